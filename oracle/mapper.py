@@ -1,0 +1,106 @@
+"""Applying the fitted cross-model KV mapper (oracle; test infrastructure only).
+
+What is computed, for target layer l, K/V, head h and every token with absolute
+position t (the same t in source and target, Sec. 3.3):
+
+1. x_j = source cache of layer sel[l][j], head h, token t, for j = 0..k-1
+   (the top-k selected source layers, ascending; Sec. 3.2).
+2. Keys only: x_j <- R_{Theta_s}(t)^{-1} x_j  (strip the source RoPE; Sec. 3.3).
+3. X = [x_0 || ... || x_{k-1}]  (cross-layer concatenation, Sec. 3.2).
+4. y = X W^{l,h} + b^{l,h}  (Eq. ridge_kv, row-vector convention of Sec. 2.3).
+5. Keys only: y <- R_{Theta_t}(t) y  (re-apply the target RoPE; the composition
+   K_t = (K_s R_s^{-1}(t) W_K + b_K) R_t(t) of Sec. 3.3: the bias is inside the
+   rotated bracket).  Values are never rotated.
+
+Two feature layouts:
+* ``"per_head"``   -- x_j is head h of layer sel[l][j] only: F = k d.
+* ``"cross_head"`` -- x_j is all KV heads of layer sel[l][j], head-minor
+                      (the paper's d_s = k n_kv d; Sec. 3.1, Sec. 3.2, Appendix
+                      "Run information", source-feature row): F = k H d.
+The per-head map equals the cross-head map with W zero outside head h's rows.
+
+Two rounding models:
+* ``"exact"``   -- everything in float64.
+* ``"bf16fwd"`` -- the paper's forward runs in bf16 (Appendix "Run information"):
+                   the stripped keys are materialised in bf16 (round-to-nearest-even)
+                   before the contraction.  Values are already bf16 inputs, and the
+                   contraction, bias and re-rotation stay exact.  This is the one point
+                   where a bf16 forward rounds an operand of the contraction.
+"""
+import numpy as np
+
+from . import bf16, rope
+
+
+def map_tokens(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
+               mode="exact", style="half", head_mix="per_head"):
+    """Map a set of tokens.
+
+    src_k, src_v : float64 [L_s][H][N][d]  -- stored (rotated) source keys, values.
+    positions    : int [N]                 -- absolute positions of the N tokens.
+    sel          : int [L_t][k]            -- selected source layers, ascending.
+    W            : float64 [L_t][2][H][F][d]  (index 0 = K, 1 = V).
+    b            : float64 [L_t][2][H][d] or None (zero bias).
+    Returns (out_k, out_v), float64 [L_t][H][N][d].
+    """
+    src_k = np.asarray(src_k, dtype=np.float64)
+    src_v = np.asarray(src_v, dtype=np.float64)
+    pos = np.asarray(positions)
+    sel = np.asarray(sel)
+    Ls, H, N, d = src_k.shape
+    Lt, k = sel.shape
+    stripped = rope.rotate(src_k, pos[None, None, :], theta_s, inverse=True, style=style)
+    feats = (stripped, src_v)
+    out = np.empty((2, Lt, H, N, d), dtype=np.float64)
+    for l in range(Lt):
+        for kv in range(2):
+            for h in range(H):
+                if head_mix == "per_head":
+                    parts = [feats[kv][s, h] for s in sel[l]]
+                elif head_mix == "cross_head":
+                    parts = [feats[kv][s, hh] for s in sel[l] for hh in range(H)]
+                else:
+                    raise ValueError(head_mix)
+                X = np.concatenate(parts, axis=-1)
+                if mode == "bf16fwd" and kv == 0:
+                    X = bf16.round_to_bf16_value(X)
+                elif mode not in ("exact", "bf16fwd"):
+                    raise ValueError(mode)
+                Y = X @ W[l, kv, h]
+                if b is not None:
+                    Y = Y + b[l, kv, h]
+                if kv == 0:
+                    Y = rope.rotate(Y, pos, theta_t, style=style)
+                out[kv, l, h] = Y
+    return out[0], out[1]
+
+
+def map_cache(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
+              mode="exact", style="half", head_mix="per_head"):
+    """Contiguous-cache form: src [L_s][B][H][T][d], positions [B][T] ->
+    (out_k, out_v) [L_t][B][H][T][d]."""
+    src_k = np.asarray(src_k, dtype=np.float64)
+    src_v = np.asarray(src_v, dtype=np.float64)
+    Ls, B, H, T, d = src_k.shape
+    pos = np.asarray(positions).reshape(B * T)
+
+    def tok(x):  # [L][B][H][T][d] -> [L][H][B*T][d]
+        return x.transpose(0, 2, 1, 3, 4).reshape(x.shape[0], H, B * T, d)
+
+    ok, ov = map_tokens(tok(src_k), tok(src_v), pos, sel, W, b, theta_s, theta_t,
+                        mode, style, head_mix)
+    Lt = ok.shape[0]
+
+    def untok(y):
+        return y.reshape(Lt, H, B, T, d).transpose(0, 2, 1, 3, 4)
+
+    return untok(ok), untok(ov)
+
+
+def mapper_params(L_t, n_kv_t, d_t, k, n_kv_s=None, d_s=None, head_mix="cross_head"):
+    """Mapper size, K plus V (Appendix C, serving cost):
+    cross-head  2 L_t n_kv^t (k n_kv^s d_h^s) d_h^t;  per-head  2 L_t n_kv^t (k d_h^s) d_h^t."""
+    n_kv_s = n_kv_t if n_kv_s is None else n_kv_s
+    d_s = d_t if d_s is None else d_s
+    feat = k * n_kv_s * d_s if head_mix == "cross_head" else k * d_s
+    return 2 * L_t * n_kv_t * feat * d_t

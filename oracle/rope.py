@@ -1,0 +1,61 @@
+"""RoPE rotation R_Theta(t) and its inverse (oracle; test infrastructure only).
+
+Sec. 3.3 (content-space mapping): the cache stores rotated keys
+k_RoPE(t) = R_Theta(t) k_content; the inverse R_Theta(t)^{-1} = R_Theta(-t) strips
+the rotation exactly because R is orthogonal.
+
+Standard RoPE (Su et al., cited in Sec. 3.3) rotates channel pair i by the angle
+t * omega_i with omega_i = theta^(-2i/d), i = 0 .. d/2-1, as the complex product
+(a + i b) * exp(i t omega_i), i.e.  a' = a cos - b sin,  b' = a sin + b cos.
+
+Pair layout (the paper does not state one):
+* ``"half"``        -- pairs (i, i + d/2): the layout of the Qwen3 / Llama checkpoints.
+* ``"interleaved"`` -- pairs (2i, 2i+1).
+"""
+import numpy as np
+
+
+def inv_freq(theta, d):
+    """omega_i = theta^(-2i/d) for i in [0, d/2), float64."""
+    i = np.arange(d // 2, dtype=np.float64)
+    return np.power(np.float64(theta), -2.0 * i / d)
+
+
+def angles(positions, theta, d):
+    """t * omega_i in float64; shape positions.shape + (d/2,)."""
+    p = np.asarray(positions, dtype=np.float64)
+    return p[..., None] * inv_freq(theta, d)
+
+
+def _pairs(x, style):
+    d = x.shape[-1]
+    if style == "half":
+        return x[..., : d // 2], x[..., d // 2:]
+    if style == "interleaved":
+        return x[..., 0::2], x[..., 1::2]
+    raise ValueError(style)
+
+
+def _unpairs(a, b, style):
+    if style == "half":
+        return np.concatenate([a, b], axis=-1)
+    out = np.empty(a.shape[:-1] + (2 * a.shape[-1],), dtype=np.float64)
+    out[..., 0::2] = a
+    out[..., 1::2] = b
+    return out
+
+
+def rotate(x, positions, theta, inverse=False, style="half"):
+    """Apply R_Theta(t) (or its inverse) to the last axis of ``x``.
+
+    ``x``: float64 [..., d]; ``positions``: integer array broadcastable to x.shape[:-1].
+    ``inverse=True`` applies R_Theta(t)^{-1} = R_Theta(-t) (the RoPE strip of Sec. 3.3).
+    """
+    x = np.asarray(x, dtype=np.float64)
+    d = x.shape[-1]
+    ang = angles(np.broadcast_to(np.asarray(positions), x.shape[:-1]), theta, d)
+    if inverse:
+        ang = -ang
+    c, s = np.cos(ang), np.sin(ang)
+    a, b = _pairs(x, style)
+    return _unpairs(a * c - b * s, a * s + b * c, style)

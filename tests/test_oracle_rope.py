@@ -1,0 +1,137 @@
+"""Pins for oracle.rope and oracle.bf16 (CPU only).
+
+RoPE is pinned against the complex-number definition of Su et al. (Sec. 3.3 cites it:
+pair i is multiplied by exp(i t omega_i)), against a textbook 2x2 rotation matrix,
+and by the group identities R(-t) R(t) = I, R(a) R(b) = R(a + b), R(0) = I and
+orthogonality (pair norms preserved).  bf16 rounding is pinned against hand-worked
+bit patterns and against torch's binary32 -> bfloat16 conversion.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import bf16, rope
+
+
+def _rng(seed=0):
+    return np.random.default_rng(seed)
+
+
+@pytest.mark.parametrize("style", ["half", "interleaved"])
+def test_inverse_is_identity(style):
+    x = _rng(1).standard_normal((3, 5, 64))
+    pos = _rng(2).integers(0, 40000, size=(3, 5))
+    y = rope.rotate(rope.rotate(x, pos, 1e6, style=style), pos, 1e6, inverse=True, style=style)
+    assert np.max(np.abs(y - x)) < 1e-12
+
+
+@pytest.mark.parametrize("style", ["half", "interleaved"])
+def test_pair_norms_preserved(style):
+    d = 32
+    x = _rng(3).standard_normal((7, d))
+    pos = np.arange(7) * 4099
+    y = rope.rotate(x, pos, 5e5, style=style)
+    if style == "half":
+        nx = x[:, : d // 2] ** 2 + x[:, d // 2:] ** 2
+        ny = y[:, : d // 2] ** 2 + y[:, d // 2:] ** 2
+    else:
+        nx = x[:, 0::2] ** 2 + x[:, 1::2] ** 2
+        ny = y[:, 0::2] ** 2 + y[:, 1::2] ** 2
+    assert np.allclose(nx, ny, rtol=1e-13, atol=1e-13)
+
+
+def test_position_zero_is_exact_identity():
+    x = _rng(4).standard_normal((4, 128))
+    y = rope.rotate(x, np.zeros(4, dtype=np.int64), 1e6)
+    assert np.array_equal(x, y)
+    y = rope.rotate(x, np.zeros(4, dtype=np.int64), 1e6, inverse=True)
+    assert np.array_equal(x, y)
+
+
+def test_angle_additivity():
+    x = _rng(5).standard_normal((6, 64))
+    a = np.array([0, 1, 17, 255, 1000, 32767])
+    b = np.array([3, 0, 9, 1, 31000, 1])
+    y1 = rope.rotate(rope.rotate(x, a, 1e4), b, 1e4)
+    y2 = rope.rotate(x, a + b, 1e4)
+    assert np.max(np.abs(y1 - y2)) < 1e-10
+
+
+def test_complex_multiplication_definition():
+    """Pair i of the half-split layout is (x[i] + 1j x[i+d/2]) * exp(1j t theta^(-2i/d))."""
+    d, theta = 16, 10000.0
+    x = _rng(6).standard_normal((9, d))
+    pos = np.array([0, 1, 2, 5, 77, 1023, 4096, 20000, 32767])
+    z = x[:, : d // 2] + 1j * x[:, d // 2:]
+    w = np.array([[theta ** (-2.0 * i / d) for i in range(d // 2)]])
+    zr = z * np.exp(1j * pos[:, None] * w)
+    expect = np.concatenate([zr.real, zr.imag], axis=1)
+    got = rope.rotate(x, pos, theta)
+    assert np.max(np.abs(got - expect)) < 1e-12
+    # the inverse multiplies by the conjugate
+    zi = z * np.exp(-1j * pos[:, None] * w)
+    got_i = rope.rotate(x, pos, theta, inverse=True)
+    assert np.max(np.abs(got_i - np.concatenate([zi.real, zi.imag], axis=1))) < 1e-12
+
+
+def test_first_pair_rotates_by_position_radians():
+    """omega_0 = 1, so pair 0 rotates by exactly t radians: a textbook 2x2 rotation."""
+    for t in [1, 3, 100, 32767]:
+        a, b = 0.3, -1.7
+        x = np.zeros((1, 8))
+        x[0, 0], x[0, 4] = a, b
+        y = rope.rotate(x, np.array([t]), 1e6)
+        rot = np.array([[math.cos(t), -math.sin(t)], [math.sin(t), math.cos(t)]])
+        ea, eb = rot @ np.array([a, b])
+        assert abs(y[0, 0] - ea) < 1e-14 and abs(y[0, 4] - eb) < 1e-14
+
+
+def test_half_and_interleaved_agree_under_permutation():
+    d = 64
+    x = _rng(7).standard_normal((5, d))
+    pos = np.array([0, 3, 999, 12345, 32000])
+    perm = np.empty(d, dtype=np.int64)  # interleaved index 2i <- half i, 2i+1 <- half i+d/2
+    perm[0::2] = np.arange(d // 2)
+    perm[1::2] = np.arange(d // 2) + d // 2
+    yh = rope.rotate(x, pos, 1e6, style="half")
+    yi = rope.rotate(x[:, perm], pos, 1e6, style="interleaved")
+    assert np.max(np.abs(yh[:, perm] - yi)) < 1e-14
+
+
+def test_inverse_frequencies():
+    w = rope.inv_freq(1e6, 128)
+    assert w[0] == 1.0
+    assert abs(w[32] - 1e6 ** -0.5) < 1e-18
+    assert abs(w[63] / w[62] - 1e6 ** (-2.0 / 128)) < 1e-14
+
+
+# ---------------------------------------------------------------- bf16 ----------
+
+def test_bf16_hand_worked_patterns():
+    vals = [1.0, -2.0, 1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8, 1.0 + 2.0 ** -8 + 2.0 ** -30,
+            3.0, 0.0, 2.0 ** -130, 65280.0]
+    expect = [0x3F80, 0xC000, 0x3F80, 0x3F82, 0x3F81, 0x4040, 0x0000, 0x0008, 0x477F]
+    assert list(bf16.encode(np.array(vals))) == expect
+
+
+def test_bf16_decode_roundtrip_all_finite_patterns():
+    bits = np.arange(0, 1 << 16, dtype=np.uint32).astype(np.uint16)
+    v = bf16.decode(bits)
+    fin = np.isfinite(v)
+    back = bf16.encode(v[fin])
+    # +0 / -0 keep their sign bit
+    assert np.array_equal(back, bits[fin])
+
+
+def test_bf16_rne_matches_torch_from_binary32():
+    """For binary32 inputs one-step rounding equals torch's float32 -> bfloat16 cast."""
+    x = (_rng(8).standard_normal(200000) * np.exp(_rng(9).uniform(-20, 20, 200000))).astype(np.float32)
+    # include exact ties: 9-bit odd significands sit half-way between two bf16 values
+    odd = np.arange(128, 256, dtype=np.float32) * 2 + 1
+    ties = np.concatenate([odd * np.float32(2.0 ** e) for e in (-9, -20, 3, 40)])
+    x = np.concatenate([x, ties, -ties])
+    expect = torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    got = bf16.encode(x.astype(np.float64))
+    assert np.array_equal(got, expect)
