@@ -1,0 +1,187 @@
+/*
+ * kvx -- cross-model KV-cache mapper, GB300 (sm_103a) C ABI.
+ *
+ * Applies the closed-form per-head ridge mapper of "Cross-Model KV Cache Transfer in
+ * LLM Families: A Closed-Form Linear Mapping for Prefill Reuse" (arXiv 2608.03893) to
+ * a prefilled source KV cache and writes the target model's KV cache:
+ *
+ *   for every target layer l, KV head h and token with absolute position t
+ *     X_K = [ R_s(t)^-1 K_s^{sel[l][0]}[h] || ... || R_s(t)^-1 K_s^{sel[l][k-1]}[h] ]
+ *     X_V = [ V_s^{sel[l][0]}[h]           || ... || V_s^{sel[l][k-1]}[h] ]
+ *     K_t^l[h] = R_t(t) (X_K W_K^{l,h} + b_K^{l,h})          (Sec. 3.3 composition)
+ *     V_t^l[h] =         X_V W_V^{l,h} + b_V^{l,h}            (Eq. ridge_kv, Sec. 3.1)
+ *
+ * sel[l] are the top-k source layers of target layer l (Sec. 3.2); R_theta(t) is the
+ * RoPE rotation of pair i by t * theta^(-2i/d) (Sec. 3.3); source and target tokens
+ * share the absolute position t (Sec. 3.3).  X is a row vector (Sec. 2.3, Eq.
+ * single_source_ols).  For bf16 caches the stripped keys are rounded to bf16
+ * (round-to-nearest-even) before the contraction: the one operand a bf16 forward
+ * (Appendix "Run information", precision row) materialises; the contraction
+ * accumulates in fp32 and the output is rounded once to the cache dtype.
+ *
+ * Conventions for every call:
+ *  - No call throws; every call returns a kvx_status (or a documented value).
+ *  - Device pointers must be 16-byte aligned, caches must have head_dim contiguous,
+ *    and every other stride must be a multiple of 8 elements (16 bytes for bf16).
+ *  - A kvx_ctx must not be used from two host threads at once, nor mapped on two
+ *    streams at the same time (both launches share the context's status word).
+ *  - kvx_last_error() returns a thread-local, human-readable description of the last
+ *    non-OK status returned on the calling thread.
+ */
+#ifndef KVX_H
+#define KVX_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define KVX_API __attribute__((visibility("default")))
+#else
+#define KVX_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct kvx_ctx kvx_ctx;
+
+typedef enum {
+  KVX_OK = 0,
+  KVX_ERR_INVALID_ARG = 1,   /* a bad argument, detected on the host; nothing launched */
+  KVX_ERR_UNSUPPORTED = 2,   /* valid request that this build cannot run (e.g. shape) */
+  KVX_ERR_OOM = 3,           /* cudaMalloc failed in kvx_create */
+  KVX_ERR_CUDA = 4,          /* a CUDA runtime or launch error */
+  KVX_ERR_TIMEOUT = 5,       /* device: a bounded wait in a kernel ran out */
+  KVX_ERR_DEVICE_BOUNDS = 6  /* device: position < 0 or block-table entry outside the pool */
+} kvx_status;
+
+typedef enum { KVX_F32 = 0, KVX_BF16 = 1 } kvx_dtype;
+
+/* Pair layout of the RoPE rotation (the paper does not state one).
+ * HALF: pairs (i, i + d/2) (Qwen3 / Llama checkpoints).  INTERLEAVED: pairs (2i, 2i+1). */
+typedef enum { KVX_ROPE_HALF = 0, KVX_ROPE_INTERLEAVED = 1 } kvx_rope_style;
+
+/* Feature layout.  PER_HEAD: head h of the k selected layers, F = k * head_dim.
+ * CROSS_HEAD: all KV heads of the k selected layers, head-minor, F = k * n_kv * head_dim
+ * (the paper's d_s = k n_kv d_h, Sec. 3.1 / Sec. 3.2). */
+typedef enum { KVX_PER_HEAD = 0, KVX_CROSS_HEAD = 1 } kvx_head_mix;
+
+/* Which kernel kvx_map launches.  AUTO picks the tensor-core (tcgen05) kernel when the
+ * shape allows it (bf16 caches and weights, head_dim 128, PER_HEAD, HALF) and the
+ * fp32 SIMT kernel otherwise. */
+typedef enum { KVX_KERNEL_AUTO = 0, KVX_KERNEL_SIMT = 1, KVX_KERNEL_TCGEN05 = 2 } kvx_kernel;
+
+/* Mapper description, read by kvx_create.  All pointers are HOST pointers; the
+ * context copies what it needs, so they may be freed when kvx_create returns. */
+typedef struct {
+  int32_t src_layers;        /* L_s */
+  int32_t tgt_layers;        /* L_t */
+  int32_t n_kv_heads;        /* n_kv = n_kv^s = n_kv^t (matched KV, Sec. 2.1) */
+  int32_t head_dim;          /* d = d_h^s = d_h^t, even */
+  int32_t k;                 /* source layers per target layer, 1 <= k <= L_s */
+  int32_t rope_style;        /* kvx_rope_style */
+  double src_rope_theta;     /* Theta of the source model's RoPE */
+  double tgt_rope_theta;     /* Theta of the target model's RoPE */
+  int32_t cache_dtype;       /* kvx_dtype of the source and target caches */
+  int32_t weight_dtype;      /* kvx_dtype of W and b below */
+  int32_t head_mix;          /* kvx_head_mix */
+  int32_t reserved;          /* must be 0 */
+  /* [L_t][k] selected source layers, distinct, each in [0, L_s); row block j of W
+   * belongs to selection[l][j].  NULL: take the top-k of selection_scores. */
+  const int32_t* selection;
+  /* [L_t][L_s] scores (head-averaged R^2, Sec. 3.2); used only if selection is NULL. */
+  const double* selection_scores;
+  /* [L_t][2][n_kv][F][d] in weight_dtype; index 0 of axis 1 is K, 1 is V. */
+  const void* W;
+  /* [L_t][2][n_kv][d] in weight_dtype, or NULL for a zero bias (Sec. 3.1: the
+   * centred fit gives b = mean(Y) - mean(X) W*). */
+  const void* b;
+} kvx_config;
+
+/* Source cache, DEVICE memory owned by the caller: element (layer l, batch b, head h,
+ * token t, channel c) of K (V) is at k[l*stride[0] + b*stride[1] + h*stride[2] +
+ * t*stride[3] + c] (v[...]).  Strides in elements; K and V share them.  The keys are
+ * the stored (RoPE-rotated) keys.  Must stay valid until the stream work completes. */
+typedef struct {
+  const void* k;
+  const void* v;
+  int64_t stride[4];
+} kvx_src;
+
+/* Target cache, DEVICE memory owned by the caller.
+ * paged == 0 (contiguous): token t of sequence b goes to
+ *   k[l*stride[0] + b*stride[1] + h*stride[2] + t*stride[3] + c].
+ * paged == 1: the token at position p of sequence b goes to physical block
+ *   blk = block_table[b * max_blocks_per_seq + p / block_size], slot p % block_size:
+ *   k[l*stride[0] + blk*stride[1] + h*stride[2] + (p % block_size)*stride[3] + c].
+ *   block_table is DEVICE int32 [batch][max_blocks_per_seq]; an entry outside
+ *   [0, n_blocks) or a logical block >= max_blocks_per_seq sets KVX_ERR_DEVICE_BOUNDS
+ *   in the status word and that row is not written.
+ * Only the mapped tokens are written; every other element is left untouched, which is
+ * what lets successive turns of a conversation append to one cache (Sec. 4.5). */
+typedef struct {
+  int32_t paged;
+  int32_t block_size;
+  void* k;
+  void* v;
+  int64_t stride[4];
+  const int32_t* block_table;
+  int32_t max_blocks_per_seq;
+  int32_t n_blocks;
+} kvx_tgt;
+
+/* Build a mapper on CUDA device `device`: validates the configuration, takes the
+ * selection (given, or the top-k of the scores, Sec. 3.2), and copies W and b to the
+ * device in the kernels' layouts.  The context owns all of its device memory.
+ * Errors: INVALID_ARG (bad dims, k, selection, NULL W), UNSUPPORTED (head_dim > 256 or
+ * odd), OOM, CUDA.  On error *out is set to NULL. */
+KVX_API kvx_status kvx_create(const kvx_config* cfg, int device, kvx_ctx** out);
+
+/* Map `batch` sequences of `tokens_per_seq` tokens each (Eq. ridge_kv with the Sec. 3.3
+ * RoPE composition).  positions: DEVICE int32 [batch][tokens_per_seq], the absolute
+ * position of each token, shared by source and target (Sec. 3.3); for a contiguous
+ * target the token index t also addresses the output row.  Asynchronous on `stream`
+ * (a cudaStream_t; NULL = the legacy default stream).  Host-detected errors return
+ * before any launch (INVALID_ARG, UNSUPPORTED); launch failures return CUDA;
+ * device-detected errors go to the status word read by kvx_get_status.
+ * batch == 0 or tokens_per_seq == 0 is a no-op returning OK. */
+KVX_API kvx_status kvx_map(kvx_ctx* ctx, const kvx_src* src, int32_t batch, int32_t tokens_per_seq,
+                   const int32_t* positions, const kvx_tgt* tgt, void* stream);
+
+/* Free the context and its device memory (synchronises the device first). NULL is OK. */
+KVX_API kvx_status kvx_destroy(kvx_ctx* ctx);
+
+/* Top-k source-layer selection (Sec. 3.2), on the host: for each target layer the k
+ * highest scores; ties go to the lower source index; each row of out[L_t][k] is
+ * returned in ascending source-layer order.  INVALID_ARG for NULL or k outside
+ * [1, L_s]. */
+KVX_API kvx_status kvx_select_topk(const double* scores, int32_t tgt_layers, int32_t src_layers,
+                           int32_t k, int32_t* out);
+
+/* Copy the context's selection table to host out[L_t][k]. */
+KVX_API kvx_status kvx_get_selection(const kvx_ctx* ctx, int32_t* out);
+
+/* Choose the kernel for later kvx_map calls (kvx_kernel).  UNSUPPORTED if the
+ * configuration cannot run on the requested kernel. */
+KVX_API kvx_status kvx_set_kernel(kvx_ctx* ctx, int32_t kernel);
+
+/* Synchronise `stream`, return the device status word (KVX_OK or the first
+ * device-detected error since the last call) and reset it to KVX_OK. */
+KVX_API kvx_status kvx_get_status(kvx_ctx* ctx, void* stream);
+
+/* Mapper size in parameters, K plus V (Appendix C, "Serving cost"):
+ * CROSS_HEAD 2 L_t n_kv (k n_kv d) d;  PER_HEAD 2 L_t n_kv (k d) d.  -1 on bad input. */
+KVX_API int64_t kvx_mapper_params(int32_t tgt_layers, int32_t n_kv_heads, int32_t head_dim, int32_t k,
+                          int32_t head_mix);
+
+/* Static description of a status code. */
+KVX_API const char* kvx_status_string(kvx_status s);
+
+/* Thread-local description of the last error on this thread ("" if none). */
+KVX_API const char* kvx_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KVX_H */

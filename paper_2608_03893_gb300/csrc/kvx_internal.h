@@ -1,0 +1,86 @@
+// Internal declarations shared by the host library and the kernels of libkvx.
+#pragma once
+
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "../../include/kvx.h"
+
+namespace kvx {
+
+constexpr int kMaxHeadDim = 256;
+constexpr int kMaxPairs = kMaxHeadDim / 2;
+
+// RoPE inverse frequencies omega_i = theta^(-2i/d) as an unevaluated sum hi + lo of two
+// floats (hi = fl32(omega), lo = fl32(omega - hi)), plus the two-float split of 2*pi
+// used to reduce t * omega into [-pi, pi] with fused multiply-adds (Cody-Waite).
+struct RopeTables {
+  float ws_hi[kMaxPairs], ws_lo[kMaxPairs];  // source theta
+  float wt_hi[kMaxPairs], wt_lo[kMaxPairs];  // target theta
+  float two_pi_hi, two_pi_lo, inv_two_pi;
+};
+
+// Everything a kernel needs about one kvx_map call.
+struct MapArgs {
+  const void* src_k;
+  const void* src_v;
+  int64_t ss[4];            // source strides (layer, batch, head, token), elements
+  void* tgt_k;
+  void* tgt_v;
+  int64_t ts[4];            // target strides (layer, batch|block, head, token|slot)
+  int32_t paged, block_size, max_blocks, n_blocks;
+  const int32_t* block_table;
+  const int32_t* pos;       // [B][T]
+  int32_t B, T;
+};
+
+// Tensor-core plan: a schedule of source-tile loads into a ring of shared-memory slots,
+// shared by every work unit (it depends only on the selection table).
+struct TcPlan {
+  int32_t n_slots = 0;        // source-tile slots in shared memory
+  int32_t n_loads = 0;        // loads per work unit
+  std::vector<int32_t> load_layer;      // [n_loads] source layer of load e
+  std::vector<int32_t> load_slot;       // [n_loads] slot it lands in
+  std::vector<int32_t> load_first_use;  // [n_loads] first target layer using it
+  std::vector<int32_t> layer_slots;     // [L_t][k] slot of selection j at layer l
+  std::vector<int32_t> layer_loads_end; // [L_t] loads issued before layer l may run
+  std::vector<int32_t> slot_release;    // [L_t][n_slots] 1 if layer l is the last use
+                                        //   of slot s before its next load
+};
+
+}  // namespace kvx
+
+struct kvx_ctx {
+  int device = 0;
+  int Ls = 0, Lt = 0, H = 0, d = 0, k = 0, F = 0;
+  int rope_style = 0, cache_dtype = 0, weight_dtype = 0, head_mix = 0;
+  double theta_s = 0, theta_t = 0;
+  int kernel = KVX_KERNEL_AUTO;
+  bool tc_eligible = false;
+  std::vector<int32_t> sel;          // host copy [L_t][k]
+  kvx::RopeTables rope{};
+  // device memory owned by the context
+  int32_t* d_sel = nullptr;          // [L_t][k]
+  void* d_W = nullptr;               // [L_t][2][H][F][d] as given (SIMT kernel)
+  float* d_b = nullptr;              // [L_t][2][H][d] fp32 (zeros when b == NULL)
+  void* d_Wt = nullptr;              // tensor-core layout (bf16), see kvx_tc.cu
+  int32_t* d_plan = nullptr;         // tensor-core schedule tables
+  int32_t* d_status = nullptr;       // device status word
+  kvx::TcPlan plan;
+  int sm_count = 0;
+};
+
+namespace kvx {
+void set_error(const std::string& msg);
+
+// SIMT fp32 kernel (any head_dim <= 256, fp32 or bf16 caches/weights, both layouts).
+kvx_status launch_simt(const kvx_ctx* ctx, const MapArgs& a, cudaStream_t stream);
+
+// Tensor-core kernel (bf16, head_dim 128, per-head, half-split pairs).
+bool tc_supported(const kvx_ctx* ctx, std::string* why);
+kvx_status tc_prepare(kvx_ctx* ctx, const void* W_host);   // repack W, build the plan
+kvx_status launch_tc(const kvx_ctx* ctx, const MapArgs& a, cudaStream_t stream);
+}  // namespace kvx

@@ -1,0 +1,251 @@
+"""ctypes binding of the kvx C ABI (include/kvx.h): argument marshalling only.
+
+Each ``kvx_*`` function here calls the C function of the same name in
+``lib/libkvx.so`` and raises ``KvxError`` when it returns a status other than
+``KVX_OK``.  Every step of the mapping runs in the library's CUDA kernels; nothing in
+this module computes any part of it, and there is no fallback: if the shared library
+is missing the first call raises.
+
+The ``*_from_tensors`` helpers turn torch tensors (used here only as device memory)
+into the plain pointer-and-stride structs of the ABI.
+"""
+import ctypes
+import os
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "lib", "libkvx.so")
+
+KVX_OK, KVX_ERR_INVALID_ARG, KVX_ERR_UNSUPPORTED, KVX_ERR_OOM = 0, 1, 2, 3
+KVX_ERR_CUDA, KVX_ERR_TIMEOUT, KVX_ERR_DEVICE_BOUNDS = 4, 5, 6
+KVX_F32, KVX_BF16 = 0, 1
+KVX_ROPE_HALF, KVX_ROPE_INTERLEAVED = 0, 1
+KVX_PER_HEAD, KVX_CROSS_HEAD = 0, 1
+KVX_KERNEL_AUTO, KVX_KERNEL_SIMT, KVX_KERNEL_TCGEN05 = 0, 1, 2
+
+
+class KvxError(RuntimeError):
+    def __init__(self, status, where, detail):
+        super().__init__("%s: status %d (%s) %s" % (where, status, _status_name(status), detail))
+        self.status = status
+
+
+class kvx_config(ctypes.Structure):
+    _fields_ = [
+        ("src_layers", ctypes.c_int32), ("tgt_layers", ctypes.c_int32),
+        ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("k", ctypes.c_int32),
+        ("rope_style", ctypes.c_int32), ("src_rope_theta", ctypes.c_double),
+        ("tgt_rope_theta", ctypes.c_double), ("cache_dtype", ctypes.c_int32),
+        ("weight_dtype", ctypes.c_int32), ("head_mix", ctypes.c_int32), ("reserved", ctypes.c_int32),
+        ("selection", ctypes.c_void_p), ("selection_scores", ctypes.c_void_p),
+        ("W", ctypes.c_void_p), ("b", ctypes.c_void_p),
+    ]
+
+
+class kvx_src(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("stride", ctypes.c_int64 * 4)]
+
+
+class kvx_tgt(ctypes.Structure):
+    _fields_ = [
+        ("paged", ctypes.c_int32), ("block_size", ctypes.c_int32),
+        ("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("stride", ctypes.c_int64 * 4),
+        ("block_table", ctypes.c_void_p), ("max_blocks_per_seq", ctypes.c_int32),
+        ("n_blocks", ctypes.c_int32),
+    ]
+
+
+_lib = None
+
+EXPORTED = ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
+            "kvx_set_kernel", "kvx_get_status", "kvx_mapper_params", "kvx_status_string",
+            "kvx_last_error")
+
+
+def lib():
+    """Load libkvx.so (once).  Raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError("libkvx.so not found at %s: build it with "
+                           "`python -m paper_2608_03893_gb300.build`" % LIB_PATH)
+    L = ctypes.CDLL(LIB_PATH)
+    vp, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+    L.kvx_create.argtypes = [ctypes.POINTER(kvx_config), ctypes.c_int, ctypes.POINTER(vp)]
+    L.kvx_map.argtypes = [vp, ctypes.POINTER(kvx_src), i32, i32, vp, ctypes.POINTER(kvx_tgt), vp]
+    L.kvx_destroy.argtypes = [vp]
+    L.kvx_select_topk.argtypes = [vp, i32, i32, i32, vp]
+    L.kvx_get_selection.argtypes = [vp, vp]
+    L.kvx_set_kernel.argtypes = [vp, i32]
+    L.kvx_get_status.argtypes = [vp, vp]
+    L.kvx_mapper_params.argtypes = [i32, i32, i32, i32, i32]
+    L.kvx_mapper_params.restype = i64
+    L.kvx_status_string.argtypes = [ctypes.c_int]
+    L.kvx_status_string.restype = ctypes.c_char_p
+    L.kvx_last_error.argtypes = []
+    L.kvx_last_error.restype = ctypes.c_char_p
+    for name in ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
+                 "kvx_set_kernel", "kvx_get_status"):
+        getattr(L, name).restype = ctypes.c_int
+    _lib = L
+    return L
+
+
+def _status_name(s):
+    try:
+        return lib().kvx_status_string(s).decode()
+    except Exception:
+        return str(s)
+
+
+def _check(status, where):
+    if status != KVX_OK:
+        raise KvxError(status, where, lib().kvx_last_error().decode())
+
+
+def _ptr(x):
+    """Address of a numpy array or torch tensor (or None)."""
+    if x is None:
+        return None
+    if hasattr(x, "data_ptr"):
+        return x.data_ptr()
+    return x.ctypes.data
+
+
+# ------------------------------------------------------------------ ABI calls ----
+
+def kvx_create(cfg, device=0):
+    """cfg: kvx_config (host pointers inside must stay alive during the call)."""
+    out = ctypes.c_void_p()
+    _check(lib().kvx_create(ctypes.byref(cfg), int(device), ctypes.byref(out)), "kvx_create")
+    return out
+
+
+def kvx_map(ctx, src, batch, tokens_per_seq, positions_ptr, tgt, stream=0):
+    _check(lib().kvx_map(ctx, ctypes.byref(src), int(batch), int(tokens_per_seq), positions_ptr,
+                         ctypes.byref(tgt), stream), "kvx_map")
+
+
+def kvx_destroy(ctx):
+    _check(lib().kvx_destroy(ctx), "kvx_destroy")
+
+
+def kvx_select_topk(scores, k):
+    """scores: float64 numpy [L_t][L_s] (C-contiguous) -> int32 numpy [L_t][k]."""
+    import numpy as np
+    s = np.ascontiguousarray(scores, dtype=np.float64)
+    out = np.empty((s.shape[0], k), dtype=np.int32)
+    _check(lib().kvx_select_topk(_ptr(s), s.shape[0], s.shape[1], int(k), _ptr(out)),
+           "kvx_select_topk")
+    return out
+
+
+def kvx_get_selection(ctx, tgt_layers, k):
+    import numpy as np
+    out = np.empty((tgt_layers, k), dtype=np.int32)
+    _check(lib().kvx_get_selection(ctx, _ptr(out)), "kvx_get_selection")
+    return out
+
+
+def kvx_set_kernel(ctx, kernel):
+    _check(lib().kvx_set_kernel(ctx, int(kernel)), "kvx_set_kernel")
+
+
+def kvx_get_status(ctx, stream=0):
+    """Returns the device status (int); does not raise for device-detected errors."""
+    return lib().kvx_get_status(ctx, stream)
+
+
+def kvx_mapper_params(tgt_layers, n_kv_heads, head_dim, k, head_mix=KVX_PER_HEAD):
+    return lib().kvx_mapper_params(tgt_layers, n_kv_heads, head_dim, k, head_mix)
+
+
+def kvx_status_string(status):
+    return lib().kvx_status_string(int(status)).decode()
+
+
+def kvx_last_error():
+    return lib().kvx_last_error().decode()
+
+
+# ---------------------------------------------------------- tensor marshalling ----
+
+_DTYPES = {"f32": KVX_F32, "bf16": KVX_BF16}
+
+
+def dtype_code(t):
+    import torch
+    if t.dtype == torch.float32:
+        return KVX_F32
+    if t.dtype == torch.bfloat16:
+        return KVX_BF16
+    raise TypeError("unsupported dtype %s" % t.dtype)
+
+
+def config_from_tensors(*, src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t,
+                        cache_dtype, W, b=None, selection=None, scores=None,
+                        rope_style=KVX_ROPE_HALF, head_mix=KVX_PER_HEAD):
+    """Build a kvx_config from host tensors.  Returns (cfg, keepalive) -- hold
+    ``keepalive`` until kvx_create returns."""
+    import numpy as np
+    import torch
+    Wc = W.detach().to("cpu").contiguous()
+    bc = None if b is None else b.detach().to("cpu").to(Wc.dtype).contiguous()
+    sel = None if selection is None else np.ascontiguousarray(selection, dtype=np.int32)
+    sc = None if scores is None else np.ascontiguousarray(scores, dtype=np.float64)
+    if sel is None and sc is None:
+        raise ValueError("need selection or scores")
+    cfg = kvx_config()
+    cfg.src_layers, cfg.tgt_layers, cfg.n_kv_heads = src_layers, tgt_layers, n_kv_heads
+    cfg.head_dim, cfg.k, cfg.rope_style = head_dim, k, rope_style
+    cfg.src_rope_theta, cfg.tgt_rope_theta = float(theta_s), float(theta_t)
+    cfg.cache_dtype = _DTYPES[cache_dtype] if isinstance(cache_dtype, str) else int(cache_dtype)
+    cfg.weight_dtype = dtype_code(Wc)
+    cfg.head_mix, cfg.reserved = head_mix, 0
+    cfg.selection = _ptr(sel)
+    cfg.selection_scores = _ptr(sc)
+    cfg.W = _ptr(Wc)
+    cfg.b = _ptr(bc)
+    return cfg, (Wc, bc, sel, sc, torch)
+
+
+def src_from_tensors(k, v):
+    """Source caches [L][B][H][T][d] (any strides with d contiguous)."""
+    if k.stride() != v.stride() or k.shape != v.shape or k.stride(-1) != 1:
+        raise ValueError("source K and V must share shape and strides, head_dim contiguous")
+    s = kvx_src()
+    s.k, s.v = k.data_ptr(), v.data_ptr()
+    for i in range(4):
+        s.stride[i] = k.stride(i)
+    return s
+
+
+def tgt_from_tensors(k, v):
+    """Contiguous target caches [L][B][H][T][d]."""
+    if k.stride() != v.stride() or k.shape != v.shape or k.stride(-1) != 1:
+        raise ValueError("target K and V must share shape and strides, head_dim contiguous")
+    t = kvx_tgt()
+    t.paged, t.block_size = 0, 0
+    t.k, t.v = k.data_ptr(), v.data_ptr()
+    for i in range(4):
+        t.stride[i] = k.stride(i)
+    t.block_table, t.max_blocks_per_seq, t.n_blocks = None, 0, 0
+    return t
+
+
+def tgt_paged_from_tensors(k, v, block_table, block_size):
+    """Paged target pools [L][n_blocks][H][block_size][d] (strides taken from the
+    tensors) and a device int32 block table [B][max_blocks_per_seq]."""
+    if k.stride() != v.stride() or k.shape != v.shape or k.stride(-1) != 1:
+        raise ValueError("target K and V pools must share shape and strides")
+    if k.shape[3] != block_size:
+        raise ValueError("pool slot axis must equal block_size")
+    t = kvx_tgt()
+    t.paged, t.block_size = 1, int(block_size)
+    t.k, t.v = k.data_ptr(), v.data_ptr()
+    for i in range(4):
+        t.stride[i] = k.stride(i)
+    t.block_table = block_table.data_ptr()
+    t.max_blocks_per_seq = block_table.shape[1]
+    t.n_blocks = k.shape[1]
+    return t

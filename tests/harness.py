@@ -1,0 +1,106 @@
+"""Test-side glue: run the CUDA path through the C ABI and the oracle on the same
+seeded inputs, and compare with the stated tolerances.
+
+Tolerances (the mapped output of a workload is compared element by element):
+* fp32 caches: max |gpu - ref| <= 1e-4 * RMS(ref), ref in the oracle's "exact" mode;
+* bf16 caches: |gpu - ref| <= 2^-7 |ref| + 1e-3 RMS(ref) for every element, ref in the
+  oracle's "bf16fwd" mode (stripped keys rounded to bf16 before the contraction).
+RMS(ref) is taken over every compared element of K and V together.
+"""
+import numpy as np
+import torch
+
+from oracle import bf16 as obf16
+from oracle import mapper as omap
+from paper_2608_03893_gb300 import kvx
+from paper_2608_03893_gb300 import synthetic as syn
+
+BF16_REL = 2.0 ** -7
+BF16_ABS_RMS = 1e-3
+F32_ABS_RMS = 1e-4
+
+
+def to_f64(t):
+    """Exact float64 copy of a CPU/GPU tensor of float32 or bfloat16."""
+    t = t.detach().contiguous().cpu()
+    if t.dtype == torch.bfloat16:
+        return obf16.decode(t.view(torch.int16).numpy().view(np.uint16))
+    return t.numpy().astype(np.float64)
+
+
+def make_ctx(w, kernel=kvx.KVX_KERNEL_AUTO, selection=None, W=None, b=None, scores=None,
+             device=0, rope_style=kvx.KVX_ROPE_HALF):
+    if W is None:
+        W, b = syn.weights(w)
+    if selection is None and scores is None:
+        scores = syn.selection_scores(w)
+    cfg, keep = kvx.config_from_tensors(
+        src_layers=w.Ls, tgt_layers=w.Lt, n_kv_heads=w.H, head_dim=w.d, k=w.k,
+        theta_s=w.theta_s, theta_t=w.theta_t, cache_dtype=w.cache_dtype, W=W, b=b,
+        selection=selection, scores=scores, rope_style=rope_style)
+    ctx = kvx.kvx_create(cfg, device)
+    if kernel != kvx.KVX_KERNEL_AUTO:
+        kvx.kvx_set_kernel(ctx, kernel)
+    sel = kvx.kvx_get_selection(ctx, w.Lt, w.k)
+    return ctx, sel, W, b
+
+
+def run_contiguous(ctx, w, sk, sv, pos_np, out_dtype=None, tgt=None):
+    dev = sk.device
+    pos = torch.from_numpy(np.ascontiguousarray(pos_np, dtype=np.int32)).to(dev)
+    B, T = pos_np.shape
+    if tgt is None:
+        dt = out_dtype or sk.dtype
+        tk = torch.full((w.Lt, B, w.H, T, w.d), float("nan"), dtype=dt, device=dev)
+        tv = torch.full_like(tk, float("nan"))
+    else:
+        tk, tv = tgt
+    stream = torch.cuda.current_stream().cuda_stream
+    kvx.kvx_map(ctx, kvx.src_from_tensors(sk, sv), B, T, pos.data_ptr(),
+                kvx.tgt_from_tensors(tk, tv), stream)
+    status = kvx.kvx_get_status(ctx, stream)
+    return tk, tv, status
+
+
+def oracle_full(w, sk, sv, pos_np, sel, W, b, style="half"):
+    mode = "exact" if w.cache_dtype == "f32" else "bf16fwd"
+    return omap.map_cache(to_f64(sk), to_f64(sv), pos_np, sel, to_f64(W),
+                          None if b is None else to_f64(b), w.theta_s, w.theta_t, mode=mode,
+                          style=style)
+
+
+def check(w, got, ref):
+    """got/ref: lists of float64 arrays of equal shapes. Returns (ok, worst ratio, rms)."""
+    g = np.concatenate([x.ravel() for x in got])
+    r = np.concatenate([x.ravel() for x in ref])
+    rms = float(np.sqrt(np.mean(r * r)))
+    err = np.abs(g - r)
+    if w.cache_dtype == "f32":
+        bound = F32_ABS_RMS * rms + 0 * r
+    else:
+        bound = BF16_REL * np.abs(r) + BF16_ABS_RMS * rms
+    bad = ~(err <= bound)          # NaN counts as a failure
+    ratio = float(np.max(err / bound)) if np.all(np.isfinite(err)) else float("inf")
+    return (not bad.any()), ratio, rms, int(bad.sum())
+
+
+def sample_rows(w, n, seed=0, turn_T=None):
+    """Token rows (b, t) to check at full size: first and last tiles, tile borders,
+    the ragged tail and random rows."""
+    T = w.T if turn_T is None else turn_T
+    rng = np.random.default_rng(1000 + seed)
+    fixed = [(0, 0), (0, 1), (0, 127), (0, 128), (w.B - 1, T - 1), (w.B - 1, T - 2),
+             (w.B - 1, (T - 1) // 128 * 128)]
+    rand = [(int(rng.integers(0, w.B)), int(rng.integers(0, T))) for _ in range(n)]
+    rows = sorted(set((b, t) for b, t in fixed + rand if 0 <= t < T))
+    return np.array(rows, dtype=np.int64)
+
+
+def oracle_rows(w, rows, pos_np, sel, W, b, turn=None):
+    """Oracle output at chosen token rows: returns (ok, ov) [L_t][H][n][d]."""
+    mode = "exact" if w.cache_dtype == "f32" else "bf16fwd"
+    sk = to_f64(syn.source_rows(w, 0, rows, turn=turn))
+    sv = to_f64(syn.source_rows(w, 1, rows, turn=turn))
+    p = pos_np[rows[:, 0], rows[:, 1]]
+    return omap.map_tokens(sk, sv, p, sel, to_f64(W), None if b is None else to_f64(b),
+                           w.theta_s, w.theta_t, mode=mode)

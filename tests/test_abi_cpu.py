@@ -1,0 +1,145 @@
+"""C-ABI library, host side only (no GPU): it builds, loads, exports every symbol that
+include/kvx.h declares, and its host logic (selection, size formula, argument
+validation before any CUDA call) matches the oracle and the paper."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import mapper as omap
+from oracle import selection as osel
+from paper_2608_03893_gb300 import build as kbuild
+from paper_2608_03893_gb300 import kvx
+from paper_2608_03893_gb300 import synthetic as syn
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    kbuild.build()
+    kvx.lib()
+
+
+def _declared_functions():
+    text = open(os.path.join(ROOT, "include", "kvx.h")).read()
+    return sorted(set(re.findall(r"KVX_API\s+[\w\s\*]+?\b(kvx_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_binding_names():
+    decl = _declared_functions()
+    assert decl == sorted(kvx.EXPORTED)
+
+
+def test_library_exports_every_declared_symbol():
+    L = kvx.lib()
+    for name in _declared_functions():
+        assert hasattr(L, name), name
+    # and nothing else of ours leaks out
+    out = os.popen("nm -D --defined-only %s" % kvx.LIB_PATH).read()
+    ours = sorted(set(re.findall(r" T (kvx_\w+)", out)))
+    assert ours == _declared_functions()
+
+
+def test_status_strings():
+    for s in range(7):
+        assert kvx.kvx_status_string(s).startswith("KVX_")
+    assert "unknown" in kvx.kvx_status_string(99)
+
+
+def test_select_topk_matches_oracle_on_every_workload():
+    for name in syn.WORKLOADS:
+        w = syn.workload(name)
+        S = syn.selection_scores(w)
+        assert np.array_equal(kvx.kvx_select_topk(S, w.k), osel.select_topk(S, w.k)), name
+    # the swept k of the headline shape
+    w = syn.workload("qwen3_14b_32b_t32768_k4")
+    S = syn.selection_scores(w)
+    for k in (1, 2, 3, 4, 7, 40):
+        assert np.array_equal(kvx.kvx_select_topk(S, k), osel.select_topk(S, k))
+
+
+def test_select_topk_ties_heavy_integer_scores():
+    rng = np.random.default_rng(5)
+    for _ in range(200):
+        lt, ls = int(rng.integers(1, 9)), int(rng.integers(1, 12))
+        k = int(rng.integers(1, ls + 1))
+        S = rng.integers(0, 3, size=(lt, ls)).astype(np.float64)
+        assert np.array_equal(kvx.kvx_select_topk(S, k), osel.select_topk(S, k))
+
+
+def test_select_topk_rejects_bad_arguments():
+    with pytest.raises(kvx.KvxError) as e:
+        kvx.kvx_select_topk(np.zeros((3, 4)), 5)
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+    with pytest.raises(kvx.KvxError):
+        kvx.kvx_select_topk(np.full((2, 3), np.nan), 1)
+
+
+def test_mapper_params_match_paper_table_and_oracle():
+    rows = [ln.split() for ln in open(os.path.join(ROOT, "tests", "golden", "mapper_sizes.txt"))
+            if ln.strip() and not ln.startswith("#")]
+    for name, k, lt, nkv, dh, params_b, _ in rows:
+        p = kvx.kvx_mapper_params(int(lt), int(nkv), int(dh), int(k), kvx.KVX_CROSS_HEAD)
+        assert round(p / 1e9, 2) == float(params_b), name
+        assert p == omap.mapper_params(int(lt), int(nkv), int(dh), int(k), head_mix="cross_head")
+    assert kvx.kvx_mapper_params(64, 8, 128, 4, kvx.KVX_PER_HEAD) == 2 * 64 * 8 * 512 * 128
+    assert kvx.kvx_mapper_params(0, 8, 128, 4, kvx.KVX_PER_HEAD) == -1
+
+
+def _cfg(**over):
+    w = syn.workload("tiny_fp32")
+    W, b = syn.weights(w)
+    args = dict(src_layers=w.Ls, tgt_layers=w.Lt, n_kv_heads=w.H, head_dim=w.d, k=w.k,
+                theta_s=w.theta_s, theta_t=w.theta_t, cache_dtype=w.cache_dtype, W=W, b=b,
+                scores=syn.selection_scores(w))
+    args.update(over)
+    return kvx.config_from_tensors(**args)
+
+
+@pytest.mark.parametrize("field,value", [
+    ("k", 0), ("k", 5), ("head_dim", 0), ("src_layers", -1), ("rope_style", 7),
+    ("head_mix", 3), ("cache_dtype", 9), ("reserved", 1), ("src_rope_theta", float("nan")),
+    ("tgt_rope_theta", 0.5),
+])
+def test_create_rejects_invalid_config_before_touching_the_device(field, value):
+    cfg, keep = _cfg()
+    setattr(cfg, field, value)
+    with pytest.raises(kvx.KvxError) as e:
+        kvx.kvx_create(cfg, 0)
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG, kvx.kvx_last_error()
+
+
+def test_create_rejects_unsupported_head_dims():
+    for hd in (63, 258):
+        cfg, keep = _cfg()
+        cfg.head_dim = hd
+        with pytest.raises(kvx.KvxError) as e:
+            kvx.kvx_create(cfg, 0)
+        assert e.value.status == kvx.KVX_ERR_UNSUPPORTED
+
+
+def test_create_rejects_bad_selection_tables():
+    w = syn.workload("tiny_fp32")
+    for bad in ([[0, 0]] * 6, [[0, 4]] * 6, [[-1, 2]] * 6):
+        cfg, keep = _cfg(selection=np.array(bad, dtype=np.int32), scores=None)
+        with pytest.raises(kvx.KvxError) as e:
+            kvx.kvx_create(cfg, 0)
+        assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+    cfg, keep = _cfg()
+    cfg.W = None
+    with pytest.raises(kvx.KvxError):
+        kvx.kvx_create(cfg, 0)
+
+
+def test_null_arguments_are_rejected():
+    L = kvx.lib()
+    assert L.kvx_create(None, 0, None) == kvx.KVX_ERR_INVALID_ARG
+    assert L.kvx_map(None, None, 1, 1, None, None, None) == kvx.KVX_ERR_INVALID_ARG
+    assert L.kvx_destroy(None) == kvx.KVX_OK
+    assert L.kvx_get_status(None, None) == kvx.KVX_ERR_INVALID_ARG
+    assert L.kvx_set_kernel(None, 0) == kvx.KVX_ERR_INVALID_ARG
+    assert L.kvx_get_selection(None, None) == kvx.KVX_ERR_INVALID_ARG

@@ -1,0 +1,331 @@
+"""GPU parity: the CUDA path (through the C ABI) against the float64 oracle on the same
+seeded inputs.  Small shapes are compared in full; the full-size workloads are compared
+on sampled token rows (all layers, heads, K and V of each sampled token) plus checks
+that hold at any size (every row written, untouched paged slots keep their sentinel)."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import mapper as omap
+from paper_2608_03893_gb300 import kvx
+from paper_2608_03893_gb300 import synthetic as syn
+
+from harness import (check, make_ctx, oracle_full, oracle_rows, run_contiguous, sample_rows,
+                     to_f64)
+
+pytestmark = pytest.mark.gpu
+
+KERNELS = {"simt": kvx.KVX_KERNEL_SIMT, "tc": kvx.KVX_KERNEL_TCGEN05}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_03893_gb300 import build as kbuild
+    kbuild.build()
+    kvx.lib()
+    torch.cuda.set_device(0)
+
+
+def _kernel_or_skip(w, kernel):
+    ctx, sel, W, b = make_ctx(w)
+    try:
+        if kernel == kvx.KVX_KERNEL_TCGEN05:
+            try:
+                kvx.kvx_set_kernel(ctx, kernel)
+            except kvx.KvxError as e:
+                pytest.fail("tensor-core kernel unavailable for a bf16 d=128 shape: %s" % e)
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
+def _small(name, kernel, **over):
+    w = syn.workload(name, **over)
+    ctx, sel, W, b = make_ctx(w, kernel=kernel)
+    try:
+        dev = torch.device("cuda:0")
+        sk = syn.source_cache(w, 0, device=dev)
+        sv = syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w)
+        tk, tv, status = run_contiguous(ctx, w, sk, sv, pos)
+        assert status == kvx.KVX_OK
+        rk, rv = oracle_full(w, sk, sv, pos, sel, W, b)
+        ok, ratio, rms, nbad = check(w, [to_f64(tk), to_f64(tv)], [rk, rv])
+        assert ok, "%s: %d elements out of tolerance (worst %.3g x bound)" % (name, nbad, ratio)
+        return ratio
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
+# ----------------------------------------------------------------- small, full -----
+
+def test_tiny_fp32_full():
+    _small("tiny_fp32", kvx.KVX_KERNEL_AUTO)
+
+
+@pytest.mark.parametrize("kname", ["simt", "tc"])
+@pytest.mark.parametrize("over", [
+    dict(Ls=6, Lt=5, H=2, B=2, T=300, k=3),                # ragged tail, B > 1
+    dict(Ls=3, Lt=4, H=1, B=1, T=1, k=1),                  # one token
+    dict(Ls=5, Lt=7, H=2, B=3, T=129, k=2, theta_t=5e5),   # different thetas, 1-row tail
+    dict(Ls=9, Lt=6, H=3, B=1, T=640, k=4),                # several tiles
+    dict(Ls=4, Lt=9, H=2, B=1, T=256, k=4, scores="uniform"),  # random selection, reloads
+])
+def test_bf16_small_full(kname, over):
+    name = "qwen3_14b_32b_b8x1024_k4"
+    if kname == "tc":
+        _kernel_or_skip(syn.workload(name, **over), KERNELS[kname])
+    _small(name, KERNELS[kname], **over)
+
+
+def test_interleaved_pairs_simt():
+    w = syn.workload("tiny_fp32", T=100, B=2)
+    ctx, sel, W, b = make_ctx(w, rope_style=kvx.KVX_ROPE_INTERLEAVED)
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w) + 7
+        tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        rk, rv = oracle_full(w, sk, sv, pos, sel, W, b, style="interleaved")
+        assert check(w, [to_f64(tk), to_f64(tv)], [rk, rv])[0]
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
+def test_cross_head_simt():
+    w = syn.workload("tiny_fp32", T=64)
+    Wc = torch.from_numpy(np.random.default_rng(3).standard_normal(
+        (w.Lt, 2, w.H, w.k * w.H * w.d, w.d)).astype(np.float32) / np.sqrt(w.k * w.H * w.d))
+    _, b = syn.weights(w)
+    scores = syn.selection_scores(w)
+    cfg, keep = kvx.config_from_tensors(
+        src_layers=w.Ls, tgt_layers=w.Lt, n_kv_heads=w.H, head_dim=w.d, k=w.k,
+        theta_s=w.theta_s, theta_t=w.theta_t, cache_dtype=w.cache_dtype, W=Wc, b=b,
+        scores=scores, head_mix=kvx.KVX_CROSS_HEAD)
+    ctx = kvx.kvx_create(cfg, 0)
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w)
+        tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        sel = kvx.kvx_get_selection(ctx, w.Lt, w.k)
+        rk, rv = omap.map_cache(to_f64(sk), to_f64(sv), pos, sel, to_f64(Wc), to_f64(b),
+                                w.theta_s, w.theta_t, mode="exact", head_mix="cross_head")
+        assert check(w, [to_f64(tk), to_f64(tv)], [rk, rv])[0]
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
+@pytest.mark.parametrize("kname", ["simt", "tc"])
+def test_identity_map_is_bit_exact(kname):
+    """k = 1, W = I, b = 0, equal thetas: V comes back bit for bit; K too at position 0
+    (the strip and re-rotation are exact identities there)."""
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=3, Lt=3, H=2, B=1, T=200, k=1)
+    W = torch.zeros((w.Lt, 2, w.H, w.d, w.d), dtype=torch.float32)
+    W[:, :, :] = torch.eye(w.d)
+    W = W.to(torch.bfloat16)
+    sel = np.array([[2], [0], [1]], dtype=np.int32)
+    ctx, sel_out, _, _ = make_ctx(w, kernel=KERNELS[kname], selection=sel, W=W, b=None)
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = np.zeros((1, w.T), dtype=np.int32)
+        tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        for l in range(w.Lt):
+            assert torch.equal(tv[l], sv[sel[l, 0]])
+            assert torch.equal(tk[l], sk[sel[l, 0]])
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
+def test_empty_and_errors():
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=3, Lt=2, H=2, B=1, T=16, k=2)
+    ctx, sel, W, b = make_ctx(w)
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        tk = torch.zeros((w.Lt, w.B, w.H, w.T, w.d), dtype=torch.bfloat16, device=dev)
+        tv = torch.zeros_like(tk)
+        pos = torch.zeros((1, w.T), dtype=torch.int32, device=dev)
+        src, tgt = kvx.src_from_tensors(sk, sv), kvx.tgt_from_tensors(tk, tv)
+        s = torch.cuda.current_stream().cuda_stream
+        kvx.kvx_map(ctx, src, 0, w.T, pos.data_ptr(), tgt, s)       # empty batch: no-op
+        kvx.kvx_map(ctx, src, 1, 0, pos.data_ptr(), tgt, s)         # no tokens: no-op
+        assert kvx.kvx_get_status(ctx, s) == kvx.KVX_OK
+        assert torch.count_nonzero(tk) == 0
+        # misaligned pointer -> INVALID_ARG, nothing launched
+        bad = kvx.src_from_tensors(sk, sv)
+        bad.k = sk.data_ptr() + 2
+        with pytest.raises(kvx.KvxError) as e:
+            kvx.kvx_map(ctx, bad, 1, w.T, pos.data_ptr(), tgt, s)
+        assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+        # negative position -> device status DEVICE_BOUNDS, that row not written
+        pos[0, 5] = -3
+        kvx.kvx_map(ctx, src, 1, w.T, pos.data_ptr(), tgt, s)
+        assert kvx.kvx_get_status(ctx, s) == kvx.KVX_ERR_DEVICE_BOUNDS
+        assert kvx.kvx_get_status(ctx, s) == kvx.KVX_OK              # reset after read
+        assert torch.count_nonzero(tk[:, 0, :, 5]) == 0
+        assert torch.count_nonzero(tk[:, 0, :, 4]) > 0
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
+def test_generator_cpu_gpu_identical():
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=2, B=2, T=300)
+    g = syn.source_cache(w, 0, device=torch.device("cuda:0")).cpu()
+    c = syn.source_cache(w, 0, device="cpu")
+    assert torch.equal(g.view(torch.int16), c.view(torch.int16))
+
+
+# ------------------------------------------------------------ full size, sampled -----
+
+FULL = ["qwen3_14b_32b_b8x1024_k4", "qwen3_14b_32b_t32768_k1", "qwen3_14b_32b_t32768_k2",
+        "qwen3_14b_32b_t32768_k4", "llama31_8b_70b_b4x8192_k3", "llama31_70b_8b_b4x8192_k3"]
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_full_size_sampled(name):
+    w = syn.workload(name)
+    ctx, sel, W, b = make_ctx(w)            # AUTO: the kernel the bench times
+    dev = torch.device("cuda:0")
+    try:
+        sk = syn.source_cache(w, 0, device=dev)
+        sv = syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w)
+        tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        del sk, sv
+        assert not torch.isnan(tk).any() and not torch.isnan(tv).any(), "unwritten rows"
+        rows = sample_rows(w, 48)
+        rk, rv = oracle_rows(w, rows, pos, sel, W, b)
+        gk = to_f64(tk[:, rows[:, 0], :, rows[:, 1]].permute(1, 2, 0, 3))
+        gv = to_f64(tv[:, rows[:, 0], :, rows[:, 1]].permute(1, 2, 0, 3))
+        ok, ratio, rms, nbad = check(w, [gk, gv], [rk, rv])
+        assert ok, "%s: %d sampled elements out of tolerance (worst %.3g x bound)" % (name, nbad, ratio)
+    finally:
+        kvx.kvx_destroy(ctx)
+        torch.cuda.empty_cache()
+
+
+# ----------------------------------------------------------------------- paged -----
+
+def _paged_run(w, turn, L0, ctx):
+    dev = torch.device("cuda:0")
+    pos = syn.positions(w, turn, L0)
+    table, n_blocks = syn.block_table(w, pos, turn)
+    pool_k = torch.empty((w.Lt, n_blocks, w.H, w.block_size, w.d), dtype=torch.bfloat16, device=dev)
+    pool_k.view(torch.int16).fill_(0x7FBF)   # a NaN pattern the map never writes
+    pool_v = torch.empty_like(pool_k)
+    pool_v.view(torch.int16).fill_(0x7FBF)
+    sk = syn.source_cache(w, 0, device=dev, turn=turn)
+    sv = syn.source_cache(w, 1, device=dev, turn=turn)
+    tbl = torch.from_numpy(table).to(dev)
+    posd = torch.from_numpy(pos).to(dev)
+    s = torch.cuda.current_stream().cuda_stream
+    kvx.kvx_map(ctx, kvx.src_from_tensors(sk, sv), w.B, w.T, posd.data_ptr(),
+                kvx.tgt_paged_from_tensors(pool_k, pool_v, tbl, w.block_size), s)
+    st = kvx.kvx_get_status(ctx, s)
+    return pool_k, pool_v, pos, table, n_blocks, st
+
+
+def _check_paged(w, ctx, sel, W, b, turn, L0, rows):
+    pool_k, pool_v, pos, table, n_blocks, st = _paged_run(w, turn, L0, ctx)
+    assert st == kvx.KVX_OK
+    # every slot of a mapped position is written; every other slot keeps the sentinel
+    written = torch.zeros((n_blocks, w.block_size), dtype=torch.bool)
+    for bb in range(w.B):
+        blk = torch.from_numpy(table[bb, pos[bb] // w.block_size].astype(np.int64))
+        slot = torch.from_numpy((pos[bb] % w.block_size).astype(np.int64))
+        written[blk, slot] = True
+    written = written.to(pool_k.device)
+    for pool in (pool_k, pool_v):
+        sent = pool.view(torch.int16) == 0x7FBF                     # [Lt][nb][H][bs][d]
+        all_sent = sent.all(dim=-1).all(dim=2).all(dim=0)            # [nb][bs]
+        none_sent = (~sent).all(dim=-1).all(dim=2).all(dim=0)
+        assert torch.equal(all_sent, ~written), "a slot outside the mapped tokens was touched"
+        assert torch.equal(none_sent, written), "a mapped slot was not fully written"
+    rk, rv = oracle_rows(w, rows, pos, sel, W, b, turn=turn)
+    p = pos[rows[:, 0], rows[:, 1]]
+    blk = table[rows[:, 0], p // w.block_size].astype(np.int64)
+    slot = (p % w.block_size).astype(np.int64)
+    gk = to_f64(pool_k[:, blk, :, slot].permute(1, 2, 0, 3))
+    gv = to_f64(pool_v[:, blk, :, slot].permute(1, 2, 0, 3))
+    ok, ratio, rms, nbad = check(w, [gk, gv], [rk, rv])
+    assert ok, "paged turn %d: %d out of tolerance (worst %.3g)" % (turn, nbad, ratio)
+
+
+@pytest.mark.parametrize("kname", ["simt", "tc"])
+def test_paged_small_full(kname):
+    w = syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4", Ls=5, Lt=3, H=2, B=3, T=37, k=2,
+                     len_range=(3, 70))
+    if kname == "tc":
+        _kernel_or_skip(w, KERNELS[kname])
+    ctx, sel, W, b = make_ctx(w, kernel=KERNELS[kname])
+    try:
+        L0 = syn.initial_lengths(w)
+        rows = np.array([(bb, t) for bb in range(w.B) for t in range(w.T)], dtype=np.int64)
+        for turn in (0, 1):
+            _check_paged(w, ctx, sel, W, b, turn, L0, rows)
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
+@pytest.mark.parametrize("turn", [0, 7])
+def test_paged_full_size_sampled(turn):
+    w = syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4")
+    ctx, sel, W, b = make_ctx(w)
+    try:
+        L0 = syn.initial_lengths(w)
+        _check_paged(w, ctx, sel, W, b, turn, L0, sample_rows(w, 40, seed=turn))
+    finally:
+        kvx.kvx_destroy(ctx)
+        torch.cuda.empty_cache()
+
+
+def test_paged_bad_block_is_reported_and_skipped():
+    w = syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4", Ls=3, Lt=2, H=2, B=2, T=20, k=2,
+                     len_range=(5, 9))
+    ctx, sel, W, b = make_ctx(w)
+    dev = torch.device("cuda:0")
+    try:
+        L0 = syn.initial_lengths(w)
+        pos = syn.positions(w, 0, L0)
+        table, n_blocks = syn.block_table(w, pos, 0)
+        table[1, pos[1, 0] // w.block_size] = n_blocks + 5        # outside the pool
+        pool_k = torch.zeros((w.Lt, n_blocks, w.H, w.block_size, w.d), dtype=torch.bfloat16, device=dev)
+        pool_v = torch.zeros_like(pool_k)
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        tbl, posd = torch.from_numpy(table).to(dev), torch.from_numpy(pos).to(dev)
+        s = torch.cuda.current_stream().cuda_stream
+        kvx.kvx_map(ctx, kvx.src_from_tensors(sk, sv), w.B, w.T, posd.data_ptr(),
+                    kvx.tgt_paged_from_tensors(pool_k, pool_v, tbl, w.block_size), s)
+        assert kvx.kvx_get_status(ctx, s) == kvx.KVX_ERR_DEVICE_BOUNDS
+        # sequence 0 was mapped normally
+        blk0 = int(table[0, pos[0, 0] // w.block_size])
+        assert torch.count_nonzero(pool_k[:, blk0]) > 0
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
+def test_incremental_turns_equal_one_shot():
+    """Per-token independence (the map is per token): mapping turn 0 then turn 1 into a
+    contiguous cache equals mapping both turns' tokens at once."""
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=6, Lt=4, H=2, B=1, T=256, k=2)
+    ctx, sel, W, b = make_ctx(w)
+    dev = torch.device("cuda:0")
+    try:
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w)
+        full_k, full_v, st = run_contiguous(ctx, w, sk, sv, pos)
+        tk = torch.zeros_like(full_k)
+        tv = torch.zeros_like(full_v)
+        for lo, hi in ((0, 100), (100, 256)):
+            tgt = (tk[:, :, :, lo:hi], tv[:, :, :, lo:hi])
+            run_contiguous(ctx, w, sk[:, :, :, lo:hi], sv[:, :, :, lo:hi], pos[:, lo:hi], tgt=tgt)
+        assert torch.equal(tk, full_k) and torch.equal(tv, full_v)
+    finally:
+        kvx.kvx_destroy(ctx)
