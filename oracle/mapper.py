@@ -26,14 +26,50 @@ Two rounding models:
                    before the contraction.  Values are already bf16 inputs, and the
                    contraction, bias and re-rotation stay exact.  This is the one point
                    where a bf16 forward rounds an operand of the contraction.
+
+Rounding slack (bf16fwd only).  Rounding a stripped key to bf16 is a decision taken
+on a value that any implementation computes with some error.  When the exact value
+lies within that error of a bf16 rounding midpoint, both neighbours are correct
+bf16-forward results.  ``map_tokens(..., rounding_slack=delta)`` therefore also
+returns, for every output, the largest change that choosing the other neighbour for
+every such ambiguous key element can cause: sum_f (hi_f - lo_f) |W[f][c]|, where
+lo_f, hi_f are the roundings of x_f -/+ delta (|a| + |b|) (a, b the stored pair of
+x_f), and for keys the two members of each re-rotated pair add up.  Values carry no
+such decision, so their slack is zero.
 """
 import numpy as np
 
 from . import bf16, rope
 
 
+def _pair_magnitude(x, style):
+    """|a| + |b| of the RoPE pair each element belongs to (same shape as x)."""
+    d = x.shape[-1]
+    if style == "half":
+        m = np.abs(x[..., : d // 2]) + np.abs(x[..., d // 2:])
+        return np.concatenate([m, m], axis=-1)
+    m = np.abs(x[..., 0::2]) + np.abs(x[..., 1::2])
+    out = np.empty_like(x)
+    out[..., 0::2] = m
+    out[..., 1::2] = m
+    return out
+
+
+def _pair_sum(y, style):
+    """Each element replaced by the sum over its RoPE pair (bound after a rotation)."""
+    d = y.shape[-1]
+    if style == "half":
+        m = y[..., : d // 2] + y[..., d // 2:]
+        return np.concatenate([m, m], axis=-1)
+    m = y[..., 0::2] + y[..., 1::2]
+    out = np.empty_like(y)
+    out[..., 0::2] = m
+    out[..., 1::2] = m
+    return out
+
+
 def map_tokens(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
-               mode="exact", style="half", head_mix="per_head"):
+               mode="exact", style="half", head_mix="per_head", rounding_slack=None):
     """Map a set of tokens.
 
     src_k, src_v : float64 [L_s][H][N][d]  -- stored (rotated) source keys, values.
@@ -41,7 +77,8 @@ def map_tokens(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
     sel          : int [L_t][k]            -- selected source layers, ascending.
     W            : float64 [L_t][2][H][F][d]  (index 0 = K, 1 = V).
     b            : float64 [L_t][2][H][d] or None (zero bias).
-    Returns (out_k, out_v), float64 [L_t][H][N][d].
+    Returns (out_k, out_v), float64 [L_t][H][N][d]; with ``rounding_slack`` (bf16fwd
+    mode) also (slack_k, slack_v) of the same shape.
     """
     src_k = np.asarray(src_k, dtype=np.float64)
     src_v = np.asarray(src_v, dtype=np.float64)
@@ -52,6 +89,12 @@ def map_tokens(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
     stripped = rope.rotate(src_k, pos[None, None, :], theta_s, inverse=True, style=style)
     feats = (stripped, src_v)
     out = np.empty((2, Lt, H, N, d), dtype=np.float64)
+    want_slack = rounding_slack is not None and mode == "bf16fwd"
+    slack = np.zeros_like(out) if rounding_slack is not None else None
+    if want_slack:
+        delta = rounding_slack * _pair_magnitude(src_k, style)
+        amb = (bf16.round_to_bf16_value(stripped + delta) -
+               bf16.round_to_bf16_value(stripped - delta))
     for l in range(Lt):
         for kv in range(2):
             for h in range(H):
@@ -72,13 +115,21 @@ def map_tokens(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
                 if kv == 0:
                     Y = rope.rotate(Y, pos, theta_t, style=style)
                 out[kv, l, h] = Y
+                if want_slack and kv == 0:
+                    if head_mix == "per_head":
+                        A = np.concatenate([amb[s, h] for s in sel[l]], axis=-1)
+                    else:
+                        A = np.concatenate([amb[s, hh] for s in sel[l] for hh in range(H)], axis=-1)
+                    slack[0, l, h] = _pair_sum(A @ np.abs(W[l, 0, h]), style)
+    if rounding_slack is not None:
+        return out[0], out[1], slack[0], slack[1]
     return out[0], out[1]
 
 
 def map_cache(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
-              mode="exact", style="half", head_mix="per_head"):
+              mode="exact", style="half", head_mix="per_head", rounding_slack=None):
     """Contiguous-cache form: src [L_s][B][H][T][d], positions [B][T] ->
-    (out_k, out_v) [L_t][B][H][T][d]."""
+    (out_k, out_v) [L_t][B][H][T][d] (plus the two slacks with ``rounding_slack``)."""
     src_k = np.asarray(src_k, dtype=np.float64)
     src_v = np.asarray(src_v, dtype=np.float64)
     Ls, B, H, T, d = src_k.shape
@@ -87,14 +138,14 @@ def map_cache(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
     def tok(x):  # [L][B][H][T][d] -> [L][H][B*T][d]
         return x.transpose(0, 2, 1, 3, 4).reshape(x.shape[0], H, B * T, d)
 
-    ok, ov = map_tokens(tok(src_k), tok(src_v), pos, sel, W, b, theta_s, theta_t,
-                        mode, style, head_mix)
-    Lt = ok.shape[0]
+    res = map_tokens(tok(src_k), tok(src_v), pos, sel, W, b, theta_s, theta_t,
+                     mode, style, head_mix, rounding_slack)
+    Lt = res[0].shape[0]
 
     def untok(y):
         return y.reshape(Lt, H, B, T, d).transpose(0, 2, 1, 3, 4)
 
-    return untok(ok), untok(ov)
+    return tuple(untok(r) for r in res)
 
 
 def mapper_params(L_t, n_kv_t, d_t, k, n_kv_s=None, d_s=None, head_mix="cross_head"):

@@ -50,8 +50,8 @@ def _small(name, kernel, **over):
         pos = syn.positions(w)
         tk, tv, status = run_contiguous(ctx, w, sk, sv, pos)
         assert status == kvx.KVX_OK
-        rk, rv = oracle_full(w, sk, sv, pos, sel, W, b)
-        ok, ratio, rms, nbad = check(w, [to_f64(tk), to_f64(tv)], [rk, rv])
+        rk, rv, ak, av = oracle_full(w, sk, sv, pos, sel, W, b)
+        ok, ratio, rms, nbad = check(w, [to_f64(tk), to_f64(tv)], [rk, rv], [ak, av])
         assert ok, "%s: %d elements out of tolerance (worst %.3g x bound)" % (name, nbad, ratio)
         return ratio
     finally:
@@ -88,16 +88,16 @@ def test_interleaved_pairs_simt():
         pos = syn.positions(w) + 7
         tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
         assert st == kvx.KVX_OK
-        rk, rv = oracle_full(w, sk, sv, pos, sel, W, b, style="interleaved")
-        assert check(w, [to_f64(tk), to_f64(tv)], [rk, rv])[0]
+        rk, rv, ak, av = oracle_full(w, sk, sv, pos, sel, W, b, style="interleaved")
+        assert check(w, [to_f64(tk), to_f64(tv)], [rk, rv], [ak, av])[0]
     finally:
         kvx.kvx_destroy(ctx)
 
 
 def test_cross_head_simt():
     w = syn.workload("tiny_fp32", T=64)
-    Wc = torch.from_numpy(np.random.default_rng(3).standard_normal(
-        (w.Lt, 2, w.H, w.k * w.H * w.d, w.d)).astype(np.float32) / np.sqrt(w.k * w.H * w.d))
+    Wc = torch.from_numpy((np.random.default_rng(3).standard_normal(
+        (w.Lt, 2, w.H, w.k * w.H * w.d, w.d)) / np.sqrt(w.k * w.H * w.d)).astype(np.float32))
     _, b = syn.weights(w)
     scores = syn.selection_scores(w)
     cfg, keep = kvx.config_from_tensors(
@@ -201,10 +201,10 @@ def test_full_size_sampled(name):
         del sk, sv
         assert not torch.isnan(tk).any() and not torch.isnan(tv).any(), "unwritten rows"
         rows = sample_rows(w, 48)
-        rk, rv = oracle_rows(w, rows, pos, sel, W, b)
+        rk, rv, ak, av = oracle_rows(w, rows, pos, sel, W, b)
         gk = to_f64(tk[:, rows[:, 0], :, rows[:, 1]].permute(1, 2, 0, 3))
         gv = to_f64(tv[:, rows[:, 0], :, rows[:, 1]].permute(1, 2, 0, 3))
-        ok, ratio, rms, nbad = check(w, [gk, gv], [rk, rv])
+        ok, ratio, rms, nbad = check(w, [gk, gv], [rk, rv], [ak, av])
         assert ok, "%s: %d sampled elements out of tolerance (worst %.3g x bound)" % (name, nbad, ratio)
     finally:
         kvx.kvx_destroy(ctx)
@@ -248,13 +248,13 @@ def _check_paged(w, ctx, sel, W, b, turn, L0, rows):
         none_sent = (~sent).all(dim=-1).all(dim=2).all(dim=0)
         assert torch.equal(all_sent, ~written), "a slot outside the mapped tokens was touched"
         assert torch.equal(none_sent, written), "a mapped slot was not fully written"
-    rk, rv = oracle_rows(w, rows, pos, sel, W, b, turn=turn)
+    rk, rv, ak, av = oracle_rows(w, rows, pos, sel, W, b, turn=turn)
     p = pos[rows[:, 0], rows[:, 1]]
     blk = table[rows[:, 0], p // w.block_size].astype(np.int64)
     slot = (p % w.block_size).astype(np.int64)
     gk = to_f64(pool_k[:, blk, :, slot].permute(1, 2, 0, 3))
     gv = to_f64(pool_v[:, blk, :, slot].permute(1, 2, 0, 3))
-    ok, ratio, rms, nbad = check(w, [gk, gv], [rk, rv])
+    ok, ratio, rms, nbad = check(w, [gk, gv], [rk, rv], [ak, av])
     assert ok, "paged turn %d: %d out of tolerance (worst %.3g)" % (turn, nbad, ratio)
 
 

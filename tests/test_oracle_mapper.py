@@ -17,7 +17,7 @@ import math
 import numpy as np
 import pytest
 
-from oracle import bf16, mapper
+from oracle import bf16, mapper, rope
 
 
 def _problem(seed, Ls=3, Lt=4, H=2, N=6, d=8, k=2, head_mix="per_head", theta_s=1e4,
@@ -207,3 +207,39 @@ def test_map_cache_layout_roundtrip():
     for bb in range(B):
         tk, tv = mapper.map_tokens(src_k[:, bb], src_v[:, bb], pos[bb], sel, W, b, 1e4, 1e4)
         assert np.array_equal(ck[:, bb], tk) and np.array_equal(cv[:, bb], tv)
+
+
+def test_rounding_slack_is_zero_without_ambiguity_and_for_values():
+    P = _problem(44, N=10)
+    ok, ov, sk, sv = mapper.map_tokens(**P, mode="bf16fwd", rounding_slack=0.0)
+    assert np.all(sk == 0) and np.all(sv == 0)
+    ok2, ov2, sk2, sv2 = mapper.map_tokens(**P, mode="bf16fwd", rounding_slack=4e-6)
+    assert np.array_equal(ok, ok2) and np.all(sv2 == 0)
+
+
+def test_rounding_slack_covers_both_roundings_of_a_planted_midpoint():
+    """Content keys sitting exactly on a bf16 midpoint are rotated into the cache; the
+    oracle's f64 strip lands within 1e-15 of the midpoint and may round either way.
+    Both choices, evaluated directly, must lie within out +- slack."""
+    rng = np.random.default_rng(45)
+    Ls, Lt, H, N, d, k = 2, 2, 1, 3, 8, 2
+    content = bf16.round_to_bf16_value(rng.standard_normal((Ls, H, N, d)))
+    content[0, 0, :, 1] = 1.0 + 2.0 ** -8          # ties between 1 and 1 + 2^-7
+    content[1, 0, :, 6] = -(3.0 + 2.0 ** -7)        # ties between -3 and -(3 + 2^-6)
+    pos = np.array([0, 77, 30001])
+    stored = np.stack([rope.rotate(content[s], pos[None, :], 1e4) for s in range(Ls)])
+    sel = np.array([[0, 1], [0, 1]])
+    W = rng.standard_normal((Lt, 2, H, k * d, d)) / 4
+    b = rng.standard_normal((Lt, 2, H, d)) * 0.1
+    src_v = rng.standard_normal((Ls, H, N, d))
+    out_k, _, slack_k, _ = mapper.map_tokens(stored, src_v, pos, sel, W, b, 1e4, 1e4,
+                                             mode="bf16fwd", rounding_slack=4e-6)
+    for down in (True, False):
+        X = content.copy()
+        X[0, 0, :, 1] = 1.0 if down else 1.0 + 2.0 ** -7
+        X[1, 0, :, 6] = -3.0 if down else -(3.0 + 2.0 ** -6)
+        for l in range(Lt):
+            Xl = np.concatenate([X[s, 0] for s in sel[l]], axis=-1)
+            y = rope.rotate(Xl @ W[l, 0, 0] + b[l, 0, 0], pos, 1e4)
+            assert np.all(np.abs(y - out_k[l, 0]) <= slack_k[l, 0] + 1e-12)
+    assert np.all(slack_k[:, 0][:, :, [1, 5]] > 0)   # the planted pairs are flagged
