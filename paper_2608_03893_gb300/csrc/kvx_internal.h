@@ -38,17 +38,18 @@ struct MapArgs {
 };
 
 // Tensor-core plan: a schedule of source-tile loads into a ring of shared-memory slots,
-// shared by every work unit (it depends only on the selection table).
+// the same for every work unit (it depends only on the selection table).  Uses are the
+// (target layer l, selection j) pairs in l-major order.
 struct TcPlan {
-  int32_t n_slots = 0;        // source-tile slots in shared memory
-  int32_t n_loads = 0;        // loads per work unit
+  int32_t n_slots = 0;                  // source-tile slots in shared memory
+  int32_t n_wst = 0;                    // W stages in shared memory
+  int32_t n_loads = 0;                  // source-tile loads per work unit
   std::vector<int32_t> load_layer;      // [n_loads] source layer of load e
   std::vector<int32_t> load_slot;       // [n_loads] slot it lands in
-  std::vector<int32_t> load_first_use;  // [n_loads] first target layer using it
-  std::vector<int32_t> layer_slots;     // [L_t][k] slot of selection j at layer l
-  std::vector<int32_t> layer_loads_end; // [L_t] loads issued before layer l may run
-  std::vector<int32_t> slot_release;    // [L_t][n_slots] 1 if layer l is the last use
-                                        //   of slot s before its next load
+  std::vector<int32_t> load_first_use;  // [n_loads] target layer of its first use
+  std::vector<int32_t> use_slot;        // [L_t*k] slot holding the tile of use (l, j)
+  std::vector<int32_t> use_flags;       // [L_t*k] bit 0: first use of a load,
+                                        //         bit 1: last use before the slot is reloaded
 };
 
 }  // namespace kvx

@@ -70,7 +70,8 @@ def test_tiny_fp32_full():
     dict(Ls=3, Lt=4, H=1, B=1, T=1, k=1),                  # one token
     dict(Ls=5, Lt=7, H=2, B=3, T=129, k=2, theta_t=5e5),   # different thetas, 1-row tail
     dict(Ls=9, Lt=6, H=3, B=1, T=640, k=4),                # several tiles
-    dict(Ls=4, Lt=9, H=2, B=1, T=256, k=4, scores="uniform"),  # random selection, reloads
+    dict(Ls=8, Lt=9, H=2, B=1, T=256, k=4, scores="uniform"),  # random selection, reloads
+    dict(Ls=10, Lt=5, H=2, B=1, T=200, k=6),               # more selected layers than slots
 ])
 def test_bf16_small_full(kname, over):
     name = "qwen3_14b_32b_b8x1024_k4"
