@@ -1,0 +1,420 @@
+#!/usr/bin/env python3
+"""Throughput bench for the cross-model KV mapper (one JSON line on rank 0).
+
+Metric: mapped target-KV tokens/s (one token = every target layer x KV head x K and V
+written) on the Qwen3-14B->32B-shaped long-context workload: 40 -> 64 layers, 8 KV heads,
+head_dim 128, bf16, one sequence of 32768 tokens at positions 0..32767, k = 4 selected
+source layers per target layer.  A step is one kvx_map call over the whole workload.
+
+* value: device throughput, inputs resident in HBM, K steps timed with CUDA events on
+  the launching stream between a barrier + synchronize on both sides (max over ranks).
+  Every step reads 5.4 GB of source cache and writes 8.6 GB of target cache, far more
+  than the 129 MB L2, so no flush is needed between steps.
+* e2e: the same metric through the C ABI with host buffers: each step copies the source
+  caches and positions from pinned host memory, maps, and copies the target cache back.
+* roofline: algorithmic FLOPs and bytes of one launch (tensor-core and HBM bounds)
+  against MEASURED_PEAKS.json; traffic from the committed ncu summary when it was taken
+  on the current kernel source.
+* cpu_baseline: the float64 oracle on a bounded sample of the same workload's tokens.
+* --impl reference: the oracle as the reference arm.
+
+Multi-GPU (torchrun): every rank maps its own replica (weak scaling, no collective on
+the data path; a MAX all-reduce of the elapsed time only).
+"""
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_03893_gb300 import kvx  # noqa: E402
+from paper_2608_03893_gb300 import synthetic as syn  # noqa: E402
+
+METRIC = "mapped target-KV tokens/s"
+UNIT = "tokens/s"
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "tc_map_kernel_qwen3_14b_32b_traffic.txt")
+KERNEL_SOURCES = ["paper_2608_03893_gb300/csrc/kvx_tc.cu", "paper_2608_03893_gb300/csrc/kvx_rope.cuh",
+                  "paper_2608_03893_gb300/csrc/kvx_internal.h"]
+
+
+def algorithmic(w):
+    """FLOPs and bytes of one launch (per-unit figures times the tokens of the launch)."""
+    e = 2  # bf16
+    tok = w.n_tokens
+    flop_per_tok = 2 * w.Lt * w.H * 2 * w.F * w.d              # K and V contractions
+    src_per_tok = 2 * w.Ls * w.H * w.d * e                       # every source layer read once
+    tgt_per_tok = 2 * w.Lt * w.H * w.d * e                       # target written once
+    w_bytes = w.Lt * 2 * w.H * w.F * w.d * e + w.Lt * 2 * w.H * w.d * e
+    return dict(flop=flop_per_tok * tok, bytes=(src_per_tok + tgt_per_tok + 4) * tok + w_bytes,
+                flop_per_token=flop_per_tok, bytes_per_token=src_per_tok + tgt_per_tok + 4,
+                weight_bytes=w_bytes)
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sustained=d.get("bf16_tflops_sustained"),
+                    source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, source="fallback")
+
+
+def kernel_hash():
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        h.update(open(os.path.join(ROOT, f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def committed_traffic(workload):
+    """dram bytes per launch from the committed ncu summary, if taken on this kernel."""
+    if not os.path.exists(TRAFFIC_FILE):
+        return None
+    kv = {}
+    for ln in open(TRAFFIC_FILE):
+        if ":" in ln and not ln.startswith("#"):
+            a, b = ln.split(":", 1)
+            kv[a.strip()] = b.strip()
+    if kv.get("kernel_source_sha256_16") != kernel_hash() or kv.get("workload") != workload:
+        return None
+    try:
+        return float(kv["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        rows = []
+        for ln in (self.out or "").splitlines():
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append(dict(sm=float(parts[1]), smax=float(parts[2]), power=float(parts[3]),
+                                 hw=parts[5], hwt=parts[6], swt=parts[7], pcap=parts[8]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"]}
+        loaded = [r for r in rows if r["power"] > 200.0] or rows
+        reasons = set()
+        for r in loaded:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                              ("swt", "sw_thermal_slowdown"), ("pcap", "sw_power_cap")):
+                if r[key].lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(r["sm"] for r in loaded),
+                "sm_max_mhz": max(r["smax"] for r in rows), "reasons": sorted(reasons),
+                "samples": len(rows), "samples_under_load": len(loaded),
+                "power_w_max": max(r["power"] for r in rows)}
+
+
+def dist_setup(n_gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        return rank, world, local, dist
+    return 0, 1, 0, None
+
+
+def barrier(dist):
+    if dist is not None:
+        dist.barrier()
+
+
+def max_over_ranks(x, dist, dev):
+    if dist is None:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------ oracle leg ----
+
+def oracle_sample_rate(w, budget_s, seed=0, ctx_sel=None):
+    """Time the float64 oracle (as it stands) on a bounded sample of the workload's
+    tokens.  Returns (tokens/s, tokens, seconds, threads)."""
+    from oracle import bf16 as obf16
+    from oracle import mapper as omap
+    from oracle import selection as osel
+    W, b = syn.weights(w)
+    Wf = obf16.decode(W.view(torch.int16).numpy().view(np.uint16)) if W.dtype == torch.bfloat16 else W.double().numpy()
+    bf = obf16.decode(b.view(torch.int16).numpy().view(np.uint16)) if b.dtype == torch.bfloat16 else b.double().numpy()
+    sel = osel.select_topk(syn.selection_scores(w), w.k)
+    pos = syn.positions(w)
+    rng = np.random.default_rng(seed)
+
+    def run(n):
+        rows = np.stack([rng.integers(0, w.B, n), rng.integers(0, w.T, n)], axis=1)
+        sk = syn.source_rows(w, 0, rows)
+        sv = syn.source_rows(w, 1, rows)
+        skf = obf16.decode(sk.view(torch.int16).numpy().view(np.uint16))
+        svf = obf16.decode(sv.view(torch.int16).numpy().view(np.uint16))
+        p = pos[rows[:, 0], rows[:, 1]]
+        t0 = time.perf_counter()
+        omap.map_tokens(skf, svf, p, sel, Wf, bf, w.theta_s, w.theta_t, mode="bf16fwd")
+        return time.perf_counter() - t0
+
+    n, dt = 8, run(8)
+    while dt < 0.2 * budget_s and n < w.n_tokens:
+        n = min(w.n_tokens, int(n * min(8.0, max(2.0, 0.5 * budget_s / max(dt, 1e-3)))))
+        dt = run(n)
+    return n / dt, n, dt, blas_threads()
+
+
+def blas_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        info = threadpool_info()
+        if info:
+            return int(max(i.get("num_threads", 1) for i in info))
+    except Exception:
+        pass
+    for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS"):
+        if os.environ.get(var, "").isdigit():
+            return int(os.environ[var])
+    return os.cpu_count() or 1
+
+
+def reference_arm(args, w, config):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    from oracle import bf16 as obf16
+    from oracle import mapper as omap
+    from oracle import selection as osel
+    # size one step so that warmup + steps stay within a few minutes
+    rate, n_cal, dt_cal, cores = oracle_sample_rate(w, budget_s=2.0)
+    per_step = max(1, min(w.n_tokens, int(rate * 150.0 / max(1, args.steps + args.warmup))))
+    W, b = syn.weights(w)
+    Wf = obf16.decode(W.view(torch.int16).numpy().view(np.uint16))
+    bf = obf16.decode(b.view(torch.int16).numpy().view(np.uint16))
+    sel = osel.select_topk(syn.selection_scores(w), w.k)
+    pos = syn.positions(w)
+    rng = np.random.default_rng(7)
+    times, toks = [], 0
+    for i in range(args.warmup + args.steps):
+        rows = np.stack([rng.integers(0, w.B, per_step), rng.integers(0, w.T, per_step)], axis=1)
+        skf = obf16.decode(syn.source_rows(w, 0, rows).view(torch.int16).numpy().view(np.uint16))
+        svf = obf16.decode(syn.source_rows(w, 1, rows).view(torch.int16).numpy().view(np.uint16))
+        t0 = time.perf_counter()
+        omap.map_tokens(skf, svf, pos[rows[:, 0], rows[:, 1]], sel, Wf, bf, w.theta_s, w.theta_t,
+                        mode="bf16fwd")
+        dt = time.perf_counter() - t0
+        if i >= args.warmup:
+            times.append(dt)
+            toks += per_step
+    total = sum(times)
+    value = toks / total
+    sample = "%d random tokens per step (of %d), float64 oracle, numpy BLAS" % (per_step, w.n_tokens)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / len(times),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": config,
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# -------------------------------------------------------------------- GPU leg -----
+
+def make_mapper(w, dev_index):
+    W, b = syn.weights(w)
+    cfg, keep = kvx.config_from_tensors(
+        src_layers=w.Ls, tgt_layers=w.Lt, n_kv_heads=w.H, head_dim=w.d, k=w.k, theta_s=w.theta_s,
+        theta_t=w.theta_t, cache_dtype=w.cache_dtype, W=W, b=b, scores=syn.selection_scores(w))
+    return kvx.kvx_create(cfg, dev_index)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="kvx", choices=["kvx", "reference"])
+    ap.add_argument("--workload", default=syn.HEADLINE)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=None)
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)
+    w = syn.workload(args.workload)
+    alg = algorithmic(w)
+    config = {"workload": w.name, "src_layers": w.Ls, "tgt_layers": w.Lt, "kv_heads": w.H,
+              "head_dim": w.d, "k": w.k, "batch": w.B, "seq_len": w.T, "tokens_per_step": w.n_tokens,
+              "rope_theta": w.theta_t, "layout": "paged" if w.paged else "contiguous",
+              "parallelism": "replicas x%d" % args.gpus,
+              "l2": "no flush: each step streams %.1f GB (source read + target write) vs 129 MB L2"
+                    % (alg["bytes"] / 1e9)}
+    if args.impl == "reference":
+        return reference_arm(args, w, config)
+
+    rank, world, local, dist = dist_setup(args.gpus)
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    sp = stream.cuda_stream
+
+    ctx = make_mapper(w, local)
+    sk = syn.source_cache(w, 0, device=dev)
+    sv = syn.source_cache(w, 1, device=dev)
+    pos_np = syn.positions(w)
+    pos = torch.from_numpy(pos_np).to(dev)
+    tk = torch.empty((w.Lt, w.B, w.H, w.T, w.d), dtype=torch.bfloat16, device=dev)
+    tv = torch.empty_like(tk)
+    src, tgt = kvx.src_from_tensors(sk, sv), kvx.tgt_from_tensors(tk, tv)
+
+    def step():
+        kvx.kvx_map(ctx, src, w.B, w.T, pos.data_ptr(), tgt, sp)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    assert kvx.kvx_get_status(ctx, sp) == kvx.KVX_OK
+    assert not torch.isnan(tk).any().item()
+
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        barrier(dist)
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for _ in range(args.steps):
+            step()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        barrier(dist)
+    ms = ev0.elapsed_time(ev1)
+    ms = max_over_ranks(ms, dist, dev)
+    st = kvx.kvx_get_status(ctx, sp)
+    ms_step = ms / args.steps
+    value = world * w.n_tokens * args.steps / (ms / 1e3)
+
+    # ---- e2e: host buffers through the C ABI, copies inside the timed region
+    e2e_steps = args.e2e_steps or max(3, min(args.steps, 40))
+    hk = torch.empty(sk.shape, dtype=sk.dtype, pin_memory=True)
+    hv = torch.empty(sv.shape, dtype=sv.dtype, pin_memory=True)
+    hk.copy_(sk)
+    hv.copy_(sv)
+    hpos = torch.from_numpy(pos_np).pin_memory()
+    ok_ = torch.empty(tk.shape, dtype=tk.dtype, pin_memory=True)
+    ov_ = torch.empty(tv.shape, dtype=tv.dtype, pin_memory=True)
+    h2d = hk.numel() * 2 + hv.numel() * 2 + hpos.numel() * 4
+    d2h = ok_.numel() * 2 + ov_.numel() * 2
+
+    def e2e_step():
+        sk.copy_(hk, non_blocking=True)
+        sv.copy_(hv, non_blocking=True)
+        pos.copy_(hpos, non_blocking=True)
+        kvx.kvx_map(ctx, src, w.B, w.T, pos.data_ptr(), tgt, sp)
+        ok_.copy_(tk, non_blocking=True)
+        ov_.copy_(tv, non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize()
+    barrier(dist)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(dist)
+    ems = max_over_ranks(e0.elapsed_time(e1), dist, dev)
+    e2e_value = world * w.n_tokens * e2e_steps / (ems / 1e3)
+    del hk, hv, ok_, ov_
+
+    kvx.kvx_destroy(ctx)
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return 0
+
+    peaks = load_peaks()
+    t_tc = alg["flop"] / (peaks["bf16"] * 1e12)
+    t_hbm = alg["bytes"] / (peaks["hbm"] * 1e9)
+    launch_s = ms_step / 1e3                  # one launch per step
+    bound = "tensor" if t_tc >= t_hbm else "hbm"
+    if bound == "tensor":
+        achieved, peak, unit = alg["flop"] / launch_s / 1e12, peaks["bf16"], "TFLOP/s"
+    else:
+        achieved, peak, unit = alg["bytes"] / launch_s / 1e9, peaks["hbm"], "GB/s"
+    roofline = {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+                "frac": achieved / peak, "traffic": committed_traffic(w.name),
+                "peak_source": "%s (bf16 burst; HBM copy)" % peaks["source"],
+                "roofline_ms": 1e3 * max(t_tc, t_hbm),
+                "other": {"hbm_achieved_gbs": alg["bytes"] / launch_s / 1e9, "hbm_peak_gbs": peaks["hbm"],
+                          "hbm_frac": alg["bytes"] / launch_s / 1e9 / peaks["hbm"],
+                          "tensor_achieved_tflops": alg["flop"] / launch_s / 1e12,
+                          "tensor_frac": alg["flop"] / launch_s / 1e12 / peaks["bf16"]},
+                "algorithmic": {"flop_per_launch": alg["flop"], "bytes_per_launch": alg["bytes"],
+                                "flop_per_token": alg["flop_per_token"],
+                                "bytes_per_token": alg["bytes_per_token"],
+                                "weight_bytes": alg["weight_bytes"]}}
+    cpu = None
+    if not args.no_cpu_baseline:
+        rate, n, dt, cores = oracle_sample_rate(w, budget_s=12.0)
+        cpu = {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": "%d random tokens of the workload (all %d layers x %d heads x K,V), "
+                         "float64 numpy oracle, %.1f s" % (n, w.Lt, w.H, dt)}
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config,
+            "clocks": clk.summary(), "status": kvx.kvx_status_string(st),
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "steps": e2e_steps, "ms_per_step": ems / e2e_steps},
+            "gpu_launches": args.steps, "roofline": roofline, "cpu_baseline": cpu,
+            "kernel": "tc_map_kernel (tcgen05, sm_103a)"}
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

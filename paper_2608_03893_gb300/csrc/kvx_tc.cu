@@ -173,6 +173,29 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
+// L2 prefetch of one tensor-map tile (no shared memory, no barrier).
+__device__ __forceinline__ void tma_prefetch_5d(const CUtensorMap* map, int c0, int c1, int c2, int c3, int c4) {
+  asm volatile("cp.async.bulk.prefetch.tensor.5d.L2.global.tile [%0, {%1, %2, %3, %4, %5}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4)
+               : "memory");
+}
+
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int c0, int c1) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(c0), "r"(c1)
+               : "memory");
+}
+
+// 16-byte global store that bypasses L1 and is marked evict-first in L2 (the target
+// cache is written once and not read by this kernel).
+__device__ __forceinline__ void st_global_stream(void* ptr, uint4 v, uint64_t policy) {
+  asm volatile("st.global.L1::no_allocate.L2::cache_hint.v4.b32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(ptr),
+               "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "l"(policy)
+               : "memory");
+}
+
 __device__ __forceinline__ void tc_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -244,9 +267,13 @@ struct Unit {
   int b, t0, h, kv;
 };
 
+// Units are visited u = blockIdx.x + i * gridDim.x.  With an even grid, u & 1 would pin
+// every CTA to K or to V units; flipping it every round makes each CTA alternate, which
+// balances the (heavier) key units across CTAs.  u and u ^ 1 share u / grid, so the
+// mapping stays a bijection.
 __device__ __forceinline__ Unit decode_unit(int u, int H, int tiles) {
   Unit r;
-  r.kv = u & 1;
+  r.kv = (u & 1) ^ ((gridDim.x & 1) ? 0 : static_cast<int>((u / gridDim.x) & 1));
   int rest = u >> 1;
   r.h = rest % H;
   rest /= H;
@@ -318,12 +345,28 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
       const uint64_t pol = policy_evict_first();
       uint32_t loaded = 0, empty_par = 0, full_cnt_par = 0;
       bool ok = true;
+      constexpr int kPrefetch = 4;   // source tiles pulled into L2 ahead of their TMA load
+      auto prefetch = [&](int u, int e) {
+        if (e >= P.n_loads) {
+          e -= P.n_loads;
+          u += gridDim.x;
+        }
+        if (u >= n_units) return;
+        const Unit pu = decode_unit(u, H, tiles);
+        const CUtensorMap* ptm = pu.kv ? &P.tm_v : &P.tm_k;
+        const int L = __ldg(&P.load_layer[e]);
+        tma_prefetch_5d(ptm, 0, pu.t0, pu.h, pu.b, L);
+        tma_prefetch_5d(ptm, 64, pu.t0, pu.h, pu.b, L);
+      };
+      if (blockIdx.x < n_units)
+        for (int e = 0; e < kPrefetch && e < P.n_loads; ++e) prefetch(blockIdx.x, e);
       for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
         const Unit un = decode_unit(u, H, tiles);
         const CUtensorMap* tm = un.kv ? &P.tm_v : &P.tm_k;
         for (int e = 0; e < P.n_loads; ++e) {
           const int s = __ldg(&P.load_slot[e]);
           const int L = __ldg(&P.load_layer[e]);
+          prefetch(u, e + kPrefetch);
           if ((loaded >> s) & 1u) {
             if (!wait_bar(smem_u32(&empty[s]), (empty_par >> s) & 1u, abort_flag, P.status)) {
               ok = false;
@@ -362,6 +405,13 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
                 !wait_bar(smem_u32(&wempty[st]), (round - 1) & 1u, abort_flag, P.status)) {
               ok = false;
               break;
+            }
+            // pull the same chunk of the next layer (or of the next unit's layer 0) into L2
+            if (l + 1 < Lt) {
+              tma_prefetch_2d(&P.tm_w, c * 64, (((l + 1) * 2 + un.kv) * H + un.h) * kD);
+            } else if (u + static_cast<int>(gridDim.x) < n_units) {
+              const Unit nu = decode_unit(u + gridDim.x, H, tiles);
+              tma_prefetch_2d(&P.tm_w, c * 64, (nu.kv * H + nu.h) * kD);
             }
             mbar_expect_tx(smem_u32(&wfull[st]), kWStageBytes);
             tma_load_2d(smem_u32(wst + static_cast<size_t>(st) * kWStageBytes), &P.tm_w,
@@ -446,6 +496,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     uint32_t full_par = 0, li = 0;
     float cs[32], sn[32];
     bool ok = true;
+    const uint64_t st_pol = policy_evict_first();
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
       const Unit un = decode_unit(u, H, tiles);
       const int t = un.t0 + r;
@@ -583,8 +634,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
                                           pack_bf16x2(ylo[j + 4], ylo[j + 5]), pack_bf16x2(ylo[j + 6], ylo[j + 7]));
               const uint4 v1 = make_uint4(pack_bf16x2(yhi[j], yhi[j + 1]), pack_bf16x2(yhi[j + 2], yhi[j + 3]),
                                           pack_bf16x2(yhi[j + 4], yhi[j + 5]), pack_bf16x2(yhi[j + 6], yhi[j + 7]));
-              *reinterpret_cast<uint4*>(out + 16 * rnd + j) = v0;
-              *reinterpret_cast<uint4*>(out + 64 + 16 * rnd + j) = v1;
+              st_global_stream(out + 16 * rnd + j, v0, st_pol);
+              st_global_stream(out + 64 + 16 * rnd + j, v1, st_pol);
             }
           }
         }
