@@ -180,6 +180,53 @@ KVX_API const char* kvx_status_string(kvx_status s);
 /* Thread-local description of the last error on this thread ("" if none). */
 KVX_API const char* kvx_last_error(void);
 
+/* ---- Mapping with no device allocation (the paper has no counterpart) -------------
+ *
+ * kvx_create allocates device memory (weight copies, tables, a status word).  Some
+ * callers cannot let a library do that: processes whose framework has reserved nearly
+ * all device memory for its own pool up front (so a cudaMalloc from a library fails or
+ * fragments the pool), and latency-critical serving paths that cannot afford the
+ * implicit device synchronisation of cudaMalloc / cudaFree.  kvx_map_noalloc serves them:
+ * the caller passes everything in its own buffers (caches, positions, W and bias on the
+ * device, the selection table on the host) and the library allocates nothing.  The map
+ * runs on the fp32 SIMT kernel, with the same results as kvx_map with KVX_KERNEL_SIMT.
+ *
+ * The little device memory it needs besides the caller's buffers -- a status word and a
+ * copy of the selection table -- lives in one fixed array inside libkvx
+ * (KVX_NOALLOC_SCRATCH_BYTES, kept by every GPU that loads the library until the process
+ * exits).  Consequences:
+ *  - The first call on a device looks up that array's device address (cudaGetSymbolAddress,
+ *    with the device made current); make that first call before any stream capture.
+ *  - Every call on a device shares the array: calls that may overlap on the GPU (other
+ *    streams, other host threads) race on it and must be serialised by the caller.  Each
+ *    call clears the status word and rewrites the selection copy before its launch.
+ *  - tgt_layers * k may not exceed KVX_NOALLOC_MAX_SELECTION (INVALID_ARG otherwise).
+ */
+#define KVX_NOALLOC_MAX_SELECTION 16384
+#define KVX_NOALLOC_SCRATCH_BYTES (256 + 4 * KVX_NOALLOC_MAX_SELECTION)
+
+typedef struct {
+  int32_t src_layers, tgt_layers, n_kv_heads, head_dim, k;
+  int32_t rope_style;          /* kvx_rope_style */
+  double src_rope_theta, tgt_rope_theta;
+  int32_t cache_dtype;         /* kvx_dtype of the caches */
+  int32_t weight_dtype;        /* kvx_dtype of W */
+  int32_t head_mix;            /* kvx_head_mix */
+  int32_t reserved;            /* must be 0 */
+  const int32_t* selection;    /* HOST [L_t][k], distinct layers in [0, L_s); row block j of W <-> selection[l][j] */
+  const void* W;               /* DEVICE [L_t][2][n_kv][F][d] in weight_dtype, 16-byte aligned */
+  const float* b;              /* DEVICE fp32 [L_t][2][n_kv][d] (pass zeros for no bias), 16-byte aligned */
+} kvx_noalloc_mapper;
+
+/* Map as kvx_map does, allocating nothing.  src, tgt, positions, batch and
+ * tokens_per_seq are as for kvx_map; `device` is the CUDA device that owns every pointer.
+ * Asynchronous on `stream` unless device_status is non-NULL: then the call waits for the
+ * stream and stores the device-detected status (KVX_OK, KVX_ERR_DEVICE_BOUNDS) there.
+ * Host-detected errors return before any launch. */
+KVX_API kvx_status kvx_map_noalloc(const kvx_noalloc_mapper* m, int device, const kvx_src* src,
+                                   int32_t batch, int32_t tokens_per_seq, const int32_t* positions,
+                                   const kvx_tgt* tgt, void* stream, int32_t* device_status);
+
 #ifdef __cplusplus
 }
 #endif

@@ -59,7 +59,7 @@ static float bf16_to_float(uint16_t v) {
   return f;
 }
 
-static void fill_rope(kvx_ctx* c) {
+void fill_rope(kvx_ctx* c) {
   const int half = c->d / 2;
   for (int i = 0; i < half; ++i) {
     const double e = -2.0 * i / c->d;

@@ -77,6 +77,9 @@ struct kvx_ctx {
 namespace kvx {
 void set_error(const std::string& msg);
 
+// Fills ctx->rope from ctx->d, ctx->theta_s and ctx->theta_t.
+void fill_rope(kvx_ctx* c);
+
 // SIMT fp32 kernel (any head_dim <= 256, fp32 or bf16 caches/weights, both layouts).
 kvx_status launch_simt(const kvx_ctx* ctx, const MapArgs& a, cudaStream_t stream);
 

@@ -54,11 +54,22 @@ class kvx_tgt(ctypes.Structure):
     ]
 
 
+class kvx_noalloc_mapper(ctypes.Structure):
+    _fields_ = [
+        ("src_layers", ctypes.c_int32), ("tgt_layers", ctypes.c_int32),
+        ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("k", ctypes.c_int32),
+        ("rope_style", ctypes.c_int32), ("src_rope_theta", ctypes.c_double),
+        ("tgt_rope_theta", ctypes.c_double), ("cache_dtype", ctypes.c_int32),
+        ("weight_dtype", ctypes.c_int32), ("head_mix", ctypes.c_int32), ("reserved", ctypes.c_int32),
+        ("selection", ctypes.c_void_p), ("W", ctypes.c_void_p), ("b", ctypes.c_void_p),
+    ]
+
+
 _lib = None
 
 EXPORTED = ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
             "kvx_set_kernel", "kvx_get_status", "kvx_mapper_params", "kvx_status_string",
-            "kvx_last_error")
+            "kvx_last_error", "kvx_map_noalloc")
 
 
 def lib():
@@ -84,8 +95,10 @@ def lib():
     L.kvx_status_string.restype = ctypes.c_char_p
     L.kvx_last_error.argtypes = []
     L.kvx_last_error.restype = ctypes.c_char_p
+    L.kvx_map_noalloc.argtypes = [ctypes.POINTER(kvx_noalloc_mapper), ctypes.c_int, ctypes.POINTER(kvx_src),
+                                  i32, i32, vp, ctypes.POINTER(kvx_tgt), vp, ctypes.POINTER(i32)]
     for name in ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
-                 "kvx_set_kernel", "kvx_get_status"):
+                 "kvx_set_kernel", "kvx_get_status", "kvx_map_noalloc"):
         getattr(L, name).restype = ctypes.c_int
     _lib = L
     return L
@@ -124,6 +137,17 @@ def kvx_create(cfg, device=0):
 def kvx_map(ctx, src, batch, tokens_per_seq, positions_ptr, tgt, stream=0):
     _check(lib().kvx_map(ctx, ctypes.byref(src), int(batch), int(tokens_per_seq), positions_ptr,
                          ctypes.byref(tgt), stream), "kvx_map")
+
+
+def kvx_map_noalloc(mapper, device, src, batch, tokens_per_seq, positions_ptr, tgt, stream=0,
+                    want_status=True):
+    """Map with no allocation by the library (see include/kvx.h).  Returns the device
+    status when ``want_status`` (the call then waits for the stream), else None."""
+    st = ctypes.c_int32(-1)
+    _check(lib().kvx_map_noalloc(ctypes.byref(mapper), int(device), ctypes.byref(src), int(batch),
+                                 int(tokens_per_seq), positions_ptr, ctypes.byref(tgt), stream,
+                                 ctypes.byref(st) if want_status else None), "kvx_map_noalloc")
+    return st.value if want_status else None
 
 
 def kvx_destroy(ctx):
