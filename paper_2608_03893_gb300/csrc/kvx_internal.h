@@ -41,7 +41,8 @@ struct MapArgs {
 // the same for every work unit (it depends only on the selection table).  Uses are the
 // (target layer l, selection j) pairs in l-major order.
 struct TcPlan {
-  int32_t n_slots = 0;                  // source-tile slots in shared memory
+  int32_t n_slots = 0;                  // source-tile slots (tensor memory)
+  int32_t n_land = 0;                   // source landing buffers in shared memory
   int32_t n_wst = 0;                    // W stages in shared memory
   int32_t n_loads = 0;                  // source-tile loads per work unit
   std::vector<int32_t> load_layer;      // [n_loads] source layer of load e

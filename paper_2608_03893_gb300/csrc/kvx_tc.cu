@@ -1,38 +1,48 @@
 // Tensor-core mapping kernel for sm_103a (tcgen05 + TMEM + TMA), bf16 caches and
-// weights, head_dim 128, per-head features, half-split RoPE pairs.
+// weights, head_dim 128, per-head features, half-split RoPE pairs, k <= 4.
 //
-// What it computes is Eq. ridge_kv with the Sec. 3.3 RoPE composition:
+// It computes Eq. ridge_kv with the Sec. 3.3 RoPE composition,
 //   K_t^{l,h} = R_t(t) ( [R_s(t)^-1 K_s^{sel[l][j]}[h]]_j W_K^{l,h} + b_K^{l,h} ),
 //   V_t^{l,h} =          [V_s^{sel[l][j]}[h]]_j W_V^{l,h} + b_V^{l,h},
 // with the stripped keys rounded to bf16 before the contraction and fp32 accumulation.
 //
-// Work unit = (sequence b, 128-token tile, head h, K|V).  A persistent CTA walks all
-// target layers of a unit.  The k source tiles a target layer concatenates are
-// 128 x 128 bf16 tiles in shared memory; a host-built schedule (Belady over the
-// sequence of (layer, j) uses) keeps every source tile resident for as long as later
-// target layers select it, so each source layer is read from HBM once per token tile
-// and shared by all target layers that select it (Sec. 3.2 selection is near
-// proportional depth, so a ring of k+1 slots almost never reloads).
+// Work unit = (sequence b, 128-token tile, head h, K|V).  A persistent CTA walks every
+// target layer of a unit.  The k source tiles a target layer concatenates are the A
+// operand of the contraction and live in tensor memory: four 64-column TMEM slots, each
+// holding a 128-token x 128-feature bf16 tile (lane = token, two features per column).
+// A host-built schedule (Belady over the sequence of (layer, j) uses) keeps every source
+// tile resident while later target layers still select it, so each source layer is
+// read from HBM once per token tile and shared by all target layers that select it.  A
+// slot is released as soon as the MMAs of its tile's last use complete, so the tile a
+// layer adds is written while the rest of the previous layer still computes.
 //
-// The contraction of target layer l is the GEMM D[128 tok x 128 ch] = X[128 x kd] W[kd x 128]
-// on tcgen05 (cta_group::1, M = N = 128, K = 16 per instruction), A = source slots
-// (K-major, 128-byte swizzle, as TMA lands them), B = W^T streamed through a ring of
-// 16 KB stages (128 output channels x 64 features), D = fp32 in TMEM, double buffered.
+// Contraction of target layer l: D[128 tok x 128 ch] = X[128 x kd] W[kd x 128] on tcgen05
+// (cta_group::1, M = N = 128, K = 16 per instruction: the full-rate shape), A from TMEM,
+// B = W^T from a ring of 16 KB shared-memory stages (128 output channels x 64 features,
+// 128-byte swizzle), D in one of two 128-column fp32 TMEM accumulators.
 //
 // Warp roles (384 threads):
-//   warp 0      TMA producer of source tiles (one thread)
-//   warp 1      MMA issuer (one thread)
-//   warp 2      TMEM allocator
-//   warp 3      TMA producer of W stages (one thread)
-//   warps 4-11  two "transform" warpgroups.  Thread (group g, row r) owns token row r
-//               (= TMEM lane r) and RoPE pairs i in [32g, 32g+32) (channels i, i+64):
-//               it strips the source RoPE from key tiles in place (fp32, round to
-//               bf16) and runs the epilogue (TMEM -> registers, + bias, target RoPE for
-//               keys, bf16, 16-byte global stores, contiguous or paged).
+//   warp 0      TMA producer of raw source tiles into shared-memory landing buffers
+//               (plus TMA L2 prefetch of tiles a few loads ahead)
+//   warp 1      TMEM allocator (all 512 columns) and MMA issuer (one thread)
+//   warp 2      TMA producer of W^T stages and of each layer's bias row (plus L2
+//               prefetch of the next layer's W)
+//   warp 3      idle
+//   warps 4-11  two transform warpgroups (one warp per TMEM lane quarter, warp % 4).
+//               Thread (group g, row r) owns token row r (= TMEM lane r) and the 32 RoPE
+//               pairs 32g .. 32g+31 (channels i and i + 64).
+//               Prologue: landing buffer -> registers -> (keys) strip the source RoPE in
+//               fp32, round to bf16 -> tcgen05.st into the tile's TMEM slot.
+//               Epilogue: TMEM -> registers, + bias, (keys) target RoPE, bf16, into a
+//               double-buffered shared-memory staging tile written out by a TMA store
+//               (contiguous targets), or 16-byte stores through the block table (paged).
+//               Transform thread 0 issues the TMA stores; a staged tile holding a row
+//               with an out-of-range position is instead written row by row by its warp,
+//               skipping the bad rows.
 //
-// Every mbarrier wait is bounded: after kTimeoutNs the kernel raises KVX_ERR_TIMEOUT
-// in the status word, sets a shared abort flag that every role polls, waits (again
-// bounded) for its own TMA copies and MMAs in flight, frees TMEM and returns.
+// Every mbarrier wait is bounded: after 4 s the kernel raises KVX_ERR_TIMEOUT in the
+// status word, sets a shared abort flag that every role polls, waits (again bounded)
+// for its own TMA copies and MMAs in flight, frees TMEM and returns.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
@@ -44,224 +54,51 @@
 #include <vector>
 
 #include "kvx_internal.h"
+#include "kvx_ptx.cuh"
 #include "kvx_rope.cuh"
 
 namespace kvx {
 namespace {
 
+using namespace ptx;
+
 constexpr int kThreads = 384;
-constexpr int kTileM = 128;                      // tokens per work unit
-constexpr int kD = 128;                          // head_dim of this kernel
-constexpr uint32_t kSlotBytes = kTileM * kD * 2; // 32 KB: two 64-column SW128 halves
-constexpr uint32_t kHalfBytes = kSlotBytes / 2;  // 16 KB
-constexpr uint32_t kWStageBytes = 128 * 64 * 2;  // 16 KB: 128 channels x 64 features
-constexpr int kMaxSlots = 8;
+constexpr int kFirstTransformWarp = 4;
+constexpr int kTileM = 128;                         // tokens per work unit
+constexpr int kD = 128;                             // head_dim of this kernel
+constexpr uint32_t kLandBytes = kTileM * kD * 2;    // 32 KB raw tile: two 64-column SW128 halves
+constexpr uint32_t kHalfBytes = kLandBytes / 2;     // 16 KB
+constexpr uint32_t kWStageBytes = kD * 64 * 2;      // 16 KB: 128 output channels x 64 features
+constexpr uint32_t kOutBytes = kTileM * kD * 2;     // 32 KB staging tile (two SW128 boxes)
+constexpr int kOutBufs = 2;
+constexpr int kTSlots = 4;                          // TMEM source-tile slots (64 columns each)
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kAccCols = 128;                  // one fp32 accumulator
+constexpr int kAccBufs = 2;
+constexpr uint32_t kSlotCol0 = kAccBufs * kAccCols; // 256: first source-slot column
+constexpr int kLand = 2;                            // landing buffers
 constexpr int kMaxWStages = 8;
-constexpr uint32_t kTmemCols = 256;              // two 128-column fp32 accumulators
-constexpr uint64_t kTimeoutNs = 4000000000ull;   // 4 s
-constexpr size_t kSmemLimit = 232448;            // 227 KB opt-in per CTA
+constexpr int kSrcPrefetch = 6;                     // source loads prefetched into L2 ahead
+constexpr int kBiasSlots = 4;                       // per-layer bias rows staged ahead (512 B each)
+constexpr uint32_t kBiasBytes = kD * 4;
+constexpr size_t kSmemLimit = 232448;               // 227 KB opt-in per CTA
 
 struct TcParams {
-  CUtensorMap tm_k;   // source keys   [L_s][B][H][T][128] bf16, box 64 x 128
-  CUtensorMap tm_v;   // source values
-  CUtensorMap tm_w;   // W^T           [L_t*2*H*128][F] bf16, box 64 x 128
+  CUtensorMap tm_k;      // source keys   [L_s][B][H][T][128] bf16, box 64 x 128
+  CUtensorMap tm_v;      // source values
+  CUtensorMap tm_w;      // W^T [L_t*2*H*128][F] bf16, box 64 x 128
+  CUtensorMap tm_out_k;  // target keys   [L_t][B][H][T][128] bf16, box 64 x 128 (contiguous only)
+  CUtensorMap tm_out_v;  // target values
   MapArgs a;
-  const int32_t* load_layer;   // [n_loads]
-  const int32_t* load_slot;    // [n_loads]
+  const int32_t* load_layer;   // [n_loads] source layer of load e
+  const int32_t* load_slot;    // [n_loads] TMEM slot
   const int32_t* load_first;   // [n_loads] first target layer using the load
-  const int32_t* use_slot;     // [L_t*k]
-  const int32_t* use_flags;    // [L_t*k] bit 0: first use of a load; bit 1: release after
+  const uint32_t* use_pack;    // [L_t] per use j: 5 bits at 5j = slot | 8 first use | 16 release after
   const float* bias;           // [L_t][2][H][128] fp32
   int32_t* status;
-  int32_t Lt, H, k, n_slots, n_wst, n_loads, tiles_per_seq, n_units, same_theta;
+  int32_t Lt, H, k, n_wst, n_loads, tiles_per_seq, n_units, same_theta;
   RopeTables rope;
 };
-
-// ------------------------------------------------------------------ PTX wrappers --
-
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-               : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ uint32_t mbar_try_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok;
-}
-
-__device__ __forceinline__ uint64_t global_timer() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-
-// Bounded wait for the phase of the given parity.  false = timed out or aborted.
-__device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile uint32_t* abort_flag,
-                                         int32_t* status) {
-  if (mbar_try_wait(bar, parity)) return true;
-  uint64_t t0 = 0;
-  for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 127u) == 0) {
-      if (*abort_flag) return false;
-      const uint64_t now = global_timer();
-      if (t0 == 0) {
-        t0 = now;
-      } else if (now - t0 > kTimeoutNs) {
-        *abort_flag = 1u;
-        atomicCAS(status, 0, KVX_ERR_TIMEOUT);
-        return false;
-      }
-    }
-  }
-}
-
-// Teardown wait: ignores the abort flag, still bounded in time.
-__device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
-  const uint64_t t0 = global_timer();
-  while (!mbar_try_wait(bar, parity))
-    if (global_timer() - t0 > kTimeoutNs) break;
-}
-
-__device__ __forceinline__ uint64_t policy_evict_first() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-
-__device__ __forceinline__ uint64_t policy_evict_last() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-
-__device__ __forceinline__ void tma_load_5d(uint32_t dst, const CUtensorMap* map, uint32_t bar, int c0,
-                                            int c1, int c2, int c3, int c4, uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.5d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1, {%2, %3, %4, %5, %6}], [%7], %8;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4), "r"(bar),
-      "l"(policy)
-      : "memory");
-}
-
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar, int c0,
-                                            int c1, uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar), "l"(policy)
-      : "memory");
-}
-
-// L2 prefetch of one tensor-map tile (no shared memory, no barrier).
-__device__ __forceinline__ void tma_prefetch_5d(const CUtensorMap* map, int c0, int c1, int c2, int c3, int c4) {
-  asm volatile("cp.async.bulk.prefetch.tensor.5d.L2.global.tile [%0, {%1, %2, %3, %4, %5}];" ::"l"(
-                   reinterpret_cast<uint64_t>(map)),
-               "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4)
-               : "memory");
-}
-
-__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int c0, int c1) {
-  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
-                   reinterpret_cast<uint64_t>(map)),
-               "r"(c0), "r"(c1)
-               : "memory");
-}
-
-// 16-byte global store that bypasses L1 and is marked evict-first in L2 (the target
-// cache is written once and not read by this kernel).
-__device__ __forceinline__ void st_global_stream(void* ptr, uint4 v, uint64_t policy) {
-  asm volatile("st.global.L1::no_allocate.L2::cache_hint.v4.b32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(ptr),
-               "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "l"(policy)
-               : "memory");
-}
-
-__device__ __forceinline__ void tc_fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-
-__device__ __forceinline__ void tc_commit(uint32_t bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-               : "memory");
-}
-
-__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
-                                       uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
-// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row core groups 1024 B
-// apart (stride byte offset), leading byte offset unused for this layout (1), descriptor
-// version 1 (bits 46-47), swizzle mode 2 = 128B (bits 61-63).  Tiles are 1024-aligned.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-  return static_cast<uint64_t>((saddr >> 4) & 0x3FFFu) | (static_cast<uint64_t>(1) << 16) |
-         (static_cast<uint64_t>(1024 >> 4) << 32) | (static_cast<uint64_t>(1) << 46) |
-         (static_cast<uint64_t>(2) << 61);
-}
-
-// Instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1), B bf16 (bits
-// 10-12 = 1), both K-major, N >> 3 at bits 17-22, M >> 4 at bits 24-28.
-__host__ __device__ constexpr uint32_t make_idesc(int M, int N) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(N >> 3) << 17) |
-         (static_cast<uint32_t>(M >> 4) << 24);
-}
-
-// Two 16-column TMEM loads (32 lanes x 32 bit each) and the wait, in one asm block so
-// the registers are complete when it returns.
-__device__ __forceinline__ void tmem_ld_2x16(uint32_t taddr_lo, uint32_t taddr_hi, uint32_t (&lo)[16],
-                                             uint32_t (&hi)[16]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%32];\n\t"
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-      "{%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%33];\n\t"
-      "tcgen05.wait::ld.sync.aligned;"
-      : "=r"(lo[0]), "=r"(lo[1]), "=r"(lo[2]), "=r"(lo[3]), "=r"(lo[4]), "=r"(lo[5]), "=r"(lo[6]),
-        "=r"(lo[7]), "=r"(lo[8]), "=r"(lo[9]), "=r"(lo[10]), "=r"(lo[11]), "=r"(lo[12]), "=r"(lo[13]),
-        "=r"(lo[14]), "=r"(lo[15]), "=r"(hi[0]), "=r"(hi[1]), "=r"(hi[2]), "=r"(hi[3]), "=r"(hi[4]),
-        "=r"(hi[5]), "=r"(hi[6]), "=r"(hi[7]), "=r"(hi[8]), "=r"(hi[9]), "=r"(hi[10]), "=r"(hi[11]),
-        "=r"(hi[12]), "=r"(hi[13]), "=r"(hi[14]), "=r"(hi[15])
-      : "r"(taddr_lo), "r"(taddr_hi)
-      : "memory");
-}
-
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
-  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<const uint32_t*>(&v);
-}
-
-__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
-
-__device__ __forceinline__ void report(int32_t* status, int code) { atomicCAS(status, 0, code); }
 
 struct Unit {
   int b, t0, h, kv;
@@ -282,51 +119,72 @@ __device__ __forceinline__ Unit decode_unit(int u, int H, int tiles) {
   return r;
 }
 
+__device__ __forceinline__ void report(int32_t* status, int code) { atomicCAS(status, 0, code); }
+
 // ------------------------------------------------------------------------ kernel --
 
 __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_constant__ TcParams P) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const int S = P.n_slots, NW = P.n_wst;
-  uint8_t* slots = smem;
-  uint8_t* wst = smem + static_cast<size_t>(S) * kSlotBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(wst + static_cast<size_t>(NW) * kWStageBytes);
-  uint64_t* full = bars;                  // [S] TMA landed
-  uint64_t* ready = full + S;             // [S] keys stripped (K units)
-  uint64_t* empty = ready + S;            // [S] slot released by the MMA
-  uint64_t* wfull = empty + S;            // [NW]
-  uint64_t* wempty = wfull + NW;          // [NW]
-  uint64_t* accf = wempty + NW;           // [2]
-  uint64_t* acce = accf + 2;              // [2]
-  uint64_t* drain = acce + 2;             // [1]
+  const int NW = P.n_wst;
+  uint8_t* land = smem;
+  uint8_t* wst = land + kLand * kLandBytes;
+  uint8_t* outst = wst + static_cast<size_t>(NW) * kWStageBytes;
+  float* bias_ring = reinterpret_cast<float*>(outst + kOutBufs * kOutBytes);   // [4][128] fp32
+  uint64_t* bars = reinterpret_cast<uint64_t*>(bias_ring + kBiasSlots * kD);
+  uint64_t* land_full = bars;                    // [2] TMA landed
+  uint64_t* land_empty = land_full + kLand;      // [2] transform read it (8 warps)
+  uint64_t* tready = land_empty + kLand;         // [4] TMEM tile written (8 warps)
+  uint64_t* tfree = tready + kTSlots;            // [4] TMEM tile released by the MMA
+  uint64_t* wfull = tfree + kTSlots;             // [NW]
+  uint64_t* wempty = wfull + NW;                 // [NW]
+  uint64_t* accf = wempty + NW;                  // [2] accumulator ready
+  uint64_t* acce = accf + kAccBufs;              // [2] accumulator drained (8 warps)
+  uint64_t* stage_full = acce + kAccBufs;        // [2] staging tile written (8 warps)
+  uint64_t* stage_free = stage_full + kOutBufs;  // [2] staging tile read by its store
+  uint64_t* bias_full = stage_free + kOutBufs;   // [4] bias row landed
+  uint64_t* bias_empty = bias_full + kBiasSlots; // [4] bias row used (8 warps)
+  uint64_t* drain = bias_empty + kBiasSlots;     // [1]
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
   volatile uint32_t* abort_flag = tmem_holder + 1;
+  uint32_t* bad_mask = tmem_holder + 2;          // [2][4] rows of a staged tile with a bad position
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < S; ++s) {
-      mbar_init(smem_u32(&full[s]), 1);
-      mbar_init(smem_u32(&ready[s]), 8);
-      mbar_init(smem_u32(&empty[s]), 1);
+    for (int i = 0; i < kLand; ++i) {
+      mbar_init(smem_u32(&land_full[i]), 1);
+      mbar_init(smem_u32(&land_empty[i]), 8);
     }
-    for (int s = 0; s < NW; ++s) {
-      mbar_init(smem_u32(&wfull[s]), 1);
-      mbar_init(smem_u32(&wempty[s]), 1);
+    for (int i = 0; i < kTSlots; ++i) {
+      mbar_init(smem_u32(&tready[i]), 8);
+      mbar_init(smem_u32(&tfree[i]), 1);
     }
-    for (int a = 0; a < 2; ++a) {
-      mbar_init(smem_u32(&accf[a]), 1);
-      mbar_init(smem_u32(&acce[a]), 8);
+    for (int i = 0; i < NW; ++i) {
+      mbar_init(smem_u32(&wfull[i]), 1);
+      mbar_init(smem_u32(&wempty[i]), 1);
+    }
+    for (int i = 0; i < kAccBufs; ++i) {
+      mbar_init(smem_u32(&accf[i]), 1);
+      mbar_init(smem_u32(&acce[i]), 8);
+    }
+    for (int i = 0; i < kOutBufs; ++i) {
+      mbar_init(smem_u32(&stage_full[i]), 8);
+      mbar_init(smem_u32(&stage_free[i]), 1);
+    }
+    for (int i = 0; i < kBiasSlots; ++i) {
+      mbar_init(smem_u32(&bias_full[i]), 1);
+      mbar_init(smem_u32(&bias_empty[i]), 8);
     }
     mbar_init(smem_u32(drain), 1);
     *abort_flag = 0u;
+    for (int i = 0; i < 2 * 4; ++i) bad_mask[i] = 0u;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    fence_proxy_async_smem();
   }
-  if (warp == 2) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                     smem_u32(tmem_holder)),
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_holder)),
                  "r"(kTmemCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
@@ -343,11 +201,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     // ------------------------------------------------ source-tile producer --------
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
-      uint32_t loaded = 0, empty_par = 0, full_cnt_par = 0;
+      uint32_t gl = 0;
       bool ok = true;
-      constexpr int kPrefetch = 4;   // source tiles pulled into L2 ahead of their TMA load
       auto prefetch = [&](int u, int e) {
-        if (e >= P.n_loads) {
+        while (e >= P.n_loads) {
           e -= P.n_loads;
           u += gridDim.x;
         }
@@ -358,155 +215,162 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
         tma_prefetch_5d(ptm, 0, pu.t0, pu.h, pu.b, L);
         tma_prefetch_5d(ptm, 64, pu.t0, pu.h, pu.b, L);
       };
-      if (blockIdx.x < n_units)
-        for (int e = 0; e < kPrefetch && e < P.n_loads; ++e) prefetch(blockIdx.x, e);
+      if (static_cast<int>(blockIdx.x) < n_units)
+        for (int e = 0; e < kSrcPrefetch; ++e) prefetch(blockIdx.x, e);
       for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
         const Unit un = decode_unit(u, H, tiles);
         const CUtensorMap* tm = un.kv ? &P.tm_v : &P.tm_k;
-        for (int e = 0; e < P.n_loads; ++e) {
-          const int s = __ldg(&P.load_slot[e]);
+        for (int e = 0; e < P.n_loads; ++e, ++gl) {
+          prefetch(u, e + kSrcPrefetch);
+          const int lb = gl % kLand;
+          const uint32_t round = gl / kLand;
+          if (round > 0 && !wait_bar(smem_u32(&land_empty[lb]), (round - 1) & 1u, abort_flag, P.status,
+                                     KVX_ERR_TIMEOUT)) {
+            ok = false;
+            break;
+          }
           const int L = __ldg(&P.load_layer[e]);
-          prefetch(u, e + kPrefetch);
-          if ((loaded >> s) & 1u) {
-            if (!wait_bar(smem_u32(&empty[s]), (empty_par >> s) & 1u, abort_flag, P.status)) {
+          const uint32_t dst = smem_u32(land + static_cast<size_t>(lb) * kLandBytes);
+          mbar_expect_tx(smem_u32(&land_full[lb]), kLandBytes);
+          tma_load_5d(dst, tm, smem_u32(&land_full[lb]), 0, un.t0, un.h, un.b, L, pol);
+          tma_load_5d(dst + kHalfBytes, tm, smem_u32(&land_full[lb]), 64, un.t0, un.h, un.b, L, pol);
+        }
+      }
+      if (!ok) {  // the last min(gl, kLand) landing buffers may still be filling
+        const uint32_t first = gl > static_cast<uint32_t>(kLand) ? gl - kLand : 0;
+        for (uint32_t i = first; i < gl; ++i) drain_wait(smem_u32(&land_full[i % kLand]), (i / kLand) & 1u);
+      }
+    }
+  } else if (warp == 2) {
+    // --------------------------------------------------- W and bias producer ------
+    if (lane == 0) {
+      const uint64_t pol = policy_evict_last();
+      uint32_t wi = 0, bl = 0;
+      bool ok = true;
+      const int chunks = 2 * k;  // 64-feature chunks of F = 128 k
+      for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+        const Unit un = decode_unit(u, H, tiles);
+        for (int l = 0; ok && l < Lt; ++l, ++bl) {
+          const int row0 = ((l * 2 + un.kv) * H + un.h) * kD;
+          {  // this layer's bias row into the bias ring
+            const int bs = bl % kBiasSlots;
+            const uint32_t round = bl / kBiasSlots;
+            if (round > 0 &&
+                !wait_bar(smem_u32(&bias_empty[bs]), (round - 1) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
               ok = false;
               break;
             }
-            empty_par ^= 1u << s;
+            mbar_expect_tx(smem_u32(&bias_full[bs]), kBiasBytes);
+            bulk_load(smem_u32(bias_ring + bs * kD), P.bias + static_cast<size_t>(row0), kBiasBytes,
+                      smem_u32(&bias_full[bs]));
           }
-          const uint32_t dst = smem_u32(slots + static_cast<size_t>(s) * kSlotBytes);
-          mbar_expect_tx(smem_u32(&full[s]), kSlotBytes);
-          tma_load_5d(dst, tm, smem_u32(&full[s]), 0, un.t0, un.h, un.b, L, pol);
-          tma_load_5d(dst + kHalfBytes, tm, smem_u32(&full[s]), 64, un.t0, un.h, un.b, L, pol);
-          loaded |= 1u << s;
-          full_cnt_par ^= 1u << s;
-        }
-      }
-      if (!ok) {  // wait for the copies still in flight into each slot
-        for (int s = 0; s < S; ++s)
-          if ((loaded >> s) & 1u) drain_wait(smem_u32(&full[s]), ((full_cnt_par >> s) & 1u) ^ 1u);
-      }
-    }
-  } else if (warp == 3) {
-    // ------------------------------------------------------------ W producer ------
-    if (lane == 0) {
-      const uint64_t pol = policy_evict_last();
-      uint32_t wi = 0;
-      bool ok = true;
-      const int chunks = 2 * k;
-      for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-        const Unit un = decode_unit(u, H, tiles);
-        for (int l = 0; ok && l < Lt; ++l) {
-          const int row0 = ((l * 2 + un.kv) * H + un.h) * kD;
+          int next_row0 = -1;
+          if (l + 1 < Lt) {
+            next_row0 = (((l + 1) * 2 + un.kv) * H + un.h) * kD;
+          } else if (u + static_cast<int>(gridDim.x) < n_units) {
+            const Unit nu = decode_unit(u + gridDim.x, H, tiles);
+            next_row0 = (nu.kv * H + nu.h) * kD;
+          }
           for (int c = 0; c < chunks; ++c, ++wi) {
             const int st = wi % NW;
             const uint32_t round = wi / NW;
             if (round > 0 &&
-                !wait_bar(smem_u32(&wempty[st]), (round - 1) & 1u, abort_flag, P.status)) {
+                !wait_bar(smem_u32(&wempty[st]), (round - 1) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
               ok = false;
               break;
             }
-            // pull the same chunk of the next layer (or of the next unit's layer 0) into L2
-            if (l + 1 < Lt) {
-              tma_prefetch_2d(&P.tm_w, c * 64, (((l + 1) * 2 + un.kv) * H + un.h) * kD);
-            } else if (u + static_cast<int>(gridDim.x) < n_units) {
-              const Unit nu = decode_unit(u + gridDim.x, H, tiles);
-              tma_prefetch_2d(&P.tm_w, c * 64, (nu.kv * H + nu.h) * kD);
-            }
+            if (next_row0 >= 0) tma_prefetch_2d(&P.tm_w, c * 64, next_row0);
             mbar_expect_tx(smem_u32(&wfull[st]), kWStageBytes);
-            tma_load_2d(smem_u32(wst + static_cast<size_t>(st) * kWStageBytes), &P.tm_w,
-                        smem_u32(&wfull[st]), c * 64, row0, pol);
+            tma_load_2d(smem_u32(wst + static_cast<size_t>(st) * kWStageBytes), &P.tm_w, smem_u32(&wfull[st]),
+                        c * 64, row0, pol);
           }
         }
       }
       if (!ok) {
-        // the last min(wi, NW) stages may still be landing
         const uint32_t first = wi > static_cast<uint32_t>(NW) ? wi - NW : 0;
         for (uint32_t i = first; i < wi; ++i) drain_wait(smem_u32(&wfull[i % NW]), (i / NW) & 1u);
+        const uint32_t bfirst = bl > static_cast<uint32_t>(kBiasSlots) ? bl - kBiasSlots : 0;
+        for (uint32_t i = bfirst; i < bl; ++i) drain_wait(smem_u32(&bias_full[i % kBiasSlots]), (i / kBiasSlots) & 1u);
       }
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA ---------
     if (lane == 0) {
       constexpr uint32_t idesc = make_idesc(kTileM, kD);
-      uint32_t full_par = 0, ready_par = 0, wi = 0, li = 0;
+      uint32_t ready_par = 0, wi = 0, li = 0;
       bool ok = true, issued = false;
+      uint32_t pack_next = __ldg(&P.use_pack[0]);
       for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-        const Unit un = decode_unit(u, H, tiles);
         for (int l = 0; ok && l < Lt; ++l, ++li) {
-          const uint32_t a = li & 1u;
-          if (li >= 2 && !wait_bar(smem_u32(&acce[a]), ((li >> 1) - 1) & 1u, abort_flag, P.status)) {
+          const uint32_t pack = pack_next;
+          pack_next = __ldg(&P.use_pack[l + 1 < Lt ? l + 1 : 0]);   // schedule word of the next layer
+          const uint32_t buf = li & 1u;
+          if (li >= 2 && !wait_bar(smem_u32(&acce[buf]), ((li >> 1) - 1) & 1u, abort_flag, P.status,
+                                   KVX_ERR_TIMEOUT)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t d_tmem = tmem_base + a * kD;
+          const uint32_t d_tmem = tmem_base + buf * kAccCols;
           for (int j = 0; ok && j < k; ++j) {
-            const int s = __ldg(&P.use_slot[l * k + j]);
-            const int fl = __ldg(&P.use_flags[l * k + j]);
-            if (fl & 1) {
-              bool w_ok;
-              if (un.kv == 0) {
-                w_ok = wait_bar(smem_u32(&ready[s]), (ready_par >> s) & 1u, abort_flag, P.status);
-                ready_par ^= 1u << s;
-              } else {
-                w_ok = wait_bar(smem_u32(&full[s]), (full_par >> s) & 1u, abort_flag, P.status);
-              }
-              full_par ^= 1u << s;
-              if (!w_ok) {
+            const uint32_t f = (pack >> (5 * j)) & 31u;
+            const uint32_t s = f & 7u;
+            if (f & 8u) {  // first use of the tile: wait until the transform wrote it
+              if (!wait_bar(smem_u32(&tready[s]), (ready_par >> s) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
                 ok = false;
                 break;
               }
+              ready_par ^= 1u << s;
               tc_fence_after();
             }
-            const uint32_t a_base = smem_u32(slots + static_cast<size_t>(s) * kSlotBytes);
-            for (int half = 0; half < 2; ++half, ++wi) {
+            const uint32_t a_col = tmem_base + kSlotCol0 + s * 64;
+            for (int c2 = 0; c2 < 2; ++c2, ++wi) {
               const int st = wi % NW;
-              if (!wait_bar(smem_u32(&wfull[st]), (wi / NW) & 1u, abort_flag, P.status)) {
+              if (!wait_bar(smem_u32(&wfull[st]), (wi / NW) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
                 ok = false;
                 break;
               }
-              tc_fence_after();
               const uint32_t b_base = smem_u32(wst + static_cast<size_t>(st) * kWStageBytes);
 #pragma unroll
-              for (int kk = 0; kk < 4; ++kk) {
-                tc_mma(d_tmem, sw128_desc(a_base + half * kHalfBytes + kk * 32), sw128_desc(b_base + kk * 32),
-                       idesc, (j | half | kk) != 0);
-              }
+              for (int kk = 0; kk < 4; ++kk)
+                tc_mma_ts(d_tmem, a_col + c2 * 32 + kk * 8, sw128_desc(b_base + kk * 32), idesc, (j | c2 | kk) != 0);
               issued = true;
               tc_commit(smem_u32(&wempty[st]));
             }
-            if (ok && (fl & 2)) tc_commit(smem_u32(&empty[s]));
+            if (ok && (f & 16u)) tc_commit(smem_u32(&tfree[s]));   // last use before a reload
           }
-          if (ok) tc_commit(smem_u32(&accf[a]));
+          if (ok) tc_commit(smem_u32(&accf[buf]));
         }
       }
-      // make sure every MMA (and every commit) has completed before TMEM is freed
+      // every MMA (and every commit) must have completed before TMEM is freed
       if (issued || !ok) {
         tc_commit(smem_u32(drain));
         drain_wait(smem_u32(drain), 0);
       }
     }
-  } else if (warp >= 4) {
+  } else if (warp >= kFirstTransformWarp) {
     // ------------------------------------------------------- transform warps ------
-    const int g = (warp - 4) >> 2;          // column group: pairs [32g, 32g+32)
-    const int q = warp & 3;                 // TMEM lane quarter
-    const int r = q * 32 + lane;            // token row within the tile
+    const int g = (warp - kFirstTransformWarp) >> 2; // pair group: pairs 32g .. 32g+31
+    const int q = warp & 3;                          // TMEM lane quarter this warp may access
+    const int r = q * 32 + lane;                     // token row within the tile
     const uint32_t lane_addr = static_cast<uint32_t>(q * 32) << 16;
-    uint32_t full_par = 0, li = 0;
+    const uint64_t st_pol = policy_evict_first();
+    uint32_t gl = 0, lay = 0, tl_loaded = 0, tfree_par = 0;
+    bool prev_store_pending = false;   // first transform warp: the previous layer's TMA store may still read its buffer
     float cs[32], sn[32];
     bool ok = true;
-    const uint64_t st_pol = policy_evict_first();
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
       const Unit un = decode_unit(u, H, tiles);
       const int t = un.t0 + r;
       bool valid = t < A.T;
+      bool bad = false;
       int p = 0;
       if (valid) {
         p = __ldg(&A.pos[static_cast<int64_t>(un.b) * A.T + t]);
         if (p < 0 || p >= (1 << 24)) {
           report(P.status, KVX_ERR_DEVICE_BOUNDS);
           valid = false;
+          bad = true;
           p = 0;
         }
       }
@@ -516,7 +380,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           row_off = un.b * A.ts[1] + un.h * A.ts[2] + static_cast<int64_t>(t) * A.ts[3];
         } else {
           const int lb = p / A.block_size;
-          const int blk = lb < A.max_blocks ? __ldg(&A.block_table[static_cast<int64_t>(un.b) * A.max_blocks + lb]) : -1;
+          const int blk =
+              lb < A.max_blocks ? __ldg(&A.block_table[static_cast<int64_t>(un.b) * A.max_blocks + lb]) : -1;
           if (blk < 0 || blk >= A.n_blocks) {
             report(P.status, KVX_ERR_DEVICE_BOUNDS);
             valid = false;
@@ -526,127 +391,250 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           }
         }
       }
+      const bool use_tma = !A.paged;   // contiguous targets: staged tiles + TMA stores
       if (un.kv == 0) {
 #pragma unroll
-        for (int j = 0; j < 32; ++j)
-          rope_sincos(p, P.rope.wt_hi[32 * g + j], P.rope.wt_lo[32 * g + j], P.rope.two_pi_hi,
-                      P.rope.two_pi_lo, P.rope.inv_two_pi, &sn[j], &cs[j]);
+        for (int m = 0; m < 32; ++m) {
+          const int i = 32 * g + m;
+          rope_sincos(p, P.rope.wt_hi[i], P.rope.wt_lo[i], P.rope.two_pi_hi, P.rope.two_pi_lo, P.rope.inv_two_pi,
+                      &sn[m], &cs[m]);
+        }
       }
       __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(un.kv ? A.tgt_v : A.tgt_k);
+      const CUtensorMap* tm_out = un.kv ? &P.tm_out_v : &P.tm_out_k;
       int e = 0;
-      for (int l = 0; ok && l < Lt; ++l, ++li) {
-        // strip the key tiles that layer l + 1 needs first
+      for (int l = 0; ok && l < Lt; ++l, ++lay) {
+        // prologue: the source tiles whose first use is at most layer l + 1
         while (e < P.n_loads && __ldg(&P.load_first[e]) <= l + 1) {
-          const int s = __ldg(&P.load_slot[e]);
+          const int lb = gl % kLand;
+          bool w_ok = wait_bar(smem_u32(&land_full[lb]), (gl / kLand) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT);
+          if (!__all_sync(0xffffffffu, w_ok)) {
+            ok = false;
+            break;
+          }
+          uint32_t wa[16], wb[16];   // a: features 32g + [0,32) of the pairs, b: features + 64
+          {
+            const uint8_t* row = land + static_cast<size_t>(lb) * kLandBytes + r * 128;
+#pragma unroll
+            for (int ci = 0; ci < 4; ++ci) {
+              const int phys = ((4 * g + ci) ^ (r & 7)) << 4;
+              const uint4 va = *reinterpret_cast<const uint4*>(row + phys);
+              const uint4 vb = *reinterpret_cast<const uint4*>(row + kHalfBytes + phys);
+              wa[4 * ci] = va.x;
+              wa[4 * ci + 1] = va.y;
+              wa[4 * ci + 2] = va.z;
+              wa[4 * ci + 3] = va.w;
+              wb[4 * ci] = vb.x;
+              wb[4 * ci + 1] = vb.y;
+              wb[4 * ci + 2] = vb.z;
+              wb[4 * ci + 3] = vb.w;
+            }
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&land_empty[lb]));
+          ++gl;
           if (un.kv == 0) {
-            const bool w_ok = wait_bar(smem_u32(&full[s]), (full_par >> s) & 1u, abort_flag, P.status);
+#pragma unroll
+            for (int w = 0; w < 16; ++w) {
+              const int m0 = 2 * w, m1 = 2 * w + 1;
+              float c0, s0, c1, s1;
+              if (P.same_theta) {
+                c0 = cs[m0];
+                s0 = sn[m0];
+                c1 = cs[m1];
+                s1 = sn[m1];
+              } else {
+                const int i0 = 32 * g + m0, i1 = 32 * g + m1;
+                rope_sincos(p, P.rope.ws_hi[i0], P.rope.ws_lo[i0], P.rope.two_pi_hi, P.rope.two_pi_lo,
+                            P.rope.inv_two_pi, &s0, &c0);
+                rope_sincos(p, P.rope.ws_hi[i1], P.rope.ws_lo[i1], P.rope.two_pi_hi, P.rope.two_pi_lo,
+                            P.rope.inv_two_pi, &s1, &c1);
+              }
+              const float a0 = bf16_lo(wa[w]), a1 = bf16_hi(wa[w]);
+              const float b0 = bf16_lo(wb[w]), b1 = bf16_hi(wb[w]);
+              // rotation by -t*omega: a' = a c + b s, b' = b c - a s
+              wa[w] = pack_bf16x2(__fmaf_rn(a0, c0, __fmul_rn(b0, s0)), __fmaf_rn(a1, c1, __fmul_rn(b1, s1)));
+              wb[w] = pack_bf16x2(__fmaf_rn(b0, c0, -__fmul_rn(a0, s0)), __fmaf_rn(b1, c1, -__fmul_rn(a1, s1)));
+            }
+          }
+          const int s = __ldg(&P.load_slot[e]);
+          if ((tl_loaded >> s) & 1u) {
+            w_ok = wait_bar(smem_u32(&tfree[s]), (tfree_par >> s) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT);
+            tfree_par ^= 1u << s;
             if (!__all_sync(0xffffffffu, w_ok)) {
               ok = false;
               break;
             }
-            uint8_t* row = slots + static_cast<size_t>(s) * kSlotBytes + r * 128;
-#pragma unroll
-            for (int c4 = 0; c4 < 4; ++c4) {
-              const int phys = ((4 * g + c4) ^ (r & 7)) << 4;
-              uint4* pa = reinterpret_cast<uint4*>(row + phys);
-              uint4* pb = reinterpret_cast<uint4*>(row + kHalfBytes + phys);
-              uint4 va = *pa, vb = *pb;
-              uint32_t wa[4] = {va.x, va.y, va.z, va.w}, wb[4] = {vb.x, vb.y, vb.z, vb.w};
-#pragma unroll
-              for (int m = 0; m < 4; ++m) {
-                float ca0, sa0, ca1, sa1;
-                const int j0 = 8 * c4 + 2 * m;
-                if (P.same_theta) {
-                  ca0 = cs[j0];
-                  sa0 = sn[j0];
-                  ca1 = cs[j0 + 1];
-                  sa1 = sn[j0 + 1];
-                } else {
-                  rope_sincos(p, P.rope.ws_hi[32 * g + j0], P.rope.ws_lo[32 * g + j0], P.rope.two_pi_hi,
-                              P.rope.two_pi_lo, P.rope.inv_two_pi, &sa0, &ca0);
-                  rope_sincos(p, P.rope.ws_hi[32 * g + j0 + 1], P.rope.ws_lo[32 * g + j0 + 1],
-                              P.rope.two_pi_hi, P.rope.two_pi_lo, P.rope.inv_two_pi, &sa1, &ca1);
-                }
-                const float a0 = bf16_lo(wa[m]), a1 = bf16_hi(wa[m]);
-                const float b0 = bf16_lo(wb[m]), b1 = bf16_hi(wb[m]);
-                // rotation by -t*omega: a' = a c + b s, b' = b c - a s
-                wa[m] = pack_bf16x2(__fmaf_rn(a0, ca0, __fmul_rn(b0, sa0)), __fmaf_rn(a1, ca1, __fmul_rn(b1, sa1)));
-                wb[m] = pack_bf16x2(__fmaf_rn(b0, ca0, -__fmul_rn(a0, sa0)), __fmaf_rn(b1, ca1, -__fmul_rn(a1, sa1)));
-              }
-              *pa = make_uint4(wa[0], wa[1], wa[2], wa[3]);
-              *pb = make_uint4(wb[0], wb[1], wb[2], wb[3]);
-            }
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&ready[s]));
+            tc_fence_after();
           }
-          full_par ^= 1u << s;
+          tl_loaded |= 1u << s;
+          const uint32_t scol = tmem_base + lane_addr + kSlotCol0 + s * 64;
+          tmem_st_x16(scol + 16 * g, wa);        // features 32g .. 32g+31
+          tmem_st_x16(scol + 32 + 16 * g, wb);   // features 64 + 32g .. 64 + 32g+31
+          tmem_wait_st();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&tready[s]));
           ++e;
         }
         if (!ok) break;
         // epilogue of layer l
-        const uint32_t a = li & 1u;
-        const bool w_ok = wait_bar(smem_u32(&accf[a]), (li >> 1) & 1u, abort_flag, P.status);
-        if (!__all_sync(0xffffffffu, w_ok)) {
-          ok = false;
-          break;
+        const uint32_t ob_i = lay & 1u;
+        uint8_t* ob = outst + ob_i * kOutBytes;
+        const uint32_t bslot = lay % kBiasSlots;
+        const float* bias = bias_ring + bslot * kD;
+        {
+          const bool w_ok = wait_bar(smem_u32(&bias_full[bslot]), (lay / kBiasSlots) & 1u, abort_flag, P.status,
+                                     KVX_ERR_TIMEOUT);
+          if (!__all_sync(0xffffffffu, w_ok)) {
+            ok = false;
+            break;
+          }
+        }
+        if (use_tma && lay >= 2) {   // the store that last read this staging buffer is done
+          const bool w_ok = wait_bar(smem_u32(&stage_free[ob_i]), ((lay >> 1) - 1) & 1u, abort_flag, P.status,
+                                     KVX_ERR_TIMEOUT);
+          if (!__all_sync(0xffffffffu, w_ok)) {
+            ok = false;
+            break;
+          }
+        }
+        const uint32_t buf = lay & 1u;
+        {
+          const bool w_ok = wait_bar(smem_u32(&accf[buf]), (lay >> 1) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT);
+          if (!__all_sync(0xffffffffu, w_ok)) {
+            ok = false;
+            break;
+          }
         }
         tc_fence_after();
-        const uint32_t col = tmem_base + a * kD + 32 * g;
-        const float* bias = P.bias + (static_cast<size_t>(l * 2 + un.kv) * H + un.h) * kD + 32 * g;
-        __nv_bfloat16* out = dst + static_cast<int64_t>(l) * A.ts[0] + row_off + 32 * g;
+        const uint32_t col = tmem_base + lane_addr + buf * kAccCols + 32 * g;
 #pragma unroll
         for (int rnd = 0; rnd < 2; ++rnd) {
           uint32_t lo[16], hi[16];
-          tmem_ld_2x16(col + 16 * rnd + lane_addr, col + 64 + 16 * rnd + lane_addr, lo, hi);
-          if (rnd == 1) {  // the accumulator is free for the next layer's MMAs
+          tmem_ld_2x16(col + 16 * rnd, col + 64 + 16 * rnd, lo, hi);
+          if (rnd == 1) {  // the accumulator is free for the MMAs of layer l + 2
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&acce[a]));
+            if (lane == 0) mbar_arrive(smem_u32(&acce[buf]));
           }
-          if (valid) {
-            float ylo[16], yhi[16];
+          const int c_lo = 32 * g + 16 * rnd;   // channels c_lo + [0,16) and 64 + c_lo + [0,16)
+          float ylo[16], yhi[16];
 #pragma unroll
-            for (int j = 0; j < 16; j += 4) {
-              const float4 b0 = __ldg(reinterpret_cast<const float4*>(bias + 16 * rnd + j));
-              const float4 b1 = __ldg(reinterpret_cast<const float4*>(bias + 64 + 16 * rnd + j));
-              ylo[j] = __fadd_rn(__uint_as_float(lo[j]), b0.x);
-              ylo[j + 1] = __fadd_rn(__uint_as_float(lo[j + 1]), b0.y);
-              ylo[j + 2] = __fadd_rn(__uint_as_float(lo[j + 2]), b0.z);
-              ylo[j + 3] = __fadd_rn(__uint_as_float(lo[j + 3]), b0.w);
-              yhi[j] = __fadd_rn(__uint_as_float(hi[j]), b1.x);
-              yhi[j + 1] = __fadd_rn(__uint_as_float(hi[j + 1]), b1.y);
-              yhi[j + 2] = __fadd_rn(__uint_as_float(hi[j + 2]), b1.z);
-              yhi[j + 3] = __fadd_rn(__uint_as_float(hi[j + 3]), b1.w);
+          for (int j = 0; j < 16; j += 4) {
+            const float4 b0 = *reinterpret_cast<const float4*>(bias + c_lo + j);
+            const float4 b1 = *reinterpret_cast<const float4*>(bias + 64 + c_lo + j);
+            ylo[j] = __fadd_rn(__uint_as_float(lo[j]), b0.x);
+            ylo[j + 1] = __fadd_rn(__uint_as_float(lo[j + 1]), b0.y);
+            ylo[j + 2] = __fadd_rn(__uint_as_float(lo[j + 2]), b0.z);
+            ylo[j + 3] = __fadd_rn(__uint_as_float(lo[j + 3]), b0.w);
+            yhi[j] = __fadd_rn(__uint_as_float(hi[j]), b1.x);
+            yhi[j + 1] = __fadd_rn(__uint_as_float(hi[j + 1]), b1.y);
+            yhi[j + 2] = __fadd_rn(__uint_as_float(hi[j + 2]), b1.z);
+            yhi[j + 3] = __fadd_rn(__uint_as_float(hi[j + 3]), b1.w);
+          }
+          if (un.kv == 0) {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const float c = cs[16 * rnd + j], sv = sn[16 * rnd + j];
+              const float y0 = ylo[j], y1 = yhi[j];
+              ylo[j] = __fmaf_rn(y0, c, -__fmul_rn(y1, sv));
+              yhi[j] = __fmaf_rn(y0, sv, __fmul_rn(y1, c));
             }
-            if (un.kv == 0) {
-#pragma unroll
-              for (int j = 0; j < 16; ++j) {
-                const float c = cs[16 * rnd + j], sv = sn[16 * rnd + j];
-                const float y0 = ylo[j], y1 = yhi[j];
-                ylo[j] = __fmaf_rn(y0, c, -__fmul_rn(y1, sv));
-                yhi[j] = __fmaf_rn(y0, sv, __fmul_rn(y1, c));
+          }
+          uint4 v[4];
+          v[0] = make_uint4(pack_bf16x2(ylo[0], ylo[1]), pack_bf16x2(ylo[2], ylo[3]), pack_bf16x2(ylo[4], ylo[5]),
+                            pack_bf16x2(ylo[6], ylo[7]));
+          v[1] = make_uint4(pack_bf16x2(ylo[8], ylo[9]), pack_bf16x2(ylo[10], ylo[11]),
+                            pack_bf16x2(ylo[12], ylo[13]), pack_bf16x2(ylo[14], ylo[15]));
+          v[2] = make_uint4(pack_bf16x2(yhi[0], yhi[1]), pack_bf16x2(yhi[2], yhi[3]), pack_bf16x2(yhi[4], yhi[5]),
+                            pack_bf16x2(yhi[6], yhi[7]));
+          v[3] = make_uint4(pack_bf16x2(yhi[8], yhi[9]), pack_bf16x2(yhi[10], yhi[11]),
+                            pack_bf16x2(yhi[12], yhi[13]), pack_bf16x2(yhi[14], yhi[15]));
+          if (use_tma) {
+            // staging tile: box 0 = channels 0..63, box 1 = channels 64..127, rows of 128 B,
+            // 128-byte swizzle (16-byte chunk index XOR row % 8)
+            const int ch = c_lo >> 3;  // 16-byte chunk of channel c_lo within a box row
+            uint8_t* row0 = ob + r * 128;
+            *reinterpret_cast<uint4*>(row0 + ((ch ^ (r & 7)) << 4)) = v[0];
+            *reinterpret_cast<uint4*>(row0 + (((ch + 1) ^ (r & 7)) << 4)) = v[1];
+            *reinterpret_cast<uint4*>(row0 + kHalfBytes + ((ch ^ (r & 7)) << 4)) = v[2];
+            *reinterpret_cast<uint4*>(row0 + kHalfBytes + (((ch + 1) ^ (r & 7)) << 4)) = v[3];
+          } else if (valid) {
+            __nv_bfloat16* out = dst + static_cast<int64_t>(l) * A.ts[0] + row_off;
+            st_global_hint(out + c_lo, v[0], st_pol);
+            st_global_hint(out + c_lo + 8, v[1], st_pol);
+            st_global_hint(out + 64 + c_lo, v[2], st_pol);
+            st_global_hint(out + 64 + c_lo + 8, v[3], st_pol);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&bias_empty[bslot]));
+        if (use_tma) {
+          // hand the staged tile to transform thread 0 (the first transform warp)
+          if (bad && g == 0) atomicOr(&bad_mask[ob_i * 4 + (r >> 5)], 1u << (r & 31));
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&stage_full[ob_i]));
+          if (warp == kFirstTransformWarp) {
+            const bool w_ok = wait_bar(smem_u32(&stage_full[ob_i]), (lay >> 1) & 1u, abort_flag, P.status,
+                                       KVX_ERR_TIMEOUT);
+            if (!__all_sync(0xffffffffu, w_ok)) {
+              ok = false;
+              break;
+            }
+            const uint32_t m0 = bad_mask[ob_i * 4], m1 = bad_mask[ob_i * 4 + 1], m2 = bad_mask[ob_i * 4 + 2],
+                           m3 = bad_mask[ob_i * 4 + 3];
+            const bool clean = (m0 | m1 | m2 | m3) == 0u;
+            if (clean) {
+              if (lane == 0) {
+                const uint32_t src = smem_u32(ob);
+                tma_store_5d(tm_out, src, 0, un.t0, un.h, un.b, l);
+                tma_store_5d(tm_out, src + kHalfBytes, 64, un.t0, un.h, un.b, l);
+                bulk_commit_group();
               }
+            } else {
+              // write the rows with a valid position one by one (lane j: rows j, j+32, ...)
+              __nv_bfloat16* base_out = dst + static_cast<int64_t>(l) * A.ts[0];
+              for (int rr = lane; rr < kTileM; rr += 32) {
+                const uint32_t mw = rr < 32 ? m0 : rr < 64 ? m1 : rr < 96 ? m2 : m3;
+                const int trow = un.t0 + rr;
+                if (trow >= A.T || ((mw >> (rr & 31)) & 1u)) continue;
+                __nv_bfloat16* orow =
+                    base_out + un.b * A.ts[1] + un.h * A.ts[2] + static_cast<int64_t>(trow) * A.ts[3];
+                for (int c16 = 0; c16 < 16; ++c16) {   // 16-byte chunk c16 of the 256-byte row
+                  const int box = c16 >> 3, chk = c16 & 7;
+                  const uint4 v = *reinterpret_cast<const uint4*>(ob + box * kHalfBytes + rr * 128 +
+                                                                  ((chk ^ (rr & 7)) << 4));
+                  st_global_hint(orow + 8 * c16, v, st_pol);
+                }
+              }
+              __syncwarp();
+              if (lane == 0)
+                for (int i = 0; i < 4; ++i) bad_mask[ob_i * 4 + i] = 0u;
             }
-#pragma unroll
-            for (int j = 0; j < 16; j += 8) {
-              const uint4 v0 = make_uint4(pack_bf16x2(ylo[j], ylo[j + 1]), pack_bf16x2(ylo[j + 2], ylo[j + 3]),
-                                          pack_bf16x2(ylo[j + 4], ylo[j + 5]), pack_bf16x2(ylo[j + 6], ylo[j + 7]));
-              const uint4 v1 = make_uint4(pack_bf16x2(yhi[j], yhi[j + 1]), pack_bf16x2(yhi[j + 2], yhi[j + 3]),
-                                          pack_bf16x2(yhi[j + 4], yhi[j + 5]), pack_bf16x2(yhi[j + 6], yhi[j + 7]));
-              st_global_stream(out + 16 * rnd + j, v0, st_pol);
-              st_global_stream(out + 64 + 16 * rnd + j, v1, st_pol);
+            // Release staging buffers exactly once per use: the previous layer's buffer
+            // once its TMA store has read it, this layer's buffer at once if it was
+            // written out row by row (no store reads it).
+            if (lane == 0) {
+              if (prev_store_pending) {
+                if (clean) bulk_wait_read_but_last(); else bulk_wait_read_all();
+                mbar_arrive(smem_u32(&stage_free[ob_i ^ 1u]));
+              }
+              if (!clean) mbar_arrive(smem_u32(&stage_free[ob_i]));
             }
+            prev_store_pending = clean;
           }
         }
       }
     }
+    if (warp == kFirstTransformWarp && lane == 0) bulk_wait_all();
   }
 
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (warp == 2) {
+  if (warp == 1) {
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(kTmemCols)
                  : "memory");
   }
@@ -668,14 +656,20 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return fn;
 }
 
-size_t smem_bytes(int n_slots, int n_wst) {
-  const size_t bars = (3 * n_slots + 2 * n_wst + 5) * 8 + 16;
-  return 1024 + static_cast<size_t>(n_slots) * kSlotBytes + static_cast<size_t>(n_wst) * kWStageBytes + bars;
+size_t smem_bytes(int n_wst) {
+  const size_t bars =
+      (2 * kLand + 2 * kTSlots + 2 * n_wst + 2 * kAccBufs + 2 * kOutBufs + 2 * kBiasSlots + 1) * 8 + 48;
+  return 1024 + static_cast<size_t>(kLand) * kLandBytes + static_cast<size_t>(n_wst) * kWStageBytes +
+         kOutBufs * static_cast<size_t>(kOutBytes) + kBiasSlots * kBiasBytes + bars;
 }
 
-// Belady schedule of source-tile loads over the use sequence (l, j), l-major.
-void build_plan(const kvx_ctx* c, int n_slots, TcPlan* plan) {
-  const int Lt = c->Lt, k = c->k, n_uses = Lt * k;
+// Belady schedule of source-tile loads over the use sequence (l, j), l-major, into
+// kTSlots TMEM slots.  The victim is the resident tile whose next use is farthest away;
+// among equals, the one whose last use is earliest (its slot frees soonest).  A slot is
+// released right after the MMAs of its tile's last use before the reload, so with
+// k <= kTSlots a victim always exists and every wait ends.
+void build_plan(const kvx_ctx* c, TcPlan* plan) {
+  const int Lt = c->Lt, k = c->k, n_uses = Lt * k, S = kTSlots;
   std::vector<int> src(n_uses), next_use(n_uses);
   for (int u = 0; u < n_uses; ++u) src[u] = c->sel[u];
   std::vector<int> seen(c->Ls, INT_MAX);
@@ -683,28 +677,28 @@ void build_plan(const kvx_ctx* c, int n_slots, TcPlan* plan) {
     next_use[u] = seen[src[u]];
     seen[src[u]] = u;
   }
-  plan->n_slots = n_slots;
+  plan->n_slots = S;
   plan->load_layer.clear();
   plan->load_slot.clear();
   plan->load_first_use.clear();
   plan->use_slot.assign(n_uses, -1);
   plan->use_flags.assign(n_uses, 0);
-  std::vector<int> slot_src(n_slots, -1), slot_next(n_slots, INT_MAX), slot_last(n_slots, -1);
+  std::vector<int> slot_src(S, -1), slot_next(S, INT_MAX), slot_last(S, -1);
   for (int u = 0; u < n_uses; ++u) {
     const int l = u / k;
     int s = -1;
-    for (int i = 0; i < n_slots; ++i)
+    for (int i = 0; i < S; ++i)
       if (slot_src[i] == src[u]) s = i;
     if (s < 0) {
-      // victim: an empty slot, else the one whose next use is farthest away
       int best = -1;
-      for (int i = 0; i < n_slots; ++i) {
-        const int key = slot_src[i] < 0 ? INT_MAX : slot_next[i];
-        if (best < 0 || key > (slot_src[best] < 0 ? INT_MAX : slot_next[best])) best = i;
+      for (int i = 0; i < S; ++i) {
         if (slot_src[i] < 0) {
           best = i;
           break;
         }
+        if (best < 0 || slot_next[i] > slot_next[best] ||
+            (slot_next[i] == slot_next[best] && slot_last[i] < slot_last[best]))
+          best = i;
       }
       s = best;
       if (slot_src[s] >= 0) plan->use_flags[slot_last[s]] |= 2;
@@ -718,7 +712,7 @@ void build_plan(const kvx_ctx* c, int n_slots, TcPlan* plan) {
     slot_next[s] = next_use[u];
     slot_last[s] = u;
   }
-  for (int i = 0; i < n_slots; ++i)
+  for (int i = 0; i < S; ++i)
     if (slot_src[i] >= 0) plan->use_flags[slot_last[i]] |= 2;
   plan->n_loads = static_cast<int>(plan->load_layer.size());
 }
@@ -731,6 +725,7 @@ bool tc_supported(const kvx_ctx* c, std::string* why) {
   else if (c->d != kD) w = "needs head_dim 128";
   else if (c->head_mix != KVX_PER_HEAD) w = "needs per-head features";
   else if (c->rope_style != KVX_ROPE_HALF) w = "needs half-split RoPE pairs";
+  else if (c->k > kTSlots) w = "needs k <= 4 (one target layer's source tiles must fit in tensor memory)";
   else if (static_cast<int64_t>(c->Lt) * 2 * c->H * kD > INT_MAX) w = "too many W rows";
   if (why) *why = w;
   return w.empty();
@@ -743,10 +738,10 @@ kvx_status tc_prepare(kvx_ctx* c, const void* W_host) {
   std::vector<uint16_t> wt(blocks * F * kD);
   const uint16_t* w = static_cast<const uint16_t*>(W_host);
   for (size_t blk = 0; blk < blocks; ++blk) {
-    const uint16_t* src = w + blk * F * kD;
-    uint16_t* dst = wt.data() + blk * F * kD;
+    const uint16_t* srcb = w + blk * F * kD;
+    uint16_t* dstb = wt.data() + blk * F * kD;
     for (size_t f = 0; f < F; ++f)
-      for (int n = 0; n < kD; ++n) dst[static_cast<size_t>(n) * F + f] = src[f * kD + n];
+      for (int n = 0; n < kD; ++n) dstb[static_cast<size_t>(n) * F + f] = srcb[f * kD + n];
   }
   cudaError_t e = cudaMalloc(&c->d_Wt, wt.size() * 2);
   if (e != cudaSuccess) {
@@ -757,20 +752,27 @@ kvx_status tc_prepare(kvx_ctx* c, const void* W_host) {
     set_error(std::string("kvx_create: upload W^T: ") + cudaGetErrorString(e));
     return KVX_ERR_CUDA;
   }
-  // slots and W stages within the shared-memory budget
-  int n_wst = 4;
-  int n_slots = std::min<int>(kMaxSlots, c->k + 2);
-  while (n_slots > 1 && smem_bytes(n_slots, n_wst) > kSmemLimit) --n_slots;
-  while (n_wst < kMaxWStages && smem_bytes(n_slots, n_wst + 1) <= kSmemLimit) ++n_wst;
-  build_plan(c, n_slots, &c->plan);
+  // as many W stages as the shared-memory budget allows
+  int n_wst = 2;
+  while (n_wst < kMaxWStages && smem_bytes(n_wst + 1) <= kSmemLimit) ++n_wst;
+  build_plan(c, &c->plan);
   c->plan.n_wst = n_wst;
+  c->plan.n_land = kLand;
   const TcPlan& p = c->plan;
+  // per target layer, one word: 5 bits per use j (slot | 8 first use | 16 release after)
+  std::vector<int32_t> pack(c->Lt, 0);
+  for (int l = 0; l < c->Lt; ++l)
+    for (int j = 0; j < c->k; ++j) {
+      const int u = l * c->k + j;
+      const uint32_t f = static_cast<uint32_t>(p.use_slot[u]) | ((p.use_flags[u] & 1) ? 8u : 0u) |
+                         ((p.use_flags[u] & 2) ? 16u : 0u);
+      pack[l] |= static_cast<int32_t>(f << (5 * j));
+    }
   std::vector<int32_t> tab;
   tab.insert(tab.end(), p.load_layer.begin(), p.load_layer.end());
   tab.insert(tab.end(), p.load_slot.begin(), p.load_slot.end());
   tab.insert(tab.end(), p.load_first_use.begin(), p.load_first_use.end());
-  tab.insert(tab.end(), p.use_slot.begin(), p.use_slot.end());
-  tab.insert(tab.end(), p.use_flags.begin(), p.use_flags.end());
+  tab.insert(tab.end(), pack.begin(), pack.end());
   if ((e = cudaMalloc(&c->d_plan, tab.size() * 4)) != cudaSuccess) {
     set_error(std::string("kvx_create: cudaMalloc plan: ") + cudaGetErrorString(e));
     return KVX_ERR_OOM;
@@ -790,48 +792,62 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   }
   TcParams P;
   std::memset(&P, 0, sizeof(P));
+  const cuuint32_t ones[5] = {1, 1, 1, 1, 1};
   // source maps: dims (d, T, H, B, L_s), strides in bytes for dims 1..4
   const cuuint64_t sdims[5] = {static_cast<cuuint64_t>(kD), static_cast<cuuint64_t>(a.T),
                                static_cast<cuuint64_t>(c->H), static_cast<cuuint64_t>(a.B),
                                static_cast<cuuint64_t>(c->Ls)};
   const cuuint64_t sstr[4] = {static_cast<cuuint64_t>(a.ss[3]) * 2, static_cast<cuuint64_t>(a.ss[2]) * 2,
                               static_cast<cuuint64_t>(a.ss[1]) * 2, static_cast<cuuint64_t>(a.ss[0]) * 2};
-  const cuuint32_t sbox[5] = {64, kTileM, 1, 1, 1};
-  const cuuint32_t ones[5] = {1, 1, 1, 1, 1};
+  const cuuint32_t box[5] = {64, kTileM, 1, 1, 1};
   for (int kv = 0; kv < 2; ++kv) {
     CUresult r = encode(kv ? &P.tm_v : &P.tm_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5,
-                        const_cast<void*>(kv ? a.src_v : a.src_k), sdims, sstr, sbox, ones,
-                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                        const_cast<void*>(kv ? a.src_v : a.src_k), sdims, sstr, box, ones,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) {
       set_error("kvx_map: source tensor map rejected (strides or sizes)");
       return KVX_ERR_UNSUPPORTED;
     }
   }
+  if (!a.paged) {  // target maps for the TMA-store epilogue: dims (d, T, H, B, L_t)
+    const cuuint64_t tdims[5] = {static_cast<cuuint64_t>(kD), static_cast<cuuint64_t>(a.T),
+                                 static_cast<cuuint64_t>(c->H), static_cast<cuuint64_t>(a.B),
+                                 static_cast<cuuint64_t>(c->Lt)};
+    const cuuint64_t tstr[4] = {static_cast<cuuint64_t>(a.ts[3]) * 2, static_cast<cuuint64_t>(a.ts[2]) * 2,
+                                static_cast<cuuint64_t>(a.ts[1]) * 2, static_cast<cuuint64_t>(a.ts[0]) * 2};
+    for (int kv = 0; kv < 2; ++kv) {
+      CUresult r = encode(kv ? &P.tm_out_v : &P.tm_out_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5,
+                          kv ? a.tgt_v : a.tgt_k, tdims, tstr, box, ones, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      if (r != CUDA_SUCCESS) {
+        set_error("kvx_map: target tensor map rejected (strides or sizes)");
+        return KVX_ERR_UNSUPPORTED;
+      }
+    }
+  }
   const cuuint64_t wdims[2] = {static_cast<cuuint64_t>(c->F), static_cast<cuuint64_t>(c->Lt) * 2 * c->H * kD};
   const cuuint64_t wstr[1] = {static_cast<cuuint64_t>(c->F) * 2};
-  const cuuint32_t wbox[2] = {64, 128};
+  const cuuint32_t wbox[2] = {64, kD};
   CUresult r = encode(&P.tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, c->d_Wt, wdims, wstr, wbox, ones,
-                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
     set_error("kvx_map: weight tensor map rejected");
     return KVX_ERR_CUDA;
   }
   const TcPlan& p = c->plan;
-  const int n_uses = c->Lt * c->k;
   P.a = a;
   P.load_layer = c->d_plan;
   P.load_slot = c->d_plan + p.n_loads;
   P.load_first = c->d_plan + 2 * p.n_loads;
-  P.use_slot = c->d_plan + 3 * p.n_loads;
-  P.use_flags = c->d_plan + 3 * p.n_loads + n_uses;
+  P.use_pack = reinterpret_cast<const uint32_t*>(c->d_plan + 3 * p.n_loads);
   P.bias = c->d_b;
   P.status = c->d_status;
   P.Lt = c->Lt;
   P.H = c->H;
   P.k = c->k;
-  P.n_slots = p.n_slots;
   P.n_wst = p.n_wst;
   P.n_loads = p.n_loads;
   P.tiles_per_seq = (a.T + kTileM - 1) / kTileM;
@@ -843,7 +859,7 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   P.n_units = static_cast<int>(units);
   P.same_theta = c->theta_s == c->theta_t;
   P.rope = c->rope;
-  const size_t smem = smem_bytes(P.n_slots, P.n_wst);
+  const size_t smem = smem_bytes(P.n_wst);
   cudaError_t e = cudaFuncSetAttribute(tc_map_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) {

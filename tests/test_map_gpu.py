@@ -71,11 +71,21 @@ def test_tiny_fp32_full():
     dict(Ls=5, Lt=7, H=2, B=3, T=129, k=2, theta_t=5e5),   # different thetas, 1-row tail
     dict(Ls=9, Lt=6, H=3, B=1, T=640, k=4),                # several tiles
     dict(Ls=8, Lt=9, H=2, B=1, T=256, k=4, scores="uniform"),  # random selection, reloads
-    dict(Ls=10, Lt=5, H=2, B=1, T=200, k=6),               # more selected layers than slots
+    dict(Ls=10, Lt=5, H=2, B=1, T=200, k=5),               # beyond the tensor-core kernel: SIMT
 ])
 def test_bf16_small_full(kname, over):
     name = "qwen3_14b_32b_b8x1024_k4"
     if kname == "tc":
+        if over["k"] > 4:
+            w = syn.workload(name, **over)
+            ctx, _, _, _ = make_ctx(w)
+            try:
+                with pytest.raises(kvx.KvxError) as e:
+                    kvx.kvx_set_kernel(ctx, KERNELS[kname])
+                assert e.value.status == kvx.KVX_ERR_UNSUPPORTED
+            finally:
+                kvx.kvx_destroy(ctx)
+            return
         _kernel_or_skip(syn.workload(name, **over), KERNELS[kname])
     _small(name, KERNELS[kname], **over)
 
