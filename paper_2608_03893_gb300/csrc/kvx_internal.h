@@ -49,8 +49,8 @@ struct TcPlan {
   std::vector<int32_t> load_slot;       // [n_loads] slot it lands in
   std::vector<int32_t> load_first_use;  // [n_loads] target layer of its first use
   std::vector<int32_t> use_slot;        // [L_t*k] slot holding the tile of use (l, j)
-  std::vector<int32_t> use_flags;       // [L_t*k] bit 0: first use of a load,
-                                        //         bit 1: last use before the slot is reloaded
+  std::vector<int32_t> use_flags;       // [L_t*k] bit 0: first use of the tile by its issuer,
+                                        //         bit 2: release the slot after this use
 };
 
 }  // namespace kvx

@@ -34,7 +34,7 @@
 //               Prologue: landing buffer -> registers -> (keys) strip the source RoPE in
 //               fp32, round to bf16 -> tcgen05.st into the tile's TMEM slot.
 //               Epilogue: TMEM -> registers, + bias, (keys) target RoPE, bf16, into a
-//               double-buffered shared-memory staging tile written out by a TMA store
+//               shared-memory staging tile written out by a TMA store
 //               (contiguous targets), or 16-byte stores through the block table (paged).
 //               Transform thread 0 issues the TMA stores; a staged tile holding a row
 //               with an out-of-range position is instead written row by row by its warp,
@@ -70,18 +70,32 @@ constexpr uint32_t kLandBytes = kTileM * kD * 2;    // 32 KB raw tile: two 64-co
 constexpr uint32_t kHalfBytes = kLandBytes / 2;     // 16 KB
 constexpr uint32_t kWStageBytes = kD * 64 * 2;      // 16 KB: 128 output channels x 64 features
 constexpr uint32_t kOutBytes = kTileM * kD * 2;     // 32 KB staging tile (two SW128 boxes)
-constexpr int kOutBufs = 2;
+constexpr int kOutBufs = 2;                         // staging tiles (1 or 2)
 constexpr int kTSlots = 4;                          // TMEM source-tile slots (64 columns each)
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccCols = 128;                  // one fp32 accumulator
 constexpr int kAccBufs = 2;
 constexpr uint32_t kSlotCol0 = kAccBufs * kAccCols; // 256: first source-slot column
-constexpr int kLand = 2;                            // landing buffers
-constexpr int kMaxWStages = 8;
+constexpr int kLand = 1;                            // landing buffers (tiles are L2-prefetched ahead)
+constexpr int kIssuers = 2;                         // MMA-issuing threads (even / odd target layers)
 constexpr int kSrcPrefetch = 6;                     // source loads prefetched into L2 ahead
 constexpr int kBiasSlots = 4;                       // per-layer bias rows staged ahead (512 B each)
 constexpr uint32_t kBiasBytes = kD * 4;
 constexpr size_t kSmemLimit = 232448;               // 227 KB opt-in per CTA
+
+constexpr int kRing = 4;                            // W stages per issuer ring (two uses)
+constexpr int kNW = kRing * kIssuers;               // W stages in shared memory
+
+// Dynamic shared memory: the 128-byte-swizzled buffers need 1024-byte alignment, which
+// the base of the dynamic window has (the kernel checks it) since nothing else is placed
+// before it; no slack is reserved.
+constexpr size_t smem_bytes() {
+  return static_cast<size_t>(kLand) * kLandBytes + static_cast<size_t>(kNW) * kWStageBytes +
+         kOutBufs * static_cast<size_t>(kOutBytes) + kBiasSlots * kBiasBytes +
+         (2 * kLand + 2 * kTSlots * kIssuers + 2 * kNW + 2 * kAccBufs + 2 * kOutBufs + 2 * kBiasSlots +
+          kIssuers) * 8 + 48;
+}
+static_assert(smem_bytes() <= kSmemLimit, "shared-memory layout exceeds the per-CTA limit");
 
 struct TcParams {
   CUtensorMap tm_k;      // source keys   [L_s][B][H][T][128] bf16, box 64 x 128
@@ -96,7 +110,7 @@ struct TcParams {
   const uint32_t* use_pack;    // [L_t] per use j: 5 bits at 5j = slot | 8 first use | 16 release after
   const float* bias;           // [L_t][2][H][128] fp32
   int32_t* status;
-  int32_t Lt, H, k, n_wst, n_loads, tiles_per_seq, n_units, same_theta;
+  int32_t Lt, H, k, n_loads, tiles_per_seq, n_units, same_theta;
   RopeTables rope;
 };
 
@@ -104,18 +118,19 @@ struct Unit {
   int b, t0, h, kv;
 };
 
-// Units are visited u = blockIdx.x + i * gridDim.x.  With an even grid, u & 1 would pin
-// every CTA to K or to V units; flipping it every round makes each CTA alternate, which
-// balances the (heavier) key units across CTAs.  u and u ^ 1 share u / grid, so the
-// mapping stays a bijection.
-__device__ __forceinline__ Unit decode_unit(int u, int H, int tiles) {
+// Units are visited u = blockIdx.x + i * gridDim.x, token tile fastest, then sequence,
+// head, and K|V outermost.  The CTAs running at any moment then work on one or two
+// (K|V, head) pairs, so the W^T rows they stream (8 MB per pair at L_t = 64, k = 4) stay
+// in L2 even when the CTAs drift to different target layers; every CTA still gets
+// nearly equal numbers of (heavier) key and value units.
+__device__ __forceinline__ Unit decode_unit(int u, int H, int B, int tiles) {
   Unit r;
-  r.kv = (u & 1) ^ ((gridDim.x & 1) ? 0 : static_cast<int>((u / gridDim.x) & 1));
-  int rest = u >> 1;
+  r.t0 = (u % tiles) * kTileM;
+  int rest = u / tiles;
+  r.b = rest % B;
+  rest /= B;
   r.h = rest % H;
-  rest /= H;
-  r.t0 = (rest % tiles) * kTileM;
-  r.b = rest / tiles;
+  r.kv = rest / H;
   return r;
 }
 
@@ -124,28 +139,30 @@ __device__ __forceinline__ void report(int32_t* status, int code) { atomicCAS(st
 // ------------------------------------------------------------------------ kernel --
 
 __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_constant__ TcParams P) {
-  extern __shared__ __align__(1024) uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const int NW = P.n_wst;
+  extern __shared__ __align__(1024) uint8_t smem[];
+  if (smem_u32(smem) & 1023u) {   // uniform over the CTA: every thread returns here
+    if (threadIdx.x == 0) report(P.status, KVX_ERR_UNSUPPORTED);
+    return;
+  }
   uint8_t* land = smem;
-  uint8_t* wst = land + kLand * kLandBytes;
-  uint8_t* outst = wst + static_cast<size_t>(NW) * kWStageBytes;
+  uint8_t* wst = land + kLand * kLandBytes;            // [2 rings][kRing] W stages
+  uint8_t* outst = wst + static_cast<size_t>(kNW) * kWStageBytes;
   float* bias_ring = reinterpret_cast<float*>(outst + kOutBufs * kOutBytes);   // [4][128] fp32
   uint64_t* bars = reinterpret_cast<uint64_t*>(bias_ring + kBiasSlots * kD);
   uint64_t* land_full = bars;                    // [2] TMA landed
   uint64_t* land_empty = land_full + kLand;      // [2] transform read it (8 warps)
-  uint64_t* tready = land_empty + kLand;         // [4] TMEM tile written (8 warps)
-  uint64_t* tfree = tready + kTSlots;            // [4] TMEM tile released by the MMA
-  uint64_t* wfull = tfree + kTSlots;             // [NW]
-  uint64_t* wempty = wfull + NW;                 // [NW]
-  uint64_t* accf = wempty + NW;                  // [2] accumulator ready
+  uint64_t* tready = land_empty + kLand;         // [4][2] TMEM tile written for issuer i (8 warps)
+  uint64_t* tfree = tready + kTSlots * kIssuers; // [4][2] TMEM tile released by issuer i
+  uint64_t* wfull = tfree + kTSlots * kIssuers;  // [2][kRing]
+  uint64_t* wempty = wfull + kNW;                // [2][kRing]
+  uint64_t* accf = wempty + kNW;                 // [2] accumulator ready
   uint64_t* acce = accf + kAccBufs;              // [2] accumulator drained (8 warps)
   uint64_t* stage_full = acce + kAccBufs;        // [2] staging tile written (8 warps)
   uint64_t* stage_free = stage_full + kOutBufs;  // [2] staging tile read by its store
   uint64_t* bias_full = stage_free + kOutBufs;   // [4] bias row landed
   uint64_t* bias_empty = bias_full + kBiasSlots; // [4] bias row used (8 warps)
-  uint64_t* drain = bias_empty + kBiasSlots;     // [1]
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* drain = bias_empty + kBiasSlots;     // [2] per issuer
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + kIssuers);
   volatile uint32_t* abort_flag = tmem_holder + 1;
   uint32_t* bad_mask = tmem_holder + 2;          // [2][4] rows of a staged tile with a bad position
 
@@ -157,11 +174,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
       mbar_init(smem_u32(&land_full[i]), 1);
       mbar_init(smem_u32(&land_empty[i]), 8);
     }
-    for (int i = 0; i < kTSlots; ++i) {
-      mbar_init(smem_u32(&tready[i]), 8);
-      mbar_init(smem_u32(&tfree[i]), 1);
-    }
-    for (int i = 0; i < NW; ++i) {
+    for (int i = 0; i < kTSlots * kIssuers; ++i) mbar_init(smem_u32(&tready[i]), 8);
+    for (int i = 0; i < kTSlots * kIssuers; ++i) mbar_init(smem_u32(&tfree[i]), 1);
+    for (int i = 0; i < kNW; ++i) {
       mbar_init(smem_u32(&wfull[i]), 1);
       mbar_init(smem_u32(&wempty[i]), 1);
     }
@@ -177,7 +192,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
       mbar_init(smem_u32(&bias_full[i]), 1);
       mbar_init(smem_u32(&bias_empty[i]), 8);
     }
-    mbar_init(smem_u32(drain), 1);
+    for (int i = 0; i < kIssuers; ++i) mbar_init(smem_u32(&drain[i]), 1);
     *abort_flag = 0u;
     for (int i = 0; i < 2 * 4; ++i) bad_mask[i] = 0u;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -209,7 +224,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           u += gridDim.x;
         }
         if (u >= n_units) return;
-        const Unit pu = decode_unit(u, H, tiles);
+        const Unit pu = decode_unit(u, H, A.B, tiles);
         const CUtensorMap* ptm = pu.kv ? &P.tm_v : &P.tm_k;
         const int L = __ldg(&P.load_layer[e]);
         tma_prefetch_5d(ptm, 0, pu.t0, pu.h, pu.b, L);
@@ -218,7 +233,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
       if (static_cast<int>(blockIdx.x) < n_units)
         for (int e = 0; e < kSrcPrefetch; ++e) prefetch(blockIdx.x, e);
       for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-        const Unit un = decode_unit(u, H, tiles);
+        const Unit un = decode_unit(u, H, A.B, tiles);
         const CUtensorMap* tm = un.kv ? &P.tm_v : &P.tm_k;
         for (int e = 0; e < P.n_loads; ++e, ++gl) {
           prefetch(u, e + kSrcPrefetch);
@@ -245,11 +260,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     // --------------------------------------------------- W and bias producer ------
     if (lane == 0) {
       const uint64_t pol = policy_evict_last();
-      uint32_t wi = 0, bl = 0;
+      uint32_t wi[kIssuers] = {0, 0}, bl = 0;   // stages filled per ring (ring = layer % 2)
       bool ok = true;
       const int chunks = 2 * k;  // 64-feature chunks of F = 128 k
       for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-        const Unit un = decode_unit(u, H, tiles);
+        const Unit un = decode_unit(u, H, A.B, tiles);
         for (int l = 0; ok && l < Lt; ++l, ++bl) {
           const int row0 = ((l * 2 + un.kv) * H + un.h) * kD;
           {  // this layer's bias row into the bias ring
@@ -268,12 +283,13 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           if (l + 1 < Lt) {
             next_row0 = (((l + 1) * 2 + un.kv) * H + un.h) * kD;
           } else if (u + static_cast<int>(gridDim.x) < n_units) {
-            const Unit nu = decode_unit(u + gridDim.x, H, tiles);
+            const Unit nu = decode_unit(u + gridDim.x, H, A.B, tiles);
             next_row0 = (nu.kv * H + nu.h) * kD;
           }
-          for (int c = 0; c < chunks; ++c, ++wi) {
-            const int st = wi % NW;
-            const uint32_t round = wi / NW;
+          const int ring = l % kIssuers;
+          for (int c = 0; c < chunks; ++c, ++wi[ring]) {
+            const int st = ring * kRing + static_cast<int>(wi[ring] % kRing);
+            const uint32_t round = wi[ring] / kRing;
             if (round > 0 &&
                 !wait_bar(smem_u32(&wempty[st]), (round - 1) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
               ok = false;
@@ -287,65 +303,82 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
         }
       }
       if (!ok) {
-        const uint32_t first = wi > static_cast<uint32_t>(NW) ? wi - NW : 0;
-        for (uint32_t i = first; i < wi; ++i) drain_wait(smem_u32(&wfull[i % NW]), (i / NW) & 1u);
+        for (int ring = 0; ring < kIssuers; ++ring) {
+          const uint32_t first = wi[ring] > static_cast<uint32_t>(kRing) ? wi[ring] - kRing : 0;
+          for (uint32_t i = first; i < wi[ring]; ++i)
+            drain_wait(smem_u32(&wfull[ring * kRing + i % kRing]), (i / kRing) & 1u);
+        }
         const uint32_t bfirst = bl > static_cast<uint32_t>(kBiasSlots) ? bl - kBiasSlots : 0;
         for (uint32_t i = bfirst; i < bl; ++i) drain_wait(smem_u32(&bias_full[i % kBiasSlots]), (i / kBiasSlots) & 1u);
       }
     }
-  } else if (warp == 1) {
-    // ---------------------------------------------------------------- MMA ---------
+  } else if (warp == 1 || warp == 3) {
+    // --------------------------------------------------------- MMA issuers --------
+    // Warp 1 issues the even target layers into accumulator 0, warp 3 the odd ones into
+    // accumulator 1.  A thread that reads shared memory (an mbarrier wait) while its own
+    // MMAs are queued stalls for about as long as they take to start, so a single issuer
+    // leaves the tensor pipe idle at every wait; with two issuers on different SM
+    // sub-partitions the other one's queued MMAs cover it.
+    const int iss = warp == 1 ? 0 : 1;
     if (lane == 0) {
       constexpr uint32_t idesc = make_idesc(kTileM, kD);
-      uint32_t ready_par = 0, wi = 0, li = 0;
+      const uint32_t d_tmem = tmem_base + iss * kAccCols;
+      uint32_t ready_par = 0, acc_n = 0, wi = 0;   // wi: stages consumed from this issuer's ring
       bool ok = true, issued = false;
-      uint32_t pack_next = __ldg(&P.use_pack[0]);
+      uint32_t pack_next = iss < Lt ? __ldg(&P.use_pack[iss]) : 0u;
       for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-        for (int l = 0; ok && l < Lt; ++l, ++li) {
+        for (int l = iss; ok && l < Lt; l += kIssuers, ++acc_n) {
           const uint32_t pack = pack_next;
-          pack_next = __ldg(&P.use_pack[l + 1 < Lt ? l + 1 : 0]);   // schedule word of the next layer
-          const uint32_t buf = li & 1u;
-          if (li >= 2 && !wait_bar(smem_u32(&acce[buf]), ((li >> 1) - 1) & 1u, abort_flag, P.status,
-                                   KVX_ERR_TIMEOUT)) {
+          const int ln = l + kIssuers < Lt ? l + kIssuers : iss;
+          pack_next = __ldg(&P.use_pack[ln]);   // schedule word of this issuer's next layer
+          if (acc_n >= 1 && !wait_bar(smem_u32(&acce[iss]), (acc_n - 1) & 1u, abort_flag, P.status,
+                                      KVX_ERR_TIMEOUT)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t d_tmem = tmem_base + buf * kAccCols;
-          for (int j = 0; ok && j < k; ++j) {
+          for (int j = 0; j < k; ++j, wi += 2) {
+            // use bits: slot | 4 first use of the tile by this issuer | 16 release the
+            // slot after this use.  The transform warps signal tready[slot][issuer] only
+            // for the loads this issuer uses, so it waits for every phase in order.
             const uint32_t f = (pack >> (5 * j)) & 31u;
-            const uint32_t s = f & 7u;
-            if (f & 8u) {  // first use of the tile: wait until the transform wrote it
-              if (!wait_bar(smem_u32(&tready[s]), (ready_par >> s) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
+            const uint32_t s = f & 3u;
+            if (f & 4u) {
+              if (!wait_bar(smem_u32(&tready[s * kIssuers + iss]), (ready_par >> s) & 1u, abort_flag, P.status,
+                            KVX_ERR_TIMEOUT)) {
                 ok = false;
                 break;
               }
               ready_par ^= 1u << s;
-              tc_fence_after();
+              tc_fence_after();   // the tile was written by other threads' tcgen05.st
+            }
+            const uint32_t st0 = iss * kRing + wi % kRing, st1 = iss * kRing + (wi + 1) % kRing;
+            if (!wait_bar(smem_u32(&wfull[st0]), (wi / kRing) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT) ||
+                !wait_bar(smem_u32(&wfull[st1]), ((wi + 1) / kRing) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
+              ok = false;
+              break;
             }
             const uint32_t a_col = tmem_base + kSlotCol0 + s * 64;
-            for (int c2 = 0; c2 < 2; ++c2, ++wi) {
-              const int st = wi % NW;
-              if (!wait_bar(smem_u32(&wfull[st]), (wi / NW) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
-                ok = false;
-                break;
-              }
-              const uint32_t b_base = smem_u32(wst + static_cast<size_t>(st) * kWStageBytes);
+            const uint32_t b0 = smem_u32(wst + static_cast<size_t>(st0) * kWStageBytes);
+            const uint32_t b1 = smem_u32(wst + static_cast<size_t>(st1) * kWStageBytes);
 #pragma unroll
-              for (int kk = 0; kk < 4; ++kk)
-                tc_mma_ts(d_tmem, a_col + c2 * 32 + kk * 8, sw128_desc(b_base + kk * 32), idesc, (j | c2 | kk) != 0);
-              issued = true;
-              tc_commit(smem_u32(&wempty[st]));
-            }
-            if (ok && (f & 16u)) tc_commit(smem_u32(&tfree[s]));   // last use before a reload
+            for (int kk = 0; kk < 4; ++kk)
+              tc_mma_ts(d_tmem, a_col + kk * 8, sw128_desc(b0 + kk * 32), idesc, (j | kk) != 0);
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              tc_mma_ts(d_tmem, a_col + 32 + kk * 8, sw128_desc(b1 + kk * 32), idesc, true);
+            issued = true;
+            tc_commit(smem_u32(&wempty[st0]));
+            tc_commit(smem_u32(&wempty[st1]));
+            if (f & 16u) tc_commit(smem_u32(&tfree[s * kIssuers + iss]));
           }
-          if (ok) tc_commit(smem_u32(&accf[buf]));
+          if (ok) tc_commit(smem_u32(&accf[iss]));
         }
       }
-      // every MMA (and every commit) must have completed before TMEM is freed
+      // every MMA (and every commit) of this issuer must have completed before TMEM is freed
       if (issued || !ok) {
-        tc_commit(smem_u32(drain));
-        drain_wait(smem_u32(drain), 0);
+        tc_commit(smem_u32(&drain[iss]));
+        drain_wait(smem_u32(&drain[iss]), 0);
       }
     }
   } else if (warp >= kFirstTransformWarp) {
@@ -355,12 +388,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     const int r = q * 32 + lane;                     // token row within the tile
     const uint32_t lane_addr = static_cast<uint32_t>(q * 32) << 16;
     const uint64_t st_pol = policy_evict_first();
-    uint32_t gl = 0, lay = 0, tl_loaded = 0, tfree_par = 0;
+    uint32_t gl = 0, lay = 0, tl_loaded = 0, tfree_par = 0, acc_n0 = 0, acc_n1 = 0;
     bool prev_store_pending = false;   // first transform warp: the previous layer's TMA store may still read its buffer
     float cs[32], sn[32];
     bool ok = true;
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-      const Unit un = decode_unit(u, H, tiles);
+      const Unit un = decode_unit(u, H, A.B, tiles);
       const int t = un.t0 + r;
       bool valid = t < A.T;
       bool bad = false;
@@ -457,10 +490,19 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
               wb[w] = pack_bf16x2(__fmaf_rn(b0, c0, -__fmul_rn(a0, s0)), __fmaf_rn(b1, c1, -__fmul_rn(a1, s1)));
             }
           }
-          const int s = __ldg(&P.load_slot[e]);
+          // load word: slot | 4 << i if issuer i used the slot's previous tile (wait for its
+          // release) | 16 << i if issuer i uses this tile (signal tready[slot][i])
+          const uint32_t lw = static_cast<uint32_t>(__ldg(&P.load_slot[e]));
+          const int s = static_cast<int>(lw & 3u);
           if ((tl_loaded >> s) & 1u) {
-            w_ok = wait_bar(smem_u32(&tfree[s]), (tfree_par >> s) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT);
-            tfree_par ^= 1u << s;
+#pragma unroll
+            for (int i = 0; i < kIssuers; ++i) {
+              if (!((lw >> (2 + i)) & 1u)) continue;
+              const int bi = s * kIssuers + i;
+              w_ok = w_ok && wait_bar(smem_u32(&tfree[bi]), (tfree_par >> bi) & 1u, abort_flag, P.status,
+                                      KVX_ERR_TIMEOUT);
+              tfree_par ^= 1u << bi;
+            }
             if (!__all_sync(0xffffffffu, w_ok)) {
               ok = false;
               break;
@@ -474,12 +516,16 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           tmem_wait_st();
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive(smem_u32(&tready[s]));
+          if (lane == 0) {
+#pragma unroll
+            for (int i = 0; i < kIssuers; ++i)
+              if ((lw >> (4 + i)) & 1u) mbar_arrive(smem_u32(&tready[s * kIssuers + i]));
+          }
           ++e;
         }
         if (!ok) break;
         // epilogue of layer l
-        const uint32_t ob_i = lay & 1u;
+        const uint32_t ob_i = lay % kOutBufs;
         uint8_t* ob = outst + ob_i * kOutBytes;
         const uint32_t bslot = lay % kBiasSlots;
         const float* bias = bias_ring + bslot * kD;
@@ -491,17 +537,19 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
             break;
           }
         }
-        if (use_tma && lay >= 2) {   // the store that last read this staging buffer is done
-          const bool w_ok = wait_bar(smem_u32(&stage_free[ob_i]), ((lay >> 1) - 1) & 1u, abort_flag, P.status,
+        if (use_tma && lay >= static_cast<uint32_t>(kOutBufs)) {   // the last store from this buffer has read it
+          const bool w_ok = wait_bar(smem_u32(&stage_free[ob_i]), ((lay / kOutBufs) - 1) & 1u, abort_flag, P.status,
                                      KVX_ERR_TIMEOUT);
           if (!__all_sync(0xffffffffu, w_ok)) {
             ok = false;
             break;
           }
         }
-        const uint32_t buf = lay & 1u;
+        const uint32_t buf = static_cast<uint32_t>(l) & 1u;   // accumulator of issuer l % 2
         {
-          const bool w_ok = wait_bar(smem_u32(&accf[buf]), (lay >> 1) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT);
+          const uint32_t acc_par = (buf ? acc_n1 : acc_n0) & 1u;
+          if (buf) ++acc_n1; else ++acc_n0;
+          const bool w_ok = wait_bar(smem_u32(&accf[buf]), acc_par, abort_flag, P.status, KVX_ERR_TIMEOUT);
           if (!__all_sync(0xffffffffu, w_ok)) {
             ok = false;
             break;
@@ -513,7 +561,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
         for (int rnd = 0; rnd < 2; ++rnd) {
           uint32_t lo[16], hi[16];
           tmem_ld_2x16(col + 16 * rnd, col + 64 + 16 * rnd, lo, hi);
-          if (rnd == 1) {  // the accumulator is free for the MMAs of layer l + 2
+          if (rnd == 1) {  // the accumulator is free for the issuer's next layer
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&acce[buf]));
@@ -577,7 +625,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           __syncwarp();
           if (lane == 0) mbar_arrive(smem_u32(&stage_full[ob_i]));
           if (warp == kFirstTransformWarp) {
-            const bool w_ok = wait_bar(smem_u32(&stage_full[ob_i]), (lay >> 1) & 1u, abort_flag, P.status,
+            const bool w_ok = wait_bar(smem_u32(&stage_full[ob_i]), (lay / kOutBufs) & 1u, abort_flag, P.status,
                                        KVX_ERR_TIMEOUT);
             if (!__all_sync(0xffffffffu, w_ok)) {
               ok = false;
@@ -613,15 +661,21 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
               if (lane == 0)
                 for (int i = 0; i < 4; ++i) bad_mask[ob_i * 4 + i] = 0u;
             }
-            // Release staging buffers exactly once per use: the previous layer's buffer
-            // once its TMA store has read it, this layer's buffer at once if it was
-            // written out row by row (no store reads it).
+            // Release each staging buffer exactly once per use, once nothing reads it any
+            // more.  One buffer: after this layer's store has read it.  Two buffers: the
+            // previous layer's buffer once its store has read it, this layer's buffer at
+            // once if it was written out row by row (no store reads it).
             if (lane == 0) {
-              if (prev_store_pending) {
-                if (clean) bulk_wait_read_but_last(); else bulk_wait_read_all();
-                mbar_arrive(smem_u32(&stage_free[ob_i ^ 1u]));
+              if constexpr (kOutBufs == 1) {
+                if (clean) bulk_wait_read_all();
+                mbar_arrive(smem_u32(&stage_free[0]));
+              } else {
+                if (prev_store_pending) {
+                  if (clean) bulk_wait_read_but_last(); else bulk_wait_read_all();
+                  mbar_arrive(smem_u32(&stage_free[ob_i ^ 1u]));
+                }
+                if (!clean) mbar_arrive(smem_u32(&stage_free[ob_i]));
               }
-              if (!clean) mbar_arrive(smem_u32(&stage_free[ob_i]));
             }
             prev_store_pending = clean;
           }
@@ -656,18 +710,18 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return fn;
 }
 
-size_t smem_bytes(int n_wst) {
-  const size_t bars =
-      (2 * kLand + 2 * kTSlots + 2 * n_wst + 2 * kAccBufs + 2 * kOutBufs + 2 * kBiasSlots + 1) * 8 + 48;
-  return 1024 + static_cast<size_t>(kLand) * kLandBytes + static_cast<size_t>(n_wst) * kWStageBytes +
-         kOutBufs * static_cast<size_t>(kOutBytes) + kBiasSlots * kBiasBytes + bars;
-}
-
 // Belady schedule of source-tile loads over the use sequence (l, j), l-major, into
-// kTSlots TMEM slots.  The victim is the resident tile whose next use is farthest away;
-// among equals, the one whose last use is earliest (its slot frees soonest).  A slot is
-// released right after the MMAs of its tile's last use before the reload, so with
-// k <= kTSlots a victim always exists and every wait ends.
+// kTSlots TMEM slots: the victim is the resident tile whose next use is farthest away;
+// among equals, the one whose last use is earliest.  Use (l, j) is issued by issuer l % 2.
+// Before a tile is overwritten, every issuer that read it releases the slot (a commit
+// after its last use of the tile) and the transform warps wait for exactly those
+// releases.  The final tiles of a unit are released for the first loads of the next one.
+// All waits follow the (l, j) order, and with k <= kTSlots a victim always exists, so
+// every wait ends.
+//   use_flags:  1 first use of the tile by its issuer (wait for tready[slot][issuer]),
+//               4 release the slot after the use
+//   load_slot:  slot | 4 << i if issuer i must release the slot's previous tile first
+//               | 16 << i if issuer i uses the tile (the transform signals its tready)
 void build_plan(const kvx_ctx* c, TcPlan* plan) {
   const int Lt = c->Lt, k = c->k, n_uses = Lt * k, S = kTSlots;
   std::vector<int> src(n_uses), next_use(n_uses);
@@ -683,9 +737,10 @@ void build_plan(const kvx_ctx* c, TcPlan* plan) {
   plan->load_first_use.clear();
   plan->use_slot.assign(n_uses, -1);
   plan->use_flags.assign(n_uses, 0);
-  std::vector<int> slot_src(S, -1), slot_next(S, INT_MAX), slot_last(S, -1);
+  std::vector<int> slot_src(S, -1), slot_next(S, INT_MAX), slot_last(S, -1), slot_load(S, -1), slot_first_load(S, -1);
+  std::vector<int> last_by(S * kIssuers, -1);   // [slot][issuer] last use of the current tile
   for (int u = 0; u < n_uses; ++u) {
-    const int l = u / k;
+    const int l = u / k, iss = l % kIssuers;
     int s = -1;
     for (int i = 0; i < S; ++i)
       if (slot_src[i] == src[u]) s = i;
@@ -701,19 +756,41 @@ void build_plan(const kvx_ctx* c, TcPlan* plan) {
           best = i;
       }
       s = best;
-      if (slot_src[s] >= 0) plan->use_flags[slot_last[s]] |= 2;
+      int word = s;
+      for (int i = 0; i < kIssuers; ++i) {
+        const int lu = last_by[s * kIssuers + i];
+        if (lu >= 0) {
+          plan->use_flags[lu] |= 4;
+          word |= 4 << i;
+        }
+        last_by[s * kIssuers + i] = -1;
+      }
+      if (slot_first_load[s] < 0) slot_first_load[s] = static_cast<int>(plan->load_slot.size());
       plan->load_layer.push_back(src[u]);
-      plan->load_slot.push_back(s);
+      plan->load_slot.push_back(word);
       plan->load_first_use.push_back(l);
       slot_src[s] = src[u];
-      plan->use_flags[u] |= 1;
+      slot_load[s] = static_cast<int>(plan->load_slot.size()) - 1;
     }
+    if (last_by[s * kIssuers + iss] < 0) {
+      plan->use_flags[u] |= 1;
+      plan->load_slot[slot_load[s]] |= 16 << iss;
+    }
+    last_by[s * kIssuers + iss] = u;
     plan->use_slot[u] = s;
     slot_next[s] = next_use[u];
     slot_last[s] = u;
   }
-  for (int i = 0; i < S; ++i)
-    if (slot_src[i] >= 0) plan->use_flags[slot_last[i]] |= 2;
+  for (int s = 0; s < S; ++s) {
+    if (slot_src[s] < 0) continue;
+    for (int i = 0; i < kIssuers; ++i) {
+      const int lu = last_by[s * kIssuers + i];
+      if (lu >= 0) {
+        plan->use_flags[lu] |= 4;
+        plan->load_slot[slot_first_load[s]] |= 4 << i;
+      }
+    }
+  }
   plan->n_loads = static_cast<int>(plan->load_layer.size());
 }
 
@@ -752,20 +829,18 @@ kvx_status tc_prepare(kvx_ctx* c, const void* W_host) {
     set_error(std::string("kvx_create: upload W^T: ") + cudaGetErrorString(e));
     return KVX_ERR_CUDA;
   }
-  // as many W stages as the shared-memory budget allows
-  int n_wst = 2;
-  while (n_wst < kMaxWStages && smem_bytes(n_wst + 1) <= kSmemLimit) ++n_wst;
   build_plan(c, &c->plan);
-  c->plan.n_wst = n_wst;
+  c->plan.n_wst = kNW;   // two rings of kRing stages
   c->plan.n_land = kLand;
   const TcPlan& p = c->plan;
-  // per target layer, one word: 5 bits per use j (slot | 8 first use | 16 release after)
+  // per target layer, one word: 5 bits per use j (slot | 4 first use by its issuer |
+  // 16 release after)
   std::vector<int32_t> pack(c->Lt, 0);
   for (int l = 0; l < c->Lt; ++l)
     for (int j = 0; j < c->k; ++j) {
       const int u = l * c->k + j;
-      const uint32_t f = static_cast<uint32_t>(p.use_slot[u]) | ((p.use_flags[u] & 1) ? 8u : 0u) |
-                         ((p.use_flags[u] & 2) ? 16u : 0u);
+      const uint32_t f = static_cast<uint32_t>(p.use_slot[u]) | ((p.use_flags[u] & 1) ? 4u : 0u) |
+                         ((p.use_flags[u] & 4) ? 16u : 0u);
       pack[l] |= static_cast<int32_t>(f << (5 * j));
     }
   std::vector<int32_t> tab;
@@ -848,7 +923,6 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   P.Lt = c->Lt;
   P.H = c->H;
   P.k = c->k;
-  P.n_wst = p.n_wst;
   P.n_loads = p.n_loads;
   P.tiles_per_seq = (a.T + kTileM - 1) / kTileM;
   const int64_t units = static_cast<int64_t>(a.B) * P.tiles_per_seq * c->H * 2;
@@ -859,7 +933,7 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   P.n_units = static_cast<int>(units);
   P.same_theta = c->theta_s == c->theta_t;
   P.rope = c->rope;
-  const size_t smem = smem_bytes(P.n_wst);
+  const size_t smem = smem_bytes();
   cudaError_t e = cudaFuncSetAttribute(tc_map_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) {
