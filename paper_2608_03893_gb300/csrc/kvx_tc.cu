@@ -69,8 +69,10 @@ constexpr int kD = 128;                             // head_dim of this kernel
 constexpr uint32_t kLandBytes = kTileM * kD * 2;    // 32 KB raw tile: two 64-column SW128 halves
 constexpr uint32_t kHalfBytes = kLandBytes / 2;     // 16 KB
 constexpr uint32_t kWStageBytes = kD * 64 * 2;      // 16 KB: 128 output channels x 64 features
-constexpr uint32_t kOutBytes = kTileM * kD * 2;     // 32 KB staging tile (two SW128 boxes)
-constexpr int kOutBufs = 2;                         // staging tiles (1 or 2)
+constexpr uint32_t kPieceBytes = 32 * 64;           // 2 KB: 32 rows x 32 channels, 64-byte swizzle
+constexpr uint32_t kWarpStageBytes = 2 * kPieceBytes; // one transform warp's share of an output tile
+constexpr int kTransformWarps = 8;
+constexpr uint32_t kOutBytes = 2 * kTransformWarps * kWarpStageBytes;   // 64 KB: two per warp
 constexpr int kTSlots = 4;                          // TMEM source-tile slots (64 columns each)
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccCols = 128;                  // one fp32 accumulator
@@ -91,9 +93,8 @@ constexpr int kNW = kRing * kIssuers;               // W stages in shared memory
 // before it; no slack is reserved.
 constexpr size_t smem_bytes() {
   return static_cast<size_t>(kLand) * kLandBytes + static_cast<size_t>(kNW) * kWStageBytes +
-         kOutBufs * static_cast<size_t>(kOutBytes) + kBiasSlots * kBiasBytes +
-         (2 * kLand + 2 * kTSlots * kIssuers + 2 * kNW + 2 * kAccBufs + 2 * kOutBufs + 2 * kBiasSlots +
-          kIssuers) * 8 + 48;
+         kOutBytes + kBiasSlots * kBiasBytes +
+         (2 * kLand + 2 * kTSlots * kIssuers + 2 * kNW + 2 * kAccBufs + 2 * kBiasSlots + kIssuers) * 8 + 16;
 }
 static_assert(smem_bytes() <= kSmemLimit, "shared-memory layout exceeds the per-CTA limit");
 
@@ -147,7 +148,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
   uint8_t* land = smem;
   uint8_t* wst = land + kLand * kLandBytes;            // [2 rings][kRing] W stages
   uint8_t* outst = wst + static_cast<size_t>(kNW) * kWStageBytes;
-  float* bias_ring = reinterpret_cast<float*>(outst + kOutBufs * kOutBytes);   // [4][128] fp32
+  float* bias_ring = reinterpret_cast<float*>(outst + kOutBytes);   // [4][128] fp32
   uint64_t* bars = reinterpret_cast<uint64_t*>(bias_ring + kBiasSlots * kD);
   uint64_t* land_full = bars;                    // [2] TMA landed
   uint64_t* land_empty = land_full + kLand;      // [2] transform read it (8 warps)
@@ -157,14 +158,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
   uint64_t* wempty = wfull + kNW;                // [2][kRing]
   uint64_t* accf = wempty + kNW;                 // [2] accumulator ready
   uint64_t* acce = accf + kAccBufs;              // [2] accumulator drained (8 warps)
-  uint64_t* stage_full = acce + kAccBufs;        // [2] staging tile written (8 warps)
-  uint64_t* stage_free = stage_full + kOutBufs;  // [2] staging tile read by its store
-  uint64_t* bias_full = stage_free + kOutBufs;   // [4] bias row landed
+  uint64_t* bias_full = acce + kAccBufs;         // [4] bias row landed
   uint64_t* bias_empty = bias_full + kBiasSlots; // [4] bias row used (8 warps)
   uint64_t* drain = bias_empty + kBiasSlots;     // [2] per issuer
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + kIssuers);
   volatile uint32_t* abort_flag = tmem_holder + 1;
-  uint32_t* bad_mask = tmem_holder + 2;          // [2][4] rows of a staged tile with a bad position
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -184,17 +182,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
       mbar_init(smem_u32(&accf[i]), 1);
       mbar_init(smem_u32(&acce[i]), 8);
     }
-    for (int i = 0; i < kOutBufs; ++i) {
-      mbar_init(smem_u32(&stage_full[i]), 8);
-      mbar_init(smem_u32(&stage_free[i]), 1);
-    }
     for (int i = 0; i < kBiasSlots; ++i) {
       mbar_init(smem_u32(&bias_full[i]), 1);
       mbar_init(smem_u32(&bias_empty[i]), 8);
     }
     for (int i = 0; i < kIssuers; ++i) mbar_init(smem_u32(&drain[i]), 1);
     *abort_flag = 0u;
-    for (int i = 0; i < 2 * 4; ++i) bad_mask[i] = 0u;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     fence_proxy_async_smem();
   }
@@ -258,58 +251,111 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     }
   } else if (warp == 2) {
     // --------------------------------------------------- W and bias producer ------
+    // One thread feeds three independent streams and polls each one's next free slot
+    // without blocking: the W ring of each issuer (the 2k stages of every layer of its
+    // parity, in order) and the per-layer bias rows (every layer, in order).  Blocking on
+    // one ring would starve the other issuer.
     if (lane == 0) {
       const uint64_t pol = policy_evict_last();
-      uint32_t wi[kIssuers] = {0, 0}, bl = 0;   // stages filled per ring (ring = layer % 2)
-      bool ok = true;
       const int chunks = 2 * k;  // 64-feature chunks of F = 128 k
-      for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-        const Unit un = decode_unit(u, H, A.B, tiles);
-        for (int l = 0; ok && l < Lt; ++l, ++bl) {
-          const int row0 = ((l * 2 + un.kv) * H + un.h) * kD;
-          {  // this layer's bias row into the bias ring
-            const int bs = bl % kBiasSlots;
-            const uint32_t round = bl / kBiasSlots;
-            if (round > 0 &&
-                !wait_bar(smem_u32(&bias_empty[bs]), (round - 1) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
-              ok = false;
-              break;
+      int wu[kIssuers], wl[kIssuers], wc[kIssuers], wkv[kIssuers], wh[kIssuers];
+      uint32_t wn[kIssuers];     // stages filled into ring r
+      for (int r = 0; r < kIssuers; ++r) {
+        wu[r] = blockIdx.x;
+        wl[r] = r;
+        wc[r] = 0;
+        wn[r] = 0;
+        const Unit un = decode_unit(wu[r] < n_units ? wu[r] : 0, H, A.B, tiles);
+        wkv[r] = un.kv;
+        wh[r] = un.h;
+      }
+      int bu = blockIdx.x, blay = 0;
+      uint32_t bn = 0;           // bias rows filled
+      Unit bun = decode_unit(bu < n_units ? bu : 0, H, A.B, tiles);
+      bool ok = true;
+      uint64_t t_idle = 0;
+      uint32_t spins = 0;
+      for (;;) {
+        bool busy = false, progress = false;
+#pragma unroll
+        for (int r = 0; r < kIssuers; ++r) {
+          if (wl[r] >= Lt || wu[r] >= n_units) continue;   // done (or issuer r has no layer)
+          busy = true;
+          const int st = r * kRing + static_cast<int>(wn[r] % kRing);
+          const uint32_t round = wn[r] / kRing;
+          if (round > 0 && !mbar_test_wait(smem_u32(&wempty[st]), (round - 1) & 1u)) continue;
+          // L2 prefetch of the same chunk of this ring's next layer
+          int nl = wl[r] + kIssuers, nu = wu[r], nkv = wkv[r], nh = wh[r];
+          if (nl >= Lt) {
+            nl = r;
+            nu += gridDim.x;
+            if (nu < n_units) {
+              const Unit nun = decode_unit(nu, H, A.B, tiles);
+              nkv = nun.kv;
+              nh = nun.h;
             }
+          }
+          if (nu < n_units) tma_prefetch_2d(&P.tm_w, wc[r] * 64, ((nl * 2 + nkv) * H + nh) * kD);
+          mbar_expect_tx(smem_u32(&wfull[st]), kWStageBytes);
+          tma_load_2d(smem_u32(wst + static_cast<size_t>(st) * kWStageBytes), &P.tm_w, smem_u32(&wfull[st]),
+                      wc[r] * 64, ((wl[r] * 2 + wkv[r]) * H + wh[r]) * kD, pol);
+          ++wn[r];
+          if (++wc[r] == chunks) {
+            wc[r] = 0;
+            wl[r] = nl;
+            wu[r] = nu;
+            wkv[r] = nkv;
+            wh[r] = nh;
+          }
+          progress = true;
+        }
+        if (bu < n_units) {
+          busy = true;
+          const int bs = static_cast<int>(bn % kBiasSlots);
+          const uint32_t round = bn / kBiasSlots;
+          if (round == 0 || mbar_test_wait(smem_u32(&bias_empty[bs]), (round - 1) & 1u)) {
+            const int row0 = ((blay * 2 + bun.kv) * H + bun.h) * kD;
             mbar_expect_tx(smem_u32(&bias_full[bs]), kBiasBytes);
             bulk_load(smem_u32(bias_ring + bs * kD), P.bias + static_cast<size_t>(row0), kBiasBytes,
                       smem_u32(&bias_full[bs]));
-          }
-          int next_row0 = -1;
-          if (l + 1 < Lt) {
-            next_row0 = (((l + 1) * 2 + un.kv) * H + un.h) * kD;
-          } else if (u + static_cast<int>(gridDim.x) < n_units) {
-            const Unit nu = decode_unit(u + gridDim.x, H, A.B, tiles);
-            next_row0 = (nu.kv * H + nu.h) * kD;
-          }
-          const int ring = l % kIssuers;
-          for (int c = 0; c < chunks; ++c, ++wi[ring]) {
-            const int st = ring * kRing + static_cast<int>(wi[ring] % kRing);
-            const uint32_t round = wi[ring] / kRing;
-            if (round > 0 &&
-                !wait_bar(smem_u32(&wempty[st]), (round - 1) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
-              ok = false;
-              break;
+            ++bn;
+            if (++blay == Lt) {
+              blay = 0;
+              bu += gridDim.x;
+              if (bu < n_units) bun = decode_unit(bu, H, A.B, tiles);
             }
-            if (next_row0 >= 0) tma_prefetch_2d(&P.tm_w, c * 64, next_row0);
-            mbar_expect_tx(smem_u32(&wfull[st]), kWStageBytes);
-            tma_load_2d(smem_u32(wst + static_cast<size_t>(st) * kWStageBytes), &P.tm_w, smem_u32(&wfull[st]),
-                        c * 64, row0, pol);
+            progress = true;
+          }
+        }
+        if (!busy) break;
+        if (progress) {
+          spins = 0;
+          t_idle = 0;
+          continue;
+        }
+        if ((++spins & 63u) == 0) {   // bounded: no slot freed for 4 s raises KVX_ERR_TIMEOUT
+          if (*abort_flag) {
+            ok = false;
+            break;
+          }
+          const uint64_t now = global_timer();
+          if (t_idle == 0) {
+            t_idle = now;
+          } else if (now - t_idle > kTimeoutNs) {
+            *abort_flag = 1u;
+            report(P.status, KVX_ERR_TIMEOUT);
+            ok = false;
+            break;
           }
         }
       }
-      if (!ok) {
-        for (int ring = 0; ring < kIssuers; ++ring) {
-          const uint32_t first = wi[ring] > static_cast<uint32_t>(kRing) ? wi[ring] - kRing : 0;
-          for (uint32_t i = first; i < wi[ring]; ++i)
-            drain_wait(smem_u32(&wfull[ring * kRing + i % kRing]), (i / kRing) & 1u);
+      if (!ok) {   // the most recent fills of each ring may still be landing
+        for (int r = 0; r < kIssuers; ++r) {
+          const uint32_t first = wn[r] > static_cast<uint32_t>(kRing) ? wn[r] - kRing : 0;
+          for (uint32_t i = first; i < wn[r]; ++i) drain_wait(smem_u32(&wfull[r * kRing + i % kRing]), (i / kRing) & 1u);
         }
-        const uint32_t bfirst = bl > static_cast<uint32_t>(kBiasSlots) ? bl - kBiasSlots : 0;
-        for (uint32_t i = bfirst; i < bl; ++i) drain_wait(smem_u32(&bias_full[i % kBiasSlots]), (i / kBiasSlots) & 1u);
+        const uint32_t bfirst = bn > static_cast<uint32_t>(kBiasSlots) ? bn - kBiasSlots : 0;
+        for (uint32_t i = bfirst; i < bn; ++i) drain_wait(smem_u32(&bias_full[i % kBiasSlots]), (i / kBiasSlots) & 1u);
       }
     }
   } else if (warp == 1 || warp == 3) {
@@ -389,7 +435,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     const uint32_t lane_addr = static_cast<uint32_t>(q * 32) << 16;
     const uint64_t st_pol = policy_evict_first();
     uint32_t gl = 0, lay = 0, tl_loaded = 0, tfree_par = 0, acc_n0 = 0, acc_n1 = 0;
-    bool prev_store_pending = false;   // first transform warp: the previous layer's TMA store may still read its buffer
+    uint8_t* wstage = outst + static_cast<size_t>(warp - kFirstTransformWarp) * 2 * kWarpStageBytes;
     float cs[32], sn[32];
     bool ok = true;
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
@@ -424,7 +470,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           }
         }
       }
-      const bool use_tma = !A.paged;   // contiguous targets: staged tiles + TMA stores
+      // contiguous targets: each warp stages its 32 rows and writes them with TMA stores,
+      // unless one of its rows has an out-of-range position: then its valid rows are
+      // written directly (rows past the sequence end are clipped by the tensor map)
+      const bool warp_tma = !A.paged && __ballot_sync(0xffffffffu, bad) == 0u;
       if (un.kv == 0) {
 #pragma unroll
         for (int m = 0; m < 32; ++m) {
@@ -525,20 +574,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
         }
         if (!ok) break;
         // epilogue of layer l
-        const uint32_t ob_i = lay % kOutBufs;
-        uint8_t* ob = outst + ob_i * kOutBytes;
         const uint32_t bslot = lay % kBiasSlots;
         const float* bias = bias_ring + bslot * kD;
         {
           const bool w_ok = wait_bar(smem_u32(&bias_full[bslot]), (lay / kBiasSlots) & 1u, abort_flag, P.status,
-                                     KVX_ERR_TIMEOUT);
-          if (!__all_sync(0xffffffffu, w_ok)) {
-            ok = false;
-            break;
-          }
-        }
-        if (use_tma && lay >= static_cast<uint32_t>(kOutBufs)) {   // the last store from this buffer has read it
-          const bool w_ok = wait_bar(smem_u32(&stage_free[ob_i]), ((lay / kOutBufs) - 1) & 1u, abort_flag, P.status,
                                      KVX_ERR_TIMEOUT);
           if (!__all_sync(0xffffffffu, w_ok)) {
             ok = false;
@@ -556,6 +595,13 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           }
         }
         tc_fence_after();
+        // this warp's staging buffer for the layer; the store that read it two layers ago
+        // (this thread's bulk group before last) must be done reading
+        uint8_t* sb = wstage + (lay & 1u) * kWarpStageBytes;
+        if (!A.paged && lay >= 2) {
+          if (lane == 0) bulk_wait_read_but_last();
+          __syncwarp();
+        }
         const uint32_t col = tmem_base + lane_addr + buf * kAccCols + 32 * g;
 #pragma unroll
         for (int rnd = 0; rnd < 2; ++rnd) {
@@ -599,15 +645,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
                             pack_bf16x2(yhi[6], yhi[7]));
           v[3] = make_uint4(pack_bf16x2(yhi[8], yhi[9]), pack_bf16x2(yhi[10], yhi[11]),
                             pack_bf16x2(yhi[12], yhi[13]), pack_bf16x2(yhi[14], yhi[15]));
-          if (use_tma) {
-            // staging tile: box 0 = channels 0..63, box 1 = channels 64..127, rows of 128 B,
-            // 128-byte swizzle (16-byte chunk index XOR row % 8)
-            const int ch = c_lo >> 3;  // 16-byte chunk of channel c_lo within a box row
-            uint8_t* row0 = ob + r * 128;
-            *reinterpret_cast<uint4*>(row0 + ((ch ^ (r & 7)) << 4)) = v[0];
-            *reinterpret_cast<uint4*>(row0 + (((ch + 1) ^ (r & 7)) << 4)) = v[1];
-            *reinterpret_cast<uint4*>(row0 + kHalfBytes + ((ch ^ (r & 7)) << 4)) = v[2];
-            *reinterpret_cast<uint4*>(row0 + kHalfBytes + (((ch + 1) ^ (r & 7)) << 4)) = v[3];
+          if (warp_tma) {
+            // two 32-row x 64-byte pieces (channels 32g.. and 64+32g..), 64-byte swizzle:
+            // 16-byte chunk index XOR (row / 2) % 4
+            const int sw = (lane >> 1) & 3;
+            uint8_t* prow = sb + lane * 64;
+            *reinterpret_cast<uint4*>(prow + (((2 * rnd) ^ sw) << 4)) = v[0];
+            *reinterpret_cast<uint4*>(prow + (((2 * rnd + 1) ^ sw) << 4)) = v[1];
+            *reinterpret_cast<uint4*>(prow + kPieceBytes + (((2 * rnd) ^ sw) << 4)) = v[2];
+            *reinterpret_cast<uint4*>(prow + kPieceBytes + (((2 * rnd + 1) ^ sw) << 4)) = v[3];
           } else if (valid) {
             __nv_bfloat16* out = dst + static_cast<int64_t>(l) * A.ts[0] + row_off;
             st_global_hint(out + c_lo, v[0], st_pol);
@@ -618,71 +664,25 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&bias_empty[bslot]));
-        if (use_tma) {
-          // hand the staged tile to transform thread 0 (the first transform warp)
-          if (bad && g == 0) atomicOr(&bad_mask[ob_i * 4 + (r >> 5)], 1u << (r & 31));
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(smem_u32(&stage_full[ob_i]));
-          if (warp == kFirstTransformWarp) {
-            const bool w_ok = wait_bar(smem_u32(&stage_full[ob_i]), (lay / kOutBufs) & 1u, abort_flag, P.status,
-                                       KVX_ERR_TIMEOUT);
-            if (!__all_sync(0xffffffffu, w_ok)) {
-              ok = false;
-              break;
+        if (!A.paged) {
+          // every contiguous-target layer commits one bulk group per warp (empty when the
+          // warp wrote its rows directly), so "all but the last" above means this buffer
+          if (warp_tma) {
+            fence_proxy_async_smem();
+            __syncwarp();
+          }
+          if (lane == 0) {
+            if (warp_tma && un.t0 + 32 * q < A.T) {   // skip a box wholly past the sequence end
+              const uint32_t src = smem_u32(sb);
+              tma_store_5d(tm_out, src, 32 * g, un.t0 + 32 * q, un.h, un.b, l);
+              tma_store_5d(tm_out, src + kPieceBytes, 64 + 32 * g, un.t0 + 32 * q, un.h, un.b, l);
             }
-            const uint32_t m0 = bad_mask[ob_i * 4], m1 = bad_mask[ob_i * 4 + 1], m2 = bad_mask[ob_i * 4 + 2],
-                           m3 = bad_mask[ob_i * 4 + 3];
-            const bool clean = (m0 | m1 | m2 | m3) == 0u;
-            if (clean) {
-              if (lane == 0) {
-                const uint32_t src = smem_u32(ob);
-                tma_store_5d(tm_out, src, 0, un.t0, un.h, un.b, l);
-                tma_store_5d(tm_out, src + kHalfBytes, 64, un.t0, un.h, un.b, l);
-                bulk_commit_group();
-              }
-            } else {
-              // write the rows with a valid position one by one (lane j: rows j, j+32, ...)
-              __nv_bfloat16* base_out = dst + static_cast<int64_t>(l) * A.ts[0];
-              for (int rr = lane; rr < kTileM; rr += 32) {
-                const uint32_t mw = rr < 32 ? m0 : rr < 64 ? m1 : rr < 96 ? m2 : m3;
-                const int trow = un.t0 + rr;
-                if (trow >= A.T || ((mw >> (rr & 31)) & 1u)) continue;
-                __nv_bfloat16* orow =
-                    base_out + un.b * A.ts[1] + un.h * A.ts[2] + static_cast<int64_t>(trow) * A.ts[3];
-                for (int c16 = 0; c16 < 16; ++c16) {   // 16-byte chunk c16 of the 256-byte row
-                  const int box = c16 >> 3, chk = c16 & 7;
-                  const uint4 v = *reinterpret_cast<const uint4*>(ob + box * kHalfBytes + rr * 128 +
-                                                                  ((chk ^ (rr & 7)) << 4));
-                  st_global_hint(orow + 8 * c16, v, st_pol);
-                }
-              }
-              __syncwarp();
-              if (lane == 0)
-                for (int i = 0; i < 4; ++i) bad_mask[ob_i * 4 + i] = 0u;
-            }
-            // Release each staging buffer exactly once per use, once nothing reads it any
-            // more.  One buffer: after this layer's store has read it.  Two buffers: the
-            // previous layer's buffer once its store has read it, this layer's buffer at
-            // once if it was written out row by row (no store reads it).
-            if (lane == 0) {
-              if constexpr (kOutBufs == 1) {
-                if (clean) bulk_wait_read_all();
-                mbar_arrive(smem_u32(&stage_free[0]));
-              } else {
-                if (prev_store_pending) {
-                  if (clean) bulk_wait_read_but_last(); else bulk_wait_read_all();
-                  mbar_arrive(smem_u32(&stage_free[ob_i ^ 1u]));
-                }
-                if (!clean) mbar_arrive(smem_u32(&stage_free[ob_i]));
-              }
-            }
-            prev_store_pending = clean;
+            bulk_commit_group();
           }
         }
       }
     }
-    if (warp == kFirstTransformWarp && lane == 0) bulk_wait_all();
+    if (!A.paged && lane == 0) bulk_wait_all();   // this warp's stores are complete
   }
 
   tc_fence_before();
@@ -885,7 +885,8 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
       return KVX_ERR_UNSUPPORTED;
     }
   }
-  if (!a.paged) {  // target maps for the TMA-store epilogue: dims (d, T, H, B, L_t)
+  if (!a.paged) {  // target maps for the per-warp TMA stores: dims (d, T, H, B, L_t), box 32 x 32
+    const cuuint32_t tbox[5] = {32, 32, 1, 1, 1};
     const cuuint64_t tdims[5] = {static_cast<cuuint64_t>(kD), static_cast<cuuint64_t>(a.T),
                                  static_cast<cuuint64_t>(c->H), static_cast<cuuint64_t>(a.B),
                                  static_cast<cuuint64_t>(c->Lt)};
@@ -893,8 +894,8 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
                                 static_cast<cuuint64_t>(a.ts[1]) * 2, static_cast<cuuint64_t>(a.ts[0]) * 2};
     for (int kv = 0; kv < 2; ++kv) {
       CUresult r = encode(kv ? &P.tm_out_v : &P.tm_out_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5,
-                          kv ? a.tgt_v : a.tgt_k, tdims, tstr, box, ones, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                          kv ? a.tgt_v : a.tgt_k, tdims, tstr, tbox, ones, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
       if (r != CUDA_SUCCESS) {
         set_error("kvx_map: target tensor map rejected (strides or sizes)");
