@@ -23,6 +23,7 @@ the data path; a MAX all-reduce of the elapsed time only).
 """
 import argparse
 import hashlib
+import re
 import json
 import os
 import statistics
@@ -68,10 +69,23 @@ def load_peaks():
     return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, source="fallback")
 
 
-def kernel_hash():
+def code_only(text):
+    """Source text without // comments and blank lines (a comment edit keeps the hash)."""
+    out = []
+    for ln in text.splitlines():
+        ln = re.sub(r"//.*$", "", ln).rstrip()
+        if ln:
+            out.append(ln)
+    return "\n".join(out)
+
+
+def kernel_hash(read=None):
+    """sha256 (16 hex digits) of the tensor-core kernel's code, the key of the committed
+    traffic figure."""
+    read = read or (lambda f: open(os.path.join(ROOT, f), encoding="utf-8").read())
     h = hashlib.sha256()
     for f in KERNEL_SOURCES:
-        h.update(open(os.path.join(ROOT, f), "rb").read())
+        h.update(code_only(read(f)).encode())
     return h.hexdigest()[:16]
 
 

@@ -18,27 +18,27 @@
 //
 // Contraction of target layer l: D[128 tok x 128 ch] = X[128 x kd] W[kd x 128] on tcgen05
 // (cta_group::1, M = N = 128, K = 16 per instruction: the full-rate shape), A from TMEM,
-// B = W^T from a ring of 16 KB shared-memory stages (128 output channels x 64 features,
-// 128-byte swizzle), D in one of two 128-column fp32 TMEM accumulators.
+// B = W^T from shared-memory stages of 16 KB (128 output channels x 64 features, 128-byte
+// swizzle), D in one of two 128-column fp32 TMEM accumulators.
 //
 // Warp roles (384 threads):
-//   warp 0      TMA producer of raw source tiles into shared-memory landing buffers
+//   warp 0      TMA producer of raw source tiles into the shared-memory landing buffer
 //               (plus TMA L2 prefetch of tiles a few loads ahead)
-//   warp 1      TMEM allocator (all 512 columns) and MMA issuer (one thread)
-//   warp 2      TMA producer of W^T stages and of each layer's bias row (plus L2
-//               prefetch of the next layer's W)
-//   warp 3      idle
+//   warp 1      TMEM allocator (all 512 columns); issuer of the even target layers
+//   warp 3      issuer of the odd target layers.  Each issuer owns one accumulator, one
+//               ring of W stages and one tready/tfree barrier per slot.
+//   warp 2      one thread feeding three streams without blocking: the W ring of each
+//               issuer and the per-layer bias rows (plus L2 prefetch of upcoming W)
 //   warps 4-11  two transform warpgroups (one warp per TMEM lane quarter, warp % 4).
 //               Thread (group g, row r) owns token row r (= TMEM lane r) and the 32 RoPE
 //               pairs 32g .. 32g+31 (channels i and i + 64).
 //               Prologue: landing buffer -> registers -> (keys) strip the source RoPE in
 //               fp32, round to bf16 -> tcgen05.st into the tile's TMEM slot.
-//               Epilogue: TMEM -> registers, + bias, (keys) target RoPE, bf16, into a
-//               shared-memory staging tile written out by a TMA store
-//               (contiguous targets), or 16-byte stores through the block table (paged).
-//               Transform thread 0 issues the TMA stores; a staged tile holding a row
-//               with an out-of-range position is instead written row by row by its warp,
-//               skipping the bad rows.
+//               Epilogue: TMEM -> registers, + bias, (keys) target RoPE, bf16.  For a
+//               contiguous target each warp stages its 32 rows x 2 x 32 channels
+//               (64-byte swizzle) and writes them with its own TMA stores; a warp with a
+//               row at an out-of-range position writes its valid rows directly.  Paged
+//               targets take 16-byte stores through the block table.
 //
 // Every mbarrier wait is bounded: after 4 s the kernel raises KVX_ERR_TIMEOUT in the
 // status word, sets a shared abort flag that every role polls, waits (again bounded)
