@@ -23,7 +23,6 @@
 //
 // Warp roles (384 threads):
 //   warp 0      TMA producer of raw source tiles into the shared-memory landing buffer
-//               (plus TMA L2 prefetch of tiles a few loads ahead)
 //   warp 1      TMEM allocator (all 512 columns); issuer of the even target layers
 //   warp 3      issuer of the odd target layers.  Each issuer owns one accumulator, one
 //               ring of W stages and one tready/tfree barrier per slot.
@@ -72,20 +71,20 @@ constexpr uint32_t kWStageBytes = kD * 64 * 2;      // 16 KB: 128 output channel
 constexpr uint32_t kPieceBytes = 32 * 64;           // 2 KB: 32 rows x 32 channels, 64-byte swizzle
 constexpr uint32_t kWarpStageBytes = 2 * kPieceBytes; // one transform warp's share of an output tile
 constexpr int kTransformWarps = 8;
-constexpr uint32_t kOutBytes = 2 * kTransformWarps * kWarpStageBytes;   // 64 KB: two per warp
+constexpr int kStageBufs = 1;                       // staging buffers per transform warp
+constexpr uint32_t kOutBytes = kStageBufs * kTransformWarps * kWarpStageBytes;
 constexpr int kTSlots = 4;                          // TMEM source-tile slots (64 columns each)
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccCols = 128;                  // one fp32 accumulator
 constexpr int kAccBufs = 2;
 constexpr uint32_t kSlotCol0 = kAccBufs * kAccCols; // 256: first source-slot column
-constexpr int kLand = 1;                            // landing buffers (tiles are L2-prefetched ahead)
+constexpr int kLand = 2;                            // landing buffers for raw source tiles
 constexpr int kIssuers = 2;                         // MMA-issuing threads (even / odd target layers)
-constexpr int kSrcPrefetch = 6;                     // source loads prefetched into L2 ahead
 constexpr int kBiasSlots = 4;                       // per-layer bias rows staged ahead (512 B each)
 constexpr uint32_t kBiasBytes = kD * 4;
 constexpr size_t kSmemLimit = 232448;               // 227 KB opt-in per CTA
 
-constexpr int kRing = 4;                            // W stages per issuer ring (two uses)
+constexpr int kRing = 4;                            // W stages per issuer ring
 constexpr int kNW = kRing * kIssuers;               // W stages in shared memory
 
 // Dynamic shared memory: the 128-byte-swizzled buffers need 1024-byte alignment, which
@@ -97,6 +96,7 @@ constexpr size_t smem_bytes() {
          (2 * kLand + 2 * kTSlots * kIssuers + 2 * kNW + 2 * kAccBufs + 2 * kBiasSlots + kIssuers) * 8 + 16;
 }
 static_assert(smem_bytes() <= kSmemLimit, "shared-memory layout exceeds the per-CTA limit");
+static_assert(kRing >= 2, "each W ring must hold one use (two stages)");
 
 struct TcParams {
   CUtensorMap tm_k;      // source keys   [L_s][B][H][T][128] bf16, box 64 x 128
@@ -107,7 +107,6 @@ struct TcParams {
   MapArgs a;
   const int32_t* load_layer;   // [n_loads] source layer of load e
   const int32_t* load_slot;    // [n_loads] TMEM slot
-  const int32_t* load_first;   // [n_loads] first target layer using the load
   const uint32_t* use_pack;    // [L_t] per use j: 5 bits at 5j = slot | 8 first use | 16 release after
   const float* bias;           // [L_t][2][H][128] fp32
   int32_t* status;
@@ -211,33 +210,21 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
       const uint64_t pol = policy_evict_first();
       uint32_t gl = 0;
       bool ok = true;
-      auto prefetch = [&](int u, int e) {
-        while (e >= P.n_loads) {
-          e -= P.n_loads;
-          u += gridDim.x;
-        }
-        if (u >= n_units) return;
-        const Unit pu = decode_unit(u, H, A.B, tiles);
-        const CUtensorMap* ptm = pu.kv ? &P.tm_v : &P.tm_k;
-        const int L = __ldg(&P.load_layer[e]);
-        tma_prefetch_5d(ptm, 0, pu.t0, pu.h, pu.b, L);
-        tma_prefetch_5d(ptm, 64, pu.t0, pu.h, pu.b, L);
-      };
-      if (static_cast<int>(blockIdx.x) < n_units)
-        for (int e = 0; e < kSrcPrefetch; ++e) prefetch(blockIdx.x, e);
+      // No L2 prefetch of upcoming source tiles: under this kernel's streaming traffic a
+      // tile prefetched a few loads ahead was often evicted before its load (about 1 GB of
+      // extra DRAM reads per 8192 tokens), so each tile is read once, by its TMA load.
       for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
         const Unit un = decode_unit(u, H, A.B, tiles);
         const CUtensorMap* tm = un.kv ? &P.tm_v : &P.tm_k;
         for (int e = 0; e < P.n_loads; ++e, ++gl) {
-          prefetch(u, e + kSrcPrefetch);
           const int lb = gl % kLand;
           const uint32_t round = gl / kLand;
+          const int L = __ldg(&P.load_layer[e]);
           if (round > 0 && !wait_bar(smem_u32(&land_empty[lb]), (round - 1) & 1u, abort_flag, P.status,
                                      KVX_ERR_TIMEOUT)) {
             ok = false;
             break;
           }
-          const int L = __ldg(&P.load_layer[e]);
           const uint32_t dst = smem_u32(land + static_cast<size_t>(lb) * kLandBytes);
           mbar_expect_tx(smem_u32(&land_full[lb]), kLandBytes);
           tma_load_5d(dst, tm, smem_u32(&land_full[lb]), 0, un.t0, un.h, un.b, L, pol);
@@ -435,7 +422,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     const uint32_t lane_addr = static_cast<uint32_t>(q * 32) << 16;
     const uint64_t st_pol = policy_evict_first();
     uint32_t gl = 0, lay = 0, tl_loaded = 0, tfree_par = 0, acc_n0 = 0, acc_n1 = 0;
-    uint8_t* wstage = outst + static_cast<size_t>(warp - kFirstTransformWarp) * 2 * kWarpStageBytes;
+    uint8_t* wstage = outst + static_cast<size_t>(warp - kFirstTransformWarp) * kStageBufs * kWarpStageBytes;
     float cs[32], sn[32];
     bool ok = true;
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
@@ -485,9 +472,18 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
       __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(un.kv ? A.tgt_v : A.tgt_k);
       const CUtensorMap* tm_out = un.kv ? &P.tm_out_v : &P.tm_out_k;
       int e = 0;
+      uint32_t pk_next = __ldg(&P.use_pack[0]);
       for (int l = 0; ok && l < Lt; ++l, ++lay) {
-        // prologue: the source tiles whose first use is at most layer l + 1
-        while (e < P.n_loads && __ldg(&P.load_first[e]) <= l + 1) {
+        // Schedule word of layer l (read one layer ahead): bits 20.. count the loads to
+        // write before its epilogue, those first used by layer l + 1 (and, for layer 0,
+        // by layer 0).
+        const uint32_t pk = pk_next;
+        pk_next = __ldg(&P.use_pack[l + 1 < Lt ? l + 1 : 0]);
+        const int e_end = e + static_cast<int>(pk >> 20);
+        for (; e < e_end; ++e) {   // prologue
+          // load word: slot | 4 << i if issuer i used the slot's previous tile (wait for its
+          // release) | 16 << i if issuer i uses this tile (signal tready[slot][i])
+          const uint32_t lw = static_cast<uint32_t>(__ldg(&P.load_slot[e]));
           const int lb = gl % kLand;
           bool w_ok = wait_bar(smem_u32(&land_full[lb]), (gl / kLand) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT);
           if (!__all_sync(0xffffffffu, w_ok)) {
@@ -539,9 +535,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
               wb[w] = pack_bf16x2(__fmaf_rn(b0, c0, -__fmul_rn(a0, s0)), __fmaf_rn(b1, c1, -__fmul_rn(a1, s1)));
             }
           }
-          // load word: slot | 4 << i if issuer i used the slot's previous tile (wait for its
-          // release) | 16 << i if issuer i uses this tile (signal tready[slot][i])
-          const uint32_t lw = static_cast<uint32_t>(__ldg(&P.load_slot[e]));
           const int s = static_cast<int>(lw & 3u);
           if ((tl_loaded >> s) & 1u) {
 #pragma unroll
@@ -570,7 +563,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
             for (int i = 0; i < kIssuers; ++i)
               if ((lw >> (4 + i)) & 1u) mbar_arrive(smem_u32(&tready[s * kIssuers + i]));
           }
-          ++e;
         }
         if (!ok) break;
         // epilogue of layer l
@@ -595,11 +587,13 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           }
         }
         tc_fence_after();
-        // this warp's staging buffer for the layer; the store that read it two layers ago
-        // (this thread's bulk group before last) must be done reading
-        uint8_t* sb = wstage + (lay & 1u) * kWarpStageBytes;
-        if (!A.paged && lay >= 2) {
-          if (lane == 0) bulk_wait_read_but_last();
+        // this warp's staging buffer for the layer; the store that last read it (this
+        // thread's bulk group kStageBufs layers ago) must be done reading
+        uint8_t* sb = wstage + (lay % kStageBufs) * kWarpStageBytes;
+        if (!A.paged && lay >= static_cast<uint32_t>(kStageBufs)) {
+          if (lane == 0) {
+            if constexpr (kStageBufs == 1) bulk_wait_read_all(); else bulk_wait_read_but_last();
+          }
           __syncwarp();
         }
         const uint32_t col = tmem_base + lane_addr + buf * kAccCols + 32 * g;
@@ -666,7 +660,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
         if (lane == 0) mbar_arrive(smem_u32(&bias_empty[bslot]));
         if (!A.paged) {
           // every contiguous-target layer commits one bulk group per warp (empty when the
-          // warp wrote its rows directly), so "all but the last" above means this buffer
+          // warp wrote its rows directly), so the group count above identifies the buffer
           if (warp_tma) {
             fence_proxy_async_smem();
             __syncwarp();
@@ -843,6 +837,10 @@ kvx_status tc_prepare(kvx_ctx* c, const void* W_host) {
                          ((p.use_flags[u] & 4) ? 16u : 0u);
       pack[l] |= static_cast<int32_t>(f << (5 * j));
     }
+  // bits 20..: loads the transform warps write before the epilogue of layer l
+  std::vector<int32_t> before(c->Lt, 0);
+  for (int e = 0; e < p.n_loads; ++e) ++before[std::max(p.load_first_use[e] - 1, 0)];
+  for (int l = 0; l < c->Lt; ++l) pack[l] |= before[l] << 20;
   std::vector<int32_t> tab;
   tab.insert(tab.end(), p.load_layer.begin(), p.load_layer.end());
   tab.insert(tab.end(), p.load_slot.begin(), p.load_slot.end());
@@ -917,7 +915,6 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   P.a = a;
   P.load_layer = c->d_plan;
   P.load_slot = c->d_plan + p.n_loads;
-  P.load_first = c->d_plan + 2 * p.n_loads;
   P.use_pack = reinterpret_cast<const uint32_t*>(c->d_plan + 3 * p.n_loads);
   P.bias = c->d_b;
   P.status = c->d_status;

@@ -90,6 +90,31 @@ def test_bf16_small_full(kname, over):
     _small(name, KERNELS[kname], **over)
 
 
+@pytest.mark.parametrize("over", [
+    dict(Ls=6, Lt=5, H=2, B=2, T=300, k=3),
+    dict(Ls=9, Lt=6, H=3, B=1, T=640, k=4),
+    dict(Ls=8, Lt=9, H=2, B=1, T=256, k=4, scores="uniform"),
+])
+def test_tc_small_repeated(over):
+    """Eight launches of one small shape (one work unit per CTA, so every role starts cold):
+    a race between the kernel's roles shows up as a launch that differs from the oracle."""
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", **over)
+    _kernel_or_skip(w, kvx.KVX_KERNEL_TCGEN05)
+    ctx, sel, W, b = make_ctx(w, kernel=kvx.KVX_KERNEL_TCGEN05)
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w)
+        rk, rv, ak, av = oracle_full(w, sk, sv, pos, sel, W, b)
+        for rep in range(8):
+            tk, tv, status = run_contiguous(ctx, w, sk, sv, pos)
+            assert status == kvx.KVX_OK
+            ok, ratio, rms, nbad = check(w, [to_f64(tk), to_f64(tv)], [rk, rv], [ak, av])
+            assert ok, "launch %d: %d elements out of tolerance (worst %.3g x bound)" % (rep, nbad, ratio)
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
 def test_interleaved_pairs_simt():
     w = syn.workload("tiny_fp32", T=100, B=2)
     ctx, sel, W, b = make_ctx(w, rope_style=kvx.KVX_ROPE_INTERLEAVED)
@@ -281,6 +306,9 @@ def test_paged_small_full(kname):
         rows = np.array([(bb, t) for bb in range(w.B) for t in range(w.T)], dtype=np.int64)
         for turn in (0, 1):
             _check_paged(w, ctx, sel, W, b, turn, L0, rows)
+        if kname == "tc":   # repeated launches: a race between roles shows up as a differing launch
+            for rep in range(6):
+                _check_paged(w, ctx, sel, W, b, rep % 2, L0, rows)
     finally:
         kvx.kvx_destroy(ctx)
 
