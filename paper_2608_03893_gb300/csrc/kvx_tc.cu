@@ -22,12 +22,14 @@
 // swizzle), D in one of two 128-column fp32 TMEM accumulators.
 //
 // Warp roles (384 threads):
-//   warp 0      TMA producer of raw source tiles into the shared-memory landing buffer
+//   warp 0      one thread polling two streams without blocking: TMA loads of raw source
+//               tiles into the two landing buffers, and each layer's bias row
 //   warp 1      TMEM allocator (all 512 columns); issuer of the even target layers
 //   warp 3      issuer of the odd target layers.  Each issuer owns one accumulator, one
 //               ring of W stages and one tready/tfree barrier per slot.
-//   warp 2      one thread feeding three streams without blocking: the W ring of each
-//               issuer and the per-layer bias rows (plus L2 prefetch of upcoming W)
+//   warp 2      one thread polling the two W rings without blocking, one per issuer (plus
+//               L2 prefetch of upcoming W).  A poll of shared memory costs hundreds of
+//               cycles under this kernel's traffic, so each poller serves few streams.
 //   warps 4-11  two transform warpgroups (one warp per TMEM lane quarter, warp % 4).
 //               Thread (group g, row r) owns token row r (= TMEM lane r) and the 32 RoPE
 //               pairs 32g .. 32g+31 (channels i and i + 64).
@@ -205,96 +207,41 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
   const MapArgs& A = P.a;
 
   if (warp == 0) {
-    // ------------------------------------------------ source-tile producer --------
+    // ------------------------------------------- source-tile and bias producer ------
+    // One thread polls two streams without blocking: the source tiles of the schedule
+    // into the landing buffers, and every layer's bias row into the bias ring.  There is
+    // no L2 prefetch of upcoming source tiles: under this kernel's streaming traffic a
+    // tile prefetched a few loads ahead was often evicted before its load.
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
-      uint32_t gl = 0;
-      bool ok = true;
-      // No L2 prefetch of upcoming source tiles: under this kernel's streaming traffic a
-      // tile prefetched a few loads ahead was often evicted before its load (about 1 GB of
-      // extra DRAM reads per 8192 tokens), so each tile is read once, by its TMA load.
-      for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-        const Unit un = decode_unit(u, H, A.B, tiles);
-        const CUtensorMap* tm = un.kv ? &P.tm_v : &P.tm_k;
-        for (int e = 0; e < P.n_loads; ++e, ++gl) {
-          const int lb = gl % kLand;
-          const uint32_t round = gl / kLand;
-          const int L = __ldg(&P.load_layer[e]);
-          if (round > 0 && !wait_bar(smem_u32(&land_empty[lb]), (round - 1) & 1u, abort_flag, P.status,
-                                     KVX_ERR_TIMEOUT)) {
-            ok = false;
-            break;
-          }
-          const uint32_t dst = smem_u32(land + static_cast<size_t>(lb) * kLandBytes);
-          mbar_expect_tx(smem_u32(&land_full[lb]), kLandBytes);
-          tma_load_5d(dst, tm, smem_u32(&land_full[lb]), 0, un.t0, un.h, un.b, L, pol);
-          tma_load_5d(dst + kHalfBytes, tm, smem_u32(&land_full[lb]), 64, un.t0, un.h, un.b, L, pol);
-        }
-      }
-      if (!ok) {  // the last min(gl, kLand) landing buffers may still be filling
-        const uint32_t first = gl > static_cast<uint32_t>(kLand) ? gl - kLand : 0;
-        for (uint32_t i = first; i < gl; ++i) drain_wait(smem_u32(&land_full[i % kLand]), (i / kLand) & 1u);
-      }
-    }
-  } else if (warp == 2) {
-    // --------------------------------------------------- W and bias producer ------
-    // One thread feeds three independent streams and polls each one's next free slot
-    // without blocking: the W ring of each issuer (the 2k stages of every layer of its
-    // parity, in order) and the per-layer bias rows (every layer, in order).  Blocking on
-    // one ring would starve the other issuer.
-    if (lane == 0) {
-      const uint64_t pol = policy_evict_last();
-      const int chunks = 2 * k;  // 64-feature chunks of F = 128 k
-      int wu[kIssuers], wl[kIssuers], wc[kIssuers], wkv[kIssuers], wh[kIssuers];
-      uint32_t wn[kIssuers];     // stages filled into ring r
-      for (int r = 0; r < kIssuers; ++r) {
-        wu[r] = blockIdx.x;
-        wl[r] = r;
-        wc[r] = 0;
-        wn[r] = 0;
-        const Unit un = decode_unit(wu[r] < n_units ? wu[r] : 0, H, A.B, tiles);
-        wkv[r] = un.kv;
-        wh[r] = un.h;
-      }
-      int bu = blockIdx.x, blay = 0;
-      uint32_t bn = 0;           // bias rows filled
-      Unit bun = decode_unit(bu < n_units ? bu : 0, H, A.B, tiles);
+      uint32_t gl = 0, bn = 0;
+      int su = blockIdx.x, se = 0, bu = blockIdx.x, blay = 0;
+      Unit sun = decode_unit(su < n_units ? su : 0, H, A.B, tiles);
+      Unit bun = sun;
       bool ok = true;
       uint64_t t_idle = 0;
       uint32_t spins = 0;
       for (;;) {
         bool busy = false, progress = false;
-#pragma unroll
-        for (int r = 0; r < kIssuers; ++r) {
-          if (wl[r] >= Lt || wu[r] >= n_units) continue;   // done (or issuer r has no layer)
+        if (su < n_units && P.n_loads > 0) {
           busy = true;
-          const int st = r * kRing + static_cast<int>(wn[r] % kRing);
-          const uint32_t round = wn[r] / kRing;
-          if (round > 0 && !mbar_test_wait(smem_u32(&wempty[st]), (round - 1) & 1u)) continue;
-          // L2 prefetch of the same chunk of this ring's next layer
-          int nl = wl[r] + kIssuers, nu = wu[r], nkv = wkv[r], nh = wh[r];
-          if (nl >= Lt) {
-            nl = r;
-            nu += gridDim.x;
-            if (nu < n_units) {
-              const Unit nun = decode_unit(nu, H, A.B, tiles);
-              nkv = nun.kv;
-              nh = nun.h;
+          const int lb = static_cast<int>(gl % kLand);
+          const uint32_t round = gl / kLand;
+          if (round == 0 || mbar_test_wait(smem_u32(&land_empty[lb]), (round - 1) & 1u)) {
+            const int L = __ldg(&P.load_layer[se]);
+            const CUtensorMap* tm = sun.kv ? &P.tm_v : &P.tm_k;
+            const uint32_t dst = smem_u32(land + static_cast<size_t>(lb) * kLandBytes);
+            mbar_expect_tx(smem_u32(&land_full[lb]), kLandBytes);
+            tma_load_5d(dst, tm, smem_u32(&land_full[lb]), 0, sun.t0, sun.h, sun.b, L, pol);
+            tma_load_5d(dst + kHalfBytes, tm, smem_u32(&land_full[lb]), 64, sun.t0, sun.h, sun.b, L, pol);
+            ++gl;
+            if (++se == P.n_loads) {
+              se = 0;
+              su += gridDim.x;
+              if (su < n_units) sun = decode_unit(su, H, A.B, tiles);
             }
+            progress = true;
           }
-          if (nu < n_units) tma_prefetch_2d(&P.tm_w, wc[r] * 64, ((nl * 2 + nkv) * H + nh) * kD);
-          mbar_expect_tx(smem_u32(&wfull[st]), kWStageBytes);
-          tma_load_2d(smem_u32(wst + static_cast<size_t>(st) * kWStageBytes), &P.tm_w, smem_u32(&wfull[st]),
-                      wc[r] * 64, ((wl[r] * 2 + wkv[r]) * H + wh[r]) * kD, pol);
-          ++wn[r];
-          if (++wc[r] == chunks) {
-            wc[r] = 0;
-            wl[r] = nl;
-            wu[r] = nu;
-            wkv[r] = nkv;
-            wh[r] = nh;
-          }
-          progress = true;
         }
         if (bu < n_units) {
           busy = true;
@@ -336,13 +283,96 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           }
         }
       }
+      if (!ok) {   // the most recent loads and bias rows may still be landing
+        const uint32_t first = gl > static_cast<uint32_t>(kLand) ? gl - kLand : 0;
+        for (uint32_t i = first; i < gl; ++i) drain_wait(smem_u32(&land_full[i % kLand]), (i / kLand) & 1u);
+        const uint32_t bfirst = bn > static_cast<uint32_t>(kBiasSlots) ? bn - kBiasSlots : 0;
+        for (uint32_t i = bfirst; i < bn; ++i) drain_wait(smem_u32(&bias_full[i % kBiasSlots]), (i / kBiasSlots) & 1u);
+      }
+    }
+  } else if (warp == 2) {
+    // ----------------------------------------------------------- W producer ------
+    // One thread polls the W ring of each issuer (the 2k stages of every layer of its
+    // parity, in order) without blocking: a blocking wait on one ring would starve the
+    // other issuer.
+    if (lane == 0) {
+      const uint64_t pol = policy_evict_last();
+      const int chunks = 2 * k;  // 64-feature chunks of F = 128 k
+      int wu[kIssuers], wl[kIssuers], wc[kIssuers], wkv[kIssuers], wh[kIssuers];
+      uint32_t wn[kIssuers];     // stages filled into ring r
+      for (int r = 0; r < kIssuers; ++r) {
+        wu[r] = blockIdx.x;
+        wl[r] = r;
+        wc[r] = 0;
+        wn[r] = 0;
+        const Unit un = decode_unit(wu[r] < n_units ? wu[r] : 0, H, A.B, tiles);
+        wkv[r] = un.kv;
+        wh[r] = un.h;
+      }
+      bool ok = true;
+      uint64_t t_idle = 0;
+      uint32_t spins = 0;
+      for (;;) {
+        bool busy = false, progress = false;
+#pragma unroll
+        for (int r = 0; r < kIssuers; ++r) {
+          if (wl[r] >= Lt || wu[r] >= n_units) continue;   // done (or issuer r has no layer)
+          busy = true;
+          const int st = r * kRing + static_cast<int>(wn[r] % kRing);
+          const uint32_t round = wn[r] / kRing;
+          if (round > 0 && !mbar_test_wait(smem_u32(&wempty[st]), (round - 1) & 1u)) continue;
+          // L2 prefetch of the same chunk of this ring's next layer
+          int nl = wl[r] + kIssuers, nu = wu[r], nkv = wkv[r], nh = wh[r];
+          if (nl >= Lt) {
+            nl = r;
+            nu += gridDim.x;
+            if (nu < n_units) {
+              const Unit nun = decode_unit(nu, H, A.B, tiles);
+              nkv = nun.kv;
+              nh = nun.h;
+            }
+          }
+          if (nu < n_units) tma_prefetch_2d(&P.tm_w, wc[r] * 64, ((nl * 2 + nkv) * H + nh) * kD);
+          mbar_expect_tx(smem_u32(&wfull[st]), kWStageBytes);
+          tma_load_2d(smem_u32(wst + static_cast<size_t>(st) * kWStageBytes), &P.tm_w, smem_u32(&wfull[st]),
+                      wc[r] * 64, ((wl[r] * 2 + wkv[r]) * H + wh[r]) * kD, pol);
+          ++wn[r];
+          if (++wc[r] == chunks) {
+            wc[r] = 0;
+            wl[r] = nl;
+            wu[r] = nu;
+            wkv[r] = nkv;
+            wh[r] = nh;
+          }
+          progress = true;
+        }
+        if (!busy) break;
+        if (progress) {
+          spins = 0;
+          t_idle = 0;
+          continue;
+        }
+        if ((++spins & 63u) == 0) {   // bounded: no slot freed for 4 s raises KVX_ERR_TIMEOUT
+          if (*abort_flag) {
+            ok = false;
+            break;
+          }
+          const uint64_t now = global_timer();
+          if (t_idle == 0) {
+            t_idle = now;
+          } else if (now - t_idle > kTimeoutNs) {
+            *abort_flag = 1u;
+            report(P.status, KVX_ERR_TIMEOUT);
+            ok = false;
+            break;
+          }
+        }
+      }
       if (!ok) {   // the most recent fills of each ring may still be landing
         for (int r = 0; r < kIssuers; ++r) {
           const uint32_t first = wn[r] > static_cast<uint32_t>(kRing) ? wn[r] - kRing : 0;
           for (uint32_t i = first; i < wn[r]; ++i) drain_wait(smem_u32(&wfull[r * kRing + i % kRing]), (i / kRing) & 1u);
         }
-        const uint32_t bfirst = bn > static_cast<uint32_t>(kBiasSlots) ? bn - kBiasSlots : 0;
-        for (uint32_t i = bfirst; i < bn; ++i) drain_wait(smem_u32(&bias_full[i % kBiasSlots]), (i / kBiasSlots) & 1u);
       }
     }
   } else if (warp == 1 || warp == 3) {
