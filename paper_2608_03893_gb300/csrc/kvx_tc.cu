@@ -18,8 +18,9 @@
 //
 // Contraction of target layer l: D[128 tok x 128 ch] = X[128 x kd] W[kd x 128] on tcgen05
 // (cta_group::1, M = N = 128, K = 16 per instruction: the full-rate shape), A from TMEM,
-// B = W^T from shared-memory stages of 16 KB (128 output channels x 64 features, 128-byte
-// swizzle), D in one of two 128-column fp32 TMEM accumulators.
+// B = W^T from 32 KB shared-memory stages, one per use (128 output channels x 128 features
+// as two 64-feature halves, 128-byte swizzle), D in one of two 128-column fp32 TMEM
+// accumulators.  W needs no L2 prefetch: the CTAs in flight share one (K|V, head) block.
 //
 // Warp roles (384 threads):
 //   warp 0      one thread polling two streams without blocking: TMA loads of raw source
@@ -27,9 +28,9 @@
 //   warp 1      TMEM allocator (all 512 columns); issuer of the even target layers
 //   warp 3      issuer of the odd target layers.  Each issuer owns one accumulator, one
 //               ring of W stages and one tready/tfree barrier per slot.
-//   warp 2      one thread polling the two W rings without blocking, one per issuer (plus
-//               L2 prefetch of upcoming W).  A poll of shared memory costs hundreds of
-//               cycles under this kernel's traffic, so each poller serves few streams.
+//   warp 2      one thread polling the two W rings without blocking, one per issuer.  A
+//               poll of shared memory costs hundreds of cycles under this kernel's
+//               traffic, so each poller serves few streams.
 //   warps 4-11  two transform warpgroups (one warp per TMEM lane quarter, warp % 4).
 //               Thread (group g, row r) owns token row r (= TMEM lane r) and the 32 RoPE
 //               pairs 32g .. 32g+31 (channels i and i + 64).
@@ -69,7 +70,7 @@ constexpr int kTileM = 128;                         // tokens per work unit
 constexpr int kD = 128;                             // head_dim of this kernel
 constexpr uint32_t kLandBytes = kTileM * kD * 2;    // 32 KB raw tile: two 64-column SW128 halves
 constexpr uint32_t kHalfBytes = kLandBytes / 2;     // 16 KB
-constexpr uint32_t kWStageBytes = kD * 64 * 2;      // 16 KB: 128 output channels x 64 features
+constexpr uint32_t kWStageBytes = kD * 128 * 2;     // 32 KB: one use (two 64-feature halves)
 constexpr uint32_t kPieceBytes = 32 * 64;           // 2 KB: 32 rows x 32 channels, 64-byte swizzle
 constexpr uint32_t kWarpStageBytes = 2 * kPieceBytes; // one transform warp's share of an output tile
 constexpr int kTransformWarps = 8;
@@ -86,7 +87,7 @@ constexpr int kBiasSlots = 4;                       // per-layer bias rows stage
 constexpr uint32_t kBiasBytes = kD * 4;
 constexpr size_t kSmemLimit = 232448;               // 227 KB opt-in per CTA
 
-constexpr int kRing = 4;                            // W stages per issuer ring
+constexpr int kRing = 2;                            // W stages (uses) per issuer ring
 constexpr int kNW = kRing * kIssuers;               // W stages in shared memory
 
 // Dynamic shared memory: the 128-byte-swizzled buffers need 1024-byte alignment, which
@@ -98,7 +99,7 @@ constexpr size_t smem_bytes() {
          (2 * kLand + 2 * kTSlots * kIssuers + 2 * kNW + 2 * kAccBufs + 2 * kBiasSlots + kIssuers) * 8 + 16;
 }
 static_assert(smem_bytes() <= kSmemLimit, "shared-memory layout exceeds the per-CTA limit");
-static_assert(kRing >= 2, "each W ring must hold one use (two stages)");
+static_assert(kRing >= 2, "each W ring must hold two uses");
 
 struct TcParams {
   CUtensorMap tm_k;      // source keys   [L_s][B][H][T][128] bf16, box 64 x 128
@@ -297,7 +298,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     // other issuer.
     if (lane == 0) {
       const uint64_t pol = policy_evict_last();
-      const int chunks = 2 * k;  // 64-feature chunks of F = 128 k
+      const int chunks = k;      // uses per layer, one 128-feature stage each
       int wu[kIssuers], wl[kIssuers], wc[kIssuers], wkv[kIssuers], wh[kIssuers];
       uint32_t wn[kIssuers];     // stages filled into ring r
       for (int r = 0; r < kIssuers; ++r) {
@@ -332,10 +333,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
               nh = nun.h;
             }
           }
-          if (nu < n_units) tma_prefetch_2d(&P.tm_w, wc[r] * 64, ((nl * 2 + nkv) * H + nh) * kD);
           mbar_expect_tx(smem_u32(&wfull[st]), kWStageBytes);
-          tma_load_2d(smem_u32(wst + static_cast<size_t>(st) * kWStageBytes), &P.tm_w, smem_u32(&wfull[st]),
-                      wc[r] * 64, ((wl[r] * 2 + wkv[r]) * H + wh[r]) * kD, pol);
+          const uint32_t wdst = smem_u32(wst + static_cast<size_t>(st) * kWStageBytes);
+          const int wrow = ((wl[r] * 2 + wkv[r]) * H + wh[r]) * kD;
+          tma_load_2d(wdst, &P.tm_w, smem_u32(&wfull[st]), wc[r] * 128, wrow, pol);
+          tma_load_2d(wdst + kWStageBytes / 2, &P.tm_w, smem_u32(&wfull[st]), wc[r] * 128 + 64, wrow, pol);
           ++wn[r];
           if (++wc[r] == chunks) {
             wc[r] = 0;
@@ -386,7 +388,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     if (lane == 0) {
       constexpr uint32_t idesc = make_idesc(kTileM, kD);
       const uint32_t d_tmem = tmem_base + iss * kAccCols;
-      uint32_t ready_par = 0, acc_n = 0, wi = 0;   // wi: stages consumed from this issuer's ring
+      uint32_t ready_par = 0, acc_n = 0, wi = 0;   // wi: W stages (uses) consumed from this issuer's ring
       bool ok = true, issued = false;
       uint32_t pack_next = iss < Lt ? __ldg(&P.use_pack[iss]) : 0u;
       for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
@@ -400,7 +402,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
             break;
           }
           tc_fence_after();
-          for (int j = 0; j < k; ++j, wi += 2) {
+          for (int j = 0; j < k; ++j, ++wi) {
             // use bits: slot | 4 first use of the tile by this issuer | 16 release the
             // slot after this use.  The transform warps signal tready[slot][issuer] only
             // for the loads this issuer uses, so it waits for every phase in order.
@@ -415,15 +417,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
               ready_par ^= 1u << s;
               tc_fence_after();   // the tile was written by other threads' tcgen05.st
             }
-            const uint32_t st0 = iss * kRing + wi % kRing, st1 = iss * kRing + (wi + 1) % kRing;
-            if (!wait_bar(smem_u32(&wfull[st0]), (wi / kRing) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT) ||
-                !wait_bar(smem_u32(&wfull[st1]), ((wi + 1) / kRing) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
+            const uint32_t st0 = iss * kRing + wi % kRing;
+            if (!wait_bar(smem_u32(&wfull[st0]), (wi / kRing) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
               ok = false;
               break;
             }
             const uint32_t a_col = tmem_base + kSlotCol0 + s * 64;
             const uint32_t b0 = smem_u32(wst + static_cast<size_t>(st0) * kWStageBytes);
-            const uint32_t b1 = smem_u32(wst + static_cast<size_t>(st1) * kWStageBytes);
+            const uint32_t b1 = b0 + kWStageBytes / 2;
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
               tc_mma_ts(d_tmem, a_col + kk * 8, sw128_desc(b0 + kk * 32), idesc, (j | kk) != 0);
@@ -432,7 +433,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
               tc_mma_ts(d_tmem, a_col + 32 + kk * 8, sw128_desc(b1 + kk * 32), idesc, true);
             issued = true;
             tc_commit(smem_u32(&wempty[st0]));
-            tc_commit(smem_u32(&wempty[st1]));
             if (f & 16u) tc_commit(smem_u32(&tfree[s * kIssuers + iss]));
           }
           if (ok) tc_commit(smem_u32(&accf[iss]));
