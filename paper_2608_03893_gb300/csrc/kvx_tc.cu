@@ -22,7 +22,7 @@
 // as two 64-feature halves, 128-byte swizzle), D in one of two 128-column fp32 TMEM
 // accumulators.  W needs no L2 prefetch: the CTAs in flight share one (K|V, head) block.
 //
-// Warp roles (384 threads):
+// Warp roles (512 threads; per-warpgroup register shares set with setmaxnreg):
 //   warp 0      one thread polling two streams without blocking: TMA loads of raw source
 //               tiles into the two landing buffers, and each layer's bias row
 //   warp 1      TMEM allocator (all 512 columns); issuer of the even target layers
@@ -31,16 +31,18 @@
 //   warp 2      one thread polling the two W rings without blocking, one per issuer.  A
 //               poll of shared memory costs hundreds of cycles under this kernel's
 //               traffic, so each poller serves few streams.
-//   warps 4-11  two transform warpgroups (one warp per TMEM lane quarter, warp % 4).
+//   warps 4-11  epilogue, two warpgroups (one warp per TMEM lane quarter, warp % 4).
 //               Thread (group g, row r) owns token row r (= TMEM lane r) and the 32 RoPE
-//               pairs 32g .. 32g+31 (channels i and i + 64).
-//               Prologue: landing buffer -> registers -> (keys) strip the source RoPE in
-//               fp32, round to bf16 -> tcgen05.st into the tile's TMEM slot.
-//               Epilogue: TMEM -> registers, + bias, (keys) target RoPE, bf16.  For a
-//               contiguous target each warp stages its 32 rows x 2 x 32 channels
-//               (64-byte swizzle) and writes them with its own TMA stores; a warp with a
-//               row at an out-of-range position writes its valid rows directly.  Paged
-//               targets take 16-byte stores through the block table.
+//               pairs 32g .. 32g+31 (channels i and i + 64): TMEM -> registers, + bias,
+//               (keys) target RoPE, bf16.  For a contiguous target each warp stages its
+//               32 rows x 2 x 32 channels (64-byte swizzle) and writes them with its own
+//               TMA stores; a warp with a row at an out-of-range position writes its valid
+//               rows directly.  Paged targets take 16-byte stores through the block table.
+//   warps 12-15 prologue, one warpgroup (one warp per lane quarter); thread r owns token
+//               row r and all 64 pairs: landing buffer -> registers -> (keys) strip the
+//               source RoPE in fp32, round to bf16 -> tcgen05.st into the tile's TMEM slot.
+//               Running the prologue on its own warps takes it off the epilogue's per-layer
+//               chain of waits, loads and stores.
 //
 // Every mbarrier wait is bounded: after 4 s the kernel raises KVX_ERR_TIMEOUT in the
 // status word, sets a shared abort flag that every role polls, waits (again bounded)
@@ -64,18 +66,26 @@ namespace {
 
 using namespace ptx;
 
-constexpr int kThreads = 384;
-constexpr int kFirstTransformWarp = 4;
+constexpr int kThreads = 512;
+constexpr int kFirstEpiWarp = 4;                    // warps 4-11: epilogue
+constexpr int kEpiWarps = 8;
+constexpr int kFirstProWarp = 12;                   // warps 12-15: prologue
+constexpr int kProWarps = 4;
+// Registers per thread of each warpgroup (setmaxnreg): the control warps give up most of
+// theirs so that the epilogue keeps its cos/sin of 32 pairs and the prologue its cos/sin
+// of all 64 pairs in registers.  The shares add up to the launch's 128 x 512.
+constexpr uint32_t kRegsCtl = 32, kRegsEpi = 152, kRegsPro = 176;
+static_assert(kRegsCtl * 128 + kRegsEpi * 256 + kRegsPro * 128 <= 128u * kThreads,
+              "register split exceeds the launch's register file share");
 constexpr int kTileM = 128;                         // tokens per work unit
 constexpr int kD = 128;                             // head_dim of this kernel
 constexpr uint32_t kLandBytes = kTileM * kD * 2;    // 32 KB raw tile: two 64-column SW128 halves
 constexpr uint32_t kHalfBytes = kLandBytes / 2;     // 16 KB
 constexpr uint32_t kWStageBytes = kD * 128 * 2;     // 32 KB: one use (two 64-feature halves)
 constexpr uint32_t kPieceBytes = 32 * 64;           // 2 KB: 32 rows x 32 channels, 64-byte swizzle
-constexpr uint32_t kWarpStageBytes = 2 * kPieceBytes; // one transform warp's share of an output tile
-constexpr int kTransformWarps = 8;
-constexpr int kStageBufs = 1;                       // staging buffers per transform warp
-constexpr uint32_t kOutBytes = kStageBufs * kTransformWarps * kWarpStageBytes;
+constexpr uint32_t kWarpStageBytes = 2 * kPieceBytes; // one epilogue warp's share of an output tile
+constexpr int kStageBufs = 1;                       // staging buffers per epilogue warp
+constexpr uint32_t kOutBytes = kStageBufs * kEpiWarps * kWarpStageBytes;
 constexpr int kTSlots = 4;                          // TMEM source-tile slots (64 columns each)
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccCols = 128;                  // one fp32 accumulator
@@ -110,10 +120,10 @@ struct TcParams {
   MapArgs a;
   const int32_t* load_layer;   // [n_loads] source layer of load e
   const int32_t* load_slot;    // [n_loads] TMEM slot
-  const uint32_t* use_pack;    // [L_t] per use j: 5 bits at 5j = slot | 8 first use | 16 release after
+  const uint32_t* use_pack;    // [L_t] per use j: 5 bits at 5j = slot | 4 first use | 16 release after
   const float* bias;           // [L_t][2][H][128] fp32
   int32_t* status;
-  int32_t Lt, H, k, n_loads, tiles_per_seq, n_units, same_theta;
+  int32_t Lt, H, k, n_loads, tiles_per_seq, n_units;
   RopeTables rope;
 };
 
@@ -153,8 +163,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
   float* bias_ring = reinterpret_cast<float*>(outst + kOutBytes);   // [4][128] fp32
   uint64_t* bars = reinterpret_cast<uint64_t*>(bias_ring + kBiasSlots * kD);
   uint64_t* land_full = bars;                    // [2] TMA landed
-  uint64_t* land_empty = land_full + kLand;      // [2] transform read it (8 warps)
-  uint64_t* tready = land_empty + kLand;         // [4][2] TMEM tile written for issuer i (8 warps)
+  uint64_t* land_empty = land_full + kLand;      // [2] prologue read it (4 warps)
+  uint64_t* tready = land_empty + kLand;         // [4][2] TMEM tile written for issuer i (4 warps)
   uint64_t* tfree = tready + kTSlots * kIssuers; // [4][2] TMEM tile released by issuer i
   uint64_t* wfull = tfree + kTSlots * kIssuers;  // [2][kRing]
   uint64_t* wempty = wfull + kNW;                // [2][kRing]
@@ -172,9 +182,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
   if (threadIdx.x == 0) {
     for (int i = 0; i < kLand; ++i) {
       mbar_init(smem_u32(&land_full[i]), 1);
-      mbar_init(smem_u32(&land_empty[i]), 8);
+      mbar_init(smem_u32(&land_empty[i]), kProWarps);
     }
-    for (int i = 0; i < kTSlots * kIssuers; ++i) mbar_init(smem_u32(&tready[i]), 8);
+    for (int i = 0; i < kTSlots * kIssuers; ++i) mbar_init(smem_u32(&tready[i]), kProWarps);
     for (int i = 0; i < kTSlots * kIssuers; ++i) mbar_init(smem_u32(&tfree[i]), 1);
     for (int i = 0; i < kNW; ++i) {
       mbar_init(smem_u32(&wfull[i]), 1);
@@ -182,11 +192,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     }
     for (int i = 0; i < kAccBufs; ++i) {
       mbar_init(smem_u32(&accf[i]), 1);
-      mbar_init(smem_u32(&acce[i]), 8);
+      mbar_init(smem_u32(&acce[i]), kEpiWarps);
     }
     for (int i = 0; i < kBiasSlots; ++i) {
       mbar_init(smem_u32(&bias_full[i]), 1);
-      mbar_init(smem_u32(&bias_empty[i]), 8);
+      mbar_init(smem_u32(&bias_empty[i]), kEpiWarps);
     }
     for (int i = 0; i < kIssuers; ++i) mbar_init(smem_u32(&drain[i]), 1);
     *abort_flag = 0u;
@@ -206,7 +216,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
   const int Lt = P.Lt, k = P.k, H = P.H;
   const int n_units = P.n_units, tiles = P.tiles_per_seq;
   const MapArgs& A = P.a;
-
+  // Each warpgroup takes its register share (every warp of it executes the same
+  // setmaxnreg) before its warps go their separate ways.
+  if (warp < kFirstEpiWarp) {
+  setmaxnreg_dec<kRegsCtl>();
   if (warp == 0) {
     // ------------------------------------------- source-tile and bias producer ------
     // One thread polls two streams without blocking: the source tiles of the schedule
@@ -322,7 +335,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           const int st = r * kRing + static_cast<int>(wn[r] % kRing);
           const uint32_t round = wn[r] / kRing;
           if (round > 0 && !mbar_test_wait(smem_u32(&wempty[st]), (round - 1) & 1u)) continue;
-          // L2 prefetch of the same chunk of this ring's next layer
+          // the layer (and unit) this ring fills after the current one
           int nl = wl[r] + kIssuers, nu = wu[r], nkv = wkv[r], nh = wh[r];
           if (nl >= Lt) {
             nl = r;
@@ -377,7 +390,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
         }
       }
     }
-  } else if (warp == 1 || warp == 3) {
+  } else {   // warps 1 and 3
     // --------------------------------------------------------- MMA issuers --------
     // Warp 1 issues the even target layers into accumulator 0, warp 3 the odd ones into
     // accumulator 1.  A thread that reads shared memory (an mbarrier wait) while its own
@@ -404,7 +417,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           tc_fence_after();
           for (int j = 0; j < k; ++j, ++wi) {
             // use bits: slot | 4 first use of the tile by this issuer | 16 release the
-            // slot after this use.  The transform warps signal tready[slot][issuer] only
+            // slot after this use.  The prologue warps signal tready[slot][issuer] only
             // for the loads this issuer uses, so it waits for every phase in order.
             const uint32_t f = (pack >> (5 * j)) & 31u;
             const uint32_t s = f & 3u;
@@ -444,15 +457,17 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
         drain_wait(smem_u32(&drain[iss]), 0);
       }
     }
-  } else if (warp >= kFirstTransformWarp) {
-    // ------------------------------------------------------- transform warps ------
-    const int g = (warp - kFirstTransformWarp) >> 2; // pair group: pairs 32g .. 32g+31
+  }
+  } else if (warp < kFirstProWarp) {
+    setmaxnreg_inc<kRegsEpi>();
+    // -------------------------------------------------------- epilogue warps ------
+    const int g = (warp - kFirstEpiWarp) >> 2;       // pair group: pairs 32g .. 32g+31
     const int q = warp & 3;                          // TMEM lane quarter this warp may access
     const int r = q * 32 + lane;                     // token row within the tile
     const uint32_t lane_addr = static_cast<uint32_t>(q * 32) << 16;
     const uint64_t st_pol = policy_evict_first();
-    uint32_t gl = 0, lay = 0, tl_loaded = 0, tfree_par = 0, acc_n0 = 0, acc_n1 = 0;
-    uint8_t* wstage = outst + static_cast<size_t>(warp - kFirstTransformWarp) * kStageBufs * kWarpStageBytes;
+    uint32_t lay = 0, acc_n0 = 0, acc_n1 = 0;
+    uint8_t* wstage = outst + static_cast<size_t>(warp - kFirstEpiWarp) * kStageBufs * kWarpStageBytes;
     float cs[32], sn[32];
     bool ok = true;
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
@@ -501,101 +516,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
       }
       __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(un.kv ? A.tgt_v : A.tgt_k);
       const CUtensorMap* tm_out = un.kv ? &P.tm_out_v : &P.tm_out_k;
-      int e = 0;
-      uint32_t pk_next = __ldg(&P.use_pack[0]);
       for (int l = 0; ok && l < Lt; ++l, ++lay) {
-        // Schedule word of layer l (read one layer ahead): bits 20.. count the loads to
-        // write before its epilogue, those first used by layer l + 1 (and, for layer 0,
-        // by layer 0).
-        const uint32_t pk = pk_next;
-        pk_next = __ldg(&P.use_pack[l + 1 < Lt ? l + 1 : 0]);
-        const int e_end = e + static_cast<int>(pk >> 20);
-        for (; e < e_end; ++e) {   // prologue
-          // load word: slot | 4 << i if issuer i used the slot's previous tile (wait for its
-          // release) | 16 << i if issuer i uses this tile (signal tready[slot][i])
-          const uint32_t lw = static_cast<uint32_t>(__ldg(&P.load_slot[e]));
-          const int lb = gl % kLand;
-          bool w_ok = wait_bar(smem_u32(&land_full[lb]), (gl / kLand) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT);
-          if (!__all_sync(0xffffffffu, w_ok)) {
-            ok = false;
-            break;
-          }
-          uint32_t wa[16], wb[16];   // a: features 32g + [0,32) of the pairs, b: features + 64
-          {
-            const uint8_t* row = land + static_cast<size_t>(lb) * kLandBytes + r * 128;
-#pragma unroll
-            for (int ci = 0; ci < 4; ++ci) {
-              const int phys = ((4 * g + ci) ^ (r & 7)) << 4;
-              const uint4 va = *reinterpret_cast<const uint4*>(row + phys);
-              const uint4 vb = *reinterpret_cast<const uint4*>(row + kHalfBytes + phys);
-              wa[4 * ci] = va.x;
-              wa[4 * ci + 1] = va.y;
-              wa[4 * ci + 2] = va.z;
-              wa[4 * ci + 3] = va.w;
-              wb[4 * ci] = vb.x;
-              wb[4 * ci + 1] = vb.y;
-              wb[4 * ci + 2] = vb.z;
-              wb[4 * ci + 3] = vb.w;
-            }
-          }
-          __syncwarp();
-          if (lane == 0) mbar_arrive(smem_u32(&land_empty[lb]));
-          ++gl;
-          if (un.kv == 0) {
-#pragma unroll
-            for (int w = 0; w < 16; ++w) {
-              const int m0 = 2 * w, m1 = 2 * w + 1;
-              float c0, s0, c1, s1;
-              if (P.same_theta) {
-                c0 = cs[m0];
-                s0 = sn[m0];
-                c1 = cs[m1];
-                s1 = sn[m1];
-              } else {
-                const int i0 = 32 * g + m0, i1 = 32 * g + m1;
-                rope_sincos(p, P.rope.ws_hi[i0], P.rope.ws_lo[i0], P.rope.two_pi_hi, P.rope.two_pi_lo,
-                            P.rope.inv_two_pi, &s0, &c0);
-                rope_sincos(p, P.rope.ws_hi[i1], P.rope.ws_lo[i1], P.rope.two_pi_hi, P.rope.two_pi_lo,
-                            P.rope.inv_two_pi, &s1, &c1);
-              }
-              const float a0 = bf16_lo(wa[w]), a1 = bf16_hi(wa[w]);
-              const float b0 = bf16_lo(wb[w]), b1 = bf16_hi(wb[w]);
-              // rotation by -t*omega: a' = a c + b s, b' = b c - a s
-              wa[w] = pack_bf16x2(__fmaf_rn(a0, c0, __fmul_rn(b0, s0)), __fmaf_rn(a1, c1, __fmul_rn(b1, s1)));
-              wb[w] = pack_bf16x2(__fmaf_rn(b0, c0, -__fmul_rn(a0, s0)), __fmaf_rn(b1, c1, -__fmul_rn(a1, s1)));
-            }
-          }
-          const int s = static_cast<int>(lw & 3u);
-          if ((tl_loaded >> s) & 1u) {
-#pragma unroll
-            for (int i = 0; i < kIssuers; ++i) {
-              if (!((lw >> (2 + i)) & 1u)) continue;
-              const int bi = s * kIssuers + i;
-              w_ok = w_ok && wait_bar(smem_u32(&tfree[bi]), (tfree_par >> bi) & 1u, abort_flag, P.status,
-                                      KVX_ERR_TIMEOUT);
-              tfree_par ^= 1u << bi;
-            }
-            if (!__all_sync(0xffffffffu, w_ok)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-          }
-          tl_loaded |= 1u << s;
-          const uint32_t scol = tmem_base + lane_addr + kSlotCol0 + s * 64;
-          tmem_st_x16(scol + 16 * g, wa);        // features 32g .. 32g+31
-          tmem_st_x16(scol + 32 + 16 * g, wb);   // features 64 + 32g .. 64 + 32g+31
-          tmem_wait_st();
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) {
-#pragma unroll
-            for (int i = 0; i < kIssuers; ++i)
-              if ((lw >> (4 + i)) & 1u) mbar_arrive(smem_u32(&tready[s * kIssuers + i]));
-          }
-        }
-        if (!ok) break;
-        // epilogue of layer l
         const uint32_t bslot = lay % kBiasSlots;
         const float* bias = bias_ring + bslot * kD;
         {
@@ -707,6 +628,103 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
       }
     }
     if (!A.paged && lane == 0) bulk_wait_all();   // this warp's stores are complete
+  } else {
+    setmaxnreg_inc<kRegsPro>();
+    // -------------------------------------------------------- prologue warps ------
+    // Thread (quarter q, lane) owns token row r = 32q + lane (TMEM lane r) and all 64 RoPE
+    // pairs.  For every load of the schedule, in order: landing buffer -> registers ->
+    // (keys) strip the source RoPE in fp32, round to bf16 -> tcgen05.st into the tile's
+    // TMEM slot.  These warps run ahead of the epilogue, limited only by the landing
+    // buffers and by the release of each slot's previous tile.
+    const int q = warp & 3;
+    const int r = q * 32 + lane;
+    const uint32_t lane_addr = static_cast<uint32_t>(q * 32) << 16;
+    uint32_t gl = 0, tl_loaded = 0, tfree_par = 0;
+    float cs[64], sn[64];   // cos / sin of the source angle of pair i of row r
+    bool ok = true;
+    for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+      const Unit un = decode_unit(u, H, A.B, tiles);
+      if (un.kv == 0) {
+        // a row past the sequence end or at an out-of-range position (which the epilogue
+        // reports) is rotated by angle 0: its output is never written
+        const int t = un.t0 + r;
+        int p = t < A.T ? __ldg(&A.pos[static_cast<int64_t>(un.b) * A.T + t]) : 0;
+        if (p < 0 || p >= (1 << 24)) p = 0;
+#pragma unroll
+        for (int i = 0; i < 64; ++i)
+          rope_sincos(p, P.rope.ws_hi[i], P.rope.ws_lo[i], P.rope.two_pi_hi, P.rope.two_pi_lo, P.rope.inv_two_pi,
+                      &sn[i], &cs[i]);
+      }
+      for (int e = 0; ok && e < P.n_loads; ++e) {
+        // load word: slot | 4 << i if issuer i used the slot's previous tile (wait for its
+        // release) | 16 << i if issuer i uses this tile (signal tready[slot][i])
+        const uint32_t lw = static_cast<uint32_t>(__ldg(&P.load_slot[e]));
+        const int s = static_cast<int>(lw & 3u);
+        const int lb = gl % kLand;
+        bool w_ok = wait_bar(smem_u32(&land_full[lb]), (gl / kLand) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT);
+        if ((tl_loaded >> s) & 1u) {
+#pragma unroll
+          for (int i = 0; i < kIssuers; ++i) {
+            if (!((lw >> (2 + i)) & 1u)) continue;
+            const int bi = s * kIssuers + i;
+            w_ok = w_ok && wait_bar(smem_u32(&tfree[bi]), (tfree_par >> bi) & 1u, abort_flag, P.status,
+                                    KVX_ERR_TIMEOUT);
+            tfree_par ^= 1u << bi;
+          }
+        }
+        if (!__all_sync(0xffffffffu, w_ok)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        tl_loaded |= 1u << s;
+        const uint8_t* row = land + static_cast<size_t>(lb) * kLandBytes + r * 128;
+        const uint32_t scol = tmem_base + lane_addr + kSlotCol0 + s * 64;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {   // features 16c .. 16c+15 (a) and 64 + 16c .. 64 + 16c+15 (b)
+          uint32_t wa[8], wb[8];
+#pragma unroll
+          for (int ci = 0; ci < 2; ++ci) {
+            const int phys = ((2 * c + ci) ^ (r & 7)) << 4;
+            const uint4 va = *reinterpret_cast<const uint4*>(row + phys);
+            const uint4 vb = *reinterpret_cast<const uint4*>(row + kHalfBytes + phys);
+            wa[4 * ci] = va.x;
+            wa[4 * ci + 1] = va.y;
+            wa[4 * ci + 2] = va.z;
+            wa[4 * ci + 3] = va.w;
+            wb[4 * ci] = vb.x;
+            wb[4 * ci + 1] = vb.y;
+            wb[4 * ci + 2] = vb.z;
+            wb[4 * ci + 3] = vb.w;
+          }
+          if (un.kv == 0) {
+#pragma unroll
+            for (int w = 0; w < 8; ++w) {   // pairs 16c + 2w and 16c + 2w + 1
+              const int m0 = 16 * c + 2 * w, m1 = m0 + 1;
+              const float a0 = bf16_lo(wa[w]), a1 = bf16_hi(wa[w]);
+              const float b0 = bf16_lo(wb[w]), b1 = bf16_hi(wb[w]);
+              // rotation by -t*omega: a' = a c + b s, b' = b c - a s
+              wa[w] = pack_bf16x2(__fmaf_rn(a0, cs[m0], __fmul_rn(b0, sn[m0])),
+                                  __fmaf_rn(a1, cs[m1], __fmul_rn(b1, sn[m1])));
+              wb[w] = pack_bf16x2(__fmaf_rn(b0, cs[m0], -__fmul_rn(a0, sn[m0])),
+                                  __fmaf_rn(b1, cs[m1], -__fmul_rn(a1, sn[m1])));
+            }
+          }
+          tmem_st_x8(scol + 8 * c, wa);        // TMEM columns 8c .. 8c+7
+          tmem_st_x8(scol + 32 + 8 * c, wb);   // TMEM columns 32 + 8c .. 32 + 8c+7
+        }
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(smem_u32(&land_empty[lb]));
+#pragma unroll
+          for (int i = 0; i < kIssuers; ++i)
+            if ((lw >> (4 + i)) & 1u) mbar_arrive(smem_u32(&tready[s * kIssuers + i]));
+        }
+        ++gl;
+      }
+    }
   }
 
   tc_fence_before();
@@ -738,14 +756,14 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
 // kTSlots TMEM slots: the victim is the resident tile whose next use is farthest away;
 // among equals, the one whose last use is earliest.  Use (l, j) is issued by issuer l % 2.
 // Before a tile is overwritten, every issuer that read it releases the slot (a commit
-// after its last use of the tile) and the transform warps wait for exactly those
+// after its last use of the tile) and the prologue warps wait for exactly those
 // releases.  The final tiles of a unit are released for the first loads of the next one.
 // All waits follow the (l, j) order, and with k <= kTSlots a victim always exists, so
 // every wait ends.
 //   use_flags:  1 first use of the tile by its issuer (wait for tready[slot][issuer]),
 //               4 release the slot after the use
 //   load_slot:  slot | 4 << i if issuer i must release the slot's previous tile first
-//               | 16 << i if issuer i uses the tile (the transform signals its tready)
+//               | 16 << i if issuer i uses the tile (the prologue signals its tready)
 void build_plan(const kvx_ctx* c, TcPlan* plan) {
   const int Lt = c->Lt, k = c->k, n_uses = Lt * k, S = kTSlots;
   std::vector<int> src(n_uses), next_use(n_uses);
@@ -867,10 +885,6 @@ kvx_status tc_prepare(kvx_ctx* c, const void* W_host) {
                          ((p.use_flags[u] & 4) ? 16u : 0u);
       pack[l] |= static_cast<int32_t>(f << (5 * j));
     }
-  // bits 20..: loads the transform warps write before the epilogue of layer l
-  std::vector<int32_t> before(c->Lt, 0);
-  for (int e = 0; e < p.n_loads; ++e) ++before[std::max(p.load_first_use[e] - 1, 0)];
-  for (int l = 0; l < c->Lt; ++l) pack[l] |= before[l] << 20;
   std::vector<int32_t> tab;
   tab.insert(tab.end(), p.load_layer.begin(), p.load_layer.end());
   tab.insert(tab.end(), p.load_slot.begin(), p.load_slot.end());
@@ -959,7 +973,6 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
     return KVX_ERR_UNSUPPORTED;
   }
   P.n_units = static_cast<int>(units);
-  P.same_theta = c->theta_s == c->theta_t;
   P.rope = c->rope;
   const size_t smem = smem_bytes();
   cudaError_t e = cudaFuncSetAttribute(tc_map_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -967,6 +980,19 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   if (e != cudaSuccess) {
     set_error(std::string("kvx_map: smem attribute: ") + cudaGetErrorString(e));
     return KVX_ERR_CUDA;
+  }
+  // The warpgroups' register shares (setmaxnreg) are drawn from what the launch holds: a
+  // build that launched with fewer registers per thread would leave an increase waiting.
+  cudaFuncAttributes fa;
+  e = cudaFuncGetAttributes(&fa, tc_map_kernel);
+  if (e != cudaSuccess) {
+    set_error(std::string("kvx_map: kernel attributes: ") + cudaGetErrorString(e));
+    return KVX_ERR_CUDA;
+  }
+  if (static_cast<uint32_t>(fa.numRegs) * kThreads < kRegsCtl * 128 + kRegsEpi * 256 + kRegsPro * 128) {
+    set_error("kvx_map: tensor-core kernel built with " + std::to_string(fa.numRegs) +
+              " registers per thread, too few for its warpgroup register split");
+    return KVX_ERR_UNSUPPORTED;
   }
   const int grid = static_cast<int>(std::min<int64_t>(units, c->sm_count));
   tc_map_kernel<<<grid, kThreads, smem, stream>>>(P);
