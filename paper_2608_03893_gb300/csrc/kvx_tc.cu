@@ -573,12 +573,20 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
             yhi[j + 3] = __fadd_rn(__uint_as_float(hi[j + 3]), b1.w);
           }
           if (un.kv == 0) {
+            // target RoPE, two pairs per f32x2 instruction (each lane rounds like the
+            // scalar fmul / fma it replaces): y0' = y0 c - y1 s, y1' = y0 s + y1 c
 #pragma unroll
-            for (int j = 0; j < 16; ++j) {
-              const float c = cs[16 * rnd + j], sv = sn[16 * rnd + j];
-              const float y0 = ylo[j], y1 = yhi[j];
-              ylo[j] = __fmaf_rn(y0, c, -__fmul_rn(y1, sv));
-              yhi[j] = __fmaf_rn(y0, sv, __fmul_rn(y1, c));
+            for (int j = 0; j < 16; j += 2) {
+              const float2 c = make_float2(cs[16 * rnd + j], cs[16 * rnd + j + 1]);
+              const float2 sv = make_float2(sn[16 * rnd + j], sn[16 * rnd + j + 1]);
+              const float2 y0 = make_float2(ylo[j], ylo[j + 1]), y1 = make_float2(yhi[j], yhi[j + 1]);
+              const float2 u = __fmul2_rn(y1, sv);
+              const float2 r0 = __ffma2_rn(y0, c, make_float2(-u.x, -u.y));
+              const float2 r1 = __ffma2_rn(y0, sv, __fmul2_rn(y1, c));
+              ylo[j] = r0.x;
+              ylo[j + 1] = r0.y;
+              yhi[j] = r1.x;
+              yhi[j + 1] = r1.y;
             }
           }
           uint4 v[4];
