@@ -115,8 +115,8 @@ struct TcParams {
   CUtensorMap tm_k;      // source keys   [L_s][B][H][T][128] bf16, box 64 x 128
   CUtensorMap tm_v;      // source values
   CUtensorMap tm_w;      // W^T [L_t*2*H*128][F] bf16, box 64 x 128
-  CUtensorMap tm_out_k;  // target keys   [L_t][B][H][T][128] bf16, box 64 x 128 (contiguous only)
-  CUtensorMap tm_out_v;  // target values
+  CUtensorMap tm_out_k;  // target keys as (64 ch, T, 2 halves, B*H or H, L_t), box 32 x 32 x 2 x 1 x 1
+  CUtensorMap tm_out_v;  // target values (contiguous targets whose (batch, head) dims merge)
   MapArgs a;
   const int32_t* load_layer;   // [n_loads] source layer of load e
   const int32_t* load_slot;    // [n_loads] TMEM slot
@@ -124,6 +124,7 @@ struct TcParams {
   const float* bias;           // [L_t][2][H][128] fp32
   int32_t* status;
   int32_t Lt, H, k, n_loads, tiles_per_seq, n_units;
+  int32_t out_bh;        // TMA-store head coordinate: 0 none (direct stores), 1 h (B = 1), 2 b*H + h
   RopeTables rope;
 };
 
@@ -505,7 +506,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
       // contiguous targets: each warp stages its 32 rows and writes them with TMA stores,
       // unless one of its rows has an out-of-range position: then its valid rows are
       // written directly (rows past the sequence end are clipped by the tensor map)
-      const bool warp_tma = !A.paged && __ballot_sync(0xffffffffu, bad) == 0u;
+      const bool warp_tma = P.out_bh != 0 && __ballot_sync(0xffffffffu, bad) == 0u;
       if (un.kv == 0) {
 #pragma unroll
         for (int m = 0; m < 32; ++m) {
@@ -626,9 +627,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           }
           if (lane == 0) {
             if (warp_tma && un.t0 + 32 * q < A.T) {   // skip a box wholly past the sequence end
-              const uint32_t src = smem_u32(sb);
-              tma_store_5d(tm_out, src, 32 * g, un.t0 + 32 * q, un.h, un.b, l);
-              tma_store_5d(tm_out, src + kPieceBytes, 64 + 32 * g, un.t0 + 32 * q, un.h, un.b, l);
+              // one box: both 32-row x 32-channel pieces (channels 32g.. and 64 + 32g..)
+              const int bh = P.out_bh == 2 ? un.b * H + un.h : un.h;
+              tma_store_5d(tm_out, smem_u32(sb), 32 * g, un.t0 + 32 * q, 0, bh, l);
             }
             bulk_commit_group();
           }
@@ -935,13 +936,20 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
       return KVX_ERR_UNSUPPORTED;
     }
   }
-  if (!a.paged) {  // target maps for the per-warp TMA stores: dims (d, T, H, B, L_t), box 32 x 32
-    const cuuint32_t tbox[5] = {32, 32, 1, 1, 1};
-    const cuuint64_t tdims[5] = {static_cast<cuuint64_t>(kD), static_cast<cuuint64_t>(a.T),
-                                 static_cast<cuuint64_t>(c->H), static_cast<cuuint64_t>(a.B),
+  // Target maps for the per-warp TMA stores: dims (64 channels, T, 2 halves, heads, L_t),
+  // so that one box (32 channels x 32 rows x both halves, 4 KB) holds a warp's share of a
+  // layer.  The inner box extent equals the 64-byte swizzle span.  The batch folds into
+  // the head dim when B = 1 or the batch stride is H head strides; other contiguous layouts
+  // take direct stores.
+  P.out_bh = 0;
+  if (!a.paged && (a.B == 1 || a.ts[1] == static_cast<int64_t>(c->H) * a.ts[2])) {
+    P.out_bh = a.B == 1 ? 1 : 2;
+    const cuuint32_t tbox[5] = {32, 32, 2, 1, 1};
+    const cuuint64_t tdims[5] = {64, static_cast<cuuint64_t>(a.T), 2,
+                                 static_cast<cuuint64_t>(c->H) * static_cast<cuuint64_t>(a.B),
                                  static_cast<cuuint64_t>(c->Lt)};
-    const cuuint64_t tstr[4] = {static_cast<cuuint64_t>(a.ts[3]) * 2, static_cast<cuuint64_t>(a.ts[2]) * 2,
-                                static_cast<cuuint64_t>(a.ts[1]) * 2, static_cast<cuuint64_t>(a.ts[0]) * 2};
+    const cuuint64_t tstr[4] = {static_cast<cuuint64_t>(a.ts[3]) * 2, 64 * 2, static_cast<cuuint64_t>(a.ts[2]) * 2,
+                                static_cast<cuuint64_t>(a.ts[0]) * 2};
     for (int kv = 0; kv < 2; ++kv) {
       CUresult r = encode(kv ? &P.tm_out_v : &P.tm_out_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5,
                           kv ? a.tgt_v : a.tgt_k, tdims, tstr, tbox, ones, CU_TENSOR_MAP_INTERLEAVE_NONE,

@@ -368,3 +368,31 @@ def test_incremental_turns_equal_one_shot():
         assert torch.equal(tk, full_k) and torch.equal(tv, full_v)
     finally:
         kvx.kvx_destroy(ctx)
+
+
+@pytest.mark.parametrize("kname", ["simt", "tc"])
+def test_target_layouts_bit_identical(kname):
+    """Target caches in other strided layouts ([L][H][B][T][d] and [L][B][T][H][d] viewed as
+    (L, B, H, T, d)) get the same bits as the contiguous one: the tensor-core kernel writes
+    those through its direct-store path, the contiguous one through per-warp TMA stores."""
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=6, Lt=5, H=2, B=2, T=300, k=3)
+    _kernel_or_skip(w, KERNELS[kname])
+    ctx, sel, W, b = make_ctx(w, kernel=KERNELS[kname])
+    dev = torch.device("cuda:0")
+    try:
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w)
+        ref_k, ref_v, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        shapes = {"lhbtd": (w.Lt, w.H, w.B, w.T, w.d), "lbthd": (w.Lt, w.B, w.T, w.H, w.d)}
+        perms = {"lhbtd": (0, 2, 1, 3, 4), "lbthd": (0, 1, 3, 2, 4)}
+        for name, shape in shapes.items():
+            bk = torch.full(shape, float("nan"), dtype=sk.dtype, device=dev)
+            bv = torch.full_like(bk, float("nan"))
+            tk, tv = bk.permute(*perms[name]), bv.permute(*perms[name])
+            assert tk.shape == ref_k.shape
+            _, _, st = run_contiguous(ctx, w, sk, sv, pos, tgt=(tk, tv))
+            assert st == kvx.KVX_OK
+            assert torch.equal(tk, ref_k) and torch.equal(tv, ref_v), name
+    finally:
+        kvx.kvx_destroy(ctx)
