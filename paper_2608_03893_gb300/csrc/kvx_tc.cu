@@ -710,13 +710,16 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
 #pragma unroll
             for (int w = 0; w < 8; ++w) {   // pairs 16c + 2w and 16c + 2w + 1
               const int m0 = 16 * c + 2 * w, m1 = m0 + 1;
-              const float a0 = bf16_lo(wa[w]), a1 = bf16_hi(wa[w]);
-              const float b0 = bf16_lo(wb[w]), b1 = bf16_hi(wb[w]);
-              // rotation by -t*omega: a' = a c + b s, b' = b c - a s
-              wa[w] = pack_bf16x2(__fmaf_rn(a0, cs[m0], __fmul_rn(b0, sn[m0])),
-                                  __fmaf_rn(a1, cs[m1], __fmul_rn(b1, sn[m1])));
-              wb[w] = pack_bf16x2(__fmaf_rn(b0, cs[m0], -__fmul_rn(a0, sn[m0])),
-                                  __fmaf_rn(b1, cs[m1], -__fmul_rn(a1, sn[m1])));
+              const float2 a = make_float2(bf16_lo(wa[w]), bf16_hi(wa[w]));
+              const float2 b = make_float2(bf16_lo(wb[w]), bf16_hi(wb[w]));
+              const float2 cc = make_float2(cs[m0], cs[m1]), ss = make_float2(sn[m0], sn[m1]);
+              // rotation by -t*omega: a' = a c + b s, b' = b c - a s, two pairs per f32x2
+              // instruction (each lane rounds like the scalar fmul / fma)
+              const float2 as = __fmul2_rn(a, ss);
+              const float2 ra = __ffma2_rn(a, cc, __fmul2_rn(b, ss));
+              const float2 rb = __ffma2_rn(b, cc, make_float2(-as.x, -as.y));
+              wa[w] = pack_bf16x2(ra.x, ra.y);
+              wb[w] = pack_bf16x2(rb.x, rb.y);
             }
           }
           tmem_st_x8(scol + 8 * c, wa);        // TMEM columns 8c .. 8c+7
