@@ -6,28 +6,39 @@
 //   V_t^{l,h} =          [V_s^{sel[l][j]}[h]]_j W_V^{l,h} + b_V^{l,h},
 // with the stripped keys rounded to bf16 before the contraction and fp32 accumulation.
 //
-// Work unit = (sequence b, 128-token tile, head h, K|V).  A persistent CTA walks every
-// target layer of a unit.  The k source tiles a target layer concatenates are the A
-// operand of the contraction and live in tensor memory: four 64-column TMEM slots, each
-// holding a 128-token x 128-feature bf16 tile (lane = token, two features per column).
-// A host-built schedule (Belady over the sequence of (layer, j) uses) keeps every source
-// tile resident while later target layers still select it, so each source layer is
-// read from HBM once per token tile and shared by all target layers that select it.  A
-// slot is released as soon as the MMAs of its tile's last use complete, so the tile a
-// layer adds is written while the rest of the previous layer still computes.
+// The kernel runs as clusters of two CTAs (one per SM).  Work unit = (sequence b, pair of
+// adjacent 128-token tiles, head h, K|V); CTA rank r of the cluster takes tile 2p + r.  A
+// persistent cluster walks every target layer of a unit.  The k source tiles a target
+// layer concatenates are the A operand of the contraction and live in tensor memory: four
+// 64-column TMEM slots per CTA, each holding a 128-token x 128-feature bf16 tile (lane =
+// token, two features per column).  A host-built schedule (Belady over the sequence of
+// (layer, j) uses) keeps every source tile resident while later target layers still
+// select it, so each source layer is read from HBM once per token tile and shared by all
+// target layers that select it.  A slot is released as soon as the MMAs of its tile's
+// last use complete, so the tile a layer adds is written while the rest of the previous
+// layer still computes.
 //
-// Contraction of target layer l: D[128 tok x 128 ch] = X[128 x kd] W[kd x 128] on tcgen05
-// (cta_group::1, M = N = 128, K = 16 per instruction: the full-rate shape), A from TMEM,
-// B = W^T from 32 KB shared-memory stages, one per use (128 output channels x 128 features
-// as two 64-feature halves, 128-byte swizzle), D in one of two 128-column fp32 TMEM
-// accumulators.  W needs no L2 prefetch: the CTAs in flight share one (K|V, head) block.
+// Contraction of target layer l for both CTAs' tiles: D[256 tok x 128 ch] =
+// X[256 x kd] W[kd x 128] as tcgen05 pair MMAs (cta_group::2, M = 256, N = 128, K = 16 per
+// instruction), issued by the rank-0 CTA.  Each CTA supplies its 128 rows of A from its own
+// TMEM and 64 of the 128 output channels of B = W^T from its own 16 KB shared-memory stage
+// (64 rows x 128 features as two 64-feature halves, 128-byte swizzle); D lands in each
+// CTA's own two 128-column fp32 TMEM accumulators.  Sharing B halves each SM's W traffic
+// from L2 and the shared memory it needs per use, so each issuer's ring holds four uses.
+// W needs no L2 prefetch: the clusters in flight share one (K|V, head) block.
+//
+// Cross-CTA hand-offs: both CTAs' W loads complete on the rank-0 CTA's stage barrier;
+// both CTAs' prologue and epilogue warps arrive on the rank-0 CTA's tready / acce
+// barriers; the rank-0 issuers' commits arrive on the wempty / tfree / accf barriers of
+// both CTAs (multicast).
 //
 // Warp roles (512 threads; per-warpgroup register shares set with setmaxnreg):
 //   warp 0      one thread polling two streams without blocking: TMA loads of raw source
 //               tiles into the two landing buffers, and each layer's bias row
-//   warp 1      TMEM allocator (all 512 columns); issuer of the even target layers
-//   warp 3      issuer of the odd target layers.  Each issuer owns one accumulator, one
-//               ring of W stages and one tready/tfree barrier per slot.
+//   warp 1      TMEM allocator (all 512 columns, jointly with the peer CTA); in the rank-0
+//               CTA, issuer of the even target layers
+//   warp 3      in the rank-0 CTA, issuer of the odd target layers.  Each issuer owns one
+//               accumulator, one ring of W stages and one tready/tfree barrier per slot.
 //   warp 2      one thread polling the two W rings without blocking, one per issuer.  A
 //               poll of shared memory costs hundreds of cycles under this kernel's
 //               traffic, so each poller serves few streams.
@@ -74,14 +85,15 @@ constexpr int kProWarps = 4;
 // Registers per thread of each warpgroup (setmaxnreg): the control warps give up most of
 // theirs so that the epilogue keeps its cos/sin of 32 pairs and the prologue its cos/sin
 // of all 64 pairs in registers.  The shares add up to the launch's 128 x 512.
-constexpr uint32_t kRegsCtl = 32, kRegsEpi = 152, kRegsPro = 176;
+constexpr uint32_t kRegsCtl = 48, kRegsEpi = 144, kRegsPro = 176;
 static_assert(kRegsCtl * 128 + kRegsEpi * 256 + kRegsPro * 128 <= 128u * kThreads,
               "register split exceeds the launch's register file share");
 constexpr int kTileM = 128;                         // tokens per work unit
 constexpr int kD = 128;                             // head_dim of this kernel
 constexpr uint32_t kLandBytes = kTileM * kD * 2;    // 32 KB raw tile: two 64-column SW128 halves
 constexpr uint32_t kHalfBytes = kLandBytes / 2;     // 16 KB
-constexpr uint32_t kWStageBytes = kD * 128 * 2;     // 32 KB: one use (two 64-feature halves)
+constexpr uint32_t kWStageBytes = (kD / 2) * 128 * 2; // 16 KB: this CTA's 64 output rows of one use
+                                                      // (two 64-feature halves)
 constexpr uint32_t kPieceBytes = 32 * 64;           // 2 KB: 32 rows x 32 channels, 64-byte swizzle
 constexpr uint32_t kWarpStageBytes = 2 * kPieceBytes; // one epilogue warp's share of an output tile
 constexpr int kStageBufs = 1;                       // staging buffers per epilogue warp
@@ -97,7 +109,7 @@ constexpr int kBiasSlots = 4;                       // per-layer bias rows stage
 constexpr uint32_t kBiasBytes = kD * 4;
 constexpr size_t kSmemLimit = 232448;               // 227 KB opt-in per CTA
 
-constexpr int kRing = 2;                            // W stages (uses) per issuer ring
+constexpr int kRing = 4;                            // W stages (uses) per issuer ring
 constexpr int kNW = kRing * kIssuers;               // W stages in shared memory
 
 // Dynamic shared memory: the 128-byte-swizzled buffers need 1024-byte alignment, which
@@ -123,7 +135,7 @@ struct TcParams {
   const uint32_t* use_pack;    // [L_t] per use j: 5 bits at 5j = slot | 4 first use | 16 release after
   const float* bias;           // [L_t][2][H][128] fp32
   int32_t* status;
-  int32_t Lt, H, k, n_loads, tiles_per_seq, n_units;
+  int32_t Lt, H, k, n_loads, tiles_per_seq, n_units;   // tiles_per_seq / n_units count pairs of token tiles
   int32_t out_bh;        // TMA-store head coordinate: 0 none (direct stores), 1 h (B = 1), 2 b*H + h
   RopeTables rope;
 };
@@ -132,15 +144,16 @@ struct Unit {
   int b, t0, h, kv;
 };
 
-// Units are visited u = blockIdx.x + i * gridDim.x, token tile fastest, then sequence,
-// head, and K|V outermost.  The CTAs running at any moment then work on one or two
-// (K|V, head) pairs, so the W^T rows they stream (8 MB per pair at L_t = 64, k = 4) stay
-// in L2 even when the CTAs drift to different target layers; every CTA still gets
-// nearly equal numbers of (heavier) key and value units.
-__device__ __forceinline__ Unit decode_unit(int u, int H, int B, int tiles) {
+// Units (tile pairs) are visited u = cluster + i * clusters, tile pair fastest, then
+// sequence, head, and K|V outermost.  The clusters running at any moment then work on one
+// or two (K|V, head) pairs, so the W^T rows they stream (8 MB per pair at L_t = 64, k = 4)
+// stay in L2 even when the clusters drift to different target layers; every cluster still
+// gets nearly equal numbers of (heavier) key and value units.  Rank 1's tile of the last
+// pair lies past the sequence end when the tile count is odd: its rows are all masked.
+__device__ __forceinline__ Unit decode_unit(int u, int H, int B, int pairs, uint32_t rank) {
   Unit r;
-  r.t0 = (u % tiles) * kTileM;
-  int rest = u / tiles;
+  r.t0 = (2 * (u % pairs) + static_cast<int>(rank)) * kTileM;   // past the end for an odd tile count
+  int rest = u / pairs;
   r.b = rest % B;
   rest /= B;
   r.h = rest % H;
@@ -152,7 +165,8 @@ __device__ __forceinline__ void report(int32_t* status, int code) { atomicCAS(st
 
 // ------------------------------------------------------------------------ kernel --
 
-__global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_constant__ TcParams P) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    tc_map_kernel(const __grid_constant__ TcParams P) {
   extern __shared__ __align__(1024) uint8_t smem[];
   if (smem_u32(smem) & 1023u) {   // uniform over the CTA: every thread returns here
     if (threadIdx.x == 0) report(P.status, KVX_ERR_UNSUPPORTED);
@@ -165,12 +179,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
   uint64_t* bars = reinterpret_cast<uint64_t*>(bias_ring + kBiasSlots * kD);
   uint64_t* land_full = bars;                    // [2] TMA landed
   uint64_t* land_empty = land_full + kLand;      // [2] prologue read it (4 warps)
-  uint64_t* tready = land_empty + kLand;         // [4][2] TMEM tile written for issuer i (4 warps)
+  uint64_t* tready = land_empty + kLand;         // [4][2] TMEM tile written for issuer i (4 warps x 2 CTAs)
   uint64_t* tfree = tready + kTSlots * kIssuers; // [4][2] TMEM tile released by issuer i
   uint64_t* wfull = tfree + kTSlots * kIssuers;  // [2][kRing]
   uint64_t* wempty = wfull + kNW;                // [2][kRing]
   uint64_t* accf = wempty + kNW;                 // [2] accumulator ready
-  uint64_t* acce = accf + kAccBufs;              // [2] accumulator drained (8 warps)
+  uint64_t* acce = accf + kAccBufs;              // [2] accumulator drained (8 warps x 2 CTAs)
   uint64_t* bias_full = acce + kAccBufs;         // [4] bias row landed
   uint64_t* bias_empty = bias_full + kBiasSlots; // [4] bias row used (8 warps)
   uint64_t* drain = bias_empty + kBiasSlots;     // [2] per issuer
@@ -179,13 +193,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();        // 0: issues the pair's MMAs
+  const int unit0 = blockIdx.x >> 1, unit_step = gridDim.x >> 1;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < kLand; ++i) {
       mbar_init(smem_u32(&land_full[i]), 1);
       mbar_init(smem_u32(&land_empty[i]), kProWarps);
     }
-    for (int i = 0; i < kTSlots * kIssuers; ++i) mbar_init(smem_u32(&tready[i]), kProWarps);
+    for (int i = 0; i < kTSlots * kIssuers; ++i) mbar_init(smem_u32(&tready[i]), 2 * kProWarps);
     for (int i = 0; i < kTSlots * kIssuers; ++i) mbar_init(smem_u32(&tfree[i]), 1);
     for (int i = 0; i < kNW; ++i) {
       mbar_init(smem_u32(&wfull[i]), 1);
@@ -193,7 +209,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     }
     for (int i = 0; i < kAccBufs; ++i) {
       mbar_init(smem_u32(&accf[i]), 1);
-      mbar_init(smem_u32(&acce[i]), kEpiWarps);
+      mbar_init(smem_u32(&acce[i]), 2 * kEpiWarps);
     }
     for (int i = 0; i < kBiasSlots; ++i) {
       mbar_init(smem_u32(&bias_full[i]), 1);
@@ -205,13 +221,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     fence_proxy_async_smem();
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_holder)),
+    // one warp of each CTA of the pair allocates, collectively, the same columns in both
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_holder)),
                  "r"(kTmemCols)
                  : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
   }
   tc_fence_before();
   __syncthreads();
+  cluster_sync();   // the peer's barriers are initialised before any arrival from this CTA
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
   const int Lt = P.Lt, k = P.k, H = P.H;
@@ -230,8 +248,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
       uint32_t gl = 0, bn = 0;
-      int su = blockIdx.x, se = 0, bu = blockIdx.x, blay = 0;
-      Unit sun = decode_unit(su < n_units ? su : 0, H, A.B, tiles);
+      int su = unit0, se = 0, bu = unit0, blay = 0;
+      Unit sun = decode_unit(su < n_units ? su : 0, H, A.B, tiles, rank);
       Unit bun = sun;
       bool ok = true;
       uint64_t t_idle = 0;
@@ -252,8 +270,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
             ++gl;
             if (++se == P.n_loads) {
               se = 0;
-              su += gridDim.x;
-              if (su < n_units) sun = decode_unit(su, H, A.B, tiles);
+              su += unit_step;
+              if (su < n_units) sun = decode_unit(su, H, A.B, tiles, rank);
             }
             progress = true;
           }
@@ -270,8 +288,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
             ++bn;
             if (++blay == Lt) {
               blay = 0;
-              bu += gridDim.x;
-              if (bu < n_units) bun = decode_unit(bu, H, A.B, tiles);
+              bu += unit_step;
+              if (bu < n_units) bun = decode_unit(bu, H, A.B, tiles, rank);
             }
             progress = true;
           }
@@ -316,11 +334,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
       int wu[kIssuers], wl[kIssuers], wc[kIssuers], wkv[kIssuers], wh[kIssuers];
       uint32_t wn[kIssuers];     // stages filled into ring r
       for (int r = 0; r < kIssuers; ++r) {
-        wu[r] = blockIdx.x;
+        wu[r] = unit0;
         wl[r] = r;
         wc[r] = 0;
         wn[r] = 0;
-        const Unit un = decode_unit(wu[r] < n_units ? wu[r] : 0, H, A.B, tiles);
+        const Unit un = decode_unit(wu[r] < n_units ? wu[r] : 0, H, A.B, tiles, rank);
         wkv[r] = un.kv;
         wh[r] = un.h;
       }
@@ -340,18 +358,21 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           int nl = wl[r] + kIssuers, nu = wu[r], nkv = wkv[r], nh = wh[r];
           if (nl >= Lt) {
             nl = r;
-            nu += gridDim.x;
+            nu += unit_step;
             if (nu < n_units) {
-              const Unit nun = decode_unit(nu, H, A.B, tiles);
+              const Unit nun = decode_unit(nu, H, A.B, tiles, rank);
               nkv = nun.kv;
               nh = nun.h;
             }
           }
-          mbar_expect_tx(smem_u32(&wfull[st]), kWStageBytes);
+          // this CTA's 64 of the use's 128 output rows; both CTAs' halves complete on the
+          // rank-0 CTA's wfull, which expects the bytes of both
+          if (rank == 0) mbar_expect_tx(smem_u32(&wfull[st]), 2 * kWStageBytes);
           const uint32_t wdst = smem_u32(wst + static_cast<size_t>(st) * kWStageBytes);
-          const int wrow = ((wl[r] * 2 + wkv[r]) * H + wh[r]) * kD;
-          tma_load_2d(wdst, &P.tm_w, smem_u32(&wfull[st]), wc[r] * 128, wrow, pol);
-          tma_load_2d(wdst + kWStageBytes / 2, &P.tm_w, smem_u32(&wfull[st]), wc[r] * 128 + 64, wrow, pol);
+          const uint32_t wbar = mapa_shared(smem_u32(&wfull[st]), 0);
+          const int wrow = ((wl[r] * 2 + wkv[r]) * H + wh[r]) * kD + static_cast<int>(rank) * (kD / 2);
+          tma_load_2d_pair(wdst, &P.tm_w, wbar, wc[r] * 128, wrow, pol);
+          tma_load_2d_pair(wdst + kWStageBytes / 2, &P.tm_w, wbar, wc[r] * 128 + 64, wrow, pol);
           ++wn[r];
           if (++wc[r] == chunks) {
             wc[r] = 0;
@@ -384,7 +405,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           }
         }
       }
-      if (!ok) {   // the most recent fills of each ring may still be landing
+      if (!ok && rank == 0) {   // the most recent fills of each ring (both CTAs' halves) may still be landing
         for (int r = 0; r < kIssuers; ++r) {
           const uint32_t first = wn[r] > static_cast<uint32_t>(kRing) ? wn[r] - kRing : 0;
           for (uint32_t i = first; i < wn[r]; ++i) drain_wait(smem_u32(&wfull[r * kRing + i % kRing]), (i / kRing) & 1u);
@@ -399,19 +420,19 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     // leaves the tensor pipe idle at every wait; with two issuers on different SM
     // sub-partitions the other one's queued MMAs cover it.
     const int iss = warp == 1 ? 0 : 1;
-    if (lane == 0) {
-      constexpr uint32_t idesc = make_idesc(kTileM, kD);
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = make_idesc(2 * kTileM, kD);   // M = 256: both CTAs' token tiles
       const uint32_t d_tmem = tmem_base + iss * kAccCols;
       uint32_t ready_par = 0, acc_n = 0, wi = 0;   // wi: W stages (uses) consumed from this issuer's ring
       bool ok = true, issued = false;
       uint32_t pack_next = iss < Lt ? __ldg(&P.use_pack[iss]) : 0u;
-      for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+      for (int u = unit0; ok && u < n_units; u += unit_step) {
         for (int l = iss; ok && l < Lt; l += kIssuers, ++acc_n) {
           const uint32_t pack = pack_next;
           const int ln = l + kIssuers < Lt ? l + kIssuers : iss;
           pack_next = __ldg(&P.use_pack[ln]);   // schedule word of this issuer's next layer
           if (acc_n >= 1 && !wait_bar(smem_u32(&acce[iss]), (acc_n - 1) & 1u, abort_flag, P.status,
-                                      KVX_ERR_TIMEOUT)) {
+                                         KVX_ERR_TIMEOUT)) {
             ok = false;
             break;
           }
@@ -423,8 +444,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
             const uint32_t f = (pack >> (5 * j)) & 31u;
             const uint32_t s = f & 3u;
             if (f & 4u) {
-              if (!wait_bar(smem_u32(&tready[s * kIssuers + iss]), (ready_par >> s) & 1u, abort_flag, P.status,
-                            KVX_ERR_TIMEOUT)) {
+              if (!wait_bar(smem_u32(&tready[s * kIssuers + iss]), (ready_par >> s) & 1u, abort_flag,
+                               P.status, KVX_ERR_TIMEOUT)) {
                 ok = false;
                 break;
               }
@@ -441,20 +462,20 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
             const uint32_t b1 = b0 + kWStageBytes / 2;
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
-              tc_mma_ts(d_tmem, a_col + kk * 8, sw128_desc(b0 + kk * 32), idesc, (j | kk) != 0);
+              tc_mma_ts_pair(d_tmem, a_col + kk * 8, sw128_desc(b0 + kk * 32), idesc, (j | kk) != 0);
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
-              tc_mma_ts(d_tmem, a_col + 32 + kk * 8, sw128_desc(b1 + kk * 32), idesc, true);
+              tc_mma_ts_pair(d_tmem, a_col + 32 + kk * 8, sw128_desc(b1 + kk * 32), idesc, true);
             issued = true;
-            tc_commit(smem_u32(&wempty[st0]));
-            if (f & 16u) tc_commit(smem_u32(&tfree[s * kIssuers + iss]));
+            tc_commit_pair(smem_u32(&wempty[st0]), 3);
+            if (f & 16u) tc_commit_pair(smem_u32(&tfree[s * kIssuers + iss]), 3);
           }
-          if (ok) tc_commit(smem_u32(&accf[iss]));
+          if (ok) tc_commit_pair(smem_u32(&accf[iss]), 3);
         }
       }
       // every MMA (and every commit) of this issuer must have completed before TMEM is freed
       if (issued || !ok) {
-        tc_commit(smem_u32(&drain[iss]));
+        tc_commit_pair(smem_u32(&drain[iss]), 1);
         drain_wait(smem_u32(&drain[iss]), 0);
       }
     }
@@ -471,8 +492,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     uint8_t* wstage = outst + static_cast<size_t>(warp - kFirstEpiWarp) * kStageBufs * kWarpStageBytes;
     float cs[32], sn[32];
     bool ok = true;
-    for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-      const Unit un = decode_unit(u, H, A.B, tiles);
+    for (int u = unit0; ok && u < n_units; u += unit_step) {
+      const Unit un = decode_unit(u, H, A.B, tiles, rank);
       const int t = un.t0 + r;
       bool valid = t < A.T;
       bool bad = false;
@@ -556,7 +577,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           if (rnd == 1) {  // the accumulator is free for the issuer's next layer
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&acce[buf]));
+            if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&acce[buf]), 0));
           }
           const int c_lo = 32 * g + 16 * rnd;   // channels c_lo + [0,16) and 64 + c_lo + [0,16)
           float ylo[16], yhi[16];
@@ -651,8 +672,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
     uint32_t gl = 0, tl_loaded = 0, tfree_par = 0;
     float cs[64], sn[64];   // cos / sin of the source angle of pair i of row r
     bool ok = true;
-    for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-      const Unit un = decode_unit(u, H, A.B, tiles);
+    for (int u = unit0; ok && u < n_units; u += unit_step) {
+      const Unit un = decode_unit(u, H, A.B, tiles, rank);
       if (un.kv == 0) {
         // a row past the sequence end or at an out-of-range position (which the epilogue
         // reports) is rotated by angle 0: its output is never written
@@ -732,7 +753,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
           mbar_arrive(smem_u32(&land_empty[lb]));
 #pragma unroll
           for (int i = 0; i < kIssuers; ++i)
-            if ((lw >> (4 + i)) & 1u) mbar_arrive(smem_u32(&tready[s * kIssuers + i]));
+            if ((lw >> (4 + i)) & 1u) mbar_arrive_cluster(mapa_shared(smem_u32(&tready[s * kIssuers + i]), 0));
         }
         ++gl;
       }
@@ -741,9 +762,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_map_kernel(const __grid_consta
 
   tc_fence_before();
   __syncthreads();
+  cluster_sync();   // no arrival or MMA of either CTA still targets the other
   tc_fence_after();
   if (warp == 1) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(kTmemCols)
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(kTmemCols)
                  : "memory");
   }
 }
@@ -966,7 +988,7 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   }
   const cuuint64_t wdims[2] = {static_cast<cuuint64_t>(c->F), static_cast<cuuint64_t>(c->Lt) * 2 * c->H * kD};
   const cuuint64_t wstr[1] = {static_cast<cuuint64_t>(c->F) * 2};
-  const cuuint32_t wbox[2] = {64, kD};
+  const cuuint32_t wbox[2] = {64, kD / 2};   // one CTA's 64 output rows x 64 features
   CUresult r = encode(&P.tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, c->d_Wt, wdims, wstr, wbox, ones,
                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                       CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -985,7 +1007,8 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   P.H = c->H;
   P.k = c->k;
   P.n_loads = p.n_loads;
-  P.tiles_per_seq = (a.T + kTileM - 1) / kTileM;
+  // work units are pairs of adjacent 128-token tiles (one per CTA of a cluster)
+  P.tiles_per_seq = (a.T + 2 * kTileM - 1) / (2 * kTileM);
   const int64_t units = static_cast<int64_t>(a.B) * P.tiles_per_seq * c->H * 2;
   if (units > INT_MAX) {
     set_error("kvx_map: too many work units");
@@ -1013,7 +1036,7 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
               " registers per thread, too few for its warpgroup register split");
     return KVX_ERR_UNSUPPORTED;
   }
-  const int grid = static_cast<int>(std::min<int64_t>(units, c->sm_count));
+  const int grid = 2 * static_cast<int>(std::min<int64_t>(units, std::max(c->sm_count / 2, 1)));   // CTA pairs
   tc_map_kernel<<<grid, kThreads, smem, stream>>>(P);
   e = cudaGetLastError();
   if (e != cudaSuccess) {
