@@ -405,7 +405,11 @@ def main():
                 "other": {"hbm_achieved_gbs": alg["bytes"] / launch_s / 1e9, "hbm_peak_gbs": peaks["hbm"],
                           "hbm_frac": alg["bytes"] / launch_s / 1e9 / peaks["hbm"],
                           "tensor_achieved_tflops": alg["flop"] / launch_s / 1e12,
-                          "tensor_frac": alg["flop"] / launch_s / 1e12 / peaks["bf16"]},
+                          "tensor_frac": alg["flop"] / launch_s / 1e12 / peaks["bf16"],
+                          # against cuBLAS run back to back under the power cap (the
+                          # regime a long bench run settles in); context, not the headline
+                          "tensor_frac_of_sustained": (alg["flop"] / launch_s / 1e12 / peaks["bf16_sustained"]
+                                                       if peaks.get("bf16_sustained") else None)},
                 "algorithmic": {"flop_per_launch": alg["flop"], "bytes_per_launch": alg["bytes"],
                                 "flop_per_token": alg["flop_per_token"],
                                 "bytes_per_token": alg["bytes_per_token"],
