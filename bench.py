@@ -211,7 +211,7 @@ def oracle_sample_rate(w, budget_s, seed=0, ctx_sel=None):
         svf = obf16.decode(sv.view(torch.int16).numpy().view(np.uint16))
         p = pos[rows[:, 0], rows[:, 1]]
         t0 = time.perf_counter()
-        omap.map_tokens(skf, svf, p, sel, Wf, bf, w.theta_s, w.theta_t, mode="bf16fwd")
+        omap.map_tokens(skf, svf, p, sel, Wf, bf, w.theta_s, w.theta_t, mode="bf16fwd", head_mix=w.head_mix)
         return time.perf_counter() - t0
 
     n, dt = 8, run(8)
@@ -258,7 +258,7 @@ def reference_arm(args, w, config):
         svf = obf16.decode(syn.source_rows(w, 1, rows).view(torch.int16).numpy().view(np.uint16))
         t0 = time.perf_counter()
         omap.map_tokens(skf, svf, pos[rows[:, 0], rows[:, 1]], sel, Wf, bf, w.theta_s, w.theta_t,
-                        mode="bf16fwd")
+                        mode="bf16fwd", head_mix=w.head_mix)
         dt = time.perf_counter() - t0
         if i >= args.warmup:
             times.append(dt)
@@ -283,7 +283,8 @@ def make_mapper(w, dev_index):
     W, b = syn.weights(w)
     cfg, keep = kvx.config_from_tensors(
         src_layers=w.Ls, tgt_layers=w.Lt, n_kv_heads=w.H, head_dim=w.d, k=w.k, theta_s=w.theta_s,
-        theta_t=w.theta_t, cache_dtype=w.cache_dtype, W=W, b=b, scores=syn.selection_scores(w))
+        theta_t=w.theta_t, cache_dtype=w.cache_dtype, W=W, b=b, scores=syn.selection_scores(w),
+        head_mix=kvx.KVX_CROSS_HEAD if w.head_mix == "cross_head" else kvx.KVX_PER_HEAD)
     return kvx.kvx_create(cfg, dev_index)
 
 
@@ -426,8 +427,11 @@ def main():
             "clocks": clk.summary(), "status": kvx.kvx_status_string(st),
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "steps": e2e_steps, "ms_per_step": ems / e2e_steps},
-            "gpu_launches": args.steps, "roofline": roofline, "cpu_baseline": cpu,
-            "kernel": "tc_map_kernel (tcgen05, sm_103a)"}
+            # one launch per step (per-head); the cross-head map is a key-strip kernel then the GEMMs
+            "gpu_launches": args.steps * (2 if w.head_mix == "cross_head" else 1), "roofline": roofline,
+            "cpu_baseline": cpu,
+            "kernel": ("xh_strip_kernel + tc_xh_kernel (tcgen05 pair GEMM, sm_103a)" if w.head_mix == "cross_head"
+                       else "tc_map_kernel (tcgen05, sm_103a)")}
     print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()

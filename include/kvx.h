@@ -66,9 +66,13 @@ typedef enum { KVX_ROPE_HALF = 0, KVX_ROPE_INTERLEAVED = 1 } kvx_rope_style;
  * (the paper's d_s = k n_kv d_h, Sec. 3.1 / Sec. 3.2). */
 typedef enum { KVX_PER_HEAD = 0, KVX_CROSS_HEAD = 1 } kvx_head_mix;
 
-/* Which kernel kvx_map launches.  AUTO picks the tensor-core (tcgen05) kernel when the
- * shape allows it (bf16 caches and weights, head_dim 128, PER_HEAD, HALF) and the
- * fp32 SIMT kernel otherwise. */
+/* Which kernel kvx_map launches.  AUTO picks a tensor-core (tcgen05) kernel when the
+ * shape allows it (bf16 caches and weights, head_dim 128, HALF; PER_HEAD with k <= 4, or
+ * CROSS_HEAD with an even head count and a contiguous target) and the fp32 SIMT kernel
+ * otherwise.  The CROSS_HEAD tensor-core kernel keeps a workspace for the stripped source
+ * keys (L_s * B * n_kv * T * head_dim bf16) in the context, allocated by the first
+ * kvx_map that needs it (a blocking cudaMalloc) and grown when a later call needs more;
+ * kvx_destroy frees it. */
 typedef enum { KVX_KERNEL_AUTO = 0, KVX_KERNEL_SIMT = 1, KVX_KERNEL_TCGEN05 = 2 } kvx_kernel;
 
 /* Mapper description, read by kvx_create.  All pointers are HOST pointers; the

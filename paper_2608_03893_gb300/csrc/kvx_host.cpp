@@ -83,6 +83,7 @@ static void free_ctx(kvx_ctx* c) {
   cudaFree(c->d_Wt);
   cudaFree(c->d_plan);
   cudaFree(c->d_status);
+  cudaFree(c->d_ws);
   delete c;
 }
 
@@ -241,8 +242,9 @@ kvx_status kvx_create(const kvx_config* cfg, int device, kvx_ctx** out) {
 
   std::string why;
   ctx->tc_eligible = tc_supported(ctx, &why);
-  if (ctx->tc_eligible) {
-    kvx_status s = tc_prepare(ctx, c.W);
+  ctx->xh_eligible = xh_supported(ctx, &why);
+  if (ctx->tc_eligible || ctx->xh_eligible) {
+    kvx_status s = ctx->tc_eligible ? tc_prepare(ctx, c.W) : repack_wt(ctx, c.W);
     if (s != KVX_OK) {
       free_ctx(ctx);
       return s;
@@ -275,9 +277,9 @@ kvx_status kvx_set_kernel(kvx_ctx* ctx, int32_t kernel) {
   if (!ctx) return fail(KVX_ERR_INVALID_ARG, "kvx_set_kernel: NULL ctx");
   if (kernel != KVX_KERNEL_AUTO && kernel != KVX_KERNEL_SIMT && kernel != KVX_KERNEL_TCGEN05)
     return fail(KVX_ERR_INVALID_ARG, "kvx_set_kernel: unknown kernel");
-  if (kernel == KVX_KERNEL_TCGEN05 && !ctx->tc_eligible) {
+  if (kernel == KVX_KERNEL_TCGEN05 && !ctx->tc_eligible && !ctx->xh_eligible) {
     std::string why;
-    tc_supported(ctx, &why);
+    if (ctx->head_mix == KVX_CROSS_HEAD) xh_supported(ctx, &why); else tc_supported(ctx, &why);
     return fail(KVX_ERR_UNSUPPORTED, "kvx_set_kernel: tensor-core kernel unavailable: " + why);
   }
   ctx->kernel = kernel;
@@ -349,6 +351,10 @@ kvx_status kvx_map(kvx_ctx* ctx, const kvx_src* src, int32_t batch, int32_t toke
   DeviceGuard guard(ctx->device);
   if (guard.err != cudaSuccess) return cuda_fail(guard.err, "kvx_map: cudaSetDevice");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // cross-head: the tensor-core kernel writes contiguous targets; AUTO maps paged ones
+  // with the SIMT kernel, an explicit TCGEN05 choice gets KVX_ERR_UNSUPPORTED from it
+  if (ctx->xh_eligible && (ctx->kernel == KVX_KERNEL_TCGEN05 || (ctx->kernel == KVX_KERNEL_AUTO && !a.paged)))
+    return launch_xh(ctx, a, st);
   const bool use_tc = ctx->kernel == KVX_KERNEL_TCGEN05 || (ctx->kernel == KVX_KERNEL_AUTO && ctx->tc_eligible);
   return use_tc ? launch_tc(ctx, a, st) : launch_simt(ctx, a, st);
 }

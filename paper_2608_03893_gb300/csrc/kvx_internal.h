@@ -62,6 +62,7 @@ struct kvx_ctx {
   double theta_s = 0, theta_t = 0;
   int kernel = KVX_KERNEL_AUTO;
   bool tc_eligible = false;
+  bool xh_eligible = false;         // cross-head tensor-core kernel
   std::vector<int32_t> sel;          // host copy [L_t][k]
   kvx::RopeTables rope{};
   // device memory owned by the context
@@ -71,6 +72,8 @@ struct kvx_ctx {
   void* d_Wt = nullptr;              // tensor-core layout (bf16), see kvx_tc.cu
   int32_t* d_plan = nullptr;         // tensor-core schedule tables
   int32_t* d_status = nullptr;       // device status word
+  void* d_ws = nullptr;              // cross-head kernel: source keys with the RoPE stripped
+  size_t ws_bytes = 0;
   kvx::TcPlan plan;
   int sm_count = 0;
 };
@@ -88,4 +91,14 @@ kvx_status launch_simt(const kvx_ctx* ctx, const MapArgs& a, cudaStream_t stream
 bool tc_supported(const kvx_ctx* ctx, std::string* why);
 kvx_status tc_prepare(kvx_ctx* ctx, const void* W_host);   // repack W, build the plan
 kvx_status launch_tc(const kvx_ctx* ctx, const MapArgs& a, cudaStream_t stream);
+// W [L_t][2][H][F][d] -> W^T [L_t][2][H][d][F] bf16 in ctx->d_Wt (both tensor-core kernels).
+kvx_status repack_wt(kvx_ctx* ctx, const void* W_host);
+// cuTensorMapEncodeTiled from the driver (as void*: PFN_cuTensorMapEncodeTiled_v12000), or NULL.
+void* tensor_map_encoder();
+
+// Tensor-core kernel for the cross-head feature layout (bf16, head_dim 128, half-split
+// pairs, even head count, contiguous targets): a source-key RoPE strip into a workspace,
+// then one pair-MMA GEMM per (target layer, K|V).
+bool xh_supported(const kvx_ctx* ctx, std::string* why);
+kvx_status launch_xh(kvx_ctx* ctx, const MapArgs& a, cudaStream_t stream);
 }  // namespace kvx

@@ -872,6 +872,8 @@ void build_plan(const kvx_ctx* c, TcPlan* plan) {
 
 }  // namespace
 
+void* tensor_map_encoder() { return reinterpret_cast<void*>(get_encode()); }
+
 bool tc_supported(const kvx_ctx* c, std::string* why) {
   std::string w;
   if (c->cache_dtype != KVX_BF16 || c->weight_dtype != KVX_BF16) w = "needs bf16 caches and weights";
@@ -884,7 +886,7 @@ bool tc_supported(const kvx_ctx* c, std::string* why) {
   return w.empty();
 }
 
-kvx_status tc_prepare(kvx_ctx* c, const void* W_host) {
+kvx_status repack_wt(kvx_ctx* c, const void* W_host) {
   // W [L_t][2][H][F][128] -> W^T [L_t][2][H][128][F] (B operand, K-major)
   const size_t F = c->F;
   const size_t blocks = static_cast<size_t>(c->Lt) * 2 * c->H;
@@ -905,6 +907,13 @@ kvx_status tc_prepare(kvx_ctx* c, const void* W_host) {
     set_error(std::string("kvx_create: upload W^T: ") + cudaGetErrorString(e));
     return KVX_ERR_CUDA;
   }
+  return KVX_OK;
+}
+
+kvx_status tc_prepare(kvx_ctx* c, const void* W_host) {
+  kvx_status st = repack_wt(c, W_host);
+  if (st != KVX_OK) return st;
+  cudaError_t e;
   build_plan(c, &c->plan);
   c->plan.n_wst = kNW;   // two rings of kRing stages
   c->plan.n_land = kLand;

@@ -119,11 +119,12 @@ class Workload:
     turns: int = 1
     block_size: int = 16
     len_range: tuple = (0, 0)   # initial per-sequence lengths (paged), inclusive
+    head_mix: str = "per_head"  # "per_head" (F = k d) | "cross_head" (F = k H d, the paper's)
     notes: str = field(default="", compare=False)
 
     @property
     def F(self):
-        return self.k * self.d
+        return self.k * self.d * (self.H if self.head_mix == "cross_head" else 1)
 
     @property
     def n_tokens(self):
@@ -152,6 +153,12 @@ WORKLOADS = {
     "qwen3_32b_14b_paged_b16_turn2048_k4": Workload(
         "qwen3_32b_14b_paged_b16_turn2048_k4", 64, 40, 8, 128, 4, 16, 2048, 1e6, 1e6, "bf16",
         "bf16", "depth", 0.01, 4, paged=True, turns=8, block_size=16, len_range=(2048, 16384)),
+    # the paper's mapper layout (every KV head of the selected layers feeds every target
+    # head); k = 8 is the Qwen3 14B -> 32B pair of its latency table
+    "qwen3_14b_32b_t32768_k4_xhead": Workload("qwen3_14b_32b_t32768_k4_xhead", 40, 64, 8, 128, 4, 1, 32768,
+                                              1e6, 1e6, "bf16", "bf16", "depth", 0.01, 2, head_mix="cross_head"),
+    "qwen3_14b_32b_t32768_k8_xhead": Workload("qwen3_14b_32b_t32768_k8_xhead", 40, 64, 8, 128, 8, 1, 32768,
+                                              1e6, 1e6, "bf16", "bf16", "depth", 0.01, 2, head_mix="cross_head"),
 }
 
 HEADLINE = "qwen3_14b_32b_t32768_k4"

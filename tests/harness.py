@@ -45,7 +45,8 @@ def make_ctx(w, kernel=kvx.KVX_KERNEL_AUTO, selection=None, W=None, b=None, scor
     cfg, keep = kvx.config_from_tensors(
         src_layers=w.Ls, tgt_layers=w.Lt, n_kv_heads=w.H, head_dim=w.d, k=w.k,
         theta_s=w.theta_s, theta_t=w.theta_t, cache_dtype=w.cache_dtype, W=W, b=b,
-        selection=selection, scores=scores, rope_style=rope_style)
+        selection=selection, scores=scores, rope_style=rope_style,
+        head_mix=kvx.KVX_CROSS_HEAD if w.head_mix == "cross_head" else kvx.KVX_PER_HEAD)
     ctx = kvx.kvx_create(cfg, device)
     if kernel != kvx.KVX_KERNEL_AUTO:
         kvx.kvx_set_kernel(ctx, kernel)
@@ -75,7 +76,7 @@ def oracle_full(w, sk, sv, pos_np, sel, W, b, style="half"):
     mode = "exact" if w.cache_dtype == "f32" else "bf16fwd"
     return omap.map_cache(to_f64(sk), to_f64(sv), pos_np, sel, to_f64(W),
                           None if b is None else to_f64(b), w.theta_s, w.theta_t, mode=mode,
-                          style=style, rounding_slack=STRIP_DELTA)
+                          style=style, head_mix=w.head_mix, rounding_slack=STRIP_DELTA)
 
 
 def check(w, got, ref, slack=None):
@@ -116,4 +117,5 @@ def oracle_rows(w, rows, pos_np, sel, W, b, turn=None):
     sv = to_f64(syn.source_rows(w, 1, rows, turn=turn))
     p = pos_np[rows[:, 0], rows[:, 1]]
     return omap.map_tokens(sk, sv, p, sel, to_f64(W), None if b is None else to_f64(b),
-                           w.theta_s, w.theta_t, mode=mode, rounding_slack=STRIP_DELTA)
+                           w.theta_s, w.theta_t, mode=mode, head_mix=w.head_mix,
+                           rounding_slack=STRIP_DELTA)

@@ -396,3 +396,72 @@ def test_target_layouts_bit_identical(kname):
             assert torch.equal(tk, ref_k) and torch.equal(tv, ref_v), name
     finally:
         kvx.kvx_destroy(ctx)
+
+
+# -------------------------------------------------------- cross-head (NEXT-1) -----
+
+@pytest.mark.parametrize("over", [
+    dict(Ls=3, Lt=4, H=2, B=1, T=300, k=2),                # ragged tail, odd tile count
+    dict(Ls=5, Lt=3, H=4, B=2, T=129, k=3, theta_t=5e5),   # B > 1, different thetas, 1-row tail
+    dict(Ls=4, Lt=2, H=2, B=1, T=1, k=1),                  # one token
+    dict(Ls=6, Lt=3, H=8, B=1, T=256, k=4),                # eight heads, two full tiles
+    dict(Ls=9, Lt=2, H=2, B=1, T=200, k=8, scores="uniform"),   # k = 8: 16 K steps, random selection
+])
+def test_cross_head_tc_small(over):
+    """Cross-head tensor-core path (key strip, pair GEMM, epilogue) against the float64
+    oracle on every output element, three launches each."""
+    w = syn.workload("qwen3_14b_32b_t32768_k4_xhead", **over)
+    ctx, sel, W, b = make_ctx(w, kernel=kvx.KVX_KERNEL_TCGEN05)
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w)
+        rk, rv, ak, av = oracle_full(w, sk, sv, pos, sel, W, b)
+        for rep in range(3):
+            tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+            assert st == kvx.KVX_OK
+            ok, ratio, rms, nbad = check(w, [to_f64(tk), to_f64(tv)], [rk, rv], [ak, av])
+            assert ok, "launch %d: %d elements out of tolerance (worst %.3g x bound)" % (rep, nbad, ratio)
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
+def test_cross_head_tc_paged_is_refused_but_auto_maps_it():
+    """The cross-head tensor-core kernel writes contiguous targets: an explicit TCGEN05
+    choice on a paged target is refused before any launch, AUTO maps it with SIMT."""
+    w = syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4", Ls=4, Lt=2, H=2, B=2, T=20, k=2,
+                     len_range=(3, 40), head_mix="cross_head")
+    ctx, sel, W, b = make_ctx(w, kernel=kvx.KVX_KERNEL_TCGEN05)
+    try:
+        with pytest.raises(kvx.KvxError) as e:
+            _paged_run(w, 0, syn.initial_lengths(w), ctx)
+        assert e.value.status == kvx.KVX_ERR_UNSUPPORTED
+        kvx.kvx_set_kernel(ctx, kvx.KVX_KERNEL_AUTO)
+        _check_paged(w, ctx, sel, W, b, 0, syn.initial_lengths(w), sample_rows(w, 12, turn_T=w.T))
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
+def test_cross_head_full_size_sampled():
+    """The cross-head bench workload (Qwen3-14B -> 32B shapes, k = 4, 32768 tokens): sampled
+    rows against the oracle, every row written."""
+    w = syn.workload("qwen3_14b_32b_t32768_k4_xhead")
+    ctx, sel, W, b = make_ctx(w)
+    dev = torch.device("cuda:0")
+    try:
+        sk = syn.source_cache(w, 0, device=dev)
+        sv = syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w)
+        tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        del sk, sv
+        assert not torch.isnan(tk).any() and not torch.isnan(tv).any(), "unwritten rows"
+        rows = sample_rows(w, 6)
+        rk, rv, ak, av = oracle_rows(w, rows, pos, sel, W, b)
+        gk = to_f64(tk[:, rows[:, 0], :, rows[:, 1]].permute(1, 2, 0, 3))
+        gv = to_f64(tv[:, rows[:, 0], :, rows[:, 1]].permute(1, 2, 0, 3))
+        ok, ratio, rms, nbad = check(w, [gk, gv], [rk, rv], [ak, av])
+        assert ok, "%d sampled elements out of tolerance (worst %.3g x bound)" % (nbad, ratio)
+    finally:
+        kvx.kvx_destroy(ctx)
+        torch.cuda.empty_cache()
