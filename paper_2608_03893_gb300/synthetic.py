@@ -155,6 +155,8 @@ WORKLOADS = {
         "bf16", "depth", 0.01, 4, paged=True, turns=8, block_size=16, len_range=(2048, 16384)),
     # the paper's mapper layout (every KV head of the selected layers feeds every target
     # head); k = 8 is the Qwen3 14B -> 32B pair of its latency table
+    "qwen3_14b_32b_b8x1024_k4_xhead": Workload("qwen3_14b_32b_b8x1024_k4_xhead", 40, 64, 8, 128, 4, 8, 1024,
+                                               1e6, 1e6, "bf16", "bf16", "depth", 0.01, 1, head_mix="cross_head"),
     "qwen3_14b_32b_t32768_k4_xhead": Workload("qwen3_14b_32b_t32768_k4_xhead", 40, 64, 8, 128, 4, 1, 32768,
                                               1e6, 1e6, "bf16", "bf16", "depth", 0.01, 2, head_mix="cross_head"),
     "qwen3_14b_32b_t32768_k8_xhead": Workload("qwen3_14b_32b_t32768_k8_xhead", 40, 64, 8, 128, 8, 1, 32768,
