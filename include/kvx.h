@@ -178,6 +178,33 @@ KVX_API kvx_status kvx_get_status(kvx_ctx* ctx, void* stream);
 KVX_API int64_t kvx_mapper_params(int32_t tgt_layers, int32_t n_kv_heads, int32_t head_dim, int32_t k,
                           int32_t head_mix);
 
+/* Ridge fit of the per-head mapper on calibration caches (Sec. 3.1, Eq. Wstar; Sec. 3.3
+ * for the keys): for every target layer l, K|V and head h, over the N = batch *
+ * tokens_per_seq calibration tokens, X = the k selected source layers' head h (keys with
+ * the source RoPE stripped) concatenated in selection order, Y = head h of target layer l
+ * (keys with the target RoPE stripped), both centred by their column means;
+ *   W = (Xc^T Xc + lambda I)^{-1} Xc^T Yc  (lambda on the unnormalised sum),
+ *   b = mean(Y) - mean(X) W.
+ * `src` holds the source caches [L_s][B][H][T][d] and `tgt` the target caches
+ * [L_t][B][H][T][d] of the same tokens (kvx_src layout, bf16, d = 128, 16-byte aligned);
+ * `positions` device [batch][tokens_per_seq].  `selection` (host [L_t][k], 1 <= k <= 4)
+ * as in kvx_config.  Outputs on the device, fp32: W [L_t][2][H][k*d][d] and
+ * b [L_t][2][H][d] (the kvx_config layouts).  Cross-products accumulate in fp32 on
+ * centred values; the factorisation and the solves run in fp64.  Runs on `stream` and
+ * synchronises it before returning (an offline step; it allocates stream-ordered
+ * workspace of about L_t*2*H*(k*k + k)*64 KB plus 8 MB per SM).  INVALID_ARG for bad
+ * arguments or when a system is not positive definite (lambda = 0 with too few tokens);
+ * DEVICE_BOUNDS when a position is outside [0, 2^24). */
+typedef struct {
+  int32_t src_layers, tgt_layers, n_kv_heads, head_dim, k;
+  double src_rope_theta, tgt_rope_theta;
+  double lambda;                 /* >= 0; the paper's value is 0.01 */
+  const int32_t* selection;      /* host [tgt_layers][k], entries in [0, src_layers) */
+} kvx_fit_config;
+KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, const kvx_src* tgt, int32_t batch,
+                                 int32_t tokens_per_seq, const int32_t* positions, float* W, float* b,
+                                 void* stream);
+
 /* Static description of a status code. */
 KVX_API const char* kvx_status_string(kvx_status s);
 

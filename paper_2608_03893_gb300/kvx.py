@@ -65,11 +65,20 @@ class kvx_noalloc_mapper(ctypes.Structure):
     ]
 
 
+class kvx_fit_config(ctypes.Structure):
+    _fields_ = [
+        ("src_layers", ctypes.c_int32), ("tgt_layers", ctypes.c_int32),
+        ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("k", ctypes.c_int32),
+        ("src_rope_theta", ctypes.c_double), ("tgt_rope_theta", ctypes.c_double),
+        ("lambda_", ctypes.c_double), ("selection", ctypes.c_void_p),
+    ]
+
+
 _lib = None
 
 EXPORTED = ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
             "kvx_set_kernel", "kvx_get_status", "kvx_mapper_params", "kvx_status_string",
-            "kvx_last_error", "kvx_map_noalloc")
+            "kvx_last_error", "kvx_map_noalloc", "kvx_fit_ridge")
 
 
 def lib():
@@ -97,8 +106,10 @@ def lib():
     L.kvx_last_error.restype = ctypes.c_char_p
     L.kvx_map_noalloc.argtypes = [ctypes.POINTER(kvx_noalloc_mapper), ctypes.c_int, ctypes.POINTER(kvx_src),
                                   i32, i32, vp, ctypes.POINTER(kvx_tgt), vp, ctypes.POINTER(i32)]
+    L.kvx_fit_ridge.argtypes = [ctypes.POINTER(kvx_fit_config), ctypes.POINTER(kvx_src), ctypes.POINTER(kvx_src),
+                                i32, i32, vp, vp, vp, vp]
     for name in ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
-                 "kvx_set_kernel", "kvx_get_status", "kvx_map_noalloc"):
+                 "kvx_set_kernel", "kvx_get_status", "kvx_map_noalloc", "kvx_fit_ridge"):
         getattr(L, name).restype = ctypes.c_int
     _lib = L
     return L
@@ -273,3 +284,16 @@ def tgt_paged_from_tensors(k, v, block_table, block_size):
     t.max_blocks_per_seq = block_table.shape[1]
     t.n_blocks = k.shape[1]
     return t
+
+
+def kvx_fit_ridge(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, selection,
+                  src, tgt, batch, tokens_per_seq, positions_ptr, W_ptr, b_ptr, stream=0):
+    """Ridge fit on calibration caches (see include/kvx.h): src / tgt are kvx_src, selection a
+    host int32 [L_t][k] array, W_ptr / b_ptr device fp32 buffers [L_t][2][H][k*d][d] and
+    [L_t][2][H][d].  Blocks until the fit is done."""
+    import numpy as np
+    sel = np.ascontiguousarray(selection, dtype=np.int32)
+    cfg = kvx_fit_config(int(src_layers), int(tgt_layers), int(n_kv_heads), int(head_dim), int(k),
+                         float(theta_s), float(theta_t), float(lam), _ptr(sel))
+    _check(lib().kvx_fit_ridge(ctypes.byref(cfg), ctypes.byref(src), ctypes.byref(tgt), int(batch),
+                               int(tokens_per_seq), positions_ptr, W_ptr, b_ptr, stream), "kvx_fit_ridge")

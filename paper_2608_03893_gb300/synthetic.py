@@ -216,6 +216,12 @@ def source_cache(w, kv, device="cpu", turn=None, out=None):
     return out
 
 
+def target_cache(w, kv, device="cpu"):
+    """Calibration target cache [L_t][B][H][T][d] for a ridge fit: the source-cache recipe
+    for L_t layers under seed w.seed + 1000 (independent of the source cache)."""
+    return source_cache(replace(w, Ls=w.Lt, seed=w.seed + 1000, paged=False), kv, device=device)
+
+
 def source_rows(w, kv, rows, turn=None):
     """Source values for chosen token rows, on the CPU, identical to ``source_cache``.
 

@@ -143,3 +143,27 @@ def test_null_arguments_are_rejected():
     assert L.kvx_get_status(None, None) == kvx.KVX_ERR_INVALID_ARG
     assert L.kvx_set_kernel(None, 0) == kvx.KVX_ERR_INVALID_ARG
     assert L.kvx_get_selection(None, None) == kvx.KVX_ERR_INVALID_ARG
+
+
+def test_fit_ridge_rejects_bad_arguments_before_touching_the_device():
+    """kvx_fit_ridge validates everything on the host first (no GPU is needed to see it)."""
+    good = dict(src_layers=4, tgt_layers=3, n_kv_heads=2, head_dim=128, k=2, theta_s=1e6, theta_t=1e6,
+                lam=0.01, selection=np.array([[0, 1], [1, 2], [2, 3]], dtype=np.int32))
+    buf = np.zeros(64, dtype=np.float32)          # a 16-byte aligned stand-in for device pointers
+    src = kvx.kvx_src(buf.ctypes.data, buf.ctypes.data, (ctypes.c_int64 * 4)(4096, 4096, 256, 128))
+    cases = [dict(head_dim=64), dict(k=5), dict(k=0), dict(lam=-1.0), dict(theta_t=1.0),
+             dict(selection=np.array([[0, 4], [1, 2], [2, 3]], dtype=np.int32)),
+             dict(src_layers=1)]
+    for over in cases:
+        a = dict(good, **over)
+        with pytest.raises(kvx.KvxError) as e:
+            kvx.kvx_fit_ridge(a["src_layers"], a["tgt_layers"], a["n_kv_heads"], a["head_dim"], a["k"],
+                              a["theta_s"], a["theta_t"], a["lam"], a["selection"], src, src, 1, 16,
+                              buf.ctypes.data, buf.ctypes.data, buf.ctypes.data)
+        assert e.value.status == kvx.KVX_ERR_INVALID_ARG, over
+    with pytest.raises(kvx.KvxError) as e:                 # NULL output
+        a = good
+        kvx.kvx_fit_ridge(a["src_layers"], a["tgt_layers"], a["n_kv_heads"], a["head_dim"], a["k"],
+                          a["theta_s"], a["theta_t"], a["lam"], a["selection"], src, src, 1, 16,
+                          buf.ctypes.data, None, buf.ctypes.data)
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG

@@ -1,0 +1,115 @@
+"""GPU parity of the ridge fit (kvx_fit_ridge, through the C ABI) against the float64 oracle
+(oracle.ridge.fit_ridge on RoPE-stripped features built with oracle.rope), on seeded
+synthetic calibration caches.
+
+Tolerance (derived from the arithmetic): the GPU accumulates the centred cross-products
+of N tokens in fp32, so every entry of Xc^T Xc and Xc^T Yc carries a relative error of at
+most about N u (u = 2^-24) of the Cauchy-Schwarz scale sqrt(G_ii G_jj); the fp64
+factorisation and solves add nothing comparable.  The solution of the perturbed system then
+differs by at most kappa(A) times that normwise relative error, so the test bounds
+max |W_gpu - W_ref| by 8 kappa N u max |W_ref| (+ the same relative bound on the bias,
+scaled by the largest feature mean)."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import bf16 as obf16
+from oracle import ridge as oridge
+from oracle import rope as orope
+from paper_2608_03893_gb300 import kvx
+from paper_2608_03893_gb300 import synthetic as syn
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_03893_gb300 import build as kbuild
+    kbuild.build()
+    kvx.lib()
+    torch.cuda.set_device(0)
+
+
+def _f64(t):
+    return obf16.decode(t.cpu().view(torch.int16).numpy().view(np.uint16))
+
+
+def _features(w, cache, kv, theta, pos):
+    """[L][B][H][T][d] cache -> float64 [L][H][N][d] with keys RoPE-stripped."""
+    x = _f64(cache)                                   # [L][B][H][T][d]
+    L, B, H, T, d = x.shape
+    x = x.transpose(0, 2, 1, 3, 4).reshape(L, H, B * T, d)
+    if kv == 0:
+        x = orope.rotate(x, pos.reshape(-1)[None, None, :], theta, inverse=True)
+    return x
+
+
+def _run_fit(w, lam, sel):
+    dev = torch.device("cuda:0")
+    sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+    tk, tv = syn.target_cache(w, 0, device=dev), syn.target_cache(w, 1, device=dev)
+    pos = syn.positions(w)
+    posd = torch.from_numpy(pos).to(dev)
+    F = w.k * w.d
+    W = torch.full((w.Lt, 2, w.H, F, w.d), float("nan"), dtype=torch.float32, device=dev)
+    b = torch.full((w.Lt, 2, w.H, w.d), float("nan"), dtype=torch.float32, device=dev)
+    s = torch.cuda.current_stream().cuda_stream
+    kvx.kvx_fit_ridge(w.Ls, w.Lt, w.H, w.d, w.k, w.theta_s, w.theta_t, lam, sel,
+                      kvx.src_from_tensors(sk, sv), kvx.src_from_tensors(tk, tv), w.B, w.T,
+                      posd.data_ptr(), W.data_ptr(), b.data_ptr(), s)
+    return (sk, sv, tk, tv, pos), W.cpu().double().numpy(), b.cpu().double().numpy()
+
+
+def _check_systems(w, lam, sel, caches, Wg, bg, systems):
+    sk, sv, tk, tv, pos = caches
+    feats = {}
+    N = w.B * w.T
+    for (l, kv, h) in systems:
+        if kv not in feats:
+            feats[kv] = (_features(w, sk if kv == 0 else sv, kv, w.theta_s, pos),
+                         _features(w, tk if kv == 0 else tv, kv, w.theta_t, pos))
+        xs, xt = feats[kv]
+        X = np.concatenate([xs[s, h] for s in sel[l]], axis=-1)
+        Y = xt[l, h]
+        Wr, br = oridge.fit_ridge(X, Y, lam)
+        Xc = X - X.mean(axis=0)
+        A = Xc.T @ Xc + lam * np.eye(X.shape[1])
+        kappa = np.linalg.cond(A)
+        rel = 8.0 * kappa * N * 2.0 ** -24
+        errW = np.max(np.abs(Wg[l, kv, h] - Wr))
+        assert errW <= rel * np.max(np.abs(Wr)), \
+            "W (%d,%d,%d): err %.3g > %.3g (kappa %.3g)" % (l, kv, h, errW, rel * np.max(np.abs(Wr)), kappa)
+        bscale = np.max(np.abs(br)) + np.max(np.abs(X.mean(axis=0))) * np.sum(np.abs(Wr), axis=0).max()
+        errb = np.max(np.abs(bg[l, kv, h] - br))
+        assert errb <= rel * bscale, "b (%d,%d,%d): err %.3g > %.3g" % (l, kv, h, errb, rel * bscale)
+
+
+@pytest.mark.parametrize("over,lam", [
+    (dict(Ls=4, Lt=3, H=2, B=2, T=300, k=2), 0.01),                 # B > 1, ragged tiles
+    (dict(Ls=5, Lt=2, H=2, B=1, T=700, k=3, theta_t=5e5), 1.0),     # different thetas, larger lambda
+    (dict(Ls=6, Lt=3, H=1, B=1, T=200, k=4), 0.01),                 # F = 512 > N: lambda keeps it SPD
+    (dict(Ls=3, Lt=2, H=2, B=1, T=64, k=1), 0.0),                   # no regularisation, N < F
+])
+def test_fit_small_every_system(over, lam):
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", **over)
+    sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
+    if lam == 0.0 and w.B * w.T <= w.k * w.d:
+        over = dict(over, T=4 * w.k * w.d)                            # keep it positive definite
+        w = syn.workload("qwen3_14b_32b_b8x1024_k4", **over)
+    caches, Wg, bg = _run_fit(w, lam, sel)
+    assert np.all(np.isfinite(Wg)) and np.all(np.isfinite(bg)), "unwritten outputs"
+    systems = [(l, kv, h) for l in range(w.Lt) for kv in range(2) for h in range(w.H)]
+    _check_systems(w, lam, sel, caches, Wg, bg, systems)
+
+
+def test_fit_headline_shapes_sampled():
+    """Qwen3-14B -> 32B layer and head counts, k = 4, 4096 calibration tokens: every system
+    fitted on the GPU, six of them checked against the oracle."""
+    w = syn.workload("qwen3_14b_32b_t32768_k4", T=4096)
+    sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
+    caches, Wg, bg = _run_fit(w, 0.01, sel)
+    assert np.all(np.isfinite(Wg)) and np.all(np.isfinite(bg))
+    systems = [(0, 0, 0), (0, 1, 7), (31, 0, 3), (40, 1, 5), (63, 0, 7), (63, 1, 0)]
+    _check_systems(w, 0.01, sel, caches, Wg, bg, systems)
