@@ -288,6 +288,64 @@ def make_mapper(w, dev_index):
     return kvx.kvx_create(cfg, dev_index)
 
 
+FP32_FFMA_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12   # SMs x FP32 lanes x 2 FLOP x max SM clock
+
+
+def fit_bench(args, w):
+    """Ridge fit of every (target layer, K|V, head) on N = B*T calibration tokens of the
+    workload's shapes.  One step = one kvx_fit_ridge call (mean, Gram and solve kernels,
+    synchronous).  Roofline: the Gram blocks' fp32 FFMA work against the FP32 peak derived
+    from the unit counts (152 SMs x 128 lanes x 2 x 2070 MHz); the fp64 solve is listed."""
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(0)
+    sp = torch.cuda.current_stream(dev).cuda_stream
+    sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+    tk, tv = syn.target_cache(w, 0, device=dev), syn.target_cache(w, 1, device=dev)
+    pos = torch.from_numpy(syn.positions(w)).to(dev)
+    sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
+    F = w.k * w.d
+    W = torch.empty((w.Lt, 2, w.H, F, w.d), dtype=torch.float32, device=dev)
+    b = torch.empty((w.Lt, 2, w.H, w.d), dtype=torch.float32, device=dev)
+    src, tgt = kvx.src_from_tensors(sk, sv), kvx.src_from_tensors(tk, tv)
+
+    def step():
+        kvx.kvx_fit_ridge(w.Ls, w.Lt, w.H, w.d, w.k, w.theta_s, w.theta_t, 0.01, sel, src, tgt, w.B, w.T,
+                          pos.data_ptr(), W.data_ptr(), b.data_ptr(), sp)
+
+    for _ in range(args.warmup):
+        step()
+    steps = max(1, min(args.steps, 20))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(0) as clk:
+        torch.cuda.synchronize()
+        e0.record()
+        for _ in range(steps):
+            step()
+        e1.record()
+        torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    n_sys = w.Lt * 2 * w.H
+    N = w.n_tokens
+    gram_flop = n_sys * (w.k * (w.k + 1) // 2 + w.k) * 2.0 * N * w.d * w.d
+    solve_flop = n_sys * (F ** 3 / 3.0 + 2.0 * F * F * w.d)
+    achieved = gram_flop / (ms / 1e3) / 1e12
+    line = {"metric": "ridge-fit calibration tokens/s", "value": N / (ms / 1e3), "unit": "tokens/s", "n_gpus": 1,
+            "steps": steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16 caches, fp32 Gram, fp64 solve",
+            "data": "synthetic",
+            "config": {"workload": w.name + " (fit)", "src_layers": w.Ls, "tgt_layers": w.Lt, "kv_heads": w.H,
+                       "head_dim": w.d, "k": w.k, "calibration_tokens": N, "systems": n_sys, "lambda": 0.01},
+            "clocks": clk.summary(),
+            "gpu_launches": 3 * steps,
+            "roofline": {"bound": "alu", "achieved": achieved, "peak": FP32_FFMA_PEAK_TFLOPS, "unit": "TFLOP/s",
+                         "frac": achieved / FP32_FFMA_PEAK_TFLOPS, "traffic": None,
+                         "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz",
+                         "algorithmic": {"gram_flop_per_step": gram_flop, "solve_fp64_flop_per_step": solve_flop}},
+            "kernel": "fit_mean_kernel + fit_gram_kernel + fit_solve_kernel"}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -297,9 +355,13 @@ def main():
     ap.add_argument("--workload", default=syn.HEADLINE)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=None)
+    ap.add_argument("--fit", action="store_true",
+                    help="time the ridge fit (kvx_fit_ridge) on the workload's shapes instead of the map")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     w = syn.workload(args.workload)
+    if args.fit:
+        return fit_bench(args, w)
     alg = algorithmic(w)
     config = {"workload": w.name, "src_layers": w.Ls, "tgt_layers": w.Lt, "kv_heads": w.H,
               "head_dim": w.d, "k": w.k, "batch": w.B, "seq_len": w.T, "tokens_per_step": w.n_tokens,
