@@ -326,7 +326,13 @@ def fit_bench(args, w):
     ms = e0.elapsed_time(e1) / steps
     n_sys = w.Lt * 2 * w.H
     N = w.n_tokens
-    gram_flop = n_sys * (w.k * (w.k + 1) // 2 + w.k) * 2.0 * N * w.d * w.d
+    # Source-pair blocks XsaᵀXsb depend only on the two source layers, so every distinct
+    # pair of the selection is one Gram block per (K|V, head); each target layer adds its
+    # k cross blocks XᵀY.  A block is N d² fused multiply-adds.
+    sel_np = np.asarray(sel).reshape(w.Lt, w.k)
+    pairs = {(max(int(a), int(c)), min(int(a), int(c))) for row in sel_np for i, a in enumerate(row) for c in row[:i + 1]}
+    gram_flop = 2 * w.H * (len(pairs) + w.Lt * w.k) * 2.0 * N * w.d * w.d
+    gram_flop_unshared = n_sys * (w.k * (w.k + 1) // 2 + w.k) * 2.0 * N * w.d * w.d
     solve_flop = n_sys * (F ** 3 / 3.0 + 2.0 * F * F * w.d)
     achieved = gram_flop / (ms / 1e3) / 1e12
     line = {"metric": "ridge-fit calibration tokens/s", "value": N / (ms / 1e3), "unit": "tokens/s", "n_gpus": 1,
@@ -340,7 +346,9 @@ def fit_bench(args, w):
             "roofline": {"bound": "alu", "achieved": achieved, "peak": FP32_FFMA_PEAK_TFLOPS, "unit": "TFLOP/s",
                          "frac": achieved / FP32_FFMA_PEAK_TFLOPS, "traffic": None,
                          "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz",
-                         "algorithmic": {"gram_flop_per_step": gram_flop, "solve_fp64_flop_per_step": solve_flop}},
+                         "algorithmic": {"gram_flop_per_step": gram_flop, "gram_blocks_source_pairs": len(pairs),
+                                         "gram_flop_without_pair_sharing": gram_flop_unshared,
+                                         "solve_fp64_flop_per_step": solve_flop}},
             "kernel": "fit_mean_kernel + fit_gram_kernel + fit_solve_kernel"}
     print(json.dumps(line), flush=True)
     return 0

@@ -12,8 +12,9 @@
 // 1. fit_mean_kernel: fp64 column sums of every (side, K|V, layer, head) over the tokens;
 //    a thread owns one RoPE pair (channels i and i + 64) of one row and a chunk of tokens,
 //    strips the rotation in fp32 and adds into fp64 with one atomic per chunk.
-// 2. fit_gram_kernel: one CTA per 128 x 128 block of Xc^T Xc (lower triangle of the
-//    k x k block grid) or of Xc^T Yc; the token loop stages 32-token tiles of both
+// 2. fit_gram_kernel: one CTA per 128 x 128 block: a (source layer, source layer) block of
+//    Xc^T Xc, computed once for every target layer whose selection holds both layers, or
+//    a (source layer, target layer) block of Xc^T Yc; the token loop stages 32-token tiles of both
 //    operands in shared memory already stripped and centred (fp32), and 256 threads each
 //    accumulate an 8 x 8 register tile with FFMA.  fp32 accumulation of centred values.
 // 3. fit_solve_kernel: one CTA per system at a time (persistent); the block grid is
@@ -29,6 +30,7 @@
 #include <climits>
 #include <cmath>
 #include <string>
+#include <vector>
 
 #include "kvx_internal.h"
 #include "kvx_ptx.cuh"
@@ -59,7 +61,10 @@ struct FitParams {
   int32_t Ls, Lt, H, k, B, T;
   RopeTables rope;
   double* sums;                     // [2 sides][2 kv][L][H][128]: side 0 L = L_s, side 1 L = L_t
-  float* gram;                      // [L_t][2][H][k*k blocks][128][128]  (lower blocks used)
+  float* gram;                      // [2][H][n_pairs][128][128]: source-pair blocks
+  const int32_t* pairs;             // [n_pairs][2] source layers (sa >= sb)
+  const int32_t* pair_of;           // [L_t][k][k] pair of block (bi, bj), bi >= bj
+  int32_t n_pairs;
   float* xty;                       // [L_t][2][H][k][128][128]
   double* scratch;                  // per CTA: F x F matrix + F x 128 right-hand sides
   float* W;                         // [L_t][2][H][F][128]
@@ -129,9 +134,9 @@ __global__ void __launch_bounds__(kFPairs) fit_mean_kernel(const __grid_constant
 }
 
 // ------------------------------------------------------------- Gram blocks --
-// grid: (k(k+1)/2 + k blocks, L_t * 2 * H systems), 256 threads, 32 KB shared memory.
-// Block index q < k(k+1)/2: the (bi, bj) block of Xc^T Xc with bi >= bj (row-major over
-// the lower triangle); q >= k(k+1)/2: block bi = q - k(k+1)/2 of Xc^T Yc.
+// grid: (n_pairs + L_t k, 2 H), 256 threads, 33 KB shared memory.  x < n_pairs: the
+// source-pair block (pairs[x][0], pairs[x][1]) of Xc^T Xc; otherwise the block (l, bi) of
+// Xc^T Yc, x - n_pairs = l k + bi.
 struct Operand {
   const FitCache* c;
   int side, layer;
@@ -175,22 +180,12 @@ __global__ void __launch_bounds__(256) fit_gram_kernel(const __grid_constant__ F
   __shared__ __align__(16) float ta[kGTok * kFD];
   __shared__ __align__(16) float tb[kGTok * kFD];
   __shared__ float mean_a[kFD], mean_b[kFD];
-  const int sys = blockIdx.y;                     // ((l * 2 + kv) * H + h)
-  const int h = sys % P.H;
-  const int kv = (sys / P.H) & 1;
-  const int l = sys / (2 * P.H);
-  const int ntri = P.k * (P.k + 1) / 2;
+  const int kv = blockIdx.y / P.H, h = blockIdx.y % P.H;
   const int q = blockIdx.x;
-  int bi, bj = -1;
-  if (q < ntri) {                                 // lower-triangle block (bi, bj), bj <= bi
-    bi = 0;
-    while ((bi + 1) * (bi + 2) / 2 <= q) ++bi;
-    bj = q - bi * (bi + 1) / 2;
-  } else {
-    bi = q - ntri;
-  }
-  const Operand oa{&P.src, 0, __ldg(&P.sel[l * P.k + bi])};
-  const Operand ob = bj >= 0 ? Operand{&P.src, 0, __ldg(&P.sel[l * P.k + bj])} : Operand{&P.tgt, 1, l};
+  const bool is_pair = q < P.n_pairs;
+  const int l = is_pair ? 0 : (q - P.n_pairs) / P.k, bi = is_pair ? 0 : (q - P.n_pairs) % P.k;
+  const Operand oa{&P.src, 0, is_pair ? __ldg(&P.pairs[2 * q]) : __ldg(&P.sel[l * P.k + bi])};
+  const Operand ob = is_pair ? Operand{&P.src, 0, __ldg(&P.pairs[2 * q + 1])} : Operand{&P.tgt, 1, l};
   const int64_t N = static_cast<int64_t>(P.B) * P.T;
   const double inv_n = 1.0 / static_cast<double>(N);
   if (threadIdx.x < kFD) {
@@ -223,8 +218,8 @@ __global__ void __launch_bounds__(256) fit_gram_kernel(const __grid_constant__ F
     }
     __syncthreads();
   }
-  float* out = bj >= 0 ? P.gram + ((static_cast<size_t>(sys) * P.k + bi) * P.k + bj) * kFD * kFD
-                       : P.xty + (static_cast<size_t>(sys) * P.k + bi) * kFD * kFD;
+  float* out = is_pair ? P.gram + ((static_cast<size_t>(kv) * P.H + h) * P.n_pairs + q) * kFD * kFD
+                       : P.xty + (((static_cast<size_t>(l) * 2 + kv) * P.H + h) * P.k + bi) * kFD * kFD;
 #pragma unroll
   for (int x = 0; x < 8; ++x) {
     float4* o = reinterpret_cast<float4*>(out + static_cast<size_t>(8 * ty + x) * kFD + 8 * tx);
@@ -257,8 +252,10 @@ __global__ void __launch_bounds__(256) fit_solve_kernel(const __grid_constant__ 
       const int r = static_cast<int>(e / F), c = static_cast<int>(e % F);
       if (c > r) continue;
       const int bi = r / kFD, bj = c / kFD;
-      const float g = P.gram[((static_cast<size_t>(sys) * P.k + bi) * P.k + bj) * kFD * kFD +
-                             static_cast<size_t>(r % kFD) * kFD + (c % kFD)];
+      const int pr = __ldg(&P.pair_of[(l * P.k + bi) * P.k + bj]);   // < 0: stored transposed
+      const size_t blk = ((static_cast<size_t>(kv) * P.H + h) * P.n_pairs + (pr >= 0 ? pr : -1 - pr)) * kFD * kFD;
+      const float g = pr >= 0 ? P.gram[blk + static_cast<size_t>(r % kFD) * kFD + (c % kFD)]
+                              : P.gram[blk + static_cast<size_t>(c % kFD) * kFD + (r % kFD)];
       A[e] = static_cast<double>(g) + (r == c ? P.lambda : 0.0);
     }
     for (int64_t e = tid; e < static_cast<int64_t>(F) * kFD; e += blockDim.x) {
@@ -437,12 +434,40 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
   const size_t n_sys = static_cast<size_t>(cfg->tgt_layers) * 2 * cfg->n_kv_heads;
   const int Lmax = std::max(cfg->src_layers, cfg->tgt_layers);
   const size_t sums_n = static_cast<size_t>(2) * (cfg->src_layers + cfg->tgt_layers) * cfg->n_kv_heads * kFD;
-  const size_t gram_n = n_sys * cfg->k * cfg->k * kFD * kFD;
+  // the distinct (source layer, source layer) blocks of all target layers' Xc^T Xc
+  const int kk = cfg->k;
+  std::vector<int32_t> pair_list, pair_of(static_cast<size_t>(cfg->tgt_layers) * kk * kk, -1);
+  {
+    std::vector<int32_t> index(static_cast<size_t>(cfg->src_layers) * cfg->src_layers, -1);
+    for (int l = 0; l < cfg->tgt_layers; ++l)
+      for (int bi = 0; bi < kk; ++bi)
+        for (int bj = 0; bj <= bi; ++bj) {
+          int sa = cfg->selection[l * kk + bi], sb = cfg->selection[l * kk + bj];
+          int ia = bi, ib = bj;
+          if (sa < sb) {   // keep the block's rows on the larger layer; transpose in the solve
+            std::swap(sa, sb);
+            std::swap(ia, ib);
+          }
+          int32_t& idx = index[static_cast<size_t>(sa) * cfg->src_layers + sb];
+          if (idx < 0) {
+            idx = static_cast<int32_t>(pair_list.size() / 2);
+            pair_list.push_back(sa);
+            pair_list.push_back(sb);
+          }
+          pair_of[(static_cast<size_t>(l) * kk + bi) * kk + bj] = ia == bi ? idx : -1 - idx;
+        }
+  }
+  const int n_pairs = static_cast<int>(pair_list.size() / 2);
+  P.n_pairs = n_pairs;
+  const size_t gram_n = static_cast<size_t>(2) * cfg->n_kv_heads * n_pairs * kFD * kFD;
   const size_t xty_n = n_sys * cfg->k * kFD * kFD;
   const int solve_grid = static_cast<int>(std::min<size_t>(n_sys, static_cast<size_t>(sms)));
   const size_t scratch_n = static_cast<size_t>(solve_grid) * (static_cast<size_t>(F) * F + static_cast<size_t>(F) * kFD);
   const size_t sel_n = static_cast<size_t>(cfg->tgt_layers) * cfg->k;
-  const size_t bytes = sums_n * 8 + scratch_n * 8 + (gram_n + xty_n) * 4 + sel_n * 4 + 16;
+  std::vector<int32_t> tab(cfg->selection, cfg->selection + sel_n);
+  tab.insert(tab.end(), pair_list.begin(), pair_list.end());
+  tab.insert(tab.end(), pair_of.begin(), pair_of.end());
+  const size_t bytes = sums_n * 8 + scratch_n * 8 + (gram_n + xty_n) * 4 + tab.size() * 4 + 16;
   char* ws = nullptr;
   if ((e = cudaMallocAsync(reinterpret_cast<void**>(&ws), bytes, st)) != cudaSuccess) {
     set_error(std::string("kvx_fit_ridge: workspace: ") + cudaGetErrorString(e));
@@ -454,12 +479,14 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
   P.xty = P.gram + gram_n;
   int32_t* dsel = reinterpret_cast<int32_t*>(P.xty + xty_n);
   P.sel = dsel;
-  P.status = dsel + sel_n;
+  P.pairs = dsel + sel_n;
+  P.pair_of = P.pairs + pair_list.size();
+  P.status = dsel + tab.size();
   kvx_status result = KVX_OK;
   do {
     if ((e = cudaMemsetAsync(P.sums, 0, sums_n * 8, st)) != cudaSuccess ||
         (e = cudaMemsetAsync(P.status, 0, 4, st)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(dsel, cfg->selection, sel_n * 4, cudaMemcpyHostToDevice, st)) != cudaSuccess) {
+        (e = cudaMemcpyAsync(dsel, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice, st)) != cudaSuccess) {
       set_error(std::string("kvx_fit_ridge: setup: ") + cudaGetErrorString(e));
       result = KVX_ERR_CUDA;
       break;
@@ -467,7 +494,7 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
     const int64_t N = static_cast<int64_t>(batch) * tokens_per_seq;
     const dim3 mgrid(static_cast<unsigned>((N + kFChunk - 1) / kFChunk), static_cast<unsigned>(4 * Lmax * cfg->n_kv_heads));
     fit_mean_kernel<<<mgrid, kFPairs, 0, st>>>(P, Lmax);
-    const dim3 ggrid(static_cast<unsigned>(cfg->k * (cfg->k + 1) / 2 + cfg->k), static_cast<unsigned>(n_sys));
+    const dim3 ggrid(static_cast<unsigned>(n_pairs + cfg->tgt_layers * kk), static_cast<unsigned>(2 * cfg->n_kv_heads));
     fit_gram_kernel<<<ggrid, 256, 0, st>>>(P);
     const size_t smem = static_cast<size_t>(kNB) * kNB * 8 + static_cast<size_t>(F - kNB) * kNB * 8;
     if ((e = cudaFuncSetAttribute(fit_solve_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem))) !=
