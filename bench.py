@@ -288,7 +288,9 @@ def make_mapper(w, dev_index):
     return kvx.kvx_create(cfg, dev_index)
 
 
-FP32_FFMA_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12   # SMs x FP32 lanes x 2 FLOP x max SM clock
+
+
+FP64_PEAK_TFLOPS = 1.25    # nominal GB300 FP64 rate
 
 
 def fit_bench(args, w):
@@ -316,14 +318,17 @@ def fit_bench(args, w):
         step()
     steps = max(1, min(args.steps, 20))
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    phase = [0.0] * 4
     with ClockSampler(0) as clk:
         torch.cuda.synchronize()
         e0.record()
         for _ in range(steps):
             step()
+            phase = [a + b for a, b in zip(phase, kvx.kvx_last_phase_ms())]
         e1.record()
         torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / steps
+    phase = [p / steps for p in phase]
     n_sys = w.Lt * 2 * w.H
     N = w.n_tokens
     # Source-pair blocks XsaᵀXsb depend only on the two source layers, so every distinct
@@ -334,22 +339,31 @@ def fit_bench(args, w):
     gram_flop = 2 * w.H * (len(pairs) + w.Lt * w.k) * 2.0 * N * w.d * w.d
     gram_flop_unshared = n_sys * (w.k * (w.k + 1) // 2 + w.k) * 2.0 * N * w.d * w.d
     solve_flop = n_sys * (F ** 3 / 3.0 + 2.0 * F * F * w.d)
-    achieved = gram_flop / (ms / 1e3) / 1e12
+    # dominant kernel: the fp64 solve (Cholesky + two triangular solves per system)
+    achieved = solve_flop / (phase[3] / 1e3) / 1e12
+    # the Gram kernel issues four bf16 MMAs per product (hi/lo split of both operands)
+    gram_tc_tflops = 4.0 * gram_flop / (phase[2] / 1e3) / 1e12
+    pk = load_peaks()
     line = {"metric": "ridge-fit calibration tokens/s", "value": N / (ms / 1e3), "unit": "tokens/s", "n_gpus": 1,
             "steps": steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "bf16 caches, fp32 Gram, fp64 solve",
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16 caches, bf16x2-split tensor-core Gram (fp32 accumulate), fp64 solve",
             "data": "synthetic",
             "config": {"workload": w.name + " (fit)", "src_layers": w.Ls, "tgt_layers": w.Lt, "kv_heads": w.H,
                        "head_dim": w.d, "k": w.k, "calibration_tokens": N, "systems": n_sys, "lambda": 0.01},
             "clocks": clk.summary(),
-            "gpu_launches": 3 * steps,
-            "roofline": {"bound": "alu", "achieved": achieved, "peak": FP32_FFMA_PEAK_TFLOPS, "unit": "TFLOP/s",
-                         "frac": achieved / FP32_FFMA_PEAK_TFLOPS, "traffic": None,
-                         "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz",
-                         "algorithmic": {"gram_flop_per_step": gram_flop, "gram_blocks_source_pairs": len(pairs),
-                                         "gram_flop_without_pair_sharing": gram_flop_unshared,
-                                         "solve_fp64_flop_per_step": solve_flop}},
-            "kernel": "fit_mean_kernel + fit_gram_kernel + fit_solve_kernel"}
+            "gpu_launches": 4 * steps,
+            "phase_ms": {"column_sums": phase[0], "pack": phase[1], "gram_tc": phase[2], "solve": phase[3]},
+            "roofline": {"bound": "alu", "achieved": achieved, "peak": FP64_PEAK_TFLOPS, "unit": "TFLOP/s",
+                         "frac": achieved / FP64_PEAK_TFLOPS, "traffic": None,
+                         "kernel": "fit_solve_kernel",
+                         "peak_source": "nominal GB300 FP64 rate (not measured; no FP64 tensor path)",
+                         "algorithmic": {"solve_fp64_flop_per_step": solve_flop, "gram_flop_per_step": gram_flop,
+                                         "gram_blocks_source_pairs": len(pairs),
+                                         "gram_flop_without_pair_sharing": gram_flop_unshared},
+                         "other": {"gram_tc_kernel": {"bound": "tensor", "achieved": gram_tc_tflops,
+                                                      "peak": pk["bf16"], "frac": gram_tc_tflops / pk["bf16"],
+                                                      "unit": "TFLOP/s (bf16 MMA, four per product)"}}},
+            "kernel": "gram_pack_kernel<0> + gram_pack_kernel<1> + gram_tc_kernel + fit_solve_kernel"}
     print(json.dumps(line), flush=True)
     return 0
 

@@ -189,12 +189,16 @@ KVX_API int64_t kvx_mapper_params(int32_t tgt_layers, int32_t n_kv_heads, int32_
  * [L_t][B][H][T][d] of the same tokens (kvx_src layout, bf16, d = 128, 16-byte aligned);
  * `positions` device [batch][tokens_per_seq].  `selection` (host [L_t][k], 1 <= k <= 4)
  * as in kvx_config.  Outputs on the device, fp32: W [L_t][2][H][k*d][d] and
- * b [L_t][2][H][d] (the kvx_config layouts).  Cross-products accumulate in fp32 on
- * centred values; the factorisation and the solves run in fp64.  Runs on `stream` and
- * synchronises it before returning (an offline step; it allocates stream-ordered
- * workspace of about L_t*2*H*(k*k + k)*64 KB plus 8 MB per SM).  INVALID_ARG for bad
- * arguments or when a system is not positive definite (lambda = 0 with too few tokens);
- * DEVICE_BOUNDS when a position is outside [0, 2^24). */
+ * b [L_t][2][H][d] (the kvx_config layouts).  Cross-products of the centred values run
+ * on the tensor cores from a bf16 hi + lo split of each value (within 2^-17 of it) and
+ * accumulate in fp32; the factorisation and the solves run in fp64.  Runs on `stream` and
+ * synchronises it before returning (an offline step).  Stream-ordered workspace: the
+ * blocks (at most L_t*2*H*(k*(k+1)/2 + k)*64 KB), 8 MB per SM, and the packed operands
+ * (4 bytes per token, channel, K|V, head and used layer of either model), at most half the
+ * free device memory or 32 GB, the tokens taken in chunks beyond that.  INVALID_ARG for
+ * bad arguments or when a system is not positive definite (lambda = 0 with too few
+ * tokens); DEVICE_BOUNDS when a position is outside [0, 2^24); OOM when the workspace
+ * cannot be allocated. */
 typedef struct {
   int32_t src_layers, tgt_layers, n_kv_heads, head_dim, k;
   double src_rope_theta, tgt_rope_theta;
@@ -204,6 +208,12 @@ typedef struct {
 KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, const kvx_src* tgt, int32_t batch,
                                  int32_t tokens_per_seq, const int32_t* positions, float* W, float* b,
                                  void* stream);
+
+/* Device time in milliseconds of the phases of the last successful kvx_fit_ridge or
+ * kvx_r2_probe call on this thread, from CUDA events on the call's stream: ms[0] column
+ * sums, ms[1] operand packing, ms[2] tensor-core Gram blocks, ms[3] the solves (fit) or
+ * the scores (probe).  `ms` host float[4].  INVALID_ARG if ms is NULL. */
+KVX_API kvx_status kvx_last_phase_ms(float* ms);
 
 /* Static description of a status code. */
 KVX_API const char* kvx_status_string(kvx_status s);

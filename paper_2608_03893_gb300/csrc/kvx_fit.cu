@@ -8,16 +8,12 @@
 //   W = (Xc^T Xc + lambda I)^{-1} Xc^T Yc,   b = mean(Y) - mean(X) W.
 // bf16 caches, head_dim 128, half-split pairs.
 //
-// Three kernels, all in this file:
-// 1. fit_mean_kernel: fp64 column sums of every (side, K|V, layer, head) over the tokens;
-//    a thread owns one RoPE pair (channels i and i + 64) of one row and a chunk of tokens,
-//    strips the rotation in fp32 and adds into fp64 with one atomic per chunk.
-// 2. fit_gram_kernel: one CTA per 128 x 128 block: a (source layer, source layer) block of
-//    Xc^T Xc, computed once for every target layer whose selection holds both layers, or
-//    a (source layer, target layer) block of Xc^T Yc; the token loop stages 32-token tiles of both
-//    operands in shared memory already stripped and centred (fp32), and 256 threads each
-//    accumulate an 8 x 8 register tile with FFMA.  fp32 accumulation of centred values.
-// 3. fit_solve_kernel: one CTA per system at a time (persistent); the block grid is
+// Steps:
+// 1. Column sums and the centred Gram blocks on the tensor cores (kvx_gram.cu): a block
+//    (source layer, source layer) of Xc^T Xc depends only on the two layers, K|V and the
+//    head, so every distinct pair of the selection is computed once and shared by all
+//    target layers whose selection holds both; the k blocks of Xc^T Yc are per target layer.
+// 2. fit_solve_kernel: one CTA per system at a time (persistent); the block grid is
 //    widened to fp64 into a per-CTA scratch matrix, lambda added, factorised by a blocked
 //    right-looking Cholesky (32-column panels: diagonal block in shared memory, panel by
 //    forward substitution, trailing update), then the two triangular solves for the d
@@ -34,7 +30,6 @@
 
 #include "kvx_internal.h"
 #include "kvx_ptx.cuh"
-#include "kvx_rope.cuh"
 
 namespace kvx {
 namespace {
@@ -42,24 +37,11 @@ namespace {
 using namespace ptx;
 
 constexpr int kFD = 128;            // head_dim
-constexpr int kFPairs = kFD / 2;    // RoPE pairs per head
-constexpr int kFChunk = 1024;       // tokens per block of the mean kernel
-constexpr int kGTok = 32;           // tokens per stage of the Gram kernel
 constexpr int kNB = 32;             // Cholesky panel width
 
-// Where one operand row lives: side 0 = source (selected layers), 1 = target.
-struct FitCache {
-  const __nv_bfloat16* k;
-  const __nv_bfloat16* v;
-  int64_t s[4];                     // strides (layer, batch, head, token), elements
-};
-
 struct FitParams {
-  FitCache src, tgt;
-  const int32_t* pos;               // [B][T]
   const int32_t* sel;               // [L_t][k]
   int32_t Ls, Lt, H, k, B, T;
-  RopeTables rope;
   double* sums;                     // [2 sides][2 kv][L][H][128]: side 0 L = L_s, side 1 L = L_t
   float* gram;                      // [2][H][n_pairs][128][128]: source-pair blocks
   const int32_t* pairs;             // [n_pairs][2] source layers (sa >= sb)
@@ -79,154 +61,7 @@ __device__ __forceinline__ size_t sums_index(const FitParams& P, int side, int k
   return base + ((static_cast<size_t>(kv) * L + layer) * P.H + h) * kFD;
 }
 
-// Token n (0 .. B*T-1) of row (layer, head) of one cache, RoPE pair i: the pair's two
-// channels as stored, and the position of the token.
-__device__ __forceinline__ const __nv_bfloat16* row_ptr(const FitCache& c, int kv, int layer, int h, int b, int t) {
-  return (kv ? c.v : c.k) + layer * c.s[0] + b * c.s[1] + h * c.s[2] + static_cast<int64_t>(t) * c.s[3];
-}
-
 __device__ __forceinline__ void report_fit(int32_t* status, int code) { atomicCAS(status, 0, code); }
-
-// Keys: the stored pair (a, b) rotated by -t omega_i (strip); values unchanged.
-__device__ __forceinline__ void strip_pair(float a, float b, float c, float s, float* ra, float* rb) {
-  *ra = __fmaf_rn(a, c, __fmul_rn(b, s));
-  *rb = __fmaf_rn(b, c, -__fmul_rn(a, s));
-}
-
-// --------------------------------------------------------------- column sums --
-// grid: (token chunks, rows), row = ((side * 2 + kv) * Lmax + layer) * H + h; 64 threads.
-__global__ void __launch_bounds__(kFPairs) fit_mean_kernel(const __grid_constant__ FitParams P, int Lmax) {
-  const int row = blockIdx.y;
-  const int h = row % P.H;
-  const int rest = row / P.H;
-  const int layer = rest % Lmax;
-  const int sk = rest / Lmax;            // side * 2 + kv
-  const int side = sk >> 1, kv = sk & 1;
-  if (layer >= (side == 0 ? P.Ls : P.Lt)) return;
-  const FitCache& c = side == 0 ? P.src : P.tgt;
-  const int i = threadIdx.x;             // pair: channels i and i + 64
-  const float* w_hi = side == 0 ? P.rope.ws_hi : P.rope.wt_hi;
-  const float* w_lo = side == 0 ? P.rope.ws_lo : P.rope.wt_lo;
-  const int64_t N = static_cast<int64_t>(P.B) * P.T;
-  const int64_t n0 = static_cast<int64_t>(blockIdx.x) * kFChunk;
-  const int64_t n1 = min(N, n0 + kFChunk);
-  double sa = 0.0, sb = 0.0;
-  for (int64_t n = n0; n < n1; ++n) {
-    const int b = static_cast<int>(n / P.T), t = static_cast<int>(n % P.T);
-    const __nv_bfloat16* r = row_ptr(c, kv, layer, h, b, t);
-    float a = __bfloat162float(r[i]), bb = __bfloat162float(r[i + kFPairs]);
-    if (kv == 0) {
-      int p = __ldg(&P.pos[n]);
-      if (p < 0 || p >= (1 << 24)) {
-        report_fit(P.status, KVX_ERR_DEVICE_BOUNDS);
-        p = 0;
-      }
-      float s, cs;
-      rope_sincos(p, w_hi[i], w_lo[i], P.rope.two_pi_hi, P.rope.two_pi_lo, P.rope.inv_two_pi, &s, &cs);
-      strip_pair(a, bb, cs, s, &a, &bb);
-    }
-    sa += a;
-    sb += bb;
-  }
-  double* out = P.sums + sums_index(P, side, kv, layer, h);
-  atomicAdd(&out[i], sa);
-  atomicAdd(&out[i + kFPairs], sb);
-}
-
-// ------------------------------------------------------------- Gram blocks --
-// grid: (n_pairs + L_t k, 2 H), 256 threads, 33 KB shared memory.  x < n_pairs: the
-// source-pair block (pairs[x][0], pairs[x][1]) of Xc^T Xc; otherwise the block (l, bi) of
-// Xc^T Yc, x - n_pairs = l k + bi.
-struct Operand {
-  const FitCache* c;
-  int side, layer;
-};
-
-// Stage tokens n0 .. n0+31 of one operand (head h, K|V kv) into dst[32][128] as fp32,
-// keys stripped, centred by `mean` (fp32 [128]); rows past N are zero.
-__device__ __forceinline__ void stage_tile(const FitParams& P, const Operand& o, int kv, int h, int64_t n0,
-                                           const float* mean, float* dst) {
-  const int i = threadIdx.x & (kFPairs - 1);      // pair
-  const int t0 = threadIdx.x >> 6;                // 0..3
-  const int64_t N = static_cast<int64_t>(P.B) * P.T;
-  const float* w_hi = o.side == 0 ? P.rope.ws_hi : P.rope.wt_hi;
-  const float* w_lo = o.side == 0 ? P.rope.ws_lo : P.rope.wt_lo;
-#pragma unroll 2
-  for (int m = 0; m < kGTok / 4; ++m) {
-    const int tt = t0 + 4 * m;
-    const int64_t n = n0 + tt;
-    float a = 0.f, bb = 0.f;
-    if (n < N) {
-      const int b = static_cast<int>(n / P.T), t = static_cast<int>(n % P.T);
-      const __nv_bfloat16* r = row_ptr(*o.c, kv, o.layer, h, b, t);
-      a = __bfloat162float(r[i]);
-      bb = __bfloat162float(r[i + kFPairs]);
-      if (kv == 0) {
-        int p = __ldg(&P.pos[n]);
-        if (p < 0 || p >= (1 << 24)) p = 0;       // reported by the mean kernel
-        float s, cs;
-        rope_sincos(p, w_hi[i], w_lo[i], P.rope.two_pi_hi, P.rope.two_pi_lo, P.rope.inv_two_pi, &s, &cs);
-        strip_pair(a, bb, cs, s, &a, &bb);
-      }
-      a -= mean[i];
-      bb -= mean[i + kFPairs];
-    }
-    dst[tt * kFD + i] = a;
-    dst[tt * kFD + i + kFPairs] = bb;
-  }
-}
-
-__global__ void __launch_bounds__(256) fit_gram_kernel(const __grid_constant__ FitParams P) {
-  __shared__ __align__(16) float ta[kGTok * kFD];
-  __shared__ __align__(16) float tb[kGTok * kFD];
-  __shared__ float mean_a[kFD], mean_b[kFD];
-  const int kv = blockIdx.y / P.H, h = blockIdx.y % P.H;
-  const int q = blockIdx.x;
-  const bool is_pair = q < P.n_pairs;
-  const int l = is_pair ? 0 : (q - P.n_pairs) / P.k, bi = is_pair ? 0 : (q - P.n_pairs) % P.k;
-  const Operand oa{&P.src, 0, is_pair ? __ldg(&P.pairs[2 * q]) : __ldg(&P.sel[l * P.k + bi])};
-  const Operand ob = is_pair ? Operand{&P.src, 0, __ldg(&P.pairs[2 * q + 1])} : Operand{&P.tgt, 1, l};
-  const int64_t N = static_cast<int64_t>(P.B) * P.T;
-  const double inv_n = 1.0 / static_cast<double>(N);
-  if (threadIdx.x < kFD) {
-    mean_a[threadIdx.x] = static_cast<float>(P.sums[sums_index(P, 0, kv, oa.layer, h) + threadIdx.x] * inv_n);
-    mean_b[threadIdx.x] = static_cast<float>(P.sums[sums_index(P, ob.side, kv, ob.layer, h) + threadIdx.x] * inv_n);
-  }
-  __syncthreads();
-  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;   // output rows 8ty.., columns 8tx..
-  float acc[8][8];
-#pragma unroll
-  for (int x = 0; x < 8; ++x)
-#pragma unroll
-    for (int y = 0; y < 8; ++y) acc[x][y] = 0.f;
-  for (int64_t n0 = 0; n0 < N; n0 += kGTok) {
-    stage_tile(P, oa, kv, h, n0, mean_a, ta);
-    stage_tile(P, ob, kv, h, n0, mean_b, tb);
-    __syncthreads();
-#pragma unroll 4
-    for (int t = 0; t < kGTok; ++t) {
-      const float4 a0 = *reinterpret_cast<const float4*>(&ta[t * kFD + 8 * ty]);
-      const float4 a1 = *reinterpret_cast<const float4*>(&ta[t * kFD + 8 * ty + 4]);
-      const float4 b0 = *reinterpret_cast<const float4*>(&tb[t * kFD + 8 * tx]);
-      const float4 b1 = *reinterpret_cast<const float4*>(&tb[t * kFD + 8 * tx + 4]);
-      const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-      const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
-#pragma unroll
-      for (int x = 0; x < 8; ++x)
-#pragma unroll
-        for (int y = 0; y < 8; ++y) acc[x][y] = __fmaf_rn(av[x], bv[y], acc[x][y]);
-    }
-    __syncthreads();
-  }
-  float* out = is_pair ? P.gram + ((static_cast<size_t>(kv) * P.H + h) * P.n_pairs + q) * kFD * kFD
-                       : P.xty + (((static_cast<size_t>(l) * 2 + kv) * P.H + h) * P.k + bi) * kFD * kFD;
-#pragma unroll
-  for (int x = 0; x < 8; ++x) {
-    float4* o = reinterpret_cast<float4*>(out + static_cast<size_t>(8 * ty + x) * kFD + 8 * tx);
-    o[0] = make_float4(acc[x][0], acc[x][1], acc[x][2], acc[x][3]);
-    o[1] = make_float4(acc[x][4], acc[x][5], acc[x][6], acc[x][7]);
-  }
-}
 
 // ------------------------------------------------------------------- solve --
 // Persistent: CTA c handles systems c, c + gridDim.x, ...  F = 128 k (k <= 4).  Dynamic
@@ -414,25 +249,29 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
   fill_rope(&tmp);
 
   FitParams P{};
-  P.src = FitCache{static_cast<const __nv_bfloat16*>(src->k), static_cast<const __nv_bfloat16*>(src->v),
-                   {src->stride[0], src->stride[1], src->stride[2], src->stride[3]}};
-  P.tgt = FitCache{static_cast<const __nv_bfloat16*>(tgt->k), static_cast<const __nv_bfloat16*>(tgt->v),
-                   {tgt->stride[0], tgt->stride[1], tgt->stride[2], tgt->stride[3]}};
-  P.pos = positions;
+  GramSpec G;
+  G.cache[0] = GramCache{src->k, src->v, {src->stride[0], src->stride[1], src->stride[2], src->stride[3]}};
+  G.cache[1] = GramCache{tgt->k, tgt->v, {tgt->stride[0], tgt->stride[1], tgt->stride[2], tgt->stride[3]}};
+  G.pos = positions;
+  G.B = batch;
+  G.T = tokens_per_seq;
+  G.H = cfg->n_kv_heads;
+  G.Ls = cfg->src_layers;
+  G.Lt = cfg->tgt_layers;
+  G.rope = tmp.rope;
+  G.sm_count = sms;
   P.Ls = cfg->src_layers;
   P.Lt = cfg->tgt_layers;
   P.H = cfg->n_kv_heads;
   P.k = cfg->k;
   P.B = batch;
   P.T = tokens_per_seq;
-  P.rope = tmp.rope;
   P.W = W;
   P.b = b;
   P.lambda = cfg->lambda;
 
   const int F = cfg->k * kFD;
   const size_t n_sys = static_cast<size_t>(cfg->tgt_layers) * 2 * cfg->n_kv_heads;
-  const int Lmax = std::max(cfg->src_layers, cfg->tgt_layers);
   const size_t sums_n = static_cast<size_t>(2) * (cfg->src_layers + cfg->tgt_layers) * cfg->n_kv_heads * kFD;
   // the distinct (source layer, source layer) blocks of all target layers' Xc^T Xc
   const int kk = cfg->k;
@@ -483,6 +322,7 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
   P.pair_of = P.pairs + pair_list.size();
   P.status = dsel + tab.size();
   kvx_status result = KVX_OK;
+  PhaseTimer timer(st);
   do {
     if ((e = cudaMemsetAsync(P.sums, 0, sums_n * 8, st)) != cudaSuccess ||
         (e = cudaMemsetAsync(P.status, 0, 4, st)) != cudaSuccess ||
@@ -491,11 +331,46 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
       result = KVX_ERR_CUDA;
       break;
     }
-    const int64_t N = static_cast<int64_t>(batch) * tokens_per_seq;
-    const dim3 mgrid(static_cast<unsigned>((N + kFChunk - 1) / kFChunk), static_cast<unsigned>(4 * Lmax * cfg->n_kv_heads));
-    fit_mean_kernel<<<mgrid, kFPairs, 0, st>>>(P, Lmax);
-    const dim3 ggrid(static_cast<unsigned>(n_pairs + cfg->tgt_layers * kk), static_cast<unsigned>(2 * cfg->n_kv_heads));
-    fit_gram_kernel<<<ggrid, 256, 0, st>>>(P);
+    // operands: the selected source layers, then every target layer
+    std::vector<int32_t> slot_of_src(cfg->src_layers, -1);
+    for (size_t i = 0; i < sel_n; ++i) slot_of_src[cfg->selection[i]] = 0;
+    for (int L = 0; L < cfg->src_layers; ++L)
+      if (slot_of_src[L] == 0) {
+        slot_of_src[L] = static_cast<int32_t>(G.slot_side.size());
+        G.slot_side.push_back(0);
+        G.slot_layer.push_back(L);
+      }
+    const int32_t tslot0 = static_cast<int32_t>(G.slot_side.size());
+    for (int l = 0; l < cfg->tgt_layers; ++l) {
+      G.slot_side.push_back(1);
+      G.slot_layer.push_back(l);
+    }
+    G.sums = P.sums;
+    G.status = P.status;
+    std::vector<GramBlock> blocks;
+    blocks.reserve(static_cast<size_t>(2) * cfg->n_kv_heads * (n_pairs + sel_n));
+    for (int kv = 0; kv < 2; ++kv)
+      for (int h = 0; h < cfg->n_kv_heads; ++h) {
+        for (int q = 0; q < n_pairs; ++q)
+          blocks.push_back(GramBlock{slot_of_src[pair_list[2 * q]], slot_of_src[pair_list[2 * q + 1]], kv, h,
+                                     P.gram + ((static_cast<size_t>(kv) * cfg->n_kv_heads + h) * n_pairs + q) * kFD * kFD});
+        for (int l = 0; l < cfg->tgt_layers; ++l)
+          for (int bi = 0; bi < kk; ++bi)
+            blocks.push_back(GramBlock{slot_of_src[cfg->selection[l * kk + bi]], tslot0 + l, kv, h,
+                                       P.xty + (((static_cast<size_t>(l) * 2 + kv) * cfg->n_kv_heads + h) * kk + bi) *
+                                                   kFD * kFD});
+      }
+    size_t free_b = 0, total_b = 0;
+    if ((e = cudaMemGetInfo(&free_b, &total_b)) != cudaSuccess) {
+      set_error(std::string("kvx_fit_ridge: memory query: ") + cudaGetErrorString(e));
+      result = KVX_ERR_CUDA;
+      break;
+    }
+    const size_t budget = std::min<size_t>(free_b / 2, static_cast<size_t>(32) << 30);
+    if ((result = gram_sums(G, st, &timer)) != KVX_OK || (result = gram_blocks(G, blocks, budget, st, &timer)) != KVX_OK) {
+      set_error(std::string("kvx_fit_ridge: ") + kvx_last_error());
+      break;
+    }
     const size_t smem = static_cast<size_t>(kNB) * kNB * 8 + static_cast<size_t>(F - kNB) * kNB * 8;
     if ((e = cudaFuncSetAttribute(fit_solve_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem))) !=
         cudaSuccess) {
@@ -503,7 +378,9 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
       result = KVX_ERR_CUDA;
       break;
     }
+    timer.begin(3);
     fit_solve_kernel<<<solve_grid, 256, smem, st>>>(P);
+    timer.end();
     if ((e = cudaGetLastError()) != cudaSuccess) {
       set_error(std::string("kvx_fit_ridge: launch: ") + cudaGetErrorString(e));
       result = KVX_ERR_CUDA;
@@ -519,8 +396,11 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
     if (dstat == kNotSpd) {
       set_error("kvx_fit_ridge: a system is not positive definite (lambda = 0 with too few tokens?)");
       result = KVX_ERR_INVALID_ARG;
-    } else if (dstat != 0) {
+    } else if (dstat == KVX_ERR_DEVICE_BOUNDS) {
       set_error("kvx_fit_ridge: a position is outside [0, 2^24)");
+      result = KVX_ERR_DEVICE_BOUNDS;
+    } else if (dstat != 0) {
+      set_error(std::string("kvx_fit_ridge: device status ") + kvx_status_string(static_cast<kvx_status>(dstat)));
       result = static_cast<kvx_status>(dstat);
     }
   } while (false);
@@ -529,6 +409,7 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
     set_error(std::string("kvx_fit_ridge: free: ") + cudaGetErrorString(e));
     result = KVX_ERR_CUDA;
   }
+  if (result == KVX_OK) timer.finish();
   return result;
 }
 

@@ -78,7 +78,7 @@ _lib = None
 
 EXPORTED = ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
             "kvx_set_kernel", "kvx_get_status", "kvx_mapper_params", "kvx_status_string",
-            "kvx_last_error", "kvx_map_noalloc", "kvx_fit_ridge")
+            "kvx_last_error", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms")
 
 
 def lib():
@@ -108,8 +108,9 @@ def lib():
                                   i32, i32, vp, ctypes.POINTER(kvx_tgt), vp, ctypes.POINTER(i32)]
     L.kvx_fit_ridge.argtypes = [ctypes.POINTER(kvx_fit_config), ctypes.POINTER(kvx_src), ctypes.POINTER(kvx_src),
                                 i32, i32, vp, vp, vp, vp]
+    L.kvx_last_phase_ms.argtypes = [ctypes.POINTER(ctypes.c_float)]
     for name in ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
-                 "kvx_set_kernel", "kvx_get_status", "kvx_map_noalloc", "kvx_fit_ridge"):
+                 "kvx_set_kernel", "kvx_get_status", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms"):
         getattr(L, name).restype = ctypes.c_int
     _lib = L
     return L
@@ -297,3 +298,11 @@ def kvx_fit_ridge(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, thet
                          float(theta_s), float(theta_t), float(lam), _ptr(sel))
     _check(lib().kvx_fit_ridge(ctypes.byref(cfg), ctypes.byref(src), ctypes.byref(tgt), int(batch),
                                int(tokens_per_seq), positions_ptr, W_ptr, b_ptr, stream), "kvx_fit_ridge")
+
+
+def kvx_last_phase_ms():
+    """Device milliseconds of the phases of the last fit / probe call on this thread:
+    (column sums, operand packing, tensor-core Gram blocks, solves or scores)."""
+    ms = (ctypes.c_float * 4)()
+    _check(lib().kvx_last_phase_ms(ms), "kvx_last_phase_ms")
+    return tuple(float(x) for x in ms)
