@@ -28,6 +28,7 @@
 #include <string>
 #include <vector>
 
+#include "kvx_gram.h"
 #include "kvx_internal.h"
 #include "kvx_ptx.cuh"
 
