@@ -309,10 +309,14 @@ def fit_bench(args, w):
     W = torch.empty((w.Lt, 2, w.H, F, w.d), dtype=torch.float32, device=dev)
     b = torch.empty((w.Lt, 2, w.H, w.d), dtype=torch.float32, device=dev)
     src, tgt = kvx.src_from_tensors(sk, sv), kvx.src_from_tensors(tk, tv)
+    # one caller workspace, allocated once (no per-call allocation inside the timed region)
+    ws_bytes = kvx.kvx_fit_workspace_bytes(w.Ls, w.Lt, w.H, w.d, w.k, w.theta_s, w.theta_t, 0.01, sel, w.B, w.T)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
 
     def step():
         kvx.kvx_fit_ridge(w.Ls, w.Lt, w.H, w.d, w.k, w.theta_s, w.theta_t, 0.01, sel, src, tgt, w.B, w.T,
-                          pos.data_ptr(), W.data_ptr(), b.data_ptr(), sp)
+                          pos.data_ptr(), W.data_ptr(), b.data_ptr(), sp, workspace_ptr=ws.data_ptr(),
+                          workspace_bytes=ws_bytes)
 
     for _ in range(args.warmup):
         step()
@@ -349,7 +353,8 @@ def fit_bench(args, w):
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16 caches, bf16x2-split tensor-core Gram (fp32 accumulate), fp64 solve",
             "data": "synthetic",
             "config": {"workload": w.name + " (fit)", "src_layers": w.Ls, "tgt_layers": w.Lt, "kv_heads": w.H,
-                       "head_dim": w.d, "k": w.k, "calibration_tokens": N, "systems": n_sys, "lambda": 0.01},
+                       "head_dim": w.d, "k": w.k, "calibration_tokens": N, "systems": n_sys, "lambda": 0.01,
+                       "workspace_gb": ws_bytes / 1e9},
             "clocks": clk.summary(),
             "gpu_launches": 4 * steps,
             "phase_ms": {"column_sums": phase[0], "pack": phase[1], "gram_tc": phase[2], "solve": phase[3]},
@@ -368,6 +373,67 @@ def fit_bench(args, w):
     return 0
 
 
+def probe_bench(args, w):
+    """Single-source R^2 probe (kvx_r2_probe) of every (target layer, source layer) pair on
+    N = B*T calibration tokens of the workload's shapes.  One step = one kvx_r2_probe call
+    (column sums, pack, tensor-core Gram blocks, factor / score / reduce kernels,
+    synchronous).  Roofline: the tensor-core Gram kernel (four bf16 MMAs per product) against
+    the measured bf16 peak."""
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(0)
+    sp = torch.cuda.current_stream(dev).cuda_stream
+    sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+    tk, tv = syn.target_cache(w, 0, device=dev), syn.target_cache(w, 1, device=dev)
+    pos = torch.from_numpy(syn.positions(w)).to(dev)
+    scores = torch.empty((w.Lt, w.Ls), dtype=torch.float64, device=dev)
+    src, tgt = kvx.src_from_tensors(sk, sv), kvx.src_from_tensors(tk, tv)
+    ws_bytes = kvx.kvx_r2_probe_workspace_bytes(w.Ls, w.Lt, w.H, w.d, w.theta_s, w.theta_t, w.B, w.T)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+
+    def step():
+        kvx.kvx_r2_probe(w.Ls, w.Lt, w.H, w.d, w.theta_s, w.theta_t, src, tgt, w.B, w.T, pos.data_ptr(),
+                         scores.data_ptr(), None, sp, workspace_ptr=ws.data_ptr(), workspace_bytes=ws_bytes)
+
+    for _ in range(args.warmup):
+        step()
+    steps = max(1, min(args.steps, 20))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    phase = [0.0] * 4
+    with ClockSampler(0) as clk:
+        torch.cuda.synchronize()
+        e0.record()
+        for _ in range(steps):
+            step()
+            phase = [a + b for a, b in zip(phase, kvx.kvx_last_phase_ms())]
+        e1.record()
+        torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    phase = [p / steps for p in phase]
+    N = w.n_tokens
+    blocks = 2 * w.H * w.Ls * (w.Lt + 1)              # C blocks of every pair + A of every source
+    gram_flop = blocks * 2.0 * N * w.d * w.d          # algorithmic: one product per token and entry pair
+    achieved = 4.0 * gram_flop / (phase[2] / 1e3) / 1e12
+    pk = load_peaks()
+    line = {"metric": "R2-probe calibration tokens/s", "value": N / (ms / 1e3), "unit": "tokens/s", "n_gpus": 1,
+            "steps": steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16 caches, bf16x2-split tensor-core Gram (fp32 accumulate), fp64 Cholesky, fp32 scores",
+            "data": "synthetic",
+            "config": {"workload": w.name + " (R2 probe)", "src_layers": w.Ls, "tgt_layers": w.Lt, "kv_heads": w.H,
+                       "head_dim": w.d, "calibration_tokens": N, "layer_pairs": w.Lt * w.Ls,
+                       "workspace_gb": ws_bytes / 1e9},
+            "clocks": clk.summary(),
+            "gpu_launches": 7 * steps,
+            "phase_ms": {"column_sums": phase[0], "pack": phase[1], "gram_tc": phase[2], "factor_score": phase[3]},
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": pk["bf16"], "unit": "TFLOP/s",
+                         "frac": achieved / pk["bf16"], "traffic": None, "kernel": "gram_tc_kernel",
+                         "peak_source": pk["source"] + " bf16 (four bf16 MMAs per product counted)",
+                         "algorithmic": {"gram_blocks": blocks, "gram_flop_per_step": gram_flop}},
+            "kernel": "gram_pack_kernel<0> + gram_pack_kernel<1> + gram_tc_kernel + probe kernels"}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -379,11 +445,15 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=None)
     ap.add_argument("--fit", action="store_true",
                     help="time the ridge fit (kvx_fit_ridge) on the workload's shapes instead of the map")
+    ap.add_argument("--probe", action="store_true",
+                    help="time the single-source R^2 probe (kvx_r2_probe) on the workload's shapes")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     w = syn.workload(args.workload)
     if args.fit:
         return fit_bench(args, w)
+    if args.probe:
+        return probe_bench(args, w)
     alg = algorithmic(w)
     config = {"workload": w.name, "src_layers": w.Ls, "tgt_layers": w.Lt, "kv_heads": w.H,
               "head_dim": w.d, "k": w.k, "batch": w.B, "seq_len": w.T, "tokens_per_step": w.n_tokens,

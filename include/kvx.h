@@ -196,18 +196,64 @@ KVX_API int64_t kvx_mapper_params(int32_t tgt_layers, int32_t n_kv_heads, int32_
  * blocks (at most L_t*2*H*(k*(k+1)/2 + k)*64 KB), 8 MB per SM, and the packed operands
  * (4 bytes per token, channel, K|V, head and used layer of either model), at most half the
  * free device memory or 32 GB, the tokens taken in chunks beyond that.  INVALID_ARG for
- * bad arguments or when a system is not positive definite (lambda = 0 with too few
- * tokens); DEVICE_BOUNDS when a position is outside [0, 2^24); OOM when the workspace
- * cannot be allocated. */
+ * bad arguments (a caller workspace that cannot hold 64 tokens included) or when a system
+ * is not positive definite (lambda = 0 with too few tokens); DEVICE_BOUNDS when a
+ * position is outside [0, 2^24); OOM when the workspace cannot be allocated.  With cfg->workspace the
+ * call allocates nothing: the caller's region holds every device piece. */
 typedef struct {
   int32_t src_layers, tgt_layers, n_kv_heads, head_dim, k;
   double src_rope_theta, tgt_rope_theta;
   double lambda;                 /* >= 0; the paper's value is 0.01 */
   const int32_t* selection;      /* host [tgt_layers][k], entries in [0, src_layers) */
+  void* workspace;               /* device, 256-byte aligned, or NULL (the call allocates) */
+  uint64_t workspace_bytes;      /* its size; kvx_fit_workspace_bytes gives the size that
+                                  * holds every token in one pass (less: tokens in chunks) */
 } kvx_fit_config;
 KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, const kvx_src* tgt, int32_t batch,
                                  int32_t tokens_per_seq, const int32_t* positions, float* W, float* b,
                                  void* stream);
+
+/* Workspace bytes for which kvx_fit_ridge (cfg->workspace set) packs every calibration
+ * token in one pass; -1 on invalid arguments or when no device is current. */
+KVX_API int64_t kvx_fit_workspace_bytes(const kvx_fit_config* cfg, int32_t batch, int32_t tokens_per_seq);
+
+/* Single-source R^2 probe and selection scores (Sec. 2.3, Eq. single_source_ols; Sec.
+ * 3.2) on calibration caches: for every target layer l, source layer l', K|V and head h,
+ * the OLS fit with intercept of head h of target layer l on head h of source layer l' over
+ * the N = batch * tokens_per_seq tokens (keys RoPE-stripped on both sides, theta_s for the
+ * source and theta_t for the target), scored by R^2 = 1 - SS_res / SS_tot pooled over
+ * the 128 output channels;
+ *   scores[l][l'] = (mean_h R^2_K + mean_h R^2_V) / 2,
+ * the score that kvx_select_topk / kvx_select_topk_device rank.  `src` [L_s][B][H][T][d]
+ * and `tgt` [L_t][B][H][T][d] as in kvx_fit_ridge (bf16, d = 128); `positions` device
+ * [batch][tokens_per_seq]; `scores` device double [L_t][L_s]; `r2_kv` device double
+ * [2][L_t][L_s] (the head-averaged R^2 of K and of V) or NULL.  The centred
+ * cross-products run on the tensor cores as in kvx_fit_ridge (fp32 accumulation of bf16
+ * hi + lo products); each source Gram block is factorised in fp64 and inverted, and
+ * explained = ||L^{-1} C||^2 is accumulated in fp32.  Runs on `stream` and synchronises
+ * it (an offline step).  Workspace: 2 H L_s (L_t + 2) blocks of 64 KB plus the packed
+ * operands (as kvx_fit_ridge, every layer of both models); from cfg->workspace when it is
+ * set (kvx_r2_probe_workspace_bytes: the size for one pass over the tokens), else
+ * stream-ordered allocations.  INVALID_ARG for bad arguments (a caller workspace that
+ * cannot hold 64 tokens included), for N <= 128, or when a source Gram block is singular;
+ * DEVICE_BOUNDS when a position is outside [0, 2^24); OOM when the workspace cannot be
+ * allocated. */
+typedef struct {
+  int32_t src_layers, tgt_layers, n_kv_heads, head_dim;
+  double src_rope_theta, tgt_rope_theta;
+  void* workspace;               /* device, 256-byte aligned, or NULL (the call allocates) */
+  uint64_t workspace_bytes;
+} kvx_probe_config;
+KVX_API kvx_status kvx_r2_probe(const kvx_probe_config* cfg, const kvx_src* src, const kvx_src* tgt, int32_t batch,
+                                int32_t tokens_per_seq, const int32_t* positions, double* scores, double* r2_kv,
+                                void* stream);
+KVX_API int64_t kvx_r2_probe_workspace_bytes(const kvx_probe_config* cfg, int32_t batch, int32_t tokens_per_seq);
+
+/* Top-k source-layer selection on the device, with the semantics of kvx_select_topk:
+ * `scores` device double [L_t][L_s], `out` device int32 [L_t][k], rows ascending.
+ * Synchronises `stream`.  INVALID_ARG for NULL, k outside [1, L_s] or a NaN score. */
+KVX_API kvx_status kvx_select_topk_device(const double* scores, int32_t tgt_layers, int32_t src_layers, int32_t k,
+                                          int32_t* out, void* stream);
 
 /* Device time in milliseconds of the phases of the last successful kvx_fit_ridge or
  * kvx_r2_probe call on this thread, from CUDA events on the call's stream: ms[0] column

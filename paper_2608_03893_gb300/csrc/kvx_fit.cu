@@ -198,10 +198,112 @@ __global__ void __launch_bounds__(256) fit_solve_kernel(const __grid_constant__ 
   }
 }
 
+// Host plan of a fit: the distinct source pairs, the block tables, the operand slots and
+// the sizes of every device piece (the same for the run and the workspace query).
+struct FitPlan {
+  std::vector<int32_t> pair_list, pair_of, tab, slot_of_src;
+  int n_pairs = 0, solve_grid = 0, F = 0;
+  size_t n_sys = 0, sums_n = 0, gram_n = 0, xty_n = 0, scratch_n = 0, sel_n = 0, n_blocks = 0;
+  size_t fixed_bytes = 0;          // sums, scratch, blocks, tables, status (256-aligned pieces)
+};
+
+size_t al256(size_t n) { return (n + 255) / 256 * 256; }
+
+FitPlan plan_fit(const kvx_fit_config* cfg, int sms, GramSpec* G) {
+  FitPlan p;
+  const int kk = cfg->k;
+  p.F = kk * kFD;
+  p.n_sys = static_cast<size_t>(cfg->tgt_layers) * 2 * cfg->n_kv_heads;
+  p.sums_n = static_cast<size_t>(2) * (cfg->src_layers + cfg->tgt_layers) * cfg->n_kv_heads * kFD;
+  p.pair_of.assign(static_cast<size_t>(cfg->tgt_layers) * kk * kk, -1);
+  std::vector<int32_t> index(static_cast<size_t>(cfg->src_layers) * cfg->src_layers, -1);
+  for (int l = 0; l < cfg->tgt_layers; ++l)
+    for (int bi = 0; bi < kk; ++bi)
+      for (int bj = 0; bj <= bi; ++bj) {
+        int sa = cfg->selection[l * kk + bi], sb = cfg->selection[l * kk + bj];
+        int ia = bi, ib = bj;
+        if (sa < sb) {   // keep the block's rows on the larger layer; transpose in the solve
+          std::swap(sa, sb);
+          std::swap(ia, ib);
+        }
+        int32_t& idx = index[static_cast<size_t>(sa) * cfg->src_layers + sb];
+        if (idx < 0) {
+          idx = static_cast<int32_t>(p.pair_list.size() / 2);
+          p.pair_list.push_back(sa);
+          p.pair_list.push_back(sb);
+        }
+        p.pair_of[(static_cast<size_t>(l) * kk + bi) * kk + bj] = ia == bi ? idx : -1 - idx;
+      }
+  p.n_pairs = static_cast<int>(p.pair_list.size() / 2);
+  p.gram_n = static_cast<size_t>(2) * cfg->n_kv_heads * p.n_pairs * kFD * kFD;
+  p.xty_n = p.n_sys * kk * kFD * kFD;
+  p.solve_grid = static_cast<int>(std::min<size_t>(p.n_sys, static_cast<size_t>(std::max(sms, 1))));
+  p.scratch_n = static_cast<size_t>(p.solve_grid) * (static_cast<size_t>(p.F) * p.F + static_cast<size_t>(p.F) * kFD);
+  p.sel_n = static_cast<size_t>(cfg->tgt_layers) * kk;
+  p.tab.assign(cfg->selection, cfg->selection + p.sel_n);
+  p.tab.insert(p.tab.end(), p.pair_list.begin(), p.pair_list.end());
+  p.tab.insert(p.tab.end(), p.pair_of.begin(), p.pair_of.end());
+  // operands: the selected source layers, then every target layer
+  p.slot_of_src.assign(cfg->src_layers, -1);
+  for (size_t i = 0; i < p.sel_n; ++i) p.slot_of_src[cfg->selection[i]] = 0;
+  G->slot_side.clear();
+  G->slot_layer.clear();
+  for (int L = 0; L < cfg->src_layers; ++L)
+    if (p.slot_of_src[L] == 0) {
+      p.slot_of_src[L] = static_cast<int32_t>(G->slot_side.size());
+      G->slot_side.push_back(0);
+      G->slot_layer.push_back(L);
+    }
+  for (int l = 0; l < cfg->tgt_layers; ++l) {
+    G->slot_side.push_back(1);
+    G->slot_layer.push_back(l);
+  }
+  G->H = cfg->n_kv_heads;
+  p.n_blocks = static_cast<size_t>(2) * cfg->n_kv_heads * (p.n_pairs + p.sel_n);
+  p.fixed_bytes = al256(p.sums_n * 8) + al256(p.scratch_n * 8) + al256((p.gram_n + p.xty_n) * 4) +
+                  al256(p.tab.size() * 4 + 4) + gram_fixed_bytes(*G, p.n_blocks);
+  return p;
+}
+
+const char* check_fit_config(const kvx_fit_config* cfg) {
+  if (!cfg) return "NULL argument";
+  if (cfg->head_dim != kFD) return "head_dim must be 128";
+  if (cfg->k < 1 || cfg->k > 4) return "k must be in [1, 4]";
+  if (cfg->src_layers < 1 || cfg->tgt_layers < 1 || cfg->n_kv_heads < 1 || cfg->k > cfg->src_layers)
+    return "layer / head counts out of range";
+  if (!(cfg->lambda >= 0.0) || !(cfg->src_rope_theta > 1.0) || !(cfg->tgt_rope_theta > 1.0))
+    return "lambda must be >= 0 and the RoPE bases > 1";
+  if (!cfg->selection) return "NULL selection";
+  for (int64_t i = 0; i < static_cast<int64_t>(cfg->tgt_layers) * cfg->k; ++i)
+    if (cfg->selection[i] < 0 || cfg->selection[i] >= cfg->src_layers) return "selection entry out of range";
+  if (cfg->workspace_bytes != 0 && !cfg->workspace) return "workspace_bytes without a workspace";
+  if (reinterpret_cast<uintptr_t>(cfg->workspace) & 255u) return "workspace must be 256-byte aligned";
+  return nullptr;
+}
+
+int sm_count_or_zero() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return 0;
+  return sms;
+}
+
 }  // namespace
 }  // namespace kvx
 
 extern "C" {
+
+KVX_API int64_t kvx_fit_workspace_bytes(const kvx_fit_config* cfg, int32_t batch, int32_t tokens_per_seq) {
+  using namespace kvx;
+  if (check_fit_config(cfg) || batch < 1 || tokens_per_seq < 1) return -1;
+  const int sms = sm_count_or_zero();
+  if (sms <= 0) return -1;
+  GramSpec G;
+  const FitPlan p = plan_fit(cfg, sms, &G);
+  const int64_t N = static_cast<int64_t>(batch) * tokens_per_seq;
+  const size_t np = static_cast<size_t>((N + 63) / 64 * 64);
+  return static_cast<int64_t>(p.fixed_bytes + gram_bytes_per_token(G) * np + 1024);
+}
 
 KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, const kvx_src* tgt, int32_t batch,
                                  int32_t tokens_per_seq, const int32_t* positions, float* W, float* b,
@@ -212,16 +314,8 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
     set_error(std::string("kvx_fit_ridge: ") + m);
     return KVX_ERR_INVALID_ARG;
   };
-  if (!cfg || !src || !tgt || !positions || !W || !b) return bad("NULL argument");
-  if (cfg->head_dim != kFD) return bad("head_dim must be 128");
-  if (cfg->k < 1 || cfg->k > 4) return bad("k must be in [1, 4]");
-  if (cfg->src_layers < 1 || cfg->tgt_layers < 1 || cfg->n_kv_heads < 1 || cfg->k > cfg->src_layers)
-    return bad("layer / head counts out of range");
-  if (!(cfg->lambda >= 0.0) || !(cfg->src_rope_theta > 1.0) || !(cfg->tgt_rope_theta > 1.0))
-    return bad("lambda must be >= 0 and the RoPE bases > 1");
-  if (!cfg->selection) return bad("NULL selection");
-  for (int64_t i = 0; i < static_cast<int64_t>(cfg->tgt_layers) * cfg->k; ++i)
-    if (cfg->selection[i] < 0 || cfg->selection[i] >= cfg->src_layers) return bad("selection entry out of range");
+  if (const char* why = check_fit_config(cfg)) return bad(why);
+  if (!src || !tgt || !positions || !W || !b) return bad("NULL argument");
   if (batch < 1 || tokens_per_seq < 1) return bad("batch and tokens_per_seq must be >= 1");
   const kvx_src* cs[2] = {src, tgt};
   for (const kvx_src* c : cs) {
@@ -238,9 +332,9 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
 
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   cudaError_t e;
-  int dev = 0, sms = 0;
-  if ((e = cudaGetDevice(&dev)) != cudaSuccess || (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) {
-    set_error(std::string("kvx_fit_ridge: device query: ") + cudaGetErrorString(e));
+  const int sms = sm_count_or_zero();
+  if (sms <= 0) {
+    set_error("kvx_fit_ridge: device query failed");
     return KVX_ERR_CUDA;
   }
   kvx_ctx tmp;                       // for the RoPE tables only
@@ -249,18 +343,36 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
   tmp.theta_t = cfg->tgt_rope_theta;
   fill_rope(&tmp);
 
-  FitParams P{};
   GramSpec G;
+  const FitPlan pl = plan_fit(cfg, sms, &G);
   G.cache[0] = GramCache{src->k, src->v, {src->stride[0], src->stride[1], src->stride[2], src->stride[3]}};
   G.cache[1] = GramCache{tgt->k, tgt->v, {tgt->stride[0], tgt->stride[1], tgt->stride[2], tgt->stride[3]}};
   G.pos = positions;
   G.B = batch;
   G.T = tokens_per_seq;
-  G.H = cfg->n_kv_heads;
   G.Ls = cfg->src_layers;
   G.Lt = cfg->tgt_layers;
   G.rope = tmp.rope;
   G.sm_count = sms;
+
+  // device pieces: from the caller's workspace, or one stream-ordered allocation
+  Scratch S;
+  char* own = nullptr;
+  const bool caller_ws = cfg->workspace != nullptr;
+  const size_t fit_bytes = pl.fixed_bytes - gram_fixed_bytes(G, pl.n_blocks);
+  if (caller_ws) {
+    S.p = static_cast<char*>(cfg->workspace);
+    S.bytes = static_cast<size_t>(cfg->workspace_bytes);
+    if (S.bytes < pl.fixed_bytes) return bad("workspace too small (see kvx_fit_workspace_bytes)");
+  } else {
+    if ((e = cudaMallocAsync(reinterpret_cast<void**>(&own), fit_bytes, st)) != cudaSuccess) {
+      set_error(std::string("kvx_fit_ridge: workspace: ") + cudaGetErrorString(e));
+      return KVX_ERR_OOM;
+    }
+    S.p = own;
+    S.bytes = fit_bytes;
+  }
+  FitParams P{};
   P.Ls = cfg->src_layers;
   P.Lt = cfg->tgt_layers;
   P.H = cfg->n_kv_heads;
@@ -270,109 +382,62 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
   P.W = W;
   P.b = b;
   P.lambda = cfg->lambda;
-
-  const int F = cfg->k * kFD;
-  const size_t n_sys = static_cast<size_t>(cfg->tgt_layers) * 2 * cfg->n_kv_heads;
-  const size_t sums_n = static_cast<size_t>(2) * (cfg->src_layers + cfg->tgt_layers) * cfg->n_kv_heads * kFD;
-  // the distinct (source layer, source layer) blocks of all target layers' Xc^T Xc
-  const int kk = cfg->k;
-  std::vector<int32_t> pair_list, pair_of(static_cast<size_t>(cfg->tgt_layers) * kk * kk, -1);
-  {
-    std::vector<int32_t> index(static_cast<size_t>(cfg->src_layers) * cfg->src_layers, -1);
-    for (int l = 0; l < cfg->tgt_layers; ++l)
-      for (int bi = 0; bi < kk; ++bi)
-        for (int bj = 0; bj <= bi; ++bj) {
-          int sa = cfg->selection[l * kk + bi], sb = cfg->selection[l * kk + bj];
-          int ia = bi, ib = bj;
-          if (sa < sb) {   // keep the block's rows on the larger layer; transpose in the solve
-            std::swap(sa, sb);
-            std::swap(ia, ib);
-          }
-          int32_t& idx = index[static_cast<size_t>(sa) * cfg->src_layers + sb];
-          if (idx < 0) {
-            idx = static_cast<int32_t>(pair_list.size() / 2);
-            pair_list.push_back(sa);
-            pair_list.push_back(sb);
-          }
-          pair_of[(static_cast<size_t>(l) * kk + bi) * kk + bj] = ia == bi ? idx : -1 - idx;
-        }
-  }
-  const int n_pairs = static_cast<int>(pair_list.size() / 2);
-  P.n_pairs = n_pairs;
-  const size_t gram_n = static_cast<size_t>(2) * cfg->n_kv_heads * n_pairs * kFD * kFD;
-  const size_t xty_n = n_sys * cfg->k * kFD * kFD;
-  const int solve_grid = static_cast<int>(std::min<size_t>(n_sys, static_cast<size_t>(sms)));
-  const size_t scratch_n = static_cast<size_t>(solve_grid) * (static_cast<size_t>(F) * F + static_cast<size_t>(F) * kFD);
-  const size_t sel_n = static_cast<size_t>(cfg->tgt_layers) * cfg->k;
-  std::vector<int32_t> tab(cfg->selection, cfg->selection + sel_n);
-  tab.insert(tab.end(), pair_list.begin(), pair_list.end());
-  tab.insert(tab.end(), pair_of.begin(), pair_of.end());
-  const size_t bytes = sums_n * 8 + scratch_n * 8 + (gram_n + xty_n) * 4 + tab.size() * 4 + 16;
-  char* ws = nullptr;
-  if ((e = cudaMallocAsync(reinterpret_cast<void**>(&ws), bytes, st)) != cudaSuccess) {
-    set_error(std::string("kvx_fit_ridge: workspace: ") + cudaGetErrorString(e));
-    return KVX_ERR_OOM;
-  }
-  P.sums = reinterpret_cast<double*>(ws);
-  P.scratch = P.sums + sums_n;
-  P.gram = reinterpret_cast<float*>(P.scratch + scratch_n);
-  P.xty = P.gram + gram_n;
-  int32_t* dsel = reinterpret_cast<int32_t*>(P.xty + xty_n);
+  P.n_pairs = pl.n_pairs;
+  P.sums = reinterpret_cast<double*>(S.take(pl.sums_n * 8));
+  P.scratch = reinterpret_cast<double*>(S.take(pl.scratch_n * 8));
+  P.gram = reinterpret_cast<float*>(S.take((pl.gram_n + pl.xty_n) * 4));
+  P.xty = P.gram + pl.gram_n;
+  int32_t* dsel = reinterpret_cast<int32_t*>(S.take(pl.tab.size() * 4 + 4));
   P.sel = dsel;
-  P.pairs = dsel + sel_n;
-  P.pair_of = P.pairs + pair_list.size();
-  P.status = dsel + tab.size();
+  P.pairs = dsel + pl.sel_n;
+  P.pair_of = P.pairs + pl.pair_list.size();
+  P.status = dsel + pl.tab.size();
+  if (!caller_ws) S = Scratch{};     // the Gram engine allocates its own
   kvx_status result = KVX_OK;
   PhaseTimer timer(st);
   do {
-    if ((e = cudaMemsetAsync(P.sums, 0, sums_n * 8, st)) != cudaSuccess ||
+    if ((e = cudaMemsetAsync(P.sums, 0, pl.sums_n * 8, st)) != cudaSuccess ||
         (e = cudaMemsetAsync(P.status, 0, 4, st)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(dsel, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice, st)) != cudaSuccess) {
+        (e = cudaMemcpyAsync(dsel, pl.tab.data(), pl.tab.size() * 4, cudaMemcpyHostToDevice, st)) != cudaSuccess) {
       set_error(std::string("kvx_fit_ridge: setup: ") + cudaGetErrorString(e));
       result = KVX_ERR_CUDA;
       break;
     }
-    // operands: the selected source layers, then every target layer
-    std::vector<int32_t> slot_of_src(cfg->src_layers, -1);
-    for (size_t i = 0; i < sel_n; ++i) slot_of_src[cfg->selection[i]] = 0;
-    for (int L = 0; L < cfg->src_layers; ++L)
-      if (slot_of_src[L] == 0) {
-        slot_of_src[L] = static_cast<int32_t>(G.slot_side.size());
-        G.slot_side.push_back(0);
-        G.slot_layer.push_back(L);
-      }
-    const int32_t tslot0 = static_cast<int32_t>(G.slot_side.size());
-    for (int l = 0; l < cfg->tgt_layers; ++l) {
-      G.slot_side.push_back(1);
-      G.slot_layer.push_back(l);
-    }
     G.sums = P.sums;
     G.status = P.status;
+    const int kk = cfg->k;
+    const int32_t tslot0 = static_cast<int32_t>(G.slot_side.size()) - cfg->tgt_layers;
     std::vector<GramBlock> blocks;
-    blocks.reserve(static_cast<size_t>(2) * cfg->n_kv_heads * (n_pairs + sel_n));
+    blocks.reserve(pl.n_blocks);
     for (int kv = 0; kv < 2; ++kv)
       for (int h = 0; h < cfg->n_kv_heads; ++h) {
-        for (int q = 0; q < n_pairs; ++q)
-          blocks.push_back(GramBlock{slot_of_src[pair_list[2 * q]], slot_of_src[pair_list[2 * q + 1]], kv, h,
-                                     P.gram + ((static_cast<size_t>(kv) * cfg->n_kv_heads + h) * n_pairs + q) * kFD * kFD});
+        for (int q = 0; q < pl.n_pairs; ++q)
+          blocks.push_back(GramBlock{pl.slot_of_src[pl.pair_list[2 * q]], pl.slot_of_src[pl.pair_list[2 * q + 1]], kv,
+                                     h, P.gram + ((static_cast<size_t>(kv) * cfg->n_kv_heads + h) * pl.n_pairs + q) *
+                                                     kFD * kFD});
         for (int l = 0; l < cfg->tgt_layers; ++l)
           for (int bi = 0; bi < kk; ++bi)
-            blocks.push_back(GramBlock{slot_of_src[cfg->selection[l * kk + bi]], tslot0 + l, kv, h,
+            blocks.push_back(GramBlock{pl.slot_of_src[cfg->selection[l * kk + bi]], tslot0 + l, kv, h,
                                        P.xty + (((static_cast<size_t>(l) * 2 + kv) * cfg->n_kv_heads + h) * kk + bi) *
                                                    kFD * kFD});
       }
-    size_t free_b = 0, total_b = 0;
-    if ((e = cudaMemGetInfo(&free_b, &total_b)) != cudaSuccess) {
-      set_error(std::string("kvx_fit_ridge: memory query: ") + cudaGetErrorString(e));
-      result = KVX_ERR_CUDA;
-      break;
+    size_t budget = 0;
+    if (!caller_ws) {
+      size_t free_b = 0, total_b = 0;
+      if ((e = cudaMemGetInfo(&free_b, &total_b)) != cudaSuccess) {
+        set_error(std::string("kvx_fit_ridge: memory query: ") + cudaGetErrorString(e));
+        result = KVX_ERR_CUDA;
+        break;
+      }
+      budget = std::min<size_t>(free_b / 2, static_cast<size_t>(32) << 30);
     }
-    const size_t budget = std::min<size_t>(free_b / 2, static_cast<size_t>(32) << 30);
-    if ((result = gram_sums(G, st, &timer)) != KVX_OK || (result = gram_blocks(G, blocks, budget, st, &timer)) != KVX_OK) {
+    Scratch* sp = caller_ws ? &S : nullptr;
+    if ((result = gram_sums(G, st, &timer, sp)) != KVX_OK ||
+        (result = gram_blocks(G, blocks, budget, st, &timer, sp)) != KVX_OK) {
       set_error(std::string("kvx_fit_ridge: ") + kvx_last_error());
       break;
     }
-    const size_t smem = static_cast<size_t>(kNB) * kNB * 8 + static_cast<size_t>(F - kNB) * kNB * 8;
+    const size_t smem = static_cast<size_t>(kNB) * kNB * 8 + static_cast<size_t>(pl.F - kNB) * kNB * 8;
     if ((e = cudaFuncSetAttribute(fit_solve_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem))) !=
         cudaSuccess) {
       set_error(std::string("kvx_fit_ridge: smem attribute: ") + cudaGetErrorString(e));
@@ -380,7 +445,7 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
       break;
     }
     timer.begin(3);
-    fit_solve_kernel<<<solve_grid, 256, smem, st>>>(P);
+    fit_solve_kernel<<<pl.solve_grid, 256, smem, st>>>(P);
     timer.end();
     if ((e = cudaGetLastError()) != cudaSuccess) {
       set_error(std::string("kvx_fit_ridge: launch: ") + cudaGetErrorString(e));
@@ -405,8 +470,8 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
       result = static_cast<kvx_status>(dstat);
     }
   } while (false);
-  cudaFreeAsync(ws, st);
-  if (result == KVX_OK && (e = cudaStreamSynchronize(st)) != cudaSuccess) {
+  if (own) cudaFreeAsync(own, st);
+  if ((e = cudaStreamSynchronize(st)) != cudaSuccess && result == KVX_OK) {
     set_error(std::string("kvx_fit_ridge: free: ") + cudaGetErrorString(e));
     result = KVX_ERR_CUDA;
   }

@@ -551,15 +551,32 @@ void PhaseTimer::finish() {
   for (int i = 0; i < 4; ++i) g_phase_ms[i] = ms[i];
 }
 
-kvx_status gram_sums(const GramSpec& spec, cudaStream_t stream, PhaseTimer* timer) {
+size_t gram_fixed_bytes(const GramSpec& spec, size_t n_blocks) {
+  const size_t n_slots = spec.slot_side.size();
+  auto al = [](size_t n) { return (n + 255) / 256 * 256; };
+  return al(n_slots * 2 * 4) /* gram_sums slot table */ + al(n_blocks * sizeof(GramUnit)) + al(n_slots * 2 * 4) +
+         al(n_slots * 2 * static_cast<size_t>(spec.H) * kGD * 4);
+}
+
+size_t gram_bytes_per_token(const GramSpec& spec) {
+  return spec.slot_side.size() * 2 * static_cast<size_t>(spec.H) * 2 * kGD * 2;
+}
+
+kvx_status gram_sums(const GramSpec& spec, cudaStream_t stream, PhaseTimer* timer, Scratch* scratch) {
   const int n_slots = static_cast<int>(spec.slot_side.size());
   if (n_slots == 0) return KVX_OK;
   const int64_t N = static_cast<int64_t>(spec.B) * spec.T;
   const std::vector<int32_t> tab = slot_table(spec);
   int32_t* d_tab = nullptr;
   cudaError_t e;
-  if ((e = cudaMallocAsync(reinterpret_cast<void**>(&d_tab), tab.size() * 4, stream)) != cudaSuccess)
-    return cuda_fail("column sums: workspace", e);
+  const bool own = !(scratch && scratch->p);
+  if (own) {
+    if ((e = cudaMallocAsync(reinterpret_cast<void**>(&d_tab), tab.size() * 4, stream)) != cudaSuccess)
+      return cuda_fail("column sums: workspace", e);
+  } else if (!(d_tab = reinterpret_cast<int32_t*>(scratch->take(tab.size() * 4)))) {
+    set_error("column sums: workspace too small");
+    return KVX_ERR_INVALID_ARG;
+  }
   kvx_status r = KVX_OK;
   if ((e = cudaMemcpyAsync(d_tab, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice, stream)) != cudaSuccess) {
     r = cuda_fail("column sums: slot table", e);
@@ -575,12 +592,12 @@ kvx_status gram_sums(const GramSpec& spec, cudaStream_t stream, PhaseTimer* time
     if (timer) timer->end();
     if ((e = cudaGetLastError()) != cudaSuccess) r = cuda_fail("column sums: launch", e);
   }
-  cudaFreeAsync(d_tab, stream);
+  if (own) cudaFreeAsync(d_tab, stream);
   return r;
 }
 
 kvx_status gram_blocks(const GramSpec& spec, const std::vector<GramBlock>& blocks, size_t ws_budget,
-                       cudaStream_t stream, PhaseTimer* timer) {
+                       cudaStream_t stream, PhaseTimer* timer, Scratch* scratch) {
   if (blocks.empty()) return KVX_OK;
   auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(tensor_map_encoder());
   if (!encode) {
@@ -595,10 +612,16 @@ kvx_status gram_blocks(const GramSpec& spec, const std::vector<GramBlock>& block
   }
   const int64_t N = static_cast<int64_t>(spec.B) * spec.T;
   const int64_t np_full = (N + kGChunk - 1) / kGChunk * kGChunk;
+  const bool own = !(scratch && scratch->p);
+  if (!own) {   // the fixed pieces come first; the packed operands get the rest
+    const size_t fixed = gram_fixed_bytes(spec, blocks.size()) - (n_slots * 2 * 4 + 255) / 256 * 256;
+    ws_budget = scratch->bytes > fixed + 256 ? scratch->bytes - fixed - 256 : 0;
+  }
   const int64_t np_fit = static_cast<int64_t>(ws_budget / (static_cast<size_t>(rows) * 2)) / kGChunk * kGChunk;
   if (np_fit < kGChunk) {
-    set_error("Gram blocks: the workspace budget holds less than 64 tokens of the operands");
-    return KVX_ERR_OOM;
+    set_error(own ? "Gram blocks: the workspace budget holds less than 64 tokens of the operands"
+                  : "Gram blocks: the caller's workspace holds less than 64 tokens of the operands");
+    return own ? KVX_ERR_OOM : KVX_ERR_INVALID_ARG;
   }
   const int64_t np = std::min<int64_t>(std::min(np_full, np_fit), INT_MAX / 2 / kGChunk * kGChunk);
   const int64_t n_chunks = (N + np - 1) / np;
@@ -642,16 +665,22 @@ kvx_status gram_blocks(const GramSpec& spec, const std::vector<GramBlock>& block
     return KVX_ERR_UNSUPPORTED;
   }
   const std::vector<int32_t> tab = slot_table(spec);
+  auto al = [](size_t n) { return (n + 255) / 256 * 256; };
   const size_t ws_bytes = static_cast<size_t>(rows) * static_cast<size_t>(np) * 2;
-  const size_t units_off = ws_bytes;
-  const size_t tab_off = units_off + units.size() * sizeof(GramUnit);
-  const size_t means_off = (tab_off + tab.size() * 4 + 15) / 16 * 16;
+  const size_t units_off = al(ws_bytes);
+  const size_t tab_off = units_off + al(units.size() * sizeof(GramUnit));
+  const size_t means_off = tab_off + al(tab.size() * 4);
   const size_t means_n = static_cast<size_t>(n_slots) * 2 * spec.H * kGD;
-  const size_t total = means_off + means_n * 4;
+  const size_t total = means_off + al(means_n * 4);
   char* mem = nullptr;
   cudaError_t e;
-  if ((e = cudaMallocAsync(reinterpret_cast<void**>(&mem), total, stream)) != cudaSuccess)
-    return cuda_fail("Gram blocks: workspace", e);
+  if (own) {
+    if ((e = cudaMallocAsync(reinterpret_cast<void**>(&mem), total, stream)) != cudaSuccess)
+      return cuda_fail("Gram blocks: workspace", e);
+  } else if (!(mem = scratch->take(total))) {
+    set_error("Gram blocks: the caller's workspace is too small");
+    return KVX_ERR_INVALID_ARG;
+  }
   kvx_status r = KVX_OK;
   do {
     if ((e = cudaMemcpyAsync(mem + units_off, units.data(), units.size() * sizeof(GramUnit), cudaMemcpyHostToDevice,
@@ -713,7 +742,7 @@ kvx_status gram_blocks(const GramSpec& spec, const std::vector<GramBlock>& block
       if ((e = cudaGetLastError()) != cudaSuccess) r = cuda_fail("Gram blocks: launch", e);
     }
   } while (false);
-  cudaFreeAsync(mem, stream);
+  if (own) cudaFreeAsync(mem, stream);
   return r;
 }
 

@@ -56,10 +56,31 @@ class PhaseTimer {
   std::vector<cudaEvent_t> ev_;
 };
 
+// A caller-provided device region that the offline calls carve their workspace from (256-
+// byte aligned pieces from the front); with p == NULL they allocate stream-ordered memory.
+struct Scratch {
+  char* p = nullptr;
+  size_t bytes = 0;
+  char* take(size_t n) {
+    const size_t a = (n + 255) / 256 * 256;
+    if (!p || a > bytes) return nullptr;
+    char* r = p;
+    p += a;
+    bytes -= a;
+    return r;
+  }
+};
+
+// Bytes gram_sums and gram_blocks take from a Scratch besides the packed operands (slot
+// tables, work units, means; `n_blocks` blocks), and bytes of packed operands per token.
+size_t gram_fixed_bytes(const GramSpec& spec, size_t n_blocks);
+size_t gram_bytes_per_token(const GramSpec& spec);
+
 // Column sums of every slot into spec.sums (one pass over the caches).
-kvx_status gram_sums(const GramSpec& spec, cudaStream_t stream, PhaseTimer* timer);
+kvx_status gram_sums(const GramSpec& spec, cudaStream_t stream, PhaseTimer* timer, Scratch* scratch);
 // Every block of the list (after gram_sums); the tokens are processed in chunks that
-// keep the packed-operand workspace within `ws_budget` bytes.
+// keep the packed operands within `ws_budget` bytes, or, with a Scratch, within what is
+// left of it.
 kvx_status gram_blocks(const GramSpec& spec, const std::vector<GramBlock>& blocks, size_t ws_budget,
-                       cudaStream_t stream, PhaseTimer* timer);
+                       cudaStream_t stream, PhaseTimer* timer, Scratch* scratch);
 }  // namespace kvx

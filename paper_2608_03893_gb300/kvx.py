@@ -71,6 +71,16 @@ class kvx_fit_config(ctypes.Structure):
         ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("k", ctypes.c_int32),
         ("src_rope_theta", ctypes.c_double), ("tgt_rope_theta", ctypes.c_double),
         ("lambda_", ctypes.c_double), ("selection", ctypes.c_void_p),
+        ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_uint64),
+    ]
+
+
+class kvx_probe_config(ctypes.Structure):
+    _fields_ = [
+        ("src_layers", ctypes.c_int32), ("tgt_layers", ctypes.c_int32),
+        ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+        ("src_rope_theta", ctypes.c_double), ("tgt_rope_theta", ctypes.c_double),
+        ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_uint64),
     ]
 
 
@@ -78,7 +88,8 @@ _lib = None
 
 EXPORTED = ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
             "kvx_set_kernel", "kvx_get_status", "kvx_mapper_params", "kvx_status_string",
-            "kvx_last_error", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms")
+            "kvx_last_error", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms", "kvx_r2_probe",
+            "kvx_select_topk_device", "kvx_fit_workspace_bytes", "kvx_r2_probe_workspace_bytes")
 
 
 def lib():
@@ -109,8 +120,16 @@ def lib():
     L.kvx_fit_ridge.argtypes = [ctypes.POINTER(kvx_fit_config), ctypes.POINTER(kvx_src), ctypes.POINTER(kvx_src),
                                 i32, i32, vp, vp, vp, vp]
     L.kvx_last_phase_ms.argtypes = [ctypes.POINTER(ctypes.c_float)]
+    L.kvx_r2_probe.argtypes = [ctypes.POINTER(kvx_probe_config), ctypes.POINTER(kvx_src), ctypes.POINTER(kvx_src),
+                               i32, i32, vp, vp, vp, vp]
+    L.kvx_select_topk_device.argtypes = [vp, i32, i32, i32, vp, vp]
+    L.kvx_fit_workspace_bytes.argtypes = [ctypes.POINTER(kvx_fit_config), i32, i32]
+    L.kvx_fit_workspace_bytes.restype = i64
+    L.kvx_r2_probe_workspace_bytes.argtypes = [ctypes.POINTER(kvx_probe_config), i32, i32]
+    L.kvx_r2_probe_workspace_bytes.restype = i64
     for name in ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
-                 "kvx_set_kernel", "kvx_get_status", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms"):
+                 "kvx_set_kernel", "kvx_get_status", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms",
+                 "kvx_r2_probe", "kvx_select_topk_device"):
         getattr(L, name).restype = ctypes.c_int
     _lib = L
     return L
@@ -287,15 +306,34 @@ def tgt_paged_from_tensors(k, v, block_table, block_size):
     return t
 
 
-def kvx_fit_ridge(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, selection,
-                  src, tgt, batch, tokens_per_seq, positions_ptr, W_ptr, b_ptr, stream=0):
-    """Ridge fit on calibration caches (see include/kvx.h): src / tgt are kvx_src, selection a
-    host int32 [L_t][k] array, W_ptr / b_ptr device fp32 buffers [L_t][2][H][k*d][d] and
-    [L_t][2][H][d].  Blocks until the fit is done."""
+def _fit_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, sel, workspace_ptr,
+                workspace_bytes):
+    return kvx_fit_config(int(src_layers), int(tgt_layers), int(n_kv_heads), int(head_dim), int(k),
+                          float(theta_s), float(theta_t), float(lam), _ptr(sel), workspace_ptr,
+                          int(workspace_bytes))
+
+
+def kvx_fit_workspace_bytes(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, selection,
+                            batch, tokens_per_seq):
+    """Bytes of a caller workspace that holds every calibration token in one pass (-1 on
+    invalid arguments)."""
     import numpy as np
     sel = np.ascontiguousarray(selection, dtype=np.int32)
-    cfg = kvx_fit_config(int(src_layers), int(tgt_layers), int(n_kv_heads), int(head_dim), int(k),
-                         float(theta_s), float(theta_t), float(lam), _ptr(sel))
+    cfg = _fit_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, sel, None, 0)
+    return int(lib().kvx_fit_workspace_bytes(ctypes.byref(cfg), int(batch), int(tokens_per_seq)))
+
+
+def kvx_fit_ridge(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, selection,
+                  src, tgt, batch, tokens_per_seq, positions_ptr, W_ptr, b_ptr, stream=0,
+                  workspace_ptr=None, workspace_bytes=0):
+    """Ridge fit on calibration caches (see include/kvx.h): src / tgt are kvx_src, selection a
+    host int32 [L_t][k] array, W_ptr / b_ptr device fp32 buffers [L_t][2][H][k*d][d] and
+    [L_t][2][H][d]; an optional caller workspace (device, 256-byte aligned).  Blocks until
+    the fit is done."""
+    import numpy as np
+    sel = np.ascontiguousarray(selection, dtype=np.int32)
+    cfg = _fit_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, sel, workspace_ptr,
+                      workspace_bytes)
     _check(lib().kvx_fit_ridge(ctypes.byref(cfg), ctypes.byref(src), ctypes.byref(tgt), int(batch),
                                int(tokens_per_seq), positions_ptr, W_ptr, b_ptr, stream), "kvx_fit_ridge")
 
@@ -306,3 +344,32 @@ def kvx_last_phase_ms():
     ms = (ctypes.c_float * 4)()
     _check(lib().kvx_last_phase_ms(ms), "kvx_last_phase_ms")
     return tuple(float(x) for x in ms)
+
+
+def kvx_r2_probe_workspace_bytes(src_layers, tgt_layers, n_kv_heads, head_dim, theta_s, theta_t, batch,
+                                 tokens_per_seq):
+    """Bytes of a caller workspace for one pass of the probe over the tokens (-1 on invalid
+    arguments)."""
+    cfg = kvx_probe_config(int(src_layers), int(tgt_layers), int(n_kv_heads), int(head_dim),
+                           float(theta_s), float(theta_t), None, 0)
+    return int(lib().kvx_r2_probe_workspace_bytes(ctypes.byref(cfg), int(batch), int(tokens_per_seq)))
+
+
+def kvx_r2_probe(src_layers, tgt_layers, n_kv_heads, head_dim, theta_s, theta_t, src, tgt, batch,
+                 tokens_per_seq, positions_ptr, scores_ptr, r2_kv_ptr=None, stream=0,
+                 workspace_ptr=None, workspace_bytes=0):
+    """Single-source R^2 probe (see include/kvx.h): src / tgt are kvx_src; scores_ptr a
+    device float64 [L_t][L_s] buffer, r2_kv_ptr a device float64 [2][L_t][L_s] buffer or
+    None; an optional caller workspace.  Blocks until the probe is done."""
+    cfg = kvx_probe_config(int(src_layers), int(tgt_layers), int(n_kv_heads), int(head_dim),
+                           float(theta_s), float(theta_t), workspace_ptr, int(workspace_bytes))
+    _check(lib().kvx_r2_probe(ctypes.byref(cfg), ctypes.byref(src), ctypes.byref(tgt), int(batch),
+                              int(tokens_per_seq), positions_ptr, scores_ptr, r2_kv_ptr, stream),
+           "kvx_r2_probe")
+
+
+def kvx_select_topk_device(scores_ptr, tgt_layers, src_layers, k, out_ptr, stream=0):
+    """Top-k selection on the device: scores_ptr device float64 [L_t][L_s], out_ptr device
+    int32 [L_t][k] (rows ascending, ties to the lower source index)."""
+    _check(lib().kvx_select_topk_device(scores_ptr, int(tgt_layers), int(src_layers), int(k), out_ptr, stream),
+           "kvx_select_topk_device")

@@ -167,3 +167,34 @@ def test_fit_ridge_rejects_bad_arguments_before_touching_the_device():
                           a["theta_s"], a["theta_t"], a["lam"], a["selection"], src, src, 1, 16,
                           buf.ctypes.data, None, buf.ctypes.data)
     assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+
+
+def test_r2_probe_rejects_bad_arguments_before_touching_the_device():
+    """kvx_r2_probe validates everything on the host first."""
+    good = dict(src_layers=4, tgt_layers=3, n_kv_heads=2, head_dim=128, theta_s=1e6, theta_t=1e6, batch=1, T=256)
+    buf = np.zeros(64, dtype=np.float64)          # an aligned stand-in for device pointers
+    src = kvx.kvx_src(buf.ctypes.data, buf.ctypes.data, (ctypes.c_int64 * 4)(4096, 4096, 256, 128))
+    cases = [dict(head_dim=64), dict(src_layers=0), dict(tgt_layers=0), dict(n_kv_heads=0), dict(theta_t=1.0),
+             dict(theta_s=float("inf")), dict(T=128), dict(batch=0)]
+    for over in cases:
+        a = dict(good, **over)
+        with pytest.raises(kvx.KvxError) as e:
+            kvx.kvx_r2_probe(a["src_layers"], a["tgt_layers"], a["n_kv_heads"], a["head_dim"], a["theta_s"],
+                             a["theta_t"], src, src, a["batch"], a["T"], buf.ctypes.data, buf.ctypes.data)
+        assert e.value.status == kvx.KVX_ERR_INVALID_ARG, over
+    bad_stride = kvx.kvx_src(buf.ctypes.data, buf.ctypes.data, (ctypes.c_int64 * 4)(4096, 4096, 256, 100))
+    with pytest.raises(kvx.KvxError):
+        kvx.kvx_r2_probe(4, 3, 2, 128, 1e6, 1e6, bad_stride, src, 1, 256, buf.ctypes.data, buf.ctypes.data)
+    with pytest.raises(kvx.KvxError) as e:                 # NULL scores
+        kvx.kvx_r2_probe(4, 3, 2, 128, 1e6, 1e6, src, src, 1, 256, buf.ctypes.data, None)
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+
+
+def test_select_topk_device_rejects_bad_arguments_before_touching_the_device():
+    buf = np.zeros(16, dtype=np.float64)
+    for (lt, ls, k) in [(0, 4, 1), (3, 0, 1), (3, 4, 0), (3, 4, 5)]:
+        with pytest.raises(kvx.KvxError) as e:
+            kvx.kvx_select_topk_device(buf.ctypes.data, lt, ls, k, buf.ctypes.data)
+        assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+    with pytest.raises(kvx.KvxError):
+        kvx.kvx_select_topk_device(None, 3, 4, 2, buf.ctypes.data)

@@ -116,3 +116,42 @@ def test_fit_headline_shapes_sampled():
     assert np.all(np.isfinite(Wg)) and np.all(np.isfinite(bg))
     systems = [(0, 0, 0), (0, 1, 7), (31, 0, 3), (40, 1, 5), (63, 0, 7), (63, 1, 0)]
     _check_systems(w, 0.01, sel, caches, Wg, bg, systems)
+
+
+def test_fit_caller_workspace_one_pass_and_chunked():
+    """A caller workspace of kvx_fit_workspace_bytes gives the same W and b as the call's own
+    allocation (bit-identical: the same single pass); a workspace that holds 128 tokens of
+    the packed operands runs the tokens in chunks (fp32 partial blocks added), within the
+    oracle tolerance; a workspace below the fixed pieces is refused."""
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=4, Lt=3, H=2, B=2, T=300, k=2)
+    sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
+    caches, W0, b0 = _run_fit(w, 0.01, sel)
+    sk, sv, tk, tv, pos = caches
+    dev = torch.device("cuda:0")
+    posd = torch.from_numpy(pos).to(dev)
+    args = (w.Ls, w.Lt, w.H, w.d, w.k, w.theta_s, w.theta_t, 0.01, sel)
+    full = kvx.kvx_fit_workspace_bytes(*args, w.B, w.T)
+    per64 = kvx.kvx_fit_workspace_bytes(*args, 1, 128) - kvx.kvx_fit_workspace_bytes(*args, 1, 64)
+    assert full > 0 and per64 > 0
+    s = torch.cuda.current_stream().cuda_stream
+    src, tgt = kvx.src_from_tensors(sk, sv), kvx.src_from_tensors(tk, tv)
+
+    def fit(nbytes):
+        ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+        F = w.k * w.d
+        W = torch.full((w.Lt, 2, w.H, F, w.d), float("nan"), dtype=torch.float32, device=dev)
+        b = torch.full((w.Lt, 2, w.H, w.d), float("nan"), dtype=torch.float32, device=dev)
+        kvx.kvx_fit_ridge(*args, src, tgt, w.B, w.T, posd.data_ptr(), W.data_ptr(), b.data_ptr(), s,
+                          workspace_ptr=ws.data_ptr(), workspace_bytes=nbytes)
+        return W.cpu().double().numpy(), b.cpu().double().numpy()
+
+    W1, b1 = fit(full)
+    assert np.array_equal(W1, W0) and np.array_equal(b1, b0)
+    np_full = (w.B * w.T + 63) // 64 * 64
+    W2, b2 = fit(full - (np_full // 64 - 2) * per64)          # two 64-token columns: chunks
+    systems = [(l, kv, h) for l in range(w.Lt) for kv in range(2) for h in range(w.H)]
+    _check_systems(w, 0.01, sel, caches, W2, b2, systems)
+    assert not np.array_equal(W2, W0)          # the chunked run did take another path
+    with pytest.raises(kvx.KvxError) as e:
+        fit(4096)
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG
