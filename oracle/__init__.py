@@ -19,6 +19,8 @@ defines, in float64 numpy, one function per defined quantity:
                    k selected layers, X W + b, re-apply target RoPE (Eq. ridge_kv,
                    Sec. 3.2 concatenation, Sec. 3.3 content-space composition);
                    plus the mapper-size formula of Appendix C.
+* ``mlp``       -- applying the MLP mapper of Sec. 4.3 / Appendix "Run information"
+                   (three Linear layers with ReLU on the cross-head source feature).
 
 Pins (tests/test_oracle_*.py, run with ``-m "not gpu"``) tie each function to
 something other than itself: closed forms, textbook routines, brute force and the

@@ -1,0 +1,99 @@
+"""Pins for oracle.mlp (CPU): the MLP mapper of Sec. 4.3 / Appendix "Run information".
+
+* A worked example with literal numbers (ReLU clipping, layer order, nn.Linear orientation).
+* The ReLU identity relu(z) - relu(-z) = z turns a hidden layer of [A; -A] followed by
+  [I, -I] into the linear map z A^T: the MLP then equals the (separately pinned) ridge
+  mapper oracle.mapper.map_tokens in cross-head mode, keys stripped, bias inside the
+  re-rotation.  A dropped term, a transposed weight, a wrong head or layer order or a
+  rotation in the wrong place breaks it.
+* A dead ReLU layer leaves only the last bias (rotated for keys).
+* bf16fwd mode rounds the hidden activations to bf16 values."""
+import numpy as np
+
+from oracle import bf16, mapper, mlp, rope
+
+
+def test_worked_example():
+    # x = (1, -2); layer 1 (2 -> 3): pre-activations (1 - 2 + 0.5, 2*1 + 0, -1 - 1*(-2) - 3)
+    x = np.array([[1.0, -2.0]])
+    W1 = np.array([[1.0, 1.0], [2.0, 0.0], [-1.0, -1.0]])
+    b1 = np.array([0.5, 0.0, -3.0])          # pre: (-0.5, 2, -2) -> relu (0, 2, 0)
+    W2 = np.array([[1.0, 1.0, 1.0], [0.0, -1.0, 0.0]])
+    b2 = np.array([1.0, 5.0])                # pre: (3, 3) -> relu (3, 3)
+    W3 = np.array([[2.0, -1.0]])
+    b3 = np.array([0.25])                    # 6 - 3 + 0.25
+    y = mlp.mlp_forward(x, W1, b1, W2, b2, W3, b3)
+    assert y.shape == (1, 1) and y[0, 0] == 3.25
+    b2n = np.array([1.0, -5.0])              # second unit clipped: pre (3, -7) -> (3, 0)
+    assert mlp.mlp_forward(x, W1, b1, W2, b2n, W3, b3)[0, 0] == 6.25
+
+
+def _linear_as_mlp(Wlin, b):
+    """W_lin [F][d] (row-vector map x W + b) as MLP weights with hidden = 2d."""
+    F, d = Wlin.shape
+    W1 = np.concatenate([Wlin.T, -Wlin.T], axis=0)          # [2d][F]
+    W2 = np.eye(2 * d)
+    W3 = np.concatenate([np.eye(d), -np.eye(d)], axis=1)    # [d][2d]
+    return W1, np.zeros(2 * d), W2, np.zeros(2 * d), W3, b
+
+
+def test_relu_identity_reduces_to_the_ridge_mapper():
+    rng = np.random.default_rng(5)
+    Ls, Lt, H, N, d, k = 3, 2, 2, 9, 128, 2
+    src_k = rng.standard_normal((Ls, H, N, d))
+    src_v = rng.standard_normal((Ls, H, N, d))
+    pos = rng.integers(0, 5000, size=N)
+    sel = np.array([[0, 2], [1, 2]])
+    F = k * H * d
+    W = rng.standard_normal((Lt, 2, H, F, d)) / np.sqrt(F)
+    b = rng.standard_normal((Lt, 2, H, d))
+    params = {n: [] for n in ("W1", "b1", "W2", "b2", "W3", "b3")}
+    for l in range(Lt):
+        per_l = {n: [] for n in params}
+        for kv in range(2):
+            per_kv = {n: [] for n in params}
+            for h in range(H):
+                for n, v in zip(("W1", "b1", "W2", "b2", "W3", "b3"), _linear_as_mlp(W[l, kv, h], b[l, kv, h])):
+                    per_kv[n].append(v)
+            for n in params:
+                per_l[n].append(per_kv[n])
+        for n in params:
+            params[n].append(per_l[n])
+    params = {n: np.asarray(v) for n, v in params.items()}
+    ok, ov = mlp.map_tokens_mlp(src_k, src_v, pos, sel, params, 1e6, 5e5)
+    rk, rv = mapper.map_tokens(src_k, src_v, pos, sel, W, b, 1e6, 5e5, head_mix="cross_head")
+    assert np.allclose(ok, rk, rtol=0, atol=1e-9) and np.allclose(ov, rv, rtol=0, atol=1e-9)
+
+
+def test_dead_relu_leaves_the_rotated_last_bias():
+    rng = np.random.default_rng(6)
+    Ls, Lt, H, N, d, k, hid = 2, 1, 1, 5, 128, 1, 16
+    src_k = rng.standard_normal((Ls, H, N, d))
+    src_v = rng.standard_normal((Ls, H, N, d))
+    pos = np.arange(N) * 37
+    sel = np.array([[1]])
+    F = k * H * d
+    b3 = rng.standard_normal((Lt, 2, H, d))
+    params = dict(W1=rng.standard_normal((Lt, 2, H, hid, F)) * 0.01, b1=np.full((Lt, 2, H, hid), -1e3),
+                  W2=rng.standard_normal((Lt, 2, H, hid, hid)), b2=np.zeros((Lt, 2, H, hid)),
+                  W3=rng.standard_normal((Lt, 2, H, d, hid)), b3=b3)
+    ok, ov = mlp.map_tokens_mlp(src_k, src_v, pos, sel, params, 1e6, 1e6)
+    assert np.array_equal(ov[0, 0], np.broadcast_to(b3[0, 1, 0], (N, d)))
+    want_k = rope.rotate(np.broadcast_to(b3[0, 0, 0], (N, d)), pos, 1e6)
+    assert np.allclose(ok[0, 0], want_k, rtol=0, atol=1e-12)
+
+
+def test_bf16fwd_rounds_hidden_activations():
+    rng = np.random.default_rng(8)
+    X = rng.standard_normal((7, 5))
+    W1, b1 = rng.standard_normal((6, 5)), rng.standard_normal(6)
+    W2, b2 = rng.standard_normal((6, 6)), rng.standard_normal(6)
+    W3, b3 = rng.standard_normal((2, 6)), np.zeros(2)
+    # with W3 = identity rows the output exposes the second hidden activation
+    W3e = np.eye(6)
+    h2 = mlp.mlp_forward(X, W1, b1, W2, b2, W3e, np.zeros(6), round_hidden=True)
+    assert np.array_equal(h2, bf16.round_to_bf16_value(h2))
+    exact = mlp.mlp_forward(X, W1, b1, W2, b2, W3, b3)
+    rounded = mlp.mlp_forward(X, W1, b1, W2, b2, W3, b3, round_hidden=True)
+    assert not np.array_equal(exact, rounded)
+    assert np.allclose(exact, rounded, rtol=0.05, atol=0.05)
