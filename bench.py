@@ -434,6 +434,78 @@ def probe_bench(args, w):
     return 0
 
 
+MLP_HIDDEN = 1024   # the paper's MLP baseline width
+
+
+def mlp_bench(args, w):
+    """MLP mapper apply (kvx_mlp_map): the three-layer ReLU MLP per (target layer, K|V, head)
+    on the cross-head source feature, synthetic seeded weights on the device.  One step =
+    one kvx_mlp_map call (key strip + three GEMM passes, synchronous) with a caller
+    workspace.  Roofline: tensor-bound, the GEMM FLOPs against the measured bf16 peak."""
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(0)
+    sp = torch.cuda.current_stream(dev).cuda_stream
+    sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+    pos = torch.from_numpy(syn.positions(w)).to(dev)
+    sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
+    hid, ds = MLP_HIDDEN, w.k * w.H * w.d
+    g = torch.Generator(device=dev).manual_seed(w.seed + 77)
+    shape = (w.Lt, 2, w.H)
+    P = dict(W1=torch.randn(*shape, hid, ds, generator=g, device=dev, dtype=torch.bfloat16).mul_(ds ** -0.5),
+             b1=torch.randn(*shape, hid, generator=g, device=dev).mul_(0.1),
+             W2=torch.randn(*shape, hid, hid, generator=g, device=dev, dtype=torch.bfloat16).mul_((2.0 / hid) ** 0.5),
+             b2=torch.randn(*shape, hid, generator=g, device=dev).mul_(0.1),
+             W3=torch.randn(*shape, w.d, hid, generator=g, device=dev, dtype=torch.bfloat16).mul_((2.0 / hid) ** 0.5),
+             b3=torch.randn(*shape, w.d, generator=g, device=dev).mul_(0.1))
+    tk = torch.empty((w.Lt, w.B, w.H, w.T, w.d), dtype=torch.bfloat16, device=dev)
+    tv = torch.empty_like(tk)
+    cfg = kvx.mlp_config(w.Ls, w.Lt, w.H, w.d, w.k, hid, w.theta_s, w.theta_t, sel,
+                         *(P[n].data_ptr() for n in ("W1", "b1", "W2", "b2", "W3", "b3")))
+    ws_bytes = kvx.kvx_mlp_workspace_bytes(cfg, w.B, w.T)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    cfg.workspace, cfg.workspace_bytes = ws.data_ptr(), ws_bytes
+    src, tgt = kvx.src_from_tensors(sk, sv), kvx.tgt_from_tensors(tk, tv)
+
+    def step():
+        kvx.kvx_mlp_map(cfg, src, w.B, w.T, pos.data_ptr(), tgt, sp)
+
+    for _ in range(args.warmup):
+        step()
+    steps = max(1, min(args.steps, 10))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(0) as clk:
+        torch.cuda.synchronize()
+        e0.record()
+        for _ in range(steps):
+            step()
+        e1.record()
+        torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    N = w.n_tokens
+    n_sys = w.Lt * 2 * w.H
+    flop = n_sys * N * 2.0 * (ds * hid + hid * hid + hid * w.d)
+    achieved = flop / (ms / 1e3) / 1e12
+    pk = load_peaks()
+    line = {"metric": "MLP-mapper tokens/s", "value": N / (ms / 1e3), "unit": "tokens/s", "n_gpus": 1,
+            "steps": steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16 (fp32 accumulate)", "data": "synthetic",
+            "config": {"workload": w.name + " (MLP mapper)", "src_layers": w.Ls, "tgt_layers": w.Lt,
+                       "kv_heads": w.H, "head_dim": w.d, "k": w.k, "hidden": hid, "d_s": ds, "batch": w.B,
+                       "seq_len": w.T, "weights_gb": sum(t.numel() * t.element_size() for t in P.values()) / 1e9,
+                       "workspace_gb": ws_bytes / 1e9,
+                       "l2": "no flush: each step reads %.1f GB of weights vs 129 MB L2" % (
+                           sum(t.numel() * t.element_size() for t in P.values()) / 1e9)},
+            "clocks": clk.summary(),
+            "gpu_launches": 4 * steps,
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": pk["bf16"], "unit": "TFLOP/s",
+                         "frac": achieved / pk["bf16"], "traffic": None, "kernel": "tc_mlp_kernel (3 passes) + strip",
+                         "peak_source": pk["source"] + " bf16 burst",
+                         "algorithmic": {"flop_per_step": flop, "flop_per_token": flop / N}},
+            "kernel": "xh_strip_kernel + tc_mlp_kernel x 3"}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -445,6 +517,8 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=None)
     ap.add_argument("--fit", action="store_true",
                     help="time the ridge fit (kvx_fit_ridge) on the workload's shapes instead of the map")
+    ap.add_argument("--mlp", action="store_true",
+                    help="time the MLP mapper apply (kvx_mlp_map, hidden 1024) on the workload's shapes")
     ap.add_argument("--probe", action="store_true",
                     help="time the single-source R^2 probe (kvx_r2_probe) on the workload's shapes")
     args = ap.parse_args()
@@ -454,6 +528,8 @@ def main():
         return fit_bench(args, w)
     if args.probe:
         return probe_bench(args, w)
+    if args.mlp:
+        return mlp_bench(args, w)
     alg = algorithmic(w)
     config = {"workload": w.name, "src_layers": w.Ls, "tgt_layers": w.Lt, "kv_heads": w.H,
               "head_dim": w.d, "k": w.k, "batch": w.B, "seq_len": w.T, "tokens_per_step": w.n_tokens,

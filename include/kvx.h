@@ -255,6 +255,42 @@ KVX_API int64_t kvx_r2_probe_workspace_bytes(const kvx_probe_config* cfg, int32_
 KVX_API kvx_status kvx_select_topk_device(const double* scores, int32_t tgt_layers, int32_t src_layers, int32_t k,
                                           int32_t* out, void* stream);
 
+/* MLP mapper apply (Sec. 4.3; Appendix "Run information", MLP baseline architecture):
+ * for every target layer l, K|V and head h,
+ *   y = W3 relu(W2 relu(W1 x + b1) + b2) + b3
+ * (weights in the nn.Linear layout [out][in]) on the cross-head source feature x: the k
+ * selected source layers (selection[l], in order) with all H heads each, head-minor,
+ * d_s = k H d; keys with the source RoPE stripped and rounded to bf16, values as stored.
+ * Keys are re-rotated with the target RoPE after b3.  Accumulation in fp32 on the tensor
+ * cores, each hidden activation stored in bf16 after its ReLU, output rounded once to
+ * bf16.  bf16 caches and weights, head_dim 128, half-split pairs, hidden a multiple of 256,
+ * contiguous targets (UNSUPPORTED for paged).  Weights and biases are DEVICE pointers:
+ *   W1 bf16 [L_t][2][H][hidden][d_s]    b1 fp32 [L_t][2][H][hidden]
+ *   W2 bf16 [L_t][2][H][hidden][hidden] b2 fp32 [L_t][2][H][hidden]
+ *   W3 bf16 [L_t][2][H][d][hidden]      b3 fp32 [L_t][2][H][d]
+ * (index 0 of the second axis = K), 16-byte aligned.  Workspace: the stripped source
+ * keys and two hidden buffers of 2 B T H hidden bf16 per target layer; from cfg->workspace
+ * (kvx_mlp_workspace_bytes: all target layers at once; less processes the target layers
+ * in groups) or allocated stream-ordered.  Runs on `stream` and synchronises it, returning
+ * the device status (DEVICE_BOUNDS for a position outside [0, 2^24), TIMEOUT if a wait of
+ * the kernel ran out).  batch == 0 or tokens_per_seq == 0 is a no-op. */
+typedef struct {
+  int32_t src_layers, tgt_layers, n_kv_heads, head_dim, k, hidden;
+  double src_rope_theta, tgt_rope_theta;
+  const int32_t* selection;      /* host [tgt_layers][k], entries in [0, src_layers) */
+  const void* W1;
+  const float* b1;
+  const void* W2;
+  const float* b2;
+  const void* W3;
+  const float* b3;
+  void* workspace;               /* device, 256-byte aligned, or NULL (the call allocates) */
+  uint64_t workspace_bytes;
+} kvx_mlp_config;
+KVX_API kvx_status kvx_mlp_map(const kvx_mlp_config* cfg, const kvx_src* src, int32_t batch, int32_t tokens_per_seq,
+                               const int32_t* positions, const kvx_tgt* tgt, void* stream);
+KVX_API int64_t kvx_mlp_workspace_bytes(const kvx_mlp_config* cfg, int32_t batch, int32_t tokens_per_seq);
+
 /* Device time in milliseconds of the phases of the last successful kvx_fit_ridge or
  * kvx_r2_probe call on this thread, from CUDA events on the call's stream: ms[0] column
  * sums, ms[1] operand packing, ms[2] tensor-core Gram blocks, ms[3] the solves (fit) or

@@ -41,6 +41,7 @@
 #include "kvx_internal.h"
 #include "kvx_ptx.cuh"
 #include "kvx_rope.cuh"
+#include "kvx_xh.h"
 
 namespace kvx {
 namespace {
@@ -147,30 +148,6 @@ __global__ void __launch_bounds__(256) xh_strip_kernel(const __nv_bfloat16* __re
       }
     }
   }
-}
-
-// Pair MMA with A and B both in shared memory (each CTA supplies its 128 rows of A and
-// its half of B's rows at the same offsets).  Issued by the rank-0 CTA.
-__device__ __forceinline__ void tc_mma_ss_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
-                                               uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
-// 5D tile load into this CTA's shared memory, completing on an mbarrier that may live in
-// the peer CTA (shared::cluster address).
-__device__ __forceinline__ void tma_load_5d_pair(uint32_t dst, const CUtensorMap* map, uint32_t bar_cluster, int c0,
-                                                 int c1, int c2, int c3, int c4, uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.5d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.cta_group::2.L2::cache_hint"
-      " [%0], [%1, {%2, %3, %4, %5, %6}], [%7], %8;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4), "r"(bar_cluster),
-      "l"(policy)
-      : "memory");
 }
 
 // -------------------------------------------------------------- mapping kernel --
@@ -515,6 +492,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
 
 }  // namespace
 
+void launch_key_strip(const void* src_k, const int64_t* ss, void* ws, const int32_t* pos, int Ls, int H, int B, int T,
+                      const RopeTables& rope, int sms, cudaStream_t stream) {
+  const int64_t threads = static_cast<int64_t>(B) * T * 16;
+  const int blocks = static_cast<int>(std::min<int64_t>((threads + 255) / 256, static_cast<int64_t>(sms) * 8));
+  xh_strip_kernel<<<blocks, 256, 0, stream>>>(static_cast<const __nv_bfloat16*>(src_k), ss[0], ss[1], ss[2], ss[3],
+                                              static_cast<__nv_bfloat16*>(ws), pos, Ls, H, B, T, rope);
+}
+
 bool xh_supported(const kvx_ctx* c, std::string* why) {
   std::string w;
   if (c->cache_dtype != KVX_BF16 || c->weight_dtype != KVX_BF16) w = "needs bf16 caches and weights";
@@ -633,11 +618,7 @@ kvx_status launch_xh(kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
 
   // 1. strip the source RoPE from every key into the workspace
   {
-    const int64_t threads = static_cast<int64_t>(a.B) * a.T * 16;
-    const int blocks = static_cast<int>(std::min<int64_t>((threads + 255) / 256, static_cast<int64_t>(c->sm_count) * 8));
-    xh_strip_kernel<<<blocks, 256, 0, stream>>>(static_cast<const __nv_bfloat16*>(a.src_k), a.ss[0], a.ss[1], a.ss[2],
-                                                a.ss[3], static_cast<__nv_bfloat16*>(c->d_ws), a.pos, c->Ls, c->H,
-                                                a.B, a.T, c->rope);
+    launch_key_strip(a.src_k, a.ss, c->d_ws, a.pos, c->Ls, c->H, a.B, a.T, c->rope, c->sm_count, stream);
     if ((e = cudaGetLastError()) != cudaSuccess) {
       set_error(std::string("kvx_map: strip launch: ") + cudaGetErrorString(e));
       return KVX_ERR_CUDA;

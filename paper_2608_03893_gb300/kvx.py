@@ -84,12 +84,26 @@ class kvx_probe_config(ctypes.Structure):
     ]
 
 
+class kvx_mlp_config(ctypes.Structure):
+    _fields_ = [
+        ("src_layers", ctypes.c_int32), ("tgt_layers", ctypes.c_int32),
+        ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("k", ctypes.c_int32),
+        ("hidden", ctypes.c_int32),
+        ("src_rope_theta", ctypes.c_double), ("tgt_rope_theta", ctypes.c_double),
+        ("selection", ctypes.c_void_p),
+        ("W1", ctypes.c_void_p), ("b1", ctypes.c_void_p), ("W2", ctypes.c_void_p), ("b2", ctypes.c_void_p),
+        ("W3", ctypes.c_void_p), ("b3", ctypes.c_void_p),
+        ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_uint64),
+    ]
+
+
 _lib = None
 
 EXPORTED = ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
             "kvx_set_kernel", "kvx_get_status", "kvx_mapper_params", "kvx_status_string",
             "kvx_last_error", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms", "kvx_r2_probe",
-            "kvx_select_topk_device", "kvx_fit_workspace_bytes", "kvx_r2_probe_workspace_bytes")
+            "kvx_select_topk_device", "kvx_fit_workspace_bytes", "kvx_r2_probe_workspace_bytes",
+            "kvx_mlp_map", "kvx_mlp_workspace_bytes")
 
 
 def lib():
@@ -127,9 +141,13 @@ def lib():
     L.kvx_fit_workspace_bytes.restype = i64
     L.kvx_r2_probe_workspace_bytes.argtypes = [ctypes.POINTER(kvx_probe_config), i32, i32]
     L.kvx_r2_probe_workspace_bytes.restype = i64
+    L.kvx_mlp_map.argtypes = [ctypes.POINTER(kvx_mlp_config), ctypes.POINTER(kvx_src), i32, i32, vp,
+                              ctypes.POINTER(kvx_tgt), vp]
+    L.kvx_mlp_workspace_bytes.argtypes = [ctypes.POINTER(kvx_mlp_config), i32, i32]
+    L.kvx_mlp_workspace_bytes.restype = i64
     for name in ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
                  "kvx_set_kernel", "kvx_get_status", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms",
-                 "kvx_r2_probe", "kvx_select_topk_device"):
+                 "kvx_r2_probe", "kvx_select_topk_device", "kvx_mlp_map"):
         getattr(L, name).restype = ctypes.c_int
     _lib = L
     return L
@@ -373,3 +391,26 @@ def kvx_select_topk_device(scores_ptr, tgt_layers, src_layers, k, out_ptr, strea
     int32 [L_t][k] (rows ascending, ties to the lower source index)."""
     _check(lib().kvx_select_topk_device(scores_ptr, int(tgt_layers), int(src_layers), int(k), out_ptr, stream),
            "kvx_select_topk_device")
+
+
+def mlp_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, hidden, theta_s, theta_t, selection,
+               W1_ptr, b1_ptr, W2_ptr, b2_ptr, W3_ptr, b3_ptr, workspace_ptr=None, workspace_bytes=0):
+    """kvx_mlp_config for kvx_mlp_map (weights and biases DEVICE pointers, see include/kvx.h).
+    The returned config keeps the host selection array alive."""
+    import numpy as np
+    sel = np.ascontiguousarray(selection, dtype=np.int32)
+    cfg = kvx_mlp_config(int(src_layers), int(tgt_layers), int(n_kv_heads), int(head_dim), int(k), int(hidden),
+                         float(theta_s), float(theta_t), _ptr(sel), W1_ptr, b1_ptr, W2_ptr, b2_ptr, W3_ptr,
+                         b3_ptr, workspace_ptr, int(workspace_bytes))
+    cfg._sel = sel
+    return cfg
+
+
+def kvx_mlp_workspace_bytes(cfg, batch, tokens_per_seq):
+    return int(lib().kvx_mlp_workspace_bytes(ctypes.byref(cfg), int(batch), int(tokens_per_seq)))
+
+
+def kvx_mlp_map(cfg, src, batch, tokens_per_seq, positions_ptr, tgt, stream=0):
+    """MLP mapper apply (see include/kvx.h); blocks until done."""
+    _check(lib().kvx_mlp_map(ctypes.byref(cfg), ctypes.byref(src), int(batch), int(tokens_per_seq),
+                             positions_ptr, ctypes.byref(tgt), stream), "kvx_mlp_map")

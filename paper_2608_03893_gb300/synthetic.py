@@ -161,6 +161,9 @@ WORKLOADS = {
                                               1e6, 1e6, "bf16", "bf16", "depth", 0.01, 2, head_mix="cross_head"),
     "qwen3_14b_32b_t32768_k8_xhead": Workload("qwen3_14b_32b_t32768_k8_xhead", 40, 64, 8, 128, 8, 1, 32768,
                                               1e6, 1e6, "bf16", "bf16", "depth", 0.01, 2, head_mix="cross_head"),
+    # the MLP mapper's shapes (cross-head d_s = 4096, hidden 1024): 11 GFLOP per token, 45 TFLOP a step
+    "qwen3_14b_32b_b1x4096_k4_xhead": Workload("qwen3_14b_32b_b1x4096_k4_xhead", 40, 64, 8, 128, 4, 1, 4096,
+                                              1e6, 1e6, "bf16", "bf16", "depth", 0.01, 3, head_mix="cross_head"),
 }
 
 HEADLINE = "qwen3_14b_32b_t32768_k4"

@@ -198,3 +198,39 @@ def test_select_topk_device_rejects_bad_arguments_before_touching_the_device():
         assert e.value.status == kvx.KVX_ERR_INVALID_ARG
     with pytest.raises(kvx.KvxError):
         kvx.kvx_select_topk_device(None, 3, 4, 2, buf.ctypes.data)
+
+
+def test_mlp_map_rejects_bad_arguments_before_touching_the_device():
+    """kvx_mlp_map validates its configuration on the host first."""
+    buf = np.zeros(64, dtype=np.float64)
+    p = buf.ctypes.data
+    sel = np.array([[0, 1], [1, 2]], dtype=np.int32)
+    good = dict(src_layers=3, tgt_layers=2, n_kv_heads=2, head_dim=128, k=2, hidden=256, theta_s=1e6, theta_t=1e6,
+                selection=sel)
+    src = kvx.kvx_src(p, p, (ctypes.c_int64 * 4)(4096, 4096, 256, 128))
+    tgt = kvx.kvx_tgt()
+    tgt.k, tgt.v = p, p
+    for i, s in enumerate((4096, 4096, 256, 128)):
+        tgt.stride[i] = s
+    cases = [dict(head_dim=64), dict(hidden=100), dict(hidden=0), dict(k=0), dict(k=4), dict(theta_t=0.5),
+             dict(selection=np.array([[0, 3], [1, 2]], dtype=np.int32)), dict(n_kv_heads=0)]
+    for over in cases:
+        a = dict(good, **over)
+        cfg = kvx.mlp_config(a["src_layers"], a["tgt_layers"], a["n_kv_heads"], a["head_dim"], a["k"], a["hidden"],
+                             a["theta_s"], a["theta_t"], a["selection"], p, p, p, p, p, p)
+        with pytest.raises(kvx.KvxError) as e:
+            kvx.kvx_mlp_map(cfg, src, 1, 16, p, tgt)
+        assert e.value.status == kvx.KVX_ERR_INVALID_ARG, over
+        assert kvx.kvx_mlp_workspace_bytes(cfg, 1, 16) == -1
+    cfg = kvx.mlp_config(3, 2, 2, 128, 2, 256, 1e6, 1e6, sel, p, p, None, p, p, p)   # NULL W2
+    with pytest.raises(kvx.KvxError):
+        kvx.kvx_mlp_map(cfg, src, 1, 16, p, tgt)
+    cfg = kvx.mlp_config(3, 2, 2, 128, 2, 256, 1e6, 1e6, sel, p, p, p, p, p, p)
+    assert kvx.kvx_mlp_workspace_bytes(cfg, 1, 16) > 0
+    paged = kvx.kvx_tgt()
+    paged.paged, paged.block_size, paged.k, paged.v = 1, 16, p, p
+    for i, s in enumerate((4096, 4096, 256, 128)):
+        paged.stride[i] = s
+    with pytest.raises(kvx.KvxError) as e:
+        kvx.kvx_mlp_map(cfg, src, 1, 16, p, paged)
+    assert e.value.status == kvx.KVX_ERR_UNSUPPORTED
