@@ -75,6 +75,18 @@ typedef enum { KVX_PER_HEAD = 0, KVX_CROSS_HEAD = 1 } kvx_head_mix;
  * kvx_destroy frees it. */
 typedef enum { KVX_KERNEL_AUTO = 0, KVX_KERNEL_SIMT = 1, KVX_KERNEL_TCGEN05 = 2 } kvx_kernel;
 
+/* Llama-3 RoPE frequency scaling (the rope_scaling of the Llama 3.1 checkpoints:
+ * factor 8, low_freq_factor 1, high_freq_factor 4, original_max_position 8192).  With
+ * omega_i = theta^(-2i/d) and wavelength 2 pi / omega_i: below original_max_position /
+ * high_freq_factor omega_i is kept, above original_max_position / low_freq_factor it is
+ * divided by factor, and in between it is (1 - s) omega_i / factor + s omega_i with
+ * s = (original_max_position / wavelength - low_freq_factor) / (high_freq_factor -
+ * low_freq_factor).  The paper uses Llama 3.1 pairs but does not discuss the scaling; a
+ * NULL pointer below means plain theta.  factor >= 1, 0 < low < high, position > 0. */
+typedef struct {
+  double factor, low_freq_factor, high_freq_factor, original_max_position;
+} kvx_rope_scaling;
+
 /* Mapper description, read by kvx_create.  All pointers are HOST pointers; the
  * context copies what it needs, so they may be freed when kvx_create returns. */
 typedef struct {
@@ -100,6 +112,9 @@ typedef struct {
   /* [L_t][2][n_kv][d] in weight_dtype, or NULL for a zero bias (Sec. 3.1: the
    * centred fit gives b = mean(Y) - mean(X) W*). */
   const void* b;
+  /* RoPE frequency scaling of the source / target model, or NULL (plain theta). */
+  const kvx_rope_scaling* src_rope_scaling;
+  const kvx_rope_scaling* tgt_rope_scaling;
 } kvx_config;
 
 /* Source cache, DEVICE memory owned by the caller: element (layer l, batch b, head h,
@@ -208,6 +223,8 @@ typedef struct {
   void* workspace;               /* device, 256-byte aligned, or NULL (the call allocates) */
   uint64_t workspace_bytes;      /* its size; kvx_fit_workspace_bytes gives the size that
                                   * holds every token in one pass (less: tokens in chunks) */
+  const kvx_rope_scaling* src_rope_scaling;   /* NULL: plain theta (see kvx_rope_scaling) */
+  const kvx_rope_scaling* tgt_rope_scaling;
 } kvx_fit_config;
 KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, const kvx_src* tgt, int32_t batch,
                                  int32_t tokens_per_seq, const int32_t* positions, float* W, float* b,
@@ -243,6 +260,8 @@ typedef struct {
   double src_rope_theta, tgt_rope_theta;
   void* workspace;               /* device, 256-byte aligned, or NULL (the call allocates) */
   uint64_t workspace_bytes;
+  const kvx_rope_scaling* src_rope_scaling;   /* NULL: plain theta (see kvx_rope_scaling) */
+  const kvx_rope_scaling* tgt_rope_scaling;
 } kvx_probe_config;
 KVX_API kvx_status kvx_r2_probe(const kvx_probe_config* cfg, const kvx_src* src, const kvx_src* tgt, int32_t batch,
                                 int32_t tokens_per_seq, const int32_t* positions, double* scores, double* r2_kv,
@@ -286,6 +305,8 @@ typedef struct {
   const float* b3;
   void* workspace;               /* device, 256-byte aligned, or NULL (the call allocates) */
   uint64_t workspace_bytes;
+  const kvx_rope_scaling* src_rope_scaling;   /* NULL: plain theta (see kvx_rope_scaling) */
+  const kvx_rope_scaling* tgt_rope_scaling;
 } kvx_mlp_config;
 KVX_API kvx_status kvx_mlp_map(const kvx_mlp_config* cfg, const kvx_src* src, int32_t batch, int32_t tokens_per_seq,
                                const int32_t* positions, const kvx_tgt* tgt, void* stream);
@@ -339,6 +360,8 @@ typedef struct {
   const int32_t* selection;    /* HOST [L_t][k], distinct layers in [0, L_s); row block j of W <-> selection[l][j] */
   const void* W;               /* DEVICE [L_t][2][n_kv][F][d] in weight_dtype, 16-byte aligned */
   const float* b;              /* DEVICE fp32 [L_t][2][n_kv][d] (pass zeros for no bias), 16-byte aligned */
+  const kvx_rope_scaling* src_rope_scaling;   /* NULL: plain theta */
+  const kvx_rope_scaling* tgt_rope_scaling;
 } kvx_noalloc_mapper;
 
 /* Map as kvx_map does, allocating nothing.  src, tgt, positions, batch and

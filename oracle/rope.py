@@ -11,14 +11,50 @@ t * omega_i with omega_i = theta^(-2i/d), i = 0 .. d/2-1, as the complex product
 Pair layout (the paper does not state one):
 * ``"half"``        -- pairs (i, i + d/2): the layout of the Qwen3 / Llama checkpoints.
 * ``"interleaved"`` -- pairs (2i, 2i+1).
+
+Frequency scaling.  The Llama 3.1 checkpoints of the paper's Llama pairs rescale the
+inverse frequencies ("llama3" rope scaling, published with those checkpoints; the paper
+itself does not discuss it).  ``theta`` may be a plain base or a ``RopeSpec`` carrying such
+a scaling; every function here accepts either.
 """
+from typing import NamedTuple, Optional
+
 import numpy as np
 
 
+class Llama3Scaling(NamedTuple):
+    factor: float                   # long wavelengths are divided by this
+    low_freq_factor: float
+    high_freq_factor: float
+    original_max_position: float    # context length the model was pre-trained with
+
+
+class RopeSpec(NamedTuple):
+    theta: float
+    scaling: Optional[Llama3Scaling] = None
+
+
+def llama3_scale(omega, s):
+    """Scaled inverse frequencies: with wavelength lam = 2 pi / omega, keep omega where
+    lam < P / high_freq_factor, divide by factor where lam > P / low_freq_factor, and in
+    between blend (1 - a) omega / factor + a omega with a = (P / lam - low_freq_factor) /
+    (high_freq_factor - low_freq_factor); P = original_max_position."""
+    omega = np.asarray(omega, dtype=np.float64)
+    lam = 2.0 * np.pi / omega
+    P = float(s.original_max_position)
+    a = (P / lam - s.low_freq_factor) / (s.high_freq_factor - s.low_freq_factor)
+    blend = (1.0 - a) * omega / s.factor + a * omega
+    out = np.where(lam < P / s.high_freq_factor, omega, blend)
+    return np.where(lam > P / s.low_freq_factor, omega / s.factor, out)
+
+
 def inv_freq(theta, d):
-    """omega_i = theta^(-2i/d) for i in [0, d/2), float64."""
+    """omega_i = theta^(-2i/d) for i in [0, d/2), float64 (scaled when ``theta`` is a
+    RopeSpec with a scaling)."""
+    spec = theta if isinstance(theta, RopeSpec) else RopeSpec(float(theta))
     i = np.arange(d // 2, dtype=np.float64)
-    return np.power(np.float64(theta), -2.0 * i / d)
+    omega = np.power(np.float64(spec.theta), -2.0 * i / d)
+    return omega if spec.scaling is None else llama3_scale(omega, spec.scaling)
 
 
 def angles(positions, theta, d):

@@ -277,6 +277,8 @@ const char* check_fit_config(const kvx_fit_config* cfg) {
   for (int64_t i = 0; i < static_cast<int64_t>(cfg->tgt_layers) * cfg->k; ++i)
     if (cfg->selection[i] < 0 || cfg->selection[i] >= cfg->src_layers) return "selection entry out of range";
   if (cfg->workspace_bytes != 0 && !cfg->workspace) return "workspace_bytes without a workspace";
+  if (const char* why = check_rope_scaling(cfg->src_rope_scaling)) return why;
+  if (const char* why = check_rope_scaling(cfg->tgt_rope_scaling)) return why;
   if (reinterpret_cast<uintptr_t>(cfg->workspace) & 255u) return "workspace must be 256-byte aligned";
   return nullptr;
 }
@@ -341,6 +343,7 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
   tmp.d = kFD;
   tmp.theta_s = cfg->src_rope_theta;
   tmp.theta_t = cfg->tgt_rope_theta;
+  set_rope_scaling(&tmp, cfg->src_rope_scaling, cfg->tgt_rope_scaling);
   fill_rope(&tmp);
 
   GramSpec G;

@@ -59,11 +59,43 @@ static float bf16_to_float(uint16_t v) {
   return f;
 }
 
+const char* check_rope_scaling(const kvx_rope_scaling* s) {
+  if (!s) return nullptr;
+  if (!(s->factor >= 1.0) || !std::isfinite(s->factor)) return "rope scaling factor must be finite and >= 1";
+  if (!(s->low_freq_factor > 0.0) || !(s->high_freq_factor > s->low_freq_factor) ||
+      !std::isfinite(s->high_freq_factor))
+    return "rope scaling needs 0 < low_freq_factor < high_freq_factor";
+  if (!(s->original_max_position > 0.0) || !std::isfinite(s->original_max_position))
+    return "rope scaling original_max_position must be > 0";
+  return nullptr;
+}
+
+void set_rope_scaling(kvx_ctx* c, const kvx_rope_scaling* src, const kvx_rope_scaling* tgt) {
+  c->scale_s_on = src != nullptr;
+  c->scale_t_on = tgt != nullptr;
+  if (src) c->scale_s = *src;
+  if (tgt) c->scale_t = *tgt;
+}
+
+// Llama-3 scaling of one inverse frequency (kvx_rope_scaling in kvx.h), in double.
+static double scaled_omega(double w, const kvx_rope_scaling& s) {
+  const double two_pi = 6.283185307179586476925286766559;
+  const double wavelen = two_pi / w;
+  const double lo_wavelen = s.original_max_position / s.low_freq_factor;
+  const double hi_wavelen = s.original_max_position / s.high_freq_factor;
+  if (wavelen < hi_wavelen) return w;
+  if (wavelen > lo_wavelen) return w / s.factor;
+  const double sm = (s.original_max_position / wavelen - s.low_freq_factor) / (s.high_freq_factor - s.low_freq_factor);
+  return (1.0 - sm) * w / s.factor + sm * w;
+}
+
 void fill_rope(kvx_ctx* c) {
   const int half = c->d / 2;
   for (int i = 0; i < half; ++i) {
     const double e = -2.0 * i / c->d;
-    const double ws = std::pow(c->theta_s, e), wt = std::pow(c->theta_t, e);
+    double ws = std::pow(c->theta_s, e), wt = std::pow(c->theta_t, e);
+    if (c->scale_s_on) ws = scaled_omega(ws, c->scale_s);
+    if (c->scale_t_on) wt = scaled_omega(wt, c->scale_t);
     c->rope.ws_hi[i] = static_cast<float>(ws);
     c->rope.ws_lo[i] = static_cast<float>(ws - static_cast<double>(c->rope.ws_hi[i]));
     c->rope.wt_hi[i] = static_cast<float>(wt);
@@ -153,6 +185,10 @@ kvx_status kvx_create(const kvx_config* cfg, int device, kvx_ctx** out) {
   if (c.head_mix != KVX_PER_HEAD && c.head_mix != KVX_CROSS_HEAD)
     return fail(KVX_ERR_INVALID_ARG, "kvx_create: bad head_mix");
   if (c.reserved != 0) return fail(KVX_ERR_INVALID_ARG, "kvx_create: reserved must be 0");
+  if (const char* why = check_rope_scaling(c.src_rope_scaling))
+    return fail(KVX_ERR_INVALID_ARG, std::string("kvx_create: source ") + why);
+  if (const char* why = check_rope_scaling(c.tgt_rope_scaling))
+    return fail(KVX_ERR_INVALID_ARG, std::string("kvx_create: target ") + why);
   if (!(c.src_rope_theta > 1.0) || !(c.tgt_rope_theta > 1.0) || !std::isfinite(c.src_rope_theta) ||
       !std::isfinite(c.tgt_rope_theta))
     return fail(KVX_ERR_INVALID_ARG, "kvx_create: rope thetas must be finite and > 1");
@@ -199,6 +235,7 @@ kvx_status kvx_create(const kvx_config* cfg, int device, kvx_ctx** out) {
       return s;
     }
   }
+  set_rope_scaling(ctx, c.src_rope_scaling, c.tgt_rope_scaling);
   fill_rope(ctx);
 
   DeviceGuard guard(device);

@@ -60,6 +60,8 @@ struct kvx_ctx {
   int Ls = 0, Lt = 0, H = 0, d = 0, k = 0, F = 0;
   int rope_style = 0, cache_dtype = 0, weight_dtype = 0, head_mix = 0;
   double theta_s = 0, theta_t = 0;
+  bool scale_s_on = false, scale_t_on = false;   // Llama-3 frequency scaling per side
+  kvx_rope_scaling scale_s{}, scale_t{};
   int kernel = KVX_KERNEL_AUTO;
   bool tc_eligible = false;
   bool xh_eligible = false;         // cross-head tensor-core kernel
@@ -81,7 +83,12 @@ struct kvx_ctx {
 namespace kvx {
 void set_error(const std::string& msg);
 
-// Fills ctx->rope from ctx->d, ctx->theta_s and ctx->theta_t.
+// NULL if the scaling (or NULL) is valid, else why not.
+const char* check_rope_scaling(const kvx_rope_scaling* s);
+// Copies the two optional scalings into the context (after check_rope_scaling).
+void set_rope_scaling(kvx_ctx* c, const kvx_rope_scaling* src, const kvx_rope_scaling* tgt);
+
+// Fills ctx->rope from ctx->d, ctx->theta_s, ctx->theta_t and the optional scalings.
 void fill_rope(kvx_ctx* c);
 
 // SIMT fp32 kernel (any head_dim <= 256, fp32 or bf16 caches/weights, both layouts).

@@ -392,6 +392,8 @@ const char* check_mlp_config(const kvx_mlp_config* c) {
   if (static_cast<int64_t>(c->tgt_layers) * 2 * c->n_kv_heads * c->hidden > INT_MAX / 2) return "too many weight rows";
   if (static_cast<int64_t>(c->k) * c->n_kv_heads * kMD > INT_MAX / 2) return "source feature too wide";
   if (c->workspace_bytes != 0 && !c->workspace) return "workspace_bytes without a workspace";
+  if (const char* why = check_rope_scaling(c->src_rope_scaling)) return why;
+  if (const char* why = check_rope_scaling(c->tgt_rope_scaling)) return why;
   if (reinterpret_cast<uintptr_t>(c->workspace) & 255u) return "workspace must be 256-byte aligned";
   return nullptr;
 }
@@ -516,6 +518,7 @@ KVX_API kvx_status kvx_mlp_map(const kvx_mlp_config* cfg, const kvx_src* src, in
     tmp.d = kMD;
     tmp.theta_s = cfg->src_rope_theta;
     tmp.theta_t = cfg->tgt_rope_theta;
+    set_rope_scaling(&tmp, cfg->src_rope_scaling, cfg->tgt_rope_scaling);
     fill_rope(&tmp);
     MlpParams P;
     std::memset(&P, 0, sizeof(P));

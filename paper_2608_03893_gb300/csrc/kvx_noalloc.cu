@@ -72,6 +72,10 @@ extern "C" KVX_API kvx_status kvx_map_noalloc(const kvx_noalloc_mapper* m, int d
   if (!(m->src_rope_theta > 1.0) || !(m->tgt_rope_theta > 1.0) || !std::isfinite(m->src_rope_theta) ||
       !std::isfinite(m->tgt_rope_theta))
     return fail(KVX_ERR_INVALID_ARG, "kvx_map_noalloc: rope thetas must be finite and > 1");
+  if (const char* why = kvx::check_rope_scaling(m->src_rope_scaling))
+    return fail(KVX_ERR_INVALID_ARG, (std::string("kvx_map_noalloc: source ") + why).c_str());
+  if (const char* why = kvx::check_rope_scaling(m->tgt_rope_scaling))
+    return fail(KVX_ERR_INVALID_ARG, (std::string("kvx_map_noalloc: target ") + why).c_str());
   if (!m->selection || !m->W || !m->b) return fail(KVX_ERR_INVALID_ARG, "kvx_map_noalloc: NULL selection, W or b");
   if (!aligned(m->W, 16) || !aligned(m->b, 16))
     return fail(KVX_ERR_INVALID_ARG, "kvx_map_noalloc: W and b must be 16-byte aligned");
@@ -134,6 +138,7 @@ extern "C" KVX_API kvx_status kvx_map_noalloc(const kvx_noalloc_mapper* m, int d
   view.weight_dtype = m->weight_dtype;
   view.theta_s = m->src_rope_theta;
   view.theta_t = m->tgt_rope_theta;
+  kvx::set_rope_scaling(&view, m->src_rope_scaling, m->tgt_rope_scaling);
   kvx::fill_rope(&view);
   view.d_sel = d_sel;
   view.d_W = const_cast<void*>(m->W);

@@ -236,6 +236,8 @@ const char* check_probe_config(const kvx_probe_config* cfg) {
       !std::isfinite(cfg->tgt_rope_theta))
     return "the RoPE bases must be finite and > 1";
   if (cfg->workspace_bytes != 0 && !cfg->workspace) return "workspace_bytes without a workspace";
+  if (const char* why = check_rope_scaling(cfg->src_rope_scaling)) return why;
+  if (const char* why = check_rope_scaling(cfg->tgt_rope_scaling)) return why;
   if (reinterpret_cast<uintptr_t>(cfg->workspace) & 255u) return "workspace must be 256-byte aligned";
   return nullptr;
 }
@@ -321,6 +323,7 @@ KVX_API kvx_status kvx_r2_probe(const kvx_probe_config* cfg, const kvx_src* src,
   tmp.d = kPD;
   tmp.theta_s = cfg->src_rope_theta;
   tmp.theta_t = cfg->tgt_rope_theta;
+  set_rope_scaling(&tmp, cfg->src_rope_scaling, cfg->tgt_rope_scaling);
   fill_rope(&tmp);
 
   const int Ls = cfg->src_layers, Lt = cfg->tgt_layers, H = cfg->n_kv_heads;

@@ -29,6 +29,28 @@ class KvxError(RuntimeError):
         self.status = status
 
 
+class kvx_rope_scaling(ctypes.Structure):
+    """Llama-3 RoPE frequency scaling (see include/kvx.h)."""
+    _fields_ = [("factor", ctypes.c_double), ("low_freq_factor", ctypes.c_double),
+                ("high_freq_factor", ctypes.c_double), ("original_max_position", ctypes.c_double)]
+
+
+_SCALING = [("src_rope_scaling", ctypes.POINTER(kvx_rope_scaling)),
+            ("tgt_rope_scaling", ctypes.POINTER(kvx_rope_scaling))]
+
+
+def rope_scaling(spec):
+    """kvx_rope_scaling from (factor, low_freq_factor, high_freq_factor, original_max_position),
+    or None."""
+    if not spec:
+        return None
+    return kvx_rope_scaling(*(float(x) for x in spec))
+
+
+def _scaling_ptr(s):
+    return ctypes.pointer(s) if s is not None else ctypes.POINTER(kvx_rope_scaling)()
+
+
 class kvx_config(ctypes.Structure):
     _fields_ = [
         ("src_layers", ctypes.c_int32), ("tgt_layers", ctypes.c_int32),
@@ -38,7 +60,7 @@ class kvx_config(ctypes.Structure):
         ("weight_dtype", ctypes.c_int32), ("head_mix", ctypes.c_int32), ("reserved", ctypes.c_int32),
         ("selection", ctypes.c_void_p), ("selection_scores", ctypes.c_void_p),
         ("W", ctypes.c_void_p), ("b", ctypes.c_void_p),
-    ]
+    ] + _SCALING
 
 
 class kvx_src(ctypes.Structure):
@@ -62,7 +84,7 @@ class kvx_noalloc_mapper(ctypes.Structure):
         ("tgt_rope_theta", ctypes.c_double), ("cache_dtype", ctypes.c_int32),
         ("weight_dtype", ctypes.c_int32), ("head_mix", ctypes.c_int32), ("reserved", ctypes.c_int32),
         ("selection", ctypes.c_void_p), ("W", ctypes.c_void_p), ("b", ctypes.c_void_p),
-    ]
+    ] + _SCALING
 
 
 class kvx_fit_config(ctypes.Structure):
@@ -72,7 +94,7 @@ class kvx_fit_config(ctypes.Structure):
         ("src_rope_theta", ctypes.c_double), ("tgt_rope_theta", ctypes.c_double),
         ("lambda_", ctypes.c_double), ("selection", ctypes.c_void_p),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_uint64),
-    ]
+    ] + _SCALING
 
 
 class kvx_probe_config(ctypes.Structure):
@@ -81,7 +103,7 @@ class kvx_probe_config(ctypes.Structure):
         ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
         ("src_rope_theta", ctypes.c_double), ("tgt_rope_theta", ctypes.c_double),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_uint64),
-    ]
+    ] + _SCALING
 
 
 class kvx_mlp_config(ctypes.Structure):
@@ -94,7 +116,7 @@ class kvx_mlp_config(ctypes.Structure):
         ("W1", ctypes.c_void_p), ("b1", ctypes.c_void_p), ("W2", ctypes.c_void_p), ("b2", ctypes.c_void_p),
         ("W3", ctypes.c_void_p), ("b3", ctypes.c_void_p),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_uint64),
-    ]
+    ] + _SCALING
 
 
 _lib = None
@@ -257,7 +279,7 @@ def dtype_code(t):
 
 def config_from_tensors(*, src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t,
                         cache_dtype, W, b=None, selection=None, scores=None,
-                        rope_style=KVX_ROPE_HALF, head_mix=KVX_PER_HEAD):
+                        rope_style=KVX_ROPE_HALF, head_mix=KVX_PER_HEAD, rope_scaling=None):
     """Build a kvx_config from host tensors.  Returns (cfg, keepalive) -- hold
     ``keepalive`` until kvx_create returns."""
     import numpy as np
@@ -279,7 +301,9 @@ def config_from_tensors(*, src_layers, tgt_layers, n_kv_heads, head_dim, k, thet
     cfg.selection_scores = _ptr(sc)
     cfg.W = _ptr(Wc)
     cfg.b = _ptr(bc)
-    return cfg, (Wc, bc, sel, sc, torch)
+    rs = globals()["rope_scaling"](rope_scaling)
+    cfg.src_rope_scaling = cfg.tgt_rope_scaling = _scaling_ptr(rs)
+    return cfg, (Wc, bc, sel, sc, torch, rs)
 
 
 def src_from_tensors(k, v):
@@ -325,10 +349,14 @@ def tgt_paged_from_tensors(k, v, block_table, block_size):
 
 
 def _fit_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, sel, workspace_ptr,
-                workspace_bytes):
-    return kvx_fit_config(int(src_layers), int(tgt_layers), int(n_kv_heads), int(head_dim), int(k),
-                          float(theta_s), float(theta_t), float(lam), _ptr(sel), workspace_ptr,
-                          int(workspace_bytes))
+                workspace_bytes, scaling=None):
+    cfg = kvx_fit_config(int(src_layers), int(tgt_layers), int(n_kv_heads), int(head_dim), int(k),
+                         float(theta_s), float(theta_t), float(lam), _ptr(sel), workspace_ptr,
+                         int(workspace_bytes))
+    rs = rope_scaling(scaling)
+    cfg.src_rope_scaling = cfg.tgt_rope_scaling = _scaling_ptr(rs)
+    cfg._rs = rs
+    return cfg
 
 
 def kvx_fit_workspace_bytes(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, selection,
@@ -343,7 +371,7 @@ def kvx_fit_workspace_bytes(src_layers, tgt_layers, n_kv_heads, head_dim, k, the
 
 def kvx_fit_ridge(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, selection,
                   src, tgt, batch, tokens_per_seq, positions_ptr, W_ptr, b_ptr, stream=0,
-                  workspace_ptr=None, workspace_bytes=0):
+                  workspace_ptr=None, workspace_bytes=0, rope_scaling=None):
     """Ridge fit on calibration caches (see include/kvx.h): src / tgt are kvx_src, selection a
     host int32 [L_t][k] array, W_ptr / b_ptr device fp32 buffers [L_t][2][H][k*d][d] and
     [L_t][2][H][d]; an optional caller workspace (device, 256-byte aligned).  Blocks until
@@ -351,7 +379,7 @@ def kvx_fit_ridge(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, thet
     import numpy as np
     sel = np.ascontiguousarray(selection, dtype=np.int32)
     cfg = _fit_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, sel, workspace_ptr,
-                      workspace_bytes)
+                      workspace_bytes, rope_scaling)
     _check(lib().kvx_fit_ridge(ctypes.byref(cfg), ctypes.byref(src), ctypes.byref(tgt), int(batch),
                                int(tokens_per_seq), positions_ptr, W_ptr, b_ptr, stream), "kvx_fit_ridge")
 
@@ -375,12 +403,14 @@ def kvx_r2_probe_workspace_bytes(src_layers, tgt_layers, n_kv_heads, head_dim, t
 
 def kvx_r2_probe(src_layers, tgt_layers, n_kv_heads, head_dim, theta_s, theta_t, src, tgt, batch,
                  tokens_per_seq, positions_ptr, scores_ptr, r2_kv_ptr=None, stream=0,
-                 workspace_ptr=None, workspace_bytes=0):
+                 workspace_ptr=None, workspace_bytes=0, rope_scaling=None):
     """Single-source R^2 probe (see include/kvx.h): src / tgt are kvx_src; scores_ptr a
     device float64 [L_t][L_s] buffer, r2_kv_ptr a device float64 [2][L_t][L_s] buffer or
     None; an optional caller workspace.  Blocks until the probe is done."""
     cfg = kvx_probe_config(int(src_layers), int(tgt_layers), int(n_kv_heads), int(head_dim),
                            float(theta_s), float(theta_t), workspace_ptr, int(workspace_bytes))
+    rs = globals()["rope_scaling"](rope_scaling)
+    cfg.src_rope_scaling = cfg.tgt_rope_scaling = _scaling_ptr(rs)
     _check(lib().kvx_r2_probe(ctypes.byref(cfg), ctypes.byref(src), ctypes.byref(tgt), int(batch),
                               int(tokens_per_seq), positions_ptr, scores_ptr, r2_kv_ptr, stream),
            "kvx_r2_probe")
@@ -394,7 +424,8 @@ def kvx_select_topk_device(scores_ptr, tgt_layers, src_layers, k, out_ptr, strea
 
 
 def mlp_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, hidden, theta_s, theta_t, selection,
-               W1_ptr, b1_ptr, W2_ptr, b2_ptr, W3_ptr, b3_ptr, workspace_ptr=None, workspace_bytes=0):
+               W1_ptr, b1_ptr, W2_ptr, b2_ptr, W3_ptr, b3_ptr, workspace_ptr=None, workspace_bytes=0,
+               rope_scaling=None):
     """kvx_mlp_config for kvx_mlp_map (weights and biases DEVICE pointers, see include/kvx.h).
     The returned config keeps the host selection array alive."""
     import numpy as np
@@ -403,6 +434,9 @@ def mlp_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, hidden, theta_s,
                          float(theta_s), float(theta_t), _ptr(sel), W1_ptr, b1_ptr, W2_ptr, b2_ptr, W3_ptr,
                          b3_ptr, workspace_ptr, int(workspace_bytes))
     cfg._sel = sel
+    rs = globals()["rope_scaling"](rope_scaling)
+    cfg.src_rope_scaling = cfg.tgt_rope_scaling = _scaling_ptr(rs)
+    cfg._rs = rs
     return cfg
 
 

@@ -120,6 +120,7 @@ class Workload:
     block_size: int = 16
     len_range: tuple = (0, 0)   # initial per-sequence lengths (paged), inclusive
     head_mix: str = "per_head"  # "per_head" (F = k d) | "cross_head" (F = k H d, the paper's)
+    rope_scaling: tuple = ()    # Llama-3 frequency scaling of both models, or () for plain theta
     notes: str = field(default="", compare=False)
 
     @property

@@ -19,6 +19,7 @@ import torch
 
 from oracle import bf16 as obf16
 from oracle import mapper as omap
+from oracle import rope as orope
 from paper_2608_03893_gb300 import kvx
 from paper_2608_03893_gb300 import synthetic as syn
 
@@ -36,6 +37,14 @@ def to_f64(t):
     return t.numpy().astype(np.float64)
 
 
+def rope_theta(w, side):
+    """The oracle's RoPE base for one side of a workload (a RopeSpec when it is scaled)."""
+    theta = w.theta_s if side == 0 else w.theta_t
+    if not w.rope_scaling:
+        return theta
+    return orope.RopeSpec(theta, orope.Llama3Scaling(*w.rope_scaling))
+
+
 def make_ctx(w, kernel=kvx.KVX_KERNEL_AUTO, selection=None, W=None, b=None, scores=None,
              device=0, rope_style=kvx.KVX_ROPE_HALF):
     if W is None:
@@ -46,7 +55,8 @@ def make_ctx(w, kernel=kvx.KVX_KERNEL_AUTO, selection=None, W=None, b=None, scor
         src_layers=w.Ls, tgt_layers=w.Lt, n_kv_heads=w.H, head_dim=w.d, k=w.k,
         theta_s=w.theta_s, theta_t=w.theta_t, cache_dtype=w.cache_dtype, W=W, b=b,
         selection=selection, scores=scores, rope_style=rope_style,
-        head_mix=kvx.KVX_CROSS_HEAD if w.head_mix == "cross_head" else kvx.KVX_PER_HEAD)
+        head_mix=kvx.KVX_CROSS_HEAD if w.head_mix == "cross_head" else kvx.KVX_PER_HEAD,
+        rope_scaling=w.rope_scaling or None)
     ctx = kvx.kvx_create(cfg, device)
     if kernel != kvx.KVX_KERNEL_AUTO:
         kvx.kvx_set_kernel(ctx, kernel)
@@ -75,7 +85,7 @@ def oracle_full(w, sk, sv, pos_np, sel, W, b, style="half"):
     """Returns (ref_k, ref_v, slack_k, slack_v)."""
     mode = "exact" if w.cache_dtype == "f32" else "bf16fwd"
     return omap.map_cache(to_f64(sk), to_f64(sv), pos_np, sel, to_f64(W),
-                          None if b is None else to_f64(b), w.theta_s, w.theta_t, mode=mode,
+                          None if b is None else to_f64(b), rope_theta(w, 0), rope_theta(w, 1), mode=mode,
                           style=style, head_mix=w.head_mix, rounding_slack=STRIP_DELTA)
 
 
@@ -117,5 +127,5 @@ def oracle_rows(w, rows, pos_np, sel, W, b, turn=None):
     sv = to_f64(syn.source_rows(w, 1, rows, turn=turn))
     p = pos_np[rows[:, 0], rows[:, 1]]
     return omap.map_tokens(sk, sv, p, sel, to_f64(W), None if b is None else to_f64(b),
-                           w.theta_s, w.theta_t, mode=mode, head_mix=w.head_mix,
+                           rope_theta(w, 0), rope_theta(w, 1), mode=mode, head_mix=w.head_mix,
                            rounding_slack=STRIP_DELTA)

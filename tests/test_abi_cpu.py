@@ -234,3 +234,26 @@ def test_mlp_map_rejects_bad_arguments_before_touching_the_device():
     with pytest.raises(kvx.KvxError) as e:
         kvx.kvx_mlp_map(cfg, src, 1, 16, p, paged)
     assert e.value.status == kvx.KVX_ERR_UNSUPPORTED
+
+
+@pytest.mark.parametrize("spec", [(0.5, 1.0, 4.0, 8192.0), (8.0, 4.0, 1.0, 8192.0), (8.0, 0.0, 4.0, 8192.0),
+                                  (8.0, 1.0, 4.0, 0.0), (float("inf"), 1.0, 4.0, 8192.0)])
+def test_rope_scaling_is_validated_on_the_host(spec):
+    """Invalid Llama-3 scaling parameters are refused by kvx_create, kvx_fit_ridge and
+    kvx_r2_probe before any device work."""
+    cfg, keep = _cfg()
+    rs = kvx.rope_scaling(spec)
+    cfg.tgt_rope_scaling = ctypes.pointer(rs)
+    with pytest.raises(kvx.KvxError) as e:
+        kvx.kvx_create(cfg, 0)
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+    buf = np.zeros(64, dtype=np.float64)
+    p = buf.ctypes.data
+    src = kvx.kvx_src(p, p, (ctypes.c_int64 * 4)(4096, 4096, 256, 128))
+    with pytest.raises(kvx.KvxError) as e:
+        kvx.kvx_fit_ridge(4, 3, 2, 128, 2, 1e6, 1e6, 0.01, np.array([[0, 1], [1, 2], [2, 3]], dtype=np.int32),
+                          src, src, 1, 16, p, p, p, rope_scaling=spec)
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+    with pytest.raises(kvx.KvxError) as e:
+        kvx.kvx_r2_probe(4, 3, 2, 128, 1e6, 1e6, src, src, 1, 256, p, p, rope_scaling=spec)
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG

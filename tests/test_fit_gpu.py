@@ -66,13 +66,18 @@ def _run_fit(w, lam, sel):
 
 
 def _check_systems(w, lam, sel, caches, Wg, bg, systems):
+    _check_systems_theta(w, w.theta_s, w.theta_t, lam, sel, caches, Wg, bg, systems)
+
+
+def _check_systems_theta(w, theta_s, theta_t, lam, sel, caches, Wg, bg, systems):
+    """theta_s / theta_t: plain bases or oracle.rope.RopeSpec (scaled frequencies)."""
     sk, sv, tk, tv, pos = caches
     feats = {}
     N = w.B * w.T
     for (l, kv, h) in systems:
         if kv not in feats:
-            feats[kv] = (_features(w, sk if kv == 0 else sv, kv, w.theta_s, pos),
-                         _features(w, tk if kv == 0 else tv, kv, w.theta_t, pos))
+            feats[kv] = (_features(w, sk if kv == 0 else sv, kv, theta_s, pos),
+                         _features(w, tk if kv == 0 else tv, kv, theta_t, pos))
         xs, xt = feats[kv]
         X = np.concatenate([xs[s, h] for s in sel[l]], axis=-1)
         Y = xt[l, h]
@@ -155,3 +160,28 @@ def test_fit_caller_workspace_one_pass_and_chunked():
     with pytest.raises(kvx.KvxError) as e:
         fit(4096)
     assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+
+
+def test_fit_llama3_rope_scaling():
+    """The fit strips both sides' keys with the llama3-scaled frequencies: every system of a
+    small Llama-3.1-like case at positions past 10^5 against the oracle given the same
+    scaling (the features are built with oracle.rope.RopeSpec)."""
+    spec = (8.0, 1.0, 4.0, 8192.0)
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=4, Lt=3, H=2, B=1, T=512, k=2, theta_s=5e5, theta_t=5e5)
+    sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
+    dev = torch.device("cuda:0")
+    sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+    tk, tv = syn.target_cache(w, 0, device=dev), syn.target_cache(w, 1, device=dev)
+    pos = syn.positions(w) + 150001
+    posd = torch.from_numpy(pos).to(dev)
+    F = w.k * w.d
+    W = torch.full((w.Lt, 2, w.H, F, w.d), float("nan"), dtype=torch.float32, device=dev)
+    b = torch.full((w.Lt, 2, w.H, w.d), float("nan"), dtype=torch.float32, device=dev)
+    kvx.kvx_fit_ridge(w.Ls, w.Lt, w.H, w.d, w.k, w.theta_s, w.theta_t, 0.01, sel, kvx.src_from_tensors(sk, sv),
+                      kvx.src_from_tensors(tk, tv), w.B, w.T, posd.data_ptr(), W.data_ptr(), b.data_ptr(),
+                      torch.cuda.current_stream().cuda_stream, rope_scaling=spec)
+    rs = orope.RopeSpec(w.theta_s, orope.Llama3Scaling(*spec))
+    rt = orope.RopeSpec(w.theta_t, orope.Llama3Scaling(*spec))
+    systems = [(l, kv, h) for l in range(w.Lt) for kv in range(2) for h in range(w.H)]
+    _check_systems_theta(w, rs, rt, 0.01, sel, (sk, sv, tk, tv, pos), W.cpu().double().numpy(),
+                         b.cpu().double().numpy(), systems)

@@ -465,3 +465,31 @@ def test_cross_head_full_size_sampled():
     finally:
         kvx.kvx_destroy(ctx)
         torch.cuda.empty_cache()
+
+
+# ------------------------------------------------------- Llama-3 frequency scaling -----
+
+@pytest.mark.parametrize("kname", ["simt", "tc"])
+def test_llama3_rope_scaling_small(kname):
+    """Llama 3.1 shapes (theta 5e5) with the llama3 frequency scaling on both models, at
+    positions past 10^5 so that the rescaled low frequencies turn: every output against the
+    oracle (whose inverse frequencies follow the scaling's definition), and the result
+    differs from the unscaled map."""
+    over = dict(Ls=6, Lt=5, H=2, B=2, T=300, k=3, theta_s=5e5, theta_t=5e5)
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", rope_scaling=(8.0, 1.0, 4.0, 8192.0), **over)
+    _kernel_or_skip(w, KERNELS[kname])
+    ctx, sel, W, b = make_ctx(w, kernel=KERNELS[kname])
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w) + np.array([[123457], [250001]], dtype=np.int32)
+        rk, rv, ak, av = oracle_full(w, sk, sv, pos, sel, W, b)
+        tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        ok, ratio, rms, nbad = check(w, [to_f64(tk), to_f64(tv)], [rk, rv], [ak, av])
+        assert ok, "%d elements out of tolerance (worst %.3g x bound)" % (nbad, ratio)
+        plain = syn.workload("qwen3_14b_32b_b8x1024_k4", **over)
+        pk, _, _, _ = oracle_full(plain, sk, sv, pos, sel, W, b)
+        assert np.max(np.abs(pk - rk)) > 0.1 * rms          # the scaling does change the keys
+    finally:
+        kvx.kvx_destroy(ctx)

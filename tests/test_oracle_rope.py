@@ -135,3 +135,43 @@ def test_bf16_rne_matches_torch_from_binary32():
     expect = torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
     got = bf16.encode(x.astype(np.float64))
     assert np.array_equal(got, expect)
+
+
+# ---- Llama-3 frequency scaling ------------------------------------------------------
+
+LLAMA31 = rope.Llama3Scaling(8.0, 1.0, 4.0, 8192.0)
+
+
+def test_llama3_scaling_hand_values():
+    """Worked by hand from the definition (P = 8192, low 1, high 4, factor 8): a wavelength
+    of 4096 sits between P/4 = 2048 and P/1 = 8192 with blend weight (8192/4096 - 1) / 3 =
+    1/3, so omega' = (2/3)(omega/8) + (1/3) omega = (5/12) omega; wavelength 1000 < 2048
+    keeps omega; wavelength 10000 > 8192 gives omega / 8."""
+    w = 2 * np.pi / np.array([4096.0, 1000.0, 10000.0])
+    got = rope.llama3_scale(w, LLAMA31)
+    assert np.allclose(got / w, [5.0 / 12.0, 1.0, 0.125], rtol=1e-14, atol=0)
+
+
+def test_llama3_scaling_is_continuous_and_monotone_at_the_edges():
+    P = LLAMA31.original_max_position
+    for lam in (P / LLAMA31.high_freq_factor, P / LLAMA31.low_freq_factor):
+        w = 2 * np.pi / np.array([lam * (1 - 1e-12), lam, lam * (1 + 1e-12)])
+        g = rope.llama3_scale(w, LLAMA31)
+        assert np.allclose(g, g[1], rtol=1e-9, atol=0)
+    lam = np.geomspace(10, 1e7, 4001)
+    g = rope.llama3_scale(2 * np.pi / lam, LLAMA31)
+    assert np.all(np.diff(g) < 0)                 # still strictly decreasing in wavelength
+
+
+def test_llama3_scaling_identity_and_inv_freq_plumbing():
+    w = rope.inv_freq(5e5, 128)
+    assert np.allclose(rope.llama3_scale(w, rope.Llama3Scaling(1.0, 1.0, 4.0, 8192.0)), w, rtol=1e-15, atol=0)
+    spec = rope.RopeSpec(5e5, LLAMA31)
+    ws = rope.inv_freq(spec, 128)
+    assert ws[0] == w[0] == 1.0                   # the fastest pair keeps its frequency
+    assert ws[-1] == w[-1] / 8.0                  # the slowest is divided by the factor
+    x = np.random.default_rng(1).standard_normal((3, 128))
+    pos = np.array([0, 5000, 123456])
+    y = rope.rotate(x, pos, spec)
+    assert np.allclose(rope.rotate(y, pos, spec, inverse=True), x, atol=1e-12)
+    assert np.allclose(np.linalg.norm(y, axis=-1), np.linalg.norm(x, axis=-1), atol=1e-12)
