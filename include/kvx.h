@@ -167,6 +167,26 @@ KVX_API kvx_status kvx_create(const kvx_config* cfg, int device, kvx_ctx** out);
 KVX_API kvx_status kvx_map(kvx_ctx* ctx, const kvx_src* src, int32_t batch, int32_t tokens_per_seq,
                    const int32_t* positions, const kvx_tgt* tgt, void* stream);
 
+/* ---- Mapping caches in host memory, copies overlapped with the map ---------------
+ * A pipe holds device staging for `chunk_tokens` tokens of `batch` sequences (two slots
+ * of source K, V, positions and target K, V: about 4 chunk_tokens batch n_kv d (L_s + L_t)
+ * cache elements) and three internal streams.  kvx_map_host maps host caches through it:
+ * the tokens go in chunks, and the host-to-device copy of one chunk, the map of the
+ * previous one and the device-to-host copy of the one before run at the same time.  The
+ * results equal kvx_map's on device copies of the same caches.
+ * Host layouts: src contiguous [L_s][batch][n_kv][T][d] (stride = {batch n_kv T d,
+ * n_kv T d, T d, d}), tgt contiguous [L_t][batch][n_kv][T][d] (paged: UNSUPPORTED),
+ * positions [batch][T]; pinned memory (cudaHostAlloc / cudaHostRegister) for the copies
+ * to overlap.  The work starts after the work already queued on `stream` and `stream`
+ * waits for its end, so the host targets are complete once `stream` is; the host inputs
+ * must not change until then.  Device errors go to the context's status word
+ * (kvx_get_status).  A pipe serves one caller at a time; destroy it before its context. */
+typedef struct kvx_host_pipe kvx_host_pipe;
+KVX_API kvx_status kvx_host_pipe_create(kvx_ctx* ctx, int32_t batch, int32_t chunk_tokens, kvx_host_pipe** out);
+KVX_API kvx_status kvx_map_host(kvx_host_pipe* pipe, const kvx_src* src, int32_t tokens_per_seq,
+                                const int32_t* positions, const kvx_tgt* tgt, void* stream);
+KVX_API kvx_status kvx_host_pipe_destroy(kvx_host_pipe* pipe);
+
 /* Free the context and its device memory (synchronises the device first). NULL is OK. */
 KVX_API kvx_status kvx_destroy(kvx_ctx* ctx);
 

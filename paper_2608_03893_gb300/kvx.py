@@ -125,7 +125,8 @@ EXPORTED = ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_
             "kvx_set_kernel", "kvx_get_status", "kvx_mapper_params", "kvx_status_string",
             "kvx_last_error", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms", "kvx_r2_probe",
             "kvx_select_topk_device", "kvx_fit_workspace_bytes", "kvx_r2_probe_workspace_bytes",
-            "kvx_mlp_map", "kvx_mlp_workspace_bytes")
+            "kvx_mlp_map", "kvx_mlp_workspace_bytes", "kvx_host_pipe_create", "kvx_map_host",
+            "kvx_host_pipe_destroy")
 
 
 def lib():
@@ -167,9 +168,13 @@ def lib():
                               ctypes.POINTER(kvx_tgt), vp]
     L.kvx_mlp_workspace_bytes.argtypes = [ctypes.POINTER(kvx_mlp_config), i32, i32]
     L.kvx_mlp_workspace_bytes.restype = i64
+    L.kvx_host_pipe_create.argtypes = [vp, i32, i32, ctypes.POINTER(vp)]
+    L.kvx_map_host.argtypes = [vp, ctypes.POINTER(kvx_src), i32, vp, ctypes.POINTER(kvx_tgt), vp]
+    L.kvx_host_pipe_destroy.argtypes = [vp]
     for name in ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
                  "kvx_set_kernel", "kvx_get_status", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms",
-                 "kvx_r2_probe", "kvx_select_topk_device", "kvx_mlp_map"):
+                 "kvx_r2_probe", "kvx_select_topk_device", "kvx_mlp_map", "kvx_host_pipe_create",
+                 "kvx_map_host", "kvx_host_pipe_destroy"):
         getattr(L, name).restype = ctypes.c_int
     _lib = L
     return L
@@ -448,3 +453,22 @@ def kvx_mlp_map(cfg, src, batch, tokens_per_seq, positions_ptr, tgt, stream=0):
     """MLP mapper apply (see include/kvx.h); blocks until done."""
     _check(lib().kvx_mlp_map(ctypes.byref(cfg), ctypes.byref(src), int(batch), int(tokens_per_seq),
                              positions_ptr, ctypes.byref(tgt), stream), "kvx_mlp_map")
+
+
+def kvx_host_pipe_create(ctx, batch, chunk_tokens):
+    """Staging and streams for kvx_map_host (see include/kvx.h); returns the pipe handle."""
+    out = ctypes.c_void_p()
+    _check(lib().kvx_host_pipe_create(ctx, int(batch), int(chunk_tokens), ctypes.byref(out)),
+           "kvx_host_pipe_create")
+    return out.value
+
+
+def kvx_map_host(pipe, src, tokens_per_seq, positions_ptr, tgt, stream=0):
+    """Map host caches (contiguous, ideally pinned) through a pipe; ``stream`` waits for the
+    result."""
+    _check(lib().kvx_map_host(pipe, ctypes.byref(src), int(tokens_per_seq), positions_ptr, ctypes.byref(tgt),
+                              stream), "kvx_map_host")
+
+
+def kvx_host_pipe_destroy(pipe):
+    _check(lib().kvx_host_pipe_destroy(pipe), "kvx_host_pipe_destroy")

@@ -257,3 +257,16 @@ def test_rope_scaling_is_validated_on_the_host(spec):
     with pytest.raises(kvx.KvxError) as e:
         kvx.kvx_r2_probe(4, 3, 2, 128, 1e6, 1e6, src, src, 1, 256, p, p, rope_scaling=spec)
     assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+
+
+def test_host_pipe_rejects_bad_arguments_before_touching_the_device():
+    with pytest.raises(kvx.KvxError) as e:
+        kvx.kvx_host_pipe_create(None, 1, 1024)
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+    buf = np.zeros(64, dtype=np.float64)
+    p = buf.ctypes.data
+    src = kvx.kvx_src(p, p, (ctypes.c_int64 * 4)(4096, 4096, 256, 128))
+    tgt = kvx.kvx_tgt()
+    with pytest.raises(kvx.KvxError) as e:
+        kvx.kvx_map_host(None, src, 16, p, tgt)
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG

@@ -493,3 +493,43 @@ def test_llama3_rope_scaling_small(kname):
         assert np.max(np.abs(pk - rk)) > 0.1 * rms          # the scaling does change the keys
     finally:
         kvx.kvx_destroy(ctx)
+
+
+# ------------------------------------------------------------ host-buffer pipeline -----
+
+@pytest.mark.parametrize("name,over,kernel,chunk", [
+    ("qwen3_14b_32b_b8x1024_k4", dict(Ls=6, Lt=5, H=2, B=2, T=1000, k=3), "tc", 300),     # ragged chunks
+    ("qwen3_14b_32b_b8x1024_k4", dict(Ls=6, Lt=5, H=2, B=2, T=1000, k=3), "simt", 256),
+    ("qwen3_14b_32b_t32768_k4_xhead", dict(Ls=4, Lt=3, H=2, B=1, T=700, k=2), "tc", 128),
+    ("qwen3_14b_32b_b8x1024_k4", dict(Ls=3, Lt=2, H=1, B=1, T=50, k=1), "tc", 4096),      # one short chunk
+])
+def test_map_host_equals_device_map(name, over, kernel, chunk):
+    """kvx_map_host (pinned host caches, chunked, copies overlapped with the map) writes the
+    same bytes into the host targets as kvx_map on device copies, over two calls through
+    one pipe."""
+    w = syn.workload(name, **over)
+    ctx, sel, W, b = make_ctx(w, kernel=KERNELS[kernel])
+    pipe = None
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w) + 17
+        tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        hk, hv = sk.cpu().pin_memory(), sv.cpu().pin_memory()
+        hpos = torch.from_numpy(np.ascontiguousarray(pos, dtype=np.int32)).pin_memory()
+        pipe = kvx.kvx_host_pipe_create(ctx, w.B, chunk)
+        s = torch.cuda.current_stream()
+        for rep in range(2):
+            ok_ = torch.full(tk.shape, float("nan"), dtype=tk.dtype).pin_memory()
+            ov_ = torch.full(tv.shape, float("nan"), dtype=tv.dtype).pin_memory()
+            kvx.kvx_map_host(pipe, kvx.src_from_tensors(hk, hv), w.T, hpos.data_ptr(),
+                             kvx.tgt_from_tensors(ok_, ov_), s.cuda_stream)
+            s.synchronize()
+            assert kvx.kvx_get_status(ctx, s.cuda_stream) == kvx.KVX_OK
+            assert torch.equal(ok_.view(torch.int16), tk.cpu().view(torch.int16)), rep
+            assert torch.equal(ov_.view(torch.int16), tv.cpu().view(torch.int16)), rep
+    finally:
+        if pipe:
+            kvx.kvx_host_pipe_destroy(pipe)
+        kvx.kvx_destroy(ctx)
