@@ -14,10 +14,11 @@
 //    head, so every distinct pair of the selection is computed once and shared by all
 //    target layers whose selection holds both; the k blocks of Xc^T Yc are per target layer.
 // 2. fit_solve_kernel: one CTA per system at a time (persistent); the block grid is
-//    widened to fp64 into a per-CTA scratch matrix, lambda added, factorised by a blocked
-//    right-looking Cholesky (32-column panels: diagonal block in shared memory, panel by
-//    forward substitution, trailing update), then the two triangular solves for the d
-//    right-hand sides and the bias; W and b are written in fp32.
+//    widened to float-float pairs (~48 significant bits, on the FP32 units) into a per-CTA
+//    scratch matrix, lambda added, factorised by a blocked right-looking Cholesky
+//    (32-column panels: diagonal block in shared memory, panel by forward substitution,
+//    trailing update), then the two triangular solves for the d right-hand sides and the
+//    bias; W and b are written in fp32.
 // kvx_fit_ridge runs them on the caller's stream, with stream-ordered workspace, and
 // synchronises before it returns (the fit is an offline step).
 #include <cuda_runtime.h>
@@ -65,25 +66,84 @@ __device__ __forceinline__ size_t sums_index(const FitParams& P, int side, int k
 __device__ __forceinline__ void report_fit(int32_t* status, int code) { atomicCAS(status, 0, code); }
 
 // ------------------------------------------------------------------- solve --
-// Persistent: CTA c handles systems c, c + gridDim.x, ...  F = 128 k (k <= 4).  Dynamic
-// shared memory: the 32 x 32 diagonal block and the panel below it ((F - 32) x 32), fp64.
-constexpr int kNotSpd = 100;        // internal status: a pivot <= 0 (matrix not positive definite)
+// Float-float arithmetic: a value is the unevaluated sum hi + lo of two floats
+// (|lo| <= ulp(hi) / 2), about 48 significant bits, against 53 for fp64 and far below the
+// fp32 error of the Gram blocks it solves with.  GB300 runs 64 FP32 FMAs for each FP64 FMA,
+// so the solve runs on the FP32 units: a fused multiply-add of two such pairs costs about a
+// dozen FP32 instructions.  The error-free steps are the published ones: two_sum (Knuth,
+// TAOCP vol. 2, 4.2.2), fast_two_sum (Dekker 1971, needs |a| >= |b|), two_prod by one
+// FMA; the pair arithmetic follows Dekker's and the QD library's (Hida, Li, Bailey 2001)
+// "sloppy" addition, and division / square root correct a float estimate once by the
+// residual.
+struct __align__(8) DF {
+  float hi, lo;
+};
 
-__global__ void __launch_bounds__(256) fit_solve_kernel(const __grid_constant__ FitParams P) {
-  extern __shared__ __align__(16) double fsm[];
-  double* D = fsm;                                // [32][32]
-  double* Pn = fsm + kNB * kNB;                   // [F - 32][32]
+__device__ __forceinline__ DF df_make(float a) { return DF{a, 0.f}; }
+__device__ __forceinline__ DF fast_two_sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  return DF{s, __fsub_rn(b, __fsub_rn(s, a))};
+}
+__device__ __forceinline__ DF two_sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  return DF{s, __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb))};
+}
+__device__ __forceinline__ DF df_neg(DF a) { return DF{-a.hi, -a.lo}; }
+__device__ __forceinline__ DF df_add(DF a, DF b) {
+  const DF s = two_sum(a.hi, b.hi);
+  return fast_two_sum(s.hi, __fadd_rn(s.lo, __fadd_rn(a.lo, b.lo)));
+}
+// a * b + c
+__device__ __forceinline__ DF df_fma(DF a, DF b, DF c) {
+  const float p = __fmul_rn(a.hi, b.hi);
+  float e = __fmaf_rn(a.hi, b.hi, -p);
+  e = __fmaf_rn(a.hi, b.lo, e);
+  e = __fmaf_rn(a.lo, b.hi, e);
+  const DF s = two_sum(p, c.hi);
+  return fast_two_sum(s.hi, __fadd_rn(s.lo, __fadd_rn(e, c.lo)));
+}
+// a / b: the float quotient q corrected by the residual a - q b
+__device__ __forceinline__ DF df_div(DF a, DF b) {
+  const float q1 = __fdiv_rn(a.hi, b.hi);
+  const DF r = df_fma(df_neg(df_make(q1)), b, a);
+  return fast_two_sum(q1, __fdiv_rn(r.hi, b.hi));
+}
+// sqrt(a), a > 0: s = sqrt(hi) corrected by (a - s^2) / 2s
+__device__ __forceinline__ DF df_sqrt(DF a) {
+  const float s = __fsqrt_rn(a.hi);
+  const DF r = df_fma(df_neg(df_make(s)), df_make(s), a);
+  return fast_two_sum(s, __fdiv_rn(r.hi, __fmul_rn(2.f, s)));
+}
+__device__ __forceinline__ DF df_from_double(double x) {
+  const float hi = static_cast<float>(x);
+  return DF{hi, static_cast<float>(x - static_cast<double>(hi))};
+}
+__device__ __forceinline__ double df_to_double(DF a) { return static_cast<double>(a.hi) + static_cast<double>(a.lo); }
+
+// Persistent: CTA c handles systems c, c + gridDim.x, ...  F = 128 k (k <= 4).  Dynamic
+// shared memory: the 32 x 32 diagonal block and the panel below it ((F - 32) x 32), pairs
+// of floats (8 bytes an element, as fp64 was).
+constexpr int kNotSpd = 100;        // internal status: a pivot <= 0 (matrix not positive definite)
+constexpr int kPS = kNB + 1;        // panel row stride in shared memory (pairs)
+
+__global__ void __launch_bounds__(256, 1) fit_solve_kernel(const __grid_constant__ FitParams P) {
+  extern __shared__ __align__(16) DF fsm[];
+  DF* D = fsm;                                    // [32][33]
+  DF* Pn = fsm + kNB * kPS;                       // [F - 32][33]: rows padded so a warp's 32 rows hit distinct banks
   const int F = P.k * kFD;
   const int tid = threadIdx.x;
-  double* A = P.scratch + static_cast<size_t>(blockIdx.x) * (static_cast<size_t>(F) * F + static_cast<size_t>(F) * kFD);
-  double* Z = A + static_cast<size_t>(F) * F;     // [F][128]
+  DF* A = reinterpret_cast<DF*>(P.scratch) +
+          static_cast<size_t>(blockIdx.x) * (static_cast<size_t>(F) * F + static_cast<size_t>(F) * kFD);
+  DF* Z = A + static_cast<size_t>(F) * F;         // [F][128]
   const int n_sys = P.Lt * 2 * P.H;
   const double inv_n = 1.0 / (static_cast<double>(P.B) * P.T);
+  const DF lam = df_from_double(P.lambda);
   for (int sys = blockIdx.x; sys < n_sys; sys += gridDim.x) {
     const int h = sys % P.H;
     const int kv = (sys / P.H) & 1;
     const int l = sys / (2 * P.H);
-    // 1. A = Xc^T Xc + lambda I (lower triangle) and Z = Xc^T Yc, widened to fp64
+    // 1. A = Xc^T Xc + lambda I (lower triangle) and Z = Xc^T Yc
     for (int64_t e = tid; e < static_cast<int64_t>(F) * F; e += blockDim.x) {
       const int r = static_cast<int>(e / F), c = static_cast<int>(e % F);
       if (c > r) continue;
@@ -92,52 +152,52 @@ __global__ void __launch_bounds__(256) fit_solve_kernel(const __grid_constant__ 
       const size_t blk = ((static_cast<size_t>(kv) * P.H + h) * P.n_pairs + (pr >= 0 ? pr : -1 - pr)) * kFD * kFD;
       const float g = pr >= 0 ? P.gram[blk + static_cast<size_t>(r % kFD) * kFD + (c % kFD)]
                               : P.gram[blk + static_cast<size_t>(c % kFD) * kFD + (r % kFD)];
-      A[e] = static_cast<double>(g) + (r == c ? P.lambda : 0.0);
+      A[e] = r == c ? df_add(df_make(g), lam) : df_make(g);
     }
     for (int64_t e = tid; e < static_cast<int64_t>(F) * kFD; e += blockDim.x) {
       const int r = static_cast<int>(e / kFD), j = static_cast<int>(e % kFD);
-      Z[e] = static_cast<double>(P.xty[(static_cast<size_t>(sys) * P.k + r / kFD) * kFD * kFD +
-                                       static_cast<size_t>(r % kFD) * kFD + j]);
+      Z[e] = df_make(P.xty[(static_cast<size_t>(sys) * P.k + r / kFD) * kFD * kFD + static_cast<size_t>(r % kFD) * kFD + j]);
     }
     __syncthreads();
     // 2. Cholesky A = L L^T, lower triangle in place, 32-column panels
     for (int c0 = 0; c0 < F; c0 += kNB) {
-      for (int e = tid; e < kNB * kNB; e += blockDim.x) D[e] = A[static_cast<size_t>(c0 + e / kNB) * F + c0 + e % kNB];
+      for (int e = tid; e < kNB * kNB; e += blockDim.x) D[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(c0 + e / kNB) * F + c0 + e % kNB];
       __syncthreads();
       if (tid < 32) {                             // one warp factors the diagonal block, lane = row
         for (int j = 0; j < kNB; ++j) {
           if (tid == j) {
-            const double d = D[j * kNB + j];
-            if (!(d > 0.0)) report_fit(P.status, kNotSpd);
-            D[j * kNB + j] = d > 0.0 ? sqrt(d) : 1.0;
+            const DF d = D[j * kPS + j];
+            if (!(d.hi > 0.f)) report_fit(P.status, kNotSpd);
+            D[j * kPS + j] = d.hi > 0.f ? df_sqrt(d) : df_make(1.f);
           }
           __syncwarp();
-          if (tid > j) D[tid * kNB + j] /= D[j * kNB + j];
+          if (tid > j) D[tid * kPS + j] = df_div(D[tid * kPS + j], D[j * kPS + j]);
           __syncwarp();
           if (tid > j)
-            for (int m = j + 1; m <= tid; ++m) D[tid * kNB + m] -= D[tid * kNB + j] * D[m * kNB + j];
+            for (int m = j + 1; m <= tid; ++m)
+              D[tid * kPS + m] = df_fma(df_neg(D[tid * kPS + j]), D[m * kPS + j], D[tid * kPS + m]);
           __syncwarp();
         }
       }
       __syncthreads();
       for (int e = tid; e < kNB * kNB; e += blockDim.x)
-        if (e % kNB <= e / kNB) A[static_cast<size_t>(c0 + e / kNB) * F + c0 + e % kNB] = D[e];
+        if (e % kNB <= e / kNB) A[static_cast<size_t>(c0 + e / kNB) * F + c0 + e % kNB] = D[(e / kNB) * kPS + e % kNB];
       // panel: rows below the diagonal block, P[r] L_kk^T = A[r][c0 .. c0+31]
       const int rows = F - c0 - kNB;
       for (int rr = tid; rr < rows; rr += blockDim.x) {
-        double* arow = A + static_cast<size_t>(c0 + kNB + rr) * F + c0;
-        double x[kNB];
+        DF* arow = A + static_cast<size_t>(c0 + kNB + rr) * F + c0;
+        DF x[kNB];
 #pragma unroll
         for (int c = 0; c < kNB; ++c) {
-          double v = arow[c];
+          DF v = arow[c];
 #pragma unroll
-          for (int m = 0; m < c; ++m) v -= x[m] * D[c * kNB + m];
-          x[c] = v / D[c * kNB + c];
+          for (int m = 0; m < c; ++m) v = df_fma(df_neg(x[m]), D[c * kPS + m], v);
+          x[c] = df_div(v, D[c * kPS + c]);
         }
 #pragma unroll
         for (int c = 0; c < kNB; ++c) {
           arow[c] = x[c];
-          Pn[rr * kNB + c] = x[c];
+          Pn[rr * kPS + c] = x[c];
         }
       }
       __syncthreads();
@@ -147,50 +207,126 @@ __global__ void __launch_bounds__(256) fit_solve_kernel(const __grid_constant__ 
         int ti = 0;
         while ((ti + 1) * (ti + 2) / 2 <= tile) ++ti;
         const int tj = tile - ti * (ti + 1) / 2;
-        const int ii = ti * kNB + (tid >> 3), jj = tj * kNB + (tid & 7) * 4;
-        double s[4] = {0.0, 0.0, 0.0, 0.0};
+        // thread: column jj (lane: the warp's stores are contiguous) and rows ii + 8q (warp w:
+        // ii = w), q < 4; the lane's panel row is read conflict-free (odd row stride), the
+        // warp's four rows are broadcasts
+        const int jj = tj * kNB + (tid & 31), ii = ti * kNB + (tid >> 5);
+        DF sacc[4] = {df_make(0.f), df_make(0.f), df_make(0.f), df_make(0.f)};
 #pragma unroll 8
         for (int m = 0; m < kNB; ++m) {
-          const double pi = Pn[ii * kNB + m];
+          const DF pj = Pn[jj * kPS + m];
 #pragma unroll
-          for (int q = 0; q < 4; ++q) s[q] += pi * Pn[(jj + q) * kNB + m];
+          for (int q = 0; q < 4; ++q) sacc[q] = df_fma(Pn[(ii + 8 * q) * kPS + m], pj, sacc[q]);
         }
-        double* arow = A + static_cast<size_t>(c0 + kNB + ii) * F + c0 + kNB;
 #pragma unroll
-        for (int q = 0; q < 4; ++q)
-          if (jj + q <= ii) arow[jj + q] -= s[q];
+        for (int q = 0; q < 4; ++q) {
+          DF* a = A + static_cast<size_t>(c0 + kNB + ii + 8 * q) * F + c0 + kNB + jj;
+          if (jj <= ii + 8 * q) *a = df_add(*a, df_neg(sacc[q]));
+        }
       }
       __syncthreads();
     }
-    // 3. forward solve L Y = Z, then backward L^T W = Y, in place on Z; thread = right-hand
-    //    side column (128 columns, two threads per column split the inner sums)
-    const int j = tid & (kFD - 1), half = tid >> 7;
-    for (int r = 0; r < F; ++r) {
-      const double* lrow = A + static_cast<size_t>(r) * F;
-      double sacc = 0.0;
-      for (int m = half; m < r; m += 2) sacc += lrow[m] * Z[static_cast<size_t>(m) * kFD + j];
-      Pn[tid] = sacc;                                  // scratch: partial sums of both halves
+    // 3. forward solve L Y = Z, then backward L^T W = Y, in place on Z, in 32-row blocks:
+    //    first the block's 32 x 128 entries take the products with every solved row (thread
+    //    = 4 rows x 4 right-hand-side columns, 16 independent sums), then the 32 x 32
+    //    triangle is solved row by row (thread = column).
+    const int r0 = 4 * (tid & 7), q0 = 4 * (tid >> 3);
+    auto load4 = [&](const DF* p, DF (&v)[4]) {
+      const float4 x = *reinterpret_cast<const float4*>(p), y = *reinterpret_cast<const float4*>(p + 2);
+      v[0] = DF{x.x, x.y};
+      v[1] = DF{x.z, x.w};
+      v[2] = DF{y.x, y.y};
+      v[3] = DF{y.z, y.w};
+    };
+    for (int b0 = 0; b0 < F; b0 += kNB) {
+      DF acc[4][4];
+#pragma unroll
+      for (int a = 0; a < 4; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0], acc[a]);
+      // operands of step m + 1 are loaded while step m computes
+      DF z[4], l[4];
+      if (b0 > 0) {
+        load4(&Z[q0], z);
+#pragma unroll
+        for (int a = 0; a < 4; ++a) l[a] = A[static_cast<size_t>(b0 + r0 + a) * F];
+      }
+      for (int m = 0; m < b0; ++m) {
+        DF zn[4], ln[4];
+        const int mn = m + 1 < b0 ? m + 1 : m;
+        load4(&Z[static_cast<size_t>(mn) * kFD + q0], zn);
+#pragma unroll
+        for (int a = 0; a < 4; ++a) ln[a] = A[static_cast<size_t>(b0 + r0 + a) * F + mn];
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) acc[a][c] = df_fma(df_neg(l[a]), z[c], acc[a][c]);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          z[c] = zn[c];
+          l[c] = ln[c];
+        }
+      }
+#pragma unroll
+      for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0 + c] = acc[a][c];
       __syncthreads();
-      if (half == 0) Z[static_cast<size_t>(r) * kFD + j] = (Z[static_cast<size_t>(r) * kFD + j] - Pn[j] - Pn[j + kFD]) / lrow[r];
+      if (tid < kFD) {
+        for (int i = 0; i < kNB; ++i) {
+          const DF* lrow = A + static_cast<size_t>(b0 + i) * F + b0;
+          DF v = Z[static_cast<size_t>(b0 + i) * kFD + tid];
+          for (int m = 0; m < i; ++m) v = df_fma(df_neg(lrow[m]), Z[static_cast<size_t>(b0 + m) * kFD + tid], v);
+          Z[static_cast<size_t>(b0 + i) * kFD + tid] = df_div(v, lrow[i]);
+        }
+      }
       __syncthreads();
     }
-    for (int r = F - 1; r >= 0; --r) {
-      double sacc = 0.0;
-      for (int m = r + 1 + half; m < F; m += 2) sacc += A[static_cast<size_t>(m) * F + r] * Z[static_cast<size_t>(m) * kFD + j];
-      Pn[tid] = sacc;
+    for (int b0 = F - kNB; b0 >= 0; b0 -= kNB) {
+      DF acc[4][4];
+#pragma unroll
+      for (int a = 0; a < 4; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0], acc[a]);
+      DF z[4], l[4];
+      if (b0 + kNB < F) {
+        load4(&Z[static_cast<size_t>(b0 + kNB) * kFD + q0], z);
+        load4(&A[static_cast<size_t>(b0 + kNB) * F + b0 + r0], l);   // L[m][b0 + r0 ..]: entries of L^T
+      }
+      for (int m = b0 + kNB; m < F; ++m) {
+        DF zn[4], ln[4];
+        const int mn = m + 1 < F ? m + 1 : m;
+        load4(&Z[static_cast<size_t>(mn) * kFD + q0], zn);
+        load4(&A[static_cast<size_t>(mn) * F + b0 + r0], ln);
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) acc[a][c] = df_fma(df_neg(l[a]), z[c], acc[a][c]);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          z[c] = zn[c];
+          l[c] = ln[c];
+        }
+      }
+#pragma unroll
+      for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0 + c] = acc[a][c];
       __syncthreads();
-      if (half == 0)
-        Z[static_cast<size_t>(r) * kFD + j] = (Z[static_cast<size_t>(r) * kFD + j] - Pn[j] - Pn[j + kFD]) / A[static_cast<size_t>(r) * F + r];
+      if (tid < kFD) {
+        for (int i = kNB - 1; i >= 0; --i) {
+          DF v = Z[static_cast<size_t>(b0 + i) * kFD + tid];
+          for (int m = i + 1; m < kNB; ++m)
+            v = df_fma(df_neg(A[static_cast<size_t>(b0 + m) * F + b0 + i]), Z[static_cast<size_t>(b0 + m) * kFD + tid], v);
+          Z[static_cast<size_t>(b0 + i) * kFD + tid] = df_div(v, A[static_cast<size_t>(b0 + i) * F + b0 + i]);
+        }
+      }
       __syncthreads();
     }
-    // 4. W (fp32) and b = mean(Y) - mean(X) W
+    // 4. W (fp32) and b = mean(Y) - mean(X) W (fp64)
     float* Wout = P.W + static_cast<size_t>(sys) * F * kFD;
-    for (int64_t e = tid; e < static_cast<int64_t>(F) * kFD; e += blockDim.x) Wout[e] = static_cast<float>(Z[e]);
+    for (int64_t e = tid; e < static_cast<int64_t>(F) * kFD; e += blockDim.x) Wout[e] = __fadd_rn(Z[e].hi, Z[e].lo);
     if (tid < kFD) {
       double acc = P.sums[sums_index(P, 1, kv, l, h) + tid] * inv_n;
       for (int r = 0; r < F; ++r) {
         const int layer = __ldg(&P.sel[l * P.k + r / kFD]);
-        acc -= P.sums[sums_index(P, 0, kv, layer, h) + r % kFD] * inv_n * Z[static_cast<size_t>(r) * kFD + tid];
+        acc -= P.sums[sums_index(P, 0, kv, layer, h) + r % kFD] * inv_n * df_to_double(Z[static_cast<size_t>(r) * kFD + tid]);
       }
       P.b[static_cast<size_t>(sys) * kFD + tid] = static_cast<float>(acc);
     }
@@ -440,7 +576,7 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
       set_error(std::string("kvx_fit_ridge: ") + kvx_last_error());
       break;
     }
-    const size_t smem = static_cast<size_t>(kNB) * kNB * 8 + static_cast<size_t>(pl.F - kNB) * kNB * 8;
+    const size_t smem = static_cast<size_t>(kNB) * kPS * 8 + static_cast<size_t>(pl.F - kNB) * kPS * 8;
     if ((e = cudaFuncSetAttribute(fit_solve_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem))) !=
         cudaSuccess) {
       set_error(std::string("kvx_fit_ridge: smem attribute: ") + cudaGetErrorString(e));
