@@ -523,13 +523,20 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=None)
     ap.add_argument("--fit", action="store_true",
                     help="time the ridge fit (kvx_fit_ridge) on the workload's shapes instead of the map")
+    ap.add_argument("--override", default="",
+                    help="comma-separated workload fields for a smaller case of the same kernel, e.g. "
+                         "Lt=16,T=4096 (profiling captures)")
     ap.add_argument("--mlp", action="store_true",
                     help="time the MLP mapper apply (kvx_mlp_map, hidden 1024) on the workload's shapes")
     ap.add_argument("--probe", action="store_true",
                     help="time the single-source R^2 probe (kvx_r2_probe) on the workload's shapes")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
-    w = syn.workload(args.workload)
+    over = {}
+    for kv in filter(None, args.override.split(",")):
+        key, val = kv.split("=")
+        over[key.strip()] = type(getattr(syn.WORKLOADS[args.workload], key.strip()))(val)
+    w = syn.workload(args.workload, **over)
     if args.fit:
         return fit_bench(args, w)
     if args.probe:
