@@ -440,7 +440,7 @@ def probe_bench(args, w):
 
 
 MLP_HIDDEN = 1024   # the paper's MLP baseline width
-E2E_CHUNK = 4096    # tokens per chunk of the host-buffer pipeline
+E2E_CHUNK = 2048    # tokens per chunk of the host-buffer pipeline (best of 1024..16384 in three sweeps)
 
 
 def mlp_bench(args, w):
