@@ -8,6 +8,7 @@
 #include <vector>
 
 #include "kvx_internal.h"
+#include "kvx_xh.h"
 
 namespace kvx {
 
@@ -281,7 +282,9 @@ kvx_status kvx_create(const kvx_config* cfg, int device, kvx_ctx** out) {
   ctx->tc_eligible = tc_supported(ctx, &why);
   ctx->xh_eligible = xh_supported(ctx, &why);
   if (ctx->tc_eligible || ctx->xh_eligible) {
-    kvx_status s = ctx->tc_eligible ? tc_prepare(ctx, c.W) : repack_wt(ctx, c.W);
+    kvx_status s = ctx->tc_eligible                  ? tc_prepare(ctx, c.W)
+                   : ctx->weight_dtype == KVX_F32 ? repack_wt_hilo(ctx, c.W)
+                                                  : repack_wt(ctx, c.W);
     if (s != KVX_OK) {
       free_ctx(ctx);
       return s;

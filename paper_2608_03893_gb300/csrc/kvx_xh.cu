@@ -37,6 +37,7 @@
 #include <climits>
 #include <cstring>
 #include <string>
+#include <vector>
 
 #include "kvx_internal.h"
 #include "kvx_ptx.cuh"
@@ -82,6 +83,7 @@ struct XhParams {
   const float* bias;      // [L_t][2][H][128]
   int32_t* status;
   int32_t Lt, H, k, pairs, n_units, out_bh;
+  int32_t lo_steps;       // fp32 weights: k n_kv further K steps over the same source tiles with W_lo
   RopeTables rope;
 };
 
@@ -207,7 +209,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
   cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
-  const int H = P.H, k = P.k, steps = P.k * P.H;
+  const int H = P.H, k = P.k, src_steps = P.k * P.H, steps = src_steps + P.lo_steps;
   const int n_units = P.n_units, pairs = P.pairs;
   const MapArgs& A = P.a;
 
@@ -230,7 +232,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
           const uint32_t round = sn / kXStages;
           if (round == 0 || mbar_test_wait(smem_u32(&empty[st]), (round - 1) & 1u)) {
             // step ss: source layer sel[l][ss / H], head ss % H; features ss*128 .. of W^T
-            const int j = ss / H, hs = ss % H;
+            const int j = (ss % src_steps) / H, hs = ss % H;
             const int L = __ldg(&P.sel[sun.l * k + j]);
             if (rank == 0) mbar_expect_tx(smem_u32(&full[st]), 2 * kXStageBytes);
             const uint32_t bar = mapa_shared(smem_u32(&full[st]), 0);
@@ -492,6 +494,47 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
 
 }  // namespace
 
+kvx_status repack_wt_hilo(kvx_ctx* c, const void* W_host) {
+  // W fp32 [L_t][2][H][F][128] -> W^T bf16 [L_t][2][H][128][2F]: columns [0, F) hold
+  // hi = bf16(w), columns [F, 2F) lo = bf16(w - hi), so X W = X W_hi + X W_lo to within
+  // 2^-17 of each weight (the paper keeps W in fp32)
+  const size_t F = c->F;
+  const size_t blocks = static_cast<size_t>(c->Lt) * 2 * c->H;
+  std::vector<uint16_t> wt(blocks * 2 * F * kXD);
+  const float* w = static_cast<const float*>(W_host);
+  auto bf16_rne = [](float x, float* back) {
+    uint32_t u;
+    std::memcpy(&u, &x, 4);
+    if ((u & 0x7F800000u) != 0x7F800000u) u += 0x7FFFu + ((u >> 16) & 1u);   // round to nearest even
+    const uint32_t r = u & 0xFFFF0000u;
+    std::memcpy(back, &r, 4);
+    return static_cast<uint16_t>(r >> 16);
+  };
+  for (size_t blk = 0; blk < blocks; ++blk) {
+    const float* srcb = w + blk * F * kXD;
+    uint16_t* dstb = wt.data() + blk * 2 * F * kXD;
+    for (size_t f = 0; f < F; ++f)
+      for (int n = 0; n < kXD; ++n) {
+        const float x = srcb[f * kXD + n];
+        float hi = 0.f, lo = 0.f;
+        const uint16_t h = bf16_rne(x, &hi);
+        const uint16_t l = bf16_rne(x - hi, &lo);
+        dstb[static_cast<size_t>(n) * 2 * F + f] = h;
+        dstb[static_cast<size_t>(n) * 2 * F + F + f] = l;
+      }
+  }
+  cudaError_t e = cudaMalloc(&c->d_Wt, wt.size() * 2);
+  if (e != cudaSuccess) {
+    set_error(std::string("kvx_create: cudaMalloc W^T: ") + cudaGetErrorString(e));
+    return KVX_ERR_OOM;
+  }
+  if ((e = cudaMemcpy(c->d_Wt, wt.data(), wt.size() * 2, cudaMemcpyHostToDevice)) != cudaSuccess) {
+    set_error(std::string("kvx_create: upload W^T: ") + cudaGetErrorString(e));
+    return KVX_ERR_CUDA;
+  }
+  return KVX_OK;
+}
+
 void launch_key_strip(const void* src_k, const int64_t* ss, void* ws, const int32_t* pos, int Ls, int H, int B, int T,
                       const RopeTables& rope, int sms, cudaStream_t stream) {
   const int64_t threads = static_cast<int64_t>(B) * T * 16;
@@ -502,7 +545,7 @@ void launch_key_strip(const void* src_k, const int64_t* ss, void* ws, const int3
 
 bool xh_supported(const kvx_ctx* c, std::string* why) {
   std::string w;
-  if (c->cache_dtype != KVX_BF16 || c->weight_dtype != KVX_BF16) w = "needs bf16 caches and weights";
+  if (c->cache_dtype != KVX_BF16) w = "needs bf16 caches";
   else if (c->d != kXD) w = "needs head_dim 128";
   else if (c->head_mix != KVX_CROSS_HEAD) w = "needs the cross-head feature layout";
   else if (c->rope_style != KVX_ROPE_HALF) w = "needs half-split RoPE pairs";
@@ -589,8 +632,10 @@ kvx_status launch_xh(kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
     }
   }
   {  // W^T [L_t*2*H*128][F], box 64 features x 128 rows
-    const cuuint64_t wdims[2] = {static_cast<cuuint64_t>(c->F), static_cast<cuuint64_t>(c->Lt) * 2 * c->H * kXD};
-    const cuuint64_t wstr[1] = {static_cast<cuuint64_t>(c->F) * 2};
+    // fp32 weights: W^T holds [W_hi | W_lo], 2F columns (see repack_wt_hilo)
+    const cuuint64_t wcols = static_cast<cuuint64_t>(c->F) * (c->weight_dtype == KVX_F32 ? 2 : 1);
+    const cuuint64_t wdims[2] = {wcols, static_cast<cuuint64_t>(c->Lt) * 2 * c->H * kXD};
+    const cuuint64_t wstr[1] = {wcols * 2};
     const cuuint32_t wbox[2] = {64, 128};
     CUresult r = encode(&P.tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, c->d_Wt, wdims, wstr, wbox, ones,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -614,6 +659,7 @@ kvx_status launch_xh(kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
     return KVX_ERR_UNSUPPORTED;
   }
   P.n_units = static_cast<int>(units);
+  P.lo_steps = c->weight_dtype == KVX_F32 ? c->k * c->H : 0;
   P.rope = c->rope;
 
   // 1. strip the source RoPE from every key into the workspace

@@ -533,3 +533,36 @@ def test_map_host_equals_device_map(name, over, kernel, chunk):
         if pipe:
             kvx.kvx_host_pipe_destroy(pipe)
         kvx.kvx_destroy(ctx)
+
+
+# ------------------------------------------------ fp32 weights on the tensor cores -----
+
+def test_cross_head_tc_fp32_weights_hi_lo():
+    """Cross-head tensor-core kernel with fp32 W (the paper keeps W in fp32): W^T is split
+    into bf16 hi + lo and the K loop runs twice over the source tiles, so the result follows
+    the fp32 weights.  Every output within the usual bound of the oracle given the fp32 W;
+    at least 90 % of them equal to the correctly rounded fp32-W result (the rest sit within
+    accumulation error of a rounding midpoint), where W rounded to bf16 gets visibly fewer."""
+    w = syn.workload("qwen3_14b_32b_t32768_k4_xhead", Ls=4, Lt=3, H=2, B=1, T=300, k=2)
+    Wb, b = syn.weights(w)
+    g = torch.Generator().manual_seed(5)
+    # fp32 weights off the bf16 grid, with a same-sign residual so that it shows in sums
+    W32 = (Wb.float() * (1.0 + 2.0 ** -9 * (0.5 + 0.5 * torch.rand(Wb.shape, generator=g)))).contiguous()
+    ctx, sel, _, _ = make_ctx(w, kernel=kvx.KVX_KERNEL_TCGEN05, W=W32, b=b)
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w)
+        rk, rv, ak, av = oracle_full(w, sk, sv, pos, sel, W32, b)
+        tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        ok, ratio, rms, nbad = check(w, [to_f64(tk), to_f64(tv)], [rk, rv], [ak, av])
+        assert ok, "%d elements out of tolerance (worst %.3g x bound)" % (nbad, ratio)
+        from oracle import bf16 as obf16
+        gv = to_f64(tv)
+        exact = np.mean(gv == obf16.round_to_bf16_value(rv))
+        hk_, hv_ = oracle_full(w, sk, sv, pos, sel, Wb, b)[:2]     # W rounded to bf16
+        hi_only = np.mean(obf16.round_to_bf16_value(hv_) == obf16.round_to_bf16_value(rv))
+        assert exact >= 0.9 and exact > hi_only + 0.05, (exact, hi_only)
+    finally:
+        kvx.kvx_destroy(ctx)
