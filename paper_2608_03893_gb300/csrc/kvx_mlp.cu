@@ -6,8 +6,8 @@
 // RoPE after the bias, bf16 out.  Each hidden activation is stored in bf16 after its ReLU.
 //
 // Three GEMM passes per group of target layers, each one launch of tc_mlp_kernel (clusters
-// of two CTAs, pair MMAs cta_group::2 with M = 256 tokens, operands in shared memory by TMA,
-// fp32 accumulators in TMEM):
+// of two CTAs, pair MMAs cta_group::2 with M = 256 tokens, operands in shared memory by TMA
+// in three 64 KB stages of 128 features, fp32 accumulators in TMEM):
 //   pass 1: H1[l,kv] = relu(X_l W1[l,kv,:]^T + b1)  -- one GEMM per (l, K|V) over all heads'
 //           hidden units (N = H hidden), K = k H d; A tiles straight from the stripped-key
 //           workspace / the value cache (5-D TMA, as the cross-head ridge kernel);
@@ -16,9 +16,9 @@
 // H1 and H2 live in a workspace [group layer][K|V][token][H hidden] bf16.  Work unit =
 // (output tile of 256 columns, head, pair of 128-token tiles, sequence, K|V, layer), the
 // output tile fastest so the clusters in flight share the A tiles of one token-tile pair.
-// Roles (384 threads): warp 0 TMA producer, warp 1 TMEM allocator and (rank 0) MMA issuer,
-// warps 4-11 epilogue (two warpgroups: columns 0-127 and 128-255 of a tile; in pass 3
-// RoPE pairs 0-31 and 32-63).  Every wait is bounded (KVX_ERR_TIMEOUT).
+// Roles (384 threads): warp 0 TMA producer, warp 1 TMEM allocator and (rank 0) MMA issuer
+// (eight MMAs per stage), warps 4-11 epilogue (two warpgroups: columns 0-127 and 128-255 of
+// a tile; in pass 3 RoPE pairs 0-31 and 32-63).  Every wait is bounded (KVX_ERR_TIMEOUT).
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
@@ -44,9 +44,9 @@ constexpr int kMFirstEpi = 4;
 constexpr int kMEpiWarps = 8;
 constexpr int kMD = 128;                          // head_dim
 constexpr int kMTile = 128;                       // tokens per CTA
-constexpr int kMStages = 6;
-constexpr uint32_t kMABytes = kMTile * 64 * 2;    // 128 tokens x 64 features, 16 KB
-constexpr uint32_t kMBBytes = 128 * 64 * 2;       // 128 output rows x 64 features, 16 KB
+constexpr int kMStages = 3;
+constexpr uint32_t kMABytes = kMTile * 128 * 2;   // 128 tokens x 128 features (two 64-wide halves), 32 KB
+constexpr uint32_t kMBBytes = 128 * 128 * 2;      // 128 output rows x 128 features (two halves), 32 KB
 constexpr uint32_t kMStageBytes = kMABytes + kMBBytes;
 constexpr uint32_t kMAccCols = 256;
 constexpr uint32_t kMTmemCols = 512;
@@ -113,6 +113,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kMThreads, 1)
   const int unit0 = blockIdx.x >> 1, unit_step = gridDim.x >> 1;
   const bool narrow = P.pass == 3;         // N = 128: each CTA holds 64 rows of B
   const uint32_t b_bytes = narrow ? kMBBytes / 2 : kMBBytes;
+  const uint32_t b_half = b_bytes / 2;     // one 64-feature half of B
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < kMStages; ++i) {
@@ -166,19 +167,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kMThreads, 1)
           const uint32_t b_dst = a_dst + kMABytes;
           int wrow;
           if (P.pass == 1) {
-            // feature block s: source layer sel[l][s / 2H], head (s / 2) % H, half s % 2
-            const int j = s / (2 * H), hs = (s >> 1) % H;
+            // feature block s: source layer sel[l][s / H], head s % H
+            const int j = s / H, hs = s % H;
             const int L = __ldg(&P.sel[l * P.k + j]);
-            tma_load_5d_pair(a_dst, un.kv ? &P.tm_av : &P.tm_ak, bar, 64 * (s & 1), un.t0, hs, un.b, L, pol_a);
+            const CUtensorMap* tm = un.kv ? &P.tm_av : &P.tm_ak;
+            tma_load_5d_pair(a_dst, tm, bar, 0, un.t0, hs, un.b, L, pol_a);
+            tma_load_5d_pair(a_dst + kMABytes / 2, tm, bar, 64, un.t0, hs, un.b, L, pol_a);
             wrow = (l * 2 + un.kv) * H * P.hidden + un.nt * 256;
           } else {
             const int row = static_cast<int>((static_cast<int64_t>(un.lg) * 2 + un.kv) * N +
                                              static_cast<int64_t>(un.b) * P.a.T + un.t0);
-            tma_load_2d_pair(a_dst, &P.tm_h, bar, un.h * P.hidden + 64 * s, row, pol_a);
+            tma_load_2d_pair(a_dst, &P.tm_h, bar, un.h * P.hidden + 128 * s, row, pol_a);
+            tma_load_2d_pair(a_dst + kMABytes / 2, &P.tm_h, bar, un.h * P.hidden + 128 * s + 64, row, pol_a);
             wrow = P.pass == 2 ? ((l * 2 + un.kv) * H + un.h) * P.hidden + un.nt * 256
                                : ((l * 2 + un.kv) * H + un.h) * kMD;
           }
-          tma_load_2d_pair(b_dst, &P.tm_w, bar, 64 * s, wrow + static_cast<int>(rank) * (narrow ? 64 : 128), pol_w);
+          const int brow = wrow + static_cast<int>(rank) * (narrow ? 64 : 128);
+          tma_load_2d_pair(b_dst, &P.tm_w, bar, 128 * s, brow, pol_w);
+          tma_load_2d_pair(b_dst + b_half, &P.tm_w, bar, 128 * s + 64, brow, pol_w);
         }
       }
       if (!ok && rank == 0) {   // the most recent loads may still be landing
@@ -211,8 +217,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kMThreads, 1)
           const uint32_t a0 = smem_u32(stages + static_cast<size_t>(st) * kMStageBytes);
           const uint32_t b0 = a0 + kMABytes;
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            tc_mma_ss_pair(d_tmem, sw128_desc(a0 + kk * 32), sw128_desc(b0 + kk * 32), idesc, (s | kk) != 0);
+          for (int half = 0; half < 2; ++half)
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              tc_mma_ss_pair(d_tmem, sw128_desc(a0 + half * (kMABytes / 2) + kk * 32),
+                             sw128_desc(b0 + half * b_half + kk * 32), idesc, (s | half | kk) != 0);
           issued = true;
           tc_commit_pair(smem_u32(&empty[st]), 3);
         }
@@ -619,7 +628,7 @@ KVX_API kvx_status kvx_mlp_map(const kvx_mlp_config* cfg, const kvx_src* src, in
         P.bias = pass == 1 ? cfg->b1 : pass == 2 ? cfg->b2 : cfg->b3;
         P.n_tiles = pass == 1 ? H * hid / 256 : pass == 2 ? hid / 256 : 1;
         P.heads = pass == 1 ? 1 : H;
-        P.ksteps = pass == 1 ? cfg->k * H * 2 : hid / 64;
+        P.ksteps = pass == 1 ? cfg->k * H : hid / 128;
         const int64_t units = static_cast<int64_t>(g_n) * 2 * batch * P.pairs * P.heads * P.n_tiles;
         if (units > INT_MAX) {
           set_error("kvx_mlp_map: too many work units");
