@@ -75,6 +75,15 @@ typedef enum { KVX_PER_HEAD = 0, KVX_CROSS_HEAD = 1 } kvx_head_mix;
  * kvx_destroy frees it. */
 typedef enum { KVX_KERNEL_AUTO = 0, KVX_KERNEL_SIMT = 1, KVX_KERNEL_TCGEN05 = 2 } kvx_kernel;
 
+/* RoPE numerics.  EXACT: angles t omega_i to ~1e-6 rad and the rotations in fp32 (the
+ * definition; the default).  HF: the rounding of the Hugging Face bf16 forward that wrote
+ * the caches -- the angle is the fp32 product of fp32(t) and fp32(omega_i), cos and sin of
+ * it are rounded to the cache dtype, and each product and sum of the rotation is rounded
+ * to the cache dtype (x' = r(r(a c) + r(-b s)), y' = r(r(b c) + r(a s)); the strip uses -s);
+ * the mapped keys are rounded to the cache dtype before the target rotation.  HF runs on
+ * the SIMT kernel only (AUTO picks it; TCGEN05 is UNSUPPORTED). */
+typedef enum { KVX_ROPE_EXACT = 0, KVX_ROPE_HF = 1 } kvx_rope_numerics;
+
 /* Llama-3 RoPE frequency scaling (the rope_scaling of the Llama 3.1 checkpoints:
  * factor 8, low_freq_factor 1, high_freq_factor 4, original_max_position 8192).  With
  * omega_i = theta^(-2i/d) and wavelength 2 pi / omega_i: below original_max_position /
@@ -115,6 +124,7 @@ typedef struct {
   /* RoPE frequency scaling of the source / target model, or NULL (plain theta). */
   const kvx_rope_scaling* src_rope_scaling;
   const kvx_rope_scaling* tgt_rope_scaling;
+  int32_t rope_numerics;     /* kvx_rope_numerics */
 } kvx_config;
 
 /* Source cache, DEVICE memory owned by the caller: element (layer l, batch b, head h,

@@ -19,6 +19,11 @@ Two feature layouts:
                       "Run information", source-feature row): F = k H d.
 The per-head map equals the cross-head map with W zero outside head h's rows.
 
+RoPE numerics (``rope_numerics``): ``"exact"`` (the definition above) or ``"hf"`` -- the
+rounding of the Hugging Face forward that wrote the caches (rope.rotate_hf: fp32 angle,
+cos / sin and every product and sum of the rotation rounded to the cache dtype, the mapped
+key rounded before the target rotation).
+
 Two rounding models:
 * ``"exact"``   -- everything in float64.
 * ``"bf16fwd"`` -- the paper's forward runs in bf16 (Appendix "Run information"):
@@ -69,7 +74,8 @@ def _pair_sum(y, style):
 
 
 def map_tokens(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
-               mode="exact", style="half", head_mix="per_head", rounding_slack=None):
+               mode="exact", style="half", head_mix="per_head", rounding_slack=None,
+               rope_numerics="exact"):
     """Map a set of tokens.
 
     src_k, src_v : float64 [L_s][H][N][d]  -- stored (rotated) source keys, values.
@@ -86,7 +92,12 @@ def map_tokens(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
     sel = np.asarray(sel)
     Ls, H, N, d = src_k.shape
     Lt, k = sel.shape
-    stripped = rope.rotate(src_k, pos[None, None, :], theta_s, inverse=True, style=style)
+    hf = rope_numerics == "hf"
+    if hf:   # the HF forward's strip: already rounded to bf16 (mode bf16fwd)
+        stripped = rope.rotate_hf(src_k, pos[None, None, :], theta_s, inverse=True, style=style,
+                                  bf16_cache=(mode == "bf16fwd"))
+    else:
+        stripped = rope.rotate(src_k, pos[None, None, :], theta_s, inverse=True, style=style)
     feats = (stripped, src_v)
     out = np.empty((2, Lt, H, N, d), dtype=np.float64)
     want_slack = rounding_slack is not None and mode == "bf16fwd"
@@ -113,7 +124,8 @@ def map_tokens(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
                 if b is not None:
                     Y = Y + b[l, kv, h]
                 if kv == 0:
-                    Y = rope.rotate(Y, pos, theta_t, style=style)
+                    Y = (rope.rotate_hf(Y, pos, theta_t, style=style, bf16_cache=(mode == "bf16fwd")) if hf
+                         else rope.rotate(Y, pos, theta_t, style=style))
                 out[kv, l, h] = Y
                 if want_slack and kv == 0:
                     if head_mix == "per_head":
@@ -127,7 +139,8 @@ def map_tokens(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
 
 
 def map_cache(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
-              mode="exact", style="half", head_mix="per_head", rounding_slack=None):
+              mode="exact", style="half", head_mix="per_head", rounding_slack=None,
+              rope_numerics="exact"):
     """Contiguous-cache form: src [L_s][B][H][T][d], positions [B][T] ->
     (out_k, out_v) [L_t][B][H][T][d] (plus the two slacks with ``rounding_slack``)."""
     src_k = np.asarray(src_k, dtype=np.float64)
@@ -139,7 +152,7 @@ def map_cache(src_k, src_v, positions, sel, W, b, theta_s, theta_t,
         return x.transpose(0, 2, 1, 3, 4).reshape(x.shape[0], H, B * T, d)
 
     res = map_tokens(tok(src_k), tok(src_v), pos, sel, W, b, theta_s, theta_t,
-                     mode, style, head_mix, rounding_slack)
+                     mode, style, head_mix, rounding_slack, rope_numerics)
     Lt = res[0].shape[0]
 
     def untok(y):

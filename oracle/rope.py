@@ -81,6 +81,40 @@ def _unpairs(a, b, style):
     return out
 
 
+def hf_cos_sin(positions, theta, d, bf16_cache=True):
+    """cos and sin as the Hugging Face bf16 forward forms them: the angle is the fp32
+    product of fp32(t) and fp32(omega_i) (omega_i rounded once from its exact value), its
+    cos and sin are taken exactly and rounded to the cache dtype (bf16, or fp32)."""
+    from . import bf16 as _bf16
+    w32 = inv_freq(theta, d).astype(np.float32)
+    p32 = np.asarray(positions).astype(np.float32)
+    ang = (p32[..., None] * w32).astype(np.float32).astype(np.float64)   # fp32 multiply, rounded
+    c, s = np.cos(ang), np.sin(ang)
+    if bf16_cache:
+        return _bf16.round_to_bf16_value(c), _bf16.round_to_bf16_value(s)
+    return c.astype(np.float32).astype(np.float64), s.astype(np.float32).astype(np.float64)
+
+
+def rotate_hf(x, positions, theta, inverse=False, style="half", bf16_cache=True):
+    """The rotation with the rounding of a Hugging Face forward in the cache dtype: with
+    (c, s) from hf_cos_sin and r() the rounding to the cache dtype,
+        a' = r(r(a c) - r(b s)),  b' = r(r(b c) + r(a s))      (inverse: s -> -s).
+    x is taken as a cache-dtype tensor (rounded first)."""
+    from . import bf16 as _bf16
+
+    def r(v):
+        v = np.asarray(v, dtype=np.float64)
+        return _bf16.round_to_bf16_value(v) if bf16_cache else v.astype(np.float32).astype(np.float64)
+
+    x = r(x)
+    d = x.shape[-1]
+    c, s = hf_cos_sin(np.broadcast_to(np.asarray(positions), x.shape[:-1]), theta, d, bf16_cache)
+    if inverse:
+        s = -s
+    a, b = _pairs(x, style)
+    return _unpairs(r(r(a * c) - r(b * s)), r(r(b * c) + r(a * s)), style)
+
+
 def rotate(x, positions, theta, inverse=False, style="half"):
     """Apply R_Theta(t) (or its inverse) to the last axis of ``x``.
 

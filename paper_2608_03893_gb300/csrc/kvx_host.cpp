@@ -186,6 +186,8 @@ kvx_status kvx_create(const kvx_config* cfg, int device, kvx_ctx** out) {
   if (c.head_mix != KVX_PER_HEAD && c.head_mix != KVX_CROSS_HEAD)
     return fail(KVX_ERR_INVALID_ARG, "kvx_create: bad head_mix");
   if (c.reserved != 0) return fail(KVX_ERR_INVALID_ARG, "kvx_create: reserved must be 0");
+  if (c.rope_numerics != KVX_ROPE_EXACT && c.rope_numerics != KVX_ROPE_HF)
+    return fail(KVX_ERR_INVALID_ARG, "kvx_create: bad rope_numerics");
   if (const char* why = check_rope_scaling(c.src_rope_scaling))
     return fail(KVX_ERR_INVALID_ARG, std::string("kvx_create: source ") + why);
   if (const char* why = check_rope_scaling(c.tgt_rope_scaling))
@@ -237,6 +239,7 @@ kvx_status kvx_create(const kvx_config* cfg, int device, kvx_ctx** out) {
     }
   }
   set_rope_scaling(ctx, c.src_rope_scaling, c.tgt_rope_scaling);
+  ctx->rope_numerics = c.rope_numerics;
   fill_rope(ctx);
 
   DeviceGuard guard(device);
@@ -279,8 +282,9 @@ kvx_status kvx_create(const kvx_config* cfg, int device, kvx_ctx** out) {
   }
 
   std::string why;
-  ctx->tc_eligible = tc_supported(ctx, &why);
-  ctx->xh_eligible = xh_supported(ctx, &why);
+  // the tensor-core kernels compute the RoPE exactly; the HF numerics run on the SIMT kernel
+  ctx->tc_eligible = ctx->rope_numerics == KVX_ROPE_EXACT && tc_supported(ctx, &why);
+  ctx->xh_eligible = ctx->rope_numerics == KVX_ROPE_EXACT && xh_supported(ctx, &why);
   if (ctx->tc_eligible || ctx->xh_eligible) {
     kvx_status s = ctx->tc_eligible                  ? tc_prepare(ctx, c.W)
                    : ctx->weight_dtype == KVX_F32 ? repack_wt_hilo(ctx, c.W)

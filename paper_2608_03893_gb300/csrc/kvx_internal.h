@@ -60,6 +60,7 @@ struct kvx_ctx {
   int Ls = 0, Lt = 0, H = 0, d = 0, k = 0, F = 0;
   int rope_style = 0, cache_dtype = 0, weight_dtype = 0, head_mix = 0;
   double theta_s = 0, theta_t = 0;
+  int rope_numerics = 0;                          // kvx_rope_numerics
   bool scale_s_on = false, scale_t_on = false;   // Llama-3 frequency scaling per side
   kvx_rope_scaling scale_s{}, scale_t{};
   int kernel = KVX_KERNEL_AUTO;

@@ -28,7 +28,7 @@ struct SimtParams {
   const void* W;
   const float* bias;
   int32_t* status;
-  int32_t Lt, H, d, k, F, cross, interleaved, cache_bf16, weight_bf16, tt;
+  int32_t Lt, H, d, k, F, cross, interleaved, cache_bf16, weight_bf16, tt, hf;
   RopeTables rope;
 };
 
@@ -45,6 +45,20 @@ __device__ __forceinline__ void store_elem(void* p, int64_t i, float v, int bf16
 }
 
 __device__ __forceinline__ void report(int32_t* status, int code) { atomicCAS(status, 0, code); }
+
+// Rounding to the cache dtype (bf16 round-to-nearest-even, or nothing for fp32 caches).
+__device__ __forceinline__ float rc(float x, int bf16) {
+  return bf16 ? __bfloat162float(__float2bfloat16_rn(x)) : x;
+}
+
+// HF numerics: cos and sin of the fp32 angle fp32(t) * fp32(omega), rounded to the cache
+// dtype (the library sincosf, which reduces any fp32 argument).
+__device__ __forceinline__ void hf_sincos(int t, float w, int bf16, float* s, float* c) {
+  float sv, cv;
+  sincosf(__fmul_rn(static_cast<float>(t), w), &sv, &cv);
+  *s = rc(sv, bf16);
+  *c = rc(cv, bf16);
+}
 
 __global__ void __launch_bounds__(kSimtThreads) simt_map_kernel(const __grid_constant__ SimtParams P) {
   extern __shared__ float smem[];
@@ -95,7 +109,17 @@ __global__ void __launch_bounds__(kSimtThreads) simt_map_kernel(const __grid_con
       const int64_t base = s * a.ss[0] + b * a.ss[1] + hs * a.ss[2] + static_cast<int64_t>(t0 + tt) * a.ss[3];
       xa = load_elem(src, base + ia, P.cache_bf16);
       xb = load_elem(src, base + ib, P.cache_bf16);
-      if (kv == 0) {
+      if (kv == 0 && P.hf) {
+        // the HF rotation with -sin: every product and sum rounded to the cache dtype
+        float sn, cs;
+        hf_sincos(p, P.rope.ws_hi[i], P.cache_bf16, &sn, &cs);
+        const float na = rc(__fadd_rn(rc(__fmul_rn(xa, cs), P.cache_bf16), rc(__fmul_rn(xb, sn), P.cache_bf16)),
+                            P.cache_bf16);
+        const float nb = rc(__fsub_rn(rc(__fmul_rn(xb, cs), P.cache_bf16), rc(__fmul_rn(xa, sn), P.cache_bf16)),
+                            P.cache_bf16);
+        xa = na;
+        xb = nb;
+      } else if (kv == 0) {
         float sn, cs;
         rope_sincos(p, P.rope.ws_hi[i], P.rope.ws_lo[i], P.rope.two_pi_hi, P.rope.two_pi_lo,
                     P.rope.inv_two_pi, &sn, &cs);
@@ -146,7 +170,18 @@ __global__ void __launch_bounds__(kSimtThreads) simt_map_kernel(const __grid_con
     const int ia = P.interleaved ? 2 * i : i;
     const int ib = P.interleaved ? 2 * i + 1 : i + half;
     float ya = Y[tt * d + ia], yb = Y[tt * d + ib];
-    if (kv == 0) {
+    if (kv == 0 && P.hf) {
+      // the mapped key as a cache-dtype tensor, then the HF rotation at the target angle
+      const int bf = P.cache_bf16;
+      ya = rc(ya, bf);
+      yb = rc(yb, bf);
+      float sn, cs;
+      hf_sincos(p, P.rope.wt_hi[i], bf, &sn, &cs);
+      const float na = rc(__fsub_rn(rc(__fmul_rn(ya, cs), bf), rc(__fmul_rn(yb, sn), bf)), bf);
+      const float nb = rc(__fadd_rn(rc(__fmul_rn(yb, cs), bf), rc(__fmul_rn(ya, sn), bf)), bf);
+      ya = na;
+      yb = nb;
+    } else if (kv == 0) {
       float sn, cs;
       rope_sincos(p, P.rope.wt_hi[i], P.rope.wt_lo[i], P.rope.two_pi_hi, P.rope.two_pi_lo,
                   P.rope.inv_two_pi, &sn, &cs);
@@ -196,6 +231,7 @@ kvx_status launch_simt(const kvx_ctx* ctx, const MapArgs& a, cudaStream_t stream
   P.cache_bf16 = ctx->cache_dtype == KVX_BF16;
   P.weight_bf16 = ctx->weight_dtype == KVX_BF16;
   P.rope = ctx->rope;
+  P.hf = ctx->rope_numerics == KVX_ROPE_HF;
   constexpr size_t kSmemBudget = 96 * 1024;
   const size_t per_token = (static_cast<size_t>(ctx->F) + ctx->d) * sizeof(float) + sizeof(int);
   int tt = static_cast<int>(kSmemBudget / per_token);

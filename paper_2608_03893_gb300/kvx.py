@@ -19,6 +19,7 @@ KVX_OK, KVX_ERR_INVALID_ARG, KVX_ERR_UNSUPPORTED, KVX_ERR_OOM = 0, 1, 2, 3
 KVX_ERR_CUDA, KVX_ERR_TIMEOUT, KVX_ERR_DEVICE_BOUNDS = 4, 5, 6
 KVX_F32, KVX_BF16 = 0, 1
 KVX_ROPE_HALF, KVX_ROPE_INTERLEAVED = 0, 1
+KVX_ROPE_EXACT, KVX_ROPE_HF = 0, 1
 KVX_PER_HEAD, KVX_CROSS_HEAD = 0, 1
 KVX_KERNEL_AUTO, KVX_KERNEL_SIMT, KVX_KERNEL_TCGEN05 = 0, 1, 2
 
@@ -60,7 +61,7 @@ class kvx_config(ctypes.Structure):
         ("weight_dtype", ctypes.c_int32), ("head_mix", ctypes.c_int32), ("reserved", ctypes.c_int32),
         ("selection", ctypes.c_void_p), ("selection_scores", ctypes.c_void_p),
         ("W", ctypes.c_void_p), ("b", ctypes.c_void_p),
-    ] + _SCALING
+    ] + _SCALING + [("rope_numerics", ctypes.c_int32)]
 
 
 class kvx_src(ctypes.Structure):
@@ -284,7 +285,8 @@ def dtype_code(t):
 
 def config_from_tensors(*, src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t,
                         cache_dtype, W, b=None, selection=None, scores=None,
-                        rope_style=KVX_ROPE_HALF, head_mix=KVX_PER_HEAD, rope_scaling=None):
+                        rope_style=KVX_ROPE_HALF, head_mix=KVX_PER_HEAD, rope_scaling=None,
+                        rope_numerics=0):
     """Build a kvx_config from host tensors.  Returns (cfg, keepalive) -- hold
     ``keepalive`` until kvx_create returns."""
     import numpy as np
@@ -308,6 +310,7 @@ def config_from_tensors(*, src_layers, tgt_layers, n_kv_heads, head_dim, k, thet
     cfg.b = _ptr(bc)
     rs = globals()["rope_scaling"](rope_scaling)
     cfg.src_rope_scaling = cfg.tgt_rope_scaling = _scaling_ptr(rs)
+    cfg.rope_numerics = int(rope_numerics)
     return cfg, (Wc, bc, sel, sc, torch, rs)
 
 

@@ -270,3 +270,11 @@ def test_host_pipe_rejects_bad_arguments_before_touching_the_device():
     with pytest.raises(kvx.KvxError) as e:
         kvx.kvx_map_host(None, src, 16, p, tgt)
     assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+
+
+def test_create_rejects_bad_rope_numerics():
+    cfg, keep = _cfg()
+    cfg.rope_numerics = 2
+    with pytest.raises(kvx.KvxError) as e:
+        kvx.kvx_create(cfg, 0)
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG

@@ -566,3 +566,51 @@ def test_cross_head_tc_fp32_weights_hi_lo():
         assert exact >= 0.9 and exact > hi_only + 0.05, (exact, hi_only)
     finally:
         kvx.kvx_destroy(ctx)
+
+
+# ---------------------------------------------------------------- HF RoPE numerics -----
+
+def test_hf_rope_numerics_simt():
+    """KVX_ROPE_HF (the rounding of the Hugging Face bf16 forward: fp32 angle, bf16 cos/sin,
+    each product and sum rounded) on the SIMT kernel against the oracle in the same numerics,
+    at positions past 2 * 10^4 where the fp32 angle is coarse: every output within the
+    usual bound, at least 90 % of the keys bit-equal to the oracle's (the rest follow a
+    rounding of the fp32-accumulated contraction or of cos / sin near a bf16 midpoint), far
+    more than agree with the exact-RoPE oracle.  The tensor-core kernels refuse the mode."""
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=5, Lt=4, H=2, B=2, T=200, k=2, theta_t=5e5)
+    W, b = syn.weights(w)
+    scores = syn.selection_scores(w)
+    cfg, keep = kvx.config_from_tensors(
+        src_layers=w.Ls, tgt_layers=w.Lt, n_kv_heads=w.H, head_dim=w.d, k=w.k, theta_s=w.theta_s,
+        theta_t=w.theta_t, cache_dtype=w.cache_dtype, W=W, b=b, scores=scores, rope_numerics=kvx.KVX_ROPE_HF)
+    ctx = kvx.kvx_create(cfg, 0)
+    try:
+        with pytest.raises(kvx.KvxError) as e:
+            kvx.kvx_set_kernel(ctx, kvx.KVX_KERNEL_TCGEN05)
+        assert e.value.status == kvx.KVX_ERR_UNSUPPORTED
+        sel = kvx.kvx_get_selection(ctx, w.Lt, w.k)
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w) + np.array([[20011], [31007]], dtype=np.int32)
+        tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        sk64, sv64 = to_f64(sk), to_f64(sv)
+        rk, rv = omap.map_cache(sk64, sv64, pos, sel, to_f64(W), to_f64(b), w.theta_s, w.theta_t,
+                                mode="bf16fwd", rope_numerics="hf")
+        ek, ev = omap.map_cache(sk64, sv64, pos, sel, to_f64(W), to_f64(b), w.theta_s, w.theta_t,
+                                mode="bf16fwd")
+        gk, gv = to_f64(tk), to_f64(tv)
+        ok, ratio, rms, nbad = check(w, [gv], [rv])
+        assert ok, "values: %d elements out of tolerance (worst %.3g x bound)" % (nbad, ratio)
+        # keys: a rounding taken on the other side of a bf16 midpoint (the mapped key before
+        # the rotation, or cos / sin) moves an output by a few bf16 steps of its pair's terms,
+        # so the bound scales with the pair magnitude |a| + |b| (4 steps: 2^-6 of it)
+        mag = np.concatenate([np.abs(rk[..., :64]) + np.abs(rk[..., 64:])] * 2, axis=-1)
+        err = np.abs(gk - rk)
+        assert np.all(err <= 2.0 ** -6 * mag + 1e-3 * rms), np.max(err / (2.0 ** -6 * mag + 1e-3 * rms))
+        from oracle import bf16 as obf16
+        same_hf = np.mean(gk == rk)
+        same_exact = np.mean(gk == obf16.round_to_bf16_value(ek))
+        assert same_hf >= 0.9 and same_hf > same_exact + 0.1, (same_hf, same_exact)
+    finally:
+        kvx.kvx_destroy(ctx)

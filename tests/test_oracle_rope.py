@@ -175,3 +175,39 @@ def test_llama3_scaling_identity_and_inv_freq_plumbing():
     y = rope.rotate(x, pos, spec)
     assert np.allclose(rope.rotate(y, pos, spec, inverse=True), x, atol=1e-12)
     assert np.allclose(np.linalg.norm(y, axis=-1), np.linalg.norm(x, axis=-1), atol=1e-12)
+
+
+# ---- Hugging Face numerics ------------------------------------------------------------
+
+def test_hf_rotation_worked_example():
+    """Worked by hand: pair i = 0 has omega = 1, so at t = 1 the fp32 angle is 1 rad;
+    cos 1 = 0.54030... = 1.0806 x 2^-1 rounds to 138/128 x 2^-1 = 0.5390625 in bf16 and
+    sin 1 = 0.84147... = 1.6829 x 2^-1 to 215/128 x 2^-1 = 0.83984375.  For (a, b) = (1, 1):
+    a' = r(0.5390625 - 0.83984375) = -0.30078125 (exact), b' = r(0.5390625 + 0.83984375) =
+    r(1.37890625) = 1.375 (176.5/128 is a tie, rounded to even).  For (1, 0): (c, s)."""
+    x = np.zeros((2, 128))
+    x[0, 0], x[0, 64] = 1.0, 1.0
+    x[1, 0] = 1.0
+    y = rope.rotate_hf(x, np.array([1, 1]), 1e6)
+    assert y[0, 0] == -0.30078125 and y[0, 64] == 1.375
+    assert y[1, 0] == 0.5390625 and y[1, 64] == 0.83984375
+    c, s = rope.hf_cos_sin(np.array([1]), 1e6, 128)
+    assert c[0, 0] == 0.5390625 and s[0, 0] == 0.83984375
+
+
+def test_hf_rotation_properties():
+    """Position 0 is the identity (cos 1, sin 0 exactly); results are bf16 values; the HF
+    rotation stays within the bf16 rounding of the exact one; its inverse undoes it up to
+    that rounding."""
+    rng = np.random.default_rng(4)
+    from oracle import bf16
+    x = bf16.round_to_bf16_value(rng.standard_normal((16, 128)))
+    assert np.array_equal(rope.rotate_hf(x, np.zeros(16, dtype=int), 5e5), x)
+    pos = rng.integers(0, 40000, size=16)
+    y = rope.rotate_hf(x, pos, 5e5)
+    assert np.array_equal(y, bf16.round_to_bf16_value(y))
+    ex = rope.rotate(x, pos, 5e5)
+    mag = np.concatenate([np.abs(x[:, :64]) + np.abs(x[:, 64:])] * 2, axis=-1)
+    assert np.all(np.abs(y - ex) <= 2.0 ** -6 * mag + 1e-6 * np.abs(pos)[:, None] * mag)
+    back = rope.rotate_hf(y, pos, 5e5, inverse=True)
+    assert np.all(np.abs(back - x) <= 2.0 ** -5 * mag + 1e-6 * np.abs(pos)[:, None] * mag)
