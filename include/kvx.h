@@ -255,6 +255,7 @@ typedef struct {
                                   * holds every token in one pass (less: tokens in chunks) */
   const kvx_rope_scaling* src_rope_scaling;   /* NULL: plain theta (see kvx_rope_scaling) */
   const kvx_rope_scaling* tgt_rope_scaling;
+  int32_t rope_numerics;        /* kvx_rope_numerics: the strip of both sides' keys */
 } kvx_fit_config;
 KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, const kvx_src* tgt, int32_t batch,
                                  int32_t tokens_per_seq, const int32_t* positions, float* W, float* b,
@@ -292,6 +293,7 @@ typedef struct {
   uint64_t workspace_bytes;
   const kvx_rope_scaling* src_rope_scaling;   /* NULL: plain theta (see kvx_rope_scaling) */
   const kvx_rope_scaling* tgt_rope_scaling;
+  int32_t rope_numerics;        /* kvx_rope_numerics: the strip of both sides' keys */
 } kvx_probe_config;
 KVX_API kvx_status kvx_r2_probe(const kvx_probe_config* cfg, const kvx_src* src, const kvx_src* tgt, int32_t batch,
                                 int32_t tokens_per_seq, const int32_t* positions, double* scores, double* r2_kv,

@@ -413,6 +413,7 @@ const char* check_fit_config(const kvx_fit_config* cfg) {
   for (int64_t i = 0; i < static_cast<int64_t>(cfg->tgt_layers) * cfg->k; ++i)
     if (cfg->selection[i] < 0 || cfg->selection[i] >= cfg->src_layers) return "selection entry out of range";
   if (cfg->workspace_bytes != 0 && !cfg->workspace) return "workspace_bytes without a workspace";
+  if (cfg->rope_numerics != KVX_ROPE_EXACT && cfg->rope_numerics != KVX_ROPE_HF) return "bad rope_numerics";
   if (const char* why = check_rope_scaling(cfg->src_rope_scaling)) return why;
   if (const char* why = check_rope_scaling(cfg->tgt_rope_scaling)) return why;
   if (reinterpret_cast<uintptr_t>(cfg->workspace) & 255u) return "workspace must be 256-byte aligned";
@@ -492,6 +493,7 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
   G.Ls = cfg->src_layers;
   G.Lt = cfg->tgt_layers;
   G.rope = tmp.rope;
+  G.hf = cfg->rope_numerics == KVX_ROPE_HF;
   G.sm_count = sms;
 
   // device pieces: from the caller's workspace, or one stream-ordered allocation

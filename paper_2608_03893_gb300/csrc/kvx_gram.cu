@@ -74,9 +74,11 @@ struct PackParams {
   int64_t n0;                  // first token of the chunk (pack) or 0 (sums)
   int64_t n_end;               // tokens past n_end are zero padding
   int32_t np;                  // tokens per workspace row (multiple of 64)
-  int32_t B, T, H, Ls, Lt;
+  int32_t B, T, H, Ls, Lt, hf;
   RopeTables rope;
 };
+
+__device__ __forceinline__ float rbf(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
 
 __device__ __forceinline__ void greport(int32_t* status, int code) { atomicCAS(status, 0, code); }
 
@@ -123,8 +125,14 @@ __global__ void __launch_bounds__(kGPackThreads, 2) gram_pack_kernel(const __gri
 #pragma unroll
     for (int m = 0; m < 8; ++m) {
       float sv, cv;
-      rope_sincos(p, w_hi[8 * g + m], w_lo[8 * g + m], P.rope.two_pi_hi, P.rope.two_pi_lo, P.rope.inv_two_pi, &sv,
-                  &cv);
+      if (P.hf) {   // HF numerics: cos / sin of the fp32 angle, rounded to bf16
+        sincosf(__fmul_rn(static_cast<float>(p), w_hi[8 * g + m]), &sv, &cv);
+        sv = rbf(sv);
+        cv = rbf(cv);
+      } else {
+        rope_sincos(p, w_hi[8 * g + m], w_lo[8 * g + m], P.rope.two_pi_hi, P.rope.two_pi_lo, P.rope.inv_two_pi,
+                    &sv, &cv);
+      }
       trig[trig_index(0, q, m, g, lane)] = cv;
       trig[trig_index(1, q, m, g, lane)] = sv;
     }
@@ -161,7 +169,11 @@ __global__ void __launch_bounds__(kGPackThreads, 2) gram_pack_kernel(const __gri
         for (int m = 0; m < 8; ++m) {
           const float a = (m & 1) ? bf16_hi(wa[m >> 1]) : bf16_lo(wa[m >> 1]);
           const float b = (m & 1) ? bf16_hi(wb[m >> 1]) : bf16_lo(wb[m >> 1]);
-          if (kv == 0) {   // rotation by -t omega: a' = a c + b s, b' = b c - a s
+          if (kv == 0 && P.hf) {   // the HF strip: each product and sum rounded to bf16
+            const float cv = trig[trig_index(0, q, m, g, lane)], sv = trig[trig_index(1, q, m, g, lane)];
+            va[q][m] = rbf(__fadd_rn(rbf(__fmul_rn(a, cv)), rbf(__fmul_rn(b, sv))));
+            vb[q][m] = rbf(__fsub_rn(rbf(__fmul_rn(b, cv)), rbf(__fmul_rn(a, sv))));
+          } else if (kv == 0) {   // rotation by -t omega: a' = a c + b s, b' = b c - a s
             const float cv = trig[trig_index(0, q, m, g, lane)], sv = trig[trig_index(1, q, m, g, lane)];
             va[q][m] = __fmaf_rn(a, cv, __fmul_rn(b, sv));
             vb[q][m] = __fmaf_rn(b, cv, -__fmul_rn(a, sv));
@@ -498,6 +510,7 @@ PackParams pack_params(const GramSpec& s) {
   P.H = s.H;
   P.Ls = s.Ls;
   P.Lt = s.Lt;
+  P.hf = s.hf;
   P.rope = s.rope;
   return P;
 }

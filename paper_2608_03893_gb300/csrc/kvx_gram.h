@@ -20,6 +20,7 @@ struct GramSpec {
   const int32_t* pos;               // device [B][T]
   int32_t B = 0, T = 0, H = 0, Ls = 0, Lt = 0;
   RopeTables rope{};
+  int32_t hf = 0;                   // strip with the HF numerics (kvx_rope_numerics)
   std::vector<int32_t> slot_side;   // host: the operands' (side, layer), one per slot
   std::vector<int32_t> slot_layer;
   double* sums = nullptr;           // device [2 sides][2 kv][L][H][128] (side 0: L_s rows,

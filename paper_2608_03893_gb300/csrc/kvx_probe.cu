@@ -236,6 +236,7 @@ const char* check_probe_config(const kvx_probe_config* cfg) {
       !std::isfinite(cfg->tgt_rope_theta))
     return "the RoPE bases must be finite and > 1";
   if (cfg->workspace_bytes != 0 && !cfg->workspace) return "workspace_bytes without a workspace";
+  if (cfg->rope_numerics != KVX_ROPE_EXACT && cfg->rope_numerics != KVX_ROPE_HF) return "bad rope_numerics";
   if (const char* why = check_rope_scaling(cfg->src_rope_scaling)) return why;
   if (const char* why = check_rope_scaling(cfg->tgt_rope_scaling)) return why;
   if (reinterpret_cast<uintptr_t>(cfg->workspace) & 255u) return "workspace must be 256-byte aligned";
@@ -337,6 +338,7 @@ KVX_API kvx_status kvx_r2_probe(const kvx_probe_config* cfg, const kvx_src* src,
   G.Ls = Ls;
   G.Lt = Lt;
   G.rope = tmp.rope;
+  G.hf = cfg->rope_numerics == KVX_ROPE_HF;
   G.sm_count = sms;
   const size_t blk = pl.blk;
   const bool caller_ws = cfg->workspace != nullptr;

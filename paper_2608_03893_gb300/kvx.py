@@ -95,7 +95,7 @@ class kvx_fit_config(ctypes.Structure):
         ("src_rope_theta", ctypes.c_double), ("tgt_rope_theta", ctypes.c_double),
         ("lambda_", ctypes.c_double), ("selection", ctypes.c_void_p),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_uint64),
-    ] + _SCALING
+    ] + _SCALING + [("rope_numerics", ctypes.c_int32)]
 
 
 class kvx_probe_config(ctypes.Structure):
@@ -104,7 +104,7 @@ class kvx_probe_config(ctypes.Structure):
         ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
         ("src_rope_theta", ctypes.c_double), ("tgt_rope_theta", ctypes.c_double),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_uint64),
-    ] + _SCALING
+    ] + _SCALING + [("rope_numerics", ctypes.c_int32)]
 
 
 class kvx_mlp_config(ctypes.Structure):
@@ -379,7 +379,7 @@ def kvx_fit_workspace_bytes(src_layers, tgt_layers, n_kv_heads, head_dim, k, the
 
 def kvx_fit_ridge(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, selection,
                   src, tgt, batch, tokens_per_seq, positions_ptr, W_ptr, b_ptr, stream=0,
-                  workspace_ptr=None, workspace_bytes=0, rope_scaling=None):
+                  workspace_ptr=None, workspace_bytes=0, rope_scaling=None, rope_numerics=0):
     """Ridge fit on calibration caches (see include/kvx.h): src / tgt are kvx_src, selection a
     host int32 [L_t][k] array, W_ptr / b_ptr device fp32 buffers [L_t][2][H][k*d][d] and
     [L_t][2][H][d]; an optional caller workspace (device, 256-byte aligned).  Blocks until
@@ -388,6 +388,7 @@ def kvx_fit_ridge(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, thet
     sel = np.ascontiguousarray(selection, dtype=np.int32)
     cfg = _fit_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, sel, workspace_ptr,
                       workspace_bytes, rope_scaling)
+    cfg.rope_numerics = int(rope_numerics)
     _check(lib().kvx_fit_ridge(ctypes.byref(cfg), ctypes.byref(src), ctypes.byref(tgt), int(batch),
                                int(tokens_per_seq), positions_ptr, W_ptr, b_ptr, stream), "kvx_fit_ridge")
 
@@ -411,7 +412,7 @@ def kvx_r2_probe_workspace_bytes(src_layers, tgt_layers, n_kv_heads, head_dim, t
 
 def kvx_r2_probe(src_layers, tgt_layers, n_kv_heads, head_dim, theta_s, theta_t, src, tgt, batch,
                  tokens_per_seq, positions_ptr, scores_ptr, r2_kv_ptr=None, stream=0,
-                 workspace_ptr=None, workspace_bytes=0, rope_scaling=None):
+                 workspace_ptr=None, workspace_bytes=0, rope_scaling=None, rope_numerics=0):
     """Single-source R^2 probe (see include/kvx.h): src / tgt are kvx_src; scores_ptr a
     device float64 [L_t][L_s] buffer, r2_kv_ptr a device float64 [2][L_t][L_s] buffer or
     None; an optional caller workspace.  Blocks until the probe is done."""
@@ -419,6 +420,7 @@ def kvx_r2_probe(src_layers, tgt_layers, n_kv_heads, head_dim, theta_s, theta_t,
                            float(theta_s), float(theta_t), workspace_ptr, int(workspace_bytes))
     rs = globals()["rope_scaling"](rope_scaling)
     cfg.src_rope_scaling = cfg.tgt_rope_scaling = _scaling_ptr(rs)
+    cfg.rope_numerics = int(rope_numerics)
     _check(lib().kvx_r2_probe(ctypes.byref(cfg), ctypes.byref(src), ctypes.byref(tgt), int(batch),
                               int(tokens_per_seq), positions_ptr, scores_ptr, r2_kv_ptr, stream),
            "kvx_r2_probe")

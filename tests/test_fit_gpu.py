@@ -185,3 +185,45 @@ def test_fit_llama3_rope_scaling():
     systems = [(l, kv, h) for l in range(w.Lt) for kv in range(2) for h in range(w.H)]
     _check_systems_theta(w, rs, rt, 0.01, sel, (sk, sv, tk, tv, pos), W.cpu().double().numpy(),
                          b.cpu().double().numpy(), systems)
+
+
+def test_fit_hf_rope_numerics():
+    """KVX_ROPE_HF on the fit: both sides' keys are stripped with the Hugging Face forward's
+    rounding (oracle.rope.rotate_hf, inverse) before centring; every system of a small case at
+    positions past 2 * 10^4 against the oracle's fit of those features."""
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=4, Lt=3, H=2, B=1, T=512, k=2, theta_t=5e5)
+    sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
+    dev = torch.device("cuda:0")
+    sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+    tk, tv = syn.target_cache(w, 0, device=dev), syn.target_cache(w, 1, device=dev)
+    pos = syn.positions(w) + 20011
+    posd = torch.from_numpy(pos).to(dev)
+    F = w.k * w.d
+    W = torch.full((w.Lt, 2, w.H, F, w.d), float("nan"), dtype=torch.float32, device=dev)
+    b = torch.full((w.Lt, 2, w.H, w.d), float("nan"), dtype=torch.float32, device=dev)
+    kvx.kvx_fit_ridge(w.Ls, w.Lt, w.H, w.d, w.k, w.theta_s, w.theta_t, 0.01, sel, kvx.src_from_tensors(sk, sv),
+                      kvx.src_from_tensors(tk, tv), w.B, w.T, posd.data_ptr(), W.data_ptr(), b.data_ptr(),
+                      torch.cuda.current_stream().cuda_stream, rope_numerics=kvx.KVX_ROPE_HF)
+    Wg, bg = W.cpu().double().numpy(), b.cpu().double().numpy()
+    N = w.B * w.T
+
+    def feats(cache, kv, theta):
+        x = _f64(cache)
+        L, B, H, T, d = x.shape
+        x = x.transpose(0, 2, 1, 3, 4).reshape(L, H, B * T, d)
+        if kv == 0:
+            x = orope.rotate_hf(x, pos.reshape(-1)[None, None, :], theta, inverse=True)
+        return x
+
+    for kv in range(2):
+        xs = feats(sk if kv == 0 else sv, kv, w.theta_s)
+        xt = feats(tk if kv == 0 else tv, kv, w.theta_t)
+        for l in range(w.Lt):
+            for h in range(w.H):
+                X = np.concatenate([xs[s, h] for s in sel[l]], axis=-1)
+                Wr, br = oridge.fit_ridge(X, xt[l, h], 0.01)
+                Xc = X - X.mean(axis=0)
+                kappa = np.linalg.cond(Xc.T @ Xc + 0.01 * np.eye(F))
+                rel = 8.0 * kappa * (N * 2.0 ** -24 + 2.0 ** -16)
+                err = np.max(np.abs(Wg[l, kv, h] - Wr))
+                assert err <= rel * np.max(np.abs(Wr)), (l, kv, h, err, rel * np.max(np.abs(Wr)))
