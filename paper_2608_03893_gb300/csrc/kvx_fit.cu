@@ -228,9 +228,12 @@ __global__ void __launch_bounds__(256, 1) fit_solve_kernel(const __grid_constant
     }
     // 3. forward solve L Y = Z, then backward L^T W = Y, in place on Z, in 32-row blocks:
     //    first the block's 32 x 128 entries take the products with every solved row (thread
-    //    = 4 rows x 4 right-hand-side columns, 16 independent sums), then the 32 x 32
+    //    = 4 rows x 4 right-hand-side columns, 16 independent sums; the solved rows and the
+    //    block's L entries staged through shared memory 32 at a time), then the 32 x 32
     //    triangle is solved row by row (thread = column).
     const int r0 = 4 * (tid & 7), q0 = 4 * (tid >> 3);
+    DF* Ls = fsm;                         // [32][33]: L (forward) or L^T (backward) entries
+    DF* Zs = fsm + kNB * kPS;             // [32][128]: 32 solved rows of Z
     auto load4 = [&](const DF* p, DF (&v)[4]) {
       const float4 x = *reinterpret_cast<const float4*>(p), y = *reinterpret_cast<const float4*>(p + 2);
       v[0] = DF{x.x, x.y};
@@ -238,32 +241,36 @@ __global__ void __launch_bounds__(256, 1) fit_solve_kernel(const __grid_constant
       v[2] = DF{y.x, y.y};
       v[3] = DF{y.z, y.w};
     };
+    // acc[a][c] -= sum_j Ls[r0 + a][j] Zs[j][q0 + c] over the staged chunk (Ls indexed
+    // [row][j] when `rows_major`, else [j][row])
+    auto chunk_update = [&](DF (&acc)[4][4], bool rows_major) {
+#pragma unroll 4
+      for (int j = 0; j < kNB; ++j) {
+        DF z[4], l[4];
+        load4(&Zs[j * kFD + q0], z);
+#pragma unroll
+        for (int a2 = 0; a2 < 4; ++a2) l[a2] = df_neg(rows_major ? Ls[(r0 + a2) * kPS + j] : Ls[j * kPS + r0 + a2]);
+#pragma unroll
+        for (int a2 = 0; a2 < 4; ++a2)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) acc[a2][c] = df_fma(l[a2], z[c], acc[a2][c]);
+      }
+    };
+    auto stage_z = [&](int m0) {
+      for (int e = tid; e < kNB * kFD / 2; e += blockDim.x)   // 32 rows x 128 pairs, two per thread-step
+        reinterpret_cast<float4*>(Zs)[e] = reinterpret_cast<const float4*>(Z + static_cast<size_t>(m0) * kFD)[e];
+    };
     for (int b0 = 0; b0 < F; b0 += kNB) {
       DF acc[4][4];
 #pragma unroll
       for (int a = 0; a < 4; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0], acc[a]);
-      // operands of step m + 1 are loaded while step m computes
-      DF z[4], l[4];
-      if (b0 > 0) {
-        load4(&Z[q0], z);
-#pragma unroll
-        for (int a = 0; a < 4; ++a) l[a] = A[static_cast<size_t>(b0 + r0 + a) * F];
-      }
-      for (int m = 0; m < b0; ++m) {
-        DF zn[4], ln[4];
-        const int mn = m + 1 < b0 ? m + 1 : m;
-        load4(&Z[static_cast<size_t>(mn) * kFD + q0], zn);
-#pragma unroll
-        for (int a = 0; a < 4; ++a) ln[a] = A[static_cast<size_t>(b0 + r0 + a) * F + mn];
-#pragma unroll
-        for (int a = 0; a < 4; ++a)
-#pragma unroll
-          for (int c = 0; c < 4; ++c) acc[a][c] = df_fma(df_neg(l[a]), z[c], acc[a][c]);
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          z[c] = zn[c];
-          l[c] = ln[c];
-        }
+      for (int mc = 0; mc < b0; mc += kNB) {
+        for (int e = tid; e < kNB * kNB; e += blockDim.x)
+          Ls[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(b0 + e / kNB) * F + mc + e % kNB];
+        stage_z(mc);
+        __syncthreads();
+        chunk_update(acc, true);
+        __syncthreads();
       }
 #pragma unroll
       for (int a = 0; a < 4; ++a)
@@ -284,25 +291,13 @@ __global__ void __launch_bounds__(256, 1) fit_solve_kernel(const __grid_constant
       DF acc[4][4];
 #pragma unroll
       for (int a = 0; a < 4; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0], acc[a]);
-      DF z[4], l[4];
-      if (b0 + kNB < F) {
-        load4(&Z[static_cast<size_t>(b0 + kNB) * kFD + q0], z);
-        load4(&A[static_cast<size_t>(b0 + kNB) * F + b0 + r0], l);   // L[m][b0 + r0 ..]: entries of L^T
-      }
-      for (int m = b0 + kNB; m < F; ++m) {
-        DF zn[4], ln[4];
-        const int mn = m + 1 < F ? m + 1 : m;
-        load4(&Z[static_cast<size_t>(mn) * kFD + q0], zn);
-        load4(&A[static_cast<size_t>(mn) * F + b0 + r0], ln);
-#pragma unroll
-        for (int a = 0; a < 4; ++a)
-#pragma unroll
-          for (int c = 0; c < 4; ++c) acc[a][c] = df_fma(df_neg(l[a]), z[c], acc[a][c]);
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          z[c] = zn[c];
-          l[c] = ln[c];
-        }
+      for (int mc = b0 + kNB; mc < F; mc += kNB) {
+        for (int e = tid; e < kNB * kNB; e += blockDim.x)   // L[mc + j][b0 + i]: entries of L^T
+          Ls[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(mc + e / kNB) * F + b0 + e % kNB];
+        stage_z(mc);
+        __syncthreads();
+        chunk_update(acc, false);
+        __syncthreads();
       }
 #pragma unroll
       for (int a = 0; a < 4; ++a)
@@ -578,7 +573,9 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
       set_error(std::string("kvx_fit_ridge: ") + kvx_last_error());
       break;
     }
-    const size_t smem = static_cast<size_t>(kNB) * kPS * 8 + static_cast<size_t>(pl.F - kNB) * kPS * 8;
+    // the factorisation's diagonal block and panel, or the solves' staged chunk
+    const size_t smem = std::max(static_cast<size_t>(kNB) * kPS + static_cast<size_t>(pl.F - kNB) * kPS,
+                                 static_cast<size_t>(kNB) * kPS + static_cast<size_t>(kNB) * kFD) * 8;
     if ((e = cudaFuncSetAttribute(fit_solve_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem))) !=
         cudaSuccess) {
       set_error(std::string("kvx_fit_ridge: smem attribute: ") + cudaGetErrorString(e));
