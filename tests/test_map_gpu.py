@@ -520,6 +520,11 @@ def test_map_host_equals_device_map(name, over, kernel, chunk):
         hpos = torch.from_numpy(np.ascontiguousarray(pos, dtype=np.int32)).pin_memory()
         pipe = kvx.kvx_host_pipe_create(ctx, w.B, chunk)
         s = torch.cuda.current_stream()
+        untouched = torch.full(tk.shape, 3.0, dtype=tk.dtype).pin_memory()
+        kvx.kvx_map_host(pipe, kvx.src_from_tensors(hk, hv), 0, hpos.data_ptr(),
+                         kvx.tgt_from_tensors(untouched, untouched), s.cuda_stream)   # T = 0: no-op
+        s.synchronize()
+        assert torch.all(untouched == 3.0)
         for rep in range(2):
             ok_ = torch.full(tk.shape, float("nan"), dtype=tk.dtype).pin_memory()
             ov_ = torch.full(tv.shape, float("nan"), dtype=tv.dtype).pin_memory()

@@ -208,3 +208,20 @@ def test_mlp_headline_shapes_sampled():
     cases = [(l, kv, h, np.sort(rng.choice(w.T, 48, replace=False))) for (l, kv, h) in
              [(0, 0, 0), (0, 1, 7), (21, 0, 3), (40, 1, 5), (63, 0, 7), (63, 1, 2)]]
     _check(w, 1024, sel, P, src_tok, pos.reshape(-1), (tk, tv), cases)
+
+
+def test_mlp_empty_call_writes_nothing():
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4_xhead", Ls=2, Lt=2, H=2, B=1, T=64, k=1)
+    dev = torch.device("cuda:0")
+    sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
+    sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+    P = _weights(w, 256, 14, dev)
+    tk = torch.full((w.Lt, w.B, w.H, w.T, w.d), 7.0, dtype=torch.bfloat16, device=dev)
+    tv = tk.clone()
+    pos = torch.from_numpy(syn.positions(w)).to(dev)
+    cfg = kvx.mlp_config(w.Ls, w.Lt, w.H, w.d, w.k, 256, w.theta_s, w.theta_t, sel,
+                         *(P[n].data_ptr() for n in ("W1", "b1", "W2", "b2", "W3", "b3")))
+    for (B, T) in [(0, w.T), (w.B, 0)]:
+        kvx.kvx_mlp_map(cfg, kvx.src_from_tensors(sk, sv), B, T, pos.data_ptr(), kvx.tgt_from_tensors(tk, tv),
+                        torch.cuda.current_stream().cuda_stream)
+    assert torch.all(tk == 7.0) and torch.all(tv == 7.0)

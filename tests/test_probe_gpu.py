@@ -224,3 +224,17 @@ def test_probe_caller_workspace():
     with pytest.raises(kvx.KvxError) as e:
         probe(4096)
     assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+
+
+def test_probe_reports_a_singular_source_block():
+    """A constant channel makes a centred source Gram block singular: the probe reports
+    INVALID_ARG instead of returning scores (OLS has no unique fit there)."""
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=3, Lt=2, H=1, B=1, T=300)
+    dev = torch.device("cuda:0")
+    sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+    sv[1, :, :, :, 5] = 0.75                      # value channel 5 of source layer 1: constant
+    tk, tv = syn.target_cache(w, 0, device=dev), syn.target_cache(w, 1, device=dev)
+    with pytest.raises(kvx.KvxError) as e:
+        _run_probe(w, sk, sv, tk, tv, syn.positions(w))
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+    assert "singular" in kvx.lib().kvx_last_error().decode()
