@@ -127,7 +127,10 @@ __device__ __forceinline__ double df_to_double(DF a) { return static_cast<double
 constexpr int kNotSpd = 100;        // internal status: a pivot <= 0 (matrix not positive definite)
 constexpr int kPS = kNB + 1;        // panel row stride in shared memory (pairs)
 
-__global__ void __launch_bounds__(256, 1) fit_solve_kernel(const __grid_constant__ FitParams P) {
+constexpr int kSolveThreads = 512;                 // 16 warps: enough to keep the FP32 lanes busy
+constexpr int kSolveWarps = kSolveThreads / 32;
+
+__global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __grid_constant__ FitParams P) {
   extern __shared__ __align__(16) DF fsm[];
   DF* D = fsm;                                    // [32][33]
   DF* Pn = fsm + kNB * kPS;                       // [F - 32][33]: rows padded so a warp's 32 rows hit distinct banks
@@ -207,31 +210,35 @@ __global__ void __launch_bounds__(256, 1) fit_solve_kernel(const __grid_constant
         int ti = 0;
         while ((ti + 1) * (ti + 2) / 2 <= tile) ++ti;
         const int tj = tile - ti * (ti + 1) / 2;
-        // thread: column jj (lane: the warp's stores are contiguous) and rows ii + 8q (warp w:
-        // ii = w), q < 4; the lane's panel row is read conflict-free (odd row stride), the
-        // warp's four rows are broadcasts
+        // thread: column jj (lane: the warp's stores are contiguous) and rows ii + 16q (warp w:
+        // ii = w), q < 2; the lane's panel row is read conflict-free (odd row stride), the
+        // warp's rows are broadcasts
+        constexpr int kRowsPer = kNB / kSolveWarps;
         const int jj = tj * kNB + (tid & 31), ii = ti * kNB + (tid >> 5);
-        DF sacc[4] = {df_make(0.f), df_make(0.f), df_make(0.f), df_make(0.f)};
+        DF sacc[kRowsPer];
+#pragma unroll
+        for (int q = 0; q < kRowsPer; ++q) sacc[q] = df_make(0.f);
 #pragma unroll 8
         for (int m = 0; m < kNB; ++m) {
           const DF pj = Pn[jj * kPS + m];
 #pragma unroll
-          for (int q = 0; q < 4; ++q) sacc[q] = df_fma(Pn[(ii + 8 * q) * kPS + m], pj, sacc[q]);
+          for (int q = 0; q < kRowsPer; ++q) sacc[q] = df_fma(Pn[(ii + kSolveWarps * q) * kPS + m], pj, sacc[q]);
         }
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          DF* a = A + static_cast<size_t>(c0 + kNB + ii + 8 * q) * F + c0 + kNB + jj;
-          if (jj <= ii + 8 * q) *a = df_add(*a, df_neg(sacc[q]));
+        for (int q = 0; q < kRowsPer; ++q) {
+          DF* a = A + static_cast<size_t>(c0 + kNB + ii + kSolveWarps * q) * F + c0 + kNB + jj;
+          if (jj <= ii + kSolveWarps * q) *a = df_add(*a, df_neg(sacc[q]));
         }
       }
       __syncthreads();
     }
     // 3. forward solve L Y = Z, then backward L^T W = Y, in place on Z, in 32-row blocks:
     //    first the block's 32 x 128 entries take the products with every solved row (thread
-    //    = 4 rows x 4 right-hand-side columns, 16 independent sums; the solved rows and the
+    //    = 2 rows x 4 right-hand-side columns, 8 independent sums; the solved rows and the
     //    block's L entries staged through shared memory 32 at a time), then the 32 x 32
     //    triangle is solved row by row (thread = column).
-    const int r0 = 4 * (tid & 7), q0 = 4 * (tid >> 3);
+    constexpr int kR = kNB * kFD / 4 / kSolveThreads;   // rows per thread (2)
+    const int r0 = kR * (tid % (kNB / kR)), q0 = 4 * (tid / (kNB / kR));
     DF* Ls = fsm;                         // [32][33]: L (forward) or L^T (backward) entries
     DF* Zs = fsm + kNB * kPS;             // [32][128]: 32 solved rows of Z
     auto load4 = [&](const DF* p, DF (&v)[4]) {
@@ -243,15 +250,15 @@ __global__ void __launch_bounds__(256, 1) fit_solve_kernel(const __grid_constant
     };
     // acc[a][c] -= sum_j Ls[r0 + a][j] Zs[j][q0 + c] over the staged chunk (Ls indexed
     // [row][j] when `rows_major`, else [j][row])
-    auto chunk_update = [&](DF (&acc)[4][4], bool rows_major) {
+    auto chunk_update = [&](DF (&acc)[kR][4], bool rows_major) {
 #pragma unroll 4
       for (int j = 0; j < kNB; ++j) {
-        DF z[4], l[4];
+        DF z[4], l[kR];
         load4(&Zs[j * kFD + q0], z);
 #pragma unroll
-        for (int a2 = 0; a2 < 4; ++a2) l[a2] = df_neg(rows_major ? Ls[(r0 + a2) * kPS + j] : Ls[j * kPS + r0 + a2]);
+        for (int a2 = 0; a2 < kR; ++a2) l[a2] = df_neg(rows_major ? Ls[(r0 + a2) * kPS + j] : Ls[j * kPS + r0 + a2]);
 #pragma unroll
-        for (int a2 = 0; a2 < 4; ++a2)
+        for (int a2 = 0; a2 < kR; ++a2)
 #pragma unroll
           for (int c = 0; c < 4; ++c) acc[a2][c] = df_fma(l[a2], z[c], acc[a2][c]);
       }
@@ -261,9 +268,9 @@ __global__ void __launch_bounds__(256, 1) fit_solve_kernel(const __grid_constant
         reinterpret_cast<float4*>(Zs)[e] = reinterpret_cast<const float4*>(Z + static_cast<size_t>(m0) * kFD)[e];
     };
     for (int b0 = 0; b0 < F; b0 += kNB) {
-      DF acc[4][4];
+      DF acc[kR][4];
 #pragma unroll
-      for (int a = 0; a < 4; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0], acc[a]);
+      for (int a = 0; a < kR; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0], acc[a]);
       for (int mc = 0; mc < b0; mc += kNB) {
         for (int e = tid; e < kNB * kNB; e += blockDim.x)
           Ls[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(b0 + e / kNB) * F + mc + e % kNB];
@@ -273,7 +280,7 @@ __global__ void __launch_bounds__(256, 1) fit_solve_kernel(const __grid_constant
         __syncthreads();
       }
 #pragma unroll
-      for (int a = 0; a < 4; ++a)
+      for (int a = 0; a < kR; ++a)
 #pragma unroll
         for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0 + c] = acc[a][c];
       __syncthreads();
@@ -288,9 +295,9 @@ __global__ void __launch_bounds__(256, 1) fit_solve_kernel(const __grid_constant
       __syncthreads();
     }
     for (int b0 = F - kNB; b0 >= 0; b0 -= kNB) {
-      DF acc[4][4];
+      DF acc[kR][4];
 #pragma unroll
-      for (int a = 0; a < 4; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0], acc[a]);
+      for (int a = 0; a < kR; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0], acc[a]);
       for (int mc = b0 + kNB; mc < F; mc += kNB) {
         for (int e = tid; e < kNB * kNB; e += blockDim.x)   // L[mc + j][b0 + i]: entries of L^T
           Ls[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(mc + e / kNB) * F + b0 + e % kNB];
@@ -300,7 +307,7 @@ __global__ void __launch_bounds__(256, 1) fit_solve_kernel(const __grid_constant
         __syncthreads();
       }
 #pragma unroll
-      for (int a = 0; a < 4; ++a)
+      for (int a = 0; a < kR; ++a)
 #pragma unroll
         for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0 + c] = acc[a][c];
       __syncthreads();
@@ -583,7 +590,7 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
       break;
     }
     timer.begin(3);
-    fit_solve_kernel<<<pl.solve_grid, 256, smem, st>>>(P);
+    fit_solve_kernel<<<pl.solve_grid, kSolveThreads, smem, st>>>(P);
     timer.end();
     if ((e = cudaGetLastError()) != cudaSuccess) {
       set_error(std::string("kvx_fit_ridge: launch: ") + cudaGetErrorString(e));
