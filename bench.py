@@ -16,7 +16,7 @@ source layers per target layer.  A step is one kvx_map call over the whole workl
   against MEASURED_PEAKS.json; traffic from the committed ncu summary when it was taken
   on the current kernel source.
 * cpu_baseline: the float64 oracle on a bounded sample of the same workload's tokens.
-* --impl reference: the oracle as the reference arm (see DESIGN.md).
+* --impl reference: the oracle as the reference arm.
 
 Multi-GPU (torchrun): every rank maps its own replica (weak scaling, no collective on
 the data path; a MAX all-reduce of the elapsed time only).

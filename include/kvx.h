@@ -48,7 +48,7 @@ typedef struct kvx_ctx kvx_ctx;
 typedef enum {
   KVX_OK = 0,
   KVX_ERR_INVALID_ARG = 1,   /* a bad argument, detected on the host; nothing launched */
-  KVX_ERR_UNSUPPORTED = 2,   /* valid request that this build cannot run (e.g. shape) */
+  KVX_ERR_UNSUPPORTED = 2,   /* valid request that the library cannot run (e.g. shape) */
   KVX_ERR_OOM = 3,           /* cudaMalloc failed in kvx_create */
   KVX_ERR_CUDA = 4,          /* a CUDA runtime or launch error */
   KVX_ERR_TIMEOUT = 5,       /* device: a bounded wait in a kernel ran out */
