@@ -339,6 +339,7 @@ typedef struct {
   uint64_t workspace_bytes;
   const kvx_rope_scaling* src_rope_scaling;   /* NULL: plain theta (see kvx_rope_scaling) */
   const kvx_rope_scaling* tgt_rope_scaling;
+  int32_t rope_numerics;        /* kvx_rope_numerics: source strip and target rotation of keys */
 } kvx_mlp_config;
 KVX_API kvx_status kvx_mlp_map(const kvx_mlp_config* cfg, const kvx_src* src, int32_t batch, int32_t tokens_per_seq,
                                const int32_t* positions, const kvx_tgt* tgt, void* stream);

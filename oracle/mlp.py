@@ -39,14 +39,17 @@ def mlp_forward(X, W1, b1, W2, b2, W3, b3, round_hidden=False):
     return h @ np.asarray(W3, dtype=np.float64).T + np.asarray(b3, dtype=np.float64)
 
 
-def cross_head_features(src, l, sel, kv, positions, theta_s, mode="exact"):
+def cross_head_features(src, l, sel, kv, positions, theta_s, mode="exact", rope_numerics="exact"):
     """Source feature of target layer l: src [L_s][H][N][d] (one of K / V), the k layers
     sel[l] in order, each with all H heads (head-minor): [N][k H d].  Keys are stripped
-    (and rounded to bf16 in ``"bf16fwd"`` mode)."""
+    (and rounded to bf16 in ``"bf16fwd"`` mode; ``rope_numerics="hf"``: the Hugging Face
+    forward's strip, rope.rotate_hf)."""
     parts = []
     for j in sel[l]:
         x = np.asarray(src[j], dtype=np.float64)            # [H][N][d]
-        if kv == 0:
+        if kv == 0 and rope_numerics == "hf":
+            x = rope.rotate_hf(x, np.asarray(positions)[None, :], theta_s, inverse=True)
+        elif kv == 0:
             x = rope.rotate(x, np.asarray(positions)[None, :], theta_s, inverse=True)
             if mode == "bf16fwd":
                 x = bf16.round_to_bf16_value(x)
@@ -54,7 +57,7 @@ def cross_head_features(src, l, sel, kv, positions, theta_s, mode="exact"):
     return np.concatenate(parts, axis=-1)
 
 
-def map_tokens_mlp(src_k, src_v, positions, sel, params, theta_s, theta_t, mode="exact"):
+def map_tokens_mlp(src_k, src_v, positions, sel, params, theta_s, theta_t, mode="exact", rope_numerics="exact"):
     """src_k / src_v [L_s][H][N][d], positions [N], sel [L_t][k];
     params: W1 [L_t][2][H][hidden][k H d], b1 [L_t][2][H][hidden], W2 [L_t][2][H][hidden][hidden],
     b2 [L_t][2][H][hidden], W3 [L_t][2][H][d][hidden], b3 [L_t][2][H][d].
@@ -66,12 +69,14 @@ def map_tokens_mlp(src_k, src_v, positions, sel, params, theta_s, theta_t, mode=
     for kv, src in enumerate((src_k, src_v)):
         out = []
         for l in range(Lt):
-            X = cross_head_features(src, l, sel, kv, positions, theta_s, mode)
+            X = cross_head_features(src, l, sel, kv, positions, theta_s, mode, rope_numerics)
             heads = []
             for h in range(H):
                 y = mlp_forward(X, W1[l][kv][h], b1[l][kv][h], W2[l][kv][h], b2[l][kv][h], W3[l][kv][h],
                                 b3[l][kv][h], round_hidden=(mode == "bf16fwd"))
-                if kv == 0:
+                if kv == 0 and rope_numerics == "hf":
+                    y = rope.rotate_hf(y, np.asarray(positions), theta_t)
+                elif kv == 0:
                     y = rope.rotate(y, np.asarray(positions), theta_t)
                 heads.append(y)
             out.append(np.stack(heads))

@@ -67,7 +67,7 @@ struct MlpParams {
   MapArgs a;               // positions, targets (pass 3), B, T
   const int32_t* sel;      // [L_t][k]
   int32_t* status;
-  int32_t pass, l0, H, k, hidden, pairs, n_units, n_tiles, heads, ksteps, G;
+  int32_t pass, l0, H, k, hidden, pairs, n_units, n_tiles, heads, ksteps, G, hf;
   RopeTables rope;
 };
 
@@ -302,7 +302,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kMThreads, 1)
             p = 0;
           }
         }
-        if (un.kv == 0) {
+        if (un.kv == 0 && P.hf) {   // HF numerics: cos / sin of the fp32 angle, rounded to bf16
+#pragma unroll
+          for (int m = 0; m < 32; ++m) {
+            sincosf(__fmul_rn(static_cast<float>(p), P.rope.wt_hi[32 * g + m]), &sn[m], &cs[m]);
+            sn[m] = __bfloat162float(__float2bfloat16_rn(sn[m]));
+            cs[m] = __bfloat162float(__float2bfloat16_rn(cs[m]));
+          }
+        } else if (un.kv == 0) {
 #pragma unroll
           for (int m = 0; m < 32; ++m)
             rope_sincos(p, P.rope.wt_hi[32 * g + m], P.rope.wt_lo[32 * g + m], P.rope.two_pi_hi, P.rope.two_pi_lo,
@@ -337,7 +344,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kMThreads, 1)
             yhi[j + 2] = __fadd_rn(__uint_as_float(hi[j + 2]), b1.z);
             yhi[j + 3] = __fadd_rn(__uint_as_float(hi[j + 3]), b1.w);
           }
-          if (un.kv == 0) {   // y0' = y0 c - y1 s, y1' = y0 s + y1 c
+          if (un.kv == 0 && P.hf) {   // the key as a bf16 tensor, each product and sum rounded
+            auto r = [](float x) { return __bfloat162float(__float2bfloat16_rn(x)); };
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const float c = cs[16 * rnd + j], s = sn[16 * rnd + j];
+              const float y0 = r(ylo[j]), y1 = r(yhi[j]);
+              ylo[j] = r(__fsub_rn(r(__fmul_rn(y0, c)), r(__fmul_rn(y1, s))));
+              yhi[j] = r(__fadd_rn(r(__fmul_rn(y1, c)), r(__fmul_rn(y0, s))));
+            }
+          } else if (un.kv == 0) {   // y0' = y0 c - y1 s, y1' = y0 s + y1 c
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
               const float c = cs[16 * rnd + j], s = sn[16 * rnd + j];
@@ -401,6 +417,7 @@ const char* check_mlp_config(const kvx_mlp_config* c) {
   if (static_cast<int64_t>(c->tgt_layers) * 2 * c->n_kv_heads * c->hidden > INT_MAX / 2) return "too many weight rows";
   if (static_cast<int64_t>(c->k) * c->n_kv_heads * kMD > INT_MAX / 2) return "source feature too wide";
   if (c->workspace_bytes != 0 && !c->workspace) return "workspace_bytes without a workspace";
+  if (c->rope_numerics != KVX_ROPE_EXACT && c->rope_numerics != KVX_ROPE_HF) return "bad rope_numerics";
   if (const char* why = check_rope_scaling(c->src_rope_scaling)) return why;
   if (const char* why = check_rope_scaling(c->tgt_rope_scaling)) return why;
   if (reinterpret_cast<uintptr_t>(c->workspace) & 255u) return "workspace must be 256-byte aligned";
@@ -608,7 +625,9 @@ KVX_API kvx_status kvx_mlp_map(const kvx_mlp_config* cfg, const kvx_src* src, in
     P.pairs = (tokens_per_seq + 2 * kMTile - 1) / (2 * kMTile);
     P.rope = tmp.rope;
     // strip every source key once
-    launch_key_strip(src->k, src->stride, d_strip, positions, cfg->src_layers, H, batch, tokens_per_seq, tmp.rope, sms, st);
+    P.hf = cfg->rope_numerics == KVX_ROPE_HF;
+    launch_key_strip(src->k, src->stride, d_strip, positions, cfg->src_layers, H, batch, tokens_per_seq, tmp.rope, sms, st,
+                     P.hf);
     const size_t smem = mlp_smem_bytes();
     if ((e = cudaFuncSetAttribute(tc_mlp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   static_cast<int>(smem))) != cudaSuccess) {

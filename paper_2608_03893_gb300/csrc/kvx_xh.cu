@@ -114,7 +114,7 @@ __device__ __forceinline__ void xreport(int32_t* status, int code) { atomicCAS(s
 __global__ void __launch_bounds__(256) xh_strip_kernel(const __nv_bfloat16* __restrict__ src, int64_t s_l,
                                                        int64_t s_b, int64_t s_h, int64_t s_t,
                                                        __nv_bfloat16* __restrict__ ws, const int32_t* __restrict__ pos,
-                                                       int Ls, int H, int B, int T, RopeTables rope) {
+                                                       int Ls, int H, int B, int T, RopeTables rope, int hf) {
   const int64_t n = static_cast<int64_t>(B) * T * 16;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -125,9 +125,16 @@ __global__ void __launch_bounds__(256) xh_strip_kernel(const __nv_bfloat16* __re
     if (p < 0 || p >= (1 << 24)) p = 0;   // the mapping kernel reports the position
     float c[4], s[4];
 #pragma unroll
-    for (int m = 0; m < 4; ++m)
-      rope_sincos(p, rope.ws_hi[4 * grp + m], rope.ws_lo[4 * grp + m], rope.two_pi_hi, rope.two_pi_lo,
-                  rope.inv_two_pi, &s[m], &c[m]);
+    for (int m = 0; m < 4; ++m) {
+      if (hf) {   // HF numerics: cos / sin of the fp32 angle, rounded to bf16
+        sincosf(__fmul_rn(static_cast<float>(p), rope.ws_hi[4 * grp + m]), &s[m], &c[m]);
+        s[m] = __bfloat162float(__float2bfloat16_rn(s[m]));
+        c[m] = __bfloat162float(__float2bfloat16_rn(c[m]));
+      } else {
+        rope_sincos(p, rope.ws_hi[4 * grp + m], rope.ws_lo[4 * grp + m], rope.two_pi_hi, rope.two_pi_lo,
+                    rope.inv_two_pi, &s[m], &c[m]);
+      }
+    }
     for (int L = 0; L < Ls; ++L) {
       for (int h = 0; h < H; ++h) {
         const __nv_bfloat16* row = src + L * s_l + b * s_b + h * s_h + static_cast<int64_t>(t) * s_t;
@@ -140,9 +147,17 @@ __global__ void __launch_bounds__(256) xh_strip_kernel(const __nv_bfloat16* __re
           const float a0 = bf16_lo(wa[w]), a1 = bf16_hi(wa[w]);
           const float b0 = bf16_lo(wb[w]), b1 = bf16_hi(wb[w]);
           const int m0 = 2 * w, m1 = 2 * w + 1;
-          // rotation by -t*omega: a' = a c + b s, b' = b c - a s
-          oa[w] = pack_bf16x2(__fmaf_rn(a0, c[m0], __fmul_rn(b0, s[m0])), __fmaf_rn(a1, c[m1], __fmul_rn(b1, s[m1])));
-          ob[w] = pack_bf16x2(__fmaf_rn(b0, c[m0], -__fmul_rn(a0, s[m0])), __fmaf_rn(b1, c[m1], -__fmul_rn(a1, s[m1])));
+          if (hf) {   // each product and sum rounded to bf16
+            auto r = [](float x) { return __bfloat162float(__float2bfloat16_rn(x)); };
+            oa[w] = pack_bf16x2(r(__fadd_rn(r(__fmul_rn(a0, c[m0])), r(__fmul_rn(b0, s[m0])))),
+                                r(__fadd_rn(r(__fmul_rn(a1, c[m1])), r(__fmul_rn(b1, s[m1])))));
+            ob[w] = pack_bf16x2(r(__fsub_rn(r(__fmul_rn(b0, c[m0])), r(__fmul_rn(a0, s[m0])))),
+                                r(__fsub_rn(r(__fmul_rn(b1, c[m1])), r(__fmul_rn(a1, s[m1])))));
+          } else {
+            // rotation by -t*omega: a' = a c + b s, b' = b c - a s
+            oa[w] = pack_bf16x2(__fmaf_rn(a0, c[m0], __fmul_rn(b0, s[m0])), __fmaf_rn(a1, c[m1], __fmul_rn(b1, s[m1])));
+            ob[w] = pack_bf16x2(__fmaf_rn(b0, c[m0], -__fmul_rn(a0, s[m0])), __fmaf_rn(b1, c[m1], -__fmul_rn(a1, s[m1])));
+          }
         }
         __nv_bfloat16* out = ws + ((((static_cast<int64_t>(L) * B + b) * H + h) * T + t) * kXD);
         *reinterpret_cast<uint2*>(out + 4 * grp) = make_uint2(oa[0], oa[1]);
@@ -536,11 +551,11 @@ kvx_status repack_wt_hilo(kvx_ctx* c, const void* W_host) {
 }
 
 void launch_key_strip(const void* src_k, const int64_t* ss, void* ws, const int32_t* pos, int Ls, int H, int B, int T,
-                      const RopeTables& rope, int sms, cudaStream_t stream) {
+                      const RopeTables& rope, int sms, cudaStream_t stream, int hf) {
   const int64_t threads = static_cast<int64_t>(B) * T * 16;
   const int blocks = static_cast<int>(std::min<int64_t>((threads + 255) / 256, static_cast<int64_t>(sms) * 8));
   xh_strip_kernel<<<blocks, 256, 0, stream>>>(static_cast<const __nv_bfloat16*>(src_k), ss[0], ss[1], ss[2], ss[3],
-                                              static_cast<__nv_bfloat16*>(ws), pos, Ls, H, B, T, rope);
+                                              static_cast<__nv_bfloat16*>(ws), pos, Ls, H, B, T, rope, hf);
 }
 
 bool xh_supported(const kvx_ctx* c, std::string* why) {
@@ -664,7 +679,7 @@ kvx_status launch_xh(kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
 
   // 1. strip the source RoPE from every key into the workspace
   {
-    launch_key_strip(a.src_k, a.ss, c->d_ws, a.pos, c->Ls, c->H, a.B, a.T, c->rope, c->sm_count, stream);
+    launch_key_strip(a.src_k, a.ss, c->d_ws, a.pos, c->Ls, c->H, a.B, a.T, c->rope, c->sm_count, stream, 0);
     if ((e = cudaGetLastError()) != cudaSuccess) {
       set_error(std::string("kvx_map: strip launch: ") + cudaGetErrorString(e));
       return KVX_ERR_CUDA;

@@ -6,9 +6,10 @@
 namespace kvx {
 
 // Source keys with the source RoPE stripped and rounded to bf16, written contiguously as
-// [L_s][B][H][T][128] into `ws`; `ss` the source strides (layer, batch, head, token).
+// [L_s][B][H][T][128] into `ws`; `ss` the source strides (layer, batch, head, token);
+// `hf`: the Hugging Face forward's rounding (kvx_rope_numerics).
 void launch_key_strip(const void* src_k, const int64_t* ss, void* ws, const int32_t* pos, int Ls, int H, int B, int T,
-                      const RopeTables& rope, int sms, cudaStream_t stream);
+                      const RopeTables& rope, int sms, cudaStream_t stream, int hf);
 
 // fp32 W [L_t][2][H][F][128] -> W^T bf16 [L_t][2][H][128][2F] = [W_hi | W_lo] in ctx->d_Wt,
 // for the cross-head tensor-core kernel with fp32 weights.

@@ -117,7 +117,7 @@ class kvx_mlp_config(ctypes.Structure):
         ("W1", ctypes.c_void_p), ("b1", ctypes.c_void_p), ("W2", ctypes.c_void_p), ("b2", ctypes.c_void_p),
         ("W3", ctypes.c_void_p), ("b3", ctypes.c_void_p),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_uint64),
-    ] + _SCALING
+    ] + _SCALING + [("rope_numerics", ctypes.c_int32)]
 
 
 _lib = None
@@ -435,7 +435,7 @@ def kvx_select_topk_device(scores_ptr, tgt_layers, src_layers, k, out_ptr, strea
 
 def mlp_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, hidden, theta_s, theta_t, selection,
                W1_ptr, b1_ptr, W2_ptr, b2_ptr, W3_ptr, b3_ptr, workspace_ptr=None, workspace_bytes=0,
-               rope_scaling=None):
+               rope_scaling=None, rope_numerics=0):
     """kvx_mlp_config for kvx_mlp_map (weights and biases DEVICE pointers, see include/kvx.h).
     The returned config keeps the host selection array alive."""
     import numpy as np
@@ -447,6 +447,7 @@ def mlp_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, hidden, theta_s,
     rs = globals()["rope_scaling"](rope_scaling)
     cfg.src_rope_scaling = cfg.tgt_rope_scaling = _scaling_ptr(rs)
     cfg._rs = rs
+    cfg.rope_numerics = int(rope_numerics)
     return cfg
 
 
