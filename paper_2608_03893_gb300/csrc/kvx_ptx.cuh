@@ -363,5 +363,12 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
+// x rounded to the nearest bf16 (ties to even), as a float
+__device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+__device__ __forceinline__ float2 bf16_round2(float2 v) {
+  const uint32_t w = pack_bf16x2(v.x, v.y);
+  return make_float2(bf16_lo(w), bf16_hi(w));
+}
+
 }  // namespace ptx
 }  // namespace kvx

@@ -165,6 +165,9 @@ __device__ __forceinline__ void report(int32_t* status, int code) { atomicCAS(st
 
 // ------------------------------------------------------------------------ kernel --
 
+// kHF: the Hugging Face forward's RoPE rounding (kvx_rope_numerics): cos / sin of the fp32
+// angle rounded to bf16, every product and sum of the rotations rounded to bf16.
+template <bool kHF>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     tc_map_kernel(const __grid_constant__ TcParams P) {
   extern __shared__ __align__(1024) uint8_t smem[];
@@ -532,8 +535,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int m = 0; m < 32; ++m) {
           const int i = 32 * g + m;
-          rope_sincos(p, P.rope.wt_hi[i], P.rope.wt_lo[i], P.rope.two_pi_hi, P.rope.two_pi_lo, P.rope.inv_two_pi,
-                      &sn[m], &cs[m]);
+          if constexpr (kHF) {
+            sincosf(__fmul_rn(static_cast<float>(p), P.rope.wt_hi[i]), &sn[m], &cs[m]);
+            sn[m] = bf16_round(sn[m]);
+            cs[m] = bf16_round(cs[m]);
+          } else {
+            rope_sincos(p, P.rope.wt_hi[i], P.rope.wt_lo[i], P.rope.two_pi_hi, P.rope.two_pi_lo, P.rope.inv_two_pi,
+                        &sn[m], &cs[m]);
+          }
         }
       }
       __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(un.kv ? A.tgt_v : A.tgt_k);
@@ -602,9 +611,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
               const float2 c = make_float2(cs[16 * rnd + j], cs[16 * rnd + j + 1]);
               const float2 sv = make_float2(sn[16 * rnd + j], sn[16 * rnd + j + 1]);
               const float2 y0 = make_float2(ylo[j], ylo[j + 1]), y1 = make_float2(yhi[j], yhi[j + 1]);
-              const float2 u = __fmul2_rn(y1, sv);
-              const float2 r0 = __ffma2_rn(y0, c, make_float2(-u.x, -u.y));
-              const float2 r1 = __ffma2_rn(y0, sv, __fmul2_rn(y1, c));
+              float2 r0, r1;
+              if constexpr (kHF) {   // the key as bf16, products and sums rounded to bf16
+                const float2 b0 = bf16_round2(y0), b1 = bf16_round2(y1);
+                const float2 p0 = bf16_round2(__fmul2_rn(b0, c)), p1 = bf16_round2(__fmul2_rn(b1, sv));
+                const float2 p2 = bf16_round2(__fmul2_rn(b1, c)), p3 = bf16_round2(__fmul2_rn(b0, sv));
+                r0 = make_float2(__fsub_rn(p0.x, p1.x), __fsub_rn(p0.y, p1.y));
+                r1 = make_float2(__fadd_rn(p2.x, p3.x), __fadd_rn(p2.y, p3.y));
+              } else {
+                const float2 u = __fmul2_rn(y1, sv);
+                r0 = __ffma2_rn(y0, c, make_float2(-u.x, -u.y));
+                r1 = __ffma2_rn(y0, sv, __fmul2_rn(y1, c));
+              }
               ylo[j] = r0.x;
               ylo[j + 1] = r0.y;
               yhi[j] = r1.x;
@@ -681,9 +699,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         int p = t < A.T ? __ldg(&A.pos[static_cast<int64_t>(un.b) * A.T + t]) : 0;
         if (p < 0 || p >= (1 << 24)) p = 0;
 #pragma unroll
-        for (int i = 0; i < 64; ++i)
-          rope_sincos(p, P.rope.ws_hi[i], P.rope.ws_lo[i], P.rope.two_pi_hi, P.rope.two_pi_lo, P.rope.inv_two_pi,
-                      &sn[i], &cs[i]);
+        for (int i = 0; i < 64; ++i) {
+          if constexpr (kHF) {
+            sincosf(__fmul_rn(static_cast<float>(p), P.rope.ws_hi[i]), &sn[i], &cs[i]);
+            sn[i] = bf16_round(sn[i]);
+            cs[i] = bf16_round(cs[i]);
+          } else {
+            rope_sincos(p, P.rope.ws_hi[i], P.rope.ws_lo[i], P.rope.two_pi_hi, P.rope.two_pi_lo, P.rope.inv_two_pi,
+                        &sn[i], &cs[i]);
+          }
+        }
       }
       for (int e = 0; ok && e < P.n_loads; ++e) {
         // load word: slot | 4 << i if issuer i used the slot's previous tile (wait for its
@@ -736,11 +761,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
               const float2 cc = make_float2(cs[m0], cs[m1]), ss = make_float2(sn[m0], sn[m1]);
               // rotation by -t*omega: a' = a c + b s, b' = b c - a s, two pairs per f32x2
               // instruction (each lane rounds like the scalar fmul / fma)
-              const float2 as = __fmul2_rn(a, ss);
-              const float2 ra = __ffma2_rn(a, cc, __fmul2_rn(b, ss));
-              const float2 rb = __ffma2_rn(b, cc, make_float2(-as.x, -as.y));
-              wa[w] = pack_bf16x2(ra.x, ra.y);
-              wb[w] = pack_bf16x2(rb.x, rb.y);
+              if constexpr (kHF) {   // products rounded to bf16, then the sums (by the pack)
+                const float2 ac = bf16_round2(__fmul2_rn(a, cc)), bs = bf16_round2(__fmul2_rn(b, ss));
+                const float2 bc = bf16_round2(__fmul2_rn(b, cc)), as = bf16_round2(__fmul2_rn(a, ss));
+                wa[w] = pack_bf16x2(__fadd_rn(ac.x, bs.x), __fadd_rn(ac.y, bs.y));
+                wb[w] = pack_bf16x2(__fsub_rn(bc.x, as.x), __fsub_rn(bc.y, as.y));
+              } else {
+                const float2 as = __fmul2_rn(a, ss);
+                const float2 ra = __ffma2_rn(a, cc, __fmul2_rn(b, ss));
+                const float2 rb = __ffma2_rn(b, cc, make_float2(-as.x, -as.y));
+                wa[w] = pack_bf16x2(ra.x, ra.y);
+                wb[w] = pack_bf16x2(rb.x, rb.y);
+              }
             }
           }
           tmem_st_x8(scol + 8 * c, wa);        // TMEM columns 8c .. 8c+7
@@ -1026,8 +1058,8 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   P.n_units = static_cast<int>(units);
   P.rope = c->rope;
   const size_t smem = smem_bytes();
-  cudaError_t e = cudaFuncSetAttribute(tc_map_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
+  void (*kernel)(TcParams) = c->rope_numerics == KVX_ROPE_HF ? tc_map_kernel<true> : tc_map_kernel<false>;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) {
     set_error(std::string("kvx_map: smem attribute: ") + cudaGetErrorString(e));
     return KVX_ERR_CUDA;
@@ -1035,7 +1067,7 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   // The warpgroups' register shares (setmaxnreg) are drawn from what the launch holds: a
   // build that launched with fewer registers per thread would leave an increase waiting.
   cudaFuncAttributes fa;
-  e = cudaFuncGetAttributes(&fa, tc_map_kernel);
+  e = cudaFuncGetAttributes(&fa, kernel);
   if (e != cudaSuccess) {
     set_error(std::string("kvx_map: kernel attributes: ") + cudaGetErrorString(e));
     return KVX_ERR_CUDA;
@@ -1046,7 +1078,7 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
     return KVX_ERR_UNSUPPORTED;
   }
   const int grid = 2 * static_cast<int>(std::min<int64_t>(units, std::max(c->sm_count / 2, 1)));   // CTA pairs
-  tc_map_kernel<<<grid, kThreads, smem, stream>>>(P);
+  kernel<<<grid, kThreads, smem, stream>>>(P);
   e = cudaGetLastError();
   if (e != cudaSuccess) {
     set_error(std::string("kvx_map: tensor-core launch: ") + cudaGetErrorString(e));

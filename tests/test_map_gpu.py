@@ -575,13 +575,15 @@ def test_cross_head_tc_fp32_weights_hi_lo():
 
 # ---------------------------------------------------------------- HF RoPE numerics -----
 
-def test_hf_rope_numerics_simt():
+@pytest.mark.parametrize("kname", ["simt", "tc"])
+def test_hf_rope_numerics(kname):
     """KVX_ROPE_HF (the rounding of the Hugging Face bf16 forward: fp32 angle, bf16 cos/sin,
-    each product and sum rounded) on the SIMT kernel against the oracle in the same numerics,
-    at positions past 2 * 10^4 where the fp32 angle is coarse: every output within the
-    usual bound, at least 90 % of the keys bit-equal to the oracle's (the rest follow a
-    rounding of the fp32-accumulated contraction or of cos / sin near a bf16 midpoint), far
-    more than agree with the exact-RoPE oracle.  The tensor-core kernels refuse the mode."""
+    each product and sum rounded) on the SIMT and the per-head tensor-core kernels against
+    the oracle in the same numerics, at positions past 2 * 10^4 where the fp32 angle is
+    coarse: every output within the bound, at least 90 % of the keys bit-equal to the
+    oracle's (the rest follow a rounding of the fp32-accumulated contraction or of cos / sin
+    near a bf16 midpoint), far more than agree with the exact-RoPE oracle.  The cross-head
+    tensor-core kernel refuses the mode."""
     w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=5, Lt=4, H=2, B=2, T=200, k=2, theta_t=5e5)
     W, b = syn.weights(w)
     scores = syn.selection_scores(w)
@@ -590,9 +592,7 @@ def test_hf_rope_numerics_simt():
         theta_t=w.theta_t, cache_dtype=w.cache_dtype, W=W, b=b, scores=scores, rope_numerics=kvx.KVX_ROPE_HF)
     ctx = kvx.kvx_create(cfg, 0)
     try:
-        with pytest.raises(kvx.KvxError) as e:
-            kvx.kvx_set_kernel(ctx, kvx.KVX_KERNEL_TCGEN05)
-        assert e.value.status == kvx.KVX_ERR_UNSUPPORTED
+        kvx.kvx_set_kernel(ctx, KERNELS[kname])
         sel = kvx.kvx_get_selection(ctx, w.Lt, w.k)
         dev = torch.device("cuda:0")
         sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
@@ -617,5 +617,21 @@ def test_hf_rope_numerics_simt():
         same_hf = np.mean(gk == rk)
         same_exact = np.mean(gk == obf16.round_to_bf16_value(ek))
         assert same_hf >= 0.9 and same_hf > same_exact + 0.1, (same_hf, same_exact)
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
+def test_hf_rope_numerics_refused_by_the_cross_head_tensor_core_kernel():
+    w = syn.workload("qwen3_14b_32b_t32768_k4_xhead", Ls=4, Lt=3, H=2, B=1, T=64, k=2)
+    W, b = syn.weights(w)
+    cfg, keep = kvx.config_from_tensors(
+        src_layers=w.Ls, tgt_layers=w.Lt, n_kv_heads=w.H, head_dim=w.d, k=w.k, theta_s=w.theta_s,
+        theta_t=w.theta_t, cache_dtype=w.cache_dtype, W=W, b=b, scores=syn.selection_scores(w),
+        head_mix=kvx.KVX_CROSS_HEAD, rope_numerics=kvx.KVX_ROPE_HF)
+    ctx = kvx.kvx_create(cfg, 0)
+    try:
+        with pytest.raises(kvx.KvxError) as e:
+            kvx.kvx_set_kernel(ctx, kvx.KVX_KERNEL_TCGEN05)
+        assert e.value.status == kvx.KVX_ERR_UNSUPPORTED
     finally:
         kvx.kvx_destroy(ctx)
