@@ -80,8 +80,8 @@ typedef enum { KVX_KERNEL_AUTO = 0, KVX_KERNEL_SIMT = 1, KVX_KERNEL_TCGEN05 = 2 
  * the caches -- the angle is the fp32 product of fp32(t) and fp32(omega_i), cos and sin of
  * it are rounded to the cache dtype, and each product and sum of the rotation is rounded
  * to the cache dtype (x' = r(r(a c) + r(-b s)), y' = r(r(b c) + r(a s)); the strip uses -s);
- * the mapped keys are rounded to the cache dtype before the target rotation.  HF runs on
- * the SIMT kernel only (AUTO picks it; TCGEN05 is UNSUPPORTED). */
+ * the mapped keys are rounded to the cache dtype before the target rotation.  Every map
+ * kernel, kvx_fit_ridge, kvx_r2_probe and kvx_mlp_map implement both. */
 typedef enum { KVX_ROPE_EXACT = 0, KVX_ROPE_HF = 1 } kvx_rope_numerics;
 
 /* Llama-3 RoPE frequency scaling (the rope_scaling of the Llama 3.1 checkpoints:

@@ -282,9 +282,8 @@ kvx_status kvx_create(const kvx_config* cfg, int device, kvx_ctx** out) {
   }
 
   std::string why;
-  // the per-head tensor-core kernel has both RoPE numerics; the cross-head one the exact only
   ctx->tc_eligible = tc_supported(ctx, &why);
-  ctx->xh_eligible = ctx->rope_numerics == KVX_ROPE_EXACT && xh_supported(ctx, &why);
+  ctx->xh_eligible = xh_supported(ctx, &why);
   if (ctx->tc_eligible || ctx->xh_eligible) {
     kvx_status s = ctx->tc_eligible                  ? tc_prepare(ctx, c.W)
                    : ctx->weight_dtype == KVX_F32 ? repack_wt_hilo(ctx, c.W)

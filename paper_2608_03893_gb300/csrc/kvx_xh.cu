@@ -84,6 +84,7 @@ struct XhParams {
   int32_t* status;
   int32_t Lt, H, k, pairs, n_units, out_bh;
   int32_t lo_steps;       // fp32 weights: k n_kv further K steps over the same source tiles with W_lo
+  int32_t hf;             // the Hugging Face forward's RoPE rounding (kvx_rope_numerics)
   RopeTables rope;
 };
 
@@ -386,8 +387,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
 #pragma unroll
         for (int m = 0; m < 32; ++m) {
           const int i = 32 * g + m;
-          rope_sincos(p, P.rope.wt_hi[i], P.rope.wt_lo[i], P.rope.two_pi_hi, P.rope.two_pi_lo, P.rope.inv_two_pi,
-                      &sn[m], &cs[m]);
+          if (P.hf) {   // cos / sin of the fp32 angle, rounded to bf16
+            sincosf(__fmul_rn(static_cast<float>(p), P.rope.wt_hi[i]), &sn[m], &cs[m]);
+            sn[m] = bf16_round(sn[m]);
+            cs[m] = bf16_round(cs[m]);
+          } else {
+            rope_sincos(p, P.rope.wt_hi[i], P.rope.wt_lo[i], P.rope.two_pi_hi, P.rope.two_pi_lo, P.rope.inv_two_pi,
+                        &sn[m], &cs[m]);
+          }
         }
       }
       const uint32_t bslot = bn % kXBiasSlots;
@@ -443,9 +450,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
               const float2 c = make_float2(cs[16 * rnd + j], cs[16 * rnd + j + 1]);
               const float2 sv = make_float2(sn[16 * rnd + j], sn[16 * rnd + j + 1]);
               const float2 y0 = make_float2(ylo[j], ylo[j + 1]), y1 = make_float2(yhi[j], yhi[j + 1]);
-              const float2 uu = __fmul2_rn(y1, sv);
-              const float2 r0 = __ffma2_rn(y0, c, make_float2(-uu.x, -uu.y));
-              const float2 r1 = __ffma2_rn(y0, sv, __fmul2_rn(y1, c));
+              float2 r0, r1;
+              if (P.hf) {   // the key as bf16, products and sums rounded to bf16
+                const float2 b0 = bf16_round2(y0), b1 = bf16_round2(y1);
+                const float2 p0 = bf16_round2(__fmul2_rn(b0, c)), p1 = bf16_round2(__fmul2_rn(b1, sv));
+                const float2 p2 = bf16_round2(__fmul2_rn(b1, c)), p3 = bf16_round2(__fmul2_rn(b0, sv));
+                r0 = make_float2(__fsub_rn(p0.x, p1.x), __fsub_rn(p0.y, p1.y));
+                r1 = make_float2(__fadd_rn(p2.x, p3.x), __fadd_rn(p2.y, p3.y));
+              } else {
+                const float2 uu = __fmul2_rn(y1, sv);
+                r0 = __ffma2_rn(y0, c, make_float2(-uu.x, -uu.y));
+                r1 = __ffma2_rn(y0, sv, __fmul2_rn(y1, c));
+              }
               ylo[j] = r0.x;
               ylo[j + 1] = r0.y;
               yhi[j] = r1.x;
@@ -675,11 +691,13 @@ kvx_status launch_xh(kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   }
   P.n_units = static_cast<int>(units);
   P.lo_steps = c->weight_dtype == KVX_F32 ? c->k * c->H : 0;
+  P.hf = c->rope_numerics == KVX_ROPE_HF;
   P.rope = c->rope;
 
   // 1. strip the source RoPE from every key into the workspace
   {
-    launch_key_strip(a.src_k, a.ss, c->d_ws, a.pos, c->Ls, c->H, a.B, a.T, c->rope, c->sm_count, stream, 0);
+    launch_key_strip(a.src_k, a.ss, c->d_ws, a.pos, c->Ls, c->H, a.B, a.T, c->rope, c->sm_count, stream,
+                     c->rope_numerics == KVX_ROPE_HF);
     if ((e = cudaGetLastError()) != cudaSuccess) {
       set_error(std::string("kvx_map: strip launch: ") + cudaGetErrorString(e));
       return KVX_ERR_CUDA;
