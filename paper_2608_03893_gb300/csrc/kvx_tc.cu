@@ -1,5 +1,5 @@
-// Tensor-core mapping kernel for sm_103a (tcgen05 + TMEM + TMA), bf16 caches and
-// weights, head_dim 128, per-head features, half-split RoPE pairs, k <= 4.
+// Tensor-core mapping kernel for sm_103a (tcgen05 + TMEM + TMA), bf16 caches, bf16 or
+// fp32 weights, head_dim 128, per-head features, half-split RoPE pairs, k <= 4.
 //
 // It computes Eq. ridge_kv with the Sec. 3.3 RoPE composition,
 //   K_t^{l,h} = R_t(t) ( [R_s(t)^-1 K_s^{sel[l][j]}[h]]_j W_K^{l,h} + b_K^{l,h} ),
@@ -26,6 +26,11 @@
 // CTA's own two 128-column fp32 TMEM accumulators.  Sharing B halves each SM's W traffic
 // from L2 and the shared memory it needs per use, so each issuer's ring holds four uses.
 // W needs no L2 prefetch: the clusters in flight share one (K|V, head) block.
+//
+// fp32 weights (the paper keeps W in fp32) are split on the host into bf16 hi = bf16(w)
+// and lo = bf16(w - hi); each use then takes two W stages, hi and lo, whose MMAs read the
+// same source tile and accumulate into the same TMEM accumulator, so X W = X W_hi + X W_lo
+// to within 2^-17 of each weight.
 //
 // Cross-CTA hand-offs: both CTAs' W loads complete on the rank-0 CTA's stage barrier;
 // both CTAs' prologue and epilogue warps arrive on the rank-0 CTA's tready / acce
@@ -71,6 +76,7 @@
 #include "kvx_internal.h"
 #include "kvx_ptx.cuh"
 #include "kvx_rope.cuh"
+#include "kvx_xh.h"
 
 namespace kvx {
 namespace {
@@ -126,7 +132,7 @@ static_assert(kRing >= 2, "each W ring must hold two uses");
 struct TcParams {
   CUtensorMap tm_k;      // source keys   [L_s][B][H][T][128] bf16, box 64 x 128
   CUtensorMap tm_v;      // source values
-  CUtensorMap tm_w;      // W^T [L_t*2*H*128][F] bf16, box 64 x 128
+  CUtensorMap tm_w;      // W^T [L_t*2*H*128][F] bf16 (fp32 weights: [hi | lo], 2F columns), box 64 x 64
   CUtensorMap tm_out_k;  // target keys as (64 ch, T, 2 halves, B*H or H, L_t), box 32 x 32 x 2 x 1 x 1
   CUtensorMap tm_out_v;  // target values (contiguous targets whose (batch, head) dims merge)
   MapArgs a;
@@ -167,7 +173,8 @@ __device__ __forceinline__ void report(int32_t* status, int code) { atomicCAS(st
 
 // kHF: the Hugging Face forward's RoPE rounding (kvx_rope_numerics): cos / sin of the fp32
 // angle rounded to bf16, every product and sum of the rotations rounded to bf16.
-template <bool kHF>
+// kParts: W stages per use, 1 for bf16 weights, 2 (hi, lo) for fp32 weights.
+template <bool kHF, int kParts>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     tc_map_kernel(const __grid_constant__ TcParams P) {
   extern __shared__ __align__(1024) uint8_t smem[];
@@ -328,12 +335,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 2) {
     // ----------------------------------------------------------- W producer ------
-    // One thread polls the W ring of each issuer (the 2k stages of every layer of its
-    // parity, in order) without blocking: a blocking wait on one ring would starve the
-    // other issuer.
+    // One thread polls the W ring of each issuer (the k kParts stages of every layer of
+    // its parity, in order) without blocking: a blocking wait on one ring would starve
+    // the other issuer.
     if (lane == 0) {
       const uint64_t pol = policy_evict_last();
-      const int chunks = k;      // uses per layer, one 128-feature stage each
+      const int chunks = k * kParts;   // stages per layer: one 128-feature stage per use and part
       int wu[kIssuers], wl[kIssuers], wc[kIssuers], wkv[kIssuers], wh[kIssuers];
       uint32_t wn[kIssuers];     // stages filled into ring r
       for (int r = 0; r < kIssuers; ++r) {
@@ -374,8 +381,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const uint32_t wdst = smem_u32(wst + static_cast<size_t>(st) * kWStageBytes);
           const uint32_t wbar = mapa_shared(smem_u32(&wfull[st]), 0);
           const int wrow = ((wl[r] * 2 + wkv[r]) * H + wh[r]) * kD + static_cast<int>(rank) * (kD / 2);
-          tma_load_2d_pair(wdst, &P.tm_w, wbar, wc[r] * 128, wrow, pol);
-          tma_load_2d_pair(wdst + kWStageBytes / 2, &P.tm_w, wbar, wc[r] * 128 + 64, wrow, pol);
+          // stage c of a layer: use j = c / kParts, part p = c % kParts at W^T column p F + 128 j
+          const int wx = (wc[r] % kParts) * k * 128 + (wc[r] / kParts) * 128;
+          tma_load_2d_pair(wdst, &P.tm_w, wbar, wx, wrow, pol);
+          tma_load_2d_pair(wdst + kWStageBytes / 2, &P.tm_w, wbar, wx + 64, wrow, pol);
           ++wn[r];
           if (++wc[r] == chunks) {
             wc[r] = 0;
@@ -426,7 +435,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     if (lane == 0 && rank == 0) {
       constexpr uint32_t idesc = make_idesc(2 * kTileM, kD);   // M = 256: both CTAs' token tiles
       const uint32_t d_tmem = tmem_base + iss * kAccCols;
-      uint32_t ready_par = 0, acc_n = 0, wi = 0;   // wi: W stages (uses) consumed from this issuer's ring
+      uint32_t ready_par = 0, acc_n = 0, wi = 0;   // wi: W stages consumed from this issuer's ring
       bool ok = true, issued = false;
       uint32_t pack_next = iss < Lt ? __ldg(&P.use_pack[iss]) : 0u;
       for (int u = unit0; ok && u < n_units; u += unit_step) {
@@ -440,7 +449,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             break;
           }
           tc_fence_after();
-          for (int j = 0; j < k; ++j, ++wi) {
+          for (int j = 0; ok && j < k; ++j) {
             // use bits: slot | 4 first use of the tile by this issuer | 16 release the
             // slot after this use.  The prologue warps signal tready[slot][issuer] only
             // for the loads this issuer uses, so it waits for every phase in order.
@@ -455,23 +464,26 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
               ready_par ^= 1u << s;
               tc_fence_after();   // the tile was written by other threads' tcgen05.st
             }
-            const uint32_t st0 = iss * kRing + wi % kRing;
-            if (!wait_bar(smem_u32(&wfull[st0]), (wi / kRing) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
-              ok = false;
-              break;
-            }
             const uint32_t a_col = tmem_base + kSlotCol0 + s * 64;
-            const uint32_t b0 = smem_u32(wst + static_cast<size_t>(st0) * kWStageBytes);
-            const uint32_t b1 = b0 + kWStageBytes / 2;
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-              tc_mma_ts_pair(d_tmem, a_col + kk * 8, sw128_desc(b0 + kk * 32), idesc, (j | kk) != 0);
+            for (int p = 0; p < kParts; ++p, ++wi) {   // hi (and lo) stages of this use
+              const uint32_t st0 = iss * kRing + wi % kRing;
+              if (!wait_bar(smem_u32(&wfull[st0]), (wi / kRing) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
+                ok = false;
+                break;
+              }
+              const uint32_t b0 = smem_u32(wst + static_cast<size_t>(st0) * kWStageBytes);
+              const uint32_t b1 = b0 + kWStageBytes / 2;
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-              tc_mma_ts_pair(d_tmem, a_col + 32 + kk * 8, sw128_desc(b1 + kk * 32), idesc, true);
-            issued = true;
-            tc_commit_pair(smem_u32(&wempty[st0]), 3);
-            if (f & 16u) tc_commit_pair(smem_u32(&tfree[s * kIssuers + iss]), 3);
+              for (int kk = 0; kk < 4; ++kk)
+                tc_mma_ts_pair(d_tmem, a_col + kk * 8, sw128_desc(b0 + kk * 32), idesc, (j | p | kk) != 0);
+#pragma unroll
+              for (int kk = 0; kk < 4; ++kk)
+                tc_mma_ts_pair(d_tmem, a_col + 32 + kk * 8, sw128_desc(b1 + kk * 32), idesc, true);
+              issued = true;
+              tc_commit_pair(smem_u32(&wempty[st0]), 3);
+            }
+            if (ok && (f & 16u)) tc_commit_pair(smem_u32(&tfree[s * kIssuers + iss]), 3);
           }
           if (ok) tc_commit_pair(smem_u32(&accf[iss]), 3);
         }
@@ -908,7 +920,7 @@ void* tensor_map_encoder() { return reinterpret_cast<void*>(get_encode()); }
 
 bool tc_supported(const kvx_ctx* c, std::string* why) {
   std::string w;
-  if (c->cache_dtype != KVX_BF16 || c->weight_dtype != KVX_BF16) w = "needs bf16 caches and weights";
+  if (c->cache_dtype != KVX_BF16) w = "needs bf16 caches";
   else if (c->d != kD) w = "needs head_dim 128";
   else if (c->head_mix != KVX_PER_HEAD) w = "needs per-head features";
   else if (c->rope_style != KVX_ROPE_HALF) w = "needs half-split RoPE pairs";
@@ -943,7 +955,7 @@ kvx_status repack_wt(kvx_ctx* c, const void* W_host) {
 }
 
 kvx_status tc_prepare(kvx_ctx* c, const void* W_host) {
-  kvx_status st = repack_wt(c, W_host);
+  kvx_status st = c->weight_dtype == KVX_F32 ? repack_wt_hilo(c, W_host) : repack_wt(c, W_host);
   if (st != KVX_OK) return st;
   cudaError_t e;
   build_plan(c, &c->plan);
@@ -1027,8 +1039,10 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
       }
     }
   }
-  const cuuint64_t wdims[2] = {static_cast<cuuint64_t>(c->F), static_cast<cuuint64_t>(c->Lt) * 2 * c->H * kD};
-  const cuuint64_t wstr[1] = {static_cast<cuuint64_t>(c->F) * 2};
+  // fp32 weights: W^T holds [W_hi | W_lo], 2F columns
+  const cuuint64_t wcols = static_cast<cuuint64_t>(c->F) * (c->weight_dtype == KVX_F32 ? 2 : 1);
+  const cuuint64_t wdims[2] = {wcols, static_cast<cuuint64_t>(c->Lt) * 2 * c->H * kD};
+  const cuuint64_t wstr[1] = {wcols * 2};
   const cuuint32_t wbox[2] = {64, kD / 2};   // one CTA's 64 output rows x 64 features
   CUresult r = encode(&P.tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, c->d_Wt, wdims, wstr, wbox, ones,
                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -1058,7 +1072,9 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   P.n_units = static_cast<int>(units);
   P.rope = c->rope;
   const size_t smem = smem_bytes();
-  void (*kernel)(TcParams) = c->rope_numerics == KVX_ROPE_HF ? tc_map_kernel<true> : tc_map_kernel<false>;
+  const bool hf = c->rope_numerics == KVX_ROPE_HF;
+  void (*kernel)(TcParams) = c->weight_dtype == KVX_F32 ? (hf ? tc_map_kernel<true, 2> : tc_map_kernel<false, 2>)
+                                                        : (hf ? tc_map_kernel<true, 1> : tc_map_kernel<false, 1>);
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) {
     set_error(std::string("kvx_map: smem attribute: ") + cudaGetErrorString(e));

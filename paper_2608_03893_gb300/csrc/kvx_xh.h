@@ -12,7 +12,7 @@ void launch_key_strip(const void* src_k, const int64_t* ss, void* ws, const int3
                       const RopeTables& rope, int sms, cudaStream_t stream, int hf);
 
 // fp32 W [L_t][2][H][F][128] -> W^T bf16 [L_t][2][H][128][2F] = [W_hi | W_lo] in ctx->d_Wt,
-// for the cross-head tensor-core kernel with fp32 weights.
+// for the tensor-core map kernels (cross-head and per-head) with fp32 weights.
 kvx_status repack_wt_hilo(kvx_ctx* c, const void* W_host);
 
 }  // namespace kvx

@@ -573,6 +573,39 @@ def test_cross_head_tc_fp32_weights_hi_lo():
         kvx.kvx_destroy(ctx)
 
 
+@pytest.mark.parametrize("over", [
+    dict(Ls=6, Lt=5, H=2, B=2, T=300, k=3),                 # ragged tail, B > 1
+    dict(Ls=8, Lt=9, H=2, B=1, T=256, k=4, scores="uniform"),  # k = 4, reloads
+])
+def test_per_head_tc_fp32_weights_hi_lo(over):
+    """Per-head tensor-core kernel with fp32 W: each use takes a hi and a lo W stage over
+    the same source tile, so the result follows the fp32 weights.  Every output within the
+    usual bound of the oracle given the fp32 W; at least 90 % of the values equal to the
+    correctly rounded fp32-W result, where W rounded to bf16 gets visibly fewer."""
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", **over)
+    _kernel_or_skip(w, kvx.KVX_KERNEL_TCGEN05)
+    Wb, b = syn.weights(w)
+    g = torch.Generator().manual_seed(6)
+    W32 = (Wb.float() * (1.0 + 2.0 ** -9 * (0.5 + 0.5 * torch.rand(Wb.shape, generator=g)))).contiguous()
+    ctx, sel, _, _ = make_ctx(w, kernel=kvx.KVX_KERNEL_TCGEN05, W=W32, b=b)
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w)
+        rk, rv, ak, av = oracle_full(w, sk, sv, pos, sel, W32, b)
+        tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        ok, ratio, rms, nbad = check(w, [to_f64(tk), to_f64(tv)], [rk, rv], [ak, av])
+        assert ok, "%d elements out of tolerance (worst %.3g x bound)" % (nbad, ratio)
+        from oracle import bf16 as obf16
+        exact = np.mean(to_f64(tv) == obf16.round_to_bf16_value(rv))
+        hv_ = oracle_full(w, sk, sv, pos, sel, Wb, b)[1]     # W rounded to bf16
+        hi_only = np.mean(obf16.round_to_bf16_value(hv_) == obf16.round_to_bf16_value(rv))
+        assert exact >= 0.9 and exact > hi_only + 0.05, (exact, hi_only)
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
 # ---------------------------------------------------------------- HF RoPE numerics -----
 
 @pytest.mark.parametrize("kname", ["simt", "tc"])
@@ -582,8 +615,7 @@ def test_hf_rope_numerics(kname):
     the oracle in the same numerics, at positions past 2 * 10^4 where the fp32 angle is
     coarse: every output within the bound, at least 90 % of the keys bit-equal to the
     oracle's (the rest follow a rounding of the fp32-accumulated contraction or of cos / sin
-    near a bf16 midpoint), far more than agree with the exact-RoPE oracle.  The cross-head
-    tensor-core kernel refuses the mode."""
+    near a bf16 midpoint), far more than agree with the exact-RoPE oracle."""
     w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=5, Lt=4, H=2, B=2, T=200, k=2, theta_t=5e5)
     W, b = syn.weights(w)
     scores = syn.selection_scores(w)
