@@ -188,6 +188,12 @@ def max_over_ranks(x, dist, dev):
     return float(t.item())
 
 
+def job_rate(world, tokens_per_step, steps, ms):
+    """Whole-job tokens/s: every rank maps tokens_per_step tokens per step (replicas, weak
+    scaling), over the slowest rank's elapsed ms."""
+    return world * tokens_per_step * steps / (ms / 1e3)
+
+
 # ------------------------------------------------------------------ oracle leg ----
 
 def oracle_sample_rate(w, budget_s, seed=0, ctx_sel=None):
@@ -591,7 +597,7 @@ def main():
     ms = max_over_ranks(ms, dist, dev)
     st = kvx.kvx_get_status(ctx, sp)
     ms_step = ms / args.steps
-    value = world * w.n_tokens * args.steps / (ms / 1e3)
+    value = job_rate(world, w.n_tokens, args.steps, ms)
 
     # ---- e2e: host buffers through the C ABI, copies inside the timed region
     e2e_steps = args.e2e_steps or max(3, min(args.steps, 40))
@@ -636,7 +642,7 @@ def main():
     torch.cuda.synchronize()
     barrier(dist)
     ems = max_over_ranks(e0.elapsed_time(e1), dist, dev)
-    e2e_value = world * w.n_tokens * e2e_steps / (ems / 1e3)
+    e2e_value = job_rate(world, w.n_tokens, e2e_steps, ems)
     e2e_api = "kvx_map_host (chunks of %d tokens)" % chunk if pipe is not None else "copies + kvx_map"
     if pipe is not None:
         kvx.kvx_host_pipe_destroy(pipe)
