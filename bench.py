@@ -44,7 +44,7 @@ METRIC = "mapped target-KV tokens/s"
 UNIT = "tokens/s"
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "tc_map_kernel_qwen3_14b_32b_traffic.txt")
 KERNEL_SOURCES = ["paper_2608_03893_gb300/csrc/kvx_tc.cu", "paper_2608_03893_gb300/csrc/kvx_rope.cuh",
-                  "paper_2608_03893_gb300/csrc/kvx_internal.h"]
+                  "paper_2608_03893_gb300/csrc/kvx_internal.h", "paper_2608_03893_gb300/csrc/kvx_ptx.cuh"]
 
 
 def algorithmic(w):
@@ -89,10 +89,13 @@ def kernel_hash(read=None):
     return h.hexdigest()[:16]
 
 
-def committed_traffic(workload):
-    """dram bytes per launch from the committed ncu summary, if taken on this kernel."""
-    if not os.path.exists(TRAFFIC_FILE):
+def committed_traffic(w):
+    """dram bytes per launch from the committed ncu summary, if taken on this kernel and on
+    the named workload as defined (no --override: a changed field such as the weight dtype
+    changes the kernel instance or its traffic)."""
+    if not os.path.exists(TRAFFIC_FILE) or syn.WORKLOADS.get(w.name) != w:
         return None
+    workload = w.name
     kv = {}
     for ln in open(TRAFFIC_FILE):
         if ":" in ln and not ln.startswith("#"):
@@ -664,7 +667,7 @@ def main():
     else:
         achieved, peak, unit = alg["bytes"] / launch_s / 1e9, peaks["hbm"], "GB/s"
     roofline = {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
-                "frac": achieved / peak, "traffic": committed_traffic(w.name),
+                "frac": achieved / peak, "traffic": committed_traffic(w),
                 "peak_source": "%s (bf16 burst; HBM copy)" % peaks["source"],
                 "roofline_ms": 1e3 * max(t_tc, t_hbm),
                 "other": {"hbm_achieved_gbs": alg["bytes"] / launch_s / 1e9, "hbm_peak_gbs": peaks["hbm"],
