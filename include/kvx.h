@@ -70,8 +70,9 @@ typedef enum { KVX_PER_HEAD = 0, KVX_CROSS_HEAD = 1 } kvx_head_mix;
  * shape allows it (bf16 caches, head_dim 128, HALF; PER_HEAD with k <= 4, or CROSS_HEAD
  * with an even head count and a contiguous target) and the fp32 SIMT kernel otherwise.
  * fp32 weights run on the tensor cores split into bf16 hi = bf16(w) and lo = bf16(w - hi)
- * (twice the MMAs; the contraction follows the fp32 W to within 2^-17 of each weight).  The CROSS_HEAD tensor-core kernel keeps a workspace for the stripped source
- * keys (L_s * B * n_kv * T * head_dim bf16) in the context, allocated by the first
+ * (twice the MMAs; the contraction follows the fp32 W to within 2^-17 of each weight).
+ * The CROSS_HEAD tensor-core kernel keeps a workspace for the stripped source keys
+ * (L_s * B * n_kv * T * head_dim bf16) in the context, allocated by the first
  * kvx_map that needs it (a blocking cudaMalloc) and grown when a later call needs more;
  * kvx_destroy frees it. */
 typedef enum { KVX_KERNEL_AUTO = 0, KVX_KERNEL_SIMT = 1, KVX_KERNEL_TCGEN05 = 2 } kvx_kernel;
