@@ -166,6 +166,32 @@ class ClockSampler:
                 "power_w_max": max(r["power"] for r in rows)}
 
 
+def measure_link(h_src, h_dst, d_src, d_dst, dev, reps=3):
+    """Host link bandwidth of this machine in GB/s, from pinned copies of the step's own
+    buffers: host->device alone, device->host alone, and both at once on two streams
+    (best of `reps`).  The e2e copy floor of a step follows from these."""
+    def timed(fns):
+        best = float("inf")
+        for _ in range(reps):
+            streams = [torch.cuda.Stream(dev) for _ in fns]
+            torch.cuda.synchronize(dev)
+            t0 = time.perf_counter()
+            for s, fn in zip(streams, fns):
+                with torch.cuda.stream(s):
+                    fn()
+            torch.cuda.synchronize(dev)
+            best = min(best, time.perf_counter() - t0)
+        return best
+    hb = h_src.numel() * h_src.element_size()
+    db = h_dst.numel() * h_dst.element_size()
+    t_h = timed([lambda: d_src.copy_(h_src, non_blocking=True)])
+    t_d = timed([lambda: h_dst.copy_(d_dst, non_blocking=True)])
+    t_b = timed([lambda: d_src.copy_(h_src, non_blocking=True), lambda: h_dst.copy_(d_dst, non_blocking=True)])
+    return {"h2d_gbs": hb / t_h / 1e9, "d2h_gbs": db / t_d / 1e9, "both_gbs": (hb + db) / t_b / 1e9,
+            "measured_on": "one key cache each way (%.2f GB in, %.2f GB out), pinned, best of %d"
+                           % (hb / 1e9, db / 1e9, reps)}
+
+
 def dist_setup(n_gpus):
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -646,6 +672,8 @@ def main():
     barrier(dist)
     ems = max_over_ranks(e0.elapsed_time(e1), dist, dev)
     e2e_value = job_rate(world, w.n_tokens, e2e_steps, ems)
+    link = measure_link(hk, ok_, sk, tk, dev)
+    floor_ms = max(h2d / link["h2d_gbs"], d2h / link["d2h_gbs"], (h2d + d2h) / link["both_gbs"]) / 1e6
     e2e_api = "kvx_map_host (chunks of %d tokens)" % chunk if pipe is not None else "copies + kvx_map"
     if pipe is not None:
         kvx.kvx_host_pipe_destroy(pipe)
@@ -688,12 +716,18 @@ def main():
         cpu = {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
                "sample": "%d random tokens of the workload (all %d layers x %d heads x K,V), "
                          "float64 numpy oracle, %.1f s" % (n, w.Lt, w.H, dt)}
+    clocks = clk.summary()
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config,
-            "clocks": clk.summary(), "status": kvx.kvx_status_string(st),
+            "clocks": clocks, "status": kvx.kvx_status_string(st),
+            # ms per step x median SM MHz = thousands of SM cycles per step: compares runs
+            # taken at different clocks (a power-capped long run against a short burst)
+            "kcycles_per_step": (ms_step * clocks["sm_mhz"] if clocks.get("sm_mhz") else None),
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                    "steps": e2e_steps, "ms_per_step": ems / e2e_steps, "api": e2e_api},
+                    "steps": e2e_steps, "ms_per_step": ems / e2e_steps, "api": e2e_api,
+                    "link_gbs": link, "copy_floor_ms": floor_ms,
+                    "frac_of_copy_floor": floor_ms / (ems / e2e_steps)},
             # one launch per step (per-head); the cross-head map is a key-strip kernel then the GEMMs
             "gpu_launches": args.steps * (2 if w.head_mix == "cross_head" else 1), "roofline": roofline,
             "cpu_baseline": cpu,

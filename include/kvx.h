@@ -238,7 +238,9 @@ KVX_API int64_t kvx_mapper_params(int32_t tgt_layers, int32_t n_kv_heads, int32_
  * as in kvx_config.  Outputs on the device, fp32: W [L_t][2][H][k*d][d] and
  * b [L_t][2][H][d] (the kvx_config layouts).  Cross-products of the centred values run
  * on the tensor cores from a bf16 hi + lo split of each value (within 2^-17 of it) and
- * accumulate in fp32; the factorisation and the solves run in fp64.  Runs on `stream` and
+ * accumulate in fp32; the factorisation and the solves run in float-float arithmetic (each
+ * value an unevaluated sum of two fp32 numbers, about 48 significant bits) on the FP32
+ * units, and the bias in fp64.  Runs on `stream` and
  * synchronises it before returning (an offline step).  Stream-ordered workspace: the
  * blocks (at most L_t*2*H*(k*(k+1)/2 + k)*64 KB), 8 MB per SM, and the packed operands
  * (4 bytes per token, channel, K|V, head and used layer of either model), at most half the
@@ -368,7 +370,8 @@ KVX_API const char* kvx_last_error(void);
  * implicit device synchronisation of cudaMalloc / cudaFree.  kvx_map_noalloc serves them:
  * the caller passes everything in its own buffers (caches, positions, W and bias on the
  * device, the selection table on the host) and the library allocates nothing.  The map
- * runs on the fp32 SIMT kernel, with the same results as kvx_map with KVX_KERNEL_SIMT.
+ * runs on the fp32 SIMT kernel, with the same results as kvx_map with KVX_KERNEL_SIMT
+ * on a context of the same configuration (rope_numerics included).
  *
  * The little device memory it needs besides the caller's buffers -- a status word and a
  * copy of the selection table -- lives in one fixed array inside libkvx
@@ -397,13 +400,20 @@ typedef struct {
   const float* b;              /* DEVICE fp32 [L_t][2][n_kv][d] (pass zeros for no bias), 16-byte aligned */
   const kvx_rope_scaling* src_rope_scaling;   /* NULL: plain theta */
   const kvx_rope_scaling* tgt_rope_scaling;
+  int32_t rope_numerics;       /* kvx_rope_numerics, as in kvx_config (0 = KVX_ROPE_EXACT) */
 } kvx_noalloc_mapper;
 
 /* Map as kvx_map does, allocating nothing.  src, tgt, positions, batch and
  * tokens_per_seq are as for kvx_map; `device` is the CUDA device that owns every pointer.
  * Asynchronous on `stream` unless device_status is non-NULL: then the call waits for the
  * stream and stores the device-detected status (KVX_OK, KVX_ERR_DEVICE_BOUNDS) there.
- * Host-detected errors return before any launch. */
+ * Host-detected errors return before any launch, INVALID_ARG among them for a selection
+ * row that names a source layer twice.
+ *  - The selection table is copied to the device on `stream` (cudaMemcpyAsync): when it
+ *    sits in pinned host memory the copy reads it only when the stream reaches it, so
+ *    the caller keeps it unchanged until the stream has passed this call.
+ *  - Pass device_status = NULL while `stream` is being captured: reading the status waits
+ *    for the stream, which a stream under capture does not allow. */
 KVX_API kvx_status kvx_map_noalloc(const kvx_noalloc_mapper* m, int device, const kvx_src* src,
                                    int32_t batch, int32_t tokens_per_seq, const int32_t* positions,
                                    const kvx_tgt* tgt, void* stream, int32_t* device_status);

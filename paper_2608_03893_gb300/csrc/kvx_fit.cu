@@ -450,6 +450,7 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
                                  int32_t tokens_per_seq, const int32_t* positions, float* W, float* b,
                                  void* stream) {
   using namespace kvx;
+  NvtxRange range("kvx_fit_ridge");
   set_error("");
   auto bad = [](const char* m) {
     set_error(std::string("kvx_fit_ridge: ") + m);

@@ -347,6 +347,7 @@ kvx_status kvx_get_status(kvx_ctx* ctx, void* stream) {
 
 kvx_status kvx_map(kvx_ctx* ctx, const kvx_src* src, int32_t batch, int32_t tokens_per_seq,
                    const int32_t* positions, const kvx_tgt* tgt, void* stream) {
+  NvtxRange range("kvx_map");
   g_last_error.clear();
   if (!ctx || !src || !tgt) return fail(KVX_ERR_INVALID_ARG, "kvx_map: NULL ctx/src/tgt");
   if (batch < 0 || tokens_per_seq < 0)

@@ -6,10 +6,20 @@
 #include <vector>
 
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include "../../include/kvx.h"
 
 namespace kvx {
+
+// A named NVTX range over one entry point's host work (its launches and copies show
+// under it in a timeline profiler); a no-op unless a profiler is attached.
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 constexpr int kMaxHeadDim = 256;
 constexpr int kMaxPairs = kMaxHeadDim / 2;

@@ -451,6 +451,7 @@ KVX_API int64_t kvx_mlp_workspace_bytes(const kvx_mlp_config* cfg, int32_t batch
 KVX_API kvx_status kvx_mlp_map(const kvx_mlp_config* cfg, const kvx_src* src, int32_t batch, int32_t tokens_per_seq,
                                const int32_t* positions, const kvx_tgt* tgt, void* stream) {
   using namespace kvx;
+  NvtxRange range("kvx_mlp_map");
   set_error("");
   auto bad = [](const std::string& m) {
     set_error("kvx_mlp_map: " + m);

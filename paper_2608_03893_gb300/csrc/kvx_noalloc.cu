@@ -79,9 +79,18 @@ extern "C" KVX_API kvx_status kvx_map_noalloc(const kvx_noalloc_mapper* m, int d
   if (!m->selection || !m->W || !m->b) return fail(KVX_ERR_INVALID_ARG, "kvx_map_noalloc: NULL selection, W or b");
   if (!aligned(m->W, 16) || !aligned(m->b, 16))
     return fail(KVX_ERR_INVALID_ARG, "kvx_map_noalloc: W and b must be 16-byte aligned");
+  if (m->rope_numerics != KVX_ROPE_EXACT && m->rope_numerics != KVX_ROPE_HF)
+    return fail(KVX_ERR_INVALID_ARG, "kvx_map_noalloc: bad rope_numerics");
   for (int64_t i = 0; i < static_cast<int64_t>(m->tgt_layers) * m->k; ++i)
     if (m->selection[i] < 0 || m->selection[i] >= m->src_layers)
       return fail(KVX_ERR_INVALID_ARG, "kvx_map_noalloc: selection entry outside [0, src_layers)");
+  for (int64_t l = 0; l < m->tgt_layers; ++l) {  // a row names k distinct source layers
+    const int32_t* row = m->selection + l * m->k;
+    for (int i = 0; i < m->k; ++i)
+      for (int j = 0; j < i; ++j)
+        if (row[i] == row[j])
+          return fail(KVX_ERR_INVALID_ARG, "kvx_map_noalloc: duplicate source layer in a selection row");
+  }
   if (batch < 0 || tokens_per_seq < 0) return fail(KVX_ERR_INVALID_ARG, "kvx_map_noalloc: negative sizes");
   if (device_status) *device_status = KVX_OK;
   if (batch == 0 || tokens_per_seq == 0) return KVX_OK;
@@ -138,6 +147,7 @@ extern "C" KVX_API kvx_status kvx_map_noalloc(const kvx_noalloc_mapper* m, int d
   view.weight_dtype = m->weight_dtype;
   view.theta_s = m->src_rope_theta;
   view.theta_t = m->tgt_rope_theta;
+  view.rope_numerics = m->rope_numerics;
   kvx::set_rope_scaling(&view, m->src_rope_scaling, m->tgt_rope_scaling);
   kvx::fill_rope(&view);
   view.d_sel = d_sel;

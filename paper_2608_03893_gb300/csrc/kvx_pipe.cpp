@@ -115,6 +115,7 @@ KVX_API kvx_status kvx_host_pipe_create(kvx_ctx* ctx, int32_t batch, int32_t chu
 
 KVX_API kvx_status kvx_map_host(kvx_host_pipe* p, const kvx_src* src, int32_t tokens_per_seq, const int32_t* positions,
                                 const kvx_tgt* tgt, void* stream) {
+  kvx::NvtxRange range("kvx_map_host");
   kvx::set_error("");
   if (!p || !src || !tgt || !positions) return pipe_fail(KVX_ERR_INVALID_ARG, "kvx_map_host: NULL argument");
   if (tokens_per_seq < 0) return pipe_fail(KVX_ERR_INVALID_ARG, "kvx_map_host: negative tokens_per_seq");

@@ -294,6 +294,7 @@ KVX_API kvx_status kvx_r2_probe(const kvx_probe_config* cfg, const kvx_src* src,
                                 int32_t tokens_per_seq, const int32_t* positions, double* scores, double* r2_kv,
                                 void* stream) {
   using namespace kvx;
+  NvtxRange range("kvx_r2_probe");
   set_error("");
   auto bad = [](const char* m) { return pfail(std::string("kvx_r2_probe: ") + m, KVX_ERR_INVALID_ARG); };
   if (const char* why = check_probe_config(cfg)) return bad(why);

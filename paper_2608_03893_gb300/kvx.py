@@ -85,7 +85,7 @@ class kvx_noalloc_mapper(ctypes.Structure):
         ("tgt_rope_theta", ctypes.c_double), ("cache_dtype", ctypes.c_int32),
         ("weight_dtype", ctypes.c_int32), ("head_mix", ctypes.c_int32), ("reserved", ctypes.c_int32),
         ("selection", ctypes.c_void_p), ("W", ctypes.c_void_p), ("b", ctypes.c_void_p),
-    ] + _SCALING
+    ] + _SCALING + [("rope_numerics", ctypes.c_int32)]
 
 
 class kvx_fit_config(ctypes.Structure):

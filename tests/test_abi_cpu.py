@@ -278,3 +278,35 @@ def test_create_rejects_bad_rope_numerics():
     with pytest.raises(kvx.KvxError) as e:
         kvx.kvx_create(cfg, 0)
     assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+
+
+def _noalloc_mapper(sel, **over):
+    """A kvx_noalloc_mapper for host-side validation only: W and b are placeholder
+    16-byte aligned addresses that no check before the launch dereferences."""
+    m = kvx.kvx_noalloc_mapper()
+    m.src_layers, m.tgt_layers, m.n_kv_heads, m.head_dim, m.k = 4, sel.shape[0], 2, 64, sel.shape[1]
+    m.rope_style = kvx.KVX_ROPE_HALF
+    m.src_rope_theta = m.tgt_rope_theta = 1e4
+    m.cache_dtype = m.weight_dtype = kvx.KVX_F32
+    m.head_mix = kvx.KVX_PER_HEAD
+    m.selection = sel.ctypes.data
+    m.W, m.b = 0x10000, 0x20000
+    for key, val in over.items():
+        setattr(m, key, val)
+    return m
+
+
+@pytest.mark.parametrize("sel,over,why", [
+    ([[0, 0], [1, 2]], {}, "duplicate"),
+    ([[0, 3], [2, 1]], {"rope_numerics": 2}, "rope_numerics"),
+    ([[0, 4], [1, 2]], {}, "outside"),
+    ([[0, 1], [1, 2]], {"reserved": 1}, "reserved"),
+])
+def test_noalloc_rejects_bad_mapper_before_touching_the_device(sel, over, why):
+    sel = np.ascontiguousarray(sel, dtype=np.int32)
+    m = _noalloc_mapper(sel, **over)
+    src, tgt = kvx.kvx_src(), kvx.kvx_tgt()
+    with pytest.raises(kvx.KvxError) as e:
+        kvx.kvx_map_noalloc(m, 0, src, 1, 8, 0x30000, tgt, want_status=False)
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+    assert why in kvx.kvx_last_error()
