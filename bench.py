@@ -343,18 +343,22 @@ def fit_bench(args, w):
     tk, tv = syn.target_cache(w, 0, device=dev), syn.target_cache(w, 1, device=dev)
     pos = torch.from_numpy(syn.positions(w)).to(dev)
     sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
-    F = w.k * w.d
+    cross = w.head_mix == "cross_head"
+    mix = kvx.KVX_CROSS_HEAD if cross else kvx.KVX_PER_HEAD
+    F = w.F
+    R = w.H * w.d if cross else w.d             # right-hand sides per system
     W = torch.empty((w.Lt, 2, w.H, F, w.d), dtype=torch.float32, device=dev)
     b = torch.empty((w.Lt, 2, w.H, w.d), dtype=torch.float32, device=dev)
     src, tgt = kvx.src_from_tensors(sk, sv), kvx.src_from_tensors(tk, tv)
     # one caller workspace, allocated once (no per-call allocation inside the timed region)
-    ws_bytes = kvx.kvx_fit_workspace_bytes(w.Ls, w.Lt, w.H, w.d, w.k, w.theta_s, w.theta_t, 0.01, sel, w.B, w.T)
+    ws_bytes = kvx.kvx_fit_workspace_bytes(w.Ls, w.Lt, w.H, w.d, w.k, w.theta_s, w.theta_t, 0.01, sel, w.B, w.T,
+                                           head_mix=mix)
     ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
 
     def step():
         kvx.kvx_fit_ridge(w.Ls, w.Lt, w.H, w.d, w.k, w.theta_s, w.theta_t, 0.01, sel, src, tgt, w.B, w.T,
                           pos.data_ptr(), W.data_ptr(), b.data_ptr(), sp, workspace_ptr=ws.data_ptr(),
-                          workspace_bytes=ws_bytes)
+                          workspace_bytes=ws_bytes, head_mix=mix)
 
     for _ in range(args.warmup):
         step()
@@ -371,16 +375,24 @@ def fit_bench(args, w):
         torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / steps
     phase = [p / steps for p in phase]
-    n_sys = w.Lt * 2 * w.H
+    n_sys = w.Lt * 2 * (1 if cross else w.H)
     N = w.n_tokens
     # Source-pair blocks XsaᵀXsb depend only on the two source layers, so every distinct
-    # pair of the selection is one Gram block per (K|V, head); each target layer adds its
-    # k cross blocks XᵀY.  A block is N d² fused multiply-adds.
+    # pair of the selection is one Gram block per (K|V, head) -- per (K|V, head pair) in
+    # cross-head mode, where one layer with itself needs only H(H+1)/2 of them; each target
+    # layer adds its cross blocks XᵀY (k per head, or k H H).  A block is N d² fused
+    # multiply-adds.
     sel_np = np.asarray(sel).reshape(w.Lt, w.k)
     pairs = {(max(int(a), int(c)), min(int(a), int(c))) for row in sel_np for i, a in enumerate(row) for c in row[:i + 1]}
-    gram_flop = 2 * w.H * (len(pairs) + w.Lt * w.k) * 2.0 * N * w.d * w.d
-    gram_flop_unshared = n_sys * (w.k * (w.k + 1) // 2 + w.k) * 2.0 * N * w.d * w.d
-    solve_flop = n_sys * (F ** 3 / 3.0 + 2.0 * F * F * w.d)
+    blk = 2.0 * N * w.d * w.d
+    if cross:
+        n_src_blocks = sum(w.H * (w.H + 1) // 2 if a == c else w.H * w.H for a, c in pairs)
+        gram_flop = 2 * (n_src_blocks + w.Lt * w.k * w.H * w.H) * blk
+        gram_flop_unshared = n_sys * (F // w.d) * (F // w.d + 1) // 2 * blk + 2 * w.Lt * w.k * w.H * w.H * blk
+    else:
+        gram_flop = 2 * w.H * (len(pairs) + w.Lt * w.k) * blk
+        gram_flop_unshared = n_sys * (w.k * (w.k + 1) // 2 + w.k) * blk
+    solve_flop = n_sys * (F ** 3 / 3.0 + 2.0 * F * F * R)
     # dominant kernel: the fp64 solve (Cholesky + two triangular solves per system)
     achieved = solve_flop / (phase[3] / 1e3) / 1e12
     # the Gram kernel issues four bf16 MMAs per product (hi/lo split of both operands)
@@ -392,13 +404,14 @@ def fit_bench(args, w):
             "data": "synthetic",
             "config": {"workload": w.name + " (fit)", "src_layers": w.Ls, "tgt_layers": w.Lt, "kv_heads": w.H,
                        "head_dim": w.d, "k": w.k, "calibration_tokens": N, "systems": n_sys, "lambda": 0.01,
+                       "head_mix": w.head_mix, "features": F, "rhs_per_system": R,
                        "workspace_gb": ws_bytes / 1e9},
             "clocks": clk.summary(),
             "gpu_launches": 4 * steps,
             "phase_ms": {"column_sums": phase[0], "pack": phase[1], "gram_tc": phase[2], "solve": phase[3]},
             "roofline": {"bound": "alu", "achieved": achieved, "peak": FF_PEAK_TFLOPS, "unit": "TFLOP/s",
                          "frac": achieved / FF_PEAK_TFLOPS, "traffic": None,
-                         "kernel": "fit_solve_kernel (float-float on the FP32 lanes)",
+                         "kernel": ("fit_solve_xh_kernel" if cross else "fit_solve_kernel") + " (float-float on the FP32 lanes)",
                          "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2070 MHz / 15 FP32 instructions per "
                                         "float-float FMA x 2 FLOP (the FP64-equivalent work; GB300's FP64 "
                                         "units give 1.25 TFLOP/s nominal)",
@@ -408,7 +421,8 @@ def fit_bench(args, w):
                          "other": {"gram_tc_kernel": {"bound": "tensor", "achieved": gram_tc_tflops,
                                                       "peak": pk["bf16"], "frac": gram_tc_tflops / pk["bf16"],
                                                       "unit": "TFLOP/s (bf16 MMA, four per product)"}}},
-            "kernel": "gram_pack_kernel<0> + gram_pack_kernel<1> + gram_tc_kernel + fit_solve_kernel"}
+            "kernel": "gram_pack_kernel<0> + gram_pack_kernel<1> + gram_tc_kernel + "
+                      + ("fit_solve_xh_kernel" if cross else "fit_solve_kernel")}
     print(json.dumps(line), flush=True)
     return 0
 

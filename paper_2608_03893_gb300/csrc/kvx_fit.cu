@@ -7,6 +7,10 @@
 //   Xc, Yc centred by their column means,
 //   W = (Xc^T Xc + lambda I)^{-1} Xc^T Yc,   b = mean(Y) - mean(X) W.
 // bf16 caches, head_dim 128, half-split pairs.
+// Cross-head mode (the paper's source feature, Appendix "Run information": d_s = k n_kv d):
+// x_j is every KV head of layer sel[l][j] (head-minor), Y every head of target layer l, so
+// there is one system per (l, K|V) with F = k H 128 features and H 128 right-hand sides:
+// Xc^T Xc is formed and factored once per target layer and shared by its heads (Sec. 3.1).
 //
 // Steps:
 // 1. Column sums and the centred Gram blocks on the tensor cores (kvx_gram.cu): a block
@@ -18,7 +22,8 @@
 //    scratch matrix, lambda added, factorised by a blocked right-looking Cholesky
 //    (32-column panels: diagonal block in shared memory, panel by forward substitution,
 //    trailing update), then the two triangular solves for the d right-hand sides and the
-//    bias; W and b are written in fp32.
+//    bias; W and b are written in fp32.  fit_solve_xh_kernel does the same for the
+//    cross-head systems, with the trailing update staged per 64 x 64 tile.
 // kvx_fit_ridge runs them on the caller's stream, with stream-ordered workspace, and
 // synchronises before it returns (the fit is an offline step).
 #include <cuda_runtime.h>
@@ -40,21 +45,26 @@ using namespace ptx;
 
 constexpr int kFD = 128;            // head_dim
 constexpr int kNB = 32;             // Cholesky panel width
+constexpr int64_t kMaxXhFeatures = 16384;   // cross-head F = k H 128 (2 GB of float-float matrix per CTA)
 
 struct FitParams {
   const int32_t* sel;               // [L_t][k]
   int32_t Ls, Lt, H, k, B, T;
   double* sums;                     // [2 sides][2 kv][L][H][128]: side 0 L = L_s, side 1 L = L_t
-  float* gram;                      // [2][H][n_pairs][128][128]: source-pair blocks
+  float* gram;                      // source-pair blocks: per head [2][H][n_pairs][128][128];
+                                    // cross-head [n_pairs][2][H][H][128][128] (pair (sa, sb), blocks
+                                    // (head of sa, head of sb); one layer: only row head >= column head)
   const int32_t* pairs;             // [n_pairs][2] source layers (sa >= sb)
   const int32_t* pair_of;           // [L_t][k][k] pair of block (bi, bj), bi >= bj
   int32_t n_pairs;
-  float* xty;                       // [L_t][2][H][k][128][128]
-  double* scratch;                  // per CTA: F x F matrix + F x 128 right-hand sides
+  float* xty;                       // per head [L_t][2][H][k][128][128]; cross-head
+                                    // [L_t][2][k][H (source head)][H (target head)][128][128]
+  double* scratch;                  // per CTA: F x F matrix + F x R right-hand sides
   float* W;                         // [L_t][2][H][F][128]
   float* b;                         // [L_t][2][H][128]
   double lambda;
   int32_t* status;
+  int32_t R;                        // right-hand sides per system: 128 (per head) or H 128 (cross-head)
 };
 
 __device__ __forceinline__ size_t sums_index(const FitParams& P, int side, int kv, int layer, int h) {
@@ -121,15 +131,162 @@ __device__ __forceinline__ DF df_from_double(double x) {
 }
 __device__ __forceinline__ double df_to_double(DF a) { return static_cast<double>(a.hi) + static_cast<double>(a.lo); }
 
-// Persistent: CTA c handles systems c, c + gridDim.x, ...  F = 128 k (k <= 4).  Dynamic
-// shared memory: the 32 x 32 diagonal block and the panel below it ((F - 32) x 32), pairs
-// of floats (8 bytes an element, as fp64 was).
+// Persistent solve kernels: CTA c handles systems c, c + gridDim.x, ...  Dynamic shared
+// memory holds pairs of floats (8 bytes an element, as fp64 was).
 constexpr int kNotSpd = 100;        // internal status: a pivot <= 0 (matrix not positive definite)
 constexpr int kPS = kNB + 1;        // panel row stride in shared memory (pairs)
 
 constexpr int kSolveThreads = 512;                 // 16 warps: enough to keep the FP32 lanes busy
 constexpr int kSolveWarps = kSolveThreads / 32;
 
+// Cholesky step of the 32 x 32 diagonal block at (c0, c0) of A (row-major, leading
+// dimension F, lower triangle): copied to D in shared memory, factored by one warp (lane =
+// row), written back.  A pivot <= 0 is reported and replaced by 1 so the call finishes.
+__device__ __forceinline__ void chol_diag(DF* A, int F, int c0, DF* D, int32_t* status) {
+  const int tid = threadIdx.x;
+  for (int e = tid; e < kNB * kNB; e += blockDim.x) D[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(c0 + e / kNB) * F + c0 + e % kNB];
+  __syncthreads();
+  if (tid < 32) {
+    for (int j = 0; j < kNB; ++j) {
+      if (tid == j) {
+        const DF d = D[j * kPS + j];
+        if (!(d.hi > 0.f)) report_fit(status, kNotSpd);
+        D[j * kPS + j] = d.hi > 0.f ? df_sqrt(d) : df_make(1.f);
+      }
+      __syncwarp();
+      if (tid > j) D[tid * kPS + j] = df_div(D[tid * kPS + j], D[j * kPS + j]);
+      __syncwarp();
+      if (tid > j)
+        for (int m = j + 1; m <= tid; ++m)
+          D[tid * kPS + m] = df_fma(df_neg(D[tid * kPS + j]), D[m * kPS + j], D[tid * kPS + m]);
+      __syncwarp();
+    }
+  }
+  __syncthreads();
+  for (int e = tid; e < kNB * kNB; e += blockDim.x)
+    if (e % kNB <= e / kNB) A[static_cast<size_t>(c0 + e / kNB) * F + c0 + e % kNB] = D[(e / kNB) * kPS + e % kNB];
+}
+
+// Panel below the diagonal block: every row r in [c0 + 32, F) solves x L_kk^T =
+// A[r][c0 .. c0 + 31] (thread = row), in place; with Pn the rows are also kept in shared
+// memory ([F - c0 - 32][33]).
+__device__ __forceinline__ void chol_panel(DF* A, int F, int c0, const DF* D, DF* Pn) {
+  const int rows = F - c0 - kNB;
+  for (int rr = threadIdx.x; rr < rows; rr += blockDim.x) {
+    DF* arow = A + static_cast<size_t>(c0 + kNB + rr) * F + c0;
+    DF x[kNB];
+#pragma unroll
+    for (int c = 0; c < kNB; ++c) {
+      DF v = arow[c];
+#pragma unroll
+      for (int m = 0; m < c; ++m) v = df_fma(df_neg(x[m]), D[c * kPS + m], v);
+      x[c] = df_div(v, D[c * kPS + c]);
+    }
+#pragma unroll
+    for (int c = 0; c < kNB; ++c) {
+      arow[c] = x[c];
+      if (Pn) Pn[rr * kPS + c] = x[c];
+    }
+  }
+}
+
+// The two triangular solves with the factor L (lower triangle of A, leading dimension F)
+// for 128 right-hand-side columns Z[0 .. F)[0 .. 128) (leading dimension ldz), in place:
+// forward L Y = Z, then backward L^T W = Y, in 32-row blocks.  A block first takes the
+// products with every solved row (thread = 2 rows x 4 columns, 8 independent sums; the
+// solved rows and the block's L entries staged through shared memory 32 at a time), then
+// its 32 x 32 triangle is solved row by row (thread = column).  fsm: [32][33] + [32][128].
+__device__ __forceinline__ void tri_solves(const DF* A, int F, DF* Z, int ldz, DF* fsm) {
+  const int tid = threadIdx.x;
+  constexpr int kR = kNB * kFD / 4 / kSolveThreads;   // rows per thread (2)
+  const int r0 = kR * (tid % (kNB / kR)), q0 = 4 * (tid / (kNB / kR));
+  DF* Ls = fsm;                         // [32][33]: L (forward) or L^T (backward) entries
+  DF* Zs = fsm + kNB * kPS;             // [32][128]: 32 solved rows of Z
+  auto load4 = [&](const DF* p, DF (&v)[4]) {
+    const float4 x = *reinterpret_cast<const float4*>(p), y = *reinterpret_cast<const float4*>(p + 2);
+    v[0] = DF{x.x, x.y};
+    v[1] = DF{x.z, x.w};
+    v[2] = DF{y.x, y.y};
+    v[3] = DF{y.z, y.w};
+  };
+  // acc[a][c] -= sum_j Ls[r0 + a][j] Zs[j][q0 + c] over the staged chunk (Ls indexed
+  // [row][j] when `rows_major`, else [j][row])
+  auto chunk_update = [&](DF (&acc)[kR][4], bool rows_major) {
+#pragma unroll 4
+    for (int j = 0; j < kNB; ++j) {
+      DF z[4], l[kR];
+      load4(&Zs[j * kFD + q0], z);
+#pragma unroll
+      for (int a2 = 0; a2 < kR; ++a2) l[a2] = df_neg(rows_major ? Ls[(r0 + a2) * kPS + j] : Ls[j * kPS + r0 + a2]);
+#pragma unroll
+      for (int a2 = 0; a2 < kR; ++a2)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[a2][c] = df_fma(l[a2], z[c], acc[a2][c]);
+    }
+  };
+  auto stage_z = [&](int m0) {        // 32 rows x 128 pairs, two pairs per thread-step
+    for (int e = tid; e < kNB * kFD / 2; e += blockDim.x)
+      reinterpret_cast<float4*>(Zs)[e] =
+          *reinterpret_cast<const float4*>(Z + static_cast<size_t>(m0 + e / (kFD / 2)) * ldz + 2 * (e % (kFD / 2)));
+  };
+  for (int b0 = 0; b0 < F; b0 += kNB) {
+    DF acc[kR][4];
+#pragma unroll
+    for (int a = 0; a < kR; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * ldz + q0], acc[a]);
+    for (int mc = 0; mc < b0; mc += kNB) {
+      for (int e = tid; e < kNB * kNB; e += blockDim.x)
+        Ls[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(b0 + e / kNB) * F + mc + e % kNB];
+      stage_z(mc);
+      __syncthreads();
+      chunk_update(acc, true);
+      __syncthreads();
+    }
+#pragma unroll
+    for (int a = 0; a < kR; ++a)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * ldz + q0 + c] = acc[a][c];
+    __syncthreads();
+    if (tid < kFD) {
+      for (int i = 0; i < kNB; ++i) {
+        const DF* lrow = A + static_cast<size_t>(b0 + i) * F + b0;
+        DF v = Z[static_cast<size_t>(b0 + i) * ldz + tid];
+        for (int m = 0; m < i; ++m) v = df_fma(df_neg(lrow[m]), Z[static_cast<size_t>(b0 + m) * ldz + tid], v);
+        Z[static_cast<size_t>(b0 + i) * ldz + tid] = df_div(v, lrow[i]);
+      }
+    }
+    __syncthreads();
+  }
+  for (int b0 = F - kNB; b0 >= 0; b0 -= kNB) {
+    DF acc[kR][4];
+#pragma unroll
+    for (int a = 0; a < kR; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * ldz + q0], acc[a]);
+    for (int mc = b0 + kNB; mc < F; mc += kNB) {
+      for (int e = tid; e < kNB * kNB; e += blockDim.x)   // L[mc + j][b0 + i]: entries of L^T
+        Ls[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(mc + e / kNB) * F + b0 + e % kNB];
+      stage_z(mc);
+      __syncthreads();
+      chunk_update(acc, false);
+      __syncthreads();
+    }
+#pragma unroll
+    for (int a = 0; a < kR; ++a)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * ldz + q0 + c] = acc[a][c];
+    __syncthreads();
+    if (tid < kFD) {
+      for (int i = kNB - 1; i >= 0; --i) {
+        DF v = Z[static_cast<size_t>(b0 + i) * ldz + tid];
+        for (int m = i + 1; m < kNB; ++m)
+          v = df_fma(df_neg(A[static_cast<size_t>(b0 + m) * F + b0 + i]), Z[static_cast<size_t>(b0 + m) * ldz + tid], v);
+        Z[static_cast<size_t>(b0 + i) * ldz + tid] = df_div(v, A[static_cast<size_t>(b0 + i) * F + b0 + i]);
+      }
+    }
+    __syncthreads();
+  }
+}
+
+// Per-head systems (F = 128 k <= 512): the whole panel stays in shared memory
+// ([32][33] diagonal block + [F - 32][33] panel).
 __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __grid_constant__ FitParams P) {
   extern __shared__ __align__(16) DF fsm[];
   DF* D = fsm;                                    // [32][33]
@@ -164,47 +321,11 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __gri
     __syncthreads();
     // 2. Cholesky A = L L^T, lower triangle in place, 32-column panels
     for (int c0 = 0; c0 < F; c0 += kNB) {
-      for (int e = tid; e < kNB * kNB; e += blockDim.x) D[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(c0 + e / kNB) * F + c0 + e % kNB];
-      __syncthreads();
-      if (tid < 32) {                             // one warp factors the diagonal block, lane = row
-        for (int j = 0; j < kNB; ++j) {
-          if (tid == j) {
-            const DF d = D[j * kPS + j];
-            if (!(d.hi > 0.f)) report_fit(P.status, kNotSpd);
-            D[j * kPS + j] = d.hi > 0.f ? df_sqrt(d) : df_make(1.f);
-          }
-          __syncwarp();
-          if (tid > j) D[tid * kPS + j] = df_div(D[tid * kPS + j], D[j * kPS + j]);
-          __syncwarp();
-          if (tid > j)
-            for (int m = j + 1; m <= tid; ++m)
-              D[tid * kPS + m] = df_fma(df_neg(D[tid * kPS + j]), D[m * kPS + j], D[tid * kPS + m]);
-          __syncwarp();
-        }
-      }
-      __syncthreads();
-      for (int e = tid; e < kNB * kNB; e += blockDim.x)
-        if (e % kNB <= e / kNB) A[static_cast<size_t>(c0 + e / kNB) * F + c0 + e % kNB] = D[(e / kNB) * kPS + e % kNB];
-      // panel: rows below the diagonal block, P[r] L_kk^T = A[r][c0 .. c0+31]
-      const int rows = F - c0 - kNB;
-      for (int rr = tid; rr < rows; rr += blockDim.x) {
-        DF* arow = A + static_cast<size_t>(c0 + kNB + rr) * F + c0;
-        DF x[kNB];
-#pragma unroll
-        for (int c = 0; c < kNB; ++c) {
-          DF v = arow[c];
-#pragma unroll
-          for (int m = 0; m < c; ++m) v = df_fma(df_neg(x[m]), D[c * kPS + m], v);
-          x[c] = df_div(v, D[c * kPS + c]);
-        }
-#pragma unroll
-        for (int c = 0; c < kNB; ++c) {
-          arow[c] = x[c];
-          Pn[rr * kPS + c] = x[c];
-        }
-      }
+      chol_diag(A, F, c0, D, P.status);
+      chol_panel(A, F, c0, D, Pn);
       __syncthreads();
       // trailing update: A[i][j] -= P[i] . P[j] for c0+32 <= j <= i, in 32 x 32 tiles
+      const int rows = F - c0 - kNB;
       const int nt = rows / kNB;
       for (int tile = 0; tile < nt * (nt + 1) / 2; ++tile) {
         int ti = 0;
@@ -232,95 +353,8 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __gri
       }
       __syncthreads();
     }
-    // 3. forward solve L Y = Z, then backward L^T W = Y, in place on Z, in 32-row blocks:
-    //    first the block's 32 x 128 entries take the products with every solved row (thread
-    //    = 2 rows x 4 right-hand-side columns, 8 independent sums; the solved rows and the
-    //    block's L entries staged through shared memory 32 at a time), then the 32 x 32
-    //    triangle is solved row by row (thread = column).
-    constexpr int kR = kNB * kFD / 4 / kSolveThreads;   // rows per thread (2)
-    const int r0 = kR * (tid % (kNB / kR)), q0 = 4 * (tid / (kNB / kR));
-    DF* Ls = fsm;                         // [32][33]: L (forward) or L^T (backward) entries
-    DF* Zs = fsm + kNB * kPS;             // [32][128]: 32 solved rows of Z
-    auto load4 = [&](const DF* p, DF (&v)[4]) {
-      const float4 x = *reinterpret_cast<const float4*>(p), y = *reinterpret_cast<const float4*>(p + 2);
-      v[0] = DF{x.x, x.y};
-      v[1] = DF{x.z, x.w};
-      v[2] = DF{y.x, y.y};
-      v[3] = DF{y.z, y.w};
-    };
-    // acc[a][c] -= sum_j Ls[r0 + a][j] Zs[j][q0 + c] over the staged chunk (Ls indexed
-    // [row][j] when `rows_major`, else [j][row])
-    auto chunk_update = [&](DF (&acc)[kR][4], bool rows_major) {
-#pragma unroll 4
-      for (int j = 0; j < kNB; ++j) {
-        DF z[4], l[kR];
-        load4(&Zs[j * kFD + q0], z);
-#pragma unroll
-        for (int a2 = 0; a2 < kR; ++a2) l[a2] = df_neg(rows_major ? Ls[(r0 + a2) * kPS + j] : Ls[j * kPS + r0 + a2]);
-#pragma unroll
-        for (int a2 = 0; a2 < kR; ++a2)
-#pragma unroll
-          for (int c = 0; c < 4; ++c) acc[a2][c] = df_fma(l[a2], z[c], acc[a2][c]);
-      }
-    };
-    auto stage_z = [&](int m0) {
-      for (int e = tid; e < kNB * kFD / 2; e += blockDim.x)   // 32 rows x 128 pairs, two per thread-step
-        reinterpret_cast<float4*>(Zs)[e] = reinterpret_cast<const float4*>(Z + static_cast<size_t>(m0) * kFD)[e];
-    };
-    for (int b0 = 0; b0 < F; b0 += kNB) {
-      DF acc[kR][4];
-#pragma unroll
-      for (int a = 0; a < kR; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0], acc[a]);
-      for (int mc = 0; mc < b0; mc += kNB) {
-        for (int e = tid; e < kNB * kNB; e += blockDim.x)
-          Ls[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(b0 + e / kNB) * F + mc + e % kNB];
-        stage_z(mc);
-        __syncthreads();
-        chunk_update(acc, true);
-        __syncthreads();
-      }
-#pragma unroll
-      for (int a = 0; a < kR; ++a)
-#pragma unroll
-        for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0 + c] = acc[a][c];
-      __syncthreads();
-      if (tid < kFD) {
-        for (int i = 0; i < kNB; ++i) {
-          const DF* lrow = A + static_cast<size_t>(b0 + i) * F + b0;
-          DF v = Z[static_cast<size_t>(b0 + i) * kFD + tid];
-          for (int m = 0; m < i; ++m) v = df_fma(df_neg(lrow[m]), Z[static_cast<size_t>(b0 + m) * kFD + tid], v);
-          Z[static_cast<size_t>(b0 + i) * kFD + tid] = df_div(v, lrow[i]);
-        }
-      }
-      __syncthreads();
-    }
-    for (int b0 = F - kNB; b0 >= 0; b0 -= kNB) {
-      DF acc[kR][4];
-#pragma unroll
-      for (int a = 0; a < kR; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0], acc[a]);
-      for (int mc = b0 + kNB; mc < F; mc += kNB) {
-        for (int e = tid; e < kNB * kNB; e += blockDim.x)   // L[mc + j][b0 + i]: entries of L^T
-          Ls[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(mc + e / kNB) * F + b0 + e % kNB];
-        stage_z(mc);
-        __syncthreads();
-        chunk_update(acc, false);
-        __syncthreads();
-      }
-#pragma unroll
-      for (int a = 0; a < kR; ++a)
-#pragma unroll
-        for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * kFD + q0 + c] = acc[a][c];
-      __syncthreads();
-      if (tid < kFD) {
-        for (int i = kNB - 1; i >= 0; --i) {
-          DF v = Z[static_cast<size_t>(b0 + i) * kFD + tid];
-          for (int m = i + 1; m < kNB; ++m)
-            v = df_fma(df_neg(A[static_cast<size_t>(b0 + m) * F + b0 + i]), Z[static_cast<size_t>(b0 + m) * kFD + tid], v);
-          Z[static_cast<size_t>(b0 + i) * kFD + tid] = df_div(v, A[static_cast<size_t>(b0 + i) * F + b0 + i]);
-        }
-      }
-      __syncthreads();
-    }
+    // 3. forward and backward solves for the 128 right-hand sides
+    tri_solves(A, F, Z, kFD, fsm);
     // 4. W (fp32) and b = mean(Y) - mean(X) W (fp64)
     float* Wout = P.W + static_cast<size_t>(sys) * F * kFD;
     for (int64_t e = tid; e < static_cast<int64_t>(F) * kFD; e += blockDim.x) Wout[e] = __fadd_rn(Z[e].hi, Z[e].lo);
@@ -336,22 +370,145 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __gri
   }
 }
 
+// Cross-head systems (Sec. 3.1 with the source feature of Appendix "Run information":
+// d_s = k n_kv d): one system per (target layer, K|V), F = k H 128 features (selected
+// layer-major, head-minor), R = H 128 right-hand sides (every target head of the layer),
+// so X_c^T X_c is formed and factored once per target layer and shared by its heads.
+// The matrix is too large for the panel to stay in shared memory: the trailing update
+// runs in 64 x 64 tiles whose two 64-row panel slices are staged per tile.
+constexpr int kXT = 64;                           // trailing-update tile
+__global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_xh_kernel(const __grid_constant__ FitParams P) {
+  extern __shared__ __align__(16) DF fsm[];
+  DF* D = fsm;                                    // [32][33]
+  DF* Pi = fsm + kNB * kPS;                       // [64][33]: panel rows of the tile's row block
+  DF* Pj = Pi + kXT * kPS;                        // [64][33]: panel rows of its column block
+  const int H = P.H, R = P.R;
+  const int F = P.k * H * kFD;
+  const int tid = threadIdx.x;
+  DF* A = reinterpret_cast<DF*>(P.scratch) +
+          static_cast<size_t>(blockIdx.x) * (static_cast<size_t>(F) * F + static_cast<size_t>(F) * R);
+  DF* Z = A + static_cast<size_t>(F) * F;         // [F][R]
+  const int n_sys = P.Lt * 2;
+  const double inv_n = 1.0 / (static_cast<double>(P.B) * P.T);
+  const DF lam = df_from_double(P.lambda);
+  constexpr size_t kBlk = static_cast<size_t>(kFD) * kFD;
+  for (int sys = blockIdx.x; sys < n_sys; sys += gridDim.x) {
+    const int kv = sys & 1;
+    const int l = sys >> 1;
+    // 1. A = Xc^T Xc + lambda I (lower triangle) from the source-pair blocks, Z = Xc^T Yc
+    for (int64_t e = tid; e < static_cast<int64_t>(F) * F; e += blockDim.x) {
+      const int r = static_cast<int>(e / F), c = static_cast<int>(e % F);
+      if (c > r) continue;
+      const int ur = r / kFD, uc = c / kFD;       // feature blocks (layer j, head x), ur >= uc
+      const int bi = ur / H, bj = uc / H;
+      int hr = ur % H, hc = uc % H, er = r % kFD, ec = c % kFD;
+      const int pr = __ldg(&P.pair_of[(l * P.k + bi) * P.k + bj]);
+      const int q = pr >= 0 ? pr : -1 - pr;
+      if (pr < 0) {                               // stored as (sel[bj], sel[bi]): transpose
+        const int t = hr; hr = hc; hc = t;
+        const int u = er; er = ec; ec = u;
+      }
+      if (hr < hc && __ldg(&P.pairs[2 * q]) == __ldg(&P.pairs[2 * q + 1])) {   // one layer: only hr >= hc stored
+        const int t = hr; hr = hc; hc = t;
+        const int u = er; er = ec; ec = u;
+      }
+      const float g = P.gram[(((static_cast<size_t>(q) * 2 + kv) * H + hr) * H + hc) * kBlk +
+                             static_cast<size_t>(er) * kFD + ec];
+      A[e] = r == c ? df_add(df_make(g), lam) : df_make(g);
+    }
+    for (int64_t e = tid; e < static_cast<int64_t>(F) * R; e += blockDim.x) {
+      const int r = static_cast<int>(e / R), col = static_cast<int>(e % R);
+      const int u = r / kFD, ht = col / kFD;      // u = bi * H + x
+      Z[e] = df_make(P.xty[((((static_cast<size_t>(l) * 2 + kv) * P.k * H + u) * H + ht)) * kBlk +
+                           static_cast<size_t>(r % kFD) * kFD + col % kFD]);
+    }
+    __syncthreads();
+    // 2. Cholesky, 32-column panels; trailing update in 64 x 64 tiles of the lower triangle
+    for (int c0 = 0; c0 < F; c0 += kNB) {
+      chol_diag(A, F, c0, D, P.status);
+      chol_panel(A, F, c0, D, nullptr);
+      __syncthreads();
+      const int base = c0 + kNB, rows = F - base;
+      const int nt = (rows + kXT - 1) / kXT;
+      // thread: column jj = tid % 64 of the tile, rows ii + 8q (ii = tid / 64), q < 8
+      const int jj = tid % kXT, ii = tid / kXT;
+      for (int tile = 0; tile < nt * (nt + 1) / 2; ++tile) {
+        int ti = 0;
+        while ((ti + 1) * (ti + 2) / 2 <= tile) ++ti;
+        const int tj = tile - ti * (ti + 1) / 2;
+        for (int e = tid; e < 2 * kXT * kNB; e += blockDim.x) {
+          const int s = e / (kXT * kNB), rr = (e / kNB) % kXT, m = e % kNB;
+          const int row = (s == 0 ? ti : tj) * kXT + rr;
+          (s == 0 ? Pi : Pj)[rr * kPS + m] = row < rows ? A[static_cast<size_t>(base + row) * F + c0 + m] : df_make(0.f);
+        }
+        __syncthreads();
+        constexpr int kQ = kXT * kXT / kSolveThreads;   // 8
+        DF sacc[kQ];
+#pragma unroll
+        for (int q = 0; q < kQ; ++q) sacc[q] = df_make(0.f);
+#pragma unroll 4
+        for (int m = 0; m < kNB; ++m) {
+          const DF pj = Pj[jj * kPS + m];
+#pragma unroll
+          for (int q = 0; q < kQ; ++q) sacc[q] = df_fma(Pi[(ii + 8 * q) * kPS + m], pj, sacc[q]);
+        }
+        const int gj = tj * kXT + jj;
+#pragma unroll
+        for (int q = 0; q < kQ; ++q) {
+          const int gi = ti * kXT + ii + 8 * q;
+          if (gi < rows && gj <= gi) {
+            DF* a = A + static_cast<size_t>(base + gi) * F + base + gj;
+            *a = df_add(*a, df_neg(sacc[q]));
+          }
+        }
+        __syncthreads();
+      }
+    }
+    // 3. forward and backward solves, 128 right-hand sides (one target head) at a time
+    for (int c0 = 0; c0 < R; c0 += kFD) tri_solves(A, F, Z + c0, R, fsm);
+    // 4. W (fp32, [L_t][2][H][F][128]) and b = mean(Y) - mean(X) W (fp64)
+    for (int64_t e = tid; e < static_cast<int64_t>(F) * R; e += blockDim.x) {
+      const int r = static_cast<int>(e / R), col = static_cast<int>(e % R);
+      P.W[((static_cast<size_t>(sys) * H + col / kFD) * F + r) * kFD + col % kFD] = __fadd_rn(Z[e].hi, Z[e].lo);
+    }
+    for (int col = tid; col < R; col += blockDim.x) {
+      const int ht = col / kFD, c = col % kFD;
+      double acc = P.sums[sums_index(P, 1, kv, l, ht) + c] * inv_n;
+      for (int r = 0; r < F; ++r) {
+        const int u = r / kFD;
+        const int layer = __ldg(&P.sel[l * P.k + u / H]);
+        acc -= P.sums[sums_index(P, 0, kv, layer, u % H) + r % kFD] * inv_n * df_to_double(Z[static_cast<size_t>(r) * R + col]);
+      }
+      P.b[(static_cast<size_t>(sys) * H + ht) * kFD + c] = static_cast<float>(acc);
+    }
+    __syncthreads();
+  }
+}
+
 // Host plan of a fit: the distinct source pairs, the block tables, the operand slots and
 // the sizes of every device piece (the same for the run and the workspace query).
 struct FitPlan {
   std::vector<int32_t> pair_list, pair_of, tab, slot_of_src;
-  int n_pairs = 0, solve_grid = 0, F = 0;
+  int n_pairs = 0, solve_grid = 0, F = 0, R = 0;
+  bool cross = false;
   size_t n_sys = 0, sums_n = 0, gram_n = 0, xty_n = 0, scratch_n = 0, sel_n = 0, n_blocks = 0;
   size_t fixed_bytes = 0;          // sums, scratch, blocks, tables, status (256-aligned pieces)
 };
 
 size_t al256(size_t n) { return (n + 255) / 256 * 256; }
 
+// Bytes of per-CTA solve scratch the cross-head fit may take (the grid shrinks beyond it).
+constexpr size_t kXhScratchCap = static_cast<size_t>(80) << 30;
+
 FitPlan plan_fit(const kvx_fit_config* cfg, int sms, GramSpec* G) {
   FitPlan p;
   const int kk = cfg->k;
-  p.F = kk * kFD;
-  p.n_sys = static_cast<size_t>(cfg->tgt_layers) * 2 * cfg->n_kv_heads;
+  const bool cross = cfg->head_mix == KVX_CROSS_HEAD;
+  const int H = cfg->n_kv_heads;
+  p.cross = cross;
+  p.F = kk * kFD * (cross ? H : 1);
+  p.R = cross ? H * kFD : kFD;
+  p.n_sys = static_cast<size_t>(cfg->tgt_layers) * 2 * (cross ? 1 : H);
   p.sums_n = static_cast<size_t>(2) * (cfg->src_layers + cfg->tgt_layers) * cfg->n_kv_heads * kFD;
   p.pair_of.assign(static_cast<size_t>(cfg->tgt_layers) * kk * kk, -1);
   std::vector<int32_t> index(static_cast<size_t>(cfg->src_layers) * cfg->src_layers, -1);
@@ -373,10 +530,14 @@ FitPlan plan_fit(const kvx_fit_config* cfg, int sms, GramSpec* G) {
         p.pair_of[(static_cast<size_t>(l) * kk + bi) * kk + bj] = ia == bi ? idx : -1 - idx;
       }
   p.n_pairs = static_cast<int>(p.pair_list.size() / 2);
-  p.gram_n = static_cast<size_t>(2) * cfg->n_kv_heads * p.n_pairs * kFD * kFD;
-  p.xty_n = p.n_sys * kk * kFD * kFD;
+  const size_t kBlk = static_cast<size_t>(kFD) * kFD;
+  p.gram_n = static_cast<size_t>(2) * H * (cross ? H : 1) * p.n_pairs * kBlk;
+  p.xty_n = static_cast<size_t>(cfg->tgt_layers) * 2 * H * kk * (cross ? H : 1) * kBlk;
   p.solve_grid = static_cast<int>(std::min<size_t>(p.n_sys, static_cast<size_t>(std::max(sms, 1))));
-  p.scratch_n = static_cast<size_t>(p.solve_grid) * (static_cast<size_t>(p.F) * p.F + static_cast<size_t>(p.F) * kFD);
+  const size_t per_cta = static_cast<size_t>(p.F) * p.F + static_cast<size_t>(p.F) * p.R;
+  if (cross)
+    p.solve_grid = static_cast<int>(std::max<size_t>(1, std::min<size_t>(p.solve_grid, kXhScratchCap / (per_cta * 8))));
+  p.scratch_n = static_cast<size_t>(p.solve_grid) * per_cta;
   p.sel_n = static_cast<size_t>(cfg->tgt_layers) * kk;
   p.tab.assign(cfg->selection, cfg->selection + p.sel_n);
   p.tab.insert(p.tab.end(), p.pair_list.begin(), p.pair_list.end());
@@ -397,7 +558,13 @@ FitPlan plan_fit(const kvx_fit_config* cfg, int sms, GramSpec* G) {
     G->slot_layer.push_back(l);
   }
   G->H = cfg->n_kv_heads;
-  p.n_blocks = static_cast<size_t>(2) * cfg->n_kv_heads * (p.n_pairs + p.sel_n);
+  if (cross) {   // per (pair, K|V): H x H head blocks (one layer: row head >= column head); cross: k H H per (l, K|V)
+    size_t nb = 0;
+    for (int q = 0; q < p.n_pairs; ++q) nb += p.pair_list[2 * q] == p.pair_list[2 * q + 1] ? H * (H + 1) / 2 : H * H;
+    p.n_blocks = 2 * nb + static_cast<size_t>(2) * cfg->tgt_layers * kk * H * H;
+  } else {
+    p.n_blocks = static_cast<size_t>(2) * cfg->n_kv_heads * (p.n_pairs + p.sel_n);
+  }
   p.fixed_bytes = al256(p.sums_n * 8) + al256(p.scratch_n * 8) + al256((p.gram_n + p.xty_n) * 4) +
                   al256(p.tab.size() * 4 + 4) + gram_fixed_bytes(*G, p.n_blocks);
   return p;
@@ -406,7 +573,11 @@ FitPlan plan_fit(const kvx_fit_config* cfg, int sms, GramSpec* G) {
 const char* check_fit_config(const kvx_fit_config* cfg) {
   if (!cfg) return "NULL argument";
   if (cfg->head_dim != kFD) return "head_dim must be 128";
-  if (cfg->k < 1 || cfg->k > 4) return "k must be in [1, 4]";
+  if (cfg->head_mix != KVX_PER_HEAD && cfg->head_mix != KVX_CROSS_HEAD) return "bad head_mix";
+  if (cfg->head_mix == KVX_PER_HEAD && (cfg->k < 1 || cfg->k > 4)) return "k must be in [1, 4] (per head)";
+  if (cfg->head_mix == KVX_CROSS_HEAD &&
+      (cfg->k < 1 || static_cast<int64_t>(cfg->k) * cfg->n_kv_heads * kFD > kMaxXhFeatures))
+    return "k * n_kv_heads * 128 must be in [128, 16384] (cross-head)";
   if (cfg->src_layers < 1 || cfg->tgt_layers < 1 || cfg->n_kv_heads < 1 || cfg->k > cfg->src_layers)
     return "layer / head counts out of range";
   if (!(cfg->lambda >= 0.0) || !(cfg->src_rope_theta > 1.0) || !(cfg->tgt_rope_theta > 1.0))
@@ -526,6 +697,7 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
   P.W = W;
   P.b = b;
   P.lambda = cfg->lambda;
+  P.R = pl.R;
   P.n_pairs = pl.n_pairs;
   P.sums = reinterpret_cast<double*>(S.take(pl.sums_n * 8));
   P.scratch = reinterpret_cast<double*>(S.take(pl.scratch_n * 8));
@@ -553,7 +725,33 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
     const int32_t tslot0 = static_cast<int32_t>(G.slot_side.size()) - cfg->tgt_layers;
     std::vector<GramBlock> blocks;
     blocks.reserve(pl.n_blocks);
-    for (int kv = 0; kv < 2; ++kv)
+    const int H = cfg->n_kv_heads;
+    const size_t kBlk = static_cast<size_t>(kFD) * kFD;
+    if (pl.cross) {
+      for (int q = 0; q < pl.n_pairs; ++q) {
+        const int sa = pl.pair_list[2 * q], sb = pl.pair_list[2 * q + 1];
+        for (int kv = 0; kv < 2; ++kv)
+          for (int x = 0; x < H; ++x)
+            for (int y = 0; y < H; ++y) {
+              if (sa == sb && x < y) continue;
+              GramBlock g{pl.slot_of_src[sa], pl.slot_of_src[sb], kv, x,
+                          P.gram + (((static_cast<size_t>(q) * 2 + kv) * H + x) * H + y) * kBlk};
+              g.hb = y;
+              blocks.push_back(g);
+            }
+      }
+      for (int l = 0; l < cfg->tgt_layers; ++l)
+        for (int kv = 0; kv < 2; ++kv)
+          for (int bi = 0; bi < kk; ++bi)
+            for (int x = 0; x < H; ++x)
+              for (int ht = 0; ht < H; ++ht) {
+                GramBlock g{pl.slot_of_src[cfg->selection[l * kk + bi]], tslot0 + l, kv, x,
+                            P.xty + ((((static_cast<size_t>(l) * 2 + kv) * kk + bi) * H + x) * H + ht) * kBlk};
+                g.hb = ht;
+                blocks.push_back(g);
+              }
+    }
+    for (int kv = 0; kv < 2 && !pl.cross; ++kv)
       for (int h = 0; h < cfg->n_kv_heads; ++h) {
         for (int q = 0; q < pl.n_pairs; ++q)
           blocks.push_back(GramBlock{pl.slot_of_src[pl.pair_list[2 * q]], pl.slot_of_src[pl.pair_list[2 * q + 1]], kv,
@@ -581,17 +779,20 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
       set_error(std::string("kvx_fit_ridge: ") + kvx_last_error());
       break;
     }
-    // the factorisation's diagonal block and panel, or the solves' staged chunk
-    const size_t smem = std::max(static_cast<size_t>(kNB) * kPS + static_cast<size_t>(pl.F - kNB) * kPS,
-                                 static_cast<size_t>(kNB) * kPS + static_cast<size_t>(kNB) * kFD) * 8;
-    if ((e = cudaFuncSetAttribute(fit_solve_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem))) !=
+    // the factorisation's diagonal block and panel (per head) or tile slices (cross-head),
+    // or the solves' staged chunk
+    const size_t fact = pl.cross ? static_cast<size_t>(kNB + 2 * kXT) * kPS
+                                 : static_cast<size_t>(kNB) * kPS + static_cast<size_t>(pl.F - kNB) * kPS;
+    const size_t smem = std::max(fact, static_cast<size_t>(kNB) * kPS + static_cast<size_t>(kNB) * kFD) * 8;
+    auto kernel = pl.cross ? fit_solve_xh_kernel : fit_solve_kernel;
+    if ((e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem))) !=
         cudaSuccess) {
       set_error(std::string("kvx_fit_ridge: smem attribute: ") + cudaGetErrorString(e));
       result = KVX_ERR_CUDA;
       break;
     }
     timer.begin(3);
-    fit_solve_kernel<<<pl.solve_grid, kSolveThreads, smem, st>>>(P);
+    kernel<<<pl.solve_grid, kSolveThreads, smem, st>>>(P);
     timer.end();
     if ((e = cudaGetLastError()) != cudaSuccess) {
       set_error(std::string("kvx_fit_ridge: launch: ") + cudaGetErrorString(e));

@@ -648,7 +648,8 @@ kvx_status gram_blocks(const GramSpec& spec, const std::vector<GramBlock>& block
     if (p.kv != q.kv) return p.kv < q.kv;
     if (p.h != q.h) return p.h < q.h;
     if (p.a_slot != q.a_slot) return p.a_slot < q.a_slot;
-    return p.b_slot < q.b_slot;
+    if (p.b_slot != q.b_slot) return p.b_slot < q.b_slot;
+    return p.hb < q.hb;
   });
   auto row_of = [&](int slot, int kv, int h) {
     return static_cast<int32_t>(((static_cast<int64_t>(slot) * 2 + kv) * spec.H + h) * 2 * kGD);
@@ -658,14 +659,14 @@ kvx_status gram_blocks(const GramSpec& spec, const std::vector<GramBlock>& block
     const GramBlock& p = blocks[order[i]];
     GramUnit u{};
     u.a_row = row_of(p.a_slot, p.kv, p.h);
-    u.b_row0 = row_of(p.b_slot, p.kv, p.h);
+    u.b_row0 = row_of(p.b_slot, p.kv, p.hb < 0 ? p.h : p.hb);
     u.b_row1 = -1;
     u.out0 = p.out;
     u.out1 = nullptr;
     if (i + 1 < order.size()) {
       const GramBlock& q = blocks[order[i + 1]];
       if (q.kv == p.kv && q.h == p.h && q.a_slot == p.a_slot) {
-        u.b_row1 = row_of(q.b_slot, q.kv, q.h);
+        u.b_row1 = row_of(q.b_slot, q.kv, q.hb < 0 ? q.h : q.hb);
         u.out1 = q.out;
         ++i;
       }

@@ -32,10 +32,12 @@ struct GramSpec {
   int sm_count = 0;
 };
 
-// One 128 x 128 block out[i][j] = sum_n A[n][i] B[n][j] of two centred operands (slots).
+// One 128 x 128 block out[i][j] = sum_n A[n][i] B[n][j] of two centred operands (slots):
+// A is head h of slot a_slot, B head hb of slot b_slot (hb < 0: the same head h).
 struct GramBlock {
   int32_t a_slot, b_slot, kv, h;
   float* out;                       // device, fp32 row-major
+  int32_t hb = -1;
 };
 
 // Device time of the phases of one offline call (fit or probe), from CUDA events on the

@@ -227,3 +227,92 @@ def test_fit_hf_rope_numerics():
                 rel = 8.0 * kappa * (N * 2.0 ** -24 + 2.0 ** -16)
                 err = np.max(np.abs(Wg[l, kv, h] - Wr))
                 assert err <= rel * np.max(np.abs(Wr)), (l, kv, h, err, rel * np.max(np.abs(Wr)))
+
+
+# ------------------------------------------------------------ cross-head fit -----
+
+def _run_fit_xh(w, lam, sel):
+    """kvx_fit_ridge with head_mix = KVX_CROSS_HEAD; W [L_t][2][H][k H d][d], b [L_t][2][H][d]."""
+    dev = torch.device("cuda:0")
+    sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+    tk, tv = syn.target_cache(w, 0, device=dev), syn.target_cache(w, 1, device=dev)
+    pos = syn.positions(w)
+    posd = torch.from_numpy(pos).to(dev)
+    F = w.k * w.H * w.d
+    W = torch.full((w.Lt, 2, w.H, F, w.d), float("nan"), dtype=torch.float32, device=dev)
+    b = torch.full((w.Lt, 2, w.H, w.d), float("nan"), dtype=torch.float32, device=dev)
+    kvx.kvx_fit_ridge(w.Ls, w.Lt, w.H, w.d, w.k, w.theta_s, w.theta_t, lam, sel,
+                      kvx.src_from_tensors(sk, sv), kvx.src_from_tensors(tk, tv), w.B, w.T,
+                      posd.data_ptr(), W.data_ptr(), b.data_ptr(), torch.cuda.current_stream().cuda_stream,
+                      head_mix=kvx.KVX_CROSS_HEAD)
+    return (sk, sv, tk, tv, pos), W.cpu().double().numpy(), b.cpu().double().numpy()
+
+
+def _check_xh_systems(w, lam, sel, caches, Wg, bg, systems):
+    """systems: (l, kv).  The oracle's fit of the paper's cross-head feature (every KV head of
+    the k selected layers, oracle.mlp.cross_head_features) against every target head of
+    layer l at once; every head's W and b within the kappa-scaled bound of the module
+    docstring."""
+    from oracle import mlp as omlp
+    sk, sv, tk, tv, pos = caches
+    N = w.B * w.T
+    p = pos.reshape(-1)
+    def raw(cache, j):          # layer j of a [L][B][H][T][d] cache as float64 [H][N][d], as stored
+        x = _f64(cache[j])
+        return x.transpose(1, 0, 2, 3).reshape(w.H, N, w.d)
+
+    for (l, kv) in systems:
+        src = {j: raw(sk if kv == 0 else sv, j) for j in set(sel[l].tolist())}
+        X = omlp.cross_head_features(src, l, sel, kv, p, w.theta_s)                    # keys stripped
+        yt = _features(w, (tk if kv == 0 else tv)[l:l + 1], kv, w.theta_t, pos)[0]     # [H][N][d]
+        Y = np.concatenate(list(yt), axis=-1)                                          # [N][H d], head-minor
+        Wr, br = oridge.fit_ridge(X, Y, lam)
+        Xc = X - X.mean(axis=0)
+        ev = np.linalg.eigvalsh(Xc.T @ Xc + lam * np.eye(X.shape[1]))
+        kappa = ev[-1] / ev[0]
+        rel = 8.0 * kappa * (N * 2.0 ** -24 + 2.0 ** -16)
+        for h in range(w.H):
+            wr, b_r = Wr[:, h * w.d:(h + 1) * w.d], br[h * w.d:(h + 1) * w.d]
+            errW = np.max(np.abs(Wg[l, kv, h] - wr))
+            assert errW <= rel * np.max(np.abs(wr)), \
+                "W (%d,%d,%d): err %.3g > %.3g (kappa %.3g)" % (l, kv, h, errW, rel * np.max(np.abs(wr)), kappa)
+            bscale = np.max(np.abs(b_r)) + np.max(np.abs(X.mean(axis=0))) * np.sum(np.abs(wr), axis=0).max()
+            errb = np.max(np.abs(bg[l, kv, h] - b_r))
+            assert errb <= rel * bscale, "b (%d,%d,%d): err %.3g > %.3g" % (l, kv, h, errb, rel * bscale)
+
+
+@pytest.mark.parametrize("over,lam", [
+    (dict(Ls=4, Lt=3, H=2, B=2, T=300, k=2), 0.01),                 # B > 1, ragged tiles, F = 512
+    (dict(Ls=5, Lt=2, H=3, B=1, T=900, k=2, theta_t=5e5), 1.0),     # odd head count, F = 768, larger lambda
+    (dict(Ls=6, Lt=2, H=2, B=1, T=640, k=3), 0.01),                 # F = 768 > N: lambda keeps it SPD
+])
+def test_fit_cross_head_small_every_system(over, lam):
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4_xhead", **over)
+    sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
+    caches, Wg, bg = _run_fit_xh(w, lam, sel)
+    assert np.all(np.isfinite(Wg)) and np.all(np.isfinite(bg)), "unwritten outputs"
+    _check_xh_systems(w, lam, sel, caches, Wg, bg, [(l, kv) for l in range(w.Lt) for kv in range(2)])
+
+
+def test_fit_cross_head_one_head_equals_per_head():
+    """With one KV head the cross-head feature is the per-head one: both modes of the GPU fit
+    solve the same systems (different kernels), so they agree within the fit bound."""
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=4, Lt=3, H=1, B=1, T=700, k=3)
+    sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
+    caches, Wp, bp = _run_fit(w, 0.01, sel)
+    _, Wx, bx = _run_fit_xh(w, 0.01, sel)
+    scale = np.max(np.abs(Wp))
+    assert np.max(np.abs(Wx - Wp)) <= 1e-3 * scale, np.max(np.abs(Wx - Wp)) / scale
+    _check_xh_systems(w, 0.01, sel, caches, Wx, bx, [(0, 0), (2, 1)])
+
+
+def test_fit_cross_head_qwen_shapes_sampled():
+    """Qwen3-14B -> 32B layer and head counts, k = 4 (d_s = k n_kv d = 4096, the paper's source
+    feature), 8192 calibration tokens: all 128 (layer, K|V) systems fitted on the GPU, three
+    checked against the oracle on every target head."""
+    w = syn.workload("qwen3_14b_32b_t32768_k4_xhead", T=8192)
+    sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
+    caches, Wg, bg = _run_fit_xh(w, 0.01, sel)
+    assert np.all(np.isfinite(Wg)) and np.all(np.isfinite(bg))
+    _check_xh_systems(w, 0.01, sel, caches, Wg, bg, [(0, 0), (33, 1), (63, 0)])
+    torch.cuda.empty_cache()
