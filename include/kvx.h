@@ -220,6 +220,19 @@ KVX_API kvx_status kvx_set_kernel(kvx_ctx* ctx, int32_t kernel);
  * device-detected error since the last call) and reset it to KVX_OK. */
 KVX_API kvx_status kvx_get_status(kvx_ctx* ctx, void* stream);
 
+/* Test switch of the bounded waits (the paper has no counterpart).  Every wait of the
+ * per-head tensor-core kernel gives up after 4 s, sets KVX_ERR_TIMEOUT in the status word
+ * and makes the kernel drain its copies and MMAs in flight, free its tensor memory and
+ * return.  A test exercises that path on a healthy GPU with this call:
+ *   wait_limit_ns  the bound of every wait of later kvx_map calls on ctx, in [1 ms, 4 s],
+ *                  or 0 for the default 4 s;
+ *   skip_bias_row  >= 0: the first CTA of later launches never loads its bias row of this
+ *                  index (the skip_bias_row-th (layer, unit) bias row it walks), so the
+ *                  epilogue's wait for it runs out and the launch ends with
+ *                  KVX_ERR_TIMEOUT in the status word; -1: off.
+ * INVALID_ARG for a NULL ctx or values outside those ranges.  Not for production use. */
+KVX_API kvx_status kvx_set_test_wait(kvx_ctx* ctx, uint64_t wait_limit_ns, int64_t skip_bias_row);
+
 /* Mapper size in parameters, K plus V (Appendix C, "Serving cost"):
  * CROSS_HEAD 2 L_t n_kv (k n_kv d) d;  PER_HEAD 2 L_t n_kv (k d) d.  -1 on bad input. */
 KVX_API int64_t kvx_mapper_params(int32_t tgt_layers, int32_t n_kv_heads, int32_t head_dim, int32_t k,
@@ -236,7 +249,16 @@ KVX_API int64_t kvx_mapper_params(int32_t tgt_layers, int32_t n_kv_heads, int32_
  * [L_t][B][H][T][d] of the same tokens (kvx_src layout, bf16, d = 128, 16-byte aligned);
  * `positions` device [batch][tokens_per_seq].  `selection` (host [L_t][k], 1 <= k <= 4)
  * as in kvx_config.  Outputs on the device, fp32: W [L_t][2][H][k*d][d] and
- * b [L_t][2][H][d] (the kvx_config layouts).  Cross-products of the centred values run
+ * b [L_t][2][H][d] (the kvx_config layouts).
+ * With head_mix = KVX_CROSS_HEAD the feature is the paper's cross-head concatenation
+ * (Sec. 3.1; Appendix "Run information", source-feature row: d_s = k * n_kv * d): X holds
+ * every KV head of the k selected layers (layer-major, head-minor) and is shared by all
+ * target heads of layer l, so each (l, K|V) is one system (Xc^T Xc + lambda I) W_l =
+ * Xc^T Yc_l with F = k*H*128 unknowns and H*128 right-hand sides (Xc^T Xc formed and
+ * factored once per target layer, shared across its heads, Sec. 3.1); W is written as
+ * [L_t][2][H][k*H*d][d] (k >= 1, k*H*128 <= 16384).  The solve scratch is F*(F + H*128)
+ * float pairs per concurrent system (at most 80 GB; beyond that fewer systems run at
+ * once).  Cross-products of the centred values run
  * on the tensor cores from a bf16 hi + lo split of each value (within 2^-17 of it) and
  * accumulate in fp32; the factorisation and the solves run in float-float arithmetic (each
  * value an unevaluated sum of two fp32 numbers, about 48 significant bits) on the FP32
@@ -260,6 +282,7 @@ typedef struct {
   const kvx_rope_scaling* src_rope_scaling;   /* NULL: plain theta (see kvx_rope_scaling) */
   const kvx_rope_scaling* tgt_rope_scaling;
   int32_t rope_numerics;        /* kvx_rope_numerics: the strip of both sides' keys */
+  int32_t head_mix;             /* kvx_head_mix: KVX_PER_HEAD (0) or KVX_CROSS_HEAD */
 } kvx_fit_config;
 KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, const kvx_src* tgt, int32_t batch,
                                  int32_t tokens_per_seq, const int32_t* positions, float* W, float* b,

@@ -329,6 +329,18 @@ kvx_status kvx_set_kernel(kvx_ctx* ctx, int32_t kernel) {
   return KVX_OK;
 }
 
+kvx_status kvx_set_test_wait(kvx_ctx* ctx, uint64_t wait_limit_ns, int64_t skip_bias_row) {
+  g_last_error.clear();
+  if (!ctx) return fail(KVX_ERR_INVALID_ARG, "kvx_set_test_wait: NULL ctx");
+  if (wait_limit_ns != 0 && (wait_limit_ns < 1000000ull || wait_limit_ns > 4000000000ull))
+    return fail(KVX_ERR_INVALID_ARG, "kvx_set_test_wait: wait limit outside [1 ms, 4 s]");
+  if (skip_bias_row < -1 || skip_bias_row > INT32_MAX)
+    return fail(KVX_ERR_INVALID_ARG, "kvx_set_test_wait: skip_bias_row must be -1 or a row index");
+  ctx->wait_limit_ns = wait_limit_ns;
+  ctx->skip_bias_row = skip_bias_row;
+  return KVX_OK;
+}
+
 kvx_status kvx_get_status(kvx_ctx* ctx, void* stream) {
   g_last_error.clear();
   if (!ctx) return fail(KVX_ERR_INVALID_ARG, "kvx_get_status: NULL ctx");

@@ -89,6 +89,10 @@ struct kvx_ctx {
   size_t ws_bytes = 0;
   kvx::TcPlan plan;
   int sm_count = 0;
+  // test switches (kvx_set_test_wait): the per-head tensor-core kernel's wait bound, and a
+  // bias row its first CTA never loads, which makes one of its waits run out
+  uint64_t wait_limit_ns = 0;        // 0: the default bound
+  int64_t skip_bias_row = -1;
 };
 
 namespace kvx {

@@ -68,7 +68,7 @@ __device__ __forceinline__ uint64_t global_timer() {
 // the wait ran out (then it raises KVX_ERR_TIMEOUT and the shared abort flag) or if
 // another role raised the abort flag.
 __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile uint32_t* abort_flag,
-                                         int32_t* status, int32_t timeout_code) {
+                                         int32_t* status, int32_t timeout_code, uint64_t limit_ns = kTimeoutNs) {
   if (mbar_try_wait(bar, parity)) return true;
   uint64_t t0 = 0;
   for (uint32_t it = 1;; ++it) {
@@ -78,7 +78,7 @@ __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile
       const uint64_t now = global_timer();
       if (t0 == 0) {
         t0 = now;
-      } else if (now - t0 > kTimeoutNs) {
+      } else if (now - t0 > limit_ns) {
         *abort_flag = 1u;
         atomicCAS(status, 0, timeout_code);
         return false;
@@ -88,10 +88,10 @@ __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile
 }
 
 // Teardown wait: ignores the abort flag, still bounded in time.
-__device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
+__device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity, uint64_t limit_ns = kTimeoutNs) {
   const uint64_t t0 = global_timer();
   while (!mbar_try_wait(bar, parity))
-    if (global_timer() - t0 > kTimeoutNs) break;
+    if (global_timer() - t0 > limit_ns) break;
 }
 
 // ------------------------------------------------------------------------ TMA ----

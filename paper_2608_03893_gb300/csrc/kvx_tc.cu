@@ -144,6 +144,8 @@ struct TcParams {
   int32_t Lt, H, k, n_loads, tiles_per_seq, n_units;   // tiles_per_seq / n_units count pairs of token tiles
   int32_t out_bh;        // TMA-store head coordinate: 0 none (direct stores), 1 h (B = 1), 2 b*H + h
   RopeTables rope;
+  uint64_t timeout_ns;   // bound of every wait (kTimeoutNs unless a test shortens it)
+  int32_t skip_bias;     // test only: CTA 0 never loads its bias row of this index (-1: none)
 };
 
 struct Unit {
@@ -264,6 +266,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       bool ok = true;
       uint64_t t_idle = 0;
       uint32_t spins = 0;
+      // a test's planted fault: this bias row is never loaded, so the epilogue's wait for
+      // it runs out and the whole kernel takes its abort path
+      const int64_t skip = blockIdx.x == 0 ? P.skip_bias : -1;
       for (;;) {
         bool busy = false, progress = false;
         if (su < n_units && P.n_loads > 0) {
@@ -292,9 +297,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const uint32_t round = bn / kBiasSlots;
           if (round == 0 || mbar_test_wait(smem_u32(&bias_empty[bs]), (round - 1) & 1u)) {
             const int row0 = ((blay * 2 + bun.kv) * H + bun.h) * kD;
-            mbar_expect_tx(smem_u32(&bias_full[bs]), kBiasBytes);
-            bulk_load(smem_u32(bias_ring + bs * kD), P.bias + static_cast<size_t>(row0), kBiasBytes,
-                      smem_u32(&bias_full[bs]));
+            if (static_cast<int64_t>(bn) != skip) {
+              mbar_expect_tx(smem_u32(&bias_full[bs]), kBiasBytes);
+              bulk_load(smem_u32(bias_ring + bs * kD), P.bias + static_cast<size_t>(row0), kBiasBytes,
+                        smem_u32(&bias_full[bs]));
+            }
             ++bn;
             if (++blay == Lt) {
               blay = 0;
@@ -318,7 +325,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const uint64_t now = global_timer();
           if (t_idle == 0) {
             t_idle = now;
-          } else if (now - t_idle > kTimeoutNs) {
+          } else if (now - t_idle > P.timeout_ns) {
             *abort_flag = 1u;
             report(P.status, KVX_ERR_TIMEOUT);
             ok = false;
@@ -328,9 +335,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       }
       if (!ok) {   // the most recent loads and bias rows may still be landing
         const uint32_t first = gl > static_cast<uint32_t>(kLand) ? gl - kLand : 0;
-        for (uint32_t i = first; i < gl; ++i) drain_wait(smem_u32(&land_full[i % kLand]), (i / kLand) & 1u);
+        for (uint32_t i = first; i < gl; ++i)
+          drain_wait(smem_u32(&land_full[i % kLand]), (i / kLand) & 1u, P.timeout_ns);
         const uint32_t bfirst = bn > static_cast<uint32_t>(kBiasSlots) ? bn - kBiasSlots : 0;
-        for (uint32_t i = bfirst; i < bn; ++i) drain_wait(smem_u32(&bias_full[i % kBiasSlots]), (i / kBiasSlots) & 1u);
+        for (uint32_t i = bfirst; i < bn; ++i)
+          if (static_cast<int64_t>(i) != skip)
+            drain_wait(smem_u32(&bias_full[i % kBiasSlots]), (i / kBiasSlots) & 1u, P.timeout_ns);
       }
     }
   } else if (warp == 2) {
@@ -409,7 +419,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const uint64_t now = global_timer();
           if (t_idle == 0) {
             t_idle = now;
-          } else if (now - t_idle > kTimeoutNs) {
+          } else if (now - t_idle > P.timeout_ns) {
             *abort_flag = 1u;
             report(P.status, KVX_ERR_TIMEOUT);
             ok = false;
@@ -420,7 +430,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       if (!ok && rank == 0) {   // the most recent fills of each ring (both CTAs' halves) may still be landing
         for (int r = 0; r < kIssuers; ++r) {
           const uint32_t first = wn[r] > static_cast<uint32_t>(kRing) ? wn[r] - kRing : 0;
-          for (uint32_t i = first; i < wn[r]; ++i) drain_wait(smem_u32(&wfull[r * kRing + i % kRing]), (i / kRing) & 1u);
+          for (uint32_t i = first; i < wn[r]; ++i)
+            drain_wait(smem_u32(&wfull[r * kRing + i % kRing]), (i / kRing) & 1u, P.timeout_ns);
         }
       }
     }
@@ -444,7 +455,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const int ln = l + kIssuers < Lt ? l + kIssuers : iss;
           pack_next = __ldg(&P.use_pack[ln]);   // schedule word of this issuer's next layer
           if (acc_n >= 1 && !wait_bar(smem_u32(&acce[iss]), (acc_n - 1) & 1u, abort_flag, P.status,
-                                         KVX_ERR_TIMEOUT)) {
+                                         KVX_ERR_TIMEOUT, P.timeout_ns)) {
             ok = false;
             break;
           }
@@ -457,7 +468,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             const uint32_t s = f & 3u;
             if (f & 4u) {
               if (!wait_bar(smem_u32(&tready[s * kIssuers + iss]), (ready_par >> s) & 1u, abort_flag,
-                               P.status, KVX_ERR_TIMEOUT)) {
+                               P.status, KVX_ERR_TIMEOUT, P.timeout_ns)) {
                 ok = false;
                 break;
               }
@@ -468,7 +479,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int p = 0; p < kParts; ++p, ++wi) {   // hi (and lo) stages of this use
               const uint32_t st0 = iss * kRing + wi % kRing;
-              if (!wait_bar(smem_u32(&wfull[st0]), (wi / kRing) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT)) {
+              if (!wait_bar(smem_u32(&wfull[st0]), (wi / kRing) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT,
+                            P.timeout_ns)) {
                 ok = false;
                 break;
               }
@@ -491,7 +503,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       // every MMA (and every commit) of this issuer must have completed before TMEM is freed
       if (issued || !ok) {
         tc_commit_pair(smem_u32(&drain[iss]), 1);
-        drain_wait(smem_u32(&drain[iss]), 0);
+        drain_wait(smem_u32(&drain[iss]), 0, P.timeout_ns);
       }
     }
   }
@@ -564,7 +576,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const float* bias = bias_ring + bslot * kD;
         {
           const bool w_ok = wait_bar(smem_u32(&bias_full[bslot]), (lay / kBiasSlots) & 1u, abort_flag, P.status,
-                                     KVX_ERR_TIMEOUT);
+                                     KVX_ERR_TIMEOUT, P.timeout_ns);
           if (!__all_sync(0xffffffffu, w_ok)) {
             ok = false;
             break;
@@ -574,7 +586,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         {
           const uint32_t acc_par = (buf ? acc_n1 : acc_n0) & 1u;
           if (buf) ++acc_n1; else ++acc_n0;
-          const bool w_ok = wait_bar(smem_u32(&accf[buf]), acc_par, abort_flag, P.status, KVX_ERR_TIMEOUT);
+          const bool w_ok = wait_bar(smem_u32(&accf[buf]), acc_par, abort_flag, P.status, KVX_ERR_TIMEOUT,
+                                     P.timeout_ns);
           if (!__all_sync(0xffffffffu, w_ok)) {
             ok = false;
             break;
@@ -728,14 +741,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const uint32_t lw = static_cast<uint32_t>(__ldg(&P.load_slot[e]));
         const int s = static_cast<int>(lw & 3u);
         const int lb = gl % kLand;
-        bool w_ok = wait_bar(smem_u32(&land_full[lb]), (gl / kLand) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT);
+        bool w_ok =
+            wait_bar(smem_u32(&land_full[lb]), (gl / kLand) & 1u, abort_flag, P.status, KVX_ERR_TIMEOUT, P.timeout_ns);
         if ((tl_loaded >> s) & 1u) {
 #pragma unroll
           for (int i = 0; i < kIssuers; ++i) {
             if (!((lw >> (2 + i)) & 1u)) continue;
             const int bi = s * kIssuers + i;
             w_ok = w_ok && wait_bar(smem_u32(&tfree[bi]), (tfree_par >> bi) & 1u, abort_flag, P.status,
-                                    KVX_ERR_TIMEOUT);
+                                    KVX_ERR_TIMEOUT, P.timeout_ns);
             tfree_par ^= 1u << bi;
           }
         }
@@ -1071,6 +1085,8 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   }
   P.n_units = static_cast<int>(units);
   P.rope = c->rope;
+  P.timeout_ns = c->wait_limit_ns ? c->wait_limit_ns : kTimeoutNs;
+  P.skip_bias = static_cast<int32_t>(c->skip_bias_row);
   const size_t smem = smem_bytes();
   const bool hf = c->rope_numerics == KVX_ROPE_HF;
   void (*kernel)(TcParams) = c->weight_dtype == KVX_F32 ? (hf ? tc_map_kernel<true, 2> : tc_map_kernel<false, 2>)

@@ -95,7 +95,7 @@ class kvx_fit_config(ctypes.Structure):
         ("src_rope_theta", ctypes.c_double), ("tgt_rope_theta", ctypes.c_double),
         ("lambda_", ctypes.c_double), ("selection", ctypes.c_void_p),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_uint64),
-    ] + _SCALING + [("rope_numerics", ctypes.c_int32)]
+    ] + _SCALING + [("rope_numerics", ctypes.c_int32), ("head_mix", ctypes.c_int32)]
 
 
 class kvx_probe_config(ctypes.Structure):
@@ -127,7 +127,7 @@ EXPORTED = ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_
             "kvx_last_error", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms", "kvx_r2_probe",
             "kvx_select_topk_device", "kvx_fit_workspace_bytes", "kvx_r2_probe_workspace_bytes",
             "kvx_mlp_map", "kvx_mlp_workspace_bytes", "kvx_host_pipe_create", "kvx_map_host",
-            "kvx_host_pipe_destroy")
+            "kvx_host_pipe_destroy", "kvx_set_test_wait")
 
 
 def lib():
@@ -172,6 +172,8 @@ def lib():
     L.kvx_host_pipe_create.argtypes = [vp, i32, i32, ctypes.POINTER(vp)]
     L.kvx_map_host.argtypes = [vp, ctypes.POINTER(kvx_src), i32, vp, ctypes.POINTER(kvx_tgt), vp]
     L.kvx_host_pipe_destroy.argtypes = [vp]
+    L.kvx_set_test_wait.argtypes = [vp, ctypes.c_uint64, i64]
+    L.kvx_set_test_wait.restype = ctypes.c_int
     for name in ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
                  "kvx_set_kernel", "kvx_get_status", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms",
                  "kvx_r2_probe", "kvx_select_topk_device", "kvx_mlp_map", "kvx_host_pipe_create",
@@ -225,6 +227,11 @@ def kvx_map_noalloc(mapper, device, src, batch, tokens_per_seq, positions_ptr, t
                                  int(tokens_per_seq), positions_ptr, ctypes.byref(tgt), stream,
                                  ctypes.byref(st) if want_status else None), "kvx_map_noalloc")
     return st.value if want_status else None
+
+
+def kvx_set_test_wait(ctx, wait_limit_ns, skip_bias_row=-1):
+    """Test switch of the tensor-core kernel's bounded waits (see include/kvx.h)."""
+    _check(lib().kvx_set_test_wait(ctx, int(wait_limit_ns), int(skip_bias_row)), "kvx_set_test_wait")
 
 
 def kvx_destroy(ctx):
@@ -368,27 +375,30 @@ def _fit_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_
 
 
 def kvx_fit_workspace_bytes(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, selection,
-                            batch, tokens_per_seq):
+                            batch, tokens_per_seq, head_mix=KVX_PER_HEAD):
     """Bytes of a caller workspace that holds every calibration token in one pass (-1 on
     invalid arguments)."""
     import numpy as np
     sel = np.ascontiguousarray(selection, dtype=np.int32)
     cfg = _fit_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, sel, None, 0)
+    cfg.head_mix = int(head_mix)
     return int(lib().kvx_fit_workspace_bytes(ctypes.byref(cfg), int(batch), int(tokens_per_seq)))
 
 
 def kvx_fit_ridge(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, selection,
                   src, tgt, batch, tokens_per_seq, positions_ptr, W_ptr, b_ptr, stream=0,
-                  workspace_ptr=None, workspace_bytes=0, rope_scaling=None, rope_numerics=0):
+                  workspace_ptr=None, workspace_bytes=0, rope_scaling=None, rope_numerics=0,
+                  head_mix=KVX_PER_HEAD):
     """Ridge fit on calibration caches (see include/kvx.h): src / tgt are kvx_src, selection a
-    host int32 [L_t][k] array, W_ptr / b_ptr device fp32 buffers [L_t][2][H][k*d][d] and
-    [L_t][2][H][d]; an optional caller workspace (device, 256-byte aligned).  Blocks until
-    the fit is done."""
+    host int32 [L_t][k] array, W_ptr / b_ptr device fp32 buffers [L_t][2][H][F][d] (F = k*d
+    per head, k*H*d cross-head) and [L_t][2][H][d]; an optional caller workspace (device,
+    256-byte aligned).  Blocks until the fit is done."""
     import numpy as np
     sel = np.ascontiguousarray(selection, dtype=np.int32)
     cfg = _fit_config(src_layers, tgt_layers, n_kv_heads, head_dim, k, theta_s, theta_t, lam, sel, workspace_ptr,
                       workspace_bytes, rope_scaling)
     cfg.rope_numerics = int(rope_numerics)
+    cfg.head_mix = int(head_mix)
     _check(lib().kvx_fit_ridge(ctypes.byref(cfg), ctypes.byref(src), ctypes.byref(tgt), int(batch),
                                int(tokens_per_seq), positions_ptr, W_ptr, b_ptr, stream), "kvx_fit_ridge")
 

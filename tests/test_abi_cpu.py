@@ -310,3 +310,10 @@ def test_noalloc_rejects_bad_mapper_before_touching_the_device(sel, over, why):
         kvx.kvx_map_noalloc(m, 0, src, 1, 8, 0x30000, tgt, want_status=False)
     assert e.value.status == kvx.KVX_ERR_INVALID_ARG
     assert why in kvx.kvx_last_error()
+
+
+def test_set_test_wait_rejects_bad_arguments():
+    for args in ((None, 0, -1), (1, 10, -1), (1, 5_000_000_000, -1), (1, 0, -2), (1, 0, 2 ** 40)):
+        with pytest.raises(kvx.KvxError) as e:
+            kvx.kvx_set_test_wait(*args)
+        assert e.value.status == kvx.KVX_ERR_INVALID_ARG

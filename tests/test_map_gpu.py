@@ -687,3 +687,35 @@ def test_hf_rope_numerics_cross_head_tc():
         assert same_hf >= 0.9 and same_hf > same_exact + 0.1, (same_hf, same_exact)
     finally:
         kvx.kvx_destroy(ctx)
+
+
+# ------------------------------------------------------------ bounded waits -----
+
+def test_bounded_wait_runs_out_and_the_context_recovers():
+    """The tensor-core kernel's abort path, on a healthy GPU: with the test switch its first
+    CTA never loads one bias row, so the epilogue's wait for it runs out after the shortened
+    50 ms bound.  The launch must end by itself (well within a second), the status word
+    must read KVX_ERR_TIMEOUT, and the next launch on the same context (switch off) must map
+    every element within the oracle's tolerance."""
+    import time
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=3, Lt=4, H=1, B=1, T=256, k=2)
+    ctx, sel, W, b = make_ctx(w, kernel=kvx.KVX_KERNEL_TCGEN05)
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w)
+        torch.cuda.synchronize()
+        kvx.kvx_set_test_wait(ctx, 50_000_000, skip_bias_row=1)
+        t0 = time.perf_counter()
+        tk, tv, status = run_contiguous(ctx, w, sk, sv, pos)
+        dt = time.perf_counter() - t0
+        assert status == kvx.KVX_ERR_TIMEOUT, kvx.kvx_status_string(status)
+        assert dt < 1.0, "the aborted launch took %.3f s" % dt
+        kvx.kvx_set_test_wait(ctx, 0, -1)
+        tk, tv, status = run_contiguous(ctx, w, sk, sv, pos)
+        assert status == kvx.KVX_OK
+        rk, rv, ak, av = oracle_full(w, sk, sv, pos, sel, W, b)
+        ok, ratio, rms, nbad = check(w, [to_f64(tk), to_f64(tv)], [rk, rv], [ak, av])
+        assert ok, "after the abort: %d elements out of tolerance (worst %.3g x bound)" % (nbad, ratio)
+    finally:
+        kvx.kvx_destroy(ctx)
