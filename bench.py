@@ -325,6 +325,123 @@ def make_mapper(w, dev_index):
 
 
 
+def paged_bench(args, w):
+    """Multi-turn paged handoff (Sec. 4.5): every sequence's cache lives in one paged pool
+    whose block table covers its final length (initial length + turns x T tokens); a step
+    maps all turns in order, each turn's new tokens at their absolute positions from that
+    turn's own source cache.  One launch per turn.  value = mapped tokens per step / step
+    time; the roofline is taken per launch (one turn) on the average launch time."""
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(0)
+    stream = torch.cuda.current_stream(dev)
+    sp = stream.cuda_stream
+    ctx = make_mapper(w, 0)
+    L0 = syn.initial_lengths(w)
+    table, n_blocks = syn.persistent_block_table(w, L0)
+    tbl = torch.from_numpy(table).to(dev)
+    pool_k = torch.empty((w.Lt, n_blocks, w.H, w.block_size, w.d), dtype=torch.bfloat16, device=dev)
+    pool_v = torch.empty_like(pool_k)
+    pool_k.view(torch.int16).fill_(0x7FBF)
+    pool_v.view(torch.int16).fill_(0x7FBF)
+    tgt = kvx.tgt_paged_from_tensors(pool_k, pool_v, tbl, w.block_size)
+    turns = []
+    for j in range(w.turns):
+        sk = syn.source_cache(w, 0, device=dev, turn=j)
+        sv = syn.source_cache(w, 1, device=dev, turn=j)
+        pos = torch.from_numpy(syn.positions(w, j, L0)).to(dev)
+        turns.append((sk, sv, pos, kvx.src_from_tensors(sk, sv)))
+
+    def step():
+        for sk, sv, pos, src in turns:
+            kvx.kvx_map(ctx, src, w.B, w.T, pos.data_ptr(), tgt, sp)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    assert kvx.kvx_get_status(ctx, sp) == kvx.KVX_OK
+    steps = max(1, args.steps)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(0) as clk:
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for _ in range(steps):
+            step()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1) / steps
+    st = kvx.kvx_get_status(ctx, sp)
+    tokens = w.n_tokens * w.turns
+
+    # e2e: each turn's source caches and positions copied from pinned host memory inside
+    # the timed region (one turn's host buffers, copied into every turn's device buffers),
+    # then the map; the mapped target stays in the device pool the target model reads, so
+    # the step's device-to-host read is the 4-byte status word
+    hk = torch.empty(turns[0][0].shape, dtype=torch.bfloat16, pin_memory=True)
+    hv = torch.empty_like(hk, pin_memory=True)
+    hk.copy_(turns[0][0])
+    hv.copy_(turns[0][1])
+    hpos = [torch.from_numpy(syn.positions(w, j, L0)).pin_memory() for j in range(w.turns)]
+    h2d = w.turns * (hk.numel() * 2 + hv.numel() * 2 + hpos[0].numel() * 4)
+
+    def e2e_step():
+        for (sk, sv, pos, src), hp in zip(turns, hpos):
+            sk.copy_(hk, non_blocking=True)
+            sv.copy_(hv, non_blocking=True)
+            pos.copy_(hp, non_blocking=True)
+            kvx.kvx_map(ctx, src, w.B, w.T, pos.data_ptr(), tgt, sp)
+        return kvx.kvx_get_status(ctx, sp)
+
+    e2e_steps = max(1, min(args.e2e_steps or 3, 5))
+    e2e_step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ems = e0.elapsed_time(e1) / e2e_steps
+    kvx.kvx_destroy(ctx)
+
+    alg = algorithmic(w)                       # one launch = one turn
+    peaks = load_peaks()
+    launch_s = ms / w.turns / 1e3
+    t_tc = alg["flop"] / (peaks["bf16"] * 1e12)
+    t_hbm = alg["bytes"] / (peaks["hbm"] * 1e9)
+    bound = "tensor" if t_tc >= t_hbm else "hbm"
+    if bound == "tensor":
+        achieved, peak, unit = alg["flop"] / launch_s / 1e12, peaks["bf16"], "TFLOP/s"
+    else:
+        achieved, peak, unit = alg["bytes"] / launch_s / 1e9, peaks["hbm"], "GB/s"
+    clocks = clk.summary()
+    line = {"metric": METRIC, "value": tokens / (ms / 1e3), "unit": UNIT, "n_gpus": 1, "steps": steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": w.name + " (persistent pool, %d turns per step)" % w.turns,
+                       "src_layers": w.Ls, "tgt_layers": w.Lt, "kv_heads": w.H, "head_dim": w.d, "k": w.k,
+                       "batch": w.B, "tokens_per_turn": w.T, "turns": w.turns, "tokens_per_step": tokens,
+                       "pool_blocks": n_blocks, "pool_gb": 2 * pool_k.numel() * 2 / 1e9,
+                       "initial_lengths": [int(x) for x in L0], "layout": "paged (16-token blocks)",
+                       "l2": "no flush: each turn streams %.1f GB vs 129 MB L2" % (alg["bytes"] / 1e9)},
+            "clocks": clocks, "status": kvx.kvx_status_string(st),
+            "kcycles_per_step": ms * clocks["sm_mhz"] if clocks.get("sm_mhz") else None,
+            "per_turn_ms": ms / w.turns,
+            "e2e": {"value": tokens / (ems / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4,
+                    "steps": e2e_steps, "ms_per_step": ems,
+                    "api": "per turn: pinned-host copies of the source caches and positions + kvx_map into the "
+                           "device pool; kvx_get_status read at the end of the step"},
+            "gpu_launches": steps * w.turns,
+            "roofline": {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
+                         "traffic": None, "per": "launch (one turn, %d tokens)" % w.n_tokens,
+                         "peak_source": "%s (bf16 burst; HBM copy)" % peaks["source"],
+                         "other": {"hbm_frac": alg["bytes"] / launch_s / 1e9 / peaks["hbm"],
+                                   "tensor_frac": alg["flop"] / launch_s / 1e12 / peaks["bf16"]},
+                         "algorithmic": {"flop_per_launch": alg["flop"], "bytes_per_launch": alg["bytes"]}},
+            "cpu_baseline": None, "kernel": "tc_map_kernel (tcgen05, sm_103a), paged epilogue"}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 # The solve runs in float-float arithmetic on the FP32 lanes: one pair FMA is 15 FP32
 # instructions (two_prod by FMA, two_sum, fast_two_sum), and counts as 2 FLOP.
 FF_FMA_INSTR = 15
@@ -592,6 +709,8 @@ def main():
         return probe_bench(args, w)
     if args.mlp:
         return mlp_bench(args, w)
+    if w.paged and args.impl != "reference":
+        return paged_bench(args, w)
     alg = algorithmic(w)
     config = {"workload": w.name, "src_layers": w.Ls, "tgt_layers": w.Lt, "kv_heads": w.H,
               "head_dim": w.d, "k": w.k, "batch": w.B, "seq_len": w.T, "tokens_per_step": w.n_tokens,

@@ -308,3 +308,24 @@ def block_table(w, pos, turn=0):
         table[b, touched[b]] = perm[o:o + len(touched[b])]
         o += len(touched[b])
     return table, n_blocks
+
+
+def persistent_block_table(w, lengths):
+    """Paged target cache that persists across every turn: one seeded random block table
+    covering each sequence's final length L0_b + turns * T.
+
+    Logical block i of sequence b (positions 16 i .. 16 i + 15) gets a distinct physical
+    block, in a random permutation of a pool of exactly sum_b ceil(final_b / 16) blocks,
+    including the blocks of the initial prefix that no turn maps.  Returns (table int32
+    [B][max_blocks_per_seq], -1 past a sequence's last block, n_blocks)."""
+    bs = w.block_size
+    final = np.asarray(lengths, dtype=np.int64) + w.turns * w.T
+    nb = (final + bs - 1) // bs
+    table = np.full((w.B, int(nb.max())), -1, dtype=np.int32)
+    n_blocks = int(nb.sum())
+    perm = _rng(w, STREAM_BLOCKS + 999).permutation(n_blocks).astype(np.int32)
+    o = 0
+    for b in range(w.B):
+        table[b, :nb[b]] = perm[o:o + nb[b]]
+        o += int(nb[b])
+    return table, n_blocks

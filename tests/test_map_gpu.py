@@ -719,3 +719,125 @@ def test_bounded_wait_runs_out_and_the_context_recovers():
         assert ok, "after the abort: %d elements out of tolerance (worst %.3g x bound)" % (nbad, ratio)
     finally:
         kvx.kvx_destroy(ctx)
+
+
+# ------------------------------------------------- multi-turn persistent pool -----
+
+def _persistent_turns(w, kname, rows_of_turn, check_sentinel_turns):
+    """Map all w.turns turns into one pool whose block table covers every sequence's final
+    length (Sec. 4.5: only each turn's new tokens are mapped, at their absolute positions).
+    After each turn: the checked rows of every turn so far equal the oracle (a later turn
+    must not disturb them), and, on the turns listed, every slot outside the positions
+    mapped so far keeps its sentinel while every mapped slot is fully written."""
+    ctx, sel, W, b = make_ctx(w, kernel=KERNELS[kname])
+    dev = torch.device("cuda:0")
+    try:
+        L0 = syn.initial_lengths(w)
+        table, n_blocks = syn.persistent_block_table(w, L0)
+        tbl = torch.from_numpy(table).to(dev)
+        pool_k = torch.empty((w.Lt, n_blocks, w.H, w.block_size, w.d), dtype=torch.bfloat16, device=dev)
+        pool_v = torch.empty_like(pool_k)
+        pool_k.view(torch.int16).fill_(0x7FBF)
+        pool_v.view(torch.int16).fill_(0x7FBF)
+        tgt = kvx.tgt_paged_from_tensors(pool_k, pool_v, tbl, w.block_size)
+        written = torch.zeros((n_blocks, w.block_size), dtype=torch.bool)
+        s = torch.cuda.current_stream().cuda_stream
+        refs = []
+        for turn in range(w.turns):
+            pos = syn.positions(w, turn, L0)
+            sk = syn.source_cache(w, 0, device=dev, turn=turn)
+            sv = syn.source_cache(w, 1, device=dev, turn=turn)
+            posd = torch.from_numpy(pos).to(dev)
+            kvx.kvx_map(ctx, kvx.src_from_tensors(sk, sv), w.B, w.T, posd.data_ptr(), tgt, s)
+            assert kvx.kvx_get_status(ctx, s) == kvx.KVX_OK, "turn %d" % turn
+            del sk, sv
+            for bb in range(w.B):
+                written[torch.from_numpy(table[bb, pos[bb] // w.block_size].astype(np.int64)),
+                        torch.from_numpy((pos[bb] % w.block_size).astype(np.int64))] = True
+            rows = rows_of_turn(turn)
+            rk, rv, ak, av = oracle_rows(w, rows, pos, sel, W, b, turn=turn)
+            p = pos[rows[:, 0], rows[:, 1]]
+            refs.append((rows, table[rows[:, 0], p // w.block_size].astype(np.int64),
+                         (p % w.block_size).astype(np.int64), rk, rv, ak, av))
+            for j, (rows_j, blk, slot, rk, rv, ak, av) in enumerate(refs):
+                gk = to_f64(pool_k[:, blk, :, slot].permute(1, 2, 0, 3))
+                gv = to_f64(pool_v[:, blk, :, slot].permute(1, 2, 0, 3))
+                ok, ratio, rms, nbad = check(w, [gk, gv], [rk, rv], [ak, av])
+                assert ok, "after turn %d, rows of turn %d: %d out of tolerance (worst %.3g)" % (turn, j, nbad, ratio)
+            if turn in check_sentinel_turns:
+                wd = written.to(dev)
+                for pool in (pool_k, pool_v):
+                    for l in range(w.Lt):          # one layer at a time bounds the temporaries
+                        sent = pool[l].view(torch.int16) == 0x7FBF            # [nb][H][bs][d]
+                        assert torch.equal(sent.all(dim=-1).all(dim=1), ~wd), \
+                            "turn %d layer %d: a slot outside the mapped tokens was touched" % (turn, l)
+                        assert torch.equal((~sent).all(dim=-1).all(dim=1), wd), \
+                            "turn %d layer %d: a mapped slot was not fully written" % (turn, l)
+                        del sent
+    finally:
+        kvx.kvx_destroy(ctx)
+        torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("kname", ["simt", "tc"])
+def test_paged_persistent_pool_eight_turns_small(kname):
+    w = syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4", Ls=5, Lt=3, H=2, B=3, T=37, k=2,
+                     len_range=(3, 70))
+    if kname == "tc":
+        _kernel_or_skip(w, KERNELS[kname])
+    every_row = np.array([(bb, t) for bb in range(w.B) for t in range(w.T)], dtype=np.int64)
+    _persistent_turns(w, kname, lambda turn: every_row, check_sentinel_turns=range(w.turns))
+
+
+def test_paged_persistent_pool_eight_turns_full_size_sampled():
+    """The Qwen3-32B -> 14B paged workload as specified: 16 sequences, initial lengths in
+    [2048, 16384], eight turns of 2048 new tokens into one pool sized for the final lengths
+    (about 67 GB of bf16 target cache); 24 sampled rows per turn, all earlier turns'
+    sampled rows re-checked after each turn, every slot checked after the first and the
+    last turn."""
+    w = syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4")
+    _persistent_turns(w, "tc", lambda turn: sample_rows(w, 24, seed=100 + turn),
+                      check_sentinel_turns=(0, w.turns - 1))
+
+
+# ------------------------------------------------------------ strip error bound -----
+
+def test_strip_error_within_delta_up_to_max_position():
+    """Pins STRIP_DELTA, the per-rotation error the rounding slack of the bf16 tests assumes:
+    a stored pair (a, b) rotated by the kernels' angle arithmetic (float-float angle,
+    Cody-Waite reduction, sincosf) is within delta (|a| + |b|) of the exact rotation.  With
+    fp32 caches, k = 1, W = I, b = 0 and theta_s != theta_t the map is two such rotations (strip
+    by theta_s, re-rotation by theta_t); the second acts on a pair of size at most
+    sqrt(2) (|a| + |b|) and rotations preserve the first one's error, so every key output is
+    within 2 sqrt(2) delta (|a| + |b|) of the exact oracle (plus one fp32 rounding).  Positions
+    cover 0, powers of two and their neighbours, random values and 2^24 - 1 (the largest
+    accepted); values must come back bit for bit."""
+    from harness import STRIP_DELTA
+    w = syn.workload("tiny_fp32", Ls=1, Lt=1, H=1, d=128, k=1, B=1, T=1024, theta_s=1e6, theta_t=5e5)
+    rng = np.random.default_rng(24)
+    special = [0, 1, 2, 3, (1 << 24) - 1, (1 << 24) - 2] + [(1 << e) + o for e in range(2, 24) for o in (-1, 0, 1)]
+    pos = np.array(special + list(rng.integers(0, 1 << 24, size=w.T - len(special))), dtype=np.int32)[None, :]
+    W = torch.zeros((1, 2, 1, 128, 128), dtype=torch.float32)
+    W[0, :, 0] = torch.eye(128)
+    b = torch.zeros((1, 2, 1, 128), dtype=torch.float32)
+    ctx, sel, _, _ = make_ctx(w, selection=np.zeros((1, 1), dtype=np.int32), W=W, b=b)
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        assert torch.equal(tv, sv), "values must pass through W = I unchanged"
+        x = to_f64(sk)[0, 0, 0]                                  # [T][128] stored keys
+        ref = omap.map_tokens(x[None, None], to_f64(sv)[0, 0, 0][None, None], pos[0], sel, W.double().numpy(),
+                              b.double().numpy(), w.theta_s, w.theta_t, mode="exact")[0][0, 0]   # [T][128]
+        got = to_f64(tk)[0, 0, 0]
+        mag = np.abs(x[:, :64]) + np.abs(x[:, 64:])
+        mag = np.concatenate([mag, mag], axis=1)                 # |a| + |b| of each output's pair
+        bound = 2.0 * np.sqrt(2.0) * STRIP_DELTA * mag + 2.0 ** -23 * np.abs(ref)
+        err = np.abs(got - ref)
+        ratio = err / bound
+        assert np.all(err <= bound), "worst %.3g x bound at position %d" % (
+            ratio.max(), pos[0, np.unravel_index(np.argmax(ratio), ratio.shape)[0]])
+        assert np.array_equal(got[0], x[0]), "position 0 must come back unrotated and exact"
+    finally:
+        kvx.kvx_destroy(ctx)

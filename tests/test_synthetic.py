@@ -71,3 +71,20 @@ def test_paged_block_table_is_a_permutation():
         assert sorted(used.tolist()) == list(range(n_blocks))
         for b in range(w.B):
             assert np.all(table[b, pos[b] // 16] >= 0)
+
+
+def test_persistent_block_table_is_a_permutation_over_final_lengths():
+    w = syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4", B=5, T=37, len_range=(3, 70))
+    L0 = syn.initial_lengths(w)
+    table, n_blocks = syn.persistent_block_table(w, L0)
+    final = L0 + w.turns * w.T
+    nb = (final + w.block_size - 1) // w.block_size
+    assert n_blocks == nb.sum() and table.shape == (w.B, nb.max())
+    used = np.concatenate([table[b, :nb[b]] for b in range(w.B)])
+    assert np.array_equal(np.sort(used), np.arange(n_blocks))
+    for b in range(w.B):
+        assert np.all(table[b, nb[b]:] == -1)
+    # every position any turn maps has a block
+    for turn in range(w.turns):
+        pos = syn.positions(w, turn, L0)
+        assert np.all(table[np.arange(w.B)[:, None], pos // w.block_size] >= 0)
