@@ -336,6 +336,8 @@ def paged_bench(args, w):
     stream = torch.cuda.current_stream(dev)
     sp = stream.cuda_stream
     ctx = make_mapper(w, 0)
+    kernel_id = kvx.kvx_get_kernel(ctx, paged=True)
+    kernel_name = kvx.KERNEL_NAMES[kernel_id]
     L0 = syn.initial_lengths(w)
     table, n_blocks = syn.persistent_block_table(w, L0)
     tbl = torch.from_numpy(table).to(dev)
@@ -430,14 +432,14 @@ def paged_bench(args, w):
                     "steps": e2e_steps, "ms_per_step": ems,
                     "api": "per turn: pinned-host copies of the source caches and positions + kvx_map into the "
                            "device pool; kvx_get_status read at the end of the step"},
-            "gpu_launches": steps * w.turns,
+            "gpu_launches": steps * w.turns * (2 if kernel_id == 3 else 1),
             "roofline": {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
                          "traffic": None, "per": "launch (one turn, %d tokens)" % w.n_tokens,
                          "peak_source": "%s (bf16 burst; HBM copy)" % peaks["source"],
                          "other": {"hbm_frac": alg["bytes"] / launch_s / 1e9 / peaks["hbm"],
                                    "tensor_frac": alg["flop"] / launch_s / 1e12 / peaks["bf16"]},
                          "algorithmic": {"flop_per_launch": alg["flop"], "bytes_per_launch": alg["bytes"]}},
-            "cpu_baseline": None, "kernel": "tc_map_kernel (tcgen05, sm_103a), paged epilogue"}
+            "cpu_baseline": None, "kernel": kernel_name + ", paged epilogue"}
     print(json.dumps(line), flush=True)
     return 0
 
@@ -728,6 +730,7 @@ def main():
     sp = stream.cuda_stream
 
     ctx = make_mapper(w, local)
+    kernel_id = kvx.kvx_get_kernel(ctx)
     sk = syn.source_cache(w, 0, device=dev)
     sv = syn.source_cache(w, 1, device=dev)
     pos_np = syn.positions(w)
@@ -861,11 +864,10 @@ def main():
                     "steps": e2e_steps, "ms_per_step": ems / e2e_steps, "api": e2e_api,
                     "link_gbs": link, "copy_floor_ms": floor_ms,
                     "frac_of_copy_floor": floor_ms / (ems / e2e_steps)},
-            # one launch per step (per-head); the cross-head map is a key-strip kernel then the GEMMs
-            "gpu_launches": args.steps * (2 if w.head_mix == "cross_head" else 1), "roofline": roofline,
+            # one launch per step, or a key-strip launch and the GEMMs on the cross-head kernel
+            "gpu_launches": args.steps * (2 if kernel_id == 3 else 1), "roofline": roofline,
             "cpu_baseline": cpu,
-            "kernel": ("xh_strip_kernel + tc_xh_kernel (tcgen05 pair GEMM, sm_103a)" if w.head_mix == "cross_head"
-                       else "tc_map_kernel (tcgen05, sm_103a)")}
+            "kernel": kvx.KERNEL_NAMES[kernel_id]}
     print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()

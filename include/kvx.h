@@ -68,7 +68,7 @@ typedef enum { KVX_PER_HEAD = 0, KVX_CROSS_HEAD = 1 } kvx_head_mix;
 
 /* Which kernel kvx_map launches.  AUTO picks a tensor-core (tcgen05) kernel when the
  * shape allows it (bf16 caches, head_dim 128, HALF; PER_HEAD with k <= 4, or CROSS_HEAD
- * with an even head count and a contiguous target) and the fp32 SIMT kernel otherwise.
+ * with an even head count; contiguous or paged targets) and the fp32 SIMT kernel otherwise.
  * fp32 weights run on the tensor cores split into bf16 hi = bf16(w) and lo = bf16(w - hi)
  * (twice the MMAs; the contraction follows the fp32 W to within 2^-17 of each weight).
  * The CROSS_HEAD tensor-core kernel keeps a workspace for the stripped source keys
@@ -215,6 +215,13 @@ KVX_API kvx_status kvx_get_selection(const kvx_ctx* ctx, int32_t* out);
 /* Choose the kernel for later kvx_map calls (kvx_kernel).  UNSUPPORTED if the
  * configuration cannot run on the requested kernel. */
 KVX_API kvx_status kvx_set_kernel(kvx_ctx* ctx, int32_t kernel);
+
+/* Which kernel kvx_map runs on ctx for a contiguous (paged = 0) or paged (paged = 1)
+ * target under the current kvx_set_kernel choice: *out = 1 the fp32 SIMT kernel, 2 the
+ * per-head tensor-core kernel (one launch), 3 the cross-head tensor-core kernel (a key-strip
+ * launch and a GEMM launch; per-head mappers with k > 4 run here on W widened with zeros
+ * outside each head's rows).  INVALID_ARG for a NULL argument. */
+KVX_API kvx_status kvx_get_kernel(const kvx_ctx* ctx, int32_t paged, int32_t* out);
 
 /* Synchronise `stream`, return the device status word (KVX_OK or the first
  * device-detected error since the last call) and reset it to KVX_OK. */

@@ -113,6 +113,18 @@ __device__ __forceinline__ DF df_fma(DF a, DF b, DF c) {
   const DF s = two_sum(p, c.hi);
   return fast_two_sum(s.hi, __fadd_rn(s.lo, __fadd_rn(e, c.lo)));
 }
+// Dot-product accumulation with the renormalisation deferred: c.hi + c.lo is a running
+// sum whose c.lo collects every step's rounding errors unnormalised (3 FP32 instructions
+// fewer per step than df_fma); df_norm turns it back into a pair before the sum is used.
+__device__ __forceinline__ DF df_fma_lazy(DF a, DF b, DF c) {
+  const float p = __fmul_rn(a.hi, b.hi);
+  float e = __fmaf_rn(a.hi, b.hi, -p);
+  e = __fmaf_rn(a.hi, b.lo, e);
+  e = __fmaf_rn(a.lo, b.hi, e);
+  const DF s = two_sum(p, c.hi);
+  return DF{s.hi, __fadd_rn(c.lo, __fadd_rn(s.lo, e))};
+}
+__device__ __forceinline__ DF df_norm(DF a) { return two_sum(a.hi, a.lo); }
 // a / b: the float quotient q corrected by the residual a - q b
 __device__ __forceinline__ DF df_div(DF a, DF b) {
   const float q1 = __fdiv_rn(a.hi, b.hi);
@@ -179,8 +191,8 @@ __device__ __forceinline__ void chol_panel(DF* A, int F, int c0, const DF* D, DF
     for (int c = 0; c < kNB; ++c) {
       DF v = arow[c];
 #pragma unroll
-      for (int m = 0; m < c; ++m) v = df_fma(df_neg(x[m]), D[c * kPS + m], v);
-      x[c] = df_div(v, D[c * kPS + c]);
+      for (int m = 0; m < c; ++m) v = df_fma_lazy(df_neg(x[m]), D[c * kPS + m], v);
+      x[c] = df_div(df_norm(v), D[c * kPS + c]);
     }
 #pragma unroll
     for (int c = 0; c < kNB; ++c) {
@@ -221,7 +233,7 @@ __device__ __forceinline__ void tri_solves(const DF* A, int F, DF* Z, int ldz, D
 #pragma unroll
       for (int a2 = 0; a2 < kR; ++a2)
 #pragma unroll
-        for (int c = 0; c < 4; ++c) acc[a2][c] = df_fma(l[a2], z[c], acc[a2][c]);
+        for (int c = 0; c < 4; ++c) acc[a2][c] = df_fma_lazy(l[a2], z[c], acc[a2][c]);
     }
   };
   auto stage_z = [&](int m0) {        // 32 rows x 128 pairs, two pairs per thread-step
@@ -244,14 +256,14 @@ __device__ __forceinline__ void tri_solves(const DF* A, int F, DF* Z, int ldz, D
 #pragma unroll
     for (int a = 0; a < kR; ++a)
 #pragma unroll
-      for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * ldz + q0 + c] = acc[a][c];
+      for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * ldz + q0 + c] = df_norm(acc[a][c]);
     __syncthreads();
     if (tid < kFD) {
       for (int i = 0; i < kNB; ++i) {
         const DF* lrow = A + static_cast<size_t>(b0 + i) * F + b0;
         DF v = Z[static_cast<size_t>(b0 + i) * ldz + tid];
-        for (int m = 0; m < i; ++m) v = df_fma(df_neg(lrow[m]), Z[static_cast<size_t>(b0 + m) * ldz + tid], v);
-        Z[static_cast<size_t>(b0 + i) * ldz + tid] = df_div(v, lrow[i]);
+        for (int m = 0; m < i; ++m) v = df_fma_lazy(df_neg(lrow[m]), Z[static_cast<size_t>(b0 + m) * ldz + tid], v);
+        Z[static_cast<size_t>(b0 + i) * ldz + tid] = df_div(df_norm(v), lrow[i]);
       }
     }
     __syncthreads();
@@ -271,14 +283,14 @@ __device__ __forceinline__ void tri_solves(const DF* A, int F, DF* Z, int ldz, D
 #pragma unroll
     for (int a = 0; a < kR; ++a)
 #pragma unroll
-      for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * ldz + q0 + c] = acc[a][c];
+      for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * ldz + q0 + c] = df_norm(acc[a][c]);
     __syncthreads();
     if (tid < kFD) {
       for (int i = kNB - 1; i >= 0; --i) {
         DF v = Z[static_cast<size_t>(b0 + i) * ldz + tid];
         for (int m = i + 1; m < kNB; ++m)
-          v = df_fma(df_neg(A[static_cast<size_t>(b0 + m) * F + b0 + i]), Z[static_cast<size_t>(b0 + m) * ldz + tid], v);
-        Z[static_cast<size_t>(b0 + i) * ldz + tid] = df_div(v, A[static_cast<size_t>(b0 + i) * F + b0 + i]);
+          v = df_fma_lazy(df_neg(A[static_cast<size_t>(b0 + m) * F + b0 + i]), Z[static_cast<size_t>(b0 + m) * ldz + tid], v);
+        Z[static_cast<size_t>(b0 + i) * ldz + tid] = df_div(df_norm(v), A[static_cast<size_t>(b0 + i) * F + b0 + i]);
       }
     }
     __syncthreads();
@@ -343,12 +355,12 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __gri
         for (int m = 0; m < kNB; ++m) {
           const DF pj = Pn[jj * kPS + m];
 #pragma unroll
-          for (int q = 0; q < kRowsPer; ++q) sacc[q] = df_fma(Pn[(ii + kSolveWarps * q) * kPS + m], pj, sacc[q]);
+          for (int q = 0; q < kRowsPer; ++q) sacc[q] = df_fma_lazy(Pn[(ii + kSolveWarps * q) * kPS + m], pj, sacc[q]);
         }
 #pragma unroll
         for (int q = 0; q < kRowsPer; ++q) {
           DF* a = A + static_cast<size_t>(c0 + kNB + ii + kSolveWarps * q) * F + c0 + kNB + jj;
-          if (jj <= ii + kSolveWarps * q) *a = df_add(*a, df_neg(sacc[q]));
+          if (jj <= ii + kSolveWarps * q) *a = df_add(*a, df_neg(df_norm(sacc[q])));
         }
       }
       __syncthreads();
@@ -450,7 +462,7 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_xh_kernel(const __
         for (int m = 0; m < kNB; ++m) {
           const DF pj = Pj[jj * kPS + m];
 #pragma unroll
-          for (int q = 0; q < kQ; ++q) sacc[q] = df_fma(Pi[(ii + 8 * q) * kPS + m], pj, sacc[q]);
+          for (int q = 0; q < kQ; ++q) sacc[q] = df_fma_lazy(Pi[(ii + 8 * q) * kPS + m], pj, sacc[q]);
         }
         const int gj = tj * kXT + jj;
 #pragma unroll
@@ -458,7 +470,7 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_xh_kernel(const __
           const int gi = ti * kXT + ii + 8 * q;
           if (gi < rows && gj <= gi) {
             DF* a = A + static_cast<size_t>(base + gi) * F + base + gj;
-            *a = df_add(*a, df_neg(sacc[q]));
+            *a = df_add(*a, df_neg(df_norm(sacc[q])));
           }
         }
         __syncthreads();

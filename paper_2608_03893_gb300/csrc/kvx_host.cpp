@@ -283,11 +283,31 @@ kvx_status kvx_create(const kvx_config* cfg, int device, kvx_ctx** out) {
 
   std::string why;
   ctx->tc_eligible = tc_supported(ctx, &why);
-  ctx->xh_eligible = xh_supported(ctx, &why);
+  ctx->xh_eligible = !ctx->tc_eligible && xh_supported(ctx, &why);
+  ctx->F_xh = ctx->k * ctx->H * ctx->d;
   if (ctx->tc_eligible || ctx->xh_eligible) {
+    // A per-head mapper with more selected layers than the per-head kernel holds in tensor
+    // memory runs on the cross-head kernel: W of target head h widened to the cross-head
+    // feature (every head of the k layers) with zeros outside head h's rows, which leaves
+    // the map unchanged (the extra products are exact zeros).
+    std::vector<uint8_t> wide;
+    const void* w_xh = c.W;
+    if (ctx->xh_eligible && ctx->head_mix == KVX_PER_HEAD) {
+      const size_t es = ctx->weight_dtype == KVX_BF16 ? 2 : 4, d = ctx->d, F = ctx->F, Fx = ctx->F_xh;
+      const size_t blocks = static_cast<size_t>(ctx->Lt) * 2 * ctx->H;
+      wide.assign(blocks * Fx * d * es, 0);
+      const uint8_t* w = static_cast<const uint8_t*>(c.W);
+      for (size_t blk = 0; blk < blocks; ++blk) {
+        const size_t h = blk % ctx->H;
+        for (int j = 0; j < ctx->k; ++j)   // rows of selected layer j, head h: x = (j H + h) d
+          std::memcpy(wide.data() + (blk * Fx + (j * ctx->H + h) * d) * d * es, w + (blk * F + j * d) * d * es,
+                      d * d * es);
+      }
+      w_xh = wide.data();
+    }
     kvx_status s = ctx->tc_eligible                  ? tc_prepare(ctx, c.W)
-                   : ctx->weight_dtype == KVX_F32 ? repack_wt_hilo(ctx, c.W)
-                                                  : repack_wt(ctx, c.W);
+                   : ctx->weight_dtype == KVX_F32 ? repack_wt_hilo(ctx, w_xh, ctx->F_xh)
+                                                  : repack_wt(ctx, w_xh, ctx->F_xh);
     if (s != KVX_OK) {
       free_ctx(ctx);
       return s;
@@ -326,6 +346,16 @@ kvx_status kvx_set_kernel(kvx_ctx* ctx, int32_t kernel) {
     return fail(KVX_ERR_UNSUPPORTED, "kvx_set_kernel: tensor-core kernel unavailable: " + why);
   }
   ctx->kernel = kernel;
+  return KVX_OK;
+}
+
+kvx_status kvx_get_kernel(const kvx_ctx* ctx, int32_t paged, int32_t* out) {
+  g_last_error.clear();
+  if (!ctx || !out) return fail(KVX_ERR_INVALID_ARG, "kvx_get_kernel: NULL argument");
+  (void)paged;   // every kernel writes both target kinds
+  if (ctx->xh_eligible && ctx->kernel != KVX_KERNEL_SIMT) *out = 3;
+  else if (ctx->tc_eligible && ctx->kernel != KVX_KERNEL_SIMT) *out = 2;
+  else *out = 1;
   return KVX_OK;
 }
 
@@ -407,10 +437,8 @@ kvx_status kvx_map(kvx_ctx* ctx, const kvx_src* src, int32_t batch, int32_t toke
   DeviceGuard guard(ctx->device);
   if (guard.err != cudaSuccess) return cuda_fail(guard.err, "kvx_map: cudaSetDevice");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  // cross-head: the tensor-core kernel writes contiguous targets; AUTO maps paged ones
-  // with the SIMT kernel, an explicit TCGEN05 choice gets KVX_ERR_UNSUPPORTED from it
-  if (ctx->xh_eligible && (ctx->kernel == KVX_KERNEL_TCGEN05 || (ctx->kernel == KVX_KERNEL_AUTO && !a.paged)))
-    return launch_xh(ctx, a, st);
+  // cross-head: the tensor-core kernel writes contiguous and paged targets
+  if (ctx->xh_eligible && ctx->kernel != KVX_KERNEL_SIMT) return launch_xh(ctx, a, st);
   const bool use_tc = ctx->kernel == KVX_KERNEL_TCGEN05 || (ctx->kernel == KVX_KERNEL_AUTO && ctx->tc_eligible);
   return use_tc ? launch_tc(ctx, a, st) : launch_simt(ctx, a, st);
 }

@@ -91,6 +91,9 @@ struct kvx_ctx {
   int sm_count = 0;
   // test switches (kvx_set_test_wait): the per-head tensor-core kernel's wait bound, and a
   // bias row its first CTA never loads, which makes one of its waits run out
+  int F_xh = 0;                      // feature width of the cross-head kernel's W^T: F for a
+                                     // cross-head mapper, k * H * d for a per-head one (block-
+                                     // diagonal W, zero outside head h's rows)
   uint64_t wait_limit_ns = 0;        // 0: the default bound
   int64_t skip_bias_row = -1;
 };
@@ -114,7 +117,7 @@ bool tc_supported(const kvx_ctx* ctx, std::string* why);
 kvx_status tc_prepare(kvx_ctx* ctx, const void* W_host);   // repack W, build the plan
 kvx_status launch_tc(const kvx_ctx* ctx, const MapArgs& a, cudaStream_t stream);
 // W [L_t][2][H][F][d] -> W^T [L_t][2][H][d][F] bf16 in ctx->d_Wt (both tensor-core kernels).
-kvx_status repack_wt(kvx_ctx* ctx, const void* W_host);
+kvx_status repack_wt(kvx_ctx* ctx, const void* W_host, size_t F);
 // cuTensorMapEncodeTiled from the driver (as void*: PFN_cuTensorMapEncodeTiled_v12000), or NULL.
 void* tensor_map_encoder();
 

@@ -944,9 +944,8 @@ bool tc_supported(const kvx_ctx* c, std::string* why) {
   return w.empty();
 }
 
-kvx_status repack_wt(kvx_ctx* c, const void* W_host) {
+kvx_status repack_wt(kvx_ctx* c, const void* W_host, size_t F) {
   // W [L_t][2][H][F][128] -> W^T [L_t][2][H][128][F] (B operand, K-major)
-  const size_t F = c->F;
   const size_t blocks = static_cast<size_t>(c->Lt) * 2 * c->H;
   std::vector<uint16_t> wt(blocks * F * kD);
   const uint16_t* w = static_cast<const uint16_t*>(W_host);
@@ -969,7 +968,7 @@ kvx_status repack_wt(kvx_ctx* c, const void* W_host) {
 }
 
 kvx_status tc_prepare(kvx_ctx* c, const void* W_host) {
-  kvx_status st = c->weight_dtype == KVX_F32 ? repack_wt_hilo(c, W_host) : repack_wt(c, W_host);
+  kvx_status st = c->weight_dtype == KVX_F32 ? repack_wt_hilo(c, W_host, c->F) : repack_wt(c, W_host, c->F);
   if (st != KVX_OK) return st;
   cudaError_t e;
   build_plan(c, &c->plan);

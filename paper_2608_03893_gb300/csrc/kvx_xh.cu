@@ -382,6 +382,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
           p = 0;
         }
       }
+      // the row's element offset within a target layer, without the head term: contiguous
+      // (batch, token) or paged (block through the block table, slot)
+      int64_t row_off = 0;
+      if (valid) {
+        if (!A.paged) {
+          row_off = un.b * A.ts[1] + static_cast<int64_t>(t) * A.ts[3];
+        } else {
+          const int lb = p / A.block_size;
+          const int blk =
+              lb < A.max_blocks ? __ldg(&A.block_table[static_cast<int64_t>(un.b) * A.max_blocks + lb]) : -1;
+          if (blk < 0 || blk >= A.n_blocks) {
+            xreport(P.status, KVX_ERR_DEVICE_BOUNDS);
+            valid = false;
+          } else {
+            row_off = static_cast<int64_t>(blk) * A.ts[1] + static_cast<int64_t>(p % A.block_size) * A.ts[3];
+          }
+        }
+      }
       const bool warp_tma = P.out_bh != 0 && __ballot_sync(0xffffffffu, bad) == 0u;
       if (un.kv == 0) {
 #pragma unroll
@@ -487,8 +505,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
             *reinterpret_cast<uint4*>(prow + kXPieceBytes + (((2 * rnd) ^ sw) << 4)) = v[2];
             *reinterpret_cast<uint4*>(prow + kXPieceBytes + (((2 * rnd + 1) ^ sw) << 4)) = v[3];
           } else if (valid) {
-            __nv_bfloat16* out = dst + static_cast<int64_t>(un.l) * A.ts[0] + un.b * A.ts[1] +
-                                 static_cast<int64_t>(h) * A.ts[2] + static_cast<int64_t>(t) * A.ts[3];
+            __nv_bfloat16* out = dst + static_cast<int64_t>(un.l) * A.ts[0] + row_off + static_cast<int64_t>(h) * A.ts[2];
             st_global_hint(out + c_lo, v[0], st_pol);
             st_global_hint(out + c_lo + 8, v[1], st_pol);
             st_global_hint(out + 64 + c_lo, v[2], st_pol);
@@ -525,11 +542,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
 
 }  // namespace
 
-kvx_status repack_wt_hilo(kvx_ctx* c, const void* W_host) {
+kvx_status repack_wt_hilo(kvx_ctx* c, const void* W_host, size_t F) {
   // W fp32 [L_t][2][H][F][128] -> W^T bf16 [L_t][2][H][128][2F]: columns [0, F) hold
   // hi = bf16(w), columns [F, 2F) lo = bf16(w - hi), so X W = X W_hi + X W_lo to within
   // 2^-17 of each weight (the paper keeps W in fp32)
-  const size_t F = c->F;
   const size_t blocks = static_cast<size_t>(c->Lt) * 2 * c->H;
   std::vector<uint16_t> wt(blocks * 2 * F * kXD);
   const float* w = static_cast<const float*>(W_host);
@@ -578,19 +594,18 @@ bool xh_supported(const kvx_ctx* c, std::string* why) {
   std::string w;
   if (c->cache_dtype != KVX_BF16) w = "needs bf16 caches";
   else if (c->d != kXD) w = "needs head_dim 128";
-  else if (c->head_mix != KVX_CROSS_HEAD) w = "needs the cross-head feature layout";
+  else if (c->head_mix != KVX_CROSS_HEAD && c->k <= 4)
+    w = "runs per-head mappers only for k > 4 (the per-head tensor-core kernel takes k <= 4)";
   else if (c->rope_style != KVX_ROPE_HALF) w = "needs half-split RoPE pairs";
   else if (c->H % 2 != 0) w = "needs an even number of KV heads";
-  else if (static_cast<int64_t>(c->Lt) * 2 * c->H * kXD > INT_MAX || c->F > INT_MAX / 2) w = "too many W rows";
+  else if (static_cast<int64_t>(c->Lt) * 2 * c->H * kXD > INT_MAX ||
+           static_cast<int64_t>(c->k) * c->H * kXD > INT_MAX / 2)
+    w = "too many W rows";
   if (why) *why = w;
   return w.empty();
 }
 
 kvx_status launch_xh(kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
-  if (a.paged) {
-    set_error("kvx_map: the cross-head tensor-core kernel writes contiguous targets only");
-    return KVX_ERR_UNSUPPORTED;
-  }
   auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(tensor_map_encoder());
   if (!encode) {
     set_error("kvx_map: cuTensorMapEncodeTiled unavailable");
@@ -641,9 +656,10 @@ kvx_status launch_xh(kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
       return KVX_ERR_UNSUPPORTED;
     }
   }
-  // targets: as in the per-head kernel, (64 channels, T, 2 halves, heads, L_t), box 32 x 32 x 2
+  // targets: as in the per-head kernel, (64 channels, T, 2 halves, heads, L_t), box 32 x 32 x 2;
+  // paged targets take 16-byte stores through the block table
   P.out_bh = 0;
-  if (a.B == 1 || a.ts[1] == static_cast<int64_t>(c->H) * a.ts[2]) {
+  if (!a.paged && (a.B == 1 || a.ts[1] == static_cast<int64_t>(c->H) * a.ts[2])) {
     P.out_bh = a.B == 1 ? 1 : 2;
     const cuuint32_t tbox[5] = {32, 32, 2, 1, 1};
     const cuuint64_t tdims[5] = {64, static_cast<cuuint64_t>(a.T), 2,
@@ -664,7 +680,7 @@ kvx_status launch_xh(kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   }
   {  // W^T [L_t*2*H*128][F], box 64 features x 128 rows
     // fp32 weights: W^T holds [W_hi | W_lo], 2F columns (see repack_wt_hilo)
-    const cuuint64_t wcols = static_cast<cuuint64_t>(c->F) * (c->weight_dtype == KVX_F32 ? 2 : 1);
+    const cuuint64_t wcols = static_cast<cuuint64_t>(c->F_xh) * (c->weight_dtype == KVX_F32 ? 2 : 1);
     const cuuint64_t wdims[2] = {wcols, static_cast<cuuint64_t>(c->Lt) * 2 * c->H * kXD};
     const cuuint64_t wstr[1] = {wcols * 2};
     const cuuint32_t wbox[2] = {64, 128};

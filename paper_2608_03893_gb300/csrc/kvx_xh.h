@@ -13,6 +13,6 @@ void launch_key_strip(const void* src_k, const int64_t* ss, void* ws, const int3
 
 // fp32 W [L_t][2][H][F][128] -> W^T bf16 [L_t][2][H][128][2F] = [W_hi | W_lo] in ctx->d_Wt,
 // for the tensor-core map kernels (cross-head and per-head) with fp32 weights.
-kvx_status repack_wt_hilo(kvx_ctx* c, const void* W_host);
+kvx_status repack_wt_hilo(kvx_ctx* c, const void* W_host, size_t F);
 
 }  // namespace kvx

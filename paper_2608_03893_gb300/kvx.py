@@ -127,7 +127,7 @@ EXPORTED = ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_
             "kvx_last_error", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms", "kvx_r2_probe",
             "kvx_select_topk_device", "kvx_fit_workspace_bytes", "kvx_r2_probe_workspace_bytes",
             "kvx_mlp_map", "kvx_mlp_workspace_bytes", "kvx_host_pipe_create", "kvx_map_host",
-            "kvx_host_pipe_destroy", "kvx_set_test_wait")
+            "kvx_host_pipe_destroy", "kvx_set_test_wait", "kvx_get_kernel")
 
 
 def lib():
@@ -173,6 +173,8 @@ def lib():
     L.kvx_map_host.argtypes = [vp, ctypes.POINTER(kvx_src), i32, vp, ctypes.POINTER(kvx_tgt), vp]
     L.kvx_host_pipe_destroy.argtypes = [vp]
     L.kvx_set_test_wait.argtypes = [vp, ctypes.c_uint64, i64]
+    L.kvx_get_kernel.argtypes = [vp, i32, ctypes.POINTER(i32)]
+    L.kvx_get_kernel.restype = ctypes.c_int
     L.kvx_set_test_wait.restype = ctypes.c_int
     for name in ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
                  "kvx_set_kernel", "kvx_get_status", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms",
@@ -227,6 +229,18 @@ def kvx_map_noalloc(mapper, device, src, batch, tokens_per_seq, positions_ptr, t
                                  int(tokens_per_seq), positions_ptr, ctypes.byref(tgt), stream,
                                  ctypes.byref(st) if want_status else None), "kvx_map_noalloc")
     return st.value if want_status else None
+
+
+KERNEL_NAMES = {1: "simt_map_kernel (fp32 FFMA)", 2: "tc_map_kernel (tcgen05, sm_103a)",
+                3: "xh_strip_kernel + tc_xh_kernel (tcgen05 pair GEMM, sm_103a)"}
+
+
+def kvx_get_kernel(ctx, paged=False):
+    """1 SIMT, 2 per-head tensor-core kernel, 3 cross-head tensor-core kernel (see
+    include/kvx.h): the kernel kvx_map runs on ctx."""
+    out = ctypes.c_int32(0)
+    _check(lib().kvx_get_kernel(ctx, int(bool(paged)), ctypes.byref(out)), "kvx_get_kernel")
+    return out.value
 
 
 def kvx_set_test_wait(ctx, wait_limit_ns, skip_bias_row=-1):

@@ -317,3 +317,9 @@ def test_set_test_wait_rejects_bad_arguments():
         with pytest.raises(kvx.KvxError) as e:
             kvx.kvx_set_test_wait(*args)
         assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+
+
+def test_get_kernel_rejects_null_arguments():
+    with pytest.raises(kvx.KvxError) as e:
+        kvx.kvx_get_kernel(None)
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG

@@ -76,18 +76,43 @@ def test_tiny_fp32_full():
 def test_bf16_small_full(kname, over):
     name = "qwen3_14b_32b_b8x1024_k4"
     if kname == "tc":
-        if over["k"] > 4:
-            w = syn.workload(name, **over)
-            ctx, _, _, _ = make_ctx(w)
-            try:
-                with pytest.raises(kvx.KvxError) as e:
-                    kvx.kvx_set_kernel(ctx, KERNELS[kname])
-                assert e.value.status == kvx.KVX_ERR_UNSUPPORTED
-            finally:
-                kvx.kvx_destroy(ctx)
-            return
         _kernel_or_skip(syn.workload(name, **over), KERNELS[kname])
     _small(name, KERNELS[kname], **over)
+
+
+@pytest.mark.parametrize("over", [
+    dict(Ls=10, Lt=5, H=2, B=1, T=200, k=5),                 # k = 5, one ragged tile
+    dict(Ls=12, Lt=4, H=4, B=2, T=300, k=8),                 # k = 8, B > 1
+    dict(Ls=9, Lt=3, H=2, B=1, T=257, k=8, scores="uniform", theta_t=5e5),
+])
+def test_per_head_beyond_four_layers_on_tensor_cores(over):
+    """Per-head mappers with k > 4 (more selected layers than the per-head kernel keeps in
+    tensor memory) run on the cross-head tensor-core kernel with W widened by zeros outside
+    each head's rows: AUTO picks it, every element matches the oracle, and repeated launches
+    agree."""
+    name = "qwen3_14b_32b_b8x1024_k4"
+    w = syn.workload(name, **over)
+    ctx, sel, W, b = make_ctx(w)
+    try:
+        assert kvx.kvx_get_kernel(ctx) == 3 and kvx.kvx_get_kernel(ctx, paged=True) == 3
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w)
+        rk, rv, ak, av = oracle_full(w, sk, sv, pos, sel, W, b)
+        first = None
+        for rep in range(3):
+            tk, tv, status = run_contiguous(ctx, w, sk, sv, pos)
+            assert status == kvx.KVX_OK
+            ok, ratio, rms, nbad = check(w, [to_f64(tk), to_f64(tv)], [rk, rv], [ak, av])
+            assert ok, "%d elements out of tolerance (worst %.3g x bound)" % (nbad, ratio)
+            if first is None:
+                first = (tk.clone(), tv.clone())
+            else:
+                assert torch.equal(tk, first[0]) and torch.equal(tv, first[1])
+        kvx.kvx_set_kernel(ctx, kvx.KVX_KERNEL_SIMT)
+        assert kvx.kvx_get_kernel(ctx) == 1
+    finally:
+        kvx.kvx_destroy(ctx)
 
 
 @pytest.mark.parametrize("over", [
@@ -426,20 +451,34 @@ def test_cross_head_tc_small(over):
         kvx.kvx_destroy(ctx)
 
 
-def test_cross_head_tc_paged_is_refused_but_auto_maps_it():
-    """The cross-head tensor-core kernel writes contiguous targets: an explicit TCGEN05
-    choice on a paged target is refused before any launch, AUTO maps it with SIMT."""
-    w = syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4", Ls=4, Lt=2, H=2, B=2, T=20, k=2,
-                     len_range=(3, 40), head_mix="cross_head")
-    ctx, sel, W, b = make_ctx(w, kernel=kvx.KVX_KERNEL_TCGEN05)
+@pytest.mark.parametrize("kname", ["simt", "tc"])
+def test_cross_head_paged_small_full(kname):
+    """The paper's cross-head mapper writing into a paged cache (16-token blocks, unaligned
+    starts, a block table per sequence): every slot of two turns against the oracle, untouched
+    slots keep their sentinel; the tensor-core kernel is also launched repeatedly."""
+    w = syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4", Ls=4, Lt=3, H=2, B=3, T=150, k=2,
+                     len_range=(3, 70), head_mix="cross_head")
+    ctx, sel, W, b = make_ctx(w, kernel=KERNELS[kname])
     try:
-        with pytest.raises(kvx.KvxError) as e:
-            _paged_run(w, 0, syn.initial_lengths(w), ctx)
-        assert e.value.status == kvx.KVX_ERR_UNSUPPORTED
-        kvx.kvx_set_kernel(ctx, kvx.KVX_KERNEL_AUTO)
-        _check_paged(w, ctx, sel, W, b, 0, syn.initial_lengths(w), sample_rows(w, 12, turn_T=w.T))
+        L0 = syn.initial_lengths(w)
+        rows = np.array([(bb, t) for bb in range(w.B) for t in range(w.T)], dtype=np.int64)
+        for turn in (0, 1, 0, 1):
+            _check_paged(w, ctx, sel, W, b, turn, L0, rows)
     finally:
         kvx.kvx_destroy(ctx)
+
+
+def test_cross_head_paged_full_size_sampled():
+    """Cross-head mapper (k = 4, every KV head of the selected layers) into the paged
+    Qwen3-32B -> 14B turn (16 x 2048 new tokens at their absolute positions) on the tensor
+    cores: sampled rows against the oracle, every slot checked."""
+    w = syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4", head_mix="cross_head")
+    ctx, sel, W, b = make_ctx(w, kernel=kvx.KVX_KERNEL_TCGEN05)
+    try:
+        _check_paged(w, ctx, sel, W, b, 3, syn.initial_lengths(w), sample_rows(w, 24, seed=3))
+    finally:
+        kvx.kvx_destroy(ctx)
+        torch.cuda.empty_cache()
 
 
 def test_cross_head_full_size_sampled():
