@@ -663,7 +663,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                             pack_bf16x2(yhi[6], yhi[7]));
           v[3] = make_uint4(pack_bf16x2(yhi[8], yhi[9]), pack_bf16x2(yhi[10], yhi[11]),
                             pack_bf16x2(yhi[12], yhi[13]), pack_bf16x2(yhi[14], yhi[15]));
-          if (warp_tma) {
+          if (warp_tma || A.paged) {
             // two 32-row x 64-byte pieces (channels 32g.. and 64+32g..), 64-byte swizzle:
             // 16-byte chunk index XOR (row / 2) % 4
             const int sw = (lane >> 1) & 3;
@@ -682,7 +682,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&bias_empty[bslot]));
-        if (!A.paged) {
+        if (A.paged) {
+          // Paged rows leave the staging buffer in 64-byte pieces: in store i lanes 8m ..
+          // 8m + 7 write row 4i + m, lanes 4 apart the two pieces (channels 32g.. and
+          // 64 + 32g..), so each group of four lanes writes one whole 64-byte piece.  The
+          // row's block offset comes from the lane that owns the row.
+          const int64_t lay_off = static_cast<int64_t>(l) * A.ts[0];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int rr = 4 * i + (lane >> 3);
+            const int piece = (lane >> 2) & 1, chunk = lane & 3;
+            const uint32_t off_lo = __shfl_sync(0xffffffffu, static_cast<uint32_t>(row_off), rr);
+            const uint32_t off_hi = __shfl_sync(0xffffffffu, static_cast<uint32_t>(static_cast<uint64_t>(row_off) >> 32), rr);
+            const int ok_row = __shfl_sync(0xffffffffu, valid ? 1 : 0, rr);
+            const int sw = (rr >> 1) & 3;
+            const uint4 v = *reinterpret_cast<const uint4*>(sb + rr * 64 + piece * kPieceBytes + ((chunk ^ sw) << 4));
+            if (ok_row) {
+              const int64_t roff = static_cast<int64_t>((static_cast<uint64_t>(off_hi) << 32) | off_lo);
+              st_global_hint(dst + lay_off + roff + 64 * piece + 32 * g + 8 * chunk, v, st_pol);
+            }
+          }
+          __syncwarp();   // the staging buffer is read before the next layer writes it
+        } else {
           // every contiguous-target layer commits one bulk group per warp (empty when the
           // warp wrote its rows directly), so the group count above identifies the buffer
           if (warp_tma) {
