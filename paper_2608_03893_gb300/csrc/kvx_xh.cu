@@ -1,7 +1,9 @@
 // Tensor-core path for the cross-head feature layout (the paper's mapper: every KV head of
 // the k selected source layers is a feature of every target head, d_s = k n_kv d, Sec. 3.1
 // and Sec. 3.2).  bf16 caches and weights, head_dim 128, half-split RoPE pairs, an even
-// number of KV heads, contiguous targets.
+// number of KV heads, contiguous or paged targets.  Per-head mappers with more selected
+// layers than the per-head kernel holds (k > 4) run here too, on W widened at create time
+// with zeros outside each target head's rows.
 //
 // For target layer l and K|V the map is one GEMM over the tokens,
 //   Y[tok][h d + c] = sum_{j, h'} X_{sel[l][j], h'}[tok][:] . W[l][kv][h][(j n_kv + h') d + :][c]
@@ -22,7 +24,8 @@
 //    pass-fastest and token-tile next, so the clusters in flight share one (layer, K|V)
 //    block of W^T (k n_kv d x n_kv d bf16) in L2 and the four passes of a tile share its
 //    source tiles.  Epilogue per pass: TMEM -> registers, + bias, (keys) target RoPE,
-//    bf16, one TMA store per warp and head.
+//    bf16, one TMA store per warp and head (contiguous targets) or 16-byte stores through
+//    the block table (paged targets).
 //
 // Warp roles (384 threads): warp 0 one thread polling two streams (stage loads: A and B
 // halves of both CTAs complete on the rank-0 CTA's stage barrier; each unit's bias rows);
