@@ -67,8 +67,10 @@ typedef enum { KVX_ROPE_HALF = 0, KVX_ROPE_INTERLEAVED = 1 } kvx_rope_style;
 typedef enum { KVX_PER_HEAD = 0, KVX_CROSS_HEAD = 1 } kvx_head_mix;
 
 /* Which kernel kvx_map launches.  AUTO picks a tensor-core (tcgen05) kernel when the
- * shape allows it (bf16 caches, head_dim 128, HALF; PER_HEAD with k <= 4, or CROSS_HEAD
- * with an even head count; contiguous or paged targets) and the fp32 SIMT kernel otherwise.
+ * shape allows it (bf16 caches, head_dim 128, HALF or INTERLEAVED pairs; PER_HEAD with
+ * k <= 4 on the per-head kernel; CROSS_HEAD, and PER_HEAD with k > 4 on W widened with
+ * zeros, on the cross-head kernel, which needs an even head count; contiguous or paged
+ * targets) and the fp32 SIMT kernel otherwise.
  * fp32 weights run on the tensor cores split into bf16 hi = bf16(w) and lo = bf16(w - hi)
  * (twice the MMAs; the contraction follows the fp32 W to within 2^-17 of each weight).
  * The CROSS_HEAD tensor-core kernel keeps a workspace for the stripped source keys

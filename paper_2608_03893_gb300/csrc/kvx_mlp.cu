@@ -628,7 +628,7 @@ KVX_API kvx_status kvx_mlp_map(const kvx_mlp_config* cfg, const kvx_src* src, in
     // strip every source key once
     P.hf = cfg->rope_numerics == KVX_ROPE_HF;
     launch_key_strip(src->k, src->stride, d_strip, positions, cfg->src_layers, H, batch, tokens_per_seq, tmp.rope, sms, st,
-                     P.hf);
+                     P.hf, 0);
     const size_t smem = mlp_smem_bytes();
     if ((e = cudaFuncSetAttribute(tc_mlp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   static_cast<int>(smem))) != cudaSuccess) {

@@ -1,5 +1,5 @@
 // Tensor-core mapping kernel for sm_103a (tcgen05 + TMEM + TMA), bf16 caches, bf16 or
-// fp32 weights, head_dim 128, per-head features, half-split RoPE pairs, k <= 4.
+// fp32 weights, head_dim 128, per-head features, half-split or interleaved RoPE pairs, k <= 4.
 //
 // It computes Eq. ridge_kv with the Sec. 3.3 RoPE composition,
 //   K_t^{l,h} = R_t(t) ( [R_s(t)^-1 K_s^{sel[l][j]}[h]]_j W_K^{l,h} + b_K^{l,h} ),
@@ -171,12 +171,48 @@ __device__ __forceinline__ Unit decode_unit(int u, int H, int B, int pairs, uint
 
 __device__ __forceinline__ void report(int32_t* status, int code) { atomicCAS(status, 0, code); }
 
+// Rotation of two RoPE pairs (x0.x, x1.x) and (x0.y, x1.y) by the angles with cosines c and
+// sines s, one f32x2 instruction per step (each lane rounds like the scalar fmul / fma it
+// replaces).  Strip (rotation by -t*omega): x0' = x0 c + x1 s, x1' = x1 c - x0 s; the sums
+// are left unrounded for the bf16 pack.  Apply (rotation by +t*omega): y0' = y0 c - y1 s,
+// y1' = y0 s + y1 c.  kHF: the operands are bf16 values, every product is rounded to bf16.
+template <bool kHF>
+__device__ __forceinline__ void rope_strip2(float2 x0, float2 x1, float2 c, float2 s, float2& r0, float2& r1) {
+  if constexpr (kHF) {
+    const float2 ac = bf16_round2(__fmul2_rn(x0, c)), bs = bf16_round2(__fmul2_rn(x1, s));
+    const float2 bc = bf16_round2(__fmul2_rn(x1, c)), as = bf16_round2(__fmul2_rn(x0, s));
+    r0 = make_float2(__fadd_rn(ac.x, bs.x), __fadd_rn(ac.y, bs.y));
+    r1 = make_float2(__fsub_rn(bc.x, as.x), __fsub_rn(bc.y, as.y));
+  } else {
+    const float2 as = __fmul2_rn(x0, s);
+    r0 = __ffma2_rn(x0, c, __fmul2_rn(x1, s));
+    r1 = __ffma2_rn(x1, c, make_float2(-as.x, -as.y));
+  }
+}
+
+// kHF: the mapped key is first rounded to bf16 (the tensor the forward rotates).
+template <bool kHF>
+__device__ __forceinline__ void rope_apply2(float2 y0, float2 y1, float2 c, float2 s, float2& r0, float2& r1) {
+  if constexpr (kHF) {
+    const float2 b0 = bf16_round2(y0), b1 = bf16_round2(y1);
+    const float2 p0 = bf16_round2(__fmul2_rn(b0, c)), p1 = bf16_round2(__fmul2_rn(b1, s));
+    const float2 p2 = bf16_round2(__fmul2_rn(b1, c)), p3 = bf16_round2(__fmul2_rn(b0, s));
+    r0 = make_float2(__fsub_rn(p0.x, p1.x), __fsub_rn(p0.y, p1.y));
+    r1 = make_float2(__fadd_rn(p2.x, p3.x), __fadd_rn(p2.y, p3.y));
+  } else {
+    const float2 u = __fmul2_rn(y1, s);
+    r0 = __ffma2_rn(y0, c, make_float2(-u.x, -u.y));
+    r1 = __ffma2_rn(y0, s, __fmul2_rn(y1, c));
+  }
+}
+
 // ------------------------------------------------------------------------ kernel --
 
 // kHF: the Hugging Face forward's RoPE rounding (kvx_rope_numerics): cos / sin of the fp32
 // angle rounded to bf16, every product and sum of the rotations rounded to bf16.
 // kParts: W stages per use, 1 for bf16 weights, 2 (hi, lo) for fp32 weights.
-template <bool kHF, int kParts>
+// kIL: interleaved RoPE pairs (2i, 2i+1) instead of half-split pairs (i, i + 64).
+template <bool kHF, int kParts, bool kIL>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     tc_map_kernel(const __grid_constant__ TcParams P) {
   extern __shared__ __align__(1024) uint8_t smem[];
@@ -558,7 +594,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       if (un.kv == 0) {
 #pragma unroll
         for (int m = 0; m < 32; ++m) {
-          const int i = 32 * g + m;
+          // pair of slot m: half-split pairs (c, c + 64) for c = 32g + m; interleaved pairs
+          // (c, c + 1) for the 16 even c in [32g, 32g + 32) (m < 16), then in 64 + [32g, 32g + 32)
+          const int i = kIL ? (m < 16 ? 16 * g + m : 32 + 16 * g + (m - 16)) : 32 * g + m;
           if constexpr (kHF) {
             sincosf(__fmul_rn(static_cast<float>(p), P.rope.wt_hi[i]), &sn[m], &cs[m]);
             sn[m] = bf16_round(sn[m]);
@@ -628,30 +666,36 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             yhi[j + 2] = __fadd_rn(__uint_as_float(hi[j + 2]), b1.z);
             yhi[j + 3] = __fadd_rn(__uint_as_float(hi[j + 3]), b1.w);
           }
-          if (un.kv == 0) {
-            // target RoPE, two pairs per f32x2 instruction (each lane rounds like the
-            // scalar fmul / fma it replaces): y0' = y0 c - y1 s, y1' = y0 s + y1 c
+          if (un.kv == 0 && !kIL) {
+            // target RoPE on pairs (c, c + 64): channel c_lo + j of ylo with the same of yhi
 #pragma unroll
             for (int j = 0; j < 16; j += 2) {
               const float2 c = make_float2(cs[16 * rnd + j], cs[16 * rnd + j + 1]);
               const float2 sv = make_float2(sn[16 * rnd + j], sn[16 * rnd + j + 1]);
-              const float2 y0 = make_float2(ylo[j], ylo[j + 1]), y1 = make_float2(yhi[j], yhi[j + 1]);
               float2 r0, r1;
-              if constexpr (kHF) {   // the key as bf16, products and sums rounded to bf16
-                const float2 b0 = bf16_round2(y0), b1 = bf16_round2(y1);
-                const float2 p0 = bf16_round2(__fmul2_rn(b0, c)), p1 = bf16_round2(__fmul2_rn(b1, sv));
-                const float2 p2 = bf16_round2(__fmul2_rn(b1, c)), p3 = bf16_round2(__fmul2_rn(b0, sv));
-                r0 = make_float2(__fsub_rn(p0.x, p1.x), __fsub_rn(p0.y, p1.y));
-                r1 = make_float2(__fadd_rn(p2.x, p3.x), __fadd_rn(p2.y, p3.y));
-              } else {
-                const float2 u = __fmul2_rn(y1, sv);
-                r0 = __ffma2_rn(y0, c, make_float2(-u.x, -u.y));
-                r1 = __ffma2_rn(y0, sv, __fmul2_rn(y1, c));
-              }
+              rope_apply2<kHF>(make_float2(ylo[j], ylo[j + 1]), make_float2(yhi[j], yhi[j + 1]), c, sv, r0, r1);
               ylo[j] = r0.x;
               ylo[j + 1] = r0.y;
               yhi[j] = r1.x;
               yhi[j + 1] = r1.y;
+            }
+          } else if (un.kv == 0) {
+            // target RoPE on pairs (c, c + 1): channels c_lo + j, c_lo + j + 1 of ylo (slot
+            // 8 rnd + j / 2) and of yhi (slot 16 + 8 rnd + j / 2), two pairs per step
+#pragma unroll
+            for (int j = 0; j < 16; j += 4) {
+#pragma unroll
+              for (int hv = 0; hv < 2; ++hv) {
+                float* y = hv ? yhi : ylo;
+                const int m = 16 * hv + 8 * rnd + j / 2;
+                float2 r0, r1;
+                rope_apply2<kHF>(make_float2(y[j], y[j + 2]), make_float2(y[j + 1], y[j + 3]),
+                                 make_float2(cs[m], cs[m + 1]), make_float2(sn[m], sn[m + 1]), r0, r1);
+                y[j] = r0.x;
+                y[j + 2] = r0.y;
+                y[j + 1] = r1.x;
+                y[j + 3] = r1.y;
+              }
             }
           }
           uint4 v[4];
@@ -799,27 +843,25 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             wb[4 * ci + 2] = vb.z;
             wb[4 * ci + 3] = vb.w;
           }
-          if (un.kv == 0) {
+          if (un.kv == 0 && !kIL) {
 #pragma unroll
-            for (int w = 0; w < 8; ++w) {   // pairs 16c + 2w and 16c + 2w + 1
+            for (int w = 0; w < 8; ++w) {   // pairs 16c + 2w and 16c + 2w + 1: (f, f + 64)
               const int m0 = 16 * c + 2 * w, m1 = m0 + 1;
-              const float2 a = make_float2(bf16_lo(wa[w]), bf16_hi(wa[w]));
-              const float2 b = make_float2(bf16_lo(wb[w]), bf16_hi(wb[w]));
-              const float2 cc = make_float2(cs[m0], cs[m1]), ss = make_float2(sn[m0], sn[m1]);
-              // rotation by -t*omega: a' = a c + b s, b' = b c - a s, two pairs per f32x2
-              // instruction (each lane rounds like the scalar fmul / fma)
-              if constexpr (kHF) {   // products rounded to bf16, then the sums (by the pack)
-                const float2 ac = bf16_round2(__fmul2_rn(a, cc)), bs = bf16_round2(__fmul2_rn(b, ss));
-                const float2 bc = bf16_round2(__fmul2_rn(b, cc)), as = bf16_round2(__fmul2_rn(a, ss));
-                wa[w] = pack_bf16x2(__fadd_rn(ac.x, bs.x), __fadd_rn(ac.y, bs.y));
-                wb[w] = pack_bf16x2(__fsub_rn(bc.x, as.x), __fsub_rn(bc.y, as.y));
-              } else {
-                const float2 as = __fmul2_rn(a, ss);
-                const float2 ra = __ffma2_rn(a, cc, __fmul2_rn(b, ss));
-                const float2 rb = __ffma2_rn(b, cc, make_float2(-as.x, -as.y));
-                wa[w] = pack_bf16x2(ra.x, ra.y);
-                wb[w] = pack_bf16x2(rb.x, rb.y);
-              }
+              float2 ra, rb;
+              rope_strip2<kHF>(make_float2(bf16_lo(wa[w]), bf16_hi(wa[w])), make_float2(bf16_lo(wb[w]), bf16_hi(wb[w])),
+                               make_float2(cs[m0], cs[m1]), make_float2(sn[m0], sn[m1]), ra, rb);
+              wa[w] = pack_bf16x2(ra.x, ra.y);
+              wb[w] = pack_bf16x2(rb.x, rb.y);
+            }
+          } else if (un.kv == 0) {
+#pragma unroll
+            for (int w = 0; w < 8; ++w) {   // pairs 8c + w (word wa[w]) and 32 + 8c + w (word wb[w]): (f, f + 1)
+              const int m0 = 8 * c + w, m1 = 32 + 8 * c + w;
+              float2 r0, r1;
+              rope_strip2<kHF>(make_float2(bf16_lo(wa[w]), bf16_lo(wb[w])), make_float2(bf16_hi(wa[w]), bf16_hi(wb[w])),
+                               make_float2(cs[m0], cs[m1]), make_float2(sn[m0], sn[m1]), r0, r1);
+              wa[w] = pack_bf16x2(r0.x, r1.x);
+              wb[w] = pack_bf16x2(r0.y, r1.y);
             }
           }
           tmem_st_x8(scol + 8 * c, wa);        // TMEM columns 8c .. 8c+7
@@ -958,7 +1000,6 @@ bool tc_supported(const kvx_ctx* c, std::string* why) {
   if (c->cache_dtype != KVX_BF16) w = "needs bf16 caches";
   else if (c->d != kD) w = "needs head_dim 128";
   else if (c->head_mix != KVX_PER_HEAD) w = "needs per-head features";
-  else if (c->rope_style != KVX_ROPE_HALF) w = "needs half-split RoPE pairs";
   else if (c->k > kTSlots) w = "needs k <= 4 (one target layer's source tiles must fit in tensor memory)";
   else if (static_cast<int64_t>(c->Lt) * 2 * c->H * kD > INT_MAX) w = "too many W rows";
   if (why) *why = w;
@@ -1109,8 +1150,12 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   P.skip_bias = static_cast<int32_t>(c->skip_bias_row);
   const size_t smem = smem_bytes();
   const bool hf = c->rope_numerics == KVX_ROPE_HF;
-  void (*kernel)(TcParams) = c->weight_dtype == KVX_F32 ? (hf ? tc_map_kernel<true, 2> : tc_map_kernel<false, 2>)
-                                                        : (hf ? tc_map_kernel<true, 1> : tc_map_kernel<false, 1>);
+  const bool il = c->rope_style == KVX_ROPE_INTERLEAVED;
+  void (*const kernels[8])(TcParams) = {tc_map_kernel<false, 1, false>, tc_map_kernel<true, 1, false>,
+                                        tc_map_kernel<false, 2, false>, tc_map_kernel<true, 2, false>,
+                                        tc_map_kernel<false, 1, true>,  tc_map_kernel<true, 1, true>,
+                                        tc_map_kernel<false, 2, true>,  tc_map_kernel<true, 2, true>};
+  void (*kernel)(TcParams) = kernels[(il ? 4 : 0) + (c->weight_dtype == KVX_F32 ? 2 : 0) + (hf ? 1 : 0)];
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) {
     set_error(std::string("kvx_map: smem attribute: ") + cudaGetErrorString(e));

@@ -1,6 +1,6 @@
 // Tensor-core path for the cross-head feature layout (the paper's mapper: every KV head of
 // the k selected source layers is a feature of every target head, d_s = k n_kv d, Sec. 3.1
-// and Sec. 3.2).  bf16 caches and weights, head_dim 128, half-split RoPE pairs, an even
+// and Sec. 3.2).  bf16 caches and weights, head_dim 128, half-split or interleaved RoPE pairs, an even
 // number of KV heads, contiguous or paged targets.  Per-head mappers with more selected
 // layers than the per-head kernel holds (k > 4) run here too, on W widened at create time
 // with zeros outside each target head's rows.
@@ -88,6 +88,7 @@ struct XhParams {
   int32_t Lt, H, k, pairs, n_units, out_bh;
   int32_t lo_steps;       // fp32 weights: k n_kv further K steps over the same source tiles with W_lo
   int32_t hf;             // the Hugging Face forward's RoPE rounding (kvx_rope_numerics)
+  int32_t il;             // interleaved RoPE pairs (2i, 2i+1) instead of (i, i + 64)
   RopeTables rope;
 };
 
@@ -114,11 +115,13 @@ __device__ __forceinline__ void xreport(int32_t* status, int code) { atomicCAS(s
 
 // ---------------------------------------------------------------- strip kernel --
 // Thread = (sequence b, token t, group of four RoPE pairs i0..i0+3); it rotates those
-// pairs of every (source layer, head) by -t*omega_s and rounds them to bf16.
+// pairs of every (source layer, head) by -t*omega_s and rounds them to bf16.  Half-split
+// pairs (i, i + 64) take channels 4 grp .. 4 grp + 3 and 64 + the same; interleaved pairs
+// (2i, 2i+1) take channels 8 grp .. 8 grp + 7.
 __global__ void __launch_bounds__(256) xh_strip_kernel(const __nv_bfloat16* __restrict__ src, int64_t s_l,
                                                        int64_t s_b, int64_t s_h, int64_t s_t,
                                                        __nv_bfloat16* __restrict__ ws, const int32_t* __restrict__ pos,
-                                                       int Ls, int H, int B, int T, RopeTables rope, int hf) {
+                                                       int Ls, int H, int B, int T, RopeTables rope, int hf, int il) {
   const int64_t n = static_cast<int64_t>(B) * T * 16;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -142,30 +145,56 @@ __global__ void __launch_bounds__(256) xh_strip_kernel(const __nv_bfloat16* __re
     for (int L = 0; L < Ls; ++L) {
       for (int h = 0; h < H; ++h) {
         const __nv_bfloat16* row = src + L * s_l + b * s_b + h * s_h + static_cast<int64_t>(t) * s_t;
-        const uint2 va = *reinterpret_cast<const uint2*>(row + 4 * grp);        // a: pairs' first halves
-        const uint2 vb = *reinterpret_cast<const uint2*>(row + 64 + 4 * grp);   // b: second halves
-        const uint32_t wa[2] = {va.x, va.y}, wb[2] = {vb.x, vb.y};
+        uint4 vi;
+        if (il) {
+          vi = *reinterpret_cast<const uint4*>(row + 8 * grp);
+        } else {
+          const uint2 va = *reinterpret_cast<const uint2*>(row + 4 * grp);        // first halves
+          const uint2 vb = *reinterpret_cast<const uint2*>(row + 64 + 4 * grp);   // second halves
+          vi = make_uint4(va.x, vb.x, va.y, vb.y);
+        }
         uint32_t oa[2], ob[2];
 #pragma unroll
         for (int w = 0; w < 2; ++w) {
-          const float a0 = bf16_lo(wa[w]), a1 = bf16_hi(wa[w]);
-          const float b0 = bf16_lo(wb[w]), b1 = bf16_hi(wb[w]);
+          // half-split: vi = (a01, b01, a23, b23) with a = first members; interleaved: vi
+          // = (pair 0, pair 1, pair 2, pair 3), one pair per word
+          const uint32_t u0 = w ? vi.z : vi.x, u1 = w ? vi.w : vi.y;
+          float a0, a1, b0, b1;
+          if (il) {
+            a0 = bf16_lo(u0); b0 = bf16_hi(u0); a1 = bf16_lo(u1); b1 = bf16_hi(u1);
+          } else {
+            a0 = bf16_lo(u0); a1 = bf16_hi(u0); b0 = bf16_lo(u1); b1 = bf16_hi(u1);
+          }
           const int m0 = 2 * w, m1 = 2 * w + 1;
+          float na0, na1, nb0, nb1;
           if (hf) {   // each product and sum rounded to bf16
             auto r = [](float x) { return __bfloat162float(__float2bfloat16_rn(x)); };
-            oa[w] = pack_bf16x2(r(__fadd_rn(r(__fmul_rn(a0, c[m0])), r(__fmul_rn(b0, s[m0])))),
-                                r(__fadd_rn(r(__fmul_rn(a1, c[m1])), r(__fmul_rn(b1, s[m1])))));
-            ob[w] = pack_bf16x2(r(__fsub_rn(r(__fmul_rn(b0, c[m0])), r(__fmul_rn(a0, s[m0])))),
-                                r(__fsub_rn(r(__fmul_rn(b1, c[m1])), r(__fmul_rn(a1, s[m1])))));
+            na0 = r(__fadd_rn(r(__fmul_rn(a0, c[m0])), r(__fmul_rn(b0, s[m0]))));
+            na1 = r(__fadd_rn(r(__fmul_rn(a1, c[m1])), r(__fmul_rn(b1, s[m1]))));
+            nb0 = r(__fsub_rn(r(__fmul_rn(b0, c[m0])), r(__fmul_rn(a0, s[m0]))));
+            nb1 = r(__fsub_rn(r(__fmul_rn(b1, c[m1])), r(__fmul_rn(a1, s[m1]))));
           } else {
             // rotation by -t*omega: a' = a c + b s, b' = b c - a s
-            oa[w] = pack_bf16x2(__fmaf_rn(a0, c[m0], __fmul_rn(b0, s[m0])), __fmaf_rn(a1, c[m1], __fmul_rn(b1, s[m1])));
-            ob[w] = pack_bf16x2(__fmaf_rn(b0, c[m0], -__fmul_rn(a0, s[m0])), __fmaf_rn(b1, c[m1], -__fmul_rn(a1, s[m1])));
+            na0 = __fmaf_rn(a0, c[m0], __fmul_rn(b0, s[m0]));
+            na1 = __fmaf_rn(a1, c[m1], __fmul_rn(b1, s[m1]));
+            nb0 = __fmaf_rn(b0, c[m0], -__fmul_rn(a0, s[m0]));
+            nb1 = __fmaf_rn(b1, c[m1], -__fmul_rn(a1, s[m1]));
+          }
+          if (il) {
+            oa[w] = pack_bf16x2(na0, nb0);
+            ob[w] = pack_bf16x2(na1, nb1);
+          } else {
+            oa[w] = pack_bf16x2(na0, na1);
+            ob[w] = pack_bf16x2(nb0, nb1);
           }
         }
         __nv_bfloat16* out = ws + ((((static_cast<int64_t>(L) * B + b) * H + h) * T + t) * kXD);
-        *reinterpret_cast<uint2*>(out + 4 * grp) = make_uint2(oa[0], oa[1]);
-        *reinterpret_cast<uint2*>(out + 64 + 4 * grp) = make_uint2(ob[0], ob[1]);
+        if (il) {
+          *reinterpret_cast<uint4*>(out + 8 * grp) = make_uint4(oa[0], ob[0], oa[1], ob[1]);
+        } else {
+          *reinterpret_cast<uint2*>(out + 4 * grp) = make_uint2(oa[0], oa[1]);
+          *reinterpret_cast<uint2*>(out + 64 + 4 * grp) = make_uint2(ob[0], ob[1]);
+        }
       }
     }
   }
@@ -407,7 +436,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
       if (un.kv == 0) {
 #pragma unroll
         for (int m = 0; m < 32; ++m) {
-          const int i = 32 * g + m;
+          // pair of slot m: half-split pairs (c, c + 64) for c = 32g + m; interleaved pairs
+          // (c, c + 1) for the 16 even c in [32g, 32g + 32) (m < 16), then in 64 + [32g, 32g + 32)
+          const int i = P.il ? (m < 16 ? 16 * g + m : 32 + 16 * g + (m - 16)) : 32 * g + m;
           if (P.hf) {   // cos / sin of the fp32 angle, rounded to bf16
             sincosf(__fmul_rn(static_cast<float>(p), P.rope.wt_hi[i]), &sn[m], &cs[m]);
             sn[m] = bf16_round(sn[m]);
@@ -464,29 +495,52 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
             yhi[j + 2] = __fadd_rn(__uint_as_float(hi[j + 2]), b1.z);
             yhi[j + 3] = __fadd_rn(__uint_as_float(hi[j + 3]), b1.w);
           }
-          if (un.kv == 0) {
-            // target RoPE, two pairs per f32x2 instruction: y0' = y0 c - y1 s, y1' = y0 s + y1 c
+          // target RoPE, two pairs per f32x2 instruction: y0' = y0 c - y1 s, y1' = y0 s + y1 c;
+          // HF numerics: the key as bf16, products and sums rounded to bf16
+          auto rot = [&](float2 y0, float2 y1, float2 c, float2 sv, float2& r0, float2& r1) {
+            if (P.hf) {
+              const float2 b0 = bf16_round2(y0), b1 = bf16_round2(y1);
+              const float2 p0 = bf16_round2(__fmul2_rn(b0, c)), p1 = bf16_round2(__fmul2_rn(b1, sv));
+              const float2 p2 = bf16_round2(__fmul2_rn(b1, c)), p3 = bf16_round2(__fmul2_rn(b0, sv));
+              r0 = make_float2(__fsub_rn(p0.x, p1.x), __fsub_rn(p0.y, p1.y));
+              r1 = make_float2(__fadd_rn(p2.x, p3.x), __fadd_rn(p2.y, p3.y));
+            } else {
+              const float2 uu = __fmul2_rn(y1, sv);
+              r0 = __ffma2_rn(y0, c, make_float2(-uu.x, -uu.y));
+              r1 = __ffma2_rn(y0, sv, __fmul2_rn(y1, c));
+            }
+          };
+          if (un.kv == 0 && !P.il) {   // pairs (c, c + 64): channel c_lo + j of ylo with the same of yhi
 #pragma unroll
             for (int j = 0; j < 16; j += 2) {
-              const float2 c = make_float2(cs[16 * rnd + j], cs[16 * rnd + j + 1]);
-              const float2 sv = make_float2(sn[16 * rnd + j], sn[16 * rnd + j + 1]);
-              const float2 y0 = make_float2(ylo[j], ylo[j + 1]), y1 = make_float2(yhi[j], yhi[j + 1]);
               float2 r0, r1;
-              if (P.hf) {   // the key as bf16, products and sums rounded to bf16
-                const float2 b0 = bf16_round2(y0), b1 = bf16_round2(y1);
-                const float2 p0 = bf16_round2(__fmul2_rn(b0, c)), p1 = bf16_round2(__fmul2_rn(b1, sv));
-                const float2 p2 = bf16_round2(__fmul2_rn(b1, c)), p3 = bf16_round2(__fmul2_rn(b0, sv));
-                r0 = make_float2(__fsub_rn(p0.x, p1.x), __fsub_rn(p0.y, p1.y));
-                r1 = make_float2(__fadd_rn(p2.x, p3.x), __fadd_rn(p2.y, p3.y));
-              } else {
-                const float2 uu = __fmul2_rn(y1, sv);
-                r0 = __ffma2_rn(y0, c, make_float2(-uu.x, -uu.y));
-                r1 = __ffma2_rn(y0, sv, __fmul2_rn(y1, c));
-              }
+              rot(make_float2(ylo[j], ylo[j + 1]), make_float2(yhi[j], yhi[j + 1]),
+                  make_float2(cs[16 * rnd + j], cs[16 * rnd + j + 1]), make_float2(sn[16 * rnd + j], sn[16 * rnd + j + 1]),
+                  r0, r1);
               ylo[j] = r0.x;
               ylo[j + 1] = r0.y;
               yhi[j] = r1.x;
               yhi[j + 1] = r1.y;
+            }
+          } else if (un.kv == 0) {
+            // pairs (c, c + 1): channels c_lo + j, c_lo + j + 1 of ylo (slot 8 rnd + j / 2) and
+            // of yhi (slot 16 + 8 rnd + j / 2)
+#pragma unroll
+            for (int j = 0; j < 16; j += 4) {
+              const int m = 8 * rnd + j / 2;
+              float2 r0, r1;
+              rot(make_float2(ylo[j], ylo[j + 2]), make_float2(ylo[j + 1], ylo[j + 3]), make_float2(cs[m], cs[m + 1]),
+                  make_float2(sn[m], sn[m + 1]), r0, r1);
+              ylo[j] = r0.x;
+              ylo[j + 2] = r0.y;
+              ylo[j + 1] = r1.x;
+              ylo[j + 3] = r1.y;
+              rot(make_float2(yhi[j], yhi[j + 2]), make_float2(yhi[j + 1], yhi[j + 3]),
+                  make_float2(cs[16 + m], cs[17 + m]), make_float2(sn[16 + m], sn[17 + m]), r0, r1);
+              yhi[j] = r0.x;
+              yhi[j + 2] = r0.y;
+              yhi[j + 1] = r1.x;
+              yhi[j + 3] = r1.y;
             }
           }
           uint4 v[4];
@@ -586,11 +640,11 @@ kvx_status repack_wt_hilo(kvx_ctx* c, const void* W_host, size_t F) {
 }
 
 void launch_key_strip(const void* src_k, const int64_t* ss, void* ws, const int32_t* pos, int Ls, int H, int B, int T,
-                      const RopeTables& rope, int sms, cudaStream_t stream, int hf) {
+                      const RopeTables& rope, int sms, cudaStream_t stream, int hf, int il) {
   const int64_t threads = static_cast<int64_t>(B) * T * 16;
   const int blocks = static_cast<int>(std::min<int64_t>((threads + 255) / 256, static_cast<int64_t>(sms) * 8));
   xh_strip_kernel<<<blocks, 256, 0, stream>>>(static_cast<const __nv_bfloat16*>(src_k), ss[0], ss[1], ss[2], ss[3],
-                                              static_cast<__nv_bfloat16*>(ws), pos, Ls, H, B, T, rope, hf);
+                                              static_cast<__nv_bfloat16*>(ws), pos, Ls, H, B, T, rope, hf, il);
 }
 
 bool xh_supported(const kvx_ctx* c, std::string* why) {
@@ -599,7 +653,6 @@ bool xh_supported(const kvx_ctx* c, std::string* why) {
   else if (c->d != kXD) w = "needs head_dim 128";
   else if (c->head_mix != KVX_CROSS_HEAD && c->k <= 4)
     w = "runs per-head mappers only for k > 4 (the per-head tensor-core kernel takes k <= 4)";
-  else if (c->rope_style != KVX_ROPE_HALF) w = "needs half-split RoPE pairs";
   else if (c->H % 2 != 0) w = "needs an even number of KV heads";
   else if (static_cast<int64_t>(c->Lt) * 2 * c->H * kXD > INT_MAX ||
            static_cast<int64_t>(c->k) * c->H * kXD > INT_MAX / 2)
@@ -711,12 +764,13 @@ kvx_status launch_xh(kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   P.n_units = static_cast<int>(units);
   P.lo_steps = c->weight_dtype == KVX_F32 ? c->k * c->H : 0;
   P.hf = c->rope_numerics == KVX_ROPE_HF;
+  P.il = c->rope_style == KVX_ROPE_INTERLEAVED;
   P.rope = c->rope;
 
   // 1. strip the source RoPE from every key into the workspace
   {
     launch_key_strip(a.src_k, a.ss, c->d_ws, a.pos, c->Ls, c->H, a.B, a.T, c->rope, c->sm_count, stream,
-                     c->rope_numerics == KVX_ROPE_HF);
+                     c->rope_numerics == KVX_ROPE_HF, c->rope_style == KVX_ROPE_INTERLEAVED);
     if ((e = cudaGetLastError()) != cudaSuccess) {
       set_error(std::string("kvx_map: strip launch: ") + cudaGetErrorString(e));
       return KVX_ERR_CUDA;

@@ -155,6 +155,83 @@ def test_interleaved_pairs_simt():
         kvx.kvx_destroy(ctx)
 
 
+# ------------------------------------------------------ interleaved RoPE pairs -----
+
+@pytest.mark.parametrize("name,over,weights,expect", [
+    ("qwen3_14b_32b_b8x1024_k4", dict(Ls=6, Lt=4, H=2, B=2, T=300, k=3, theta_t=5e5), "bf16", 2),
+    ("qwen3_14b_32b_b8x1024_k4", dict(Ls=6, Lt=5, H=2, B=1, T=260, k=4, scores="uniform"), "f32", 2),
+    ("qwen3_14b_32b_b8x1024_k4", dict(Ls=9, Lt=3, H=2, B=1, T=200, k=6), "bf16", 3),   # k > 4: widened W
+    ("qwen3_14b_32b_t32768_k4_xhead", dict(Ls=4, Lt=3, H=2, B=2, T=150, k=2), "bf16", 3),
+])
+def test_interleaved_pairs_tensor_cores(name, over, weights, expect):
+    """Interleaved RoPE pairs (2i, 2i+1) on the per-head (2) and cross-head (3) tensor-core
+    kernels, bf16 and fp32 (hi + lo) weights: every output element of two launches against
+    the float64 oracle in the interleaved style, at positions past 10^4; the half-split
+    oracle's keys fail the same bound (the test sees the pairing)."""
+    w = syn.workload(name, **over)
+    Wb, b = syn.weights(w)
+    W = Wb
+    if weights == "f32":
+        g = torch.Generator().manual_seed(7)
+        W = (Wb.float() * (1.0 + 2.0 ** -9 * torch.rand(Wb.shape, generator=g))).contiguous()
+    ctx, sel, _, _ = make_ctx(w, kernel=kvx.KVX_KERNEL_TCGEN05, W=W, b=b, rope_style=kvx.KVX_ROPE_INTERLEAVED)
+    try:
+        assert kvx.kvx_get_kernel(ctx) == expect
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w) + 10007
+        rk, rv, ak, av = oracle_full(w, sk, sv, pos, sel, W, b, style="interleaved")
+        for rep in range(2):
+            tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+            assert st == kvx.KVX_OK
+            ok, ratio, rms, nbad = check(w, [to_f64(tk), to_f64(tv)], [rk, rv], [ak, av])
+            assert ok, "launch %d: %d elements out of tolerance (worst %.3g x bound)" % (rep, nbad, ratio)
+        hk, _, hak, _ = oracle_full(w, sk, sv, pos, sel, W, b, style="half")
+        assert not check(w, [to_f64(tk)], [hk], [hak])[0]
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
+@pytest.mark.parametrize("kname,name", [("simt", "qwen3_14b_32b_b8x1024_k4"), ("tc", "qwen3_14b_32b_b8x1024_k4"),
+                                        ("tc", "qwen3_14b_32b_t32768_k4_xhead")])
+def test_interleaved_pairs_hf_numerics(kname, name):
+    """Interleaved pairs with KVX_ROPE_HF (fp32 angle, bf16 cos / sin, every product and sum
+    rounded) on the SIMT, per-head and cross-head kernels: values within the bound of the
+    HF oracle, keys within 4 bf16 steps of their pair's magnitude and at least 90 % of them
+    bit-equal to it, far more than agree with the exact-RoPE oracle."""
+    w = syn.workload(name, Ls=5, Lt=3, H=2, B=2, T=180, k=2, theta_t=5e5)
+    W, b = syn.weights(w)
+    mix = kvx.KVX_CROSS_HEAD if w.head_mix == "cross_head" else kvx.KVX_PER_HEAD
+    cfg, keep = kvx.config_from_tensors(
+        src_layers=w.Ls, tgt_layers=w.Lt, n_kv_heads=w.H, head_dim=w.d, k=w.k, theta_s=w.theta_s,
+        theta_t=w.theta_t, cache_dtype=w.cache_dtype, W=W, b=b, scores=syn.selection_scores(w),
+        rope_style=kvx.KVX_ROPE_INTERLEAVED, head_mix=mix, rope_numerics=kvx.KVX_ROPE_HF)
+    ctx = kvx.kvx_create(cfg, 0)
+    try:
+        kvx.kvx_set_kernel(ctx, KERNELS[kname])
+        sel = kvx.kvx_get_selection(ctx, w.Lt, w.k)
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = syn.positions(w) + np.array([[20011], [31007]], dtype=np.int32)
+        tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        sk64, sv64 = to_f64(sk), to_f64(sv)
+        common = dict(mode="bf16fwd", style="interleaved", head_mix=w.head_mix)
+        rk, rv = omap.map_cache(sk64, sv64, pos, sel, to_f64(W), to_f64(b), w.theta_s, w.theta_t,
+                                rope_numerics="hf", **common)
+        ek, _ = omap.map_cache(sk64, sv64, pos, sel, to_f64(W), to_f64(b), w.theta_s, w.theta_t, **common)
+        gk, gv = to_f64(tk), to_f64(tv)
+        ok, ratio, rms, nbad = check(w, [gv], [rv])
+        assert ok, "values: %d elements out of tolerance (worst %.3g x bound)" % (nbad, ratio)
+        mag = np.repeat(np.abs(rk[..., 0::2]) + np.abs(rk[..., 1::2]), 2, axis=-1)
+        assert np.all(np.abs(gk - rk) <= 2.0 ** -6 * mag + 1e-3 * rms)
+        from oracle import bf16 as obf16
+        same_hf, same_exact = np.mean(gk == rk), np.mean(gk == obf16.round_to_bf16_value(ek))
+        assert same_hf >= 0.9 and same_hf > same_exact + 0.1, (same_hf, same_exact)
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
 def test_cross_head_simt():
     w = syn.workload("tiny_fp32", T=64)
     Wc = torch.from_numpy((np.random.default_rng(3).standard_normal(
