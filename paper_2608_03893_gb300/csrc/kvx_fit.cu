@@ -20,9 +20,11 @@
 // 2. fit_solve_kernel: one CTA per system at a time (persistent); the block grid is
 //    widened to float-float pairs (~48 significant bits, on the FP32 units) into a per-CTA
 //    scratch matrix, lambda added, factorised by a blocked right-looking Cholesky
-//    (32-column panels: diagonal block in shared memory, panel by forward substitution,
-//    trailing update), then the two triangular solves for the d right-hand sides and the
-//    bias; W and b are written in fp32.  fit_solve_xh_kernel does the same for the
+//    (32-column panels: diagonal block in shared memory, then its inverse by one warp beside
+//    the panel by forward substitution on the others, trailing update), then the two
+//    triangular solves for the d right-hand sides in 32-row blocks (products with the
+//    solved rows, then the inverse diagonal block) and the bias; W and b are written in
+//    fp32.  fit_solve_xh_kernel does the same for the
 //    cross-head systems, with the trailing update staged per 64 x 64 tile.
 // kvx_fit_ridge runs them on the caller's stream, with stream-ordered workspace, and
 // synchronises before it returns (the fit is an offline step).
@@ -59,7 +61,8 @@ struct FitParams {
   int32_t n_pairs;
   float* xty;                       // per head [L_t][2][H][k][128][128]; cross-head
                                     // [L_t][2][k][H (source head)][H (target head)][128][128]
-  double* scratch;                  // per CTA: F x F matrix + F x R right-hand sides
+  double* scratch;                  // per CTA: F x F matrix + F x R right-hand sides + the F / 32
+                                    // inverted 32 x 32 diagonal blocks of the factor
   float* W;                         // [L_t][2][H][F][128]
   float* b;                         // [L_t][2][H][128]
   double lambda;
@@ -180,11 +183,11 @@ __device__ __forceinline__ void chol_diag(DF* A, int F, int c0, DF* D, int32_t* 
 }
 
 // Panel below the diagonal block: every row r in [c0 + 32, F) solves x L_kk^T =
-// A[r][c0 .. c0 + 31] (thread = row), in place; with Pn the rows are also kept in shared
-// memory ([F - c0 - 32][33]).
-__device__ __forceinline__ void chol_panel(DF* A, int F, int c0, const DF* D, DF* Pn) {
+// A[r][c0 .. c0 + 31] (thread first + i stride = row i), in place; with Pn the rows are
+// also kept in shared memory ([F - c0 - 32][33]).
+__device__ __forceinline__ void chol_panel(DF* A, int F, int c0, const DF* D, DF* Pn, int first, int stride) {
   const int rows = F - c0 - kNB;
-  for (int rr = threadIdx.x; rr < rows; rr += blockDim.x) {
+  for (int rr = first; rr < rows; rr += stride) {
     DF* arow = A + static_cast<size_t>(c0 + kNB + rr) * F + c0;
     DF x[kNB];
 #pragma unroll
@@ -202,18 +205,60 @@ __device__ __forceinline__ void chol_panel(DF* A, int F, int c0, const DF* D, DF
   }
 }
 
+// Inverse of the factored 32 x 32 diagonal block L_kk (lower triangle of D) by one warp,
+// lane j = column j: X[i][j] = (delta_ij - sum_{m<i} L[i][m] X[m][j]) / L[i][i] (entries
+// above the diagonal come out as exact zeros); written row-major [32][32] to inv.
+__device__ __forceinline__ void tri_inverse(const DF* D, DF* inv) {
+  const int j = threadIdx.x & 31;
+  DF x[kNB];
+#pragma unroll
+  for (int i = 0; i < kNB; ++i) {
+    DF v = df_make(i == j ? 1.f : 0.f);
+#pragma unroll
+    for (int m = 0; m < i; ++m) v = df_fma_lazy(df_neg(D[i * kPS + m]), x[m], v);
+    x[i] = df_div(df_norm(v), D[i * kPS + i]);
+    inv[i * kNB + j] = x[i];
+  }
+}
+
+// One 32-column step of the factorisation: the diagonal block (one warp), then its inverse
+// (warp 0) beside the panel (the other warps).  Ends with the CTA synchronised.
+__device__ __forceinline__ void chol_step(DF* A, int F, int c0, DF* D, DF* Pn, DF* Inv, int32_t* status) {
+  chol_diag(A, F, c0, D, status);
+  if (threadIdx.x < 32) tri_inverse(D, Inv + static_cast<size_t>(c0) * kNB);
+  else chol_panel(A, F, c0, D, Pn, threadIdx.x - 32, blockDim.x - 32);
+  __syncthreads();
+}
+
+// Asynchronous global -> shared copies (cp.async, completion tracked per thread by groups).
+__device__ __forceinline__ void cp_async8(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+constexpr int kStageDF = kNB * kPS + kNB * kFD;   // one solve stage: [32][33] L entries + [32][128] rows
+
 // The two triangular solves with the factor L (lower triangle of A, leading dimension F)
 // for 128 right-hand-side columns Z[0 .. F)[0 .. 128) (leading dimension ldz), in place:
-// forward L Y = Z, then backward L^T W = Y, in 32-row blocks.  A block first takes the
-// products with every solved row (thread = 2 rows x 4 columns, 8 independent sums; the
-// solved rows and the block's L entries staged through shared memory 32 at a time), then
-// its 32 x 32 triangle is solved row by row (thread = column).  fsm: [32][33] + [32][128].
-__device__ __forceinline__ void tri_solves(const DF* A, int F, DF* Z, int ldz, DF* fsm) {
+// forward L Y = Z, then backward L^T W = Y, in 32-row blocks.  A block takes the products
+// with the solved rows 32 at a time (chunk stages: 32 x 32 entries of L and 32 solved rows
+// staged in shared memory; thread = 2 rows x 4 columns, 8 independent sums), then is
+// multiplied by the inverse of its diagonal block (Inv, [F / 32][32][32], from the
+// factorisation; its transpose in the backward solve), the same staged product with every
+// thread busy.  Stages run through two shared-memory buffers: the next stage's operands
+// are copied asynchronously while the current one computes, except where they are the
+// rows the current stage solves (the chunk orders keep that to one stage per direction).
+// fsm: 2 x kStageDF pairs.
+__device__ __forceinline__ void tri_solves(const DF* A, int F, DF* Z, int ldz, const DF* Inv, DF* fsm) {
   const int tid = threadIdx.x;
   constexpr int kR = kNB * kFD / 4 / kSolveThreads;   // rows per thread (2)
   const int r0 = kR * (tid % (kNB / kR)), q0 = 4 * (tid / (kNB / kR));
-  DF* Ls = fsm;                         // [32][33]: L (forward) or L^T (backward) entries
-  DF* Zs = fsm + kNB * kPS;             // [32][128]: 32 solved rows of Z
+  const int nb = F / kNB;
   auto load4 = [&](const DF* p, DF (&v)[4]) {
     const float4 x = *reinterpret_cast<const float4*>(p), y = *reinterpret_cast<const float4*>(p + 2);
     v[0] = DF{x.x, x.y};
@@ -221,79 +266,104 @@ __device__ __forceinline__ void tri_solves(const DF* A, int F, DF* Z, int ldz, D
     v[2] = DF{y.x, y.y};
     v[3] = DF{y.z, y.w};
   };
-  // acc[a][c] -= sum_j Ls[r0 + a][j] Zs[j][q0 + c] over the staged chunk (Ls indexed
-  // [row][j] when `rows_major`, else [j][row])
-  auto chunk_update = [&](DF (&acc)[kR][4], bool rows_major) {
+  // acc[a][c] -/+= sum_j Ls[r0 + a][j] Zs[j][q0 + c] (Ls indexed [row][j] when `rows_major`,
+  // else [j][row])
+  auto chunk_update = [&](const DF* Ls, const DF* Zs, DF (&acc)[kR][4], bool rows_major, bool subtract) {
 #pragma unroll 4
     for (int j = 0; j < kNB; ++j) {
       DF z[4], l[kR];
       load4(&Zs[j * kFD + q0], z);
 #pragma unroll
-      for (int a2 = 0; a2 < kR; ++a2) l[a2] = df_neg(rows_major ? Ls[(r0 + a2) * kPS + j] : Ls[j * kPS + r0 + a2]);
+      for (int a2 = 0; a2 < kR; ++a2) {
+        const DF v = rows_major ? Ls[(r0 + a2) * kPS + j] : Ls[j * kPS + r0 + a2];
+        l[a2] = subtract ? df_neg(v) : v;
+      }
 #pragma unroll
       for (int a2 = 0; a2 < kR; ++a2)
 #pragma unroll
         for (int c = 0; c < 4; ++c) acc[a2][c] = df_fma_lazy(l[a2], z[c], acc[a2][c]);
     }
   };
-  auto stage_z = [&](int m0) {        // 32 rows x 128 pairs, two pairs per thread-step
-    for (int e = tid; e < kNB * kFD / 2; e += blockDim.x)
-      reinterpret_cast<float4*>(Zs)[e] =
-          *reinterpret_cast<const float4*>(Z + static_cast<size_t>(m0 + e / (kFD / 2)) * ldz + 2 * (e % (kFD / 2)));
+  // Stage (bi, u) of one direction: block bi in solve order (b = bi forward, nb - 1 - bi
+  // backward) has bi chunk stages u < bi, then its diagonal stage u = bi (mc < 0).  Chunk
+  // rows: forward mc = u (ascending), backward mc = nb - 1 - u (descending).
+  auto stage = [&](bool fwd, int bi, int u, int& b, int& mc) {
+    b = fwd ? bi : nb - 1 - bi;
+    mc = u == bi ? -1 : (fwd ? u : nb - 1 - u);
   };
-  for (int b0 = 0; b0 < F; b0 += kNB) {
-    DF acc[kR][4];
-#pragma unroll
-    for (int a = 0; a < kR; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * ldz + q0], acc[a]);
-    for (int mc = 0; mc < b0; mc += kNB) {
+  auto issue = [&](DF* buf, bool fwd, int b, int mc) {
+    DF* Ls = buf;
+    if (mc >= 0) {
+      // forward: L[b + i][mc + j] -> Ls[i][j]; backward: L[mc + j][b + i] -> Ls[j][i]
+      const int X = fwd ? b : mc, Y = fwd ? mc : b;
       for (int e = tid; e < kNB * kNB; e += blockDim.x)
-        Ls[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(b0 + e / kNB) * F + mc + e % kNB];
-      stage_z(mc);
-      __syncthreads();
-      chunk_update(acc, true);
-      __syncthreads();
+        cp_async8(&Ls[(e / kNB) * kPS + e % kNB], &A[static_cast<size_t>(X * kNB + e / kNB) * F + Y * kNB + e % kNB]);
+      float4* Zs = reinterpret_cast<float4*>(buf + kNB * kPS);
+      for (int e = tid; e < kNB * kFD / 2; e += blockDim.x)
+        cp_async16(&Zs[e], Z + static_cast<size_t>(mc * kNB + e / (kFD / 2)) * ldz + 2 * (e % (kFD / 2)));
+    } else {
+      const DF* inv = Inv + static_cast<size_t>(b) * kNB * kNB;
+      for (int e = tid; e < kNB * kNB; e += blockDim.x) cp_async8(&Ls[(e / kNB) * kPS + e % kNB], &inv[e]);
     }
-#pragma unroll
-    for (int a = 0; a < kR; ++a)
-#pragma unroll
-      for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * ldz + q0 + c] = df_norm(acc[a][c]);
-    __syncthreads();
-    if (tid < kFD) {
-      for (int i = 0; i < kNB; ++i) {
-        const DF* lrow = A + static_cast<size_t>(b0 + i) * F + b0;
-        DF v = Z[static_cast<size_t>(b0 + i) * ldz + tid];
-        for (int m = 0; m < i; ++m) v = df_fma_lazy(df_neg(lrow[m]), Z[static_cast<size_t>(b0 + m) * ldz + tid], v);
-        Z[static_cast<size_t>(b0 + i) * ldz + tid] = df_div(df_norm(v), lrow[i]);
-      }
-    }
-    __syncthreads();
-  }
-  for (int b0 = F - kNB; b0 >= 0; b0 -= kNB) {
+    cp_async_commit();
+  };
+  for (int dir = 0; dir < 2; ++dir) {
+    const bool fwd = dir == 0;
+    int bi = 0, u = 0, b = 0, mc = 0;
+    stage(fwd, bi, u, b, mc);
+    int k = 0;                                   // stages issued so far in this direction
+    issue(fsm, fwd, b, mc);
     DF acc[kR][4];
 #pragma unroll
-    for (int a = 0; a < kR; ++a) load4(&Z[static_cast<size_t>(b0 + r0 + a) * ldz + q0], acc[a]);
-    for (int mc = b0 + kNB; mc < F; mc += kNB) {
-      for (int e = tid; e < kNB * kNB; e += blockDim.x)   // L[mc + j][b0 + i]: entries of L^T
-        Ls[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(mc + e / kNB) * F + b0 + e % kNB];
-      stage_z(mc);
-      __syncthreads();
-      chunk_update(acc, false);
-      __syncthreads();
-    }
-#pragma unroll
-    for (int a = 0; a < kR; ++a)
-#pragma unroll
-      for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b0 + r0 + a) * ldz + q0 + c] = df_norm(acc[a][c]);
-    __syncthreads();
-    if (tid < kFD) {
-      for (int i = kNB - 1; i >= 0; --i) {
-        DF v = Z[static_cast<size_t>(b0 + i) * ldz + tid];
-        for (int m = i + 1; m < kNB; ++m)
-          v = df_fma_lazy(df_neg(A[static_cast<size_t>(b0 + m) * F + b0 + i]), Z[static_cast<size_t>(b0 + m) * ldz + tid], v);
-        Z[static_cast<size_t>(b0 + i) * ldz + tid] = df_div(df_norm(v), A[static_cast<size_t>(b0 + i) * F + b0 + i]);
+    for (int a = 0; a < kR; ++a) load4(&Z[static_cast<size_t>(b * kNB + r0 + a) * ldz + q0], acc[a]);
+    while (bi < nb) {
+      DF* cur = fsm + (k & 1) * kStageDF;
+      DF* nxt = fsm + ((k + 1) & 1) * kStageDF;
+      const int bi2 = u < bi ? bi : bi + 1, u2 = u < bi ? u + 1 : 0;
+      int b2 = 0, mc2 = 0;
+      const bool more = bi2 < nb;
+      if (more) stage(fwd, bi2, u2, b2, mc2);
+      // the next stage's rows are the ones this diagonal stage solves: copy them after it
+      const bool defer = more && mc < 0 && mc2 == b;
+      if (more && !defer) {
+        issue(nxt, fwd, b2, mc2);
+        cp_async_wait<1>();
+      } else {
+        cp_async_wait<0>();
       }
+      __syncthreads();
+      if (mc >= 0) {
+        chunk_update(cur, cur + kNB * kPS, acc, fwd, true);
+      } else {
+        DF* Zs = cur + kNB * kPS;
+#pragma unroll
+        for (int a = 0; a < kR; ++a)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) Zs[(r0 + a) * kFD + q0 + c] = df_norm(acc[a][c]);
+        __syncthreads();
+        DF res[kR][4];
+#pragma unroll
+        for (int a = 0; a < kR; ++a)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) res[a][c] = df_make(0.f);
+        chunk_update(cur, Zs, res, fwd, false);   // forward: L_kk^-1 [row][j]; backward: (L_kk^-1)^T
+#pragma unroll
+        for (int a = 0; a < kR; ++a)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b * kNB + r0 + a) * ldz + q0 + c] = df_norm(res[a][c]);
+      }
+      __syncthreads();
+      if (defer) issue(nxt, fwd, b2, mc2);
+      if (more && mc < 0) {   // a new block starts: its right-hand sides
+#pragma unroll
+        for (int a = 0; a < kR; ++a) load4(&Z[static_cast<size_t>(b2 * kNB + r0 + a) * ldz + q0], acc[a]);
+      }
+      bi = bi2;
+      u = u2;
+      b = b2;
+      mc = mc2;
+      ++k;
     }
-    __syncthreads();
   }
 }
 
@@ -306,8 +376,10 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __gri
   const int F = P.k * kFD;
   const int tid = threadIdx.x;
   DF* A = reinterpret_cast<DF*>(P.scratch) +
-          static_cast<size_t>(blockIdx.x) * (static_cast<size_t>(F) * F + static_cast<size_t>(F) * kFD);
+          static_cast<size_t>(blockIdx.x) * (static_cast<size_t>(F) * F + static_cast<size_t>(F) * kFD +
+                                             static_cast<size_t>(F) * kNB);
   DF* Z = A + static_cast<size_t>(F) * F;         // [F][128]
+  DF* Inv = Z + static_cast<size_t>(F) * kFD;     // [F / 32][32][32]: inverses of the diagonal blocks
   const int n_sys = P.Lt * 2 * P.H;
   const double inv_n = 1.0 / (static_cast<double>(P.B) * P.T);
   const DF lam = df_from_double(P.lambda);
@@ -333,9 +405,7 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __gri
     __syncthreads();
     // 2. Cholesky A = L L^T, lower triangle in place, 32-column panels
     for (int c0 = 0; c0 < F; c0 += kNB) {
-      chol_diag(A, F, c0, D, P.status);
-      chol_panel(A, F, c0, D, Pn);
-      __syncthreads();
+      chol_step(A, F, c0, D, Pn, Inv, P.status);
       // trailing update: A[i][j] -= P[i] . P[j] for c0+32 <= j <= i, in 32 x 32 tiles
       const int rows = F - c0 - kNB;
       const int nt = rows / kNB;
@@ -348,9 +418,13 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __gri
         // warp's rows are broadcasts
         constexpr int kRowsPer = kNB / kSolveWarps;
         const int jj = tj * kNB + (tid & 31), ii = ti * kNB + (tid >> 5);
-        DF sacc[kRowsPer];
+        DF sacc[kRowsPer], aold[kRowsPer];
 #pragma unroll
-        for (int q = 0; q < kRowsPer; ++q) sacc[q] = df_make(0.f);
+        for (int q = 0; q < kRowsPer; ++q) {   // A's entries are loaded before the products
+          sacc[q] = df_make(0.f);
+          aold[q] = jj <= ii + kSolveWarps * q ? A[static_cast<size_t>(c0 + kNB + ii + kSolveWarps * q) * F + c0 + kNB + jj]
+                                               : df_make(0.f);
+        }
 #pragma unroll 8
         for (int m = 0; m < kNB; ++m) {
           const DF pj = Pn[jj * kPS + m];
@@ -360,13 +434,13 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __gri
 #pragma unroll
         for (int q = 0; q < kRowsPer; ++q) {
           DF* a = A + static_cast<size_t>(c0 + kNB + ii + kSolveWarps * q) * F + c0 + kNB + jj;
-          if (jj <= ii + kSolveWarps * q) *a = df_add(*a, df_neg(df_norm(sacc[q])));
+          if (jj <= ii + kSolveWarps * q) *a = df_add(aold[q], df_neg(df_norm(sacc[q])));
         }
       }
       __syncthreads();
     }
     // 3. forward and backward solves for the 128 right-hand sides
-    tri_solves(A, F, Z, kFD, fsm);
+    tri_solves(A, F, Z, kFD, Inv, fsm);
     // 4. W (fp32) and b = mean(Y) - mean(X) W (fp64)
     float* Wout = P.W + static_cast<size_t>(sys) * F * kFD;
     for (int64_t e = tid; e < static_cast<int64_t>(F) * kFD; e += blockDim.x) Wout[e] = __fadd_rn(Z[e].hi, Z[e].lo);
@@ -398,8 +472,10 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_xh_kernel(const __
   const int F = P.k * H * kFD;
   const int tid = threadIdx.x;
   DF* A = reinterpret_cast<DF*>(P.scratch) +
-          static_cast<size_t>(blockIdx.x) * (static_cast<size_t>(F) * F + static_cast<size_t>(F) * R);
+          static_cast<size_t>(blockIdx.x) * (static_cast<size_t>(F) * F + static_cast<size_t>(F) * R +
+                                             static_cast<size_t>(F) * kNB);
   DF* Z = A + static_cast<size_t>(F) * F;         // [F][R]
+  DF* Inv = Z + static_cast<size_t>(F) * R;       // [F / 32][32][32]: inverses of the diagonal blocks
   const int n_sys = P.Lt * 2;
   const double inv_n = 1.0 / (static_cast<double>(P.B) * P.T);
   const DF lam = df_from_double(P.lambda);
@@ -437,9 +513,7 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_xh_kernel(const __
     __syncthreads();
     // 2. Cholesky, 32-column panels; trailing update in 64 x 64 tiles of the lower triangle
     for (int c0 = 0; c0 < F; c0 += kNB) {
-      chol_diag(A, F, c0, D, P.status);
-      chol_panel(A, F, c0, D, nullptr);
-      __syncthreads();
+      chol_step(A, F, c0, D, nullptr, Inv, P.status);
       const int base = c0 + kNB, rows = F - base;
       const int nt = (rows + kXT - 1) / kXT;
       // thread: column jj = tid % 64 of the tile, rows ii + 8q (ii = tid / 64), q < 8
@@ -453,31 +527,32 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_xh_kernel(const __
           const int row = (s == 0 ? ti : tj) * kXT + rr;
           (s == 0 ? Pi : Pj)[rr * kPS + m] = row < rows ? A[static_cast<size_t>(base + row) * F + c0 + m] : df_make(0.f);
         }
-        __syncthreads();
         constexpr int kQ = kXT * kXT / kSolveThreads;   // 8
-        DF sacc[kQ];
+        const int gj = tj * kXT + jj;
+        DF sacc[kQ], aold[kQ];
 #pragma unroll
-        for (int q = 0; q < kQ; ++q) sacc[q] = df_make(0.f);
+        for (int q = 0; q < kQ; ++q) {   // A's entries are loaded before the products
+          const int gi = ti * kXT + ii + 8 * q;
+          sacc[q] = df_make(0.f);
+          aold[q] = gi < rows && gj <= gi ? A[static_cast<size_t>(base + gi) * F + base + gj] : df_make(0.f);
+        }
+        __syncthreads();
 #pragma unroll 4
         for (int m = 0; m < kNB; ++m) {
           const DF pj = Pj[jj * kPS + m];
 #pragma unroll
           for (int q = 0; q < kQ; ++q) sacc[q] = df_fma_lazy(Pi[(ii + 8 * q) * kPS + m], pj, sacc[q]);
         }
-        const int gj = tj * kXT + jj;
 #pragma unroll
         for (int q = 0; q < kQ; ++q) {
           const int gi = ti * kXT + ii + 8 * q;
-          if (gi < rows && gj <= gi) {
-            DF* a = A + static_cast<size_t>(base + gi) * F + base + gj;
-            *a = df_add(*a, df_neg(df_norm(sacc[q])));
-          }
+          if (gi < rows && gj <= gi) A[static_cast<size_t>(base + gi) * F + base + gj] = df_add(aold[q], df_neg(df_norm(sacc[q])));
         }
         __syncthreads();
       }
     }
     // 3. forward and backward solves, 128 right-hand sides (one target head) at a time
-    for (int c0 = 0; c0 < R; c0 += kFD) tri_solves(A, F, Z + c0, R, fsm);
+    for (int c0 = 0; c0 < R; c0 += kFD) tri_solves(A, F, Z + c0, R, Inv, fsm);
     // 4. W (fp32, [L_t][2][H][F][128]) and b = mean(Y) - mean(X) W (fp64)
     for (int64_t e = tid; e < static_cast<int64_t>(F) * R; e += blockDim.x) {
       const int r = static_cast<int>(e / R), col = static_cast<int>(e % R);
@@ -546,7 +621,7 @@ FitPlan plan_fit(const kvx_fit_config* cfg, int sms, GramSpec* G) {
   p.gram_n = static_cast<size_t>(2) * H * (cross ? H : 1) * p.n_pairs * kBlk;
   p.xty_n = static_cast<size_t>(cfg->tgt_layers) * 2 * H * kk * (cross ? H : 1) * kBlk;
   p.solve_grid = static_cast<int>(std::min<size_t>(p.n_sys, static_cast<size_t>(std::max(sms, 1))));
-  const size_t per_cta = static_cast<size_t>(p.F) * p.F + static_cast<size_t>(p.F) * p.R;
+  const size_t per_cta = static_cast<size_t>(p.F) * p.F + static_cast<size_t>(p.F) * p.R + static_cast<size_t>(p.F) * kNB;
   if (cross)
     p.solve_grid = static_cast<int>(std::max<size_t>(1, std::min<size_t>(p.solve_grid, kXhScratchCap / (per_cta * 8))));
   p.scratch_n = static_cast<size_t>(p.solve_grid) * per_cta;
@@ -795,7 +870,7 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
     // or the solves' staged chunk
     const size_t fact = pl.cross ? static_cast<size_t>(kNB + 2 * kXT) * kPS
                                  : static_cast<size_t>(kNB) * kPS + static_cast<size_t>(pl.F - kNB) * kPS;
-    const size_t smem = std::max(fact, static_cast<size_t>(kNB) * kPS + static_cast<size_t>(kNB) * kFD) * 8;
+    const size_t smem = std::max(fact, static_cast<size_t>(2) * kStageDF) * 8;
     auto kernel = pl.cross ? fit_solve_xh_kernel : fit_solve_kernel;
     if ((e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem))) !=
         cudaSuccess) {
