@@ -86,8 +86,10 @@ __device__ __forceinline__ void report_fit(int32_t* status, int code) { atomicCA
 // dozen FP32 instructions.  The error-free steps are the published ones: two_sum (Knuth,
 // TAOCP vol. 2, 4.2.2), fast_two_sum (Dekker 1971, needs |a| >= |b|), two_prod by one
 // FMA; the pair arithmetic follows Dekker's and the QD library's (Hida, Li, Bailey 2001)
-// "sloppy" addition, and division / square root correct a float estimate once by the
-// residual.
+// "sloppy" addition; the reciprocal square root of the pivots refines the hardware
+// estimate by Newton's iteration (below).  The IEEE-rounded float divide and square root
+// take several hundred cycles on the dependency chains of the factorisation, so pivots
+// enter only through that reciprocal.
 struct __align__(8) DF {
   float hi, lo;
 };
@@ -128,17 +130,12 @@ __device__ __forceinline__ DF df_fma_lazy(DF a, DF b, DF c) {
   return DF{s.hi, __fadd_rn(c.lo, __fadd_rn(s.lo, e))};
 }
 __device__ __forceinline__ DF df_norm(DF a) { return two_sum(a.hi, a.lo); }
-// a / b: the float quotient q corrected by the residual a - q b
-__device__ __forceinline__ DF df_div(DF a, DF b) {
-  const float q1 = __fdiv_rn(a.hi, b.hi);
-  const DF r = df_fma(df_neg(df_make(q1)), b, a);
-  return fast_two_sum(q1, __fdiv_rn(r.hi, b.hi));
-}
-// sqrt(a), a > 0: s = sqrt(hi) corrected by (a - s^2) / 2s
-__device__ __forceinline__ DF df_sqrt(DF a) {
-  const float s = __fsqrt_rn(a.hi);
-  const DF r = df_fma(df_neg(df_make(s)), df_make(s), a);
-  return fast_two_sum(s, __fdiv_rn(r.hi, __fmul_rn(2.f, s)));
+__device__ __forceinline__ DF df_mul(DF a, DF b) {
+  const float p = __fmul_rn(a.hi, b.hi);
+  float e = __fmaf_rn(a.hi, b.hi, -p);
+  e = __fmaf_rn(a.hi, b.lo, e);
+  e = __fmaf_rn(a.lo, b.hi, e);
+  return fast_two_sum(p, e);
 }
 __device__ __forceinline__ DF df_from_double(double x) {
   const float hi = static_cast<float>(x);
@@ -152,82 +149,158 @@ constexpr int kNotSpd = 100;        // internal status: a pivot <= 0 (matrix not
 constexpr int kPS = kNB + 1;        // panel row stride in shared memory (pairs)
 
 constexpr int kSolveThreads = 512;                 // 16 warps: enough to keep the FP32 lanes busy
-constexpr int kSolveWarps = kSolveThreads / 32;
 
-// Cholesky step of the 32 x 32 diagonal block at (c0, c0) of A (row-major, leading
-// dimension F, lower triangle): copied to D in shared memory, factored by one warp (lane =
-// row), written back.  A pivot <= 0 is reported and replaced by 1 so the call finishes.
-__device__ __forceinline__ void chol_diag(DF* A, int F, int c0, DF* D, int32_t* status) {
+// 1 / sqrt(a), a > 0: y from the hardware estimate, then y += y (1 - a y^2) / 2 twice with
+// the residual in float-float (Newton's iteration for the reciprocal square root, in the
+// form of Karp and Markstein, ACM TOMS 23(4), 1997).
+__device__ __forceinline__ DF df_rsqrt(DF a) {
+  DF y = df_make(rsqrtf(a.hi));
+#pragma unroll
+  for (int it = 0; it < 2; ++it) {
+    const DF r = df_fma(df_neg(a), df_mul(y, y), df_make(1.f));   // 1 - a y^2
+    y = df_add(y, df_mul(y, df_make(__fmul_rn(0.5f, r.hi))));
+  }
+  return y;
+}
+
+// Shared-memory pieces of one factorisation step.
+struct FactSmem {
+  DF* D;        // [32][33]: the diagonal block, then its factor L_kk; D[i][32] = 1 / L[i][i]
+  DF* X;        // [32][33]: L_kk^-1 (zeros above the diagonal)
+  DF* Lc;       // [32]: the column of L formed in a step of the diagonal factorisation
+  DF* T;        // [16][17]: scratch of the inverse
+  DF* Pn;       // [pn_rows][33]: staged panel rows
+  int pn_rows;
+};
+constexpr int kFactFixedDF = 2 * kNB * kPS + kNB + 16 * 17;   // D, X, Lc, T
+
+// Cholesky of the 32 x 32 diagonal block at (c0, c0) of A (lower triangle) by the CTA:
+// step j, warp 0 forms column j of L (the pivot through a float-float reciprocal square
+// root), then every thread updates its entries (i, m), j < m <= i.  A pivot <= 0 is
+// reported and replaced by 1 so the call finishes.  Ends synchronised.
+__device__ __forceinline__ void chol_diag(const DF* A, int F, int c0, const FactSmem& S, int32_t* status) {
   const int tid = threadIdx.x;
-  for (int e = tid; e < kNB * kNB; e += blockDim.x) D[(e / kNB) * kPS + e % kNB] = A[static_cast<size_t>(c0 + e / kNB) * F + c0 + e % kNB];
+  DF* D = S.D;
+  for (int e = tid; e < kNB * kNB; e += blockDim.x) {
+    const int i = e / kNB, m = e % kNB;
+    D[i * kPS + m] = m <= i ? A[static_cast<size_t>(c0 + i) * F + c0 + m] : df_make(0.f);
+  }
   __syncthreads();
-  if (tid < 32) {
-    for (int j = 0; j < kNB; ++j) {
-      if (tid == j) {
-        const DF d = D[j * kPS + j];
-        if (!(d.hi > 0.f)) report_fit(status, kNotSpd);
-        D[j * kPS + j] = d.hi > 0.f ? df_sqrt(d) : df_make(1.f);
+  for (int j = 0; j < kNB; ++j) {
+    if (tid < kNB) {
+      const DF d = D[j * kPS + j], own = D[tid * kPS + j];
+      if (!(d.hi > 0.f) && tid == 0) report_fit(status, kNotSpd);
+      const DF y = d.hi > 0.f ? df_rsqrt(d) : df_make(1.f);
+      const DF l = tid > j ? df_mul(own, y) : (tid == j ? df_mul(d, y) : df_make(0.f));
+      __syncwarp();
+      S.Lc[tid] = l;
+      if (tid >= j) D[tid * kPS + j] = l;
+      if (tid == j) D[tid * kPS + kNB] = y;
+    }
+    __syncthreads();
+    for (int e = tid; e < kNB * kNB; e += blockDim.x) {
+      const int i = e / kNB, m = e % kNB;
+      if (j < m && m <= i) D[i * kPS + m] = df_fma(df_neg(S.Lc[i]), S.Lc[m], D[i * kPS + m]);
+    }
+    __syncthreads();
+  }
+}
+
+// X = L_kk^-1 by the CTA, for L = [[P, 0], [Q, R]] in 16 x 16 quarters: P^-1 and R^-1 by
+// forward substitution (warps 0 and 1, lane = column), then the lower-left quarter
+// -R^-1 (Q P^-1) as two 16 x 16 products; written row-major [32][32] to inv.  Ends
+// synchronised.
+__device__ __forceinline__ void tri_inverse(const FactSmem& S, DF* inv) {
+  const int tid = threadIdx.x;
+  const DF* D = S.D;
+  DF* X = S.X;
+  if (tid < 64 && (tid & 31) < 16) {
+    const int o = 16 * (tid >> 5), j = tid & 31;
+    for (int i = 0; i < 16; ++i) {
+      DF v = df_make(i == j ? 1.f : 0.f);
+      for (int m = j; m < i; ++m) v = df_fma_lazy(df_neg(D[(o + i) * kPS + o + m]), X[(o + m) * kPS + o + j], v);
+      X[(o + i) * kPS + o + j] = i >= j ? df_mul(df_norm(v), D[(o + i) * kPS + kNB]) : df_make(0.f);
+    }
+  }
+  for (int e = tid; e < 256; e += blockDim.x) X[(e / 16) * kPS + 16 + e % 16] = df_make(0.f);
+  __syncthreads();
+  if (tid < 256) {   // T = Q P^-1
+    const int r = tid / 16, c = tid % 16;
+    DF v = df_make(0.f);
+    for (int m = c; m < 16; ++m) v = df_fma_lazy(D[(16 + r) * kPS + m], X[m * kPS + c], v);
+    S.T[r * 17 + c] = df_norm(v);
+  }
+  __syncthreads();
+  if (tid < 256) {   // lower-left quarter: -R^-1 T
+    const int r = tid / 16, c = tid % 16;
+    DF v = df_make(0.f);
+    for (int m = 0; m <= r; ++m) v = df_fma_lazy(X[(16 + r) * kPS + 16 + m], S.T[m * 17 + c], v);
+    X[(16 + r) * kPS + c] = df_neg(df_norm(v));
+  }
+  __syncthreads();
+  for (int e = tid; e < kNB * kNB; e += blockDim.x) inv[e] = X[(e / kNB) * kPS + e % kNB];
+}
+
+// One 32-column step of the factorisation: the diagonal block and its inverse, then the
+// panel X = A[c0 + 32 .., c0 .. c0 + 31] L_kk^-T, a product with the inverse (no dependency
+// chains) computed from rows staged in S.Pn, S.pn_rows at a time, in 32-row tiles of 64
+// threads x 4 x 4 entries, eight tiles per round; the result goes to A and, for the rows
+// of the last chunk, stays in S.Pn (per-head systems stage every row in one chunk, so the
+// trailing update reads the whole panel from there).  Ends synchronised.
+__device__ __forceinline__ void chol_step(DF* A, int F, int c0, const FactSmem& S, DF* Inv, int32_t* status) {
+  const int tid = threadIdx.x, rows = F - c0 - kNB;
+  chol_diag(A, F, c0, S, status);
+  tri_inverse(S, Inv + static_cast<size_t>(c0) * kNB);
+  const int lt = tid & 63, ri = lt >> 3, cj = lt & 7;
+  for (int r0 = 0; r0 < rows; r0 += S.pn_rows) {
+    const int nr = min(S.pn_rows, rows - r0);
+    for (int e = tid; e < nr * (kNB / 2); e += blockDim.x) {
+      const int r = e / (kNB / 2), q = 2 * (e % (kNB / 2));
+      const float4 v = *reinterpret_cast<const float4*>(A + static_cast<size_t>(c0 + kNB + r0 + r) * F + c0 + q);
+      S.Pn[r * kPS + q] = DF{v.x, v.y};
+      S.Pn[r * kPS + q + 1] = DF{v.z, v.w};
+    }
+    __syncthreads();
+    const int tiles = (nr + kNB - 1) / kNB;
+    for (int rd = 0; rd < tiles; rd += kSolveThreads / 64) {
+      const int tile = rd + (tid >> 6);
+      DF acc[4][4];
+#pragma unroll
+      for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) acc[a][b] = df_make(0.f);
+      if (tile < tiles) {
+        const DF* prow = S.Pn + (tile * kNB + ri) * kPS;
+#pragma unroll 4
+        for (int m = 0; m < kNB; ++m) {
+          DF pi[4], pj[4];
+#pragma unroll
+          for (int a = 0; a < 4; ++a) pi[a] = prow[8 * a * kPS + m];
+#pragma unroll
+          for (int b = 0; b < 4; ++b) pj[b] = S.X[(cj + 8 * b) * kPS + m];
+#pragma unroll
+          for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int b = 0; b < 4; ++b) acc[a][b] = df_fma_lazy(pi[a], pj[b], acc[a][b]);
+        }
       }
-      __syncwarp();
-      if (tid > j) D[tid * kPS + j] = df_div(D[tid * kPS + j], D[j * kPS + j]);
-      __syncwarp();
-      if (tid > j)
-        for (int m = j + 1; m <= tid; ++m)
-          D[tid * kPS + m] = df_fma(df_neg(D[tid * kPS + j]), D[m * kPS + j], D[tid * kPS + m]);
-      __syncwarp();
+      __syncthreads();   // the tile's rows are read before they are overwritten
+      if (tile < tiles) {
+#pragma unroll
+        for (int a = 0; a < 4; ++a) {
+          const int r = tile * kNB + ri + 8 * a;
+          if (r >= nr) continue;
+#pragma unroll
+          for (int b = 0; b < 4; ++b) {
+            const DF x = df_norm(acc[a][b]);
+            S.Pn[r * kPS + cj + 8 * b] = x;
+            A[static_cast<size_t>(c0 + kNB + r0 + r) * F + c0 + cj + 8 * b] = x;
+          }
+        }
+      }
     }
+    __syncthreads();
   }
-  __syncthreads();
-  for (int e = tid; e < kNB * kNB; e += blockDim.x)
-    if (e % kNB <= e / kNB) A[static_cast<size_t>(c0 + e / kNB) * F + c0 + e % kNB] = D[(e / kNB) * kPS + e % kNB];
-}
-
-// Panel below the diagonal block: every row r in [c0 + 32, F) solves x L_kk^T =
-// A[r][c0 .. c0 + 31] (thread first + i stride = row i), in place; with Pn the rows are
-// also kept in shared memory ([F - c0 - 32][33]).
-__device__ __forceinline__ void chol_panel(DF* A, int F, int c0, const DF* D, DF* Pn, int first, int stride) {
-  const int rows = F - c0 - kNB;
-  for (int rr = first; rr < rows; rr += stride) {
-    DF* arow = A + static_cast<size_t>(c0 + kNB + rr) * F + c0;
-    DF x[kNB];
-#pragma unroll
-    for (int c = 0; c < kNB; ++c) {
-      DF v = arow[c];
-#pragma unroll
-      for (int m = 0; m < c; ++m) v = df_fma_lazy(df_neg(x[m]), D[c * kPS + m], v);
-      x[c] = df_div(df_norm(v), D[c * kPS + c]);
-    }
-#pragma unroll
-    for (int c = 0; c < kNB; ++c) {
-      arow[c] = x[c];
-      if (Pn) Pn[rr * kPS + c] = x[c];
-    }
-  }
-}
-
-// Inverse of the factored 32 x 32 diagonal block L_kk (lower triangle of D) by one warp,
-// lane j = column j: X[i][j] = (delta_ij - sum_{m<i} L[i][m] X[m][j]) / L[i][i] (entries
-// above the diagonal come out as exact zeros); written row-major [32][32] to inv.
-__device__ __forceinline__ void tri_inverse(const DF* D, DF* inv) {
-  const int j = threadIdx.x & 31;
-  DF x[kNB];
-#pragma unroll
-  for (int i = 0; i < kNB; ++i) {
-    DF v = df_make(i == j ? 1.f : 0.f);
-#pragma unroll
-    for (int m = 0; m < i; ++m) v = df_fma_lazy(df_neg(D[i * kPS + m]), x[m], v);
-    x[i] = df_div(df_norm(v), D[i * kPS + i]);
-    inv[i * kNB + j] = x[i];
-  }
-}
-
-// One 32-column step of the factorisation: the diagonal block (one warp), then its inverse
-// (warp 0) beside the panel (the other warps).  Ends with the CTA synchronised.
-__device__ __forceinline__ void chol_step(DF* A, int F, int c0, DF* D, DF* Pn, DF* Inv, int32_t* status) {
-  chol_diag(A, F, c0, D, status);
-  if (threadIdx.x < 32) tri_inverse(D, Inv + static_cast<size_t>(c0) * kNB);
-  else chol_panel(A, F, c0, D, Pn, threadIdx.x - 32, blockDim.x - 32);
-  __syncthreads();
 }
 
 // Asynchronous global -> shared copies (cp.async, completion tracked per thread by groups).
@@ -371,8 +444,9 @@ __device__ __forceinline__ void tri_solves(const DF* A, int F, DF* Z, int ldz, c
 // ([32][33] diagonal block + [F - 32][33] panel).
 __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __grid_constant__ FitParams P) {
   extern __shared__ __align__(16) DF fsm[];
-  DF* D = fsm;                                    // [32][33]
-  DF* Pn = fsm + kNB * kPS;                       // [F - 32][33]: rows padded so a warp's 32 rows hit distinct banks
+  // D, X, Lc, T, then the panel [F - 32][33] (rows padded so a warp's rows hit distinct banks)
+  const FactSmem S{fsm, fsm + kNB * kPS, fsm + 2 * kNB * kPS, fsm + 2 * kNB * kPS + kNB, fsm + kFactFixedDF, 0};
+  DF* Pn = S.Pn;
   const int F = P.k * kFD;
   const int tid = threadIdx.x;
   DF* A = reinterpret_cast<DF*>(P.scratch) +
@@ -387,55 +461,90 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __gri
     const int h = sys % P.H;
     const int kv = (sys / P.H) & 1;
     const int l = sys / (2 * P.H);
-    // 1. A = Xc^T Xc + lambda I (lower triangle) and Z = Xc^T Yc
-    for (int64_t e = tid; e < static_cast<int64_t>(F) * F; e += blockDim.x) {
-      const int r = static_cast<int>(e / F), c = static_cast<int>(e % F);
-      if (c > r) continue;
-      const int bi = r / kFD, bj = c / kFD;
-      const int pr = __ldg(&P.pair_of[(l * P.k + bi) * P.k + bj]);   // < 0: stored transposed
-      const size_t blk = ((static_cast<size_t>(kv) * P.H + h) * P.n_pairs + (pr >= 0 ? pr : -1 - pr)) * kFD * kFD;
-      const float g = pr >= 0 ? P.gram[blk + static_cast<size_t>(r % kFD) * kFD + (c % kFD)]
-                              : P.gram[blk + static_cast<size_t>(c % kFD) * kFD + (r % kFD)];
-      A[e] = r == c ? df_add(df_make(g), lam) : df_make(g);
+    // 1. A = Xc^T Xc + lambda I (the 128 x 128 blocks of the lower block triangle; the
+    //    block of two selected layers is stored once per pair, transposed when the pair
+    //    is) and Z = Xc^T Yc (contiguous per system); four entries per thread step
+    for (int bi = 0; bi < P.k; ++bi) {
+      for (int bj = 0; bj <= bi; ++bj) {
+        const int pr = __ldg(&P.pair_of[(l * P.k + bi) * P.k + bj]);   // < 0: stored transposed
+        const float* gb =
+            P.gram + ((static_cast<size_t>(kv) * P.H + h) * P.n_pairs + (pr >= 0 ? pr : -1 - pr)) * kFD * kFD;
+        for (int e = tid; e < kFD * kFD / 4; e += blockDim.x) {
+          const int er = e / (kFD / 4), ec = 4 * (e % (kFD / 4));
+          float g[4];
+          if (pr >= 0) {
+            const float4 v = *reinterpret_cast<const float4*>(gb + er * kFD + ec);
+            g[0] = v.x;
+            g[1] = v.y;
+            g[2] = v.z;
+            g[3] = v.w;
+          } else {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) g[q] = gb[(ec + q) * kFD + er];
+          }
+          DF o[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) o[q] = bi == bj && er == ec + q ? df_add(df_make(g[q]), lam) : df_make(g[q]);
+          float4* dst = reinterpret_cast<float4*>(A + static_cast<size_t>(bi * kFD + er) * F + bj * kFD + ec);
+          dst[0] = make_float4(o[0].hi, o[0].lo, o[1].hi, o[1].lo);
+          dst[1] = make_float4(o[2].hi, o[2].lo, o[3].hi, o[3].lo);
+        }
+      }
     }
-    for (int64_t e = tid; e < static_cast<int64_t>(F) * kFD; e += blockDim.x) {
-      const int r = static_cast<int>(e / kFD), j = static_cast<int>(e % kFD);
-      Z[e] = df_make(P.xty[(static_cast<size_t>(sys) * P.k + r / kFD) * kFD * kFD + static_cast<size_t>(r % kFD) * kFD + j]);
+    {
+      const float4* xs = reinterpret_cast<const float4*>(P.xty + static_cast<size_t>(sys) * P.k * kFD * kFD);
+      float4* zd = reinterpret_cast<float4*>(Z);
+      for (int e = tid; e < F * kFD / 4; e += blockDim.x) {
+        const float4 v = xs[e];
+        zd[2 * e] = make_float4(v.x, 0.f, v.y, 0.f);
+        zd[2 * e + 1] = make_float4(v.z, 0.f, v.w, 0.f);
+      }
     }
     __syncthreads();
     // 2. Cholesky A = L L^T, lower triangle in place, 32-column panels
     for (int c0 = 0; c0 < F; c0 += kNB) {
-      chol_step(A, F, c0, D, Pn, Inv, P.status);
-      // trailing update: A[i][j] -= P[i] . P[j] for c0+32 <= j <= i, in 32 x 32 tiles
+      FactSmem Sp = S;
+      Sp.pn_rows = F - c0 - kNB > 0 ? F - c0 - kNB : 1;
+      chol_step(A, F, c0, Sp, Inv, P.status);
+      // trailing update: A[i][j] -= P[i] . P[j] for c0+32 <= j <= i, in 32 x 32 tiles of the
+      // lower triangle, eight at a time; a tile is 64 threads of 4 x 4 entries (rows ri + 8a,
+      // columns cj + 8b: a warp's panel loads hit distinct banks), A's entries loaded first
       const int rows = F - c0 - kNB;
       const int nt = rows / kNB;
-      for (int tile = 0; tile < nt * (nt + 1) / 2; ++tile) {
+      const int lt = tid & 63, ri = lt >> 3, cj = lt & 7;
+      for (int tile = tid >> 6; tile < nt * (nt + 1) / 2; tile += kSolveThreads / 64) {
         int ti = 0;
         while ((ti + 1) * (ti + 2) / 2 <= tile) ++ti;
         const int tj = tile - ti * (ti + 1) / 2;
-        // thread: column jj (lane: the warp's stores are contiguous) and rows ii + 16q (warp w:
-        // ii = w), q < 2; the lane's panel row is read conflict-free (odd row stride), the
-        // warp's rows are broadcasts
-        constexpr int kRowsPer = kNB / kSolveWarps;
-        const int jj = tj * kNB + (tid & 31), ii = ti * kNB + (tid >> 5);
-        DF sacc[kRowsPer], aold[kRowsPer];
+        const int gi = ti * kNB + ri, gj = tj * kNB + cj;
+        DF acc[4][4], aold[4][4];
 #pragma unroll
-        for (int q = 0; q < kRowsPer; ++q) {   // A's entries are loaded before the products
-          sacc[q] = df_make(0.f);
-          aold[q] = jj <= ii + kSolveWarps * q ? A[static_cast<size_t>(c0 + kNB + ii + kSolveWarps * q) * F + c0 + kNB + jj]
-                                               : df_make(0.f);
-        }
-#pragma unroll 8
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+          for (int b = 0; b < 4; ++b) {
+            acc[a][b] = df_make(0.f);
+            aold[a][b] = gj + 8 * b <= gi + 8 * a ? A[static_cast<size_t>(c0 + kNB + gi + 8 * a) * F + c0 + kNB + gj + 8 * b]
+                                                  : df_make(0.f);
+          }
+#pragma unroll 4
         for (int m = 0; m < kNB; ++m) {
-          const DF pj = Pn[jj * kPS + m];
+          DF pi[4], pj[4];
 #pragma unroll
-          for (int q = 0; q < kRowsPer; ++q) sacc[q] = df_fma_lazy(Pn[(ii + kSolveWarps * q) * kPS + m], pj, sacc[q]);
+          for (int a = 0; a < 4; ++a) pi[a] = Pn[(gi + 8 * a) * kPS + m];
+#pragma unroll
+          for (int b = 0; b < 4; ++b) pj[b] = Pn[(gj + 8 * b) * kPS + m];
+#pragma unroll
+          for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int b = 0; b < 4; ++b) acc[a][b] = df_fma_lazy(pi[a], pj[b], acc[a][b]);
         }
 #pragma unroll
-        for (int q = 0; q < kRowsPer; ++q) {
-          DF* a = A + static_cast<size_t>(c0 + kNB + ii + kSolveWarps * q) * F + c0 + kNB + jj;
-          if (jj <= ii + kSolveWarps * q) *a = df_add(aold[q], df_neg(df_norm(sacc[q])));
-        }
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+          for (int b = 0; b < 4; ++b)
+            if (gj + 8 * b <= gi + 8 * a)
+              A[static_cast<size_t>(c0 + kNB + gi + 8 * a) * F + c0 + kNB + gj + 8 * b] =
+                  df_add(aold[a][b], df_neg(df_norm(acc[a][b])));
       }
       __syncthreads();
     }
@@ -463,10 +572,13 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __gri
 // The matrix is too large for the panel to stay in shared memory: the trailing update
 // runs in 64 x 64 tiles whose two 64-row panel slices are staged per tile.
 constexpr int kXT = 64;                           // trailing-update tile
+constexpr int kXPanelRows = 256;                  // panel rows staged at a time
 __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_xh_kernel(const __grid_constant__ FitParams P) {
   extern __shared__ __align__(16) DF fsm[];
-  DF* D = fsm;                                    // [32][33]
-  DF* Pi = fsm + kNB * kPS;                       // [64][33]: panel rows of the tile's row block
+  // D, X, Lc, T, then a chunk of panel rows [kXPanelRows][33]; the trailing update's slices
+  // of the panel take the chunk's place
+  const FactSmem S{fsm, fsm + kNB * kPS, fsm + 2 * kNB * kPS, fsm + 2 * kNB * kPS + kNB, fsm + kFactFixedDF, kXPanelRows};
+  DF* Pi = S.Pn;                                  // [64][33]: panel rows of the tile's row block
   DF* Pj = Pi + kXT * kPS;                        // [64][33]: panel rows of its column block
   const int H = P.H, R = P.R;
   const int F = P.k * H * kFD;
@@ -513,7 +625,7 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_xh_kernel(const __
     __syncthreads();
     // 2. Cholesky, 32-column panels; trailing update in 64 x 64 tiles of the lower triangle
     for (int c0 = 0; c0 < F; c0 += kNB) {
-      chol_step(A, F, c0, D, nullptr, Inv, P.status);
+      chol_step(A, F, c0, S, Inv, P.status);
       const int base = c0 + kNB, rows = F - base;
       const int nt = (rows + kXT - 1) / kXT;
       // thread: column jj = tid % 64 of the tile, rows ii + 8q (ii = tid / 64), q < 8
@@ -868,8 +980,7 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
     }
     // the factorisation's diagonal block and panel (per head) or tile slices (cross-head),
     // or the solves' staged chunk
-    const size_t fact = pl.cross ? static_cast<size_t>(kNB + 2 * kXT) * kPS
-                                 : static_cast<size_t>(kNB) * kPS + static_cast<size_t>(pl.F - kNB) * kPS;
+    const size_t fact = kFactFixedDF + static_cast<size_t>(pl.cross ? kXPanelRows : pl.F - kNB) * kPS;
     const size_t smem = std::max(fact, static_cast<size_t>(2) * kStageDF) * 8;
     auto kernel = pl.cross ? fit_solve_xh_kernel : fit_solve_kernel;
     if ((e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem))) !=
