@@ -19,13 +19,15 @@
 //    target layers whose selection holds both; the k blocks of Xc^T Yc are per target layer.
 // 2. fit_solve_kernel: one CTA per system at a time (persistent); the block grid is
 //    widened to float-float pairs (~48 significant bits, on the FP32 units) into a per-CTA
-//    scratch matrix, lambda added, factorised by a blocked right-looking Cholesky
-//    (32-column panels: diagonal block in shared memory, then its inverse by one warp beside
-//    the panel by forward substitution on the others, trailing update), then the two
-//    triangular solves for the d right-hand sides in 32-row blocks (products with the
-//    solved rows, then the inverse diagonal block) and the bias; W and b are written in
-//    fp32.  fit_solve_xh_kernel does the same for the
-//    cross-head systems, with the trailing update staged per 64 x 64 tile.
+//    scratch matrix, lambda added, factorised by a blocked right-looking Cholesky (32-column
+//    steps: the diagonal block factored by the CTA, its inverse, the panel as a product
+//    with that inverse, the trailing update), then the two triangular solves for the d
+//    right-hand sides in 32-row blocks (products with the solved rows, then the inverse
+//    diagonal block) and the bias; W and b are written in fp32.
+//    Cross-head systems: fit_solve_xh_kernel factorises one system per CTA (trailing
+//    update staged per 128 x 128 tile), then fit_trisolve_xh_kernel solves and writes W and
+//    b per (system, target head), so that the solves of fewer systems than SMs still fill
+//    the GPU.
 // kvx_fit_ridge runs them on the caller's stream, with stream-ordered workspace, and
 // synchronises before it returns (the fit is an offline step).
 #include <cuda_runtime.h>
@@ -68,6 +70,7 @@ struct FitParams {
   double lambda;
   int32_t* status;
   int32_t R;                        // right-hand sides per system: 128 (per head) or H 128 (cross-head)
+  int32_t sys0;                     // cross-head: first system of this launch (scratch slot = its offset)
 };
 
 __device__ __forceinline__ size_t sums_index(const FitParams& P, int side, int kv, int layer, int h) {
@@ -570,16 +573,16 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __gri
 // layer-major, head-minor), R = H 128 right-hand sides (every target head of the layer),
 // so X_c^T X_c is formed and factored once per target layer and shared by its heads.
 // The matrix is too large for the panel to stay in shared memory: the trailing update
-// runs in 64 x 64 tiles whose two 64-row panel slices are staged per tile.
-constexpr int kXT = 64;                           // trailing-update tile
-constexpr int kXPanelRows = 256;                  // panel rows staged at a time
+// runs in 128 x 128 tiles whose two 128-row panel slices are staged per tile.  One system
+// per CTA and launch (scratch slot = blockIdx.x); fit_trisolve_xh_kernel then solves.
+constexpr int kXT = 128;                          // trailing-update tile
+constexpr int kXPanelRows = 512;                  // panel rows staged at a time
+static_assert(4 * kXT <= kXPanelRows, "the trailing update's two buffers of panel slices take the panel chunk's place");
 __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_xh_kernel(const __grid_constant__ FitParams P) {
   extern __shared__ __align__(16) DF fsm[];
-  // D, X, Lc, T, then a chunk of panel rows [kXPanelRows][33]; the trailing update's slices
-  // of the panel take the chunk's place
+  // D, X, Lc, T, then a chunk of panel rows [kXPanelRows][33]; the trailing update's two
+  // buffers of panel slices ([2][128][33] each) take the chunk's place
   const FactSmem S{fsm, fsm + kNB * kPS, fsm + 2 * kNB * kPS, fsm + 2 * kNB * kPS + kNB, fsm + kFactFixedDF, kXPanelRows};
-  DF* Pi = S.Pn;                                  // [64][33]: panel rows of the tile's row block
-  DF* Pj = Pi + kXT * kPS;                        // [64][33]: panel rows of its column block
   const int H = P.H, R = P.R;
   const int F = P.k * H * kFD;
   const int tid = threadIdx.x;
@@ -589,10 +592,11 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_xh_kernel(const __
   DF* Z = A + static_cast<size_t>(F) * F;         // [F][R]
   DF* Inv = Z + static_cast<size_t>(F) * R;       // [F / 32][32][32]: inverses of the diagonal blocks
   const int n_sys = P.Lt * 2;
-  const double inv_n = 1.0 / (static_cast<double>(P.B) * P.T);
   const DF lam = df_from_double(P.lambda);
   constexpr size_t kBlk = static_cast<size_t>(kFD) * kFD;
-  for (int sys = blockIdx.x; sys < n_sys; sys += gridDim.x) {
+  {
+    const int sys = P.sys0 + static_cast<int>(blockIdx.x);
+    if (sys >= n_sys) return;
     const int kv = sys & 1;
     const int l = sys >> 1;
     // 1. A = Xc^T Xc + lambda I (lower triangle) from the source-pair blocks, Z = Xc^T Yc
@@ -623,62 +627,117 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_xh_kernel(const __
                            static_cast<size_t>(r % kFD) * kFD + col % kFD]);
     }
     __syncthreads();
-    // 2. Cholesky, 32-column panels; trailing update in 64 x 64 tiles of the lower triangle
+    // 2. Cholesky, 32-column panels; trailing update in 128 x 128 tiles of the lower triangle
     for (int c0 = 0; c0 < F; c0 += kNB) {
       chol_step(A, F, c0, S, Inv, P.status);
+      // trailing update in 128 x 128 tiles of the lower triangle: the tile's two 128-row
+      // slices of the panel staged in shared memory by cp.async, the next tile's while this
+      // one computes (two buffers); thread = 8 rows (ri + 16a) x 4 columns (cj + 32b), so a
+      // warp's row loads are broadcasts; the sums start from A's entries (loaded while the
+      // slices land) and are written back without a wait
       const int base = c0 + kNB, rows = F - base;
-      const int nt = (rows + kXT - 1) / kXT;
-      // thread: column jj = tid % 64 of the tile, rows ii + 8q (ii = tid / 64), q < 8
-      const int jj = tid % kXT, ii = tid / kXT;
-      for (int tile = 0; tile < nt * (nt + 1) / 2; ++tile) {
-        int ti = 0;
+      const int nt = (rows + kXT - 1) / kXT, ntiles = nt * (nt + 1) / 2;
+      const int ri = tid >> 5, cj = tid & 31;
+      auto tile_ij = [](int tile, int& ti, int& tj) {
+        ti = 0;
         while ((ti + 1) * (ti + 2) / 2 <= tile) ++ti;
-        const int tj = tile - ti * (ti + 1) / 2;
+        tj = tile - ti * (ti + 1) / 2;
+      };
+      auto issue_slices = [&](int tile, DF* dst) {
+        int ti, tj;
+        tile_ij(tile, ti, tj);
         for (int e = tid; e < 2 * kXT * kNB; e += blockDim.x) {
-          const int s = e / (kXT * kNB), rr = (e / kNB) % kXT, m = e % kNB;
-          const int row = (s == 0 ? ti : tj) * kXT + rr;
-          (s == 0 ? Pi : Pj)[rr * kPS + m] = row < rows ? A[static_cast<size_t>(base + row) * F + c0 + m] : df_make(0.f);
+          const int sl = e / (kXT * kNB), rr = (e / kNB) % kXT, m = e % kNB;
+          const int row = (sl == 0 ? ti : tj) * kXT + rr;
+          DF* d = dst + (sl * kXT + rr) * kPS + m;
+          if (row < rows) cp_async8(d, A + static_cast<size_t>(base + row) * F + c0 + m);
+          else *d = df_make(0.f);
         }
-        constexpr int kQ = kXT * kXT / kSolveThreads;   // 8
-        const int gj = tj * kXT + jj;
-        DF sacc[kQ], aold[kQ];
+        cp_async_commit();
+      };
+      if (ntiles > 0) issue_slices(0, S.Pn);
+      for (int tile = 0; tile < ntiles; ++tile) {
+        int ti, tj;
+        tile_ij(tile, ti, tj);
+        if (tile + 1 < ntiles) issue_slices(tile + 1, S.Pn + ((tile + 1) & 1) * 2 * kXT * kPS);
+        // this thread's entries: rows gi0 + 16a, columns gj0 + 32b of the trailing block
+        const int gi0 = ti * kXT + ri, gj0 = tj * kXT + cj;
+        DF* const a0 = A + static_cast<size_t>(base + gi0) * F + base + gj0;
+        const size_t row16 = static_cast<size_t>(16) * F;
+        DF acc[8][4];
 #pragma unroll
-        for (int q = 0; q < kQ; ++q) {   // A's entries are loaded before the products
-          const int gi = ti * kXT + ii + 8 * q;
-          sacc[q] = df_make(0.f);
-          aold[q] = gi < rows && gj <= gi ? A[static_cast<size_t>(base + gi) * F + base + gj] : df_make(0.f);
-        }
+        for (int a = 0; a < 8; ++a)
+#pragma unroll
+          for (int b = 0; b < 4; ++b)
+            acc[a][b] = gi0 + 16 * a < rows && gj0 + 32 * b <= gi0 + 16 * a ? a0[a * row16 + 32 * b] : df_make(0.f);
+        if (tile + 1 < ntiles) cp_async_wait<1>();
+        else cp_async_wait<0>();
         __syncthreads();
-#pragma unroll 4
+        const DF* Pi = S.Pn + (tile & 1) * 2 * kXT * kPS;
+        const DF* Pj = Pi + kXT * kPS;
+#pragma unroll 2
         for (int m = 0; m < kNB; ++m) {
-          const DF pj = Pj[jj * kPS + m];
+          DF pi[8], pj[4];
 #pragma unroll
-          for (int q = 0; q < kQ; ++q) sacc[q] = df_fma_lazy(Pi[(ii + 8 * q) * kPS + m], pj, sacc[q]);
+          for (int a = 0; a < 8; ++a) pi[a] = Pi[(ri + 16 * a) * kPS + m];
+#pragma unroll
+          for (int b = 0; b < 4; ++b) pj[b] = Pj[(cj + 32 * b) * kPS + m];
+#pragma unroll
+          for (int a = 0; a < 8; ++a)
+#pragma unroll
+            for (int b = 0; b < 4; ++b) acc[a][b] = df_fma_lazy(df_neg(pi[a]), pj[b], acc[a][b]);
         }
 #pragma unroll
-        for (int q = 0; q < kQ; ++q) {
-          const int gi = ti * kXT + ii + 8 * q;
-          if (gi < rows && gj <= gi) A[static_cast<size_t>(base + gi) * F + base + gj] = df_add(aold[q], df_neg(df_norm(sacc[q])));
-        }
-        __syncthreads();
+        for (int a = 0; a < 8; ++a)
+#pragma unroll
+          for (int b = 0; b < 4; ++b)
+            if (gi0 + 16 * a < rows && gj0 + 32 * b <= gi0 + 16 * a) a0[a * row16 + 32 * b] = df_norm(acc[a][b]);
+        __syncthreads();   // the buffer is free for the slices of tile + 2
       }
     }
-    // 3. forward and backward solves, 128 right-hand sides (one target head) at a time
-    for (int c0 = 0; c0 < R; c0 += kFD) tri_solves(A, F, Z + c0, R, Inv, fsm);
-    // 4. W (fp32, [L_t][2][H][F][128]) and b = mean(Y) - mean(X) W (fp64)
-    for (int64_t e = tid; e < static_cast<int64_t>(F) * R; e += blockDim.x) {
-      const int r = static_cast<int>(e / R), col = static_cast<int>(e % R);
-      P.W[((static_cast<size_t>(sys) * H + col / kFD) * F + r) * kFD + col % kFD] = __fadd_rn(Z[e].hi, Z[e].lo);
+  }
+}
+
+// Cross-head triangular solves and outputs, one unit per (system of the launch, target
+// head): the factor, its inverted diagonal blocks and the right-hand sides come from the
+// scratch slot that fit_solve_xh_kernel factored, and the H units of a system run on
+// different SMs (the factorisation occupies one SM per system; there are often fewer
+// systems than SMs).
+__global__ void __launch_bounds__(kSolveThreads, 1) fit_trisolve_xh_kernel(const __grid_constant__ FitParams P,
+                                                                           int n_slots) {
+  extern __shared__ __align__(16) DF fsm[];
+  const int H = P.H, R = P.R;
+  const int F = P.k * H * kFD;
+  const int tid = threadIdx.x;
+  const double inv_n = 1.0 / (static_cast<double>(P.B) * P.T);
+  const int n_units = n_slots * H;
+  for (int u = blockIdx.x; u < n_units; u += gridDim.x) {
+    const int slot = u / H, ht = u % H;
+    const int sys = P.sys0 + slot;
+    const int kv = sys & 1, l = sys >> 1;
+    DF* A = reinterpret_cast<DF*>(P.scratch) +
+            static_cast<size_t>(slot) * (static_cast<size_t>(F) * F + static_cast<size_t>(F) * R +
+                                         static_cast<size_t>(F) * kNB);
+    DF* Z = A + static_cast<size_t>(F) * F;
+    const DF* Inv = Z + static_cast<size_t>(F) * R;
+    DF* Zh = Z + static_cast<size_t>(ht) * kFD;   // this head's 128 columns, leading dimension R
+    tri_solves(A, F, Zh, R, Inv, fsm);
+    // W (fp32, [L_t][2][H][F][128]) and b = mean(Y) - mean(X) W (fp64) of target head ht
+    float* Wout = P.W + (static_cast<size_t>(sys) * H + ht) * F * kFD;
+    for (int64_t e = tid; e < static_cast<int64_t>(F) * kFD; e += blockDim.x) {
+      const int r = static_cast<int>(e / kFD), c = static_cast<int>(e % kFD);
+      const DF z = Zh[static_cast<size_t>(r) * R + c];
+      Wout[e] = __fadd_rn(z.hi, z.lo);
     }
-    for (int col = tid; col < R; col += blockDim.x) {
-      const int ht = col / kFD, c = col % kFD;
-      double acc = P.sums[sums_index(P, 1, kv, l, ht) + c] * inv_n;
+    if (tid < kFD) {
+      double acc = P.sums[sums_index(P, 1, kv, l, ht) + tid] * inv_n;
       for (int r = 0; r < F; ++r) {
-        const int u = r / kFD;
-        const int layer = __ldg(&P.sel[l * P.k + u / H]);
-        acc -= P.sums[sums_index(P, 0, kv, layer, u % H) + r % kFD] * inv_n * df_to_double(Z[static_cast<size_t>(r) * R + col]);
+        const int uu = r / kFD;
+        const int layer = __ldg(&P.sel[l * P.k + uu / H]);
+        acc -= P.sums[sums_index(P, 0, kv, layer, uu % H) + r % kFD] * inv_n *
+               df_to_double(Zh[static_cast<size_t>(r) * R + tid]);
       }
-      P.b[(static_cast<size_t>(sys) * H + ht) * kFD + c] = static_cast<float>(acc);
+      P.b[(static_cast<size_t>(sys) * H + ht) * kFD + tid] = static_cast<float>(acc);
     }
     __syncthreads();
   }
@@ -984,13 +1043,28 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
     const size_t smem = std::max(fact, static_cast<size_t>(2) * kStageDF) * 8;
     auto kernel = pl.cross ? fit_solve_xh_kernel : fit_solve_kernel;
     if ((e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem))) !=
-        cudaSuccess) {
+            cudaSuccess ||
+        (pl.cross && (e = cudaFuncSetAttribute(fit_trisolve_xh_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               static_cast<int>(smem))) != cudaSuccess)) {
       set_error(std::string("kvx_fit_ridge: smem attribute: ") + cudaGetErrorString(e));
       result = KVX_ERR_CUDA;
       break;
     }
     timer.begin(3);
-    kernel<<<pl.solve_grid, kSolveThreads, smem, st>>>(P);
+    if (!pl.cross) {
+      kernel<<<pl.solve_grid, kSolveThreads, smem, st>>>(P);
+    } else {
+      // waves of solve_grid systems (the scratch holds that many factors): factorise, then
+      // the triangular solves of the wave's systems, one unit per (system, target head)
+      const int n_sys = static_cast<int>(pl.n_sys);
+      for (int s0 = 0; s0 < n_sys; s0 += pl.solve_grid) {
+        P.sys0 = s0;
+        const int slots = std::min(pl.solve_grid, n_sys - s0);
+        fit_solve_xh_kernel<<<slots, kSolveThreads, smem, st>>>(P);
+        const int units = slots * static_cast<int>(cfg->n_kv_heads);
+        fit_trisolve_xh_kernel<<<std::min(units, std::max(sms, 1)), kSolveThreads, smem, st>>>(P, slots);
+      }
+    }
     timer.end();
     if ((e = cudaGetLastError()) != cudaSuccess) {
       set_error(std::string("kvx_fit_ridge: launch: ") + cudaGetErrorString(e));
