@@ -294,6 +294,22 @@ def test_fit_cross_head_small_every_system(over, lam):
     _check_xh_systems(w, lam, sel, caches, Wg, bg, [(l, kv) for l in range(w.Lt) for kv in range(2)])
 
 
+def test_fit_cross_head_more_systems_than_sms():
+    """160 cross-head systems (80 target layers x K|V) on a 152-SM GB300: the factorisation
+    runs in two waves of per-CTA scratch slots and the solves of each wave fill every SM;
+    every output is written, and systems of both waves (the first and last of each) match
+    the oracle on every target head."""
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4_xhead", Ls=6, Lt=80, H=2, B=1, T=400, k=1)
+    sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
+    caches, Wg, bg = _run_fit_xh(w, 0.01, sel)
+    assert np.all(np.isfinite(Wg)) and np.all(np.isfinite(bg)), "unwritten outputs"
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    assert 2 * w.Lt > n_sm
+    last = 2 * w.Lt - 1
+    systems = sorted({(s // 2, s % 2) for s in (0, 1, n_sm - 1, n_sm, n_sm + 1, last)})
+    _check_xh_systems(w, 0.01, sel, caches, Wg, bg, systems)
+
+
 def test_fit_cross_head_one_head_equals_per_head():
     """With one KV head the cross-head feature is the per-head one: both modes of the GPU fit
     solve the same systems (different kernels), so they agree within the fit bound."""
