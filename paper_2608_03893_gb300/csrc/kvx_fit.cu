@@ -318,6 +318,7 @@ template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 constexpr int kStageDF = kNB * kPS + kNB * kFD;   // one solve stage: [32][33] L entries + [32][128] rows
+constexpr int kStages = 3;                         // solve stage buffers
 
 // The two triangular solves with the factor L (lower triangle of A, leading dimension F)
 // for 128 right-hand-side columns Z[0 .. F)[0 .. 128) (leading dimension ldz), in place:
@@ -326,10 +327,10 @@ constexpr int kStageDF = kNB * kPS + kNB * kFD;   // one solve stage: [32][33] L
 // staged in shared memory; thread = 2 rows x 4 columns, 8 independent sums), then is
 // multiplied by the inverse of its diagonal block (Inv, [F / 32][32][32], from the
 // factorisation; its transpose in the backward solve), the same staged product with every
-// thread busy.  Stages run through two shared-memory buffers: the next stage's operands
+// thread busy.  Stages run through three shared-memory buffers: the next stage's operands
 // are copied asynchronously while the current one computes, except where they are the
 // rows the current stage solves (the chunk orders keep that to one stage per direction).
-// fsm: 2 x kStageDF pairs.
+// fsm: kStages x kStageDF pairs.
 __device__ __forceinline__ void tri_solves(const DF* A, int F, DF* Z, int ldz, const DF* Inv, DF* fsm) {
   const int tid = threadIdx.x;
   constexpr int kR = kNB * kFD / 4 / kSolveThreads;   // rows per thread (2)
@@ -393,8 +394,8 @@ __device__ __forceinline__ void tri_solves(const DF* A, int F, DF* Z, int ldz, c
 #pragma unroll
     for (int a = 0; a < kR; ++a) load4(&Z[static_cast<size_t>(b * kNB + r0 + a) * ldz + q0], acc[a]);
     while (bi < nb) {
-      DF* cur = fsm + (k & 1) * kStageDF;
-      DF* nxt = fsm + ((k + 1) & 1) * kStageDF;
+      DF* cur = fsm + (k % kStages) * kStageDF;
+      DF* nxt = fsm + ((k + 1) % kStages) * kStageDF;
       const int bi2 = u < bi ? bi : bi + 1, u2 = u < bi ? u + 1 : 0;
       int b2 = 0, mc2 = 0;
       const bool more = bi2 < nb;
@@ -428,8 +429,14 @@ __device__ __forceinline__ void tri_solves(const DF* A, int F, DF* Z, int ldz, c
 #pragma unroll
           for (int c = 0; c < 4; ++c) Z[static_cast<size_t>(b * kNB + r0 + a) * ldz + q0 + c] = df_norm(res[a][c]);
       }
-      __syncthreads();
-      if (defer) issue(nxt, fwd, b2, mc2);
+      // With three buffers the next issue targets the buffer of the stage two before this
+      // one, which every thread left before the barrier above.  A diagonal stage ends with a
+      // barrier: the next iteration issues its copies before its own barrier, and those may
+      // read the rows this stage solved.
+      if (mc < 0) {
+        __syncthreads();
+        if (defer) issue(nxt, fwd, b2, mc2);
+      }
       if (more && mc < 0) {   // a new block starts: its right-hand sides
 #pragma unroll
         for (int a = 0; a < kR; ++a) load4(&Z[static_cast<size_t>(b2 * kNB + r0 + a) * ldz + q0], acc[a]);
@@ -440,6 +447,7 @@ __device__ __forceinline__ void tri_solves(const DF* A, int F, DF* Z, int ldz, c
       mc = mc2;
       ++k;
     }
+    __syncthreads();   // the direction's last stage is done with its buffer and its rows are written
   }
 }
 
@@ -1040,7 +1048,7 @@ KVX_API kvx_status kvx_fit_ridge(const kvx_fit_config* cfg, const kvx_src* src, 
     // the factorisation's diagonal block and panel (per head) or tile slices (cross-head),
     // or the solves' staged chunk
     const size_t fact = kFactFixedDF + static_cast<size_t>(pl.cross ? kXPanelRows : pl.F - kNB) * kPS;
-    const size_t smem = std::max(fact, static_cast<size_t>(2) * kStageDF) * 8;
+    const size_t smem = std::max(fact, static_cast<size_t>(kStages) * kStageDF) * 8;
     auto kernel = pl.cross ? fit_solve_xh_kernel : fit_solve_kernel;
     if ((e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem))) !=
             cudaSuccess ||
