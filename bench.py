@@ -251,7 +251,8 @@ def oracle_sample_rate(w, budget_s, seed=0, ctx_sel=None):
         svf = obf16.decode(sv.view(torch.int16).numpy().view(np.uint16))
         p = pos[rows[:, 0], rows[:, 1]]
         t0 = time.perf_counter()
-        omap.map_tokens(skf, svf, p, sel, Wf, bf, w.theta_s, w.theta_t, mode="bf16fwd", head_mix=w.head_mix)
+        omap.map_tokens(skf, svf, p, sel, Wf, bf, w.theta_s, w.theta_t, mode="bf16fwd", head_mix=w.head_mix,
+                        style=w.rope_style)
         return time.perf_counter() - t0
 
     n, dt = 8, run(8)
@@ -298,7 +299,7 @@ def reference_arm(args, w, config):
         svf = obf16.decode(syn.source_rows(w, 1, rows).view(torch.int16).numpy().view(np.uint16))
         t0 = time.perf_counter()
         omap.map_tokens(skf, svf, pos[rows[:, 0], rows[:, 1]], sel, Wf, bf, w.theta_s, w.theta_t,
-                        mode="bf16fwd", head_mix=w.head_mix)
+                        mode="bf16fwd", head_mix=w.head_mix, style=w.rope_style)
         dt = time.perf_counter() - t0
         if i >= args.warmup:
             times.append(dt)
@@ -324,7 +325,8 @@ def make_mapper(w, dev_index):
     cfg, keep = kvx.config_from_tensors(
         src_layers=w.Ls, tgt_layers=w.Lt, n_kv_heads=w.H, head_dim=w.d, k=w.k, theta_s=w.theta_s,
         theta_t=w.theta_t, cache_dtype=w.cache_dtype, W=W, b=b, scores=syn.selection_scores(w),
-        head_mix=kvx.KVX_CROSS_HEAD if w.head_mix == "cross_head" else kvx.KVX_PER_HEAD)
+        head_mix=kvx.KVX_CROSS_HEAD if w.head_mix == "cross_head" else kvx.KVX_PER_HEAD,
+        rope_style=kvx.KVX_ROPE_INTERLEAVED if w.rope_style == "interleaved" else kvx.KVX_ROPE_HALF)
     return kvx.kvx_create(cfg, dev_index)
 
 
@@ -725,6 +727,8 @@ def main():
               "parallelism": "replicas x%d" % args.gpus,
               "l2": "no flush: each step streams %.1f GB (source read + target write) vs 129 MB L2"
                     % (alg["bytes"] / 1e9)}
+    if w.rope_style != "half":
+        config["rope_pairs"] = w.rope_style
     if args.impl == "reference":
         return reference_arm(args, w, config)
 

@@ -121,6 +121,7 @@ class Workload:
     len_range: tuple = (0, 0)   # initial per-sequence lengths (paged), inclusive
     head_mix: str = "per_head"  # "per_head" (F = k d) | "cross_head" (F = k H d, the paper's)
     rope_scaling: tuple = ()    # Llama-3 frequency scaling of both models, or () for plain theta
+    rope_style: str = "half"    # RoPE pairs: "half" (i, i + d/2) | "interleaved" (2i, 2i + 1)
     notes: str = field(default="", compare=False)
 
     @property
