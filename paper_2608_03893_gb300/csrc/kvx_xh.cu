@@ -87,6 +87,7 @@ struct XhParams {
   int32_t* status;
   int32_t Lt, H, k, pairs, n_units, out_bh;
   int32_t lo_steps;       // fp32 weights: k n_kv further K steps over the same source tiles with W_lo
+  int32_t per_head;       // per-head W widened with zeros: a pass runs only its own two source heads' steps
   int32_t hf;             // the Hugging Face forward's RoPE rounding (kvx_rope_numerics)
   int32_t il;             // interleaved RoPE pairs (2i, 2i+1) instead of (i, i + 64)
   RopeTables rope;
@@ -257,7 +258,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
   cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
-  const int H = P.H, k = P.k, src_steps = P.k * P.H, steps = src_steps + P.lo_steps;
+  // A unit's K steps: (layer j, head hs) source tiles in the feature order, then (fp32 W) the
+  // same again with W_lo.  For a per-head mapper (W widened with zeros outside each head's
+  // rows) only the pass's own heads hs = 2 pass, 2 pass + 1 meet non-zero rows, so the unit
+  // runs those 2k steps alone.
+  const int H = P.H, k = P.k, src_steps = P.k * P.H;
+  const int unit_src = P.per_head ? 2 * P.k : src_steps;
+  const int steps = unit_src * (P.lo_steps ? 2 : 1);
   const int n_units = P.n_units, pairs = P.pairs;
   const MapArgs& A = P.a;
 
@@ -279,8 +286,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
           const int st = static_cast<int>(sn % kXStages);
           const uint32_t round = sn / kXStages;
           if (round == 0 || mbar_test_wait(smem_u32(&empty[st]), (round - 1) & 1u)) {
-            // step ss: source layer sel[l][ss / H], head ss % H; features ss*128 .. of W^T
-            const int j = (ss % src_steps) / H, hs = ss % H;
+            // step ss -> feature block fb: source layer sel[l][(fb % src_steps) / H], head
+            // fb % H; W^T columns fb*128 ..
+            int fb = ss;
+            if (P.per_head) {
+              const int part = ss / unit_src, s2 = ss % unit_src;
+              fb = part * src_steps + (s2 >> 1) * H + 2 * sun.pass + (s2 & 1);
+            }
+            const int j = (fb % src_steps) / H, hs = fb % H;
             const int L = __ldg(&P.sel[sun.l * k + j]);
             if (rank == 0) mbar_expect_tx(smem_u32(&full[st]), 2 * kXStageBytes);
             const uint32_t bar = mapa_shared(smem_u32(&full[st]), 0);
@@ -290,8 +303,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
             tma_load_5d_pair(a_dst, tma, bar, 0, sun.t0, hs, sun.b, L, pol_a);
             tma_load_5d_pair(a_dst + kXABytes / 2, tma, bar, 64, sun.t0, hs, sun.b, L, pol_a);
             const int wrow = ((sun.l * 2 + sun.kv) * H + 2 * sun.pass) * kXD + static_cast<int>(rank) * 128;
-            tma_load_2d_pair(b_dst, &P.tm_w, bar, ss * kXD, wrow, pol_w);
-            tma_load_2d_pair(b_dst + kXBBytes / 2, &P.tm_w, bar, ss * kXD + 64, wrow, pol_w);
+            tma_load_2d_pair(b_dst, &P.tm_w, bar, fb * kXD, wrow, pol_w);
+            tma_load_2d_pair(b_dst + kXBBytes / 2, &P.tm_w, bar, fb * kXD + 64, wrow, pol_w);
             ++sn;
             if (++ss == steps) {
               ss = 0;
@@ -763,6 +776,7 @@ kvx_status launch_xh(kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
   }
   P.n_units = static_cast<int>(units);
   P.lo_steps = c->weight_dtype == KVX_F32 ? c->k * c->H : 0;
+  P.per_head = c->head_mix == KVX_PER_HEAD ? 1 : 0;
   P.hf = c->rope_numerics == KVX_ROPE_HF;
   P.il = c->rope_style == KVX_ROPE_INTERLEAVED;
   P.rope = c->rope;

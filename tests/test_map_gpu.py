@@ -692,6 +692,7 @@ def test_cross_head_tc_fp32_weights_hi_lo():
 @pytest.mark.parametrize("over", [
     dict(Ls=6, Lt=5, H=2, B=2, T=300, k=3),                 # ragged tail, B > 1
     dict(Ls=8, Lt=9, H=2, B=1, T=256, k=4, scores="uniform"),  # k = 4, reloads
+    dict(Ls=9, Lt=3, H=4, B=1, T=200, k=6),                 # k = 6: cross-head kernel, per-head steps, W_lo pass
 ])
 def test_per_head_tc_fp32_weights_hi_lo(over):
     """Per-head tensor-core kernel with fp32 W: each use takes a hi and a lo W stage over
