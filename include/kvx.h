@@ -265,9 +265,10 @@ KVX_API int64_t kvx_mapper_params(int32_t tgt_layers, int32_t n_kv_heads, int32_
  * target heads of layer l, so each (l, K|V) is one system (Xc^T Xc + lambda I) W_l =
  * Xc^T Yc_l with F = k*H*128 unknowns and H*128 right-hand sides (Xc^T Xc formed and
  * factored once per target layer, shared across its heads, Sec. 3.1); W is written as
- * [L_t][2][H][k*H*d][d] (k >= 1, k*H*128 <= 16384).  The solve scratch is F*(F + H*128)
- * float pairs per concurrent system (at most 80 GB; beyond that fewer systems run at
- * once).  Cross-products of the centred values run
+ * [L_t][2][H][k*H*d][d] (k >= 1, k*H*128 <= 16384).  The solve scratch is
+ * F*(F + H*128 + 32) float pairs per concurrent system (the matrix, the right-hand sides
+ * and the inverted 32 x 32 diagonal blocks of the factor; at most 80 GB, beyond which the
+ * systems are factored and solved in waves).  Cross-products of the centred values run
  * on the tensor cores from a bf16 hi + lo split of each value (within 2^-17 of it) and
  * accumulate in fp32; the factorisation and the solves run in float-float arithmetic (each
  * value an unevaluated sum of two fp32 numbers, about 48 significant bits) on the FP32
