@@ -180,7 +180,8 @@ constexpr int kFactFixedDF = 2 * kNB * kPS + kNB + 16 * 17;   // D, X, Lc, T
 // Cholesky of the 32 x 32 diagonal block at (c0, c0) of A (lower triangle) by the CTA:
 // step j, warp 0 forms column j of L (the pivot through a float-float reciprocal square
 // root), then every thread updates its entries (i, m), j < m <= i.  A pivot <= 0 is
-// reported and replaced by 1 so the call finishes.  Ends synchronised.
+// reported and its reciprocal square root taken as 1 so the call finishes.  Ends
+// synchronised.
 __device__ __forceinline__ void chol_diag(const DF* A, int F, int c0, const FactSmem& S, int32_t* status) {
   const int tid = threadIdx.x;
   DF* D = S.D;

@@ -295,15 +295,15 @@ def test_fit_cross_head_small_every_system(over, lam):
 
 
 def test_fit_cross_head_more_systems_than_sms():
-    """160 cross-head systems (80 target layers x K|V) on a 152-SM GB300: the factorisation
-    runs in two waves of per-CTA scratch slots and the solves of each wave fill every SM;
-    every output is written, and systems of both waves (the first and last of each) match
-    the oracle on every target head."""
-    w = syn.workload("qwen3_14b_32b_b8x1024_k4_xhead", Ls=6, Lt=80, H=2, B=1, T=400, k=1)
+    """More cross-head systems (target layers x K|V) than SMs (160 on a 152-SM GB300): the
+    factorisation runs in two waves of per-CTA scratch slots and the solves of each wave
+    fill every SM; every output is written, and systems of both waves (the first and last
+    of each) match the oracle on every target head."""
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4_xhead", Ls=6, Lt=n_sm // 2 + 4, H=2, B=1, T=400, k=1)
     sel = kvx.kvx_select_topk(syn.selection_scores(w), w.k)
     caches, Wg, bg = _run_fit_xh(w, 0.01, sel)
     assert np.all(np.isfinite(Wg)) and np.all(np.isfinite(bg)), "unwritten outputs"
-    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
     assert 2 * w.Lt > n_sm
     last = 2 * w.Lt - 1
     systems = sorted({(s // 2, s % 2) for s in (0, 1, n_sm - 1, n_sm, n_sm + 1, last)})
