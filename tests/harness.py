@@ -46,7 +46,9 @@ def rope_theta(w, side):
 
 
 def make_ctx(w, kernel=kvx.KVX_KERNEL_AUTO, selection=None, W=None, b=None, scores=None,
-             device=0, rope_style=kvx.KVX_ROPE_HALF):
+             device=0, rope_style=None):
+    if rope_style is None:   # the workload's pairing unless the test asks for another
+        rope_style = kvx.KVX_ROPE_INTERLEAVED if w.rope_style == "interleaved" else kvx.KVX_ROPE_HALF
     if W is None:
         W, b = syn.weights(w)
     if selection is None and scores is None:
@@ -81,8 +83,9 @@ def run_contiguous(ctx, w, sk, sv, pos_np, out_dtype=None, tgt=None):
     return tk, tv, status
 
 
-def oracle_full(w, sk, sv, pos_np, sel, W, b, style="half"):
-    """Returns (ref_k, ref_v, slack_k, slack_v)."""
+def oracle_full(w, sk, sv, pos_np, sel, W, b, style=None):
+    """Returns (ref_k, ref_v, slack_k, slack_v); style None = the workload's RoPE pairing."""
+    style = style or w.rope_style
     mode = "exact" if w.cache_dtype == "f32" else "bf16fwd"
     return omap.map_cache(to_f64(sk), to_f64(sv), pos_np, sel, to_f64(W),
                           None if b is None else to_f64(b), rope_theta(w, 0), rope_theta(w, 1), mode=mode,
@@ -128,4 +131,4 @@ def oracle_rows(w, rows, pos_np, sel, W, b, turn=None):
     p = pos_np[rows[:, 0], rows[:, 1]]
     return omap.map_tokens(sk, sv, p, sel, to_f64(W), None if b is None else to_f64(b),
                            rope_theta(w, 0), rope_theta(w, 1), mode=mode, head_mix=w.head_mix,
-                           rounding_slack=STRIP_DELTA)
+                           style=w.rope_style, rounding_slack=STRIP_DELTA)

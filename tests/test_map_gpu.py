@@ -415,6 +415,24 @@ def test_paged_small_full(kname):
         kvx.kvx_destroy(ctx)
 
 
+@pytest.mark.parametrize("head_mix,expect", [("per_head", 2), ("cross_head", 3)])
+def test_paged_interleaved_tensor_cores(head_mix, expect):
+    """Interleaved RoPE pairs into a paged target on the tensor-core kernels (per-head and
+    cross-head): every slot of two turns against the interleaved oracle, untouched slots
+    keep their sentinel."""
+    w = syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4", Ls=5, Lt=3, H=2, B=3, T=150, k=2,
+                     len_range=(3, 70), head_mix=head_mix, rope_style="interleaved")
+    ctx, sel, W, b = make_ctx(w, kernel=kvx.KVX_KERNEL_TCGEN05)
+    try:
+        assert kvx.kvx_get_kernel(ctx, paged=True) == expect
+        L0 = syn.initial_lengths(w)
+        rows = np.array([(bb, t) for bb in range(w.B) for t in range(w.T)], dtype=np.int64)
+        for turn in (0, 1):
+            _check_paged(w, ctx, sel, W, b, turn, L0, rows)
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
 @pytest.mark.parametrize("turn", [0, 7])
 def test_paged_full_size_sampled(turn):
     w = syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4")
