@@ -177,7 +177,11 @@ KVX_API kvx_status kvx_create(const kvx_config* cfg, int device, kvx_ctx** out);
  * (a cudaStream_t; NULL = the legacy default stream).  Host-detected errors return
  * before any launch (INVALID_ARG, UNSUPPORTED); launch failures return CUDA;
  * device-detected errors go to the status word read by kvx_get_status.
- * batch == 0 or tokens_per_seq == 0 is a no-op returning OK. */
+ * batch == 0 or tokens_per_seq == 0 is a no-op returning OK.
+ * kvx_map may be captured into a CUDA graph: it only encodes tensor maps on the host and
+ * launches (the cross-head kernel's workspace is allocated by the first call that needs
+ * it, so make one call of the captured shape before the capture); a replay maps whatever
+ * the captured buffers then hold. */
 KVX_API kvx_status kvx_map(kvx_ctx* ctx, const kvx_src* src, int32_t batch, int32_t tokens_per_seq,
                    const int32_t* positions, const kvx_tgt* tgt, void* stream);
 

@@ -741,6 +741,55 @@ def test_per_head_tc_fp32_weights_hi_lo(over):
         kvx.kvx_destroy(ctx)
 
 
+# ------------------------------------------------------------------ CUDA graphs -----
+
+@pytest.mark.parametrize("kname,name", [("simt", "qwen3_14b_32b_b8x1024_k4"), ("tc", "qwen3_14b_32b_b8x1024_k4"),
+                                        ("tc", "qwen3_14b_32b_t32768_k4_xhead")])
+def test_map_captured_in_a_cuda_graph(kname, name):
+    """kvx_map captured into a CUDA graph (the cross-head kernel after one eager call has
+    allocated its workspace): replays map whatever the captured buffers hold at replay
+    time, bit for bit as eager calls on the same inputs, and the status stays OK."""
+    w = syn.workload(name, Ls=5, Lt=3, H=2, B=2, T=300, k=2)
+    ctx, sel, W, b = make_ctx(w, kernel=KERNELS[kname])
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        pos = torch.from_numpy(syn.positions(w)).to(dev)
+        tk = torch.full((w.Lt, w.B, w.H, w.T, w.d), float("nan"), dtype=torch.bfloat16, device=dev)
+        tv = torch.full_like(tk, float("nan"))
+        src, tgt = kvx.src_from_tensors(sk, sv), kvx.tgt_from_tensors(tk, tv)
+        s = torch.cuda.Stream()
+        with torch.cuda.stream(s):
+            kvx.kvx_map(ctx, src, w.B, w.T, pos.data_ptr(), tgt, s.cuda_stream)   # eager reference
+        s.synchronize()
+        ek, ev = tk.clone(), tv.clone()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            kvx.kvx_map(ctx, src, w.B, w.T, pos.data_ptr(), tgt, s.cuda_stream)
+        for rep in range(2):
+            tk.fill_(float("nan"))
+            tv.fill_(float("nan"))
+            g.replay()
+            torch.cuda.synchronize()
+            assert torch.equal(tk, ek) and torch.equal(tv, ev), "replay %d differs from the eager map" % rep
+        # new inputs written into the captured buffers: the replay maps them
+        sk.copy_(sk.flip(3))
+        sv.copy_(sv.flip(3))
+        pos.copy_(pos + 1000)
+        g.replay()
+        torch.cuda.synchronize()
+        gk, gv = tk.clone(), tv.clone()
+        with torch.cuda.stream(s):
+            kvx.kvx_map(ctx, src, w.B, w.T, pos.data_ptr(), tgt, s.cuda_stream)
+        s.synchronize()
+        assert torch.equal(gk, tk) and torch.equal(gv, tv)
+        assert not torch.equal(gk, ek)
+        assert kvx.kvx_get_status(ctx, s.cuda_stream) == kvx.KVX_OK
+        del g
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
 # ---------------------------------------------------------------- HF RoPE numerics -----
 
 @pytest.mark.parametrize("kname", ["simt", "tc"])
