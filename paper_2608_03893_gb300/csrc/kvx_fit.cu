@@ -144,7 +144,6 @@ __device__ __forceinline__ DF df_from_double(double x) {
   const float hi = static_cast<float>(x);
   return DF{hi, static_cast<float>(x - static_cast<double>(hi))};
 }
-__device__ __forceinline__ double df_to_double(DF a) { return static_cast<double>(a.hi) + static_cast<double>(a.lo); }
 
 // Persistent solve kernels: CTA c handles systems c, c + gridDim.x, ...  Dynamic shared
 // memory holds pairs of floats (8 bytes an element, as fp64 was).
@@ -452,6 +451,33 @@ __device__ __forceinline__ void tri_solves(const DF* A, int F, DF* Z, int ldz, c
   }
 }
 
+// b = mean(Y) - mean(X) W for one 128-column block of solved W (Z, leading dimension ldz),
+// by the CTA in float-float: the F feature means (xmean(r), fp64 from the column sums)
+// staged in shared memory as pairs, thread = (column tid % 128, quarter tid / 128 of the
+// rows), the quarters' sums added in shared memory; ymean = this thread's column's mean of
+// Y.  Writes b[0 .. 128) in fp32.  smem: F + 4 x 128 pairs.  Ends synchronised.
+template <class XMean>
+__device__ __forceinline__ void bias_out(int F, const DF* Z, int ldz, DF* smem, DF ymean, XMean xmean, float* b) {
+  const int tid = threadIdx.x;
+  constexpr int kQuarters = kSolveThreads / kFD;
+  DF* xm = smem;
+  DF* part = smem + F;
+  for (int r = tid; r < F; r += blockDim.x) xm[r] = df_from_double(xmean(r));
+  __syncthreads();
+  const int c = tid % kFD, qtr = tid / kFD;
+  DF acc = df_make(0.f);
+  for (int r = qtr; r < F; r += kQuarters) acc = df_fma_lazy(xm[r], Z[static_cast<size_t>(r) * ldz + c], acc);
+  part[qtr * kFD + c] = df_norm(acc);
+  __syncthreads();
+  if (tid < kFD) {
+    DF v = ymean;
+#pragma unroll
+    for (int q = 0; q < kQuarters; ++q) v = df_add(v, df_neg(part[q * kFD + tid]));
+    b[tid] = __fadd_rn(v.hi, v.lo);
+  }
+  __syncthreads();
+}
+
 // Per-head systems (F = 128 k <= 512): the whole panel stays in shared memory
 // ([32][33] diagonal block + [F - 32][33] panel).
 __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __grid_constant__ FitParams P) {
@@ -562,18 +588,13 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_solve_kernel(const __gri
     }
     // 3. forward and backward solves for the 128 right-hand sides
     tri_solves(A, F, Z, kFD, Inv, fsm);
-    // 4. W (fp32) and b = mean(Y) - mean(X) W (fp64)
+    // 4. W (fp32) and b = mean(Y) - mean(X) W
     float* Wout = P.W + static_cast<size_t>(sys) * F * kFD;
     for (int64_t e = tid; e < static_cast<int64_t>(F) * kFD; e += blockDim.x) Wout[e] = __fadd_rn(Z[e].hi, Z[e].lo);
-    if (tid < kFD) {
-      double acc = P.sums[sums_index(P, 1, kv, l, h) + tid] * inv_n;
-      for (int r = 0; r < F; ++r) {
-        const int layer = __ldg(&P.sel[l * P.k + r / kFD]);
-        acc -= P.sums[sums_index(P, 0, kv, layer, h) + r % kFD] * inv_n * df_to_double(Z[static_cast<size_t>(r) * kFD + tid]);
-      }
-      P.b[static_cast<size_t>(sys) * kFD + tid] = static_cast<float>(acc);
-    }
-    __syncthreads();
+    bias_out(
+        F, Z, kFD, fsm, df_from_double(P.sums[sums_index(P, 1, kv, l, h) + (tid & (kFD - 1))] * inv_n),
+        [&](int r) { return P.sums[sums_index(P, 0, kv, __ldg(&P.sel[l * P.k + r / kFD]), h) + r % kFD] * inv_n; },
+        P.b + static_cast<size_t>(sys) * kFD);
   }
 }
 
@@ -731,24 +752,20 @@ __global__ void __launch_bounds__(kSolveThreads, 1) fit_trisolve_xh_kernel(const
     const DF* Inv = Z + static_cast<size_t>(F) * R;
     DF* Zh = Z + static_cast<size_t>(ht) * kFD;   // this head's 128 columns, leading dimension R
     tri_solves(A, F, Zh, R, Inv, fsm);
-    // W (fp32, [L_t][2][H][F][128]) and b = mean(Y) - mean(X) W (fp64) of target head ht
+    // W (fp32, [L_t][2][H][F][128]) and b = mean(Y) - mean(X) W of target head ht
     float* Wout = P.W + (static_cast<size_t>(sys) * H + ht) * F * kFD;
     for (int64_t e = tid; e < static_cast<int64_t>(F) * kFD; e += blockDim.x) {
       const int r = static_cast<int>(e / kFD), c = static_cast<int>(e % kFD);
       const DF z = Zh[static_cast<size_t>(r) * R + c];
       Wout[e] = __fadd_rn(z.hi, z.lo);
     }
-    if (tid < kFD) {
-      double acc = P.sums[sums_index(P, 1, kv, l, ht) + tid] * inv_n;
-      for (int r = 0; r < F; ++r) {
-        const int uu = r / kFD;
-        const int layer = __ldg(&P.sel[l * P.k + uu / H]);
-        acc -= P.sums[sums_index(P, 0, kv, layer, uu % H) + r % kFD] * inv_n *
-               df_to_double(Zh[static_cast<size_t>(r) * R + tid]);
-      }
-      P.b[(static_cast<size_t>(sys) * H + ht) * kFD + tid] = static_cast<float>(acc);
-    }
-    __syncthreads();
+    bias_out(
+        F, Zh, R, fsm, df_from_double(P.sums[sums_index(P, 1, kv, l, ht) + (tid & (kFD - 1))] * inv_n),
+        [&](int r) {
+          const int uu = r / kFD;
+          return P.sums[sums_index(P, 0, kv, __ldg(&P.sel[l * P.k + uu / H]), uu % H) + r % kFD] * inv_n;
+        },
+        P.b + (static_cast<size_t>(sys) * H + ht) * kFD);
   }
 }
 
