@@ -276,7 +276,7 @@ KVX_API int64_t kvx_mapper_params(int32_t tgt_layers, int32_t n_kv_heads, int32_
  * on the tensor cores from a bf16 hi + lo split of each value (within 2^-17 of it) and
  * accumulate in fp32; the factorisation and the solves run in float-float arithmetic (each
  * value an unevaluated sum of two fp32 numbers, about 48 significant bits) on the FP32
- * units, and the bias in fp64.  Runs on `stream` and
+ * units, the bias too.  Runs on `stream` and
  * synchronises it before returning (an offline step).  Stream-ordered workspace: the
  * blocks (at most L_t*2*H*(k*(k+1)/2 + k)*64 KB), 8 MB per SM, and the packed operands
  * (4 bytes per token, channel, K|V, head and used layer of either model), at most half the
