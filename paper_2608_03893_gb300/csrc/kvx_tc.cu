@@ -50,7 +50,11 @@
 //   warps 4-11  epilogue, two warpgroups (one warp per TMEM lane quarter, warp % 4).
 //               Thread (group g, row r) owns token row r (= TMEM lane r) and the 32 RoPE
 //               pairs 32g .. 32g+31 (channels i and i + 64): TMEM -> registers, + bias,
-//               (keys) target RoPE, bf16.  For a contiguous target each warp stages its
+//               (keys) target RoPE, bf16.  A key layer loads its accumulator in two
+//               halves and releases it after the second load, so the cos / sin of its
+//               32 pairs and one half fit the registers; a value layer (no cos / sin) loads
+//               both halves at once and releases the accumulator before any arithmetic.
+//               For a contiguous target each warp stages its
 //               32 rows x 2 x 32 channels (64-byte swizzle) and writes them with its own
 //               TMA stores; a warp with a row at an out-of-range position writes its valid
 //               rows directly.  Paged targets take 16-byte stores through the block table.
@@ -71,6 +75,7 @@
 #include <climits>
 #include <cstring>
 #include <mutex>
+#include <type_traits>
 #include <vector>
 
 #include "kvx_internal.h"
@@ -609,161 +614,178 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       }
       __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(un.kv ? A.tgt_v : A.tgt_k);
       const CUtensorMap* tm_out = un.kv ? &P.tm_out_v : &P.tm_out_k;
-      for (int l = 0; ok && l < Lt; ++l, ++lay) {
-        const uint32_t bslot = lay % kBiasSlots;
-        const float* bias = bias_ring + bslot * kD;
-        {
-          const bool w_ok = wait_bar(smem_u32(&bias_full[bslot]), (lay / kBiasSlots) & 1u, abort_flag, P.status,
-                                     KVX_ERR_TIMEOUT, P.timeout_ns);
-          if (!__all_sync(0xffffffffu, w_ok)) {
-            ok = false;
-            break;
+      // values need no cos / sin, so their layer loop (its own instance) holds both halves
+      // of the accumulator at once and releases it before the arithmetic
+      auto layers = [&](auto kv_tag) {
+        constexpr bool kV = decltype(kv_tag)::value;
+        for (int l = 0; ok && l < Lt; ++l, ++lay) {
+          const uint32_t bslot = lay % kBiasSlots;
+          const float* bias = bias_ring + bslot * kD;
+          {
+            const bool w_ok = wait_bar(smem_u32(&bias_full[bslot]), (lay / kBiasSlots) & 1u, abort_flag, P.status,
+                                       KVX_ERR_TIMEOUT, P.timeout_ns);
+            if (!__all_sync(0xffffffffu, w_ok)) {
+              ok = false;
+              break;
+            }
           }
-        }
-        const uint32_t buf = static_cast<uint32_t>(l) & 1u;   // accumulator of issuer l % 2
-        {
-          const uint32_t acc_par = (buf ? acc_n1 : acc_n0) & 1u;
-          if (buf) ++acc_n1; else ++acc_n0;
-          const bool w_ok = wait_bar(smem_u32(&accf[buf]), acc_par, abort_flag, P.status, KVX_ERR_TIMEOUT,
-                                     P.timeout_ns);
-          if (!__all_sync(0xffffffffu, w_ok)) {
-            ok = false;
-            break;
+          const uint32_t buf = static_cast<uint32_t>(l) & 1u;   // accumulator of issuer l % 2
+          {
+            const uint32_t acc_par = (buf ? acc_n1 : acc_n0) & 1u;
+            if (buf) ++acc_n1; else ++acc_n0;
+            const bool w_ok = wait_bar(smem_u32(&accf[buf]), acc_par, abort_flag, P.status, KVX_ERR_TIMEOUT,
+                                       P.timeout_ns);
+            if (!__all_sync(0xffffffffu, w_ok)) {
+              ok = false;
+              break;
+            }
           }
-        }
-        tc_fence_after();
-        // this warp's staging buffer for the layer; the store that last read it (this
-        // thread's bulk group kStageBufs layers ago) must be done reading
-        uint8_t* sb = wstage + (lay % kStageBufs) * kWarpStageBytes;
-        if (!A.paged && lay >= static_cast<uint32_t>(kStageBufs)) {
-          if (lane == 0) {
-            if constexpr (kStageBufs == 1) bulk_wait_read_all(); else bulk_wait_read_but_last();
+          tc_fence_after();
+          // this warp's staging buffer for the layer; the store that last read it (this
+          // thread's bulk group kStageBufs layers ago) must be done reading
+          uint8_t* sb = wstage + (lay % kStageBufs) * kWarpStageBytes;
+          if (!A.paged && lay >= static_cast<uint32_t>(kStageBufs)) {
+            if (lane == 0) {
+              if constexpr (kStageBufs == 1) bulk_wait_read_all(); else bulk_wait_read_but_last();
+            }
+            __syncwarp();
           }
-          __syncwarp();
-        }
-        const uint32_t col = tmem_base + lane_addr + buf * kAccCols + 32 * g;
-#pragma unroll
-        for (int rnd = 0; rnd < 2; ++rnd) {
-          uint32_t lo[16], hi[16];
-          tmem_ld_2x16(col + 16 * rnd, col + 64 + 16 * rnd, lo, hi);
-          if (rnd == 1) {  // the accumulator is free for the issuer's next layer
+          const uint32_t col = tmem_base + lane_addr + buf * kAccCols + 32 * g;
+          auto release = [&] {   // the accumulator is free for the issuer's next layer
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&acce[buf]), 0));
+          };
+          uint32_t lo2[kV ? 2 : 1][16], hi2[kV ? 2 : 1][16];
+          if constexpr (kV) {
+            tmem_ld_2x16(col, col + 64, lo2[0], hi2[0]);
+            tmem_ld_2x16(col + 16, col + 80, lo2[kV ? 1 : 0], hi2[kV ? 1 : 0]);
+            release();
           }
-          const int c_lo = 32 * g + 16 * rnd;   // channels c_lo + [0,16) and 64 + c_lo + [0,16)
-          float ylo[16], yhi[16];
 #pragma unroll
-          for (int j = 0; j < 16; j += 4) {
-            const float4 b0 = *reinterpret_cast<const float4*>(bias + c_lo + j);
-            const float4 b1 = *reinterpret_cast<const float4*>(bias + 64 + c_lo + j);
-            ylo[j] = __fadd_rn(__uint_as_float(lo[j]), b0.x);
-            ylo[j + 1] = __fadd_rn(__uint_as_float(lo[j + 1]), b0.y);
-            ylo[j + 2] = __fadd_rn(__uint_as_float(lo[j + 2]), b0.z);
-            ylo[j + 3] = __fadd_rn(__uint_as_float(lo[j + 3]), b0.w);
-            yhi[j] = __fadd_rn(__uint_as_float(hi[j]), b1.x);
-            yhi[j + 1] = __fadd_rn(__uint_as_float(hi[j + 1]), b1.y);
-            yhi[j + 2] = __fadd_rn(__uint_as_float(hi[j + 2]), b1.z);
-            yhi[j + 3] = __fadd_rn(__uint_as_float(hi[j + 3]), b1.w);
-          }
-          if (un.kv == 0 && !kIL) {
-            // target RoPE on pairs (c, c + 64): channel c_lo + j of ylo with the same of yhi
-#pragma unroll
-            for (int j = 0; j < 16; j += 2) {
-              const float2 c = make_float2(cs[16 * rnd + j], cs[16 * rnd + j + 1]);
-              const float2 sv = make_float2(sn[16 * rnd + j], sn[16 * rnd + j + 1]);
-              float2 r0, r1;
-              rope_apply2<kHF>(make_float2(ylo[j], ylo[j + 1]), make_float2(yhi[j], yhi[j + 1]), c, sv, r0, r1);
-              ylo[j] = r0.x;
-              ylo[j + 1] = r0.y;
-              yhi[j] = r1.x;
-              yhi[j + 1] = r1.y;
+          for (int rnd = 0; rnd < 2; ++rnd) {
+            uint32_t(&lo)[16] = lo2[kV ? rnd : 0];
+            uint32_t(&hi)[16] = hi2[kV ? rnd : 0];
+            if constexpr (!kV) {
+              tmem_ld_2x16(col + 16 * rnd, col + 64 + 16 * rnd, lo, hi);
+              if (rnd == 1) release();
             }
-          } else if (un.kv == 0) {
-            // target RoPE on pairs (c, c + 1): channels c_lo + j, c_lo + j + 1 of ylo (slot
-            // 8 rnd + j / 2) and of yhi (slot 16 + 8 rnd + j / 2), two pairs per step
+            const int c_lo = 32 * g + 16 * rnd;   // channels c_lo + [0,16) and 64 + c_lo + [0,16)
+            float ylo[16], yhi[16];
 #pragma unroll
             for (int j = 0; j < 16; j += 4) {
+              const float4 b0 = *reinterpret_cast<const float4*>(bias + c_lo + j);
+              const float4 b1 = *reinterpret_cast<const float4*>(bias + 64 + c_lo + j);
+              ylo[j] = __fadd_rn(__uint_as_float(lo[j]), b0.x);
+              ylo[j + 1] = __fadd_rn(__uint_as_float(lo[j + 1]), b0.y);
+              ylo[j + 2] = __fadd_rn(__uint_as_float(lo[j + 2]), b0.z);
+              ylo[j + 3] = __fadd_rn(__uint_as_float(lo[j + 3]), b0.w);
+              yhi[j] = __fadd_rn(__uint_as_float(hi[j]), b1.x);
+              yhi[j + 1] = __fadd_rn(__uint_as_float(hi[j + 1]), b1.y);
+              yhi[j + 2] = __fadd_rn(__uint_as_float(hi[j + 2]), b1.z);
+              yhi[j + 3] = __fadd_rn(__uint_as_float(hi[j + 3]), b1.w);
+            }
+            if (!kV && !kIL) {
+              // target RoPE on pairs (c, c + 64): channel c_lo + j of ylo with the same of yhi
 #pragma unroll
-              for (int hv = 0; hv < 2; ++hv) {
-                float* y = hv ? yhi : ylo;
-                const int m = 16 * hv + 8 * rnd + j / 2;
+              for (int j = 0; j < 16; j += 2) {
+                const float2 c = make_float2(cs[16 * rnd + j], cs[16 * rnd + j + 1]);
+                const float2 sv = make_float2(sn[16 * rnd + j], sn[16 * rnd + j + 1]);
                 float2 r0, r1;
-                rope_apply2<kHF>(make_float2(y[j], y[j + 2]), make_float2(y[j + 1], y[j + 3]),
-                                 make_float2(cs[m], cs[m + 1]), make_float2(sn[m], sn[m + 1]), r0, r1);
-                y[j] = r0.x;
-                y[j + 2] = r0.y;
-                y[j + 1] = r1.x;
-                y[j + 3] = r1.y;
+                rope_apply2<kHF>(make_float2(ylo[j], ylo[j + 1]), make_float2(yhi[j], yhi[j + 1]), c, sv, r0, r1);
+                ylo[j] = r0.x;
+                ylo[j + 1] = r0.y;
+                yhi[j] = r1.x;
+                yhi[j + 1] = r1.y;
+              }
+            } else if (!kV) {
+              // target RoPE on pairs (c, c + 1): channels c_lo + j, c_lo + j + 1 of ylo (slot
+              // 8 rnd + j / 2) and of yhi (slot 16 + 8 rnd + j / 2), two pairs per step
+#pragma unroll
+              for (int j = 0; j < 16; j += 4) {
+#pragma unroll
+                for (int hv = 0; hv < 2; ++hv) {
+                  float* y = hv ? yhi : ylo;
+                  const int m = 16 * hv + 8 * rnd + j / 2;
+                  float2 r0, r1;
+                  rope_apply2<kHF>(make_float2(y[j], y[j + 2]), make_float2(y[j + 1], y[j + 3]),
+                                   make_float2(cs[m], cs[m + 1]), make_float2(sn[m], sn[m + 1]), r0, r1);
+                  y[j] = r0.x;
+                  y[j + 2] = r0.y;
+                  y[j + 1] = r1.x;
+                  y[j + 3] = r1.y;
+                }
               }
             }
+            uint4 v[4];
+            v[0] = make_uint4(pack_bf16x2(ylo[0], ylo[1]), pack_bf16x2(ylo[2], ylo[3]), pack_bf16x2(ylo[4], ylo[5]),
+                              pack_bf16x2(ylo[6], ylo[7]));
+            v[1] = make_uint4(pack_bf16x2(ylo[8], ylo[9]), pack_bf16x2(ylo[10], ylo[11]),
+                              pack_bf16x2(ylo[12], ylo[13]), pack_bf16x2(ylo[14], ylo[15]));
+            v[2] = make_uint4(pack_bf16x2(yhi[0], yhi[1]), pack_bf16x2(yhi[2], yhi[3]), pack_bf16x2(yhi[4], yhi[5]),
+                              pack_bf16x2(yhi[6], yhi[7]));
+            v[3] = make_uint4(pack_bf16x2(yhi[8], yhi[9]), pack_bf16x2(yhi[10], yhi[11]),
+                              pack_bf16x2(yhi[12], yhi[13]), pack_bf16x2(yhi[14], yhi[15]));
+            if (warp_tma || A.paged) {
+              // two 32-row x 64-byte pieces (channels 32g.. and 64+32g..), 64-byte swizzle:
+              // 16-byte chunk index XOR (row / 2) % 4
+              const int sw = (lane >> 1) & 3;
+              uint8_t* prow = sb + lane * 64;
+              *reinterpret_cast<uint4*>(prow + (((2 * rnd) ^ sw) << 4)) = v[0];
+              *reinterpret_cast<uint4*>(prow + (((2 * rnd + 1) ^ sw) << 4)) = v[1];
+              *reinterpret_cast<uint4*>(prow + kPieceBytes + (((2 * rnd) ^ sw) << 4)) = v[2];
+              *reinterpret_cast<uint4*>(prow + kPieceBytes + (((2 * rnd + 1) ^ sw) << 4)) = v[3];
+            } else if (valid) {
+              __nv_bfloat16* out = dst + static_cast<int64_t>(l) * A.ts[0] + row_off;
+              st_global_hint(out + c_lo, v[0], st_pol);
+              st_global_hint(out + c_lo + 8, v[1], st_pol);
+              st_global_hint(out + 64 + c_lo, v[2], st_pol);
+              st_global_hint(out + 64 + c_lo + 8, v[3], st_pol);
+            }
           }
-          uint4 v[4];
-          v[0] = make_uint4(pack_bf16x2(ylo[0], ylo[1]), pack_bf16x2(ylo[2], ylo[3]), pack_bf16x2(ylo[4], ylo[5]),
-                            pack_bf16x2(ylo[6], ylo[7]));
-          v[1] = make_uint4(pack_bf16x2(ylo[8], ylo[9]), pack_bf16x2(ylo[10], ylo[11]),
-                            pack_bf16x2(ylo[12], ylo[13]), pack_bf16x2(ylo[14], ylo[15]));
-          v[2] = make_uint4(pack_bf16x2(yhi[0], yhi[1]), pack_bf16x2(yhi[2], yhi[3]), pack_bf16x2(yhi[4], yhi[5]),
-                            pack_bf16x2(yhi[6], yhi[7]));
-          v[3] = make_uint4(pack_bf16x2(yhi[8], yhi[9]), pack_bf16x2(yhi[10], yhi[11]),
-                            pack_bf16x2(yhi[12], yhi[13]), pack_bf16x2(yhi[14], yhi[15]));
-          if (warp_tma || A.paged) {
-            // two 32-row x 64-byte pieces (channels 32g.. and 64+32g..), 64-byte swizzle:
-            // 16-byte chunk index XOR (row / 2) % 4
-            const int sw = (lane >> 1) & 3;
-            uint8_t* prow = sb + lane * 64;
-            *reinterpret_cast<uint4*>(prow + (((2 * rnd) ^ sw) << 4)) = v[0];
-            *reinterpret_cast<uint4*>(prow + (((2 * rnd + 1) ^ sw) << 4)) = v[1];
-            *reinterpret_cast<uint4*>(prow + kPieceBytes + (((2 * rnd) ^ sw) << 4)) = v[2];
-            *reinterpret_cast<uint4*>(prow + kPieceBytes + (((2 * rnd + 1) ^ sw) << 4)) = v[3];
-          } else if (valid) {
-            __nv_bfloat16* out = dst + static_cast<int64_t>(l) * A.ts[0] + row_off;
-            st_global_hint(out + c_lo, v[0], st_pol);
-            st_global_hint(out + c_lo + 8, v[1], st_pol);
-            st_global_hint(out + 64 + c_lo, v[2], st_pol);
-            st_global_hint(out + 64 + c_lo + 8, v[3], st_pol);
-          }
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(&bias_empty[bslot]));
-        if (A.paged) {
-          // Paged rows leave the staging buffer in 64-byte pieces: in store i lanes 8m ..
-          // 8m + 7 write row 4i + m, lanes 4 apart the two pieces (channels 32g.. and
-          // 64 + 32g..), so each group of four lanes writes one whole 64-byte piece.  The
-          // row's block offset comes from the lane that owns the row.
-          const int64_t lay_off = static_cast<int64_t>(l) * A.ts[0];
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&bias_empty[bslot]));
+          if (A.paged) {
+            // Paged rows leave the staging buffer in 64-byte pieces: in store i lanes 8m ..
+            // 8m + 7 write row 4i + m, lanes 4 apart the two pieces (channels 32g.. and
+            // 64 + 32g..), so each group of four lanes writes one whole 64-byte piece.  The
+            // row's block offset comes from the lane that owns the row.
+            const int64_t lay_off = static_cast<int64_t>(l) * A.ts[0];
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const int rr = 4 * i + (lane >> 3);
-            const int piece = (lane >> 2) & 1, chunk = lane & 3;
-            const uint32_t off_lo = __shfl_sync(0xffffffffu, static_cast<uint32_t>(row_off), rr);
-            const uint32_t off_hi = __shfl_sync(0xffffffffu, static_cast<uint32_t>(static_cast<uint64_t>(row_off) >> 32), rr);
-            const int ok_row = __shfl_sync(0xffffffffu, valid ? 1 : 0, rr);
-            const int sw = (rr >> 1) & 3;
-            const uint4 v = *reinterpret_cast<const uint4*>(sb + rr * 64 + piece * kPieceBytes + ((chunk ^ sw) << 4));
-            if (ok_row) {
-              const int64_t roff = static_cast<int64_t>((static_cast<uint64_t>(off_hi) << 32) | off_lo);
-              st_global_hint(dst + lay_off + roff + 64 * piece + 32 * g + 8 * chunk, v, st_pol);
+            for (int i = 0; i < 8; ++i) {
+              const int rr = 4 * i + (lane >> 3);
+              const int piece = (lane >> 2) & 1, chunk = lane & 3;
+              const uint32_t off_lo = __shfl_sync(0xffffffffu, static_cast<uint32_t>(row_off), rr);
+              const uint32_t off_hi = __shfl_sync(0xffffffffu, static_cast<uint32_t>(static_cast<uint64_t>(row_off) >> 32), rr);
+              const int ok_row = __shfl_sync(0xffffffffu, valid ? 1 : 0, rr);
+              const int sw = (rr >> 1) & 3;
+              const uint4 v = *reinterpret_cast<const uint4*>(sb + rr * 64 + piece * kPieceBytes + ((chunk ^ sw) << 4));
+              if (ok_row) {
+                const int64_t roff = static_cast<int64_t>((static_cast<uint64_t>(off_hi) << 32) | off_lo);
+                st_global_hint(dst + lay_off + roff + 64 * piece + 32 * g + 8 * chunk, v, st_pol);
+              }
             }
-          }
-          __syncwarp();   // the staging buffer is read before the next layer writes it
-        } else {
-          // every contiguous-target layer commits one bulk group per warp (empty when the
-          // warp wrote its rows directly), so the group count above identifies the buffer
-          if (warp_tma) {
-            fence_proxy_async_smem();
-            __syncwarp();
-          }
-          if (lane == 0) {
-            if (warp_tma && un.t0 + 32 * q < A.T) {   // skip a box wholly past the sequence end
-              // one box: both 32-row x 32-channel pieces (channels 32g.. and 64 + 32g..)
-              const int bh = P.out_bh == 2 ? un.b * H + un.h : un.h;
-              tma_store_5d(tm_out, smem_u32(sb), 32 * g, un.t0 + 32 * q, 0, bh, l);
+            __syncwarp();   // the staging buffer is read before the next layer writes it
+          } else {
+            // every contiguous-target layer commits one bulk group per warp (empty when the
+            // warp wrote its rows directly), so the group count above identifies the buffer
+            if (warp_tma) {
+              fence_proxy_async_smem();
+              __syncwarp();
             }
-            bulk_commit_group();
+            if (lane == 0) {
+              if (warp_tma && un.t0 + 32 * q < A.T) {   // skip a box wholly past the sequence end
+                // one box: both 32-row x 32-channel pieces (channels 32g.. and 64 + 32g..)
+                const int bh = P.out_bh == 2 ? un.b * H + un.h : un.h;
+                tma_store_5d(tm_out, smem_u32(sb), 32 * g, un.t0 + 32 * q, 0, bh, l);
+              }
+              bulk_commit_group();
+            }
           }
         }
-      }
+      };
+      if (un.kv) layers(std::true_type{});
+      else layers(std::false_type{});
     }
     if (!A.paged && lane == 0) bulk_wait_all();   // this warp's stores are complete
   } else {
