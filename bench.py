@@ -22,6 +22,7 @@ Multi-GPU (torchrun): every rank maps its own replica (weak scaling, no collecti
 the data path; a MAX all-reduce of the elapsed time only).
 """
 import argparse
+import dataclasses
 import hashlib
 import re
 import json
@@ -260,6 +261,28 @@ def oracle_sample_rate(w, budget_s, seed=0, ctx_sel=None):
         n = min(w.n_tokens, int(n * min(8.0, max(2.0, 0.5 * budget_s / max(dt, 1e-3)))))
         dt = run(n)
     return n / dt, n, dt, blas_threads()
+
+
+def oracle_one_core(w, budget_s=6.0):
+    """The oracle's rate with one BLAS thread: a fresh interpreter (exec, no CUDA) with the
+    BLAS thread counts set to 1 runs oracle_sample_rate on the same workload.  Returns
+    {"value", "sample"} or None if the child fails."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               CUDA_VISIBLE_DEVICES="")
+    fields = json.dumps({k: (list(v) if isinstance(v, tuple) else v) for k, v in dataclasses.asdict(w).items()})
+    code = ("import json, sys; sys.path.insert(0, %r); import bench; "
+            "from paper_2608_03893_gb300 import synthetic as syn; "
+            "d = json.loads(sys.argv[1]); "
+            "d = {k: (tuple(v) if isinstance(v, list) else v) for k, v in d.items()}; "
+            "r = bench.oracle_sample_rate(syn.Workload(**d), budget_s=%f, seed=1); "
+            "print(json.dumps(r))" % (ROOT, budget_s))
+    try:
+        out = subprocess.run([sys.executable, "-c", code, fields], env=env, capture_output=True, text=True,
+                             timeout=120 + 10 * budget_s)
+        rate, n, dt, threads = json.loads(out.stdout.strip().splitlines()[-1])
+    except Exception:
+        return None
+    return {"value": rate, "threads": threads, "sample": "%d tokens, %.1f s" % (n, dt)}
 
 
 def blas_threads():
@@ -874,6 +897,7 @@ def main():
         cpu = {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
                "sample": "%d random tokens of the workload (all %d layers x %d heads x K,V), "
                          "float64 numpy oracle, %.1f s" % (n, w.Lt, w.H, dt)}
+        cpu["one_core"] = oracle_one_core(w)
     clocks = clk.summary()
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
