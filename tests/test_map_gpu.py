@@ -984,6 +984,32 @@ def test_paged_persistent_pool_eight_turns_full_size_sampled():
                       check_sentinel_turns=(0, w.turns - 1))
 
 
+# ------------------------------------------------- tensor cores at large positions -----
+
+@pytest.mark.parametrize("name,style", [("qwen3_14b_32b_b8x1024_k4", "half"), ("qwen3_14b_32b_b8x1024_k4", "interleaved"),
+                                        ("qwen3_14b_32b_t32768_k4_xhead", "half")])
+def test_tensor_cores_up_to_max_position(name, style):
+    """The tensor-core kernels at positions spread over [0, 2^24) including 2^24 - 1 (the
+    largest accepted) and powers of two with their neighbours: every output element within
+    the bf16 bound of the oracle (with the strip's rounding slack), values and keys."""
+    w = syn.workload(name, Ls=5, Lt=3, H=2, B=2, T=300, k=2, theta_t=5e5, rope_style=style)
+    rng = np.random.default_rng(7)
+    special = [0, 1, (1 << 24) - 1, (1 << 24) - 2] + [(1 << e) + o for e in range(10, 24) for o in (-1, 0, 1)]
+    flat = np.array(special + list(rng.integers(0, 1 << 24, size=w.B * w.T - len(special))), dtype=np.int32)
+    pos = flat.reshape(w.B, w.T)
+    ctx, sel, W, b = make_ctx(w, kernel=kvx.KVX_KERNEL_TCGEN05)
+    try:
+        dev = torch.device("cuda:0")
+        sk, sv = syn.source_cache(w, 0, device=dev), syn.source_cache(w, 1, device=dev)
+        tk, tv, st = run_contiguous(ctx, w, sk, sv, pos)
+        assert st == kvx.KVX_OK
+        rk, rv, ak, av = oracle_full(w, sk, sv, pos, sel, W, b)
+        ok, ratio, rms, nbad = check(w, [to_f64(tk), to_f64(tv)], [rk, rv], [ak, av])
+        assert ok, "%d elements out of tolerance (worst %.3g x bound)" % (nbad, ratio)
+    finally:
+        kvx.kvx_destroy(ctx)
+
+
 # ------------------------------------------------------------ strip error bound -----
 
 def test_strip_error_within_delta_up_to_max_position():
