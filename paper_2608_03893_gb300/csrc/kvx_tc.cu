@@ -50,10 +50,11 @@
 //   warps 4-11  epilogue, two warpgroups (one warp per TMEM lane quarter, warp % 4).
 //               Thread (group g, row r) owns token row r (= TMEM lane r) and the 32 RoPE
 //               pairs 32g .. 32g+31 (channels i and i + 64): TMEM -> registers, + bias,
-//               (keys) target RoPE, bf16.  A key layer loads its accumulator in two
-//               halves and releases it after the second load, so the cos / sin of its
-//               32 pairs and one half fit the registers; a value layer (no cos / sin) loads
-//               both halves at once and releases the accumulator before any arithmetic.
+//               (keys) target RoPE, bf16.  Every layer loads both halves of its
+//               accumulator at once and releases it before any arithmetic; the register
+//               split (32 / 160 / 160) gives the epilogue room for the 64 accumulator words
+//               beside a key unit's cos / sin of 32 pairs.  Key and value units run
+//               separate instances of the layer loop (values carry no cos / sin).
 //               For a contiguous target each warp stages its
 //               32 rows x 2 x 32 channels (64-byte swizzle) and writes them with its own
 //               TMA stores; a warp with a row at an out-of-range position writes its valid
@@ -94,9 +95,10 @@ constexpr int kEpiWarps = 8;
 constexpr int kFirstProWarp = 12;                   // warps 12-15: prologue
 constexpr int kProWarps = 4;
 // Registers per thread of each warpgroup (setmaxnreg): the control warps give up most of
-// theirs so that the epilogue keeps its cos/sin of 32 pairs and the prologue its cos/sin
-// of all 64 pairs in registers.  The shares add up to the launch's 128 x 512.
-constexpr uint32_t kRegsCtl = 48, kRegsEpi = 144, kRegsPro = 176;
+// theirs so that the epilogue keeps its cos/sin of 32 pairs beside a whole accumulator row
+// (64 words) and the prologue its cos/sin of all 64 pairs in registers.  The shares add up
+// to the launch's 128 x 512.
+constexpr uint32_t kRegsCtl = 32, kRegsEpi = 160, kRegsPro = 160;
 static_assert(kRegsCtl * 128 + kRegsEpi * 256 + kRegsPro * 128 <= 128u * kThreads,
               "register split exceeds the launch's register file share");
 constexpr int kTileM = 128;                         // tokens per work unit
@@ -614,8 +616,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       }
       __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(un.kv ? A.tgt_v : A.tgt_k);
       const CUtensorMap* tm_out = un.kv ? &P.tm_out_v : &P.tm_out_k;
-      // values need no cos / sin, so their layer loop (its own instance) holds both halves
-      // of the accumulator at once and releases it before the arithmetic
+      // key and value units run separate instances of the layer loop (values carry no
+      // cos / sin); each layer loads both halves of its accumulator at once and releases it
+      // to the issuer before the arithmetic
       auto layers = [&](auto kv_tag) {
         constexpr bool kV = decltype(kv_tag)::value;
         for (int l = 0; ok && l < Lt; ++l, ++lay) {
@@ -656,20 +659,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&acce[buf]), 0));
           };
-          uint32_t lo2[kV ? 2 : 1][16], hi2[kV ? 2 : 1][16];
-          if constexpr (kV) {
-            tmem_ld_2x16(col, col + 64, lo2[0], hi2[0]);
-            tmem_ld_2x16(col + 16, col + 80, lo2[kV ? 1 : 0], hi2[kV ? 1 : 0]);
-            release();
-          }
+          uint32_t lo2[2][16], hi2[2][16];
+          tmem_ld_2x16(col, col + 64, lo2[0], hi2[0]);
+          tmem_ld_2x16(col + 16, col + 80, lo2[1], hi2[1]);
+          release();
 #pragma unroll
           for (int rnd = 0; rnd < 2; ++rnd) {
-            uint32_t(&lo)[16] = lo2[kV ? rnd : 0];
-            uint32_t(&hi)[16] = hi2[kV ? rnd : 0];
-            if constexpr (!kV) {
-              tmem_ld_2x16(col + 16 * rnd, col + 64 + 16 * rnd, lo, hi);
-              if (rnd == 1) release();
-            }
+            uint32_t(&lo)[16] = lo2[rnd];
+            uint32_t(&hi)[16] = hi2[rnd];
             const int c_lo = 32 * g + 16 * rnd;   // channels c_lo + [0,16) and 64 + c_lo + [0,16)
             float ylo[16], yhi[16];
 #pragma unroll
