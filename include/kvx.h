@@ -215,6 +215,29 @@ KVX_API kvx_status kvx_destroy(kvx_ctx* ctx);
 KVX_API kvx_status kvx_select_topk(const double* scores, int32_t tgt_layers, int32_t src_layers,
                            int32_t k, int32_t* out);
 
+/* The per-head tensor-core kernel's source-tile load schedule for a selection table, as
+ * kvx_create builds it (host only; no device needed).  The gather of Sec. 3.2 reads
+ * source layers selection[l][0..k-1] for every target layer l; the kernel keeps up to
+ * four source tiles of a token tile in tensor memory and loads each tile when a use
+ * needs it, evicting the resident tile whose next use is farthest away (Belady), so a
+ * layer shared by consecutive target layers is read from HBM once per token tile.
+ *   selection   host int32 [L_t][k] (row l: distinct layers in [0, L_s)), caller-owned
+ *   n_loads     out: source-tile loads per token tile (≤ L_t·k)
+ *   load_layer  out int32 [L_t·k]: the source layer of load e (first *n_loads valid)
+ *   load_word   out int32 [L_t·k]: bits 0-1 the slot of load e; bit 2 + i set if issuer i
+ *               (issuer of the target layers l with l % 2 == i) must release the slot's
+ *               previous tile before load e (for the slot's first load of a token tile:
+ *               the last tile of the previous token tile); bit 4 + i set if issuer i uses
+ *               the loaded tile
+ *   use_word    out int32 [L_t·k]: for use (l, j) at l·k + j, bits 0-1 the slot it reads;
+ *               bit 2 set on the issuer's first use of the tile (it waits for the load);
+ *               bit 4 set on its last use (it releases the slot after the use)
+ * INVALID_ARG for a NULL pointer, sizes below 1, k > L_s, an entry out of range or a
+ * repeated layer in a row; UNSUPPORTED for k > 4.  No state is kept. */
+KVX_API kvx_status kvx_tc_load_schedule(const int32_t* selection, int32_t src_layers, int32_t tgt_layers,
+                                        int32_t k, int32_t* n_loads, int32_t* load_layer, int32_t* load_word,
+                                        int32_t* use_word);
+
 /* Copy the context's selection table to host out[L_t][k]. */
 KVX_API kvx_status kvx_get_selection(const kvx_ctx* ctx, int32_t* out);
 

@@ -938,11 +938,11 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
 //               4 release the slot after the use
 //   load_slot:  slot | 4 << i if issuer i must release the slot's previous tile first
 //               | 16 << i if issuer i uses the tile (the prologue signals its tready)
-void build_plan(const kvx_ctx* c, TcPlan* plan) {
-  const int Lt = c->Lt, k = c->k, n_uses = Lt * k, S = kTSlots;
+void build_plan(const int32_t* sel, int Ls, int Lt, int k, TcPlan* plan) {
+  const int n_uses = Lt * k, S = kTSlots;
   std::vector<int> src(n_uses), next_use(n_uses);
-  for (int u = 0; u < n_uses; ++u) src[u] = c->sel[u];
-  std::vector<int> seen(c->Ls, INT_MAX);
+  for (int u = 0; u < n_uses; ++u) src[u] = sel[u];
+  std::vector<int> seen(Ls, INT_MAX);
   for (int u = n_uses - 1; u >= 0; --u) {
     next_use[u] = seen[src[u]];
     seen[src[u]] = u;
@@ -1010,6 +1010,12 @@ void build_plan(const kvx_ctx* c, TcPlan* plan) {
   plan->n_loads = static_cast<int>(plan->load_layer.size());
 }
 
+// The issuers' 5-bit word of use u: slot | 4 first use of the tile by its issuer | 16
+// release the slot after the use.
+uint32_t use_bits(const TcPlan& p, int u) {
+  return static_cast<uint32_t>(p.use_slot[u]) | ((p.use_flags[u] & 1) ? 4u : 0u) | ((p.use_flags[u] & 4) ? 16u : 0u);
+}
+
 }  // namespace
 
 void* tensor_map_encoder() { return reinterpret_cast<void*>(get_encode()); }
@@ -1052,7 +1058,7 @@ kvx_status tc_prepare(kvx_ctx* c, const void* W_host) {
   kvx_status st = c->weight_dtype == KVX_F32 ? repack_wt_hilo(c, W_host, c->F) : repack_wt(c, W_host, c->F);
   if (st != KVX_OK) return st;
   cudaError_t e;
-  build_plan(c, &c->plan);
+  build_plan(c->sel.data(), c->Ls, c->Lt, c->k, &c->plan);
   c->plan.n_wst = kNW;   // two rings of kRing stages
   c->plan.n_land = kLand;
   const TcPlan& p = c->plan;
@@ -1062,9 +1068,7 @@ kvx_status tc_prepare(kvx_ctx* c, const void* W_host) {
   for (int l = 0; l < c->Lt; ++l)
     for (int j = 0; j < c->k; ++j) {
       const int u = l * c->k + j;
-      const uint32_t f = static_cast<uint32_t>(p.use_slot[u]) | ((p.use_flags[u] & 1) ? 4u : 0u) |
-                         ((p.use_flags[u] & 4) ? 16u : 0u);
-      pack[l] |= static_cast<int32_t>(f << (5 * j));
+      pack[l] |= static_cast<int32_t>(use_bits(p, u) << (5 * j));
     }
   std::vector<int32_t> tab;
   tab.insert(tab.end(), p.load_layer.begin(), p.load_layer.end());
@@ -1204,3 +1208,41 @@ kvx_status launch_tc(const kvx_ctx* c, const MapArgs& a, cudaStream_t stream) {
 }
 
 }  // namespace kvx
+
+extern "C" {
+
+KVX_API kvx_status kvx_tc_load_schedule(const int32_t* selection, int32_t src_layers, int32_t tgt_layers, int32_t k,
+                                        int32_t* n_loads, int32_t* load_layer, int32_t* load_word,
+                                        int32_t* use_word) {
+  kvx::set_error("");
+  auto fail = [](kvx_status s, const char* m) {
+    kvx::set_error(m);
+    return s;
+  };
+  if (!selection || !n_loads || !load_layer || !load_word || !use_word)
+    return fail(KVX_ERR_INVALID_ARG, "kvx_tc_load_schedule: NULL argument");
+  if (src_layers < 1 || tgt_layers < 1 || k < 1 || k > src_layers)
+    return fail(KVX_ERR_INVALID_ARG, "kvx_tc_load_schedule: need src_layers, tgt_layers >= 1 and k in [1, src_layers]");
+  if (k > kvx::kTSlots)
+    return fail(KVX_ERR_UNSUPPORTED, "kvx_tc_load_schedule: the per-head tensor-core kernel holds at most 4 source tiles");
+  for (int32_t l = 0; l < tgt_layers; ++l) {
+    const int32_t* row = selection + static_cast<size_t>(l) * k;
+    for (int32_t j = 0; j < k; ++j) {
+      if (row[j] < 0 || row[j] >= src_layers)
+        return fail(KVX_ERR_INVALID_ARG, "kvx_tc_load_schedule: selection entry outside [0, src_layers)");
+      for (int32_t i = 0; i < j; ++i)
+        if (row[i] == row[j]) return fail(KVX_ERR_INVALID_ARG, "kvx_tc_load_schedule: duplicate source layer in a row");
+    }
+  }
+  kvx::TcPlan plan;
+  kvx::build_plan(selection, src_layers, tgt_layers, k, &plan);
+  *n_loads = plan.n_loads;
+  for (int e = 0; e < plan.n_loads; ++e) {
+    load_layer[e] = plan.load_layer[e];
+    load_word[e] = plan.load_slot[e];
+  }
+  for (int u = 0; u < tgt_layers * k; ++u) use_word[u] = static_cast<int32_t>(kvx::use_bits(plan, u));
+  return KVX_OK;
+}
+
+}  // extern "C"

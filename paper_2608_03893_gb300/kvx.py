@@ -127,7 +127,7 @@ EXPORTED = ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_
             "kvx_last_error", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms", "kvx_r2_probe",
             "kvx_select_topk_device", "kvx_fit_workspace_bytes", "kvx_r2_probe_workspace_bytes",
             "kvx_mlp_map", "kvx_mlp_workspace_bytes", "kvx_host_pipe_create", "kvx_map_host",
-            "kvx_host_pipe_destroy", "kvx_set_test_wait", "kvx_get_kernel")
+            "kvx_host_pipe_destroy", "kvx_set_test_wait", "kvx_get_kernel", "kvx_tc_load_schedule")
 
 
 def lib():
@@ -175,6 +175,8 @@ def lib():
     L.kvx_set_test_wait.argtypes = [vp, ctypes.c_uint64, i64]
     L.kvx_get_kernel.argtypes = [vp, i32, ctypes.POINTER(i32)]
     L.kvx_get_kernel.restype = ctypes.c_int
+    L.kvx_tc_load_schedule.argtypes = [vp, i32, i32, i32, ctypes.POINTER(i32), vp, vp, vp]
+    L.kvx_tc_load_schedule.restype = ctypes.c_int
     L.kvx_set_test_wait.restype = ctypes.c_int
     for name in ("kvx_create", "kvx_map", "kvx_destroy", "kvx_select_topk", "kvx_get_selection",
                  "kvx_set_kernel", "kvx_get_status", "kvx_map_noalloc", "kvx_fit_ridge", "kvx_last_phase_ms",
@@ -260,6 +262,21 @@ def kvx_select_topk(scores, k):
     _check(lib().kvx_select_topk(_ptr(s), s.shape[0], s.shape[1], int(k), _ptr(out)),
            "kvx_select_topk")
     return out
+
+
+def kvx_tc_load_schedule(selection, src_layers):
+    """selection: int32 [L_t][k] -> (load_layer [n_loads], load_word [n_loads], use_word [L_t][k]),
+    the per-head tensor-core kernel's source-tile schedule (host only)."""
+    import numpy as np
+    sel = np.ascontiguousarray(selection, dtype=np.int32)
+    Lt, k = sel.shape
+    n = ctypes.c_int32(0)
+    layer = np.empty(Lt * k, dtype=np.int32)
+    word = np.empty(Lt * k, dtype=np.int32)
+    use = np.empty((Lt, k), dtype=np.int32)
+    _check(lib().kvx_tc_load_schedule(_ptr(sel), int(src_layers), Lt, k, ctypes.byref(n), _ptr(layer), _ptr(word),
+                                      _ptr(use)), "kvx_tc_load_schedule")
+    return layer[:n.value].copy(), word[:n.value].copy(), use
 
 
 def kvx_get_selection(ctx, tgt_layers, k):
