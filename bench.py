@@ -168,7 +168,7 @@ class ClockSampler:
 
 
 def measure_link(h_src, h_dst, d_src, d_dst, dev, reps=3):
-    """Host link bandwidth of this box in GB/s, from pinned copies of the step's own
+    """Host link bandwidth of this machine in GB/s, from pinned copies of the step's own
     buffers: host->device alone, device->host alone, and both at once on two streams
     (best of `reps`).  The e2e copy floor of a step follows from these."""
     def timed(fns):
