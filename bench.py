@@ -56,9 +56,29 @@ def algorithmic(w):
     src_per_tok = 2 * w.Ls * w.H * w.d * e                       # every source layer read once
     tgt_per_tok = 2 * w.Lt * w.H * w.d * e                       # target written once
     w_bytes = w.Lt * 2 * w.H * w.F * w.d * e + w.Lt * 2 * w.H * w.d * e
+    # looser bound: a mapper without reuse reads the k selected source tiles again for
+    # every (target layer, K|V, head) product (per head; one product per (target layer,
+    # K|V) cross-head) and writes its output: intensity k d / (k + 1) FLOP per byte per head
+    per_head = w.head_mix != "cross_head"
+    gemms, out = (2 * w.Lt * w.H, w.d) if per_head else (2 * w.Lt, w.H * w.d)
+    no_reuse_per_tok = gemms * (w.F + out) * e
     return dict(flop=flop_per_tok * tok, bytes=(src_per_tok + tgt_per_tok + 4) * tok + w_bytes,
                 flop_per_token=flop_per_tok, bytes_per_token=src_per_tok + tgt_per_tok + 4,
-                weight_bytes=w_bytes)
+                weight_bytes=w_bytes, no_reuse_bytes_per_token=no_reuse_per_tok,
+                no_reuse_intensity=flop_per_tok / no_reuse_per_tok)
+
+
+def no_reuse_bound(alg, w, peaks, ms_step):
+    """The roofline of a mapper that re-reads its source tiles for every product (the
+    looser bound, intensity k d / (k + 1)): its time, and frac = that time / the measured
+    launch time, defined as the main roofline's (above 1: faster than any mapper without
+    source reuse could be)."""
+    t_tc = alg["flop"] / (peaks["bf16"] * 1e12)
+    t_hbm = alg["no_reuse_bytes_per_token"] * w.n_tokens / (peaks["hbm"] * 1e9)
+    ms = 1e3 * max(t_tc, t_hbm)
+    return {"bytes_per_token": alg["no_reuse_bytes_per_token"],
+            "intensity_flop_per_byte": alg["no_reuse_intensity"], "roofline_ms": ms,
+            "bound": "tensor" if t_tc >= t_hbm else "hbm", "frac": ms / ms_step}
 
 
 def load_peaks():
@@ -886,7 +906,8 @@ def main():
                           # against cuBLAS run back to back under the power cap (the
                           # regime a long bench run settles in); context, not the headline
                           "tensor_frac_of_sustained": (alg["flop"] / launch_s / 1e12 / peaks["bf16_sustained"]
-                                                       if peaks.get("bf16_sustained") else None)},
+                                                       if peaks.get("bf16_sustained") else None),
+                          "no_reuse": no_reuse_bound(alg, w, peaks, ms_step)},
                 "algorithmic": {"flop_per_launch": alg["flop"], "bytes_per_launch": alg["bytes"],
                                 "flop_per_token": alg["flop_per_token"],
                                 "bytes_per_token": alg["bytes_per_token"],

@@ -52,3 +52,27 @@ def test_traffic_scale_is_the_token_ratio():
     # the per-launch figure stays close to the algorithmic bytes of the full launch
     alg = bench.algorithmic(full)["bytes"]
     assert 0.95 * alg < float(kv["dram_bytes_per_launch"]) < 1.10 * alg
+
+
+def test_no_reuse_bound_has_the_stated_intensity():
+    # per head: each (target layer, K|V, head) product reads k tiles of d channels and
+    # writes d, 2 k d d FLOP per token: intensity k d / (k + 1)
+    for name in ("qwen3_14b_32b_t32768_k4", "qwen3_14b_32b_t32768_k1", "llama31_8b_70b_b4x8192_k3"):
+        w = syn.workload(name)
+        alg = bench.algorithmic(w)
+        assert alg["no_reuse_intensity"] == w.k * w.d / (w.k + 1)
+        # reuse only lowers the bytes: source once and target once
+        assert alg["no_reuse_bytes_per_token"] >= alg["bytes_per_token"] - 4
+    # cross-head: one product per (target layer, K|V) reads k H d features and writes H d,
+    # 2 (k H d) (H d) FLOP per token: intensity k H d / (k + 1)
+    w = syn.workload("qwen3_14b_32b_t32768_k4_xhead")
+    alg = bench.algorithmic(w)
+    assert alg["no_reuse_intensity"] == w.k * w.H * w.d / (w.k + 1)
+    peaks = {"bf16": 1900.0, "hbm": 6800.0}
+    b = bench.no_reuse_bound(bench.algorithmic(syn.workload("qwen3_14b_32b_t32768_k4")),
+                             syn.workload("qwen3_14b_32b_t32768_k4"), peaks, 3.0)
+    # 1024 products x (512 + 128) x 2 B = 1,310,720 B per token; over 32768 tokens at
+    # 6.8 TB/s that is 6.316 ms, above the 2.315 ms of FLOPs; frac is bound time / measured
+    assert b["bytes_per_token"] == 1310720
+    assert b["bound"] == "hbm" and abs(b["roofline_ms"] - 32768 * 1310720 / 6.8e9) < 1e-9
+    assert abs(b["frac"] - b["roofline_ms"] / 3.0) < 1e-12
