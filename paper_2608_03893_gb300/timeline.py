@@ -15,6 +15,7 @@ import collections
 import ctypes
 import glob
 import os
+import re
 import shutil
 import subprocess
 import sys
@@ -65,6 +66,14 @@ SPANS = [
 ]
 
 
+def _anchor_re(text):
+    """A probe's anchor as a pattern that starts at a line start and ignores each line's
+    indentation (group 1: the first line's), so re-indenting the kernel keeps it valid."""
+    lines = text.split("\n")
+    rest = [(" *" + re.escape(ln.lstrip(" "))) if ln else "" for ln in lines[1:]]
+    return re.compile(r"(?m)^( *)" + "\n".join([re.escape(lines[0].lstrip(" "))] + rest))
+
+
 def instrument(src_dir):
     """Write the instrumented kvx_tc.cu into src_dir; returns the event table."""
     path = os.path.join(src_dir, "kvx_tc.cu")
@@ -92,11 +101,13 @@ def instrument(src_dir):
         "  }\n"
         "  unsigned int tr_i = 0;\n"), 1)
     for text, name, after in PROBES:
-        assert s.count(text) == 1, "kernel source changed: probe %s no longer matches" % name
+        found = list(_anchor_re(text).finditer(s))
+        assert len(found) == 1, "kernel source changed: probe %s no longer matches" % name
+        m = found[0]
         ev = events.setdefault(name, len(events) + 1)
-        ind = text[:len(text) - len(text.lstrip(" "))]
-        stamp = "%sTR(%d);\n" % (ind, ev)
-        s = s.replace(text, text + stamp if after else stamp + text, 1)
+        stamp = "%sTR(%d);\n" % (m.group(1), ev)
+        at = m.end() if after else m.start()
+        s = s[:at] + stamp + s[at:]
     anchor = "  tc_fence_before();\n  __syncthreads();\n  cluster_sync();   // no arrival or MMA of either CTA still targets the other"
     assert s.count(anchor) == 1
     s = s.replace(anchor, "  if (tr_role >= 0) g_trace_n[tr_cta][tr_role] = tr_i < %d ? tr_i : %d;\n" % (LEN, LEN) + anchor, 1)
