@@ -99,6 +99,42 @@ def test_head_averaged_r2_and_scores():
     assert S.shape == (1, 2) and abs(S[0, 0] - h) < 1e-12
 
 
+
+def test_r2_matrix_and_scores_find_planted_sources():
+    # L_s = 3 source layers, L_t = 2 target layers, H = 2 heads (sizes differ, so a
+    # transposed index fails).  Keys of target layer l are an exact linear map of source
+    # layer sigma(l), values of source layer tau(l) != sigma(l); every other layer is
+    # independent.  Per-head regression: target head 1 of layer 1 depends only on source
+    # head 0, which a same-head probe must not see.
+    rng = np.random.default_rng(21)
+    N, d, Ls, Lt, H = 2000, 3, 3, 2, 2
+    srcK = rng.standard_normal((Ls, H, N, d))
+    srcV = rng.standard_normal((Ls, H, N, d))
+    sigma, tau = [2, 0], [1, 2]
+    tgtK = np.stack([np.stack([srcK[sigma[l], h] @ rng.standard_normal((d, d)) + 0.3 for h in range(H)])
+                     for l in range(Lt)])
+    # values map d = 3 source channels to 2 target channels: the target is explained
+    # exactly, while a regression the other way round (source on target) could not be
+    tgtV = np.stack([np.stack([srcV[tau[l], h] @ rng.standard_normal((d, d - 1)) for h in range(H)])
+                     for l in range(Lt)])
+    tgtK[1, 1] = srcK[sigma[1], 0] @ rng.standard_normal((d, d))     # the other source head
+    RK, RV = r2.r2_matrix(srcK, tgtK), r2.r2_matrix(srcV, tgtV)
+    assert RK.shape == (Lt, Ls) and RV.shape == (Lt, Ls)
+    noise = 5.0 * d / N                                   # R^2 of unrelated data is ~ d / N
+    for l in range(Lt):
+        for lp in range(Ls):
+            assert (abs(RV[l, lp] - 1.0) < 1e-10) if lp == tau[l] else (RV[l, lp] < noise)
+    assert abs(RK[0, sigma[0]] - 1.0) < 1e-10
+    # layer 1: head 0 is exact, head 1 only through the other head: R^2 ~ 1/2
+    assert abs(RK[1, sigma[1]] - 0.5) < noise
+    assert all(RK[l, lp] < noise for l in range(Lt) for lp in range(Ls) if lp != sigma[l])
+    S = r2.selection_scores(srcK, srcV, tgtK, tgtV)
+    assert np.allclose(S, 0.5 * (RK + RV), rtol=0, atol=1e-15)
+    # the planted layers are the top two of each target layer, in the paper's order
+    assert [sorted(np.argsort(-S[l])[:2].tolist()) for l in range(Lt)] == \
+        [sorted([sigma[l], tau[l]]) for l in range(Lt)]
+
+
 # ----------------------------------------------------------------- ridge ---------
 
 def _linear_data(seed, N=400, F=12, d=5, noise=0.0):
