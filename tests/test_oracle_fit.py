@@ -55,6 +55,11 @@ def test_topk_uniform_scores_give_uniform_subsets():
     assert chi2 < 20.5  # 5 dof, p ~ 0.001
 
 
+def test_topk_of_every_layer_is_every_layer():
+    S = np.random.default_rng(3).uniform(size=(5, 4))
+    assert np.array_equal(selection.select_topk(S, 4), np.tile(np.arange(4), (5, 1)))
+
+
 def test_topk_rejects_bad_k():
     with pytest.raises(ValueError):
         selection.select_topk(np.zeros((2, 3)), 4)

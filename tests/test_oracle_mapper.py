@@ -196,11 +196,12 @@ def test_bf16fwd_error_bounded_by_operand_rounding():
 
 def test_map_cache_layout_roundtrip():
     rng = np.random.default_rng(43)
-    Ls, Lt, B, H, T, d, k = 3, 2, 2, 2, 5, 8, 2
+    Ls, Lt, B, H, T, d, k = 3, 3, 2, 2, 5, 8, 2           # L_t, B, H, T all different
+    B = 4
     src_k = rng.standard_normal((Ls, B, H, T, d))
     src_v = rng.standard_normal((Ls, B, H, T, d))
-    pos = np.stack([np.arange(T), np.arange(T) + 100])
-    sel = np.array([[0, 2], [1, 2]])
+    pos = np.stack([np.arange(T) + 100 * bb for bb in range(B)])
+    sel = np.array([[0, 2], [1, 2], [0, 1]])
     W = rng.standard_normal((Lt, 2, H, k * d, d))
     b = rng.standard_normal((Lt, 2, H, d))
     ck, cv = mapper.map_cache(src_k, src_v, pos, sel, W, b, 1e4, 1e4)
@@ -215,6 +216,10 @@ def test_rounding_slack_is_zero_without_ambiguity_and_for_values():
     assert np.all(sk == 0) and np.all(sv == 0)
     ok2, ov2, sk2, sv2 = mapper.map_tokens(**P, mode="bf16fwd", rounding_slack=4e-6)
     assert np.array_equal(ok, ok2) and np.all(sv2 == 0)
+    # the slack leaves the mapped cache itself unchanged, keys and values
+    ok0, ov0 = mapper.map_tokens(**P, mode="bf16fwd")
+    assert np.array_equal(ok0, ok2) and np.array_equal(ov0, ov2) and np.array_equal(ov0, ov)
+    assert not np.array_equal(ok0, ov0)
 
 
 def test_rounding_slack_covers_both_roundings_of_a_planted_midpoint():
@@ -222,24 +227,80 @@ def test_rounding_slack_covers_both_roundings_of_a_planted_midpoint():
     oracle's f64 strip lands within 1e-15 of the midpoint and may round either way.
     Both choices, evaluated directly, must lie within out +- slack."""
     rng = np.random.default_rng(45)
-    Ls, Lt, H, N, d, k = 2, 2, 1, 3, 8, 2
-    content = bf16.round_to_bf16_value(rng.standard_normal((Ls, H, N, d)))
-    content[0, 0, :, 1] = 1.0 + 2.0 ** -8          # ties between 1 and 1 + 2^-7
-    content[1, 0, :, 6] = -(3.0 + 2.0 ** -7)        # ties between -3 and -(3 + 2^-6)
+    Ls, Lt, H, N, d, k = 3, 2, 2, 3, 8, 2
+    # |content| in [0.5, 2]: a stored pair's fp32-strip uncertainty (4e-6 of |a| + |b|)
+    # stays far below half a bf16 step of either element, so the planted midpoints are
+    # the only ambiguous roundings
+    content = bf16.round_to_bf16_value(rng.choice([-1.0, 1.0], size=(Ls, H, N, d)) *
+                                       rng.uniform(0.5, 2.0, size=(Ls, H, N, d)))
+    # midpoints only in head 1: of source layer 0 (channel 1) and source layer 1 (channel 6)
+    content[0, 1, :, 1] = 1.0 + 2.0 ** -8          # ties between 1 and 1 + 2^-7
+    content[1, 1, :, 6] = -(3.0 + 2.0 ** -7)        # ties between -3 and -(3 + 2^-6)
     pos = np.array([0, 77, 30001])
     stored = np.stack([rope.rotate(content[s], pos[None, :], 1e4) for s in range(Ls)])
-    sel = np.array([[0, 1], [0, 1]])
+    sel = np.array([[0, 2], [1, 2]])               # each target layer meets one planted layer
     W = rng.standard_normal((Lt, 2, H, k * d, d)) / 4
     b = rng.standard_normal((Lt, 2, H, d)) * 0.1
     src_v = rng.standard_normal((Ls, H, N, d))
-    out_k, _, slack_k, _ = mapper.map_tokens(stored, src_v, pos, sel, W, b, 1e4, 1e4,
-                                             mode="bf16fwd", rounding_slack=4e-6)
+    out_k, out_v, slack_k, slack_v = mapper.map_tokens(stored, src_v, pos, sel, W, b, 1e4, 1e4,
+                                                       mode="bf16fwd", rounding_slack=4e-6)
     for down in (True, False):
         X = content.copy()
-        X[0, 0, :, 1] = 1.0 if down else 1.0 + 2.0 ** -7
-        X[1, 0, :, 6] = -3.0 if down else -(3.0 + 2.0 ** -6)
+        X[0, 1, :, 1] = 1.0 if down else 1.0 + 2.0 ** -7
+        X[1, 1, :, 6] = -3.0 if down else -(3.0 + 2.0 ** -6)
         for l in range(Lt):
-            Xl = np.concatenate([X[s, 0] for s in sel[l]], axis=-1)
-            y = rope.rotate(Xl @ W[l, 0, 0] + b[l, 0, 0], pos, 1e4)
-            assert np.all(np.abs(y - out_k[l, 0]) <= slack_k[l, 0] + 1e-12)
-    assert np.all(slack_k[:, 0][:, :, [1, 5]] > 0)   # the planted pairs are flagged
+            for h in range(H):
+                Xl = np.concatenate([X[s, h] for s in sel[l]], axis=-1)
+                y = rope.rotate(Xl @ W[l, 0, h] + b[l, 0, h], pos, 1e4)
+                assert np.all(np.abs(y - out_k[l, h]) <= slack_k[l, h] + 1e-12)
+    assert np.all(slack_k[:, 1] > 0)     # every output of head 1 meets a planted pair
+    assert np.all(slack_k[:, 0] == 0) and np.all(slack_v == 0)
+    # the slack is the worst case of the other rounding: |W| rows of the ambiguous feature
+    # (feature 1 of block 0 in layer 0, feature 6 of block 0 in layer 1), its bf16 step
+    # (2^-7 and 2^-6), summed over the output's RoPE pair after the rotation
+    for l, f, step in ((0, 1, 2.0 ** -7), (1, 6, 2.0 ** -6)):
+        per_c = step * np.abs(W[l, 0, 1, f])                  # [d]
+        want = np.concatenate([per_c[:4] + per_c[4:]] * 2)
+        assert np.allclose(slack_k[l, 1], np.broadcast_to(want, (N, d)), rtol=1e-12, atol=0)
+    # cross-head features with W zero outside head h's rows give the same map and slack
+    Wx = np.zeros((Lt, 2, H, k * H * d, d))
+    for l in range(Lt):
+        for h in range(H):
+            for j in range(k):
+                Wx[l, :, h, (j * H + h) * d:(j * H + h + 1) * d] = W[l, :, h, j * d:(j + 1) * d]
+    xk, xv, xsk, xsv = mapper.map_tokens(stored, src_v, pos, sel, Wx, b, 1e4, 1e4, mode="bf16fwd",
+                                         rounding_slack=4e-6, head_mix="cross_head")
+    assert np.allclose(xk, out_k, rtol=0, atol=1e-12) and np.allclose(xv, out_v, rtol=0, atol=1e-12)
+    assert np.allclose(xsk, slack_k, rtol=1e-12, atol=0) and np.all(xsv == 0)
+
+
+def test_slack_helpers_hand_values():
+    x = np.array([1.0, -2.0, 3.0, -4.0])
+    # half-split pairs (0, 2), (1, 3); interleaved pairs (0, 1), (2, 3)
+    assert mapper._pair_magnitude(x, "half").tolist() == [4.0, 6.0, 4.0, 6.0]
+    assert mapper._pair_magnitude(x, "interleaved").tolist() == [3.0, 3.0, 7.0, 7.0]
+    assert mapper._pair_sum(x, "half").tolist() == [4.0, -6.0, 4.0, -6.0]
+    assert mapper._pair_sum(x, "interleaved").tolist() == [-1.0, -1.0, -1.0, -1.0]
+
+
+def test_hf_numerics_identity_map_returns_the_source_keys():
+    """k = 1, W = I, b = 0, equal thetas with the Hugging Face rounding: the strip and
+    the re-rotation cancel up to the bf16 roundings of the two rotations (each product,
+    sum and cos / sin rounded once: well under 2^-5 of the pair magnitude), on caches
+    whose L, H, N and d all differ."""
+    rng = np.random.default_rng(47)
+    Ls, H, N, d = 2, 3, 7, 16
+    src_k = bf16.round_to_bf16_value(rng.standard_normal((Ls, H, N, d)))
+    src_v = bf16.round_to_bf16_value(rng.standard_normal((Ls, H, N, d)))
+    pos = np.array([1, 5, 77, 300, 4000, 30001, 65535])
+    sel = np.array([[1], [0]])
+    W = np.broadcast_to(np.eye(d), (2, 2, H, d, d)).copy()
+    for mode in ("exact", "bf16fwd"):
+        ok, ov = mapper.map_tokens(src_k, src_v, pos, sel, W, None, 5e5, 5e5, mode=mode, rope_numerics="hf")
+        for l, s in ((0, 1), (1, 0)):
+            mag = mapper._pair_magnitude(src_k[s], "half")
+            assert np.all(np.abs(ok[l] - src_k[s]) <= 2.0 ** -5 * mag + 1e-30)
+            assert np.array_equal(ov[l], src_v[s])
+        # the HF rounding is visible: not the exact-numerics result
+        ek, _ = mapper.map_tokens(src_k, src_v, pos, sel, W, None, 5e5, 5e5, mode=mode)
+        assert not np.array_equal(ok, ek)

@@ -28,13 +28,23 @@ def test_worked_example():
     assert mlp.mlp_forward(x, W1, b1, W2, b2n, W3, b3)[0, 0] == 6.25
 
 
-def _linear_as_mlp(Wlin, b):
-    """W_lin [F][d] (row-vector map x W + b) as MLP weights with hidden = 2d."""
+def _linear_as_mlp(Wlin, b, rng=None):
+    """W_lin [F][d] (row-vector map x W + b) as MLP weights with hidden = 2d.
+
+    z = x W_lin; layer 1 gives [relu(z + c); relu(-z - c)]; layer 2 scales both halves by
+    a positive diagonal D and adds e1, e2 >= 0 (the ReLU is then inert); layer 3 takes
+    D^-1 (first half - second half): relu(u) - relu(-u) = u leaves z + c + (e1 - e2) / D,
+    and b3 = b - c - (e1 - e2) / D.  With ``rng`` every block gets its own c, D, e1, e2."""
     F, d = Wlin.shape
-    W1 = np.concatenate([Wlin.T, -Wlin.T], axis=0)          # [2d][F]
-    W2 = np.eye(2 * d)
-    W3 = np.concatenate([np.eye(d), -np.eye(d)], axis=1)    # [d][2d]
-    return W1, np.zeros(2 * d), W2, np.zeros(2 * d), W3, b
+    if rng is None:
+        c, D, e1, e2 = np.zeros(d), np.ones(d), np.zeros(d), np.zeros(d)
+    else:
+        c, D = rng.standard_normal(d), rng.uniform(0.5, 2.0, d)
+        e1, e2 = rng.uniform(0.0, 1.0, d), rng.uniform(0.0, 1.0, d)
+    W1 = np.concatenate([Wlin.T, -Wlin.T], axis=0)                      # [2d][F]
+    W2 = np.diag(np.concatenate([D, D]))
+    W3 = np.concatenate([np.diag(1.0 / D), -np.diag(1.0 / D)], axis=1)   # [d][2d]
+    return W1, np.concatenate([c, -c]), W2, np.concatenate([e1, e2]), W3, b - c - (e1 - e2) / D
 
 
 def test_relu_identity_reduces_to_the_ridge_mapper():
@@ -53,7 +63,8 @@ def test_relu_identity_reduces_to_the_ridge_mapper():
         for kv in range(2):
             per_kv = {n: [] for n in params}
             for h in range(H):
-                for n, v in zip(("W1", "b1", "W2", "b2", "W3", "b3"), _linear_as_mlp(W[l, kv, h], b[l, kv, h])):
+                for n, v in zip(("W1", "b1", "W2", "b2", "W3", "b3"),
+                                _linear_as_mlp(W[l, kv, h], b[l, kv, h], rng)):
                     per_kv[n].append(v)
             for n in params:
                 per_l[n].append(per_kv[n])
@@ -63,6 +74,14 @@ def test_relu_identity_reduces_to_the_ridge_mapper():
     ok, ov = mlp.map_tokens_mlp(src_k, src_v, pos, sel, params, 1e6, 5e5)
     rk, rv = mapper.map_tokens(src_k, src_v, pos, sel, W, b, 1e6, 5e5, head_mix="cross_head")
     assert np.allclose(ok, rk, rtol=0, atol=1e-9) and np.allclose(ov, rv, rtol=0, atol=1e-9)
+    # the Hugging Face rounding of the strip and the re-rotation (the MLP's HF forward
+    # rounds both rotations to bf16, as the mapper's bf16 forward does): equal up to the
+    # bf16 rounding of the output, whose pre-rounding values differ in the last f64 bits
+    hk, hv = mlp.map_tokens_mlp(src_k, src_v, pos, sel, params, 1e6, 5e5, rope_numerics="hf")
+    gk, gv = mapper.map_tokens(src_k, src_v, pos, sel, W, b, 1e6, 5e5, head_mix="cross_head",
+                               mode="bf16fwd", rope_numerics="hf")
+    assert np.all(np.abs(hk - gk) <= 2.0 ** -7 * np.abs(gk) + 1e-30)
+    assert np.mean(hk == gk) > 0.99 and np.allclose(hv, rv, rtol=0, atol=1e-9)
 
 
 def test_dead_relu_leaves_the_rotated_last_bias():

@@ -137,6 +137,17 @@ def test_bf16_rne_matches_torch_from_binary32():
     assert np.array_equal(got, expect)
 
 
+def test_bf16_rne_matches_torch_across_the_subnormal_boundary():
+    """Every binary32 value on a 2^-140 grid from 2^-135 to 2^-124: bf16's subnormal
+    quantum 2^-133 below 2^-126, its 8-bit significand above (including the band just
+    under the smallest normal, where the two quanta differ)."""
+    k = np.arange(2 ** 5, 2 ** 16 + 1, dtype=np.float64)
+    x = (k * 2.0 ** -140).astype(np.float32)
+    x = np.concatenate([x, -x])
+    expect = torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(bf16.encode(x.astype(np.float64)), expect)
+
+
 # ---- Llama-3 frequency scaling ------------------------------------------------------
 
 LLAMA31 = rope.Llama3Scaling(8.0, 1.0, 4.0, 8192.0)
