@@ -1,7 +1,8 @@
 """Mutation audit of the oracle's pins (CPU; run by hand, not collected by pytest).
 
 Each mutant changes one operator on one code line of ``oracle/*.py`` (a sign, an index,
-an axis, a comparison, a constant, cos for sin, a reduction) in a private copy of the
+an axis, a comparison, a constant, cos for sin, a reduction, an argument such as theta_s
+for theta_t, a rounding point such as float32 for float64) in a private copy of the
 package, and runs the oracle pin tests against it.  A mutant the pins do not reject is a
 "survivor".  Survivors listed in EQUIVALENT compute the same result on every input the
 oracle accepts, for the reason given; any other survivor is a gap in the pins and makes
@@ -31,6 +32,12 @@ OPS = [
     (r"\bmin\(", "max("), (r"\bmax\(", "min("), (r"\bh\b", "0"), (r"\bl\b", "0"), (r"\bj\b", "0"),
     (r"np\.sum\(", "np.mean("), (r"np\.mean\(", "np.sum("), (r"\+= ", "= "), (r"\bTrue\b", "False"),
     (r"// 2\b", "// 4"), (r"- 1\b", ""), (r"\+ 1\b", ""),
+    (r"\btheta_s\b", "theta_t"), (r"\btheta_t\b", "theta_s"), (r"np\.abs\(", "("), (r"0::2", "1::2"),
+    (r"1::2", "0::2"), (r"-2\.0", "2.0"), (r"\.mean\(", ".sum("), (r"\.sum\(", ".mean("),
+    (r"\bnp\.rint\(", "np.floor("), (r"\bsqrt\(", "abs("), (r"\blower=True\b", "lower=False"),
+    (r"\bstyle=style\b", "style=\"half\""), (r"\bbf16_cache=True\b", "bf16_cache=False"),
+    (r"\bmode\b", "\"exact\""), (r"\[::-1\]", ""), (r"\bx_mean\b", "0.0"), (r"\by_mean\b", "0.0"),
+    (r"\blam\b", "lam2"), (r"\bnp\.float32\b", "np.float64"),
 ]
 
 # (file, mutated line after the change, why it computes the same result)
@@ -47,6 +54,10 @@ EQUIVALENT = [
     ("mlp.py", "return np.concatenate(parts, axis=1)", "2-D parts: axis 1 is the last"),
     ("ridge.py", "Yc = Y + y_mean",
      "W only sees Xc^T Yc and Xc^T 1 = 0 (X is centred), so the sign of the Y mean drops out; b uses y_mean itself"),
+    ("ridge.py", "Yc = Y - 0.0", "as above: Xc^T Y = Xc^T Yc for a centred Xc"),
+    ("rope.py", "ang = (p32[..., None] * w32).astype(np.float64).astype(np.float64)   # fp32 multiply, rounded",
+     "p32 and w32 are float32 arrays, so numpy's product is already the binary32 product"),
+    ("mapper.py", 'raise ValueError("exact")', "only the error message's text changes"),
     ("ridge.py", "factor = scipy.linalg.cho_factor(A, lower=False)",
      "cho_solve follows the factor's own lower / upper flag"),
     ("rope.py", "out = np.where(lam <= P / s.high_freq_factor, omega, blend)",

@@ -204,10 +204,15 @@ def test_map_cache_layout_roundtrip():
     sel = np.array([[0, 2], [1, 2], [0, 1]])
     W = rng.standard_normal((Lt, 2, H, k * d, d))
     b = rng.standard_normal((Lt, 2, H, d))
-    ck, cv = mapper.map_cache(src_k, src_v, pos, sel, W, b, 1e4, 1e4)
-    for bb in range(B):
-        tk, tv = mapper.map_tokens(src_k[:, bb], src_v[:, bb], pos[bb], sel, W, b, 1e4, 1e4)
-        assert np.array_equal(ck[:, bb], tk) and np.array_equal(cv[:, bb], tv)
+    for kw in ({}, dict(mode="bf16fwd", style="interleaved"), dict(rope_numerics="hf")):
+        ck, cv = mapper.map_cache(src_k, src_v, pos, sel, W, b, 1e4, 5e5, **kw)
+        for bb in range(B):
+            tk, tv = mapper.map_tokens(src_k[:, bb], src_v[:, bb], pos[bb], sel, W, b, 1e4, 5e5, **kw)
+            assert np.array_equal(ck[:, bb], tk) and np.array_equal(cv[:, bb], tv)
+    # and the thetas and the mode reach the map: other values give another cache
+    ck2, _ = mapper.map_cache(src_k, src_v, pos, sel, W, b, 5e5, 1e4)
+    ck3, _ = mapper.map_cache(src_k, src_v, pos, sel, W, b, 1e4, 5e5, mode="bf16fwd")
+    assert not np.array_equal(ck, ck2) and not np.array_equal(ck, ck3)
 
 
 def test_rounding_slack_is_zero_without_ambiguity_and_for_values():
@@ -279,11 +284,19 @@ def test_slack_helpers_hand_values():
     # half-split pairs (0, 2), (1, 3); interleaved pairs (0, 1), (2, 3)
     assert mapper._pair_magnitude(x, "half").tolist() == [4.0, 6.0, 4.0, 6.0]
     assert mapper._pair_magnitude(x, "interleaved").tolist() == [3.0, 3.0, 7.0, 7.0]
+    assert mapper._pair_magnitude(-x, "half").tolist() == [4.0, 6.0, 4.0, 6.0]
+    assert mapper._pair_magnitude(-x, "interleaved").tolist() == [3.0, 3.0, 7.0, 7.0]
     assert mapper._pair_sum(x, "half").tolist() == [4.0, -6.0, 4.0, -6.0]
     assert mapper._pair_sum(x, "interleaved").tolist() == [-1.0, -1.0, -1.0, -1.0]
 
 
-def test_hf_numerics_identity_map_returns_the_source_keys():
+def test_unknown_mode_is_rejected():
+    with pytest.raises(ValueError):
+        mapper.map_tokens(**_problem(48), mode="fp8")
+
+
+@pytest.mark.parametrize("style", ["half", "interleaved"])
+def test_hf_numerics_identity_map_returns_the_source_keys(style):
     """k = 1, W = I, b = 0, equal thetas with the Hugging Face rounding: the strip and
     the re-rotation cancel up to the bf16 roundings of the two rotations (each product,
     sum and cos / sin rounded once: well under 2^-5 of the pair magnitude), on caches
@@ -296,11 +309,12 @@ def test_hf_numerics_identity_map_returns_the_source_keys():
     sel = np.array([[1], [0]])
     W = np.broadcast_to(np.eye(d), (2, 2, H, d, d)).copy()
     for mode in ("exact", "bf16fwd"):
-        ok, ov = mapper.map_tokens(src_k, src_v, pos, sel, W, None, 5e5, 5e5, mode=mode, rope_numerics="hf")
+        ok, ov = mapper.map_tokens(src_k, src_v, pos, sel, W, None, 5e5, 5e5, mode=mode, style=style,
+                                   rope_numerics="hf")
         for l, s in ((0, 1), (1, 0)):
-            mag = mapper._pair_magnitude(src_k[s], "half")
+            mag = mapper._pair_magnitude(src_k[s], style)
             assert np.all(np.abs(ok[l] - src_k[s]) <= 2.0 ** -5 * mag + 1e-30)
             assert np.array_equal(ov[l], src_v[s])
         # the HF rounding is visible: not the exact-numerics result
-        ek, _ = mapper.map_tokens(src_k, src_v, pos, sel, W, None, 5e5, 5e5, mode=mode)
+        ek, _ = mapper.map_tokens(src_k, src_v, pos, sel, W, None, 5e5, 5e5, mode=mode, style=style)
         assert not np.array_equal(ok, ek)

@@ -116,3 +116,81 @@ def test_bf16fwd_rounds_hidden_activations():
     rounded = mlp.mlp_forward(X, W1, b1, W2, b2, W3, b3, round_hidden=True)
     assert not np.array_equal(exact, rounded)
     assert np.allclose(exact, rounded, rtol=0.05, atol=0.05)
+
+
+def test_bf16fwd_features_match_the_mapper_exactly():
+    """bf16fwd rounds the stripped keys before the first layer, as the mapper does.  With
+    one power-of-two entry per column of W_lin, and D a power of two, every hidden value
+    is a scaled copy of one rounded feature, so the hidden roundings change nothing and
+    the MLP equals the mapper's bf16 forward bit for bit."""
+    rng = np.random.default_rng(9)
+    Ls, Lt, H, N, d, k = 3, 2, 2, 5, 16, 2
+    src_k = bf16.round_to_bf16_value(rng.standard_normal((Ls, H, N, d)))
+    src_v = bf16.round_to_bf16_value(rng.standard_normal((Ls, H, N, d)))
+    pos = np.array([0, 3, 700, 9000, 31111])
+    sel = np.array([[0, 2], [1, 2]])
+    F = k * H * d
+    W = np.zeros((Lt, 2, H, F, d))
+    b = rng.standard_normal((Lt, 2, H, d))
+    params = {n: np.zeros((Lt, 2, H) + shp) for n, shp in
+              (("W1", (2 * d, F)), ("b1", (2 * d,)), ("W2", (2 * d, 2 * d)), ("b2", (2 * d,)),
+               ("W3", (d, 2 * d)), ("b3", (d,)))}
+    for l in range(Lt):
+        for kv in range(2):
+            for h in range(H):
+                rows = rng.integers(0, F, d)
+                W[l, kv, h, rows, np.arange(d)] = rng.choice([-1.0, 1.0], d) * 2.0 ** rng.integers(-2, 3, d)
+                D = 2.0 ** rng.integers(-2, 3, d)
+                params["W1"][l, kv, h] = np.concatenate([W[l, kv, h].T, -W[l, kv, h].T])
+                params["W2"][l, kv, h] = np.diag(np.concatenate([D, D]))
+                params["W3"][l, kv, h] = np.concatenate([np.diag(1.0 / D), -np.diag(1.0 / D)], axis=1)
+                params["b3"][l, kv, h] = b[l, kv, h]
+    ok, ov = mlp.map_tokens_mlp(src_k, src_v, pos, sel, params, 1e4, 1e6, mode="bf16fwd")
+    rk, rv = mapper.map_tokens(src_k, src_v, pos, sel, W, b, 1e4, 1e6, head_mix="cross_head", mode="bf16fwd")
+    assert np.array_equal(ok, rk) and np.array_equal(ov, rv)
+    ek, _ = mapper.map_tokens(src_k, src_v, pos, sel, W, b, 1e4, 1e6, head_mix="cross_head")
+    assert not np.array_equal(ok, ek)
+
+
+def test_bf16fwd_rounds_hidden_activations_inside_the_map():
+    # W2 = W3 = I and zero later biases: the mapped values are the second hidden layer
+    rng = np.random.default_rng(10)
+    Ls, Lt, H, N, d, k = 2, 1, 1, 6, 8, 1
+    src_k = rng.standard_normal((Ls, H, N, d))
+    src_v = rng.standard_normal((Ls, H, N, d))
+    F = k * H * d
+    params = dict(W1=rng.standard_normal((Lt, 2, H, d, F)), b1=np.full((Lt, 2, H, d), 5.0),
+                  W2=np.broadcast_to(np.eye(d), (Lt, 2, H, d, d)).copy(), b2=np.zeros((Lt, 2, H, d)),
+                  W3=np.broadcast_to(np.eye(d), (Lt, 2, H, d, d)).copy(), b3=np.zeros((Lt, 2, H, d)))
+    sel = np.array([[1]])
+    _, v16 = mlp.map_tokens_mlp(src_k, src_v, np.arange(N), sel, params, 1e4, 1e4, mode="bf16fwd")
+    _, v64 = mlp.map_tokens_mlp(src_k, src_v, np.arange(N), sel, params, 1e4, 1e4)
+    assert np.array_equal(v16, bf16.round_to_bf16_value(v16)) and not np.array_equal(v64, v16)
+    assert np.allclose(v16, v64, rtol=2.0 ** -7, atol=0)
+
+
+def test_bf16fwd_rounds_the_stripped_keys_before_the_first_layer():
+    """A first-layer unit that adds two stripped key channels: in bf16fwd the MLP sees
+    bf16(s_0) + bf16(s_1) (the operand rounding of the bf16 forward), and its hidden
+    rounding then gives bf16(bf16(s_0) + bf16(s_1)); rounding only after the sum would give
+    bf16(s_0 + s_1), which differs for some tokens.  Brute force per token from the
+    pinned strip (rope.rotate) and rounding (bf16.round_to_bf16_value)."""
+    rng = np.random.default_rng(12)
+    N, d = 256, 8
+    src_k = bf16.round_to_bf16_value(rng.standard_normal((1, 1, N, d)))
+    src_v = bf16.round_to_bf16_value(rng.standard_normal((1, 1, N, d)))
+    pos = rng.integers(1, 30000, N)
+    sel = np.array([[0]])
+    zero = lambda *shp: np.zeros((1, 2, 1) + shp)
+    params = dict(W1=zero(2, d), b1=zero(2), W2=np.broadcast_to(np.eye(2), (1, 2, 1, 2, 2)).copy(),
+                  b2=zero(2), W3=zero(d, 2), b3=zero(d))
+    params["W1"][0, :, 0, 0, :2] = 1.0            # hidden 0: s_0 + s_1
+    params["W1"][0, :, 0, 1, :2] = -1.0           # hidden 1: -(s_0 + s_1)
+    params["W3"][0, :, 0, 0] = [1.0, -1.0]        # output channel 0: relu(z) - relu(-z) = z
+    ok, _ = mlp.map_tokens_mlp(src_k, src_v, pos, sel, params, 1e4, 1e4, mode="bf16fwd")
+    z = rope.rotate(ok[0, 0], pos, 1e4, inverse=True)[:, 0]      # undo the target rotation
+    s = rope.rotate(src_k[0, 0], pos, 1e4, inverse=True)
+    r = bf16.round_to_bf16_value
+    want = r(r(s[:, 0]) + r(s[:, 1]))
+    assert np.allclose(z, want, rtol=1e-12, atol=1e-300)
+    assert np.any(r(s[:, 0] + s[:, 1]) != want)                     # the case tells them apart

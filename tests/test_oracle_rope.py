@@ -137,6 +137,18 @@ def test_bf16_rne_matches_torch_from_binary32():
     assert np.array_equal(got, expect)
 
 
+def test_bf16_overflow_rounds_to_signed_infinity():
+    big = 3.3895313892515355e38                      # the largest finite bf16, 0x7F7F
+    vals = np.array([big, -big, 3.39e38, -3.39e38, 1e39, -1e39, 3.3962e38, -3.3962e38])   # midpoint 3.39618e38
+    assert bf16.encode(vals).tolist() == [0x7F7F, 0xFF7F, 0x7F7F, 0xFF7F, 0x7F80, 0xFF80, 0x7F80, 0xFF80]
+    assert bf16.round_to_bf16_value(vals).tolist() == [big, -big, big, -big, np.inf, -np.inf, np.inf, -np.inf]
+    # binary32 values near the top of the range, both signs, against torch's cast
+    x = np.linspace(3.3e38, 3.4028234e38, 4001).astype(np.float32)
+    x = np.concatenate([x, -x])
+    expect = torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(bf16.encode(x.astype(np.float64)), expect)
+
+
 def test_bf16_rne_matches_torch_across_the_subnormal_boundary():
     """Every binary32 value on a 2^-140 grid from 2^-135 to 2^-124: bf16's subnormal
     quantum 2^-133 below 2^-126, its 8-bit significand above (including the band just
@@ -204,6 +216,31 @@ def test_hf_rotation_worked_example():
     assert y[1, 0] == 0.5390625 and y[1, 64] == 0.83984375
     c, s = rope.hf_cos_sin(np.array([1]), 1e6, 128)
     assert c[0, 0] == 0.5390625 and s[0, 0] == 0.83984375
+
+
+def test_hf_angles_are_torch_binary32_products():
+    """The Hugging Face forward forms the angle as a binary32 product of binary32(t) and
+    binary32(omega_i): computed here with torch in float32 (positions past 2^24 included,
+    where binary32(t) is itself rounded), then cos / sin in float64."""
+    d, theta = 128, 1e6
+    t = np.array([0, 1, 77, 30001, 2 ** 20 + 3, 2 ** 24 + 1, 2 ** 25 + 3, 123456789])
+    w32 = torch.from_numpy(rope.inv_freq(theta, d).astype(np.float32))
+    ang = (torch.from_numpy(t.astype(np.float32))[:, None] * w32[None, :]).double().numpy()
+    c, s = rope.hf_cos_sin(t, theta, d, bf16_cache=False)
+    assert np.array_equal(c, np.cos(ang).astype(np.float32).astype(np.float64))
+    assert np.array_equal(s, np.sin(ang).astype(np.float32).astype(np.float64))
+    cb, sb = rope.hf_cos_sin(t, theta, d)
+    assert np.array_equal(cb, bf16.round_to_bf16_value(np.cos(ang)))
+    assert np.array_equal(sb, bf16.round_to_bf16_value(np.sin(ang)))
+    # an fp64 angle would differ: the check above sees the binary32 rounding points
+    assert not np.array_equal(c, np.cos(np.outer(t, rope.inv_freq(theta, d))).astype(np.float32))
+
+
+def test_hf_rotation_with_a_binary32_cache_returns_binary32_values():
+    x = _rng(31).standard_normal((5, 64))
+    y = rope.rotate_hf(x, np.arange(5) * 1000, 1e4, bf16_cache=False)
+    assert np.array_equal(y, y.astype(np.float32).astype(np.float64))
+    assert not np.array_equal(y, bf16.round_to_bf16_value(y))
 
 
 def test_hf_rotation_properties():
