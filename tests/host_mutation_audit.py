@@ -2,8 +2,10 @@
 collected by pytest; nvcc needed, no GPU).
 
 The audited functions are the ones the CPU tests can reach without a device: the top-k
-selection, the mapper-size formula, kvx_create's host checks and selection table, and
-the per-head kernel's load-schedule builder with its entry point.  Each mutant changes
+selection, the mapper-size formula, the RoPE-scaling check, kvx_create's host checks and
+selection table, the per-head kernel's load-schedule builder with its entry point, and
+the host checks of the fit, probe, MLP and no-alloc entry points (each up to its first
+CUDA call).  Each mutant changes
 one operator on one code line of one of them (a comparison, a logical operator, a sign,
 an index, a constant, a bit of a schedule word) in a private copy of the package; the
 copy's build() recompiles that translation unit and relinks, and the CPU tests of the
@@ -26,20 +28,30 @@ import sys
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 PKG = "paper_2608_03893_gb300"
-TESTS = ["tests/test_abi_cpu.py", "tests/test_schedule_cpu.py", "tests/test_abi_validation_cpu.py"]
+TESTS = ["tests/test_abi_cpu.py", "tests/test_schedule_cpu.py", "tests/test_abi_validation_cpu.py",
+         "tests/test_abi_bounds_cpu.py"]
 
-# (file, regex of the function's first line); the function ends at the next "}" in column 0
+# (file, regex of the function's first line, text of the first line that reaches the
+# device or None); a function ends at the next "}" in column 0, or before that text
 FUNCTIONS = [
-    ("kvx_host.cpp", r"^static void topk_rows\("),
-    ("kvx_host.cpp", r"^int64_t kvx_mapper_params\("),
-    ("kvx_host.cpp", r"^kvx_status kvx_select_topk\("),
-    ("kvx_host.cpp", r"^kvx_status kvx_create\("),
-    ("kvx_tc.cu", r"^void build_plan\("),
-    ("kvx_tc.cu", r"^uint32_t use_bits\("),
-    ("kvx_tc.cu", r"^KVX_API kvx_status kvx_tc_load_schedule\("),
+    ("kvx_host.cpp", r"^static void topk_rows\(", None),
+    ("kvx_host.cpp", r"^const char\* check_rope_scaling\(", None),
+    ("kvx_host.cpp", r"^int64_t kvx_mapper_params\(", None),
+    ("kvx_host.cpp", r"^kvx_status kvx_select_topk\(", None),
+    ("kvx_host.cpp", r"^kvx_status kvx_create\(", "DeviceGuard guard(device);"),
+    ("kvx_tc.cu", r"^void build_plan\(", None),
+    ("kvx_tc.cu", r"^uint32_t use_bits\(", None),
+    ("kvx_tc.cu", r"^KVX_API kvx_status kvx_tc_load_schedule\(", None),
+    ("kvx_fit.cu", r"^const char\* check_fit_config\(", None),
+    ("kvx_fit.cu", r"^KVX_API kvx_status kvx_fit_ridge\(", "const int sms = sm_count_or_zero();"),
+    ("kvx_probe.cu", r"^const char\* check_probe_config\(", None),
+    ("kvx_probe.cu", r"^KVX_API kvx_status kvx_r2_probe\(", "cudaStream_t st = static_cast<cudaStream_t>(stream);"),
+    ("kvx_mlp.cu", r"^const char\* check_mlp_config\(", None),
+    ("kvx_mlp.cu", r"^KVX_API kvx_status kvx_mlp_map\(", "cudaStream_t st = static_cast<cudaStream_t>(stream);"),
+    ("kvx_noalloc.cu", r"^extern \"C\" KVX_API kvx_status kvx_map_noalloc\(", "cudaError_t e = cudaGetDevice(&prev);"),
 ]
-# kvx_create is audited up to the point where it reaches the device
-CREATE_STOP = "DeviceGuard guard(device);"
+# Not audited here: the checks of kvx_map and of the host pipe that follow their NULL-context
+# check need a context, and a context needs a GPU (the GPU tests exercise them).
 
 OPS = [
     (r" \+ ", " - "), (r" - ", " + "), (r" < ", " <= "), (r" > ", " >= "), (r" <= ", " < "), (r" >= ", " > "),
@@ -51,7 +63,8 @@ OPS = [
 ]
 
 # (file, mutated line, why the ABI behaves the same).  A mutated line ending in "..." matches
-# any line that starts with the text before it (error messages, whose text may change).
+# any line that starts with the text before it.  Text inside string literals (error
+# messages) is not mutated.
 EQUIVALENT = [
     ("kvx_host.cpp", "if (row[a] != row[b]) return row[a] >= row[b];", "evaluated only when the scores differ"),
     ("kvx_host.cpp", "return a <= b;", "evaluated for two different indices only"),
@@ -68,10 +81,6 @@ EQUIVALENT = [
      "with the same status"),
     ("kvx_host.cpp", "ctx->F = c.k * c.head_dim * (c.head_mix != KVX_CROSS_HEAD ? c.n_kv_heads : 1);",
      "F is used on the device path only (the GPU parity tests cover it)"),
-    ("kvx_host.cpp", "return fail(KVX_ERR_INVALID_ARG, \"...", "only an error message's text changes"),
-    ("kvx_host.cpp", "if (c.head_dim > kMaxHeadDim) return fail(KVX_ERR_UNSUPPORTED, \"...",
-     "only an error message's text changes"),
-    ("kvx_tc.cu", "return fail(KVX_ERR_INVALID_ARG, \"...", "only an error message's text changes"),
     ("kvx_tc.cu", "if (src_layers < 1 || tgt_layers < 1 || k < 1 || 1 > src_layers)",
      "k > L_s leaves an entry out of range or a repeat in a row: the same status"),
     ("kvx_tc.cu", "std::vector<int> slot_src(S, -1), slot_next(S, 0), slot_last(S, -1), slot_load(S, -1), "
@@ -85,25 +94,48 @@ EQUIVALENT = [
     ("kvx_tc.cu", "slot_last[0] = u;", "slot_last only breaks ties among equal next uses: still optimal"),
     ("kvx_tc.cu", "if (slot_src[0] < 0) continue;",
      "slot 0 holds the first load, and an empty slot has no issuer to release it"),
+    ("kvx_mlp.cu", 'if (static_cast<int64_t>(c->tgt_layers) * 2 * c->n_kv_heads * c->hidden >= INT_MAX / 2) '
+     'return "too many weight rows";', "the product is even and INT_MAX / 2 odd: they are never equal"),
+    ("kvx_mlp.cu", 'if (static_cast<int64_t>(c->k) * c->n_kv_heads * kMD >= INT_MAX / 2) return "source feature too wide";',
+     "the product is a multiple of 128 and INT_MAX / 2 odd: they are never equal"),
+    ("kvx_noalloc.cu", "if (m->src_layers < 0 || m->tgt_layers <= 0 || m->n_kv_heads <= 0 || m->head_dim <= 0 ||",
+     "src_layers = 0 fails the k check (k >= 1 > src_layers) with the same status"),
+    ("kvx_probe.cu", 'if (batch < 1 && tokens_per_seq < 1) return bad("batch and tokens_per_seq must be >= 1");',
+     "an empty batch or sequence then fails the more-than-128-tokens check with the same status"),
+    ("kvx_probe.cu", "for (int i = 0; i <= 4; ++i)",
+     "reads one element past the stride array: undefined behaviour that no call at the ABI can observe"),
 ]
 
 
 def regions(path, f):
     lines = open(path).read().split("\n")
     out = []
-    for file, pat in FUNCTIONS:
+    for file, pat, stop in FUNCTIONS:
         if file != f:
             continue
         start = next(i for i, ln in enumerate(lines) if re.match(pat, ln))
         end = next(i for i in range(start + 1, len(lines)) if lines[i] == "}")
-        if pat.startswith("^kvx_status kvx_create"):
-            end = next(i for i in range(start, end) if CREATE_STOP in lines[i])
+        if stop is not None:
+            end = next(i for i in range(start, end) if stop in lines[i])
         out.append((start, end))
     return lines, out
 
 
+def in_string(code, pos):
+    """Whether position pos of a code line lies inside a string literal."""
+    inside, i = False, 0
+    while i < pos:
+        if code[i] == "\\" and inside:
+            i += 2
+            continue
+        if code[i] == '"':
+            inside = not inside
+        i += 1
+    return inside
+
+
 def mutants():
-    for f in sorted({f for f, _ in FUNCTIONS}):
+    for f in sorted({f for f, _, _ in FUNCTIONS}):
         lines, regs = regions(os.path.join(ROOT, PKG, "csrc", f), f)
         for a, b in regs:
             for i in range(a, b):
@@ -112,6 +144,8 @@ def mutants():
                     continue
                 for pat, rep in OPS:
                     for m in re.finditer(pat, code):
+                        if in_string(code, m.start()):       # an error message's text, not code
+                            continue
                         new = lines[i][:m.start()] + re.sub(pat, rep, m.group(0)) + lines[i][m.end():]
                         if new != lines[i]:
                             yield f, i + 1, lines[i].strip(), new.strip(), "\n".join(lines[:i] + [new] + lines[i + 1:])

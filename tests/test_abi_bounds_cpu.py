@@ -184,6 +184,9 @@ def test_noalloc_call_accepted_reaches_the_device():
     assert _noalloc(m, batch=1, src=_src(stride3=64), tgt=_tgt(stride3=64), pos=BASE + 4) == kvx.KVX_ERR_CUDA
     paged = dict(paged=1, block_size=16, block_table=BASE + 20480, max_blocks_per_seq=4, n_blocks=8)
     assert _noalloc(m, batch=1, tgt=_tgt(**paged)) == kvx.KVX_ERR_CUDA
+    for i in range(3):
+        assert _noalloc(m, batch=1, src=_src(**{"stride%d" % i: 0}), tgt=_tgt(**{"stride%d" % i: 0})) == \
+            kvx.KVX_ERR_CUDA, i
 
 
 # ----------------------------------------------------------------- ridge fit ---------
@@ -271,9 +274,15 @@ def test_fit_accepted_reaches_the_device():
              dict(sel=_sel([[0, 1, 2, 3]] * 3)), dict(sel=_sel([[3]] * 3)),
              dict(sel=_sel(np.tile(np.arange(16), (2, 1))), src_layers=16, n_kv_heads=8,
                   head_mix=kvx.KVX_CROSS_HEAD)]
+    cases += [dict(sel=_sel([[0]]), src_layers=1), dict(n_kv_heads=1),
+              dict(sel=_sel([[0, 1]] * 1)), dict(sel=_sel([[2]] * 3), head_mix=kvx.KVX_CROSS_HEAD)]
     for over in cases:
         assert _fit(_fit_cfg(**over)) == kvx.KVX_ERR_CUDA, over
     assert _fit(_fit_cfg(), src=_src(stride3=128), pos=BASE + 4, W=BASE + 16, b=BASE + 16) == kvx.KVX_ERR_CUDA
+    assert _fit(_fit_cfg(), batch=1, T=1) == kvx.KVX_ERR_CUDA
+    for i in range(3):                                   # a zero stride repeats a layer, batch or head
+        assert _fit(_fit_cfg(), src=_src(**{"stride%d" % i: 0}), tgt=_src(**{"stride%d" % i: 0})) == \
+            kvx.KVX_ERR_CUDA, i
 
 
 # ----------------------------------------------------------------- R^2 probe ---------
@@ -342,6 +351,9 @@ def test_probe_accepted_reaches_the_device():
     assert _probe(c, T=129) == kvx.KVX_ERR_CUDA
     assert _probe(c, r2=None) == kvx.KVX_ERR_CUDA
     assert _probe(c, src=_src(stride3=128), pos=BASE + 4, scores=BASE + 8, r2=BASE + 8) == kvx.KVX_ERR_CUDA
+    assert _probe(c, batch=129, T=1) == kvx.KVX_ERR_CUDA
+    for i in range(3):
+        assert _probe(c, src=_src(**{"stride%d" % i: 0}), tgt=_src(**{"stride%d" % i: 0})) == kvx.KVX_ERR_CUDA, i
 
 
 # ----------------------------------------------------------------- MLP mapper --------
@@ -379,6 +391,7 @@ def test_mlp_config_bounds():
         assert _mlp_ws(_mlp_cfg(**over)) == -1, over
         assert _mlp(_mlp_cfg(**over)) == INV, over
     good = [dict(hidden=512), dict(hidden=65536), dict(src_rope_theta=1.0 + 1e-9), dict(rope_numerics=1),
+            dict(n_kv_heads=1), dict(sel=_sel([[0]] * 2), src_layers=1), dict(sel=_sel([[1, 2]]), tgt_layers=1),
             dict(workspace=BASE, workspace_bytes=1), dict(sel=_sel([[0, 1, 2]] * 2)), dict(sel=_sel([[2]] * 2))]
     good += [{w: BASE + 16} for w in ("W1", "b1", "W2", "b2", "W3", "b3")]
     for over in good:
@@ -426,3 +439,5 @@ def test_mlp_accepted_reaches_the_device():
     c = _mlp_cfg()
     assert _mlp(c) == kvx.KVX_ERR_CUDA
     assert _mlp(c, src=_src(stride3=128), tgt=_tgt(stride3=128), pos=BASE + 4) == kvx.KVX_ERR_CUDA
+    for i in range(3):
+        assert _mlp(c, src=_src(**{"stride%d" % i: 0}), tgt=_tgt(**{"stride%d" % i: 0})) == kvx.KVX_ERR_CUDA, i
