@@ -76,3 +76,80 @@ def test_no_reuse_bound_has_the_stated_intensity():
     assert b["bytes_per_token"] == 1310720
     assert b["bound"] == "hbm" and abs(b["roofline_ms"] - 32768 * 1310720 / 6.8e9) < 1e-9
     assert abs(b["frac"] - b["roofline_ms"] / 3.0) < 1e-12
+
+
+def test_algorithmic_counts_of_the_workloads():
+    """Per launch, as stated for the bench workloads: FLOP = 2 (K, V) L_t H 2 F d per token;
+    bytes = every source layer read once + the target written once + 4 B of position per
+    token, plus W and b once."""
+    w = syn.workload("qwen3_14b_32b_t32768_k4")
+    a = bench.algorithmic(w)
+    assert a["flop"] == 4_398_046_511_104 and a["flop_per_token"] == 134_217_728
+    assert a["bytes_per_token"] == 163_840 + 262_144 + 4
+    assert a["weight_bytes"] == 134_217_728 + 262_144                 # W bf16, then b
+    assert a["bytes"] == 14_093_254_656
+    # Llama-3.1 8B -> 70B shapes: more target than source layers, k = 3
+    a = bench.algorithmic(syn.workload("llama31_8b_70b_b4x8192_k3"))
+    assert a["flop"] == 4_123_168_604_160
+    assert a["bytes_per_token"] == 131_072 + 327_680 + 4
+    assert a["weight_bytes"] == 125_829_120 + 327_680
+    assert a["bytes"] == 15_158_673_408
+    # one paged turn (16 x 2048 new tokens), Qwen3-32B -> 14B shapes
+    a = bench.algorithmic(syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4"))
+    assert a["flop"] == 2_748_779_069_440 and a["bytes_per_token"] == 262_144 + 163_840 + 4
+
+
+class _Clocks(bench.ClockSampler):
+    def __init__(self, out):
+        super().__init__(0)
+        self.out = out
+
+
+def test_clock_summary():
+    # index, clocks.sm, clocks.max.sm, power.draw, reasons.active, hw, hw_thermal, sw_thermal, sw_power_cap
+    rows = ["0, 1980, 2070, 150.0, 0x0, Not Active, Not Active, Not Active, Not Active",   # idle: not under load
+            "0, 1500, 2070, 1390.0, 0x4, Not Active, Not Active, Not Active, Active",
+            "0, 1700, 2070, 1200.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+            "0, 1600, 2070, 1300.5, 0x0, Not Active, Not Active, Not Active, Not Active",
+            "0, 1650, 2070, 1250.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+            "garbage line", "0, [N/A], 2070, 900, 0x0, Not Active, Not Active, Not Active, Not Active"]
+    s = _Clocks("\n".join(rows)).summary()
+    assert s["sm_mhz"] == 1625.0                     # median of the four loaded samples
+    assert s["sm_max_mhz"] == 2070.0 and s["reasons"] == ["sw_power_cap"]
+    assert s["samples"] == 5 and s["samples_under_load"] == 4 and s["power_w_max"] == 1390.0
+    hot = rows[1].replace("Not Active, Not Active, Not Active, Active", "Active, Not Active, Active, Not Active")
+    assert _Clocks(hot).summary()["reasons"] == ["hw_slowdown", "sw_thermal_slowdown"]
+    hot = rows[1].replace("Not Active, Not Active, Not Active, Active", "Not Active, Active, Not Active, Not Active")
+    assert _Clocks(hot).summary()["reasons"] == ["hw_thermal_slowdown"]
+    # below 200 W everywhere: every sample counts; no samples at all: said so
+    idle = _Clocks(rows[0] + "\n" + rows[0].replace("1980", "1000")).summary()
+    assert idle["sm_mhz"] == 1490.0 and idle["samples_under_load"] == 2
+    assert _Clocks("").summary() == {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"]}
+    # under load means above 200 W; the maximum clock is the largest reported
+    edge = ["0, 1000, 1980, 200.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+            "0, 1800, 2070, 200.05, 0x0, Not Active, Not Active, Not Active, Not Active",
+            "0, 1900, 2010, 600.0, 0x0, Not Active, Not Active, Not Active, Not Active"]
+    e = _Clocks("\n".join(edge)).summary()
+    assert e["samples_under_load"] == 2 and e["sm_mhz"] == 1850.0 and e["sm_max_mhz"] == 2070.0
+
+
+def test_peaks_fallback_is_the_recipe_figures(monkeypatch, tmp_path):
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.load_peaks() == dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, source="fallback")
+    (tmp_path / "MEASURED_PEAKS.json").write_text('{"hbm_gbs": 6000.5, "bf16_tflops": 1800.25}')
+    assert bench.load_peaks() == dict(hbm=6000.5, bf16=1800.25, bf16_sustained=None, source="measured")
+
+
+def test_traffic_file_parsing(monkeypatch, tmp_path):
+    w = syn.workload("qwen3_14b_32b_t32768_k4")
+    f = tmp_path / "traffic.txt"
+    f.write_text("# a comment: kernel_source_sha256_16: 0000000000000000\n"
+                 "# workload: elsewhere\n"
+                 "\n"
+                 "a line of text\n"
+                 "kernel_source_sha256_16: %s\nworkload: %s\ncaptured_workload: x:y\n"
+                 "dram_bytes_per_launch: 123456789\n" % (bench.kernel_hash(), w.name))
+    monkeypatch.setattr(bench, "TRAFFIC_FILE", str(f))
+    assert bench.committed_traffic(w) == 123456789.0
+    f.write_text("kernel_source_sha256_16: %s\nworkload: %s\ndram_bytes_per_launch: n/a\n" % (bench.kernel_hash(), w.name))
+    assert bench.committed_traffic(w) is None
