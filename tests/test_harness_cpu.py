@@ -76,3 +76,35 @@ def test_sampled_rows_cover_the_tile_borders_and_the_tail():
     assert rows[:, 1].max() == 127
     rows = H.sample_rows(w, 5, turn_T=129)
     assert (w.B - 1, 128) in {tuple(r) for r in rows.tolist()}
+
+
+def test_oracle_rows_are_the_rows_of_the_full_oracle():
+    """The full-size parity tests compare sampled rows against oracle_rows; those must be
+    exactly the corresponding rows of the full oracle map (both layouts, both modes, a
+    Llama-3-scaled workload), addressed by (batch, token)."""
+    from oracle import selection as osel
+    cases = [syn.workload("tiny_fp32", B=3, T=40),
+             syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=5, Lt=3, H=2, B=2, T=37, k=2, theta_t=5e5),
+             syn.workload("qwen3_14b_32b_b8x1024_k4", Ls=4, Lt=2, H=2, B=2, T=20, k=2, rope_style="interleaved"),
+             syn.workload("llama31_8b_70b_b4x8192_k3", Ls=4, Lt=3, H=2, B=2, T=24, k=2,
+                          rope_scaling=(8.0, 1.0, 4.0, 8192.0))]
+    for w in cases:
+        W, b = syn.weights(w)
+        sel = osel.select_topk(syn.selection_scores(w), w.k)
+        pos = syn.positions(w) * 1000 + 7                  # positions far from the token index
+        rk, rv, ak, av = H.oracle_full(w, syn.source_cache(w, 0), syn.source_cache(w, 1), pos, sel, W, b)
+        rows = np.array([[0, 0], [w.B - 1, w.T - 1], [1, 3], [0, w.T // 2]])
+        ok, ov, sk, sv = H.oracle_rows(w, rows, pos, sel, W, b)
+        for n, (bb, t) in enumerate(rows):
+            assert np.array_equal(ok[:, :, n], rk[:, bb, :, t]) and np.array_equal(ov[:, :, n], rv[:, bb, :, t])
+            assert np.array_equal(sk[:, :, n], ak[:, bb, :, t]) and np.array_equal(sv[:, :, n], av[:, bb, :, t])
+        assert np.array_equal(H.to_f64(W), W.double().numpy())
+
+
+def test_rope_theta_sides():
+    w = syn.workload("qwen3_14b_32b_b8x1024_k4", theta_s=1e4, theta_t=5e5)
+    assert (H.rope_theta(w, 0), H.rope_theta(w, 1)) == (1e4, 5e5)
+    w = syn.workload("llama31_8b_70b_b4x8192_k3", theta_s=1e4, theta_t=5e5, rope_scaling=(8.0, 1.0, 4.0, 8192.0))
+    s0, s1 = H.rope_theta(w, 0), H.rope_theta(w, 1)
+    assert (s0.theta, s1.theta) == (1e4, 5e5)
+    assert tuple(s0.scaling) == tuple(s1.scaling) == (8.0, 1.0, 4.0, 8192.0)
