@@ -38,6 +38,9 @@ OPS = [
     (r"\bstyle=style\b", "style=\"half\""), (r"\bbf16_cache=True\b", "bf16_cache=False"),
     (r"\bmode\b", "\"exact\""), (r"\[::-1\]", ""), (r"\bx_mean\b", "0.0"), (r"\by_mean\b", "0.0"),
     (r"\blam\b", "lam2"), (r"\bnp\.float32\b", "np.float64"),
+    (r"axis=-1", "axis=0"), (r"\[None, :\]", "[:, None]"), (r"\[:, None\]", "[None, :]"),
+    (r"\brange\((\w+)\)", "range(1)"), (r"\*\* 2\b", "** 1"), (r": d // 2\]", "d // 2:]"),
+    (r"\bd // 2:\]", ": d // 2]"),
 ]
 
 # (file, mutated line after the change, why it computes the same result)
