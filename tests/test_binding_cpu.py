@@ -116,3 +116,15 @@ def test_errors_carry_the_status_and_the_library_message():
     assert "k must be in [1, src_layers]" in str(e.value)
     assert kvx.kvx_mapper_params(64, 8, 128, 4) == 2 * 64 * 8 * 4 * 128 * 128
     assert kvx.kvx_mapper_params(64, 8, 128, 4, kvx.KVX_CROSS_HEAD) == 2 * 64 * 8 * 4 * 8 * 128 * 128
+
+
+def test_a_missing_library_fails_loudly(monkeypatch, tmp_path):
+    # no fallback: every entry point goes through lib(), which raises without libkvx.so
+    monkeypatch.setattr(kvx, "_lib", None)
+    monkeypatch.setattr(kvx, "LIB_PATH", str(tmp_path / "libkvx.so"))
+    with pytest.raises(RuntimeError, match="libkvx.so not found"):
+        kvx.lib()
+    with pytest.raises(RuntimeError):
+        kvx.kvx_select_topk(np.zeros((2, 3)), 1)
+    with pytest.raises(RuntimeError):
+        kvx.kvx_mapper_params(64, 8, 128, 4)
