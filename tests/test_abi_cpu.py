@@ -7,7 +7,6 @@ import re
 
 import numpy as np
 import pytest
-import torch
 
 from oracle import mapper as omap
 from oracle import selection as osel

@@ -17,7 +17,6 @@ here against what fixes it independently of its code:
    while its waiter still has an earlier phase to consume (a parity wait would then
    alias the two phases).
 """
-import itertools
 import random
 
 import numpy as np
