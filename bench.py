@@ -251,15 +251,26 @@ def job_rate(world, tokens_per_step, steps, ms):
 
 # ------------------------------------------------------------------ oracle leg ----
 
+def _exact_f64(t):
+    """Exact float64 values of a CPU tensor of bfloat16 (decoded bit pattern) or float32."""
+    from oracle import bf16 as obf16
+    if t.dtype == torch.bfloat16:
+        return obf16.decode(t.contiguous().view(torch.int16).numpy().view(np.uint16))
+    return t.double().numpy()
+
+
+def _oracle_mode(w):
+    """The oracle's rounding model for a workload: the bf16 forward for bf16 caches."""
+    return "exact" if w.cache_dtype == "f32" else "bf16fwd"
+
+
 def oracle_sample_rate(w, budget_s, seed=0, ctx_sel=None):
     """Time the float64 oracle (as it stands) on a bounded sample of the workload's
     tokens.  Returns (tokens/s, tokens, seconds, threads)."""
-    from oracle import bf16 as obf16
     from oracle import mapper as omap
     from oracle import selection as osel
     W, b = syn.weights(w)
-    Wf = obf16.decode(W.view(torch.int16).numpy().view(np.uint16)) if W.dtype == torch.bfloat16 else W.double().numpy()
-    bf = obf16.decode(b.view(torch.int16).numpy().view(np.uint16)) if b.dtype == torch.bfloat16 else b.double().numpy()
+    Wf, bf = _exact_f64(W), _exact_f64(b)
     sel = osel.select_topk(syn.selection_scores(w), w.k)
     pos = syn.positions(w)
     rng = np.random.default_rng(seed)
@@ -268,11 +279,10 @@ def oracle_sample_rate(w, budget_s, seed=0, ctx_sel=None):
         rows = np.stack([rng.integers(0, w.B, n), rng.integers(0, w.T, n)], axis=1)
         sk = syn.source_rows(w, 0, rows)
         sv = syn.source_rows(w, 1, rows)
-        skf = obf16.decode(sk.view(torch.int16).numpy().view(np.uint16))
-        svf = obf16.decode(sv.view(torch.int16).numpy().view(np.uint16))
+        skf, svf = _exact_f64(sk), _exact_f64(sv)
         p = pos[rows[:, 0], rows[:, 1]]
         t0 = time.perf_counter()
-        omap.map_tokens(skf, svf, p, sel, Wf, bf, w.theta_s, w.theta_t, mode="bf16fwd", head_mix=w.head_mix,
+        omap.map_tokens(skf, svf, p, sel, Wf, bf, w.theta_s, w.theta_t, mode=_oracle_mode(w), head_mix=w.head_mix,
                         style=w.rope_style)
         return time.perf_counter() - t0
 
@@ -323,30 +333,27 @@ def reference_arm(args, w, config):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
-    from oracle import bf16 as obf16
     from oracle import mapper as omap
     from oracle import selection as osel
     # size one step so that warmup + steps stay within a few minutes
     rate, n_cal, dt_cal, cores = oracle_sample_rate(w, budget_s=2.0)
     per_step = max(1, min(w.n_tokens, int(rate * 150.0 / max(1, args.steps + args.warmup))))
     W, b = syn.weights(w)
-    Wf = obf16.decode(W.view(torch.int16).numpy().view(np.uint16))
-    bf = obf16.decode(b.view(torch.int16).numpy().view(np.uint16))
+    Wf, bf = _exact_f64(W), _exact_f64(b)
     sel = osel.select_topk(syn.selection_scores(w), w.k)
     pos = syn.positions(w)
     # one seeded sample of the workload's tokens, generated once (its generation is not
     # oracle work) and mapped by every step
     rng = np.random.default_rng(7)
     rows = np.stack([rng.integers(0, w.B, per_step), rng.integers(0, w.T, per_step)], axis=1)
-    skf = obf16.decode(syn.source_rows(w, 0, rows).view(torch.int16).numpy().view(np.uint16))
-    svf = obf16.decode(syn.source_rows(w, 1, rows).view(torch.int16).numpy().view(np.uint16))
+    skf, svf = _exact_f64(syn.source_rows(w, 0, rows)), _exact_f64(syn.source_rows(w, 1, rows))
     prow = pos[rows[:, 0], rows[:, 1]]
     times, toks = [], 0
     step_budget = 150.0 / max(1, args.steps + args.warmup)
     for i in range(args.warmup + args.steps):
         t0 = time.perf_counter()
         omap.map_tokens(skf, svf, prow, sel, Wf, bf, w.theta_s, w.theta_t,
-                        mode="bf16fwd", head_mix=w.head_mix, style=w.rope_style)
+                        mode=_oracle_mode(w), head_mix=w.head_mix, style=w.rope_style)
         dt = time.perf_counter() - t0
         if i >= args.warmup:
             times.append(dt)

@@ -153,3 +153,22 @@ def test_traffic_file_parsing(monkeypatch, tmp_path):
     assert bench.committed_traffic(w) == 123456789.0
     f.write_text("kernel_source_sha256_16: %s\nworkload: %s\ndram_bytes_per_launch: n/a\n" % (bench.kernel_hash(), w.name))
     assert bench.committed_traffic(w) is None
+
+
+def test_reference_arm_prints_the_contract_line(capsys):
+    import json
+    import types
+    w = syn.workload("tiny_fp32")
+    args = types.SimpleNamespace(steps=3, warmup=1, gpus=1)
+    config = {"workload": w.name}
+    assert bench.reference_arm(args, w, config) == 0
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["metric"] == bench.METRIC and line["unit"] == bench.UNIT
+    assert (line["n_gpus"], line["steps"], line["warmup"]) == (1, 3, 1)
+    assert line["higher_is_better"] is True and line["vs_baseline"] is None and line["dtype"] == "f64"
+    assert line["config"] == config and line["value"] > 0 and line["ms_per_step"] > 0
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["value"] == line["value"] and cb["unit"] == line["unit"] and cb["cores"] >= 1
+    assert "tokens" in cb["sample"]
+    assert line["e2e"] == {"value": line["value"], "unit": line["unit"], "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
