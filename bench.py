@@ -49,13 +49,16 @@ KERNEL_SOURCES = ["paper_2608_03893_gb300/csrc/kvx_tc.cu", "paper_2608_03893_gb3
 
 
 def algorithmic(w):
-    """FLOPs and bytes of one launch (per-unit figures times the tokens of the launch)."""
-    e = 2  # bf16
+    """FLOPs and bytes of one launch (per-unit figures times the tokens of the launch).
+    Caches count at their element size (bf16 2 bytes, fp32 4), W and b at the weights'
+    (fp32 weights are 4 bytes an element, as the bf16 hi + lo pair the kernels read)."""
+    e = 4 if w.cache_dtype == "f32" else 2
+    ew = 4 if w.weight_dtype == "f32" else 2
     tok = w.n_tokens
     flop_per_tok = 2 * w.Lt * w.H * 2 * w.F * w.d              # K and V contractions
     src_per_tok = 2 * w.Ls * w.H * w.d * e                       # every source layer read once
     tgt_per_tok = 2 * w.Lt * w.H * w.d * e                       # target written once
-    w_bytes = w.Lt * 2 * w.H * w.F * w.d * e + w.Lt * 2 * w.H * w.d * e
+    w_bytes = w.Lt * 2 * w.H * w.F * w.d * ew + w.Lt * 2 * w.H * w.d * ew
     # looser bound: a mapper without reuse reads the k selected source tiles again for
     # every (target layer, K|V, head) product (per head; one product per (target layer,
     # K|V) cross-head) and writes its output: intensity k d / (k + 1) FLOP per byte per head

@@ -94,6 +94,13 @@ def test_algorithmic_counts_of_the_workloads():
     assert a["bytes_per_token"] == 131_072 + 327_680 + 4
     assert a["weight_bytes"] == 125_829_120 + 327_680
     assert a["bytes"] == 15_158_673_408
+    # fp32 caches and weights count 4 bytes an element; fp32 weights on bf16 caches too
+    w = syn.workload("tiny_fp32")
+    a = bench.algorithmic(w)
+    assert a["bytes_per_token"] == 2 * 4 * 2 * 64 * 4 + 2 * 6 * 2 * 64 * 4 + 4
+    assert a["weight_bytes"] == (6 * 2 * 2 * 128 * 64 + 6 * 2 * 2 * 64) * 4
+    a = bench.algorithmic(syn.workload("qwen3_14b_32b_t32768_k4", weight_dtype="f32"))
+    assert a["bytes_per_token"] == 163_840 + 262_144 + 4 and a["weight_bytes"] == 2 * (134_217_728 + 262_144)
     # one paged turn (16 x 2048 new tokens), Qwen3-32B -> 14B shapes
     a = bench.algorithmic(syn.workload("qwen3_32b_14b_paged_b16_turn2048_k4"))
     assert a["flop"] == 2_748_779_069_440 and a["bytes_per_token"] == 262_144 + 163_840 + 4
